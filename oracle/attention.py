@@ -1,0 +1,111 @@
+"""Oracle decode attention (test infrastructure; see ``oracle/__init__.py``).
+
+Everything here runs in float64 on already-dequantised caches.
+
+* ``resolve_sources`` -- Sec. 2.1 (depth axis): a layer either owns a cache
+  (an *anchor*) or inherits from the nearest anchor before it; layer 1 must
+  own one (Sec. 2.2, below eq. compression).  Returns ``src[l]``.
+* ``gqa_decode`` -- one decode step of grouped-query attention for every
+  query head: query head ``h`` reads KV head ``h // G`` (contiguous groups of
+  ``G = H_q / H_kv``), scores ``s_t = sigma * <q_h, k_t>``, softmax over the
+  positions the layer reads, output ``sum_t p_t v_t``.  With a kept-position
+  list (eviction composed with compression, Sec. 3.3) only the listed
+  positions are read.
+* ``mla_decode_unabsorbed`` -- Appendix C.2: the MLA cache holds the latent
+  ``c`` truncated to its first ``d`` coordinates and the post-RoPE positional
+  key ``k^R`` shared by all heads.  Head ``h`` reconstructs its content key
+  ``W_UK^h[:, :d] c[:d]`` and value ``W_UV^h[:, :d] c[:d]`` explicitly; the
+  score adds ``<q_pe^h, k^R>``.  The GPU computes the absorbed form; the
+  algebraic identity between the two is pinned by a test.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def resolve_sources(owns):
+    """``owns[l]`` true when layer ``l`` (0-based) owns a cache.
+
+    Returns ``src`` with ``src[l] = l`` for anchors and the nearest anchor
+    index ``< l`` for inheritors.  Raises ``ValueError`` if layer 0 inherits.
+    """
+    owns = [bool(o) for o in owns]
+    if not owns or not owns[0]:
+        raise ValueError("layer 0 must own a cache")
+    src = []
+    last = 0
+    for l, o in enumerate(owns):
+        if o:
+            last = l
+        src.append(last)
+    return src
+
+
+def softmax_weights(scores: np.ndarray) -> np.ndarray:
+    """Numerically safe softmax along the last axis (float64)."""
+    s = np.asarray(scores, dtype=np.float64)
+    m = s.max(axis=-1, keepdims=True)
+    e = np.exp(s - m)
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def gqa_decode(q, k_hat, v_hat, lens, sigma, kept=None):
+    """One decode step over a GQA cache.
+
+    q      : ``[B, H_q, D]``
+    k_hat  : ``[B, H_kv, T, D]`` dequantised keys (positions >= lens[b] unused)
+    v_hat  : ``[B, H_kv, T, D]``
+    lens   : ``[B]`` valid positions per sequence
+    sigma  : softmax scale
+    kept   : optional list (per sequence) of position arrays to read instead
+             of ``0..lens[b]-1``
+    Returns ``[B, H_q, D]`` float64.
+    """
+    q = np.asarray(q, np.float64)
+    B, Hq, D = q.shape
+    Hkv = k_hat.shape[1]
+    if Hq % Hkv:
+        raise ValueError("H_q must be a multiple of H_kv")
+    G = Hq // Hkv
+    out = np.zeros((B, Hq, D), np.float64)
+    for b in range(B):
+        pos = np.arange(int(lens[b])) if kept is None else np.asarray(kept[b], np.int64)
+        if pos.size == 0:
+            continue
+        for h in range(Hq):
+            j = h // G
+            K = np.asarray(k_hat[b, j, pos], np.float64)
+            V = np.asarray(v_hat[b, j, pos], np.float64)
+            p = softmax_weights(sigma * (K @ q[b, h]))
+            out[b, h] = p @ V
+    return out
+
+
+def mla_decode_unabsorbed(q_nope, q_pe, c, k_r, w_uk, w_uv, d, lens, sigma):
+    """MLA decode step, content keys and values reconstructed explicitly.
+
+    q_nope : ``[B, H, Dn]``      q_pe : ``[B, H, dR]`` (post-RoPE)
+    c      : ``[B, T, >=d]``     latent cache (only ``[:d]`` is read)
+    k_r    : ``[B, T, dR]``      positional key (post-RoPE)
+    w_uk   : ``[H, Dn, r]``      w_uv : ``[H, Dv, r]``
+    Returns ``[B, H, Dv]`` float64.
+    """
+    q_nope = np.asarray(q_nope, np.float64)
+    q_pe = np.asarray(q_pe, np.float64)
+    B, H, _ = q_nope.shape
+    Dv = w_uv.shape[1]
+    out = np.zeros((B, H, Dv), np.float64)
+    for b in range(B):
+        T = int(lens[b])
+        if T == 0:
+            continue
+        C = np.asarray(c[b, :T, :d], np.float64)          # [T, d]
+        KR = np.asarray(k_r[b, :T], np.float64)           # [T, dR]
+        for h in range(H):
+            Wk = np.asarray(w_uk[h, :, :d], np.float64)   # [Dn, d]
+            Wv = np.asarray(w_uv[h, :, :d], np.float64)   # [Dv, d]
+            Kc = C @ Wk.T                                 # [T, Dn] content keys
+            Vh = C @ Wv.T                                 # [T, Dv] values
+            s = sigma * (Kc @ q_nope[b, h] + KR @ q_pe[b, h])
+            out[b, h] = softmax_weights(s) @ Vh
+    return out

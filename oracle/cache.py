@@ -1,0 +1,92 @@
+"""Oracle for a whole per-layer plan (test infrastructure).
+
+A plan holds one action per layer (Sec. 2.2): inherit, or produce a cache at
+some bit-width (and, for MLA, some kept width).  The plan is fixed for the
+whole generation (Sec. 2.3), so an anchor's stored state depends only on the
+tokens written to it.
+
+``anchor_state`` turns the raw keys/values written to one anchor into what
+the cache stores (codes, scales, zeros, residual) and into the float64
+dequantised keys/values attention reads.  ``plan_outputs`` resolves every
+layer's source (nearest preceding anchor, Sec. 2.1) and runs
+``attention.gqa_decode`` with that layer's own query.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import quant
+from .attention import gqa_decode, resolve_sources
+
+
+def anchor_state(k, v, lens, bits, group=None, key_axis="token", value_axis="token"):
+    """Stored and dequantised state of one GQA anchor.
+
+    k, v : ``[B, H_kv, T, D]`` values as written (float32-exact)
+    lens : ``[B]`` tokens written per sequence
+    Returns a dict with ``k_hat``/``v_hat`` (float64, zero past ``lens``) and,
+    for quantised layers, the stored ``k_codes``, ``k_scale``, ``k_zero``,
+    ``v_codes``, ``v_scale``, ``v_zero`` and (per-channel keys)
+    ``k_residual``; per-channel entries are lists indexed by sequence because
+    each sequence's group count depends on its own length.
+    """
+    k = np.asarray(k, np.float32)
+    v = np.asarray(v, np.float32)
+    B, H, T, D = k.shape
+    st = {"bits": bits, "group": group, "key_axis": key_axis, "value_axis": value_axis}
+    k_hat = np.zeros(k.shape, np.float64)
+    v_hat = np.zeros(v.shape, np.float64)
+    if bits == 16:
+        for b in range(B):
+            n = int(lens[b])
+            k_hat[b, :, :n] = k[b, :, :n]
+            v_hat[b, :, :n] = v[b, :, :n]
+        st.update(k_hat=k_hat, v_hat=v_hat)
+        return st
+    if value_axis != "token":
+        raise ValueError("values are quantised per token")
+    vc, vs, vz = quant.quantise_per_token(v, bits, group)
+    st.update(v_codes=vc, v_scale=vs, v_zero=vz)
+    vh = quant.dequantise_per_token(vc, vs, vz, group)
+    if key_axis == "token":
+        kc, ks, kz = quant.quantise_per_token(k, bits, group)
+        st.update(k_codes=kc, k_scale=ks, k_zero=kz)
+        kh = quant.dequantise_per_token(kc, ks, kz, group)
+        for b in range(B):
+            n = int(lens[b])
+            k_hat[b, :, :n] = kh[b, :, :n]
+    elif key_axis == "channel":
+        st.update(k_codes=[], k_scale=[], k_zero=[], k_residual=[])
+        for b in range(B):
+            n = int(lens[b])
+            c, s, z, r = quant.quantise_per_channel(k[b, :, :n], bits, group)
+            st["k_codes"].append(c)
+            st["k_scale"].append(s)
+            st["k_zero"].append(z)
+            st["k_residual"].append(r)
+            k_hat[b, :, :n] = quant.dequantise_per_channel(c, s, z, group, r)
+    else:
+        raise ValueError(f"unknown key axis {key_axis!r}")
+    for b in range(B):
+        n = int(lens[b])
+        v_hat[b, :, :n] = vh[b, :, :n]
+    st.update(k_hat=k_hat, v_hat=v_hat)
+    return st
+
+
+def plan_outputs(owns, states, queries, lens, sigma, kept=None):
+    """Decode output of every layer of a plan.
+
+    owns    : per-layer bool (True = anchor)
+    states  : dict anchor index -> ``anchor_state`` result
+    queries : per-layer ``[B, H_q, D]``
+    lens    : dict anchor index -> ``[B]`` lengths
+    kept    : optional dict anchor index -> per-sequence kept positions
+    """
+    src = resolve_sources(owns)
+    outs = []
+    for l, s in enumerate(src):
+        st = states[s]
+        kp = None if kept is None else kept.get(s)
+        outs.append(gqa_decode(queries[l], st["k_hat"], st["v_hat"], lens[s], sigma, kp))
+    return outs

@@ -1,0 +1,112 @@
+"""Pins for oracle/quant.py against closed forms, hand-worked cases and
+brute force (no GPU).  Each test names the mistake it would catch."""
+import numpy as np
+import pytest
+
+from oracle import quant
+
+F32 = np.float32
+
+
+def test_worked_example_two_bits():
+    # 4 values spanning 3 steps: scale = 3/3 = 1, zero = 0, codes = values.
+    c, s, z = quant.quantise_groups(np.array([0.0, 1.0, 2.0, 3.0], F32), 2)
+    assert c.tolist() == [0, 1, 2, 3] and s == F32(1) and z == F32(0)
+    # a wrong level count (2^b instead of 2^b - 1) would give scale 0.75
+
+
+def test_zero_point_is_min_and_codes_unsigned():
+    x = np.array([-3.0, -1.0, 1.0, 3.0], F32)
+    c, s, z = quant.quantise_groups(x, 2)
+    assert z == F32(-3.0) and s == F32(2.0)
+    assert c.tolist() == [0, 1, 2, 3]
+
+
+def test_round_half_to_even():
+    # ratio values 0.5, 1.5, 2.5 -> 0, 2, 2 under half-to-even (floor or
+    # half-up rounding would differ)
+    x = np.array([0.0, 0.5, 1.5, 2.5, 3.0], F32)
+    c, s, _ = quant.quantise_groups(x, 2)
+    assert s == F32(1.0)
+    assert c.tolist() == [0, 0, 2, 2, 3]
+
+
+def test_constant_group():
+    x = np.full(32, 0.375, F32)
+    c, s, z = quant.quantise_groups(x, 4)
+    assert s == F32(0) and (c == 0).all() and z == F32(0.375)
+    xh = quant.dequantise_per_token(c, s[None], z[None], 32)
+    assert (xh == 0.375).all()
+
+
+@pytest.mark.parametrize("bits", [2, 4, 8])
+def test_extremes_and_roundtrip(bits):
+    rng = np.random.default_rng(bits)
+    x = (rng.standard_normal((257, 64)) * rng.lognormal(0, 1, (257, 1))).astype(F32)
+    c, s, z = quant.quantise_groups(x, bits)
+    lev = (1 << bits) - 1
+    assert c.dtype == np.uint8 and c.max() <= lev
+    rows = np.arange(x.shape[0])
+    assert (c[rows, x.argmin(1)] == 0).all()
+    assert (c[rows, x.argmax(1)] == lev).all()
+    xh = c.astype(np.float64) * s[:, None] + z[:, None]
+    slack = 8 * np.finfo(np.float32).eps * np.abs(x).max(1)
+    err = np.abs(xh - x).max(1)
+    assert (err <= 0.5 * s.astype(np.float64) + slack).all()
+
+
+def _brute_group(vals, bits):
+    # scalar loop, one float32 op at a time
+    lev = F32((1 << bits) - 1)
+    mn = F32(min(vals)); mx = F32(max(vals))
+    sc = F32(F32(mx - mn) / lev)
+    out = []
+    for v in vals:
+        if sc == 0:
+            out.append(0)
+            continue
+        r = F32(F32(F32(v) - mn) / sc)
+        out.append(int(min(max(np.rint(r), 0), lev)))
+    return out, sc, mn
+
+
+def test_per_token_matches_brute_force():
+    rng = np.random.default_rng(7)
+    x = rng.standard_normal((3, 2, 5, 64)).astype(F32)
+    c, s, z = quant.quantise_per_token(x, 4, 32)
+    for idx in np.ndindex(3, 2, 5):
+        for g in range(2):
+            bc, bs, bz = _brute_group(list(x[idx][32 * g:32 * g + 32]), 4)
+            assert list(c[idx][32 * g:32 * g + 32]) == bc
+            assert s[idx][g] == bs and z[idx][g] == bz
+
+
+def test_per_channel_matches_brute_force_and_keeps_residual():
+    rng = np.random.default_rng(11)
+    T, D, g = 77, 8, 32          # two full groups + 13 residual positions
+    x = rng.standard_normal((T, D)).astype(F32)
+    c, s, z, r = quant.quantise_per_channel(x, 8, g)
+    assert c.shape == (64, D) and s.shape == (2, D) and r.shape == (13, D)
+    assert (r == x[64:]).all()
+    for G in range(2):
+        for ch in range(D):
+            bc, bs, bz = _brute_group(list(x[G * g:(G + 1) * g, ch]), 8)
+            assert list(c[G * g:(G + 1) * g, ch]) == bc
+            assert s[G, ch] == bs and z[G, ch] == bz
+    xh = quant.dequantise_per_channel(c, s, z, g, r)
+    assert xh.shape == x.shape and (xh[64:] == x[64:]).all()
+
+
+def test_symmetric_two_bits_has_three_levels():
+    # Appendix C.3: q = 2^(b-1) - 1; at two bits the codes are {-1, 0, 1}
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((100, 128)).astype(F32)
+    c, s = quant.quantise_symmetric(x, 2)
+    assert set(np.unique(c).tolist()) == {-1, 0, 1}
+    c4, s4 = quant.quantise_symmetric(x, 4)
+    assert c4.min() >= -7 and c4.max() <= 7
+    # the element of largest magnitude maps to +-q exactly
+    i = np.abs(x).argmax(1)
+    assert (np.abs(c4[np.arange(100), i]) == 7).all()
+    err = np.abs(quant.dequantise_symmetric(c4, s4) - x).max(1)
+    assert (err <= 0.5 * s4 + 1e-6).all()
