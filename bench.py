@@ -1,0 +1,436 @@
+"""Decode-step benchmark of the compressed-KV path on GB300.
+
+Default workload: the Qwen2.5-14B-shaped mixed plan (48 layers, 40 q / 8 kv
+heads, head_dim 128, batch 32, 8191 cached positions + 1 appended per step,
+12 bf16 + 20 int4 g32 anchors, 16 inheriting layers).  One step = append one
+position to every anchor, decode attention for all 48 layers (inheritors
+read their source anchor with their own query), then roll the appended
+position back so every step reads exactly 8192 positions.
+
+Metric: achieved HBM GB/s of algorithmic bytes (compressed cache bytes every
+layer reads, plus query/output/append traffic) per step, and ms per step.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line (rank 0).  Under torchrun each rank runs its own
+replica of the workload (independent sequences; no collective on the data
+path) and the line reports the sum over ranks divided by the slowest rank.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode-attention achieved HBM GB/s and % of GB300 peak; per-step latency (us)"
+UNIT = "GB/s"
+
+
+# ---------------------------------------------------------------------------
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def algorithmic_bytes(w, lens_after_append):
+    """Bytes one step must move: each layer reads its source anchor's records
+    at the current length (per-token formats: rec bytes per (position, kv
+    head)); queries read, outputs written; appended rows read and written."""
+    B, H, D = w.batch, w.n_kv_heads, w.head_dim
+    src = w.sources()
+    total = 0
+    per_layer = []
+    for l in range(w.n_layers):
+        a = w.layers[src[l]]
+        rec = 4 * D if a["bits"] == 16 else 2 * D * a["bits"] // 8 + 2 * 8 * D // a["group"]
+        n = w.keep if w.keep else lens_after_append
+        cache = B * H * n * rec
+        qo = B * w.n_q_heads * D * (2 + 4)
+        per_layer.append(cache)
+        total += cache + qo
+        if not a["inherit"] and w.append_per_step and not w.layers[l]["inherit"]:
+            total += B * H * D * 2 * 2 + B * H * rec
+    return total, per_layer
+
+
+class Clocks:
+    """nvidia-smi sampler running during the timed region."""
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 "--query-gpu=clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.proc or not self.path:
+            return None
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 8:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[4:8]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+def cpu_baseline(w, seconds=12.0):
+    """The oracle (NumPy/fp64, as it stands) on a bounded sample of the same
+    workload: one (sequence, kv head) unit of a bf16 anchor and one of an
+    int4 anchor, each a full decode over the context (dequantise + softmax
+    attention for the G heads).  Returns (GB/s, sample text, cores)."""
+    import numpy as np
+    import torch
+    from oracle import attention as oatt
+    from oracle import quant as oq
+    from paper_2609_37988_gb300 import workloads as W
+
+    T, D, G = w.context, w.head_dim, w.n_q_heads // w.n_kv_heads
+    kinds = {}
+    for a in w.anchors:
+        kinds.setdefault(w.layers[a]["bits"], a)
+    units = []
+    for bits, a in sorted(kinds.items()):
+        k, v = W.kv_inputs(w, a, 0, T, device="cpu")
+        kk = k[0, :, 0].float().numpy()
+        vv = v[0, :, 0].float().numpy()
+        q = W.queries(w, a)[0, :G].float().numpy()
+        if bits == 16:
+            units.append((bits, q, kk, vv, None))
+        else:
+            g = w.layers[a]["group"]
+            units.append((bits, q, oq.quantise_per_token(kk, bits, g), oq.quantise_per_token(vv, bits, g), g))
+    nbytes = 0
+    n = 0
+    t0 = time.perf_counter()
+    while True:
+        for bits, q, kq, vq, g in units:
+            if bits == 16:
+                kh, vh = kq, vq
+                nbytes += T * 4 * D
+            else:
+                kh = oq.dequantise_per_token(*kq, g)
+                vh = oq.dequantise_per_token(*vq, g)
+                nbytes += T * (2 * D * bits // 8 + 16 * D // g)
+            oatt.gqa_decode(q[None], kh[None, None], vh[None, None], [T], w.sigma)
+        n += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0))
+    sample = (f"{n} passes over one (sequence, kv head) unit of each anchor format "
+              f"({', '.join(str(b) + '-bit' for b, *_ in units)}), {T} positions, G={G} heads")
+    return nbytes / dt / 1e9, sample, cores
+
+
+def run_reference(args):
+    """--impl reference: the oracle as it stands, on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_37988_gb300 import workloads as W
+    w = W.config(args.config)
+    per = max(2.0, 60.0 / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        cpu_baseline(w, seconds=min(per, 3.0))
+    vals = []
+    for _ in range(args.steps):
+        g, sample, cores = cpu_baseline(w, seconds=per)
+        vals.append(g)
+    v = statistics.median(vals)
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+# ---------------------------------------------------------------------------
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--config", type=int, default=3)
+    ap.add_argument("--impl", default="kvk")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from __graft_entry__ import build
+    build()
+    from paper_2609_37988_gb300 import workloads as W
+    from paper_2609_37988_gb300.cache import Cache, Layer
+
+    w = W.config(args.config)
+    if w.kind != "gqa":
+        raise SystemExit("bench.py times the GQA workloads (1, 2, 3, 5)")
+    T = w.context
+    pre = T - 1 if w.append_per_step else T
+    cache = Cache(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
+                  head_dim=w.head_dim, max_batch=w.batch, max_ctx=T, layers=[Layer(**a) for a in w.layers],
+                  max_splits=64, device=dev)
+    for a in w.anchors:
+        k, v = W.kv_inputs(w, a, 0, pre, device=dev)
+        cache.append(a, k, v)
+        del k, v
+    if w.keep:
+        import numpy as np
+        for a in w.anchors:
+            idx, n = W.kept_positions(w, a, np.full(w.batch, T), device=dev)
+            cache.set_kept(a, idx, n)
+    torch.cuda.synchronize()
+    qs = [W.queries(w, l, device=dev) for l in range(w.n_layers)]
+    outs = [torch.empty((w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
+            for _ in range(w.n_layers)]
+    new_kv = {}
+    if w.append_per_step:
+        for a in w.anchors:
+            new_kv[a] = W.kv_inputs(w, a, pre, T, device=dev)
+    src = w.sources()
+
+    def step():
+        for l in range(w.n_layers):
+            if l in new_kv:
+                cache.append(l, *new_kv[l])
+            cache.decode(l, qs[l], w.sigma, out=outs[l])
+        if w.append_per_step:
+            cache.rewind(1)
+
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        step()  # eager: sets kernel attributes, occupancy queries
+        stream.synchronize()
+        splits = [cache.plan_splits(l) for l in range(w.n_layers)]
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            step()
+    torch.cuda.synchronize()
+    launches = sum(1 + (splits[l] > 1) for l in range(w.n_layers))
+    launches += len(new_kv) + (1 if w.append_per_step else 0)
+
+    step_bytes, per_layer = algorithmic_bytes(w, T)
+
+    def barrier():
+        if dist:
+            dist.barrier()
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            graph.replay()
+        stream.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with Clocks(local) as clk:
+            torch.cuda.synchronize()
+            e0.record(stream)
+            for _ in range(args.steps):
+                graph.replay()
+            e1.record(stream)
+            e1.synchronize()
+            torch.cuda.synchronize()
+        barrier()
+    ms = e0.elapsed_time(e1)
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value = step_bytes * args.steps * world / (ms / 1e3) / 1e9
+
+    # ---- per-kernel durations (events on the launching stream) -------------
+    # decode kernel alone through kvk_decode_partial + kvk_splitk_reduce
+    from paper_2609_37988_gb300.cache import splitk_reduce
+    kt = {}
+    reps = 5
+    with torch.cuda.stream(stream):
+        for l in range(w.n_layers):
+            a = src[l]
+            kind = "bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}"
+            ns = splits[l]
+            part = torch.empty((max(ns, 2), w.batch * w.n_q_heads, w.head_dim + 2), device=dev)
+            if l in new_kv:
+                cache.append(l, *new_kv[l])
+            for r in range(reps):
+                s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                s0.record(stream)
+                if ns > 1:
+                    cache.decode_partial(l, qs[l], w.sigma, ns, partials=part)
+                else:
+                    cache.decode(l, qs[l], w.sigma, out=outs[l], n_splits=1)
+                s1.record(stream)
+                s1.synchronize()
+                kt.setdefault(kind, []).append((s0.elapsed_time(s1), per_layer[l]))
+        cache.rewind(1) if w.append_per_step else None
+        torch.cuda.synchronize()
+    hbm, peak_kind = peaks()
+    totals = {k: sum(t for t, _ in v) for k, v in kt.items()}
+    dom = max(totals, key=totals.get)
+    durs = [t for t, _ in kt[dom]]
+    bts = [b for _, b in kt[dom]]
+    avg_ms = sum(durs) / len(durs)
+    achieved = (sum(bts) / len(bts)) / (avg_ms / 1e3) / 1e9
+    kernels = {}
+    for k, v in kt.items():
+        d = sum(t for t, _ in v) / len(v)
+        b = sum(x for _, x in v) / len(v)
+        kernels[k] = {"avg_us": round(d * 1e3, 2), "gbs": round(b / (d / 1e3) / 1e9, 1),
+                      "frac": round(b / (d / 1e3) / 1e9 / hbm, 4)}
+    traffic = None
+    tf = os.path.join(ROOT, "profiles", "gqa_decode_traffic.json")
+    if os.path.exists(tf):
+        with open(tf) as f:
+            tj = json.load(f)
+        if tj.get("kernel_kind") == dom and tj.get("source_hash") == _source_hash():
+            traffic = tj.get("bytes_per_launch_full")
+
+    # ---- end to end through the public API, host buffers --------------------
+    e2e = None
+    if args.e2e_steps > 0:
+        h_q = [q.cpu().pin_memory() for q in qs]
+        h_kv = {a: (k.cpu().pin_memory(), v.cpu().pin_memory()) for a, (k, v) in new_kv.items()}
+        h_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
+        d_q = [torch.empty_like(q) for q in qs]
+        d_kv = {a: (torch.empty_like(k), torch.empty_like(v)) for a, (k, v) in new_kv.items()}
+        h2d = sum(q.numel() * q.element_size() for q in h_q) + \
+            sum(k.numel() * k.element_size() * 2 for k, _ in h_kv.values())
+        d2h = sum(o.numel() * o.element_size() for o in h_out)
+        with torch.cuda.stream(stream):
+            def e2e_step():
+                for l in range(w.n_layers):
+                    d_q[l].copy_(h_q[l], non_blocking=True)
+                for a in d_kv:
+                    d_kv[a][0].copy_(h_kv[a][0], non_blocking=True)
+                    d_kv[a][1].copy_(h_kv[a][1], non_blocking=True)
+                for l in range(w.n_layers):
+                    if l in d_kv:
+                        cache.append(l, *d_kv[l])
+                    cache.decode(l, d_q[l], w.sigma, out=outs[l])
+                    h_out[l].copy_(outs[l], non_blocking=True)
+                if w.append_per_step:
+                    cache.rewind(1)
+                stream.synchronize()
+            e2e_step()
+            barrier()
+            t0 = time.perf_counter()
+            for _ in range(args.e2e_steps):
+                e2e_step()
+            dt = time.perf_counter() - t0
+        if dist:
+            t = torch.tensor([dt], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            dt = float(t.item())
+        e2e = {"value": step_bytes * args.e2e_steps * world / dt / 1e9, "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": dt / args.e2e_steps * 1e3}
+
+    err = cache.device_error()
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        g, sample, cores = cpu_baseline(w)
+        cpu = {"value": g, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
+    clocks = clk.summary()
+    if rank == 0:
+        rec = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "us_per_step": ms_step * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16/int4",
+            "data": "synthetic",
+            "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "context": T,
+                       "q_heads": w.n_q_heads, "kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+                       "anchors": {"bf16": sum(1 for a in w.anchors if w.layers[a]["bits"] == 16),
+                                   "int4": sum(1 for a in w.anchors if w.layers[a]["bits"] == 4),
+                                   "int8": sum(1 for a in w.anchors if w.layers[a]["bits"] == 8)},
+                       "inheritors": w.n_layers - len(w.anchors),
+                       "bytes_per_step": step_bytes, "cuda_graph": True,
+                       "l2": "inputs larger than L2 (each anchor >= 403 MB; step reads ~31 GB), no flush",
+                       "parallelism": f"replicas x{world}"},
+            "fraction_of_peak": value / hbm, "peak_gbs": hbm, "peak_kind": peak_kind,
+            "fraction_of_nominal_8tbs": value / 8000.0,
+            "roofline": {"bound": "hbm", "kernel": f"gqa_decode ({dom})", "achieved": achieved,
+                         "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
+                         "peak_source": f"MEASURED_PEAKS.json hbm_gbs ({peak_kind})"},
+            "kernels": kernels,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches * args.steps,
+            "clocks": clocks,
+            "device_error": err,
+        }
+        print(json.dumps(rec))
+
+
+def _source_hash():
+    import hashlib
+    h = hashlib.sha256()
+    d = os.path.join(ROOT, "paper_2609_37988_gb300", "csrc")
+    for n in sorted(os.listdir(d)):
+        if n.startswith("decode_gqa"):
+            with open(os.path.join(d, n), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+if __name__ == "__main__":
+    main()

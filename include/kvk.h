@@ -1,0 +1,268 @@
+/*
+ * kvk.h -- C ABI of the GB300-native compressed-KV decode path.
+ *
+ * The library implements the per-step decode attention that reads a
+ * per-layer compressed KV cache, and the append that writes new tokens into
+ * it, for the per-layer cache plans of KV-Kaizen (arxiv 2609.37988):
+ *
+ *   depth      a layer owns a cache (an "anchor") or inherits the nearest
+ *              anchor before it and reads it with its own query (Sec. 2.1);
+ *   precision  a cache is stored at 16, 8 or 4 bits (Sec. 2.1; grouped
+ *              asymmetric quantiser of Appendix C.3 with a scale and a zero
+ *              point per group);
+ *   rank       an MLA latent truncated to its first d coordinates plus the
+ *              post-RoPE positional key (Sec. 2.1, Appendix C.2).
+ *
+ * A plan (one action per layer, eq. (cost)-(action space) in Sec. 2.2) is
+ * fixed for the whole generation (Sec. 2.3), so the cache is laid out once.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Ownership: the caller owns every device buffer (arenas, workspace,
+ *    inputs, outputs).  The library owns only its host-side cache object.
+ *    No entry point allocates device memory.
+ *  - Asynchrony: device work is enqueued on the caller's stream and is never
+ *    synchronised, except by kvk_get_device_error.
+ *  - Validation: arguments are checked on the host before anything is
+ *    enqueued; a failed check returns an error status and enqueues nothing.
+ *    Device-side bounds violations (for example a kept position past the
+ *    sequence length) set a device error word, skip the offending access and
+ *    let the kernel finish; they never trap.
+ *  - kvk_last_error() returns a thread-local, human-readable message for the
+ *    last non-OK status returned on the calling thread.
+ *  - Pointers marked "device" must be device-accessible and 16-byte aligned.
+ *  - Layer indices are 0-based.
+ */
+#ifndef KVK_H
+#define KVK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same handle as cudaStream_t; declared opaquely so this header needs no
+ * CUDA include.  NULL is the legacy default stream. */
+typedef struct CUstream_st *kvk_stream;
+
+typedef enum {
+  KVK_OK = 0,
+  KVK_ERR_INVALID_ARG = 1,     /* null pointer, bad size, misaligned buffer  */
+  KVK_ERR_INVALID_CONFIG = 2,  /* plan rejected (e.g. layer 0 inherits)      */
+  KVK_ERR_INHERITED_LAYER = 3, /* write to a layer that owns no cache        */
+  KVK_ERR_CAPACITY = 4,        /* append would pass max_ctx                  */
+  KVK_ERR_UNSUPPORTED = 5,     /* valid request this build does not handle   */
+  KVK_ERR_CUDA = 6,            /* a CUDA runtime call failed                 */
+  KVK_ERR_DEVICE = 7           /* the device error word was set              */
+} kvk_status;
+
+enum { KVK_KIND_GQA = 0, KVK_KIND_MLA = 1 };
+enum { KVK_AXIS_TOKEN = 0, KVK_AXIS_CHANNEL = 1 };
+enum { KVK_DTYPE_F32 = 0, KVK_DTYPE_BF16 = 1 };
+
+/* Device error word values (kvk_get_device_error). */
+enum {
+  KVK_DEVERR_NONE = 0,
+  KVK_DEVERR_KEPT_RANGE = 1,   /* kept position >= sequence length           */
+  KVK_DEVERR_CAPACITY = 2,     /* append position >= capacity                */
+  KVK_DEVERR_COUNT = 4         /* per-sequence append count out of range     */
+};
+
+/* Model geometry.  GQA: n_q_heads query heads, n_kv_heads KV heads of
+ * head_dim (Sec. 2.1, Tab. backbones).  MLA: latent width latent_dim (r),
+ * positional key rope_dim (d_R), content/value head width head_dim,
+ * n_q_heads heads sharing one latent (Appendix B, C.2). */
+typedef struct {
+  int32_t kind;        /* KVK_KIND_GQA or KVK_KIND_MLA                      */
+  int32_t n_layers;    /* L                                                 */
+  int32_t n_q_heads;   /* H_q                                               */
+  int32_t n_kv_heads;  /* H_kv (GQA); ignored for MLA                       */
+  int32_t head_dim;    /* d_h: 64 or 128 (GQA); 128 (MLA content/value)     */
+  int32_t latent_dim;  /* r (MLA); ignored for GQA                          */
+  int32_t rope_dim;    /* d_R (MLA, 64); ignored for GQA                    */
+  int32_t max_batch;   /* sequences per cache                               */
+  int32_t max_ctx;     /* positions per sequence                            */
+} kvk_model_desc;
+
+/* One plan action (Sec. 2.2).  inherit=1 is the depth action; otherwise the
+ * layer owns a cache at `bits` (16 = bf16, 8 or 4 = grouped quantiser with
+ * `group` elements per scale/zero pair) and, for MLA, keeps the first
+ * `width` latent coordinates (truncate on write, Appendix C.2).  key_axis
+ * selects per-token groups (g channels of one token) or per-channel groups
+ * (g positions of one channel, KIVI keys); values are per-token.
+ * evict_capacity > 0 reserves a kept-position list of that length per
+ * sequence (eviction composed with compression, Sec. 3.3). */
+typedef struct {
+  int32_t inherit;
+  int32_t bits;
+  int32_t group;
+  int32_t key_axis;
+  int32_t value_axis;
+  int32_t width;
+  int32_t evict_capacity;
+} kvk_layer_cfg;
+
+typedef struct kvk_cache kvk_cache;
+
+/* Validate a plan and report the device bytes each layer's arena needs
+ * (0 for inheritors).  arena_bytes: host array of n_layers entries.
+ * Errors: INVALID_ARG, INVALID_CONFIG (layer 0 inherits, bits not in
+ * {16,8,4}, group not dividing head_dim, MLA width not in r/8..r), and
+ * UNSUPPORTED for valid plans outside this build (2-bit codes, per-channel
+ * values, head_dim other than 64/128, per-channel keys with eviction). */
+kvk_status kvk_cache_plan(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
+                          size_t *arena_bytes);
+
+/* Device workspace bytes for a cache whose decode calls use at most
+ * max_splits context splits.  Holds the device error word, split-K partials,
+ * the absorbed MLA query and per-unit merge counters. */
+kvk_status kvk_workspace_size(const kvk_model_desc *desc, int32_t max_splits,
+                              size_t *ws_bytes);
+
+/* Create a cache over caller-allocated arenas.  arenas: host array of
+ * n_layers device pointers (NULL for inheritors), each of at least the size
+ * kvk_cache_plan reported; workspace: device buffer of ws_bytes.  The cache
+ * starts empty; call kvk_cache_reset (or zero the arenas) before first use.
+ * The cache keeps the pointers; the caller keeps the memory alive. */
+kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
+                            void *const *arenas, void *workspace, size_t ws_bytes,
+                            int32_t max_splits, kvk_cache **out);
+kvk_status kvk_cache_destroy(kvk_cache *cache);
+
+/* Zero every sequence length, kept list, merge counter and the device error
+ * word, on `stream`. */
+kvk_status kvk_cache_reset(kvk_cache *cache, kvk_stream stream);
+
+/* src[layer]: nearest anchor at or before `layer` (Sec. 2.1). */
+kvk_status kvk_layer_source(const kvk_cache *cache, int32_t layer, int32_t *src);
+
+/* Device pointer to the int32[max_batch] sequence lengths of the anchor that
+ * `layer` reads (advanced by kvk_append). */
+kvk_status kvk_layer_lengths(const kvk_cache *cache, int32_t layer,
+                             const int32_t **lens_device);
+
+/* Append n_new positions to every sequence of anchor `layer`: quantise (or
+ * truncate, for MLA) on write.
+ *  GQA: k, v device [B, n_new, H_kv, head_dim] in in_dtype (F32 or BF16).
+ *       Per-token groups are quantised immediately; per-channel key groups
+ *       are buffered in bf16 until g positions of a group exist, then
+ *       quantised along the positions (KIVI keys, Appendix C.3).
+ *  MLA: k = latent c device [B, n_new, latent_dim] BF16 (only the first
+ *       `width` coordinates are stored, Appendix C.2), v = positional key
+ *       k^R device [B, n_new, rope_dim] BF16, post-RoPE.
+ *  B = max_batch.  n_new_per_seq: optional device int32[B]; sequence b then
+ *  appends only its first n_new_per_seq[b] <= n_new rows (ragged lengths).
+ * Errors: INHERITED_LAYER, CAPACITY (host-side bound on the lengths),
+ * INVALID_ARG. */
+kvk_status kvk_append(kvk_cache *cache, int32_t layer, const void *k, const void *v,
+                      int32_t in_dtype, int32_t n_new, const int32_t *n_new_per_seq,
+                      kvk_stream stream);
+
+/* Roll back the last n positions of every sequence of every anchor (for
+ * example a rejected speculative step), in one launch on `stream`: each
+ * length becomes max(0, length - n).  Caches with per-channel key groups
+ * return UNSUPPORTED (a quantised group cannot be re-opened). */
+kvk_status kvk_rewind(kvk_cache *cache, int32_t n, kvk_stream stream);
+
+/* The split count kvk_decode_attention / kvk_decode_attention_mla would use
+ * for `layer` with n_splits = 0 (host only; depends on the host-side bound
+ * on the anchor's lengths and on the SM count). */
+kvk_status kvk_decode_plan_splits(kvk_cache *cache, int32_t layer, int32_t *n_splits);
+
+/* Install the kept-position list of anchor `layer` (eviction, Sec. 3.3):
+ * idx device int32 [B, evict_capacity] sorted ascending, n_kept device
+ * int32[B] <= evict_capacity.  Decode then reads only those positions; an
+ * entry past the sequence length sets KVK_DEVERR_KEPT_RANGE and is skipped.
+ * n_kept == NULL clears the list (all positions are read again). */
+kvk_status kvk_set_kept(kvk_cache *cache, int32_t layer, const int32_t *idx,
+                        const int32_t *n_kept, kvk_stream stream);
+
+/* GQA decode attention of `layer` with its own query (inheritors read their
+ * source anchor, Sec. 2.1):
+ *   out[b,h,:] = sum_t softmax_t(scale * <q[b,h], k_t>) v_t
+ * over the positions of sequence b (or its kept list), KV head h / G with
+ * G = H_q / H_kv.  q: device [B, H_q, head_dim] in q_dtype; out: device
+ * float [B, H_q, head_dim].  n_splits: context splits (0 = chosen from the
+ * SM count), at most the max_splits given at creation. */
+kvk_status kvk_decode_attention(kvk_cache *cache, int32_t layer, const void *q,
+                                int32_t q_dtype, float softmax_scale, float *out,
+                                int32_t n_splits, kvk_stream stream);
+
+/* MLA decode attention of `layer` in the absorbed form (Appendix C.2):
+ *   q_lat[b,h] = W_UK[h][:, :d]^T q_nope[b,h]
+ *   s_t       = scale * (<q_lat, c_t[:d]> + <q_pe, k^R_t>)
+ *   out[b,h]  = W_UV[h][:, :d] sum_t softmax_t(s_t) c_t[:d]
+ * q_nope device bf16 [B, H, head_dim]; q_pe device bf16 [B, H, rope_dim]
+ * (post-RoPE); w_uk, w_uv device bf16 [H, head_dim, latent_dim]; out device
+ * float [B, H, head_dim]. */
+kvk_status kvk_decode_attention_mla(kvk_cache *cache, int32_t layer, const void *q_nope,
+                                    const void *q_pe, const void *w_uk, const void *w_uv,
+                                    float softmax_scale, float *out, int32_t n_splits,
+                                    kvk_stream stream);
+
+/* Split-K pieces of kvk_decode_attention (the seam a context-parallel
+ * multi-GPU variant would all-gather across).  kvk_decode_partial writes
+ * partials device float [n_splits, B*H_q, head_dim + 2]: per row the
+ * unnormalised accumulator sum_t 2^(x_t - m) v_t (head_dim floats), then m,
+ * then l = sum_t 2^(x_t - m), with x_t = scale * log2(e) * <q, k_t>.  A split
+ * that reads no position stores m = -inf, l = 0. */
+kvk_status kvk_decode_partial(kvk_cache *cache, int32_t layer, const void *q,
+                              int32_t q_dtype, float softmax_scale, float *partials,
+                              int32_t n_splits, kvk_stream stream);
+
+/* Merge split partials in the format above:
+ *   out[row] = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
+ * partials device float [n_splits, n_rows, dim + 2]; out device float
+ * [n_rows, dim].  Rows where every split is empty are written as zeros. */
+kvk_status kvk_splitk_reduce(const float *partials, int32_t n_splits, int32_t n_rows,
+                             int32_t dim, float *out, kvk_stream stream);
+
+/* Cost accounting of the cache's plan.
+ *  bits_per_token_model: sum over layers of eq. (cost), in bits per token;
+ *  bytes_per_token_stored: bytes this build stores per token, summed over
+ *      anchors, including fp32 scale/zero metadata (Tab. realized_bits
+ *      counts metadata the same way);
+ *  rho: eq. (compression) against the bf16 GQA cache of the same geometry
+ *      (for MLA, n_kv_heads * head_dim = latent_dim is used as C0's width,
+ *      the conversion rule r = n_kv d_h of Appendix B). */
+kvk_status kvk_cost(const kvk_cache *cache, double *bits_per_token_model,
+                    double *bytes_per_token_stored, double *rho);
+
+/* The same accounting for a plan before any cache exists (host only, no
+ * device call).  Validates the plan like kvk_cache_plan. */
+kvk_status kvk_plan_cost(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
+                         double *bits_per_token_model, double *bytes_per_token_stored,
+                         double *rho);
+
+/* Copy anchor `layer`'s stored state out in canonical (unpermuted) form,
+ * device to device, on `stream`.  Positions past a sequence's length hold
+ * unspecified values.  Shapes (B = max_batch, T = max_ctx, D = head_dim):
+ *  bf16 GQA:   k_out, v_out bf16 [B, H_kv, T, D]; the rest unused.
+ *  quantised:  k_out, v_out uint8 codes [B, H_kv, T, D] (one code per byte);
+ *              v_scale, v_zero float [B, H_kv, T, D/g];
+ *              per-token keys: k_scale, k_zero float [B, H_kv, T, D/g];
+ *              per-channel keys: k_scale, k_zero float [B, H_kv, T/g, D] and
+ *              k_residual bf16 [B, H_kv, g, D] (positions of the open group,
+ *              row = position mod g).
+ *  MLA:        k_out bf16 [B, T, width] latent, v_out bf16 [B, T, rope_dim].
+ * Any pointer the format does not use may be NULL. */
+kvk_status kvk_export_layer(const kvk_cache *cache, int32_t layer, void *k_out, void *v_out,
+                            float *k_scale, float *k_zero, float *v_scale, float *v_zero,
+                            void *k_residual, kvk_stream stream);
+
+/* Synchronise `stream`, read the device error word into *code and clear it.
+ * Returns KVK_ERR_DEVICE if the word was non-zero. */
+kvk_status kvk_get_device_error(kvk_cache *cache, kvk_stream stream, int32_t *code);
+
+const char *kvk_status_string(kvk_status s);
+const char *kvk_last_error(void);
+
+/* Library version string ("kvk <major>.<minor> sm_103a"). */
+const char *kvk_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVK_H */

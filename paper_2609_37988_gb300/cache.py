@@ -1,0 +1,242 @@
+"""Thin PyTorch-facing wrapper of the C ABI (include/kvk.h).
+
+PyTorch provides device memory (arenas, workspace, outputs) and the current
+CUDA stream; every computation runs in ``libkvk.so``.  A :class:`Cache`
+holds one per-layer plan (Sec. 2.2 of the paper: inherit, or a cache at some
+bit-width / kept width) for a fixed model geometry.
+"""
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+
+import torch
+
+from . import _lib
+from ._lib import (AXIS_CHANNEL, AXIS_TOKEN, DTYPE_BF16, DTYPE_F32, KIND_GQA, KIND_MLA,
+                   KVKError, LayerCfg, ModelDesc, check, load)
+
+__all__ = ["Layer", "Cache", "splitk_reduce", "KVKError"]
+
+
+@dataclass
+class Layer:
+    """One plan action.  ``inherit=True`` is the depth action; otherwise a
+    cache at ``bits`` (16, 8, 4) with quantisation ``group`` and key axis
+    ``"token"``/``"channel"``, MLA kept ``width``, optional eviction list
+    capacity."""
+    inherit: bool = False
+    bits: int = 16
+    group: int = 64
+    key_axis: str = "token"
+    width: int = 0
+    evict_capacity: int = 0
+
+    def to_c(self) -> LayerCfg:
+        return LayerCfg(int(self.inherit), self.bits, self.group,
+                        AXIS_CHANNEL if self.key_axis == "channel" else AXIS_TOKEN,
+                        AXIS_TOKEN, self.width, self.evict_capacity)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(0 if t is None else t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return DTYPE_F32
+    if t.dtype == torch.bfloat16:
+        return DTYPE_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _need(t: torch.Tensor, name: str):
+    if not (t.is_cuda and t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+
+
+class Cache:
+    """A compressed KV cache for one model geometry and one plan."""
+
+    def __init__(self, *, kind: str = "gqa", n_layers: int, n_q_heads: int, n_kv_heads: int = 1,
+                 head_dim: int = 128, latent_dim: int = 0, rope_dim: int = 0, max_batch: int,
+                 max_ctx: int, layers, max_splits: int = 64, device=None):
+        self.lib = load()
+        self.desc = ModelDesc(KIND_MLA if kind == "mla" else KIND_GQA, n_layers, n_q_heads,
+                              n_kv_heads, head_dim, latent_dim, rope_dim, max_batch, max_ctx)
+        self.kind = kind
+        self.layers = list(layers)
+        if len(self.layers) != n_layers:
+            raise ValueError("one Layer per model layer")
+        cfg = (LayerCfg * n_layers)(*[l.to_c() for l in self.layers])
+        self._cfg = cfg
+        sizes = (ctypes.c_size_t * n_layers)()
+        check(self.lib.kvk_cache_plan(ctypes.byref(self.desc), cfg, sizes))
+        ws = ctypes.c_size_t()
+        check(self.lib.kvk_workspace_size(ctypes.byref(self.desc), max_splits, ctypes.byref(ws)))
+        dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+        self.device = dev
+        self.arena_bytes = [int(s) for s in sizes]
+        # torch's caching allocator returns 512-byte aligned blocks
+        self.arenas = [torch.empty(n, dtype=torch.uint8, device=dev) if n else None
+                       for n in self.arena_bytes]
+        self.workspace = torch.empty(int(ws.value), dtype=torch.uint8, device=dev)
+        ptrs = (ctypes.c_void_p * n_layers)(*[0 if a is None else a.data_ptr() for a in self.arenas])
+        h = ctypes.c_void_p()
+        with torch.cuda.device(dev):
+            check(self.lib.kvk_cache_create(ctypes.byref(self.desc), cfg, ptrs,
+                                            _ptr(self.workspace), ws.value, max_splits,
+                                            ctypes.byref(h)))
+        self.handle = h
+        self.max_splits = max_splits
+        self.reset()
+
+    # -- lifetime ------------------------------------------------------------
+    def close(self):
+        if getattr(self, "handle", None):
+            self.lib.kvk_cache_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def reset(self, stream=None):
+        check(self.lib.kvk_cache_reset(self.handle, _stream(stream)))
+
+    # -- plan ----------------------------------------------------------------
+    def source(self, layer: int) -> int:
+        out = ctypes.c_int32()
+        check(self.lib.kvk_layer_source(self.handle, layer, ctypes.byref(out)))
+        return out.value
+
+    def lengths(self, layer: int) -> torch.Tensor:
+        """Device int32[max_batch] lengths of the anchor ``layer`` reads (a view)."""
+        src = self.source(layer)
+        return self.arenas[src][: 4 * self.desc.max_batch].view(torch.int32)
+
+    def cost(self):
+        b, s, r = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+        check(self.lib.kvk_cost(self.handle, ctypes.byref(b), ctypes.byref(s), ctypes.byref(r)))
+        return {"bits_per_token_model": b.value, "bytes_per_token_stored": s.value, "rho": r.value}
+
+    # -- writes --------------------------------------------------------------
+    def append(self, layer: int, k: torch.Tensor, v: torch.Tensor, n_per_seq: torch.Tensor = None,
+               stream=None):
+        """GQA: k, v ``[B, n, H_kv, D]`` (fp32/bf16).  MLA: k = latent
+        ``[B, n, r]`` bf16, v = positional key ``[B, n, d_R]`` bf16."""
+        _need(k, "k"); _need(v, "v")
+        n = int(k.shape[1])
+        if n_per_seq is not None:
+            _need(n_per_seq, "n_per_seq")
+        check(self.lib.kvk_append(self.handle, layer, _ptr(k), _ptr(v), _dtype_code(k), n,
+                                  _ptr(n_per_seq), _stream(stream)))
+
+    def set_kept(self, layer: int, idx: torch.Tensor = None, n_kept: torch.Tensor = None,
+                 stream=None):
+        if n_kept is not None:
+            _need(idx, "idx"); _need(n_kept, "n_kept")
+        check(self.lib.kvk_set_kept(self.handle, layer, _ptr(idx), _ptr(n_kept), _stream(stream)))
+
+    def rewind(self, n: int, stream=None):
+        """Drop the last ``n`` positions of every sequence of every anchor."""
+        check(self.lib.kvk_rewind(self.handle, n, _stream(stream)))
+
+    # -- reads ---------------------------------------------------------------
+    def plan_splits(self, layer: int) -> int:
+        out = ctypes.c_int32()
+        check(self.lib.kvk_decode_plan_splits(self.handle, layer, ctypes.byref(out)))
+        return out.value
+
+    def decode(self, layer: int, q: torch.Tensor, scale: float, out: torch.Tensor = None,
+               n_splits: int = 0, stream=None) -> torch.Tensor:
+        _need(q, "q")
+        if out is None:
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        check(self.lib.kvk_decode_attention(self.handle, layer, _ptr(q), _dtype_code(q),
+                                            float(scale), _ptr(out), n_splits, _stream(stream)))
+        return out
+
+    def decode_partial(self, layer: int, q: torch.Tensor, scale: float, n_splits: int,
+                       partials: torch.Tensor = None, stream=None) -> torch.Tensor:
+        _need(q, "q")
+        B, Hq, D = q.shape
+        if partials is None:
+            partials = torch.empty((n_splits, B * Hq, D + 2), dtype=torch.float32, device=q.device)
+        check(self.lib.kvk_decode_partial(self.handle, layer, _ptr(q), _dtype_code(q), float(scale),
+                                          _ptr(partials), n_splits, _stream(stream)))
+        return partials
+
+    def decode_mla(self, layer: int, q_nope, q_pe, w_uk, w_uv, scale: float, out=None,
+                   n_splits: int = 0, stream=None) -> torch.Tensor:
+        for t, nm in ((q_nope, "q_nope"), (q_pe, "q_pe"), (w_uk, "w_uk"), (w_uv, "w_uv")):
+            _need(t, nm)
+        if out is None:
+            out = torch.empty(q_nope.shape, dtype=torch.float32, device=q_nope.device)
+        check(self.lib.kvk_decode_attention_mla(self.handle, layer, _ptr(q_nope), _ptr(q_pe),
+                                                _ptr(w_uk), _ptr(w_uv), float(scale), _ptr(out),
+                                                n_splits, _stream(stream)))
+        return out
+
+    def export(self, layer: int, stream=None) -> dict:
+        """Stored state of anchor ``layer`` in canonical order (device tensors)."""
+        d = self.desc
+        L = self.layers[layer]
+        B, T = d.max_batch, d.max_ctx
+        dev = self.device
+        res = {}
+        if self.kind == "mla":
+            res["c"] = torch.empty((B, T, L.width), dtype=torch.bfloat16, device=dev)
+            res["k_r"] = torch.empty((B, T, d.rope_dim), dtype=torch.bfloat16, device=dev)
+            check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["c"]), _ptr(res["k_r"]),
+                                            None, None, None, None, None, _stream(stream)))
+            return res
+        H, D = d.n_kv_heads, d.head_dim
+        if L.bits == 16:
+            res["k"] = torch.empty((B, H, T, D), dtype=torch.bfloat16, device=dev)
+            res["v"] = torch.empty((B, H, T, D), dtype=torch.bfloat16, device=dev)
+            check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["k"]), _ptr(res["v"]),
+                                            None, None, None, None, None, _stream(stream)))
+            return res
+        g = L.group
+        res["k_codes"] = torch.empty((B, H, T, D), dtype=torch.uint8, device=dev)
+        res["v_codes"] = torch.empty((B, H, T, D), dtype=torch.uint8, device=dev)
+        res["v_scale"] = torch.empty((B, H, T, D // g), dtype=torch.float32, device=dev)
+        res["v_zero"] = torch.empty((B, H, T, D // g), dtype=torch.float32, device=dev)
+        if L.key_axis == "channel":
+            res["k_scale"] = torch.empty((B, H, T // g, D), dtype=torch.float32, device=dev)
+            res["k_zero"] = torch.empty((B, H, T // g, D), dtype=torch.float32, device=dev)
+            res["k_residual"] = torch.empty((B, H, g, D), dtype=torch.bfloat16, device=dev)
+        else:
+            res["k_scale"] = torch.empty((B, H, T, D // g), dtype=torch.float32, device=dev)
+            res["k_zero"] = torch.empty((B, H, T, D // g), dtype=torch.float32, device=dev)
+            res["k_residual"] = None
+        check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["k_codes"]), _ptr(res["v_codes"]),
+                                        _ptr(res["k_scale"]), _ptr(res["k_zero"]), _ptr(res["v_scale"]),
+                                        _ptr(res["v_zero"]), _ptr(res["k_residual"]), _stream(stream)))
+        return res
+
+    def device_error(self, stream=None) -> int:
+        """Synchronise, read and clear the device error word (0 = none)."""
+        code = ctypes.c_int32()
+        st = self.lib.kvk_get_device_error(self.handle, _stream(stream), ctypes.byref(code))
+        if st not in (0, 7):
+            check(st)
+        return code.value
+
+
+def splitk_reduce(partials: torch.Tensor, out: torch.Tensor = None, stream=None) -> torch.Tensor:
+    """Merge ``[n_splits, rows, dim + 2]`` partials into ``[rows, dim]``."""
+    _need(partials, "partials")
+    S, R, W = partials.shape
+    if out is None:
+        out = torch.empty((R, W - 2), dtype=torch.float32, device=partials.device)
+    check(load().kvk_splitk_reduce(_ptr(partials), S, R, W - 2, _ptr(out), _stream(stream)))
+    return out

@@ -1,0 +1,31 @@
+// decode_gqa.cu -- dispatch of the GQA decode kernel by cache format.
+#include "kernels.h"
+
+namespace kvk {
+
+cudaError_t launch_gqa_decode_b16(const GqaDecodeArgs &a, cudaStream_t st);
+cudaError_t launch_gqa_decode_b8(const GqaDecodeArgs &a, cudaStream_t st);
+cudaError_t launch_gqa_decode_b4(const GqaDecodeArgs &a, cudaStream_t st);
+int gqa_ctas_b16(int D, int kax, int gs);
+int gqa_ctas_b8(int D, int kax, int gs);
+int gqa_ctas_b4(int D, int kax, int gs);
+
+cudaError_t launch_gqa_decode(const GqaDecodeArgs &a, cudaStream_t st) {
+  switch (a.v.bits) {
+    case 16: return launch_gqa_decode_b16(a, st);
+    case 8: return launch_gqa_decode_b8(a, st);
+    case 4: return launch_gqa_decode_b4(a, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+int gqa_decode_ctas_per_sm(int bits, int D, int key_axis, int group) {
+  switch (bits) {
+    case 16: return gqa_ctas_b16(D, key_axis, group);
+    case 8: return gqa_ctas_b8(D, key_axis, group);
+    case 4: return gqa_ctas_b4(D, key_axis, group);
+    default: return 1;
+  }
+}
+
+}  // namespace kvk

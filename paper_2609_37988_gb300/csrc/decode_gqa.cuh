@@ -1,0 +1,619 @@
+// decode_gqa.cuh -- split-K decode attention over one GQA anchor (sm_103a).
+//
+// Computes, for every query head h of sequence b (Sec. 2.1 GQA; the depth
+// axis only changes which anchor is read):
+//     out[b,h] = sum_t softmax_t(sigma <q[b,h], k_t>) v_t ,  k_t/v_t of KV head h/G
+// over the positions of b (or its kept list, Sec. 3.3), with k_t and v_t
+// dequantised on the fly (grouped asymmetric codes, Appendix C.3).
+//
+// Grid (split, kv head, batch); 4 warps per CTA; each CTA streams its
+// context split in tiles of 64 positions through a cp.async ring of NST
+// shared-memory stages (16-byte copies; an eviction list turns the same
+// copies into a gather).  Warp w owns tile rows [16w, 16w+16) and keeps its
+// own online-softmax state; the four states merge in shared memory at the
+// end and either write the output (one split) or a split-K partial.
+//
+// Both products run on the tensor cores with mma.m16n8k16 (fp32 accumulate):
+//   scores  S^T[16 pos x 8 heads] = K[16 x 16 ch] * Q^T, the G <= 8 query
+//           heads of the KV head share one read of every key byte;
+//   values  O^T[16 ch x 8 heads] += V^T[16 ch x 16 pos] * P^T.
+// Codes enter the MMA as exact f16 integers (the exponent-bias trick:
+// 0x6400 | c is the half 1024 + c).  Scale and zero stay fp32 and are
+// applied outside the MMA, so quantised operands lose nothing:
+//   keys, per-token groups:   s_t = sum_g sc_tg (D'_tg - Qoff_g) + z_tg Qs_g
+//   keys, per-channel groups: scale folded into the query per group of
+//                             positions, zero term  sum_i q_i z_Gi
+//   values: P'_g = p * sc_tg per channel group (hi/lo f16 split), plus
+//           sum_t p_t z_tg added once at the end.
+// bf16 caches multiply bf16 operands directly; P is split into hi + lo
+// bf16 halves so the value product keeps ~16 significant bits.
+#pragma once
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "layout.h"
+
+namespace kvk {
+
+template <int BITS, int D, int KAX, int GS>
+struct GqaCfg {
+  static constexpr bool BF = (BITS == 16);
+  static constexpr bool QUANT = !BF;
+  static constexpr bool KPT = QUANT && KAX == 0;  // per-token key meta in record
+  static constexpr bool KPC = QUANT && KAX == 1;  // per-channel key groups
+  static constexpr int KS = D / 16;               // k-steps (= value M-blocks)
+  static constexpr int NG = QUANT ? D / GS : 1;   // channel groups per row
+  static constexpr int KB = D * BITS / 8;         // K (and V) section bytes
+  static constexpr int MB = QUANT ? ((NG * 8 + 15) & ~15) : 0;
+  static constexpr int REC = 2 * KB + (KPT ? MB : 0) + (QUANT ? MB : 0);
+  static constexpr int CPR = REC / 16;            // 16-byte chunks per record
+  static constexpr int SK = KB / 4;               // bytes of one lane's K segment
+  static constexpr int NWK = SK / 4;              // words of one lane's K segment
+  static constexpr int SV = KB / 8;               // bytes of one lane's V segment
+  static constexpr int NWV = SV / 4;
+  // shared-memory planes of one stage (row = tile position)
+  static constexpr int KSTR = KB;
+  static constexpr bool KSWZ = KB >= 128;
+  static constexpr int VSTR = KB >= 128 ? KB : (KB == 64 ? 80 : 48);
+  static constexpr int VSWZ = KB >= 256 ? 2 : (KB == 128 ? 1 : 0);
+  static constexpr int KP_OFF = 0;
+  static constexpr int VP_OFF = KP_OFF + kTile * KSTR;
+  static constexpr int KM_OFF = VP_OFF + kTile * VSTR;
+  static constexpr int VM_OFF = KM_OFF + (KPT ? kTile * MB : 0);
+  static constexpr int KG_OFF = VM_OFF + (QUANT ? kTile * MB : 0);
+  static constexpr int KG_ROWS = KPC ? kTile / GS : 0;
+  static constexpr int STAGE = KG_OFF + KG_ROWS * D * 8;
+  static constexpr int NST = STAGE >= 24576 ? 3 : 4;
+  static constexpr int Q_BYTES = 8 * D * 4;
+  static constexpr int SMEM = Q_BYTES + NST * STAGE;
+  static_assert(REC % 16 == 0, "records are 16-byte multiples");
+  static_assert(!QUANT || (GS % 16 == 0 && D % GS == 0), "groups are whole k-steps");
+  static_assert(4 * 8 * (D + 2) * 4 <= NST * STAGE, "merge scratch fits the stages");
+};
+
+__device__ __forceinline__ int kswz(bool on, int t, int u) { return on ? (u ^ ((t & 1) << 2)) : u; }
+__device__ __forceinline__ int vswz(int mode, int t, int u) {
+  if (mode == 1) return u ^ (t & 6);
+  if (mode == 2) return u ^ (((t >> 1) & 1) | (((t >> 2) & 1) << 2));
+  return u;
+}
+
+// f16 pair (1024 + lo, 1024 + hi) from two bytes picked by `sel` (PRMT).
+__device__ __forceinline__ uint32_t u8pair_f16(uint32_t x, uint32_t sel) {
+  return __byte_perm(x, 0x64646464u, sel);
+}
+__device__ __forceinline__ uint32_t nib_f16(uint32_t x, uint32_t mask) {
+  return (x & mask) | 0x64006400u;
+}
+
+template <int BITS, int D, int KAX, int GS>
+__global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) {
+  using C = GqaCfg<BITS, D, KAX, GS>;
+  constexpr bool BF = C::BF;
+  constexpr int KS = C::KS, NG = C::NG;
+  extern __shared__ __align__(128) uint8_t smem[];
+  float *q_s = reinterpret_cast<float *>(smem);
+  uint8_t *stages = smem + C::Q_BYTES;
+
+  const GqaView &v = a.v;
+  const int split = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, c = lane & 3;
+  const int len = v.lens[b];
+  const int n_items = a.gather ? min(v.kept_n[b], v.kept_cap) : len;
+  const int i0 = split * a.items_per_split;
+  // the last split runs to the end, so a launch recorded for shorter
+  // sequences (a replayed graph) still covers every position
+  const int i1 = (split == a.n_splits - 1) ? n_items : min(i0 + a.items_per_split, n_items);
+  const int Tq = C::KPC ? (len / GS) * GS : len;  // positions held as codes
+  const bool use_lo = a.q_f32 != 0;
+  const int32_t *kept = v.kept_idx + (size_t)b * v.kept_cap;
+
+  for (int e = tid; e < 8 * D; e += 128) {
+    const int h = e / D, ch = e % D;
+    float x = 0.f;
+    if (h < a.G) {
+      const size_t qi = ((size_t)b * a.Hq + (size_t)kvh * a.G + h) * D + ch;
+      x = a.q_f32 ? static_cast<const float *>(a.q)[qi]
+                  : bf16_to_f32(static_cast<const uint16_t *>(a.q)[qi]);
+    }
+    q_s[e] = x;
+  }
+  __syncthreads();
+
+  // ---- query fragments (B operand of the score MMA), head n = g ----------
+  uint32_t qb[KS][2], qbl[KS][2];
+  if constexpr (!C::KPC) {
+#pragma unroll
+    for (int js = 0; js < KS; ++js) {
+      const float *qh = q_s + g * D + 16 * js;
+      float x2 = qh[2 * c + 8], x3 = qh[2 * c + 9];
+      if (BITS == 4) { x2 *= 0.0625f; x3 *= 0.0625f; }
+      split2<BF>(qh[2 * c], qh[2 * c + 1], qb[js][0], qbl[js][0]);
+      split2<BF>(x2, x3, qb[js][1], qbl[js][1]);
+    }
+  }
+  // per-token key groups: query sums Qs and the 1024-bias offsets Qoff for
+  // the two heads (2c, 2c+1) of this lane's accumulator columns.
+  float qs[NG][2], qoff[NG][2];
+  if constexpr (C::KPT) {
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const float *qh = q_s + (2 * c + hh) * D;
+        float sq = 0.f, so = 0.f;
+        for (int ch = gi * GS; ch < (gi + 1) * GS; ++ch) {
+          const bool hs = (BITS == 4) && ((ch & 15) >= 8);
+          const float xs = hs ? qh[ch] * 0.0625f : qh[ch];
+          const __half hi = __float2half_rn(xs);
+          float xe = __half2float(hi);
+          if (use_lo) xe += __half2float(__float2half_rn(xs - xe));
+          sq += hs ? 16.f * xe : xe;
+          so += 1024.f * xe;
+        }
+        qs[gi][hh] = sq;
+        qoff[gi][hh] = so;
+      }
+  }
+
+  float acc[KS][4];
+#pragma unroll
+  for (int m = 0; m < KS; ++m) acc[m][0] = acc[m][1] = acc[m][2] = acc[m][3] = 0.f;
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float zacc[NG][2];
+#pragma unroll
+  for (int gi = 0; gi < NG; ++gi) zacc[gi][0] = zacc[gi][1] = 0.f;
+
+  const size_t slab = (size_t)b * v.Hkv + kvh;
+  const uint8_t *rec = v.rec + slab * (size_t)v.cap * C::REC;
+  const float2 *gmeta = C::KPC ? v.gmeta + slab * (size_t)(v.cap / GS) * D : nullptr;
+  const int n_tiles = i1 > i0 ? (i1 - i0 + kTile - 1) / kTile : 0;
+
+  // ---- producer: one tile of records into one stage ----------------------
+  auto issue = [&](int t, int s) {
+    const int base = i0 + t * kTile;
+    uint8_t *st = stages + s * C::STAGE;
+    for (int q = tid; q < kTile * C::CPR; q += 128) {
+      const int row = q / C::CPR, u = q - row * C::CPR;
+      const int item = base + row;
+      bool valid = item < i1;
+      int pos = item;
+      if (a.gather && valid) {
+        pos = kept[item];
+        if (pos < 0 || pos >= len) {
+          valid = false;
+          if (u == 0) set_err(a.err, 1);
+        }
+      }
+      const uint8_t *src = rec + (size_t)(valid ? pos : 0) * C::REC + 16 * u;
+      uint8_t *dst;
+      const int ub = 16 * u;
+      if (ub < C::KB) {
+        dst = st + C::KP_OFF + row * C::KSTR + 16 * kswz(C::KSWZ, row, u);
+      } else if (ub < 2 * C::KB) {
+        dst = st + C::VP_OFF + row * C::VSTR + 16 * vswz(C::VSWZ, row, u - C::KB / 16);
+      } else if (C::KPT && ub < 2 * C::KB + C::MB) {
+        dst = st + C::KM_OFF + row * C::MB + (ub - 2 * C::KB);
+      } else {
+        dst = st + C::VM_OFF + row * C::MB + (ub - 2 * C::KB - (C::KPT ? C::MB : 0));
+      }
+      cp_async16(dst, src, valid);
+    }
+    if constexpr (C::KPC) {
+      const int g0 = base / GS;
+      constexpr int CPRow = D * 8 / 16;
+      for (int q = tid; q < C::KG_ROWS * CPRow; q += 128) {
+        const int row = q / CPRow, u = q - row * CPRow;
+        const int G = g0 + row;
+        const bool valid = (G + 1) * GS <= len;
+        const uint8_t *src =
+            reinterpret_cast<const uint8_t *>(gmeta + (size_t)(valid ? G : 0) * D) + 16 * u;
+        cp_async16(st + C::KG_OFF + row * D * 8 + 16 * u, src, valid);
+      }
+    }
+  };
+
+  // ---- consumer: one warp's 16 rows of one stage --------------------------
+  auto compute = [&](int t, int s) {
+    const int base = i0 + t * kTile;
+    const int r0 = 16 * warp;
+    if (base + r0 >= i1) return;  // warp-uniform: no live row
+    const uint8_t *st = stages + s * C::STAGE;
+    const int tA = r0 + g, tB = tA + 8;
+    bool vA = base + tA < i1, vB = base + tB < i1;
+    if (a.gather) {
+      if (vA) { const int p = kept[base + tA]; vA = p >= 0 && p < len; }
+      if (vB) { const int p = kept[base + tB]; vB = p >= 0 && p < len; }
+    }
+    float s4[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint8_t *Kp = st + C::KP_OFF;
+
+    // lane's K words for rows tA / tB
+    auto load_k = [&](int t, uint32_t(&w)[C::NWK]) {
+      if constexpr (C::SK >= 16) {
+#pragma unroll
+        for (int i = 0; i < C::SK / 16; ++i) {
+          const uint4 x = *reinterpret_cast<const uint4 *>(Kp + t * C::KSTR +
+                                                           16 * kswz(C::KSWZ, t, 4 * i + c));
+          w[4 * i] = x.x; w[4 * i + 1] = x.y; w[4 * i + 2] = x.z; w[4 * i + 3] = x.w;
+        }
+      } else {
+        const uint2 x = *reinterpret_cast<const uint2 *>(Kp + t * C::KSTR + 8 * c);
+        w[0] = x.x; w[1] = x.y;
+      }
+    };
+    // A fragment registers (a0..a3) of k-step js from the two rows' words
+    auto kfrag = [&](const uint32_t(&wa)[C::NWK], const uint32_t(&wb)[C::NWK], int js,
+                     uint32_t &a0, uint32_t &a1, uint32_t &a2, uint32_t &a3) {
+      if constexpr (BITS == 16) {
+        a0 = wa[2 * js]; a2 = wa[2 * js + 1]; a1 = wb[2 * js]; a3 = wb[2 * js + 1];
+      } else if constexpr (BITS == 8) {
+        a0 = u8pair_f16(wa[js], 0x4140); a2 = u8pair_f16(wa[js], 0x4342);
+        a1 = u8pair_f16(wb[js], 0x4140); a3 = u8pair_f16(wb[js], 0x4342);
+      } else {
+        const int sh = (js & 1) * 8;
+        const uint32_t xa = wa[js >> 1] >> sh, xb = wb[js >> 1] >> sh;
+        a0 = nib_f16(xa, 0x000F000Fu); a2 = nib_f16(xa, 0x00F000F0u);
+        a1 = nib_f16(xb, 0x000F000Fu); a3 = nib_f16(xb, 0x00F000F0u);
+      }
+    };
+
+    if (C::KPC && base + r0 >= Tq) {
+      // open per-channel key group: bf16 rows of the residual plane, plain
+      // fp32 dot products (at most group-1 positions per sequence).
+      const uint8_t *res = v.resid + slab * (size_t)GS * D * 2;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int t = (k < 2 ? tA : tB);
+        const bool ok = (k < 2 ? vA : vB);
+        const int h = 2 * c + (k & 1);
+        float d = 0.f;
+        if (ok) {
+          const uint8_t *row = res + (size_t)((base + t) % GS) * D * 2;
+          for (int ch = 0; ch < D; ++ch) {
+            int by, hi;
+            k_pos(ch, 16, D, &by, &hi);
+            d += q_s[h * D + ch] * bf16_to_f32(*reinterpret_cast<const uint16_t *>(row + by));
+          }
+        }
+        s4[k] = d;
+      }
+    } else if constexpr (C::KPC) {
+      // scale of each channel folded into the query for this group of
+      // positions; zero point and 1024-bias enter as one per-head constant.
+      const float2 *kg = reinterpret_cast<const float2 *>(st + C::KG_OFF) + (r0 / GS) * D;
+      uint32_t pb[KS][2], pbl[KS][2];
+      float zpart = 0.f, opart = 0.f;
+#pragma unroll
+      for (int js = 0; js < KS; ++js) {
+        const float *qh = q_s + g * D + 16 * js;
+        const float2 *sz = kg + 16 * js;
+        float x[4];
+        const int chs[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 m2 = sz[chs[e]];
+          zpart += qh[chs[e]] * m2.y;
+          x[e] = qh[chs[e]] * m2.x;
+          if (BITS == 4 && e >= 2) x[e] *= 0.0625f;
+        }
+        split2<false>(x[0], x[1], pb[js][0], pbl[js][0]);
+        split2<false>(x[2], x[3], pb[js][1], pbl[js][1]);
+        const float2 h0 = unpack2<false>(pb[js][0]), l0 = unpack2<false>(pbl[js][0]);
+        const float2 h1 = unpack2<false>(pb[js][1]), l1 = unpack2<false>(pbl[js][1]);
+        opart += 1024.f * ((h0.x + l0.x) + (h0.y + l0.y) + (h1.x + l1.x) + (h1.y + l1.y));
+      }
+      zpart += __shfl_xor_sync(0xffffffffu, zpart, 1);
+      zpart += __shfl_xor_sync(0xffffffffu, zpart, 2);
+      opart += __shfl_xor_sync(0xffffffffu, opart, 1);
+      opart += __shfl_xor_sync(0xffffffffu, opart, 2);
+      const float corr = zpart - opart;  // head g
+      const float corr0 = __shfl_sync(0xffffffffu, corr, (2 * c) * 4);
+      const float corr1 = __shfl_sync(0xffffffffu, corr, (2 * c + 1) * 4);
+      uint32_t wa[C::NWK], wb[C::NWK];
+      load_k(tA, wa);
+      load_k(tB, wb);
+      float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int js = 0; js < KS; ++js) {
+        uint32_t a0, a1, a2, a3;
+        kfrag(wa, wb, js, a0, a1, a2, a3);
+        mma_f16(d, a0, a1, a2, a3, pb[js][0], pb[js][1]);
+        mma_f16(d, a0, a1, a2, a3, pbl[js][0], pbl[js][1]);
+      }
+      s4[0] = d[0] + corr0; s4[1] = d[1] + corr1;
+      s4[2] = d[2] + corr0; s4[3] = d[3] + corr1;
+    } else {
+      uint32_t wa[C::NWK], wb[C::NWK];
+      load_k(tA, wa);
+      load_k(tB, wb);
+      if constexpr (BF) {
+        float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int js = 0; js < KS; ++js) {
+          uint32_t a0, a1, a2, a3;
+          kfrag(wa, wb, js, a0, a1, a2, a3);
+          mma_bf16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
+          if (use_lo) mma_bf16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) s4[k] = d[k];
+      } else {
+        const float2 *kmA = reinterpret_cast<const float2 *>(st + C::KM_OFF + tA * C::MB);
+        const float2 *kmB = reinterpret_cast<const float2 *>(st + C::KM_OFF + tB * C::MB);
+        constexpr int JPG = GS / 16;  // k-steps per group
+#pragma unroll
+        for (int gi = 0; gi < NG; ++gi) {
+          float d[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int jj = 0; jj < JPG; ++jj) {
+            const int js = gi * JPG + jj;
+            uint32_t a0, a1, a2, a3;
+            kfrag(wa, wb, js, a0, a1, a2, a3);
+            mma_f16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
+            if (use_lo) mma_f16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
+          }
+          const float2 mA = kmA[gi], mB = kmB[gi];
+          s4[0] += mA.x * (d[0] - qoff[gi][0]) + mA.y * qs[gi][0];
+          s4[1] += mA.x * (d[1] - qoff[gi][1]) + mA.y * qs[gi][1];
+          s4[2] += mB.x * (d[2] - qoff[gi][0]) + mB.y * qs[gi][0];
+          s4[3] += mB.x * (d[3] - qoff[gi][1]) + mB.y * qs[gi][1];
+        }
+      }
+    }
+
+    // ---- online softmax (base-2 exponent, lazy rescaling) ------------------
+    float x[4];
+    x[0] = vA ? s4[0] * a.sig_log2 : -INFINITY;
+    x[1] = vA ? s4[1] * a.sig_log2 : -INFINITY;
+    x[2] = vB ? s4[2] * a.sig_log2 : -INFINITY;
+    x[3] = vB ? s4[3] * a.sig_log2 : -INFINITY;
+    float mt0 = fmaxf(x[0], x[2]), mt1 = fmaxf(x[1], x[3]);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      mt0 = fmaxf(mt0, __shfl_xor_sync(0xffffffffu, mt0, off));
+      mt1 = fmaxf(mt1, __shfl_xor_sync(0xffffffffu, mt1, off));
+    }
+    // Keep a stale maximum while the tile stays within 2^8 of it: the
+    // result is exact either way, and rescaling is skipped on most tiles.
+    const bool need = (mt0 > m_run[0] + 8.f) || (mt1 > m_run[1] + 8.f);
+    if (__any_sync(0xffffffffu, need)) {
+      const float n0 = fmaxf(m_run[0], mt0), n1 = fmaxf(m_run[1], mt1);
+      const float al0 = (n0 == -INFINITY) ? 1.f : exp2f(m_run[0] - n0);
+      const float al1 = (n1 == -INFINITY) ? 1.f : exp2f(m_run[1] - n1);
+#pragma unroll
+      for (int m = 0; m < KS; ++m) {
+        acc[m][0] *= al0; acc[m][2] *= al0;
+        acc[m][1] *= al1; acc[m][3] *= al1;
+      }
+      l_run[0] *= al0; l_run[1] *= al1;
+#pragma unroll
+      for (int gi = 0; gi < NG; ++gi) { zacc[gi][0] *= al0; zacc[gi][1] *= al1; }
+      m_run[0] = n0; m_run[1] = n1;
+    }
+    float p[4];
+    p[0] = (m_run[0] == -INFINITY) ? 0.f : exp2f(x[0] - m_run[0]);
+    p[1] = (m_run[1] == -INFINITY) ? 0.f : exp2f(x[1] - m_run[1]);
+    p[2] = (m_run[0] == -INFINITY) ? 0.f : exp2f(x[2] - m_run[0]);
+    p[3] = (m_run[1] == -INFINITY) ? 0.f : exp2f(x[3] - m_run[1]);
+    l_run[0] += p[0] + p[2];
+    l_run[1] += p[1] + p[3];
+
+    // ---- P^T fragments (B operand of the value MMA) ------------------------
+    // P' = p * scale per channel group (quantised) or P (bf16), split hi/lo,
+    // transposed from the score accumulator layout with movmatrix.
+    uint32_t pf[NG][4];
+    if constexpr (BF) {
+      uint32_t ht, lt, hb, lb;
+      split2<true>(p[0], p[1], ht, lt);
+      split2<true>(p[2], p[3], hb, lb);
+      pf[0][0] = movmatrix_t(ht); pf[0][1] = movmatrix_t(hb);
+      pf[0][2] = movmatrix_t(lt); pf[0][3] = movmatrix_t(lb);
+    } else {
+      const float2 *vmA = reinterpret_cast<const float2 *>(st + C::VM_OFF + tA * C::MB);
+      const float2 *vmB = reinterpret_cast<const float2 *>(st + C::VM_OFF + tB * C::MB);
+#pragma unroll
+      for (int gi = 0; gi < NG; ++gi) {
+        const float2 mA = vmA[gi], mB = vmB[gi];
+        uint32_t ht, lt, hb, lb;
+        split2<false>(p[0] * mA.x, p[1] * mA.x, ht, lt);
+        split2<false>(p[2] * mB.x, p[3] * mB.x, hb, lb);
+        pf[gi][0] = movmatrix_t(ht); pf[gi][1] = movmatrix_t(hb);
+        pf[gi][2] = movmatrix_t(lt); pf[gi][3] = movmatrix_t(lb);
+        zacc[gi][0] += p[0] * mA.y + p[2] * mB.y;
+        zacc[gi][1] += p[1] * mA.y + p[3] * mB.y;
+      }
+    }
+
+    // ---- value product: A = V^T from the lane's segments of 4 positions ----
+    const uint8_t *Vp = st + C::VP_OFF;
+    const int T0 = r0 + 2 * c, T1 = T0 + 1, T2 = T0 + 8, T3 = T0 + 9;
+    auto vload16 = [&](int t, int k) {  // k-th 16-byte chunk of lane g's segment
+      const int u = g * (C::SV / 16) + k;
+      return *reinterpret_cast<const uint4 *>(Vp + t * C::VSTR + 16 * vswz(C::VSWZ, t, u));
+    };
+    if constexpr (BITS == 16) {
+      // one word per M-block: (row g, row g+8) of one position
+#pragma unroll
+      for (int k = 0; k < C::SV / 16; ++k) {
+        const uint4 w0 = vload16(T0, k), w1 = vload16(T1, k), w2 = vload16(T2, k),
+                    w3 = vload16(T3, k);
+        const uint32_t x0[4] = {w0.x, w0.y, w0.z, w0.w}, x1[4] = {w1.x, w1.y, w1.z, w1.w};
+        const uint32_t x2[4] = {w2.x, w2.y, w2.z, w2.w}, x3[4] = {w3.x, w3.y, w3.z, w3.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int m = 4 * k + q;
+          const uint32_t a0 = __byte_perm(x0[q], x1[q], 0x5410);
+          const uint32_t a1 = __byte_perm(x0[q], x1[q], 0x7632);
+          const uint32_t a2 = __byte_perm(x2[q], x3[q], 0x5410);
+          const uint32_t a3 = __byte_perm(x2[q], x3[q], 0x7632);
+          mma_bf16(acc[m], a0, a1, a2, a3, pf[0][0], pf[0][1]);
+          mma_bf16(acc[m], a0, a1, a2, a3, pf[0][2], pf[0][3]);
+        }
+      }
+    } else {
+      uint32_t w[4][C::NWV];
+      const int Ts[4] = {T0, T1, T2, T3};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if constexpr (C::SV >= 16) {
+#pragma unroll
+          for (int k = 0; k < C::SV / 16; ++k) {
+            const uint4 x = vload16(Ts[i], k);
+            w[i][4 * k] = x.x; w[i][4 * k + 1] = x.y; w[i][4 * k + 2] = x.z; w[i][4 * k + 3] = x.w;
+          }
+        } else if constexpr (C::SV == 8) {
+          const uint2 x = *reinterpret_cast<const uint2 *>(Vp + Ts[i] * C::VSTR + 8 * g);
+          w[i][0] = x.x; w[i][1] = x.y;
+        } else {
+          w[i][0] = *reinterpret_cast<const uint32_t *>(Vp + Ts[i] * C::VSTR + 4 * g);
+        }
+      }
+      const uint32_t k1024 = 0x64006400u;
+      auto vmma = [&](int m, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3) {
+        a0 = hsub2_u32(a0, k1024); a1 = hsub2_u32(a1, k1024);
+        a2 = hsub2_u32(a2, k1024); a3 = hsub2_u32(a3, k1024);
+        const int gi = (16 * m) / GS;
+        mma_f16(acc[m], a0, a1, a2, a3, pf[gi][0], pf[gi][1]);
+        mma_f16(acc[m], a0, a1, a2, a3, pf[gi][2], pf[gi][3]);
+      };
+      if constexpr (BITS == 8) {
+        // word k of a segment: M-blocks 2k (bytes 0,1) and 2k+1 (bytes 2,3)
+#pragma unroll
+        for (int k = 0; k < C::NWV; ++k) {
+          const uint32_t X0 = __byte_perm(w[0][k], w[1][k], 0x5140);
+          const uint32_t X2 = __byte_perm(w[2][k], w[3][k], 0x5140);
+          const uint32_t Y0 = __byte_perm(w[0][k], w[1][k], 0x7362);
+          const uint32_t Y2 = __byte_perm(w[2][k], w[3][k], 0x7362);
+          vmma(2 * k, u8pair_f16(X0, 0x4140), u8pair_f16(X0, 0x4342), u8pair_f16(X2, 0x4140),
+               u8pair_f16(X2, 0x4342));
+          vmma(2 * k + 1, u8pair_f16(Y0, 0x4140), u8pair_f16(Y0, 0x4342),
+               u8pair_f16(Y2, 0x4140), u8pair_f16(Y2, 0x4342));
+        }
+      } else {
+        // word k of a segment: M-blocks 4k..4k+3, one byte each (row g low
+        // nibble, row g+8 high nibble -> 16x, undone at the end)
+#pragma unroll
+        for (int k = 0; k < C::NWV; ++k) {
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            const uint32_t sel = hh ? 0x7632 : 0x5410;
+            uint32_t X0 = __byte_perm(w[0][k], w[1][k], sel);
+            uint32_t X2 = __byte_perm(w[2][k], w[3][k], sel);
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const int m = 4 * k + 2 * hh + q;
+              vmma(m, nib_f16(X0, 0x000F000Fu), nib_f16(X0, 0x00F000F0u),
+                   nib_f16(X2, 0x000F000Fu), nib_f16(X2, 0x00F000F0u));
+              X0 >>= 8;
+              X2 >>= 8;
+            }
+          }
+        }
+      }
+    }
+  };
+
+  // ---- cp.async ring over the split's tiles --------------------------------
+#pragma unroll
+  for (int s = 0; s < C::NST - 1; ++s) {
+    if (s < n_tiles) issue(s, s);
+    cp_async_commit();
+  }
+  for (int t = 0; t < n_tiles; ++t) {
+    cp_async_wait<C::NST - 2>();
+    __syncthreads();
+    const int nt = t + C::NST - 1;
+    if (nt < n_tiles) issue(nt, nt % C::NST);
+    cp_async_commit();
+    compute(t, t % C::NST);
+  }
+  cp_async_wait<0>();
+  __syncthreads();
+
+  // ---- finish this warp's state ------------------------------------------
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    l_run[0] += __shfl_xor_sync(0xffffffffu, l_run[0], off);
+    l_run[1] += __shfl_xor_sync(0xffffffffu, l_run[1], off);
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi) {
+      zacc[gi][0] += __shfl_xor_sync(0xffffffffu, zacc[gi][0], off);
+      zacc[gi][1] += __shfl_xor_sync(0xffffffffu, zacc[gi][1], off);
+    }
+  }
+  float *red = reinterpret_cast<float *>(stages);  // [4 warps][8 heads][D + 2]
+  constexpr int RS = D + 2;
+#pragma unroll
+  for (int m = 0; m < KS; ++m) {
+    const int ch0 = 16 * m + g, ch1 = ch0 + 8;
+    const int gi = C::QUANT ? (16 * m) / GS : 0;
+    const float hs = (BITS == 4) ? 0.0625f : 1.f;
+    const float z0 = C::QUANT ? zacc[gi][0] : 0.f, z1 = C::QUANT ? zacc[gi][1] : 0.f;
+    red[(warp * 8 + 2 * c) * RS + ch0] = acc[m][0] + z0;
+    red[(warp * 8 + 2 * c + 1) * RS + ch0] = acc[m][1] + z1;
+    red[(warp * 8 + 2 * c) * RS + ch1] = acc[m][2] * hs + z0;
+    red[(warp * 8 + 2 * c + 1) * RS + ch1] = acc[m][3] * hs + z1;
+  }
+  if (g == 0) {
+    red[(warp * 8 + 2 * c) * RS + D] = m_run[0];
+    red[(warp * 8 + 2 * c) * RS + D + 1] = l_run[0];
+    red[(warp * 8 + 2 * c + 1) * RS + D] = m_run[1];
+    red[(warp * 8 + 2 * c + 1) * RS + D + 1] = l_run[1];
+  }
+  __syncthreads();
+
+  // ---- merge the four warps; write output or split partial ---------------
+  const size_t row0 = (size_t)b * a.Hq + (size_t)kvh * a.G;
+  for (int e = tid; e < a.G * RS; e += 128) {
+    const int h = e / RS, ch = e - h * RS;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, red[(w * 8 + h) * RS + D]);
+    float A = 0.f, L = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float mw = red[(w * 8 + h) * RS + D];
+        const float sc = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+        L += sc * red[(w * 8 + h) * RS + D + 1];
+        if (ch < D) A += sc * red[(w * 8 + h) * RS + ch];
+      }
+    }
+    if (a.out) {
+      if (ch < D) a.out[(row0 + h) * D + ch] = (L > 0.f) ? A / L : 0.f;
+    } else {
+      float *pr = a.partial + ((size_t)split * gridDim.z * a.Hq + row0 + h) * RS;
+      pr[ch] = (ch < D) ? A : (ch == D ? M : L);
+    }
+  }
+}
+
+template <int BITS, int D, int KAX, int GS>
+cudaError_t launch_gqa_decode_t(const GqaDecodeArgs &a, cudaStream_t st) {
+  using C = GqaCfg<BITS, D, KAX, GS>;
+  auto k = gqa_decode_kernel<BITS, D, KAX, GS>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  dim3 grid(a.n_splits, a.v.Hkv, a.v.B);
+  k<<<grid, 128, C::SMEM, st>>>(a);
+  return cudaGetLastError();
+}
+
+template <int BITS, int D, int KAX, int GS>
+int gqa_ctas_per_sm_t() {
+  using C = GqaCfg<BITS, D, KAX, GS>;
+  auto k = gqa_decode_kernel<BITS, D, KAX, GS>;
+  cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 128, C::SMEM) != cudaSuccess) n = 1;
+  return n > 0 ? n : 1;
+}
+
+}  // namespace kvk

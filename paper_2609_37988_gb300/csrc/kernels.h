@@ -1,0 +1,90 @@
+// kernels.h -- launch interface between the host library and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace kvk {
+
+// One GQA anchor as the kernels see it.
+struct GqaView {
+  uint8_t *rec;        // records base
+  float2 *gmeta;       // per-channel key (scale, zero) plane, or null
+  uint8_t *resid;      // per-channel key residual plane, or null
+  int32_t *lens;       // [B]
+  int32_t *counter;    // append completion counter
+  int32_t *kept_n;     // [B]
+  int32_t *kept_idx;   // [B * kept_cap]
+  int64_t cap;         // positions per slab
+  int kept_cap;
+  int B, Hkv, D, bits, group, key_axis, rec_bytes;
+};
+
+struct MlaView {
+  uint8_t *rec;        // [B][cap][(width + rope) bf16]
+  int32_t *lens;
+  int32_t *counter;
+  int64_t cap;
+  int B, width, rope, rec_bytes;
+};
+
+struct GqaDecodeArgs {
+  GqaView v;
+  const void *q;       // [B, Hq, D]
+  int q_f32;           // 1: q is float32, 0: bf16
+  int Hq, G;
+  float sig_log2;      // softmax scale * log2(e)
+  int n_splits;
+  int items_per_split; // multiple of kTile
+  int gather;          // read the kept list
+  float *partial;      // [n_splits, B*Hq, D+2], written when out is null
+  float *out;          // [B, Hq, D]: normalised output (single split)
+  int32_t *err;
+};
+
+// Returns cudaSuccess or the launch error.  Template dispatch on
+// (bits, D, key axis, q dtype) happens inside.
+cudaError_t launch_gqa_decode(const GqaDecodeArgs &a, cudaStream_t st);
+int gqa_decode_ctas_per_sm(int bits, int D, int key_axis, int group);
+
+struct RewindArgs {
+  int32_t *lens[64];
+  int n_anchors, B, n;
+};
+cudaError_t launch_rewind(const RewindArgs &a, cudaStream_t st);
+
+cudaError_t launch_splitk_merge(const float *partials, int n_splits, int n_rows, int dim,
+                                float *out, cudaStream_t st);
+
+// Append n_new rows per sequence (per-sequence counts optional).
+cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, int in_f32,
+                              int n_new, const int32_t *n_per_seq, int32_t *err,
+                              cudaStream_t st);
+cudaError_t launch_mla_append(const MlaView &v, const void *c, const void *kr, int latent,
+                              int n_new, const int32_t *n_per_seq, int32_t *err,
+                              cudaStream_t st);
+
+cudaError_t launch_gqa_export(const GqaView &v, void *k_out, void *v_out, float *k_scale,
+                              float *k_zero, float *v_scale, float *v_zero, void *k_resid,
+                              int max_ctx, cudaStream_t st);
+cudaError_t launch_mla_export(const MlaView &v, void *c_out, void *kr_out, int max_ctx,
+                              cudaStream_t st);
+
+struct MlaDecodeArgs {
+  MlaView v;
+  const void *q_nope;  // bf16 [B, H, Dn]
+  const void *q_pe;    // bf16 [B, H, rope]
+  const void *w_uk;    // bf16 [H, Dn, r]
+  const void *w_uv;    // bf16 [H, Dv, r]
+  int H, Dn, r;
+  float sig_log2;
+  int n_splits, items_per_split;
+  uint16_t *qlat;      // workspace bf16 [B, H, 2*width + rope] (hi | lo | pe)
+  float *partial;      // [n_splits, B*H, width+2]
+  float *olat;         // [B, H, width]
+  float *out;          // [B, H, Dv]
+  int32_t *err;
+};
+cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st);
+int mla_decode_ctas_per_sm(int width);
+
+}  // namespace kvk

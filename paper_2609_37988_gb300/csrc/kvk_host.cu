@@ -1,0 +1,676 @@
+// kvk_host.cu -- host side of the C ABI declared in include/kvk.h.
+//
+// Validates plans (Sec. 2.2: one action per layer, layer 0 owns a cache),
+// resolves every layer's source anchor (Sec. 2.1: nearest anchor at or
+// before it), plans arena layouts, chooses split counts and launches the
+// kernels on the caller's stream.  It never allocates device memory.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/kvk.h"
+#include "kernels.h"
+#include "layout.h"
+
+using namespace kvk;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+kvk_status fail(kvk_status s, const char *fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+kvk_status cuda_fail(cudaError_t e, const char *what) {
+  return fail(KVK_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+kvk_status check_desc(const kvk_model_desc *d, bool need_support = true) {
+  if (!d) return fail(KVK_ERR_INVALID_ARG, "null model descriptor");
+  if (d->kind != KVK_KIND_GQA && d->kind != KVK_KIND_MLA)
+    return fail(KVK_ERR_INVALID_ARG, "unknown model kind %d", d->kind);
+  if (d->n_layers <= 0 || d->n_q_heads <= 0 || d->max_batch <= 0 || d->max_ctx <= 0)
+    return fail(KVK_ERR_INVALID_ARG, "layers, heads, batch and context must be positive");
+  if (d->max_ctx > (1 << 28)) return fail(KVK_ERR_INVALID_ARG, "max_ctx too large");
+  if (d->kind == KVK_KIND_GQA) {
+    if (d->n_kv_heads <= 0 || d->n_q_heads % d->n_kv_heads)
+      return fail(KVK_ERR_INVALID_ARG, "n_q_heads must be a positive multiple of n_kv_heads");
+    if (d->head_dim <= 0) return fail(KVK_ERR_INVALID_ARG, "head_dim must be positive");
+    if (need_support && d->head_dim != 64 && d->head_dim != 128)
+      return fail(KVK_ERR_UNSUPPORTED, "head_dim %d (this build supports 64 and 128)", d->head_dim);
+    if (need_support && d->n_q_heads / d->n_kv_heads > 8)
+      return fail(KVK_ERR_UNSUPPORTED, "more than 8 query heads per KV head");
+  } else {
+    if (d->latent_dim < 8 || d->latent_dim % 8 || d->rope_dim < 0)
+      return fail(KVK_ERR_INVALID_ARG, "latent_dim must be a positive multiple of 8");
+    if (need_support && (d->head_dim != 128 || d->rope_dim != 64))
+      return fail(KVK_ERR_UNSUPPORTED, "MLA needs head_dim 128 and rope_dim 64");
+    if (need_support && d->n_q_heads > 16)
+      return fail(KVK_ERR_UNSUPPORTED, "MLA with more than 16 heads");
+  }
+  return KVK_OK;
+}
+
+kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
+                       bool need_support = true) {
+  if (c->inherit) {
+    if (l == 0) return fail(KVK_ERR_INVALID_CONFIG, "layer 0 must own a cache (it inherits)");
+    return KVK_OK;
+  }
+  if (d->kind == KVK_KIND_MLA) {
+    if (c->bits != 16 && c->bits != 8 && c->bits != 4 && c->bits != 2)
+      return fail(KVK_ERR_INVALID_CONFIG, "layer %d: bits %d not in {16, 8, 4, 2}", l, c->bits);
+    if (need_support && c->bits != 16)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: quantised MLA latents are not in this build", l);
+    const int r = d->latent_dim;
+    if (c->width != r && c->width != r / 2 && c->width != r / 4 && c->width != r / 8)
+      return fail(KVK_ERR_INVALID_CONFIG, "layer %d: width %d not in {r/8, r/4, r/2, r}", l, c->width);
+    if (need_support && c->width != 64 && c->width != 128 && c->width != 256 && c->width != 512)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: width %d (this build: 64..512)", l, c->width);
+    if (need_support && c->evict_capacity)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: eviction lists on MLA layers", l);
+    return KVK_OK;
+  }
+  if (c->bits != 16 && c->bits != 8 && c->bits != 4 && c->bits != 2)
+    return fail(KVK_ERR_INVALID_CONFIG, "layer %d: bits %d not in {16, 8, 4, 2}", l, c->bits);
+  if (c->bits != 16) {
+    if (c->group <= 0 || d->head_dim % c->group)
+      return fail(KVK_ERR_INVALID_CONFIG, "layer %d: group %d must divide head_dim", l, c->group);
+    if (!need_support) return KVK_OK;
+    if (c->bits == 2)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: 2-bit codes are not in this build", l);
+    if (c->group != 32 && c->group != 64)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: group %d (this build: 32, 64)", l, c->group);
+    if (c->value_axis != KVK_AXIS_TOKEN)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: values are quantised per token", l);
+    if (c->key_axis != KVK_AXIS_TOKEN && c->key_axis != KVK_AXIS_CHANNEL)
+      return fail(KVK_ERR_INVALID_CONFIG, "layer %d: unknown key axis", l);
+    if (c->key_axis == KVK_AXIS_CHANNEL && c->evict_capacity)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: per-channel keys with an eviction list", l);
+  }
+  if (c->evict_capacity < 0 || c->evict_capacity > d->max_ctx)
+    return fail(KVK_ERR_INVALID_CONFIG, "layer %d: evict_capacity out of range", l);
+  return KVK_OK;
+}
+
+ArenaLayout layer_layout(const kvk_model_desc *d, const kvk_layer_cfg *c) {
+  const bool mla = d->kind == KVK_KIND_MLA;
+  return arena_layout(mla ? 1 : 0, d->max_batch, mla ? 1 : d->n_kv_heads, d->max_ctx, d->head_dim,
+                      c->bits, c->bits == 16 ? 64 : c->group, c->key_axis, c->evict_capacity,
+                      c->width, d->rope_dim);
+}
+
+struct WsLayout {
+  size_t err, partial, qlat, olat, total;
+};
+
+WsLayout ws_layout(const kvk_model_desc *d, int max_splits) {
+  WsLayout w;
+  size_t off = 0;
+  w.err = off;
+  off += 256;
+  const bool mla = d->kind == KVK_KIND_MLA;
+  const size_t dim = mla ? (size_t)d->latent_dim : (size_t)d->head_dim;
+  w.partial = off;
+  off += align256((int64_t)max_splits * d->max_batch * d->n_q_heads * (dim + 2) * 4);
+  w.qlat = off;
+  if (mla) off += align256((int64_t)d->max_batch * d->n_q_heads * (2 * d->latent_dim + 64) * 2);
+  w.olat = off;
+  if (mla) off += align256((int64_t)d->max_batch * d->n_q_heads * d->latent_dim * 4);
+  w.total = off;
+  return w;
+}
+
+}  // namespace
+
+struct kvk_cache {
+  kvk_model_desc desc;
+  std::vector<kvk_layer_cfg> cfg;
+  std::vector<int> src;
+  std::vector<uint8_t *> arena;
+  std::vector<ArenaLayout> lay;
+  std::vector<long long> len_hi;  // host upper bound on every sequence's length
+  std::vector<int> kept_on;
+  uint8_t *ws;
+  size_t ws_bytes;
+  WsLayout wl;
+  int max_splits;
+  int sm_count;
+  int device;
+  std::vector<int> ctas;  // per layer, decode CTAs per SM (0 = not queried)
+
+  GqaView gqa_view(int l) const {
+    const ArenaLayout &A = lay[l];
+    const kvk_layer_cfg &c = cfg[l];
+    uint8_t *a = arena[l];
+    GqaView v;
+    v.rec = a + A.rec;
+    v.gmeta = A.gmeta >= 0 ? reinterpret_cast<float2 *>(a + A.gmeta) : nullptr;
+    v.resid = A.resid >= 0 ? a + A.resid : nullptr;
+    v.lens = reinterpret_cast<int32_t *>(a + A.lens);
+    v.counter = reinterpret_cast<int32_t *>(a + A.counter);
+    v.kept_n = reinterpret_cast<int32_t *>(a + A.kept_n);
+    v.kept_idx = reinterpret_cast<int32_t *>(a + A.kept_idx);
+    v.cap = A.cap;
+    v.kept_cap = c.evict_capacity;
+    v.B = desc.max_batch;
+    v.Hkv = desc.n_kv_heads;
+    v.D = desc.head_dim;
+    v.bits = c.bits;
+    v.group = c.bits == 16 ? 64 : c.group;
+    v.key_axis = c.bits == 16 ? 0 : c.key_axis;
+    v.rec_bytes = A.rec_bytes;
+    return v;
+  }
+  MlaView mla_view(int l) const {
+    const ArenaLayout &A = lay[l];
+    uint8_t *a = arena[l];
+    MlaView v;
+    v.rec = a + A.rec;
+    v.lens = reinterpret_cast<int32_t *>(a + A.lens);
+    v.counter = reinterpret_cast<int32_t *>(a + A.counter);
+    v.cap = A.cap;
+    v.B = desc.max_batch;
+    v.width = cfg[l].width;
+    v.rope = desc.rope_dim;
+    v.rec_bytes = A.rec_bytes;
+    return v;
+  }
+  int32_t *err() const { return reinterpret_cast<int32_t *>(ws + wl.err); }
+};
+
+namespace {
+
+kvk_status check_layer_index(const kvk_cache *c, int layer) {
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
+  if (layer < 0 || layer >= c->desc.n_layers)
+    return fail(KVK_ERR_INVALID_ARG, "layer %d out of range [0, %d)", layer, c->desc.n_layers);
+  return KVK_OK;
+}
+
+// Split count that best fills the GPU: whole waves of CTAs and equal tile
+// counts per split, preferring fewer splits when two choices are within 1%.
+int choose_splits(int units, int tiles, int slots, int max_splits) {
+  if (tiles <= 1) return 1;
+  const int smax = std::max(1, std::min(max_splits, tiles));
+  int best = 1;
+  double best_eff = -1.0;
+  for (int s = 1; s <= smax; ++s) {
+    const double ctas = (double)units * s;
+    const double waves = ctas / slots;
+    const double eff_w = waves / std::ceil(waves);
+    const double per = (double)tiles / s;
+    const double eff_t = per / std::ceil(per);
+    const double eff = eff_w * eff_t * (per < 2.0 ? 0.9 : 1.0);
+    if (eff > best_eff * 1.01) {
+      best_eff = eff;
+      best = s;
+    }
+  }
+  return best;
+}
+
+
+// Tiles of 64 items (positions, or kept-list entries) an anchor's decode
+// covers, from the host-side bound on its lengths.
+int layer_tiles(const kvk_cache *c, int a) {
+  const long long items = c->kept_on[a] ? c->cfg[a].evict_capacity : c->len_hi[a];
+  return (int)std::max<long long>(1, (items + kTile - 1) / kTile);
+}
+
+int auto_splits(kvk_cache *c, int a) {
+  const bool mla = c->desc.kind == KVK_KIND_MLA;
+  if (!c->ctas[a]) {
+    if (mla) {
+      c->ctas[a] = mla_decode_ctas_per_sm(c->cfg[a].width);
+    } else {
+      const kvk_layer_cfg &L = c->cfg[a];
+      c->ctas[a] = gqa_decode_ctas_per_sm(L.bits, c->desc.head_dim, L.bits == 16 ? 0 : L.key_axis,
+                                          L.bits == 16 ? 64 : L.group);
+    }
+  }
+  const int units = mla ? c->desc.max_batch : c->desc.max_batch * c->desc.n_kv_heads;
+  return choose_splits(units, layer_tiles(c, a), c->sm_count * c->ctas[a], c->max_splits);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *kvk_status_string(kvk_status s) {
+  switch (s) {
+    case KVK_OK: return "ok";
+    case KVK_ERR_INVALID_ARG: return "invalid argument";
+    case KVK_ERR_INVALID_CONFIG: return "invalid configuration";
+    case KVK_ERR_INHERITED_LAYER: return "layer inherits its cache";
+    case KVK_ERR_CAPACITY: return "capacity exceeded";
+    case KVK_ERR_UNSUPPORTED: return "unsupported";
+    case KVK_ERR_CUDA: return "CUDA error";
+    case KVK_ERR_DEVICE: return "device error word set";
+  }
+  return "unknown status";
+}
+
+const char *kvk_last_error(void) { return g_last_error.c_str(); }
+
+const char *kvk_version(void) { return "kvk 0.1 sm_103a"; }
+
+kvk_status kvk_cache_plan(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
+                          size_t *arena_bytes) {
+  kvk_status s = check_desc(desc);
+  if (s) return s;
+  if (!cfg || !arena_bytes) return fail(KVK_ERR_INVALID_ARG, "null plan or output");
+  for (int l = 0; l < desc->n_layers; ++l) {
+    s = check_layer(desc, &cfg[l], l);
+    if (s) return s;
+  }
+  for (int l = 0; l < desc->n_layers; ++l)
+    arena_bytes[l] = cfg[l].inherit ? 0 : (size_t)layer_layout(desc, &cfg[l]).total;
+  return KVK_OK;
+}
+
+kvk_status kvk_workspace_size(const kvk_model_desc *desc, int32_t max_splits, size_t *ws_bytes) {
+  kvk_status s = check_desc(desc);
+  if (s) return s;
+  if (!ws_bytes || max_splits < 1 || max_splits > 256)
+    return fail(KVK_ERR_INVALID_ARG, "max_splits must be in [1, 256]");
+  *ws_bytes = ws_layout(desc, max_splits).total;
+  return KVK_OK;
+}
+
+kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
+                            void *const *arenas, void *workspace, size_t ws_bytes,
+                            int32_t max_splits, kvk_cache **out) {
+  if (!out) return fail(KVK_ERR_INVALID_ARG, "null output handle");
+  *out = nullptr;
+  std::vector<size_t> bytes(desc ? std::max(0, desc->n_layers) : 0);
+  kvk_status s = kvk_cache_plan(desc, cfg, bytes.data());
+  if (s) return s;
+  if (max_splits < 1 || max_splits > 256) return fail(KVK_ERR_INVALID_ARG, "max_splits must be in [1, 256]");
+  if (!arenas || !workspace || !aligned16(workspace))
+    return fail(KVK_ERR_INVALID_ARG, "null or misaligned arenas/workspace");
+  const WsLayout wl = ws_layout(desc, max_splits);
+  if (ws_bytes < wl.total)
+    return fail(KVK_ERR_INVALID_ARG, "workspace too small: %zu < %zu", ws_bytes, wl.total);
+  for (int l = 0; l < desc->n_layers; ++l) {
+    if (cfg[l].inherit) continue;
+    if (!arenas[l] || (reinterpret_cast<uintptr_t>(arenas[l]) & 255u))
+      return fail(KVK_ERR_INVALID_ARG, "arena of layer %d is null or not 256-byte aligned", l);
+  }
+  kvk_cache *c = new (std::nothrow) kvk_cache();
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "out of host memory");
+  c->desc = *desc;
+  c->cfg.assign(cfg, cfg + desc->n_layers);
+  c->src.resize(desc->n_layers);
+  c->arena.assign(desc->n_layers, nullptr);
+  c->lay.resize(desc->n_layers);
+  c->len_hi.assign(desc->n_layers, 0);
+  c->kept_on.assign(desc->n_layers, 0);
+  c->ctas.assign(desc->n_layers, 0);
+  int last = 0;
+  for (int l = 0; l < desc->n_layers; ++l) {
+    if (!cfg[l].inherit) {
+      last = l;
+      c->arena[l] = static_cast<uint8_t *>(arenas[l]);
+      c->lay[l] = layer_layout(desc, &cfg[l]);
+    }
+    c->src[l] = last;
+  }
+  c->ws = static_cast<uint8_t *>(workspace);
+  c->ws_bytes = ws_bytes;
+  c->wl = wl;
+  c->max_splits = max_splits;
+  cudaError_t e = cudaGetDevice(&c->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, c->device);
+  if (e != cudaSuccess) {
+    delete c;
+    return cuda_fail(e, "querying the device");
+  }
+  *out = c;
+  return KVK_OK;
+}
+
+kvk_status kvk_cache_destroy(kvk_cache *cache) {
+  delete cache;
+  return KVK_OK;
+}
+
+kvk_status kvk_cache_reset(kvk_cache *c, kvk_stream stream) {
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  for (int l = 0; l < c->desc.n_layers; ++l) {
+    if (c->cfg[l].inherit) continue;
+    const ArenaLayout &A = c->lay[l];
+    // lens, counter and kept_n are the arena's first three 256-byte-aligned slots
+    cudaError_t e = cudaMemsetAsync(c->arena[l], 0, (size_t)A.kept_idx, st);
+    if (e != cudaSuccess) return cuda_fail(e, "resetting lengths");
+    c->len_hi[l] = 0;
+    c->kept_on[l] = 0;
+  }
+  cudaError_t e = cudaMemsetAsync(c->err(), 0, 4, st);
+  if (e != cudaSuccess) return cuda_fail(e, "resetting the error word");
+  return KVK_OK;
+}
+
+kvk_status kvk_layer_source(const kvk_cache *c, int32_t layer, int32_t *src) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (!src) return fail(KVK_ERR_INVALID_ARG, "null output");
+  *src = c->src[layer];
+  return KVK_OK;
+}
+
+kvk_status kvk_layer_lengths(const kvk_cache *c, int32_t layer, const int32_t **lens) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (!lens) return fail(KVK_ERR_INVALID_ARG, "null output");
+  const int a = c->src[layer];
+  *lens = reinterpret_cast<const int32_t *>(c->arena[a] + c->lay[a].lens);
+  return KVK_OK;
+}
+
+kvk_status kvk_append(kvk_cache *c, int32_t layer, const void *k, const void *v, int32_t in_dtype,
+                      int32_t n_new, const int32_t *n_new_per_seq, kvk_stream stream) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->cfg[layer].inherit)
+    return fail(KVK_ERR_INHERITED_LAYER, "layer %d inherits layer %d's cache", layer, c->src[layer]);
+  if (n_new < 0) return fail(KVK_ERR_INVALID_ARG, "n_new < 0");
+  if (n_new == 0) return KVK_OK;
+  if (!k || !v || !aligned16(k) || !aligned16(v))
+    return fail(KVK_ERR_INVALID_ARG, "null or misaligned k/v");
+  if (c->len_hi[layer] + n_new > c->desc.max_ctx)
+    return fail(KVK_ERR_CAPACITY, "layer %d: %lld + %d positions exceed max_ctx %d", layer,
+                c->len_hi[layer], n_new, c->desc.max_ctx);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (c->desc.kind == KVK_KIND_GQA) {
+    if (in_dtype != KVK_DTYPE_F32 && in_dtype != KVK_DTYPE_BF16)
+      return fail(KVK_ERR_INVALID_ARG, "in_dtype must be F32 or BF16");
+    e = launch_gqa_append(c->gqa_view(layer), k, v, in_dtype == KVK_DTYPE_F32, n_new,
+                          n_new_per_seq, c->err(), st);
+  } else {
+    if (in_dtype != KVK_DTYPE_BF16) return fail(KVK_ERR_INVALID_ARG, "MLA appends take BF16");
+    e = launch_mla_append(c->mla_view(layer), k, v, c->desc.latent_dim, n_new, n_new_per_seq,
+                          c->err(), st);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  c->len_hi[layer] += n_new;
+  return KVK_OK;
+}
+
+kvk_status kvk_rewind(kvk_cache *c, int32_t n, kvk_stream stream) {
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
+  if (n < 0) return fail(KVK_ERR_INVALID_ARG, "n < 0");
+  RewindArgs r;
+  r.B = c->desc.max_batch;
+  r.n = n;
+  r.n_anchors = 0;
+  for (int l = 0; l < c->desc.n_layers; ++l) {
+    const kvk_layer_cfg &L = c->cfg[l];
+    if (L.inherit) continue;
+    if (c->desc.kind == KVK_KIND_GQA && L.bits != 16 && L.key_axis == KVK_AXIS_CHANNEL)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d has per-channel key groups", l);
+  }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  for (int l = 0; l < c->desc.n_layers; ++l) {
+    if (c->cfg[l].inherit) continue;
+    r.lens[r.n_anchors++] = reinterpret_cast<int32_t *>(c->arena[l] + c->lay[l].lens);
+    c->len_hi[l] = std::max<long long>(0, c->len_hi[l] - n);
+    if (r.n_anchors == 64) {
+      cudaError_t e = launch_rewind(r, st);
+      if (e != cudaSuccess) return cuda_fail(e, "rewind launch");
+      r.n_anchors = 0;
+    }
+  }
+  if (r.n_anchors) {
+    cudaError_t e = launch_rewind(r, st);
+    if (e != cudaSuccess) return cuda_fail(e, "rewind launch");
+  }
+  return KVK_OK;
+}
+
+kvk_status kvk_decode_plan_splits(kvk_cache *c, int32_t layer, int32_t *n_splits) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (!n_splits) return fail(KVK_ERR_INVALID_ARG, "null output");
+  *n_splits = std::min(auto_splits(c, c->src[layer]), layer_tiles(c, c->src[layer]));
+  return KVK_OK;
+}
+
+kvk_status kvk_set_kept(kvk_cache *c, int32_t layer, const int32_t *idx, const int32_t *n_kept,
+                        kvk_stream stream) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->cfg[layer].inherit)
+    return fail(KVK_ERR_INHERITED_LAYER, "layer %d inherits; set the list on layer %d", layer,
+                c->src[layer]);
+  const int cap = c->cfg[layer].evict_capacity;
+  if (!n_kept) {
+    c->kept_on[layer] = 0;
+    return KVK_OK;
+  }
+  if (cap <= 0) return fail(KVK_ERR_INVALID_CONFIG, "layer %d has evict_capacity 0", layer);
+  if (!idx) return fail(KVK_ERR_INVALID_ARG, "null kept index list");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const ArenaLayout &A = c->lay[layer];
+  const size_t B = c->desc.max_batch;
+  cudaError_t e = cudaMemcpyAsync(c->arena[layer] + A.kept_idx, idx, B * cap * 4,
+                                  cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(c->arena[layer] + A.kept_n, n_kept, B * 4, cudaMemcpyDeviceToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(e, "copying the kept list");
+  c->kept_on[layer] = 1;
+  return KVK_OK;
+}
+
+static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, int32_t q_dtype,
+                                    float scale, float *out, float *partial, int32_t n_splits,
+                                    bool merge, kvk_stream stream) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->desc.kind != KVK_KIND_GQA) return fail(KVK_ERR_INVALID_ARG, "cache is not GQA");
+  if (!q || !aligned16(q)) return fail(KVK_ERR_INVALID_ARG, "null or misaligned q");
+  if (q_dtype != KVK_DTYPE_F32 && q_dtype != KVK_DTYPE_BF16)
+    return fail(KVK_ERR_INVALID_ARG, "q_dtype must be F32 or BF16");
+  if (n_splits < 0 || n_splits > c->max_splits)
+    return fail(KVK_ERR_INVALID_ARG, "n_splits %d outside [0, %d]", n_splits, c->max_splits);
+  if (!std::isfinite(scale)) return fail(KVK_ERR_INVALID_ARG, "non-finite softmax scale");
+  const int a = c->src[layer];
+  GqaDecodeArgs args;
+  args.v = c->gqa_view(a);
+  args.gather = c->kept_on[a];
+  const int tiles = layer_tiles(c, a);
+  if (n_splits == 0) n_splits = auto_splits(c, a);
+  // a partial-only call keeps the caller's split count (extra splits are
+  // empty and write m = -inf, l = 0); a full call never uses more splits
+  // than tiles.
+  if (merge) n_splits = std::min(n_splits, tiles);
+  args.q = q;
+  args.q_f32 = q_dtype == KVK_DTYPE_F32;
+  args.Hq = c->desc.n_q_heads;
+  args.G = c->desc.n_q_heads / c->desc.n_kv_heads;
+  args.sig_log2 = scale * 1.4426950408889634f;
+  args.n_splits = n_splits;
+  const int tps = (tiles + n_splits - 1) / n_splits;
+  args.items_per_split = tps * kTile;
+  args.err = c->err();
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (merge && n_splits == 1) {
+    args.out = out;  // one split: the kernel normalises and writes the output
+    args.partial = nullptr;
+  } else {
+    args.out = nullptr;
+    args.partial = partial ? partial : reinterpret_cast<float *>(c->ws + c->wl.partial);
+  }
+  cudaError_t e = launch_gqa_decode(args, st);
+  if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+  if (merge && n_splits > 1) {
+    e = launch_splitk_merge(args.partial, n_splits, c->desc.max_batch * c->desc.n_q_heads,
+                            c->desc.head_dim, out, st);
+    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+  }
+  return KVK_OK;
+}
+
+kvk_status kvk_decode_attention(kvk_cache *c, int32_t layer, const void *q, int32_t q_dtype,
+                                float softmax_scale, float *out, int32_t n_splits,
+                                kvk_stream stream) {
+  if (!out || !aligned16(out)) return fail(KVK_ERR_INVALID_ARG, "null or misaligned out");
+  return gqa_decode_common(c, layer, q, q_dtype, softmax_scale, out, nullptr, n_splits, true,
+                           stream);
+}
+
+kvk_status kvk_decode_partial(kvk_cache *c, int32_t layer, const void *q, int32_t q_dtype,
+                              float softmax_scale, float *partials, int32_t n_splits,
+                              kvk_stream stream) {
+  if (!partials || !aligned16(partials))
+    return fail(KVK_ERR_INVALID_ARG, "null or misaligned partials");
+  if (n_splits < 2) return fail(KVK_ERR_INVALID_ARG, "kvk_decode_partial needs n_splits >= 2");
+  return gqa_decode_common(c, layer, q, q_dtype, softmax_scale, nullptr, partials, n_splits,
+                           false, stream);
+}
+
+kvk_status kvk_splitk_reduce(const float *partials, int32_t n_splits, int32_t n_rows, int32_t dim,
+                             float *out, kvk_stream stream) {
+  if (!partials || !out) return fail(KVK_ERR_INVALID_ARG, "null partials or out");
+  if (n_splits < 1 || n_splits > 256 || n_rows < 1 || dim < 1)
+    return fail(KVK_ERR_INVALID_ARG, "bad sizes");
+  cudaError_t e = launch_splitk_merge(partials, n_splits, n_rows, dim, out,
+                                      reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+  return KVK_OK;
+}
+
+kvk_status kvk_decode_attention_mla(kvk_cache *c, int32_t layer, const void *q_nope,
+                                    const void *q_pe, const void *w_uk, const void *w_uv,
+                                    float softmax_scale, float *out, int32_t n_splits,
+                                    kvk_stream stream) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->desc.kind != KVK_KIND_MLA) return fail(KVK_ERR_INVALID_ARG, "cache is not MLA");
+  if (!q_nope || !q_pe || !w_uk || !w_uv || !out || !aligned16(q_nope) || !aligned16(q_pe) ||
+      !aligned16(w_uk) || !aligned16(w_uv) || !aligned16(out))
+    return fail(KVK_ERR_INVALID_ARG, "null or misaligned MLA operand");
+  if (n_splits < 0 || n_splits > c->max_splits)
+    return fail(KVK_ERR_INVALID_ARG, "n_splits %d outside [0, %d]", n_splits, c->max_splits);
+  const int a = c->src[layer];
+  MlaDecodeArgs args;
+  args.v = c->mla_view(a);
+  const int tiles = layer_tiles(c, a);
+  if (n_splits == 0) n_splits = auto_splits(c, a);
+  n_splits = std::min(n_splits, tiles);
+  args.q_nope = q_nope;
+  args.q_pe = q_pe;
+  args.w_uk = w_uk;
+  args.w_uv = w_uv;
+  args.H = c->desc.n_q_heads;
+  args.Dn = c->desc.head_dim;
+  args.r = c->desc.latent_dim;
+  args.sig_log2 = softmax_scale * 1.4426950408889634f;
+  args.n_splits = n_splits;
+  args.items_per_split = ((tiles + n_splits - 1) / n_splits) * kTile;
+  args.qlat = reinterpret_cast<uint16_t *>(c->ws + c->wl.qlat);
+  args.partial = reinterpret_cast<float *>(c->ws + c->wl.partial);
+  args.olat = reinterpret_cast<float *>(c->ws + c->wl.olat);
+  args.out = out;
+  args.err = c->err();
+  cudaError_t e = launch_mla_decode(args, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "MLA decode launch");
+  return KVK_OK;
+}
+
+kvk_status kvk_plan_cost(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
+                         double *bits_model, double *bytes_stored, double *rho) {
+  kvk_status s = check_desc(desc, false);
+  if (s) return s;
+  if (!cfg) return fail(KVK_ERR_INVALID_ARG, "null plan");
+  for (int l = 0; l < desc->n_layers; ++l) {
+    s = check_layer(desc, &cfg[l], l, false);
+    if (s) return s;
+  }
+  const kvk_model_desc &d = *desc;
+  const bool mla = d.kind == KVK_KIND_MLA;
+  double bits = 0.0, bytes = 0.0;
+  for (int l = 0; l < d.n_layers; ++l) {
+    const kvk_layer_cfg &a = cfg[l];
+    if (a.inherit) continue;  // eq. (cost): inheriting costs nothing
+    if (mla) {
+      bits += (double)(a.width + d.rope_dim) * a.bits;
+      bytes += (double)(a.width + d.rope_dim) * a.bits / 8.0;
+    } else {
+      bits += 2.0 * d.n_kv_heads * d.head_dim * a.bits;
+      double per;
+      if (a.bits == 16) {
+        per = 4.0 * d.head_dim;
+      } else {
+        // codes + one fp32 (scale, zero) pair per group, K and V
+        per = 2.0 * d.head_dim * a.bits / 8.0 + 2.0 * 8.0 * d.head_dim / a.group;
+      }
+      bytes += per * d.n_kv_heads;
+    }
+  }
+  // eq. (compression): against the bf16 GQA cache; for MLA the conversion
+  // width r = n_kv d_h of Appendix B stands for n_kv d_h.
+  const double width = mla ? (double)d.latent_dim : (double)d.n_kv_heads * d.head_dim;
+  const double c0 = d.n_layers * 2.0 * width * 16.0;
+  if (bits_model) *bits_model = bits;
+  if (bytes_stored) *bytes_stored = bytes;
+  if (rho) *rho = c0 / bits;
+  return KVK_OK;
+}
+
+kvk_status kvk_cost(const kvk_cache *c, double *bits_model, double *bytes_stored, double *rho) {
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
+  return kvk_plan_cost(&c->desc, c->cfg.data(), bits_model, bytes_stored, rho);
+}
+
+kvk_status kvk_export_layer(const kvk_cache *c, int32_t layer, void *k_out, void *v_out,
+                            float *k_scale, float *k_zero, float *v_scale, float *v_zero,
+                            void *k_residual, kvk_stream stream) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->cfg[layer].inherit)
+    return fail(KVK_ERR_INHERITED_LAYER, "layer %d inherits layer %d's cache", layer, c->src[layer]);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (c->desc.kind == KVK_KIND_GQA)
+    e = launch_gqa_export(c->gqa_view(layer), k_out, v_out, k_scale, k_zero, v_scale, v_zero,
+                          k_residual, c->desc.max_ctx, st);
+  else
+    e = launch_mla_export(c->mla_view(layer), k_out, v_out, c->desc.max_ctx, st);
+  if (e != cudaSuccess) return cuda_fail(e, "export launch");
+  return KVK_OK;
+}
+
+kvk_status kvk_get_device_error(kvk_cache *c, kvk_stream stream, int32_t *code) {
+  if (!c || !code) return fail(KVK_ERR_INVALID_ARG, "null cache or output");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int32_t h = 0;
+  cudaError_t e = cudaMemcpyAsync(&h, c->err(), 4, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->err(), 0, 4, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the device error word");
+  *code = h;
+  if (h) return fail(KVK_ERR_DEVICE, "device error word 0x%x", h);
+  return KVK_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,181 @@
+// layout.h -- stored layout of one anchor's cache (host and device).
+//
+// Every (position, KV head) of a GQA anchor is one contiguous, 16-byte
+// aligned RECORD:
+//
+//     [ K section | V section | K meta (per-token keys) | V meta ]
+//
+//   K/V section  head_dim codes at `bits` (16 = bf16 values, 8 = one code per
+//                byte, 4 = two codes per byte), in the fragment order below;
+//   meta         one float2 (scale, zero) per group of `group` channels,
+//                natural group order, padded to 16 bytes.
+//
+// Per-channel keys (KIVI layout) keep the K codes in the record and store
+// (scale, zero) per (group of `group` positions, channel) in a separate
+// group-meta plane; positions of a not-yet-full group stay bf16 in a
+// residual plane (row = position mod group) in the bf16 K fragment order.
+//
+// Records are stored [batch][kv head][position] with `cap` positions per
+// (batch, kv head) slab, so a run of positions is one contiguous block (one
+// copy per tile when streaming) and one position is 1-2 cache lines (few
+// sectors per kept position when gathering an eviction list).
+//
+// Fragment order.  The decode kernel multiplies with mma.m16n8k16: for
+// scores, A = keys (16 positions x 16 channels); for the value product,
+// A = V^T (16 channels x 16 positions).  Channels are permuted on write so
+// that the bytes one lane needs for its A fragments are contiguous:
+//
+//   K: channel ch -> k-step j = ch/16, slot s = ch%16, lane column
+//      c = (s%8)/2, element n = 4j + r with r = (s%2) + 2*(s/8), i.e. lane c
+//      holds slots {2c, 2c+1, 2c+8, 2c+9} of every k-step.  Lane c's segment
+//      (head_dim/4 elements) is split into 16-byte chunks; chunk i of lane c
+//      sits at chunk index 4i + c.  For 4-bit keys each 32-bit word holds
+//      k-steps (2w, 2w+1) with nibbles ordered so that masking with
+//      0x000F000F / 0x00F000F0 (and again after >> 8) yields the f16 pairs of
+//      the a0 / a2 registers directly.
+//   V: channel ch -> M-block m = ch/16, row rr = ch%16, lane row g = rr%8,
+//      e = rr/8; lane g's segment (head_dim/8 elements) holds (m, e) at
+//      element 2m + e.  For 4-bit values byte m of lane g's segment holds row
+//      g in the low nibble and row g+8 in the high nibble.
+//
+// An MLA anchor stores [c[:width] | k^R] in bf16, natural order, one record
+// per (batch, position).
+#pragma once
+#include <stdint.h>
+
+#if defined(__CUDACC__)
+#define KVK_HD __host__ __device__ __forceinline__
+#else
+#define KVK_HD inline
+#endif
+
+namespace kvk {
+
+constexpr int kTile = 64;  // positions per decode tile
+
+KVK_HD int sec_bytes(int bits, int D) { return D * bits / 8; }
+KVK_HD int meta_bytes(int D, int g) { return (((D / g) * 8) + 15) & ~15; }
+
+struct RecLayout {
+  int k_off, v_off, km_off, vm_off, rec;
+};
+
+// key_axis: 0 = per token, 1 = per channel.
+KVK_HD RecLayout rec_layout(int bits, int D, int g, int key_axis) {
+  RecLayout L;
+  const int s = sec_bytes(bits, D);
+  L.k_off = 0;
+  L.v_off = s;
+  int off = 2 * s;
+  if (bits == 16) {
+    L.km_off = -1;
+    L.vm_off = -1;
+    L.rec = off;
+    return L;
+  }
+  if (key_axis == 0) {
+    L.km_off = off;
+    off += meta_bytes(D, g);
+  } else {
+    L.km_off = -1;
+  }
+  L.vm_off = off;
+  off += meta_bytes(D, g);
+  L.rec = off;
+  return L;
+}
+
+// Position of channel `ch` inside the K section: byte offset, and for 4-bit
+// codes whether it is the high nibble.
+KVK_HD void k_pos(int ch, int bits, int D, int *byte, int *hi) {
+  const int j = ch >> 4, s = ch & 15;
+  const int c = (s & 7) >> 1;
+  const int r = (s & 1) | ((s >> 3) << 1);
+  const int n = 4 * j + r;
+  const int seg = D * bits / 32;  // bytes per lane segment
+  int bp;
+  *hi = 0;
+  if (bits == 16) {
+    bp = 2 * n;
+  } else if (bits == 8) {
+    bp = n;
+  } else {
+    const int w = j >> 1, jj = j & 1;
+    const int nib = (r & 1) * 4 + (r >> 1) + 2 * jj;
+    bp = 4 * w + (nib >> 1);
+    *hi = nib & 1;
+  }
+  *byte = (seg >= 16) ? 16 * (4 * (bp >> 4) + c) + (bp & 15) : seg * c + bp;
+}
+
+// Position of channel `ch` inside the V section.
+KVK_HD void v_pos(int ch, int bits, int D, int *byte, int *hi) {
+  const int m = ch >> 4, rr = ch & 15;
+  const int g = rr & 7, e = rr >> 3;
+  const int n = 2 * m + e;
+  const int seg = D * bits / 64;
+  int bp;
+  *hi = 0;
+  if (bits == 16) {
+    bp = 2 * n;
+  } else if (bits == 8) {
+    bp = n;
+  } else {
+    bp = m;
+    *hi = e;
+  }
+  *byte = seg * g + bp;
+}
+
+KVK_HD int64_t align256(int64_t x) { return (x + 255) & ~(int64_t)255; }
+
+// Offsets inside one anchor's arena.
+struct ArenaLayout {
+  int64_t lens;      // int32[B]
+  int64_t counter;   // int32 (append completion counter)
+  int64_t kept_n;    // int32[B]
+  int64_t kept_idx;  // int32[B * kept_cap]
+  int64_t rec;       // records
+  int64_t gmeta;     // float2 [B*Hkv][cap/g][D] (per-channel keys)
+  int64_t resid;     // bf16 K rows [B*Hkv][g][D] (per-channel keys)
+  int64_t total;
+  int64_t cap;       // positions per slab (max_ctx rounded up to kTile)
+  int rec_bytes;
+};
+
+// mla: records are [B][cap][(width + rope) * 2 bytes]; kv heads = 1.
+KVK_HD ArenaLayout arena_layout(int mla, int B, int Hkv, int max_ctx, int D, int bits,
+                                int g, int key_axis, int kept_cap, int width, int rope) {
+  ArenaLayout A;
+  A.cap = ((int64_t)max_ctx + kTile - 1) / kTile * kTile;
+  int64_t off = 0;
+  A.lens = off;
+  off = align256(off + 4 * (int64_t)B);
+  A.counter = off;
+  off = align256(off + 4);
+  A.kept_n = off;
+  off = align256(off + 4 * (int64_t)B);
+  A.kept_idx = off;
+  off = align256(off + 4 * (int64_t)B * kept_cap);
+  A.rec = off;
+  if (mla) {
+    A.rec_bytes = (width + rope) * 2;
+    off = align256(off + (int64_t)B * A.cap * A.rec_bytes);
+    A.gmeta = A.resid = -1;
+  } else {
+    A.rec_bytes = rec_layout(bits, D, g, key_axis).rec;
+    off = align256(off + (int64_t)B * Hkv * A.cap * A.rec_bytes);
+    if (bits != 16 && key_axis == 1) {
+      A.gmeta = off;
+      off = align256(off + (int64_t)B * Hkv * (A.cap / g) * D * 8);
+      A.resid = off;
+      off = align256(off + (int64_t)B * Hkv * g * D * 2);
+    } else {
+      A.gmeta = A.resid = -1;
+    }
+  }
+  A.total = off;
+  return A;
+}
+
+}  // namespace kvk

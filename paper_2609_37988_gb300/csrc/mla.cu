@@ -1,0 +1,491 @@
+// mla.cu -- decode attention over a truncated MLA latent cache (Appendix C.2).
+//
+// The cache stores, per (sequence, position), the latent c[:d] (d = the
+// layer's kept width, truncated on write) and the post-RoPE positional key
+// k^R, both bf16.  With the content-key up-projection absorbed into the
+// query, one decode step of head h is
+//     q_lat = W_UK[h][:, :d]^T q_nope                      (absorb)
+//     s_t   = sigma (<q_lat, c_t[:d]> + <q_pe, k^R_t>)      (latent scores)
+//     o_lat = sum_t softmax_t(s) c_t[:d]                    (latent values)
+//     out   = W_UV[h][:, :d] o_lat                          (up-projection)
+// All heads of a sequence share the latent, so every cache byte is read once
+// for all H heads and both contractions are dense enough for the tensor
+// cores (mma.m16n8k16, bf16 operands, fp32 accumulate).  fp32 operands that
+// must enter a bf16 MMA (q_lat, softmax weights, o_lat) are split into
+// hi + lo bf16 halves, so products keep ~16 significant bits.
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "layout.h"
+
+namespace kvk {
+namespace {
+
+constexpr int kRope = 64;
+constexpr int kHeads = 16;
+
+__device__ __forceinline__ int swz8(int row, int chunk) { return chunk ^ (row & 7); }
+
+// ---------------------------------------------------------------------------
+// Absorb: q_lat[b,h,i] = sum_j q_nope[b,h,j] W_UK[h,j,i], i < d.  Per CTA one
+// head and 64 latent coordinates for up to 64 sequences: M = sequences,
+// N = latent, K = Dn = 128.  Output qlat[b][h] = [hi(d) | pe(64) | lo(d)].
+template <int W>
+__global__ void __launch_bounds__(128)
+    mla_absorb_kernel(const uint16_t *__restrict__ q_nope, const uint16_t *__restrict__ q_pe,
+                      const uint16_t *__restrict__ w_uk, int B, int H, int r,
+                      uint16_t *__restrict__ qlat) {
+  constexpr int Dn = 128;
+  __shared__ __align__(16) uint16_t a_s[64 * Dn];  // [b][j], swizzled 16B chunks
+  __shared__ __align__(16) uint16_t w_s[Dn * 64];  // [j][i], swizzled
+  const int h = blockIdx.y, i0 = blockIdx.x * 64;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, c = lane & 3;
+  constexpr int QROW = 2 * W + kRope;
+  for (int b0 = 0; b0 < B; b0 += 64) {
+    // stage q_nope rows (64 sequences) and the W_UK slice
+    for (int q = tid; q < 64 * Dn / 8; q += 128) {
+      const int row = q / (Dn / 8), u = q % (Dn / 8);
+      const int b = b0 + row;
+      uint4 x = make_uint4(0, 0, 0, 0);
+      if (b < B) x = *reinterpret_cast<const uint4 *>(q_nope + ((size_t)b * H + h) * Dn + 8 * u);
+      *reinterpret_cast<uint4 *>(a_s + row * Dn + 8 * swz8(row, u)) = x;
+    }
+    for (int q = tid; q < Dn * 8; q += 128) {
+      const int j = q / 8, u = q % 8;
+      const uint4 x = *reinterpret_cast<const uint4 *>(w_uk + ((size_t)h * Dn + j) * r + i0 + 8 * u);
+      *reinterpret_cast<uint4 *>(w_s + j * 64 + 8 * swz8(j, u)) = x;
+    }
+    __syncthreads();
+    float acc[8][4];
+#pragma unroll
+    for (int n = 0; n < 8; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
+    const int mrow = 16 * warp;
+#pragma unroll
+    for (int ks = 0; ks < Dn / 16; ++ks) {
+      uint32_t a0, a1, a2, a3;
+      {
+        const int mat = lane >> 3, rr = lane & 7;
+        const int row = mrow + rr + ((mat & 1) ? 8 : 0);
+        const int ch = 2 * ks + (mat >> 1);
+        ldmatrix_x4(a0, a1, a2, a3, a_s + row * Dn + 8 * swz8(row, ch));
+      }
+#pragma unroll
+      for (int np = 0; np < 4; ++np) {  // two n-blocks per ldmatrix.x4.trans
+        uint32_t b0, b1, b2, b3;
+        const int mat = lane >> 3, rr = lane & 7;
+        const int j = 16 * ks + rr + ((mat & 1) ? 8 : 0);
+        const int ch = 2 * np + (mat >> 1);
+        ldmatrix_x4_t(b0, b1, b2, b3, w_s + j * 64 + 8 * swz8(j, ch));
+        mma_bf16(acc[2 * np], a0, a1, a2, a3, b0, b1);
+        mma_bf16(acc[2 * np + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+#pragma unroll
+    for (int n = 0; n < 8; ++n) {
+      const int i = i0 + 8 * n + 2 * c;
+#pragma unroll
+      for (int hr = 0; hr < 2; ++hr) {
+        const int b = b0 + mrow + g + 8 * hr;
+        if (b >= B) continue;
+        uint32_t hi, lo;
+        split2<true>(acc[n][2 * hr], acc[n][2 * hr + 1], hi, lo);
+        uint16_t *dst = qlat + ((size_t)b * H + h) * QROW;
+        *reinterpret_cast<uint32_t *>(dst + i) = hi;
+        *reinterpret_cast<uint32_t *>(dst + W + kRope + i) = lo;
+      }
+    }
+    if (blockIdx.x == 0) {  // copy q_pe beside the hi half
+      for (int q = tid; q < 64 * kRope; q += 128) {
+        const int row = q / kRope, e = q % kRope;
+        const int b = b0 + row;
+        if (b < B) qlat[((size_t)b * H + h) * QROW + W + e] = q_pe[((size_t)b * H + h) * kRope + e];
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Latent split-K decode.  Grid (split, sequence); 8 warps.  Tile = 64
+// positions of [c[:W] | k^R] streamed through a cp.async ring.
+//   score phase: warp (mb, nb) = (warp/2, warp%2): 16 positions x 8 heads,
+//                K = W (q_lat hi and lo) + 64 (q_pe);
+//   value phase: warp w owns (16 latent rows x 8 heads) units w, w+8, ...
+//                of O^T[W x 16], K = the tile's 64 positions (P hi and lo).
+template <int W>
+struct MlaCfg {
+  static constexpr int RB = (W + kRope) * 2;      // record bytes
+  static constexpr int NCH = RB / 16;             // 16-byte chunks per record
+  static constexpr int STAGE = kTile * RB;
+  static constexpr int NST = W >= 512 ? 2 : (W >= 256 ? 3 : 4);
+  static constexpr int QH_ROW = (W + kRope) * 2;  // bytes: hi q_lat | q_pe
+  static constexpr int QL_ROW = W * 2;            // bytes: lo q_lat
+  static constexpr int Q_BYTES = kHeads * (QH_ROW + QL_ROW);
+  static constexpr int P_BYTES = 4 * 2 * 4 * 32 * 4;
+  static constexpr int X_BYTES = 4 * kHeads * 4 * 2;  // tile maxima, row sums
+  static constexpr int SMEM = Q_BYTES + P_BYTES + X_BYTES + NST * STAGE;
+  static constexpr int UNITS = W / 8;              // (16 rows x 8 heads) value units
+  static constexpr int UPW = (UNITS + 7) / 8;      // units per warp
+  static_assert(NCH % 8 == 0, "swizzle needs 8-chunk multiples");
+};
+
+template <int W>
+__global__ void __launch_bounds__(256)
+    mla_decode_kernel(const MlaView v, const uint16_t *__restrict__ qlat, int H, float sig_log2,
+                      int items_per_split, int n_splits, float *__restrict__ partial,
+                      int32_t *err) {
+  using C = MlaCfg<W>;
+  extern __shared__ __align__(128) uint8_t smem[];
+  uint8_t *qh_s = smem;
+  uint8_t *ql_s = smem + kHeads * C::QH_ROW;
+  uint32_t *p_s = reinterpret_cast<uint32_t *>(smem + C::Q_BYTES);
+  float *tmax_s = reinterpret_cast<float *>(smem + C::Q_BYTES + C::P_BYTES);  // [4][16]
+  float *lsum_s = tmax_s + 4 * kHeads;                                         // [4][16]
+  uint8_t *stages = smem + C::Q_BYTES + C::P_BYTES + C::X_BYTES;
+
+  const int split = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, c = lane & 3;
+  const int len = v.lens[b];
+  const int i0 = split * items_per_split;
+  const int i1 = (split == n_splits - 1) ? len : min(i0 + items_per_split, len);
+  const int n_tiles = i1 > i0 ? (i1 - i0 + kTile - 1) / kTile : 0;
+  const uint8_t *rec = v.rec + (size_t)b * v.cap * C::RB;
+
+  // absorbed query [hi | pe] and [lo] into shared memory, swizzled rows
+  {
+    constexpr int QROW = 2 * W + kRope;
+    const uint16_t *qb = qlat + (size_t)b * H * QROW;
+    for (int q = tid; q < kHeads * (C::QH_ROW / 16); q += 256) {
+      const int h = q / (C::QH_ROW / 16), u = q % (C::QH_ROW / 16);
+      uint4 x = make_uint4(0, 0, 0, 0);
+      if (h < H) x = *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + 8 * u);
+      *reinterpret_cast<uint4 *>(qh_s + h * C::QH_ROW + 16 * swz8(h, u)) = x;
+    }
+    for (int q = tid; q < kHeads * (C::QL_ROW / 16); q += 256) {
+      const int h = q / (C::QL_ROW / 16), u = q % (C::QL_ROW / 16);
+      uint4 x = make_uint4(0, 0, 0, 0);
+      if (h < H) x = *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + W + kRope + 8 * u);
+      *reinterpret_cast<uint4 *>(ql_s + h * C::QL_ROW + 16 * swz8(h, u)) = x;
+    }
+  }
+
+  auto issue = [&](int t, int s) {
+    const int base = i0 + t * kTile;
+    uint8_t *st = stages + s * C::STAGE;
+    for (int q = tid; q < kTile * C::NCH; q += 256) {
+      const int row = q / C::NCH, u = q - row * C::NCH;
+      const int item = base + row;
+      const bool valid = item < i1;
+      const uint8_t *src = rec + (size_t)(valid ? item : 0) * C::RB + 16 * u;
+      cp_async16(st + row * C::RB + 16 * swz8(row, u), src, valid);
+    }
+  };
+
+  const int mb = warp >> 1, nb = warp & 1;
+  float m_run[2][2] = {{-INFINITY, -INFINITY}, {-INFINITY, -INFINITY}};  // [nb][hh]
+  float l_part[2] = {0.f, 0.f};  // this warp's rows, heads nb*8 + 2c + hh
+  float acc[C::UPW][4];
+#pragma unroll
+  for (int u = 0; u < C::UPW; ++u) acc[u][0] = acc[u][1] = acc[u][2] = acc[u][3] = 0.f;
+
+#pragma unroll
+  for (int s = 0; s < C::NST - 1; ++s) {
+    if (s < n_tiles) issue(s, s);
+    cp_async_commit();
+  }
+  for (int t = 0; t < n_tiles; ++t) {
+    cp_async_wait<C::NST - 2>();
+    __syncthreads();
+    {
+      const int nt = t + C::NST - 1;
+      if (nt < n_tiles) issue(nt, nt % C::NST);
+      cp_async_commit();
+    }
+    const uint8_t *st = stages + (t % C::NST) * C::STAGE;
+    const int base = i0 + t * kTile;
+
+    // ---- scores: 16 positions x 8 heads per warp -------------------------
+    float d[4] = {0.f, 0.f, 0.f, 0.f};
+    const int mat = lane >> 3, rr = lane & 7;
+#pragma unroll 4
+    for (int ks = 0; ks < (W + kRope) / 16; ++ks) {
+      uint32_t a0, a1, a2, a3;
+      {
+        const int row = 16 * mb + rr + ((mat & 1) ? 8 : 0);
+        ldmatrix_x4(a0, a1, a2, a3, st + row * C::RB + 16 * swz8(row, 2 * ks + (mat >> 1)));
+      }
+      const int hrow = 8 * nb + rr;
+      if (ks < W / 16) {
+        uint32_t b0, b1, b2, b3;  // hi (2 chunks) then lo (2 chunks)
+        const uint8_t *base_q = (mat < 2) ? qh_s + hrow * C::QH_ROW : ql_s + hrow * C::QL_ROW;
+        ldmatrix_x4(b0, b1, b2, b3, base_q + 16 * swz8(hrow, 2 * ks + (mat & 1)));
+        mma_bf16(d, a0, a1, a2, a3, b0, b1);
+        mma_bf16(d, a0, a1, a2, a3, b2, b3);
+      } else {
+        uint32_t b0, b1;
+        ldmatrix_x2(b0, b1, qh_s + hrow * C::QH_ROW + 16 * swz8(hrow, 2 * ks + (mat & 1)));
+        mma_bf16(d, a0, a1, a2, a3, b0, b1);
+      }
+    }
+    const bool vA = base + 16 * mb + g < i1, vB = base + 16 * mb + g + 8 < i1;
+    float x[4];
+    x[0] = vA ? d[0] * sig_log2 : -INFINITY;
+    x[1] = vA ? d[1] * sig_log2 : -INFINITY;
+    x[2] = vB ? d[2] * sig_log2 : -INFINITY;
+    x[3] = vB ? d[3] * sig_log2 : -INFINITY;
+    float mt0 = fmaxf(x[0], x[2]), mt1 = fmaxf(x[1], x[3]);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      mt0 = fmaxf(mt0, __shfl_xor_sync(0xffffffffu, mt0, off));
+      mt1 = fmaxf(mt1, __shfl_xor_sync(0xffffffffu, mt1, off));
+    }
+    if (g == 0) {
+      tmax_s[mb * kHeads + 8 * nb + 2 * c] = mt0;
+      tmax_s[mb * kHeads + 8 * nb + 2 * c + 1] = mt1;
+    }
+    __syncthreads();
+
+    // ---- running maxima: every thread derives the same values -------------
+    float alpha[2][2];
+#pragma unroll
+    for (int n2 = 0; n2 < 2; ++n2)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int h = 8 * n2 + 2 * c + hh;
+        float mt = fmaxf(fmaxf(tmax_s[h], tmax_s[kHeads + h]),
+                         fmaxf(tmax_s[2 * kHeads + h], tmax_s[3 * kHeads + h]));
+        alpha[n2][hh] = 1.f;
+        if (mt > m_run[n2][hh] + 8.f) {  // lazy: keep a stale max within 2^8
+          alpha[n2][hh] = (m_run[n2][hh] == -INFINITY) ? 0.f : exp2f(m_run[n2][hh] - mt);
+          m_run[n2][hh] = mt;
+        }
+      }
+    // ---- weights of this warp's 16 positions -> P^T fragments -------------
+    {
+      const float ma = m_run[nb][0], mb2 = m_run[nb][1];
+      l_part[0] *= alpha[nb][0];
+      l_part[1] *= alpha[nb][1];
+      float p[4];
+      p[0] = (ma == -INFINITY) ? 0.f : exp2f(x[0] - ma);
+      p[1] = (mb2 == -INFINITY) ? 0.f : exp2f(x[1] - mb2);
+      p[2] = (ma == -INFINITY) ? 0.f : exp2f(x[2] - ma);
+      p[3] = (mb2 == -INFINITY) ? 0.f : exp2f(x[3] - mb2);
+      l_part[0] += p[0] + p[2];
+      l_part[1] += p[1] + p[3];
+      uint32_t ht, lt, hb, lb;
+      split2<true>(p[0], p[1], ht, lt);
+      split2<true>(p[2], p[3], hb, lb);
+      uint32_t *pf = p_s + ((mb * 2 + nb) * 4) * 32;
+      pf[0 * 32 + lane] = movmatrix_t(ht);
+      pf[1 * 32 + lane] = movmatrix_t(hb);
+      pf[2 * 32 + lane] = movmatrix_t(lt);
+      pf[3 * 32 + lane] = movmatrix_t(lb);
+    }
+    // rescale the value accumulators of this warp's units
+#pragma unroll
+    for (int u = 0; u < C::UPW; ++u) {
+      const int unit = warp + 8 * u;
+      if (unit < C::UNITS) {
+        const int un = unit & 1;
+        acc[u][0] *= alpha[un][0]; acc[u][2] *= alpha[un][0];
+        acc[u][1] *= alpha[un][1]; acc[u][3] *= alpha[un][1];
+      }
+    }
+    __syncthreads();
+
+    // ---- values: O^T[16 latent x 8 heads] += C^T[16 x 64 pos] P^T -----------
+#pragma unroll
+    for (int u = 0; u < C::UPW; ++u) {
+      const int unit = warp + 8 * u;
+      if (unit < C::UNITS) {
+        const int mblk = unit >> 1, un = unit & 1;
+#pragma unroll
+        for (int kb = 0; kb < 4; ++kb) {
+          uint32_t a0, a1, a2, a3;
+          const int row = 16 * kb + rr + ((mat >> 1) ? 8 : 0);
+          ldmatrix_x4_t(a0, a1, a2, a3, st + row * C::RB + 16 * swz8(row, 2 * mblk + (mat & 1)));
+          const uint32_t *pf = p_s + ((kb * 2 + un) * 4) * 32;
+          mma_bf16(acc[u], a0, a1, a2, a3, pf[lane], pf[32 + lane]);
+          mma_bf16(acc[u], a0, a1, a2, a3, pf[64 + lane], pf[96 + lane]);
+        }
+      }
+    }
+  }
+  cp_async_wait<0>();
+  __syncthreads();
+
+  // ---- row sums across the four position blocks ----------------------------
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    l_part[0] += __shfl_xor_sync(0xffffffffu, l_part[0], off);
+    l_part[1] += __shfl_xor_sync(0xffffffffu, l_part[1], off);
+  }
+  if (g == 0) {
+    lsum_s[mb * kHeads + 8 * nb + 2 * c] = l_part[0];
+    lsum_s[mb * kHeads + 8 * nb + 2 * c + 1] = l_part[1];
+  }
+  __syncthreads();
+
+  const size_t RS = (size_t)W + 2;
+  const size_t prow0 = ((size_t)split * v.B + b) * H;
+#pragma unroll
+  for (int u = 0; u < C::UPW; ++u) {
+    const int unit = warp + 8 * u;
+    if (unit < C::UNITS) {
+      const int mblk = unit >> 1, un = unit & 1;
+      const int r0 = 16 * mblk + g;
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int h = 8 * un + 2 * c + hh;
+        if (h < H) {
+          float *pr = partial + (prow0 + h) * RS;
+          pr[r0] = acc[u][hh];
+          pr[r0 + 8] = acc[u][2 + hh];
+        }
+      }
+    }
+  }
+  // publish m and l: lane (g == 0, c) of warp 0 holds m for heads 2c+hh and
+  // 8+2c+hh (all threads agree on m_run).
+  if (warp == 0 && g == 0) {
+#pragma unroll
+    for (int n2 = 0; n2 < 2; ++n2)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int h = 8 * n2 + 2 * c + hh;
+        if (h < H) {
+          float *pr = partial + (prow0 + h) * RS;
+          pr[W] = m_run[n2][hh];
+          pr[W + 1] = lsum_s[h] + lsum_s[kHeads + h] + lsum_s[2 * kHeads + h] +
+                      lsum_s[3 * kHeads + h];
+        }
+      }
+  }
+  (void)err;
+}
+
+// ---------------------------------------------------------------------------
+// Up-projection: out[b,h,o] = sum_i o_lat[b,h,i] W_UV[h,o,i], i < d.
+// Per CTA one head and 16 outputs for 64 sequences: M = sequences,
+// N = outputs, K = d in chunks of 64 (o_lat split hi/lo bf16).
+template <int W>
+__global__ void __launch_bounds__(128)
+    mla_upv_kernel(const float *__restrict__ olat, const uint16_t *__restrict__ w_uv, int B,
+                   int H, int r, float *__restrict__ out) {
+  constexpr int Dv = 128;
+  __shared__ __align__(16) uint16_t ah_s[64 * 64], al_s[64 * 64];  // [b][i] chunk
+  __shared__ __align__(16) uint16_t w_s[16 * 64];                   // [o][i] chunk
+  const int h = blockIdx.y, o0 = blockIdx.x * 16;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, c = lane & 3;
+  const int mat = lane >> 3, rr = lane & 7;
+  for (int b0 = 0; b0 < B; b0 += 64) {
+    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    for (int k0 = 0; k0 < W; k0 += 64) {
+      __syncthreads();
+      for (int q = tid; q < 64 * 32; q += 128) {  // 64 rows x 32 pairs
+        const int row = q / 32, pr = q % 32;
+        const int b = b0 + row;
+        float2 x = make_float2(0.f, 0.f);
+        if (b < B) x = *reinterpret_cast<const float2 *>(olat + ((size_t)b * H + h) * W + k0 + 2 * pr);
+        uint32_t hi, lo;
+        split2<true>(x.x, x.y, hi, lo);
+        const int u = pr / 4, wi = pr % 4;
+        reinterpret_cast<uint32_t *>(ah_s + row * 64 + 8 * swz8(row, u))[wi] = hi;
+        reinterpret_cast<uint32_t *>(al_s + row * 64 + 8 * swz8(row, u))[wi] = lo;
+      }
+      for (int q = tid; q < 16 * 8; q += 128) {
+        const int o = q / 8, u = q % 8;
+        const uint4 x = *reinterpret_cast<const uint4 *>(w_uv + ((size_t)h * Dv + o0 + o) * r + k0 + 8 * u);
+        *reinterpret_cast<uint4 *>(w_s + o * 64 + 8 * swz8(o, u)) = x;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int ks = 0; ks < 4; ++ks) {
+        const int row = 16 * warp + rr + ((mat & 1) ? 8 : 0);
+        const int ch = 2 * ks + (mat >> 1);
+        uint32_t a0, a1, a2, a3, l0, l1, l2, l3;
+        ldmatrix_x4(a0, a1, a2, a3, ah_s + row * 64 + 8 * swz8(row, ch));
+        ldmatrix_x4(l0, l1, l2, l3, al_s + row * 64 + 8 * swz8(row, ch));
+        uint32_t b0, b1, b2, b3;  // n-blocks 0 and 1 (outputs o0..o0+15)
+        const int orow = rr + ((mat >> 1) ? 8 : 0);
+        ldmatrix_x4(b0, b1, b2, b3, w_s + orow * 64 + 8 * swz8(orow, 2 * ks + (mat & 1)));
+        mma_bf16(acc[0], a0, a1, a2, a3, b0, b1);
+        mma_bf16(acc[0], l0, l1, l2, l3, b0, b1);
+        mma_bf16(acc[1], a0, a1, a2, a3, b2, b3);
+        mma_bf16(acc[1], l0, l1, l2, l3, b2, b3);
+      }
+    }
+#pragma unroll
+    for (int n = 0; n < 2; ++n)
+#pragma unroll
+      for (int hr = 0; hr < 2; ++hr) {
+        const int b = b0 + 16 * warp + g + 8 * hr;
+        if (b < B) {
+          float *dst = out + ((size_t)b * H + h) * Dv + o0 + 8 * n + 2 * c;
+          dst[0] = acc[n][2 * hr];
+          dst[1] = acc[n][2 * hr + 1];
+        }
+      }
+  }
+}
+
+template <int W>
+cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
+  using C = MlaCfg<W>;
+  const int B = a.v.B;
+  mla_absorb_kernel<W><<<dim3(W / 64, a.H), 128, 0, st>>>(
+      static_cast<const uint16_t *>(a.q_nope), static_cast<const uint16_t *>(a.q_pe),
+      static_cast<const uint16_t *>(a.w_uk), B, a.H, a.r, a.qlat);
+  auto k = mla_decode_kernel<W>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  k<<<dim3(a.n_splits, B), 256, C::SMEM, st>>>(a.v, a.qlat, a.H, a.sig_log2, a.items_per_split,
+                                                a.n_splits, a.partial, a.err);
+  cudaError_t e = launch_splitk_merge(a.partial, a.n_splits, B * a.H, W, a.olat, st);
+  if (e != cudaSuccess) return e;
+  mla_upv_kernel<W><<<dim3(128 / 16, a.H), 128, 0, st>>>(
+      a.olat, static_cast<const uint16_t *>(a.w_uv), B, a.H, a.r, a.out);
+  return cudaGetLastError();
+}
+
+template <int W>
+int mla_ctas_t() {
+  using C = MlaCfg<W>;
+  auto k = mla_decode_kernel<W>;
+  cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 256, C::SMEM) != cudaSuccess) n = 1;
+  return n > 0 ? n : 1;
+}
+
+}  // namespace
+
+cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st) {
+  switch (a.v.width) {
+    case 512: return launch_mla_t<512>(a, st);
+    case 256: return launch_mla_t<256>(a, st);
+    case 128: return launch_mla_t<128>(a, st);
+    case 64: return launch_mla_t<64>(a, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+int mla_decode_ctas_per_sm(int width) {
+  switch (width) {
+    case 512: return mla_ctas_t<512>();
+    case 256: return mla_ctas_t<256>();
+    case 128: return mla_ctas_t<128>();
+    case 64: return mla_ctas_t<64>();
+    default: return 1;
+  }
+}
+
+}  // namespace kvk
