@@ -117,6 +117,22 @@ class Clocks:
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
 
 
+def reduce_max(x: float, dist=None, device=None) -> float:
+    """Maximum of ``x`` over ranks (the slowest rank sets the job time)."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(step_bytes: int, steps: int, world: int, seconds: float) -> float:
+    """Whole-job GB/s: every rank moves ``step_bytes`` per step (weak
+    scaling), divided by the slowest rank's time."""
+    return step_bytes * steps * world / seconds / 1e9
+
+
 # ---------------------------------------------------------------------------
 def cpu_baseline(w, seconds=12.0):
     """The oracle (NumPy/fp64, as it stands) on a bounded sample of the same
@@ -291,13 +307,9 @@ def main():
             e1.synchronize()
             torch.cuda.synchronize()
         barrier()
-    ms = e0.elapsed_time(e1)
-    if dist:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_max(e0.elapsed_time(e1), dist, dev)
     ms_step = ms / args.steps
-    value = step_bytes * args.steps * world / (ms / 1e3) / 1e9
+    value = job_throughput(step_bytes, args.steps, world, ms / 1e3)
 
     # ---- per-kernel durations (events on the launching stream) -------------
     # decode kernel alone through kvk_decode_partial + kvk_splitk_reduce
@@ -377,11 +389,8 @@ def main():
             for _ in range(args.e2e_steps):
                 e2e_step()
             dt = time.perf_counter() - t0
-        if dist:
-            t = torch.tensor([dt], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            dt = float(t.item())
-        e2e = {"value": step_bytes * args.e2e_steps * world / dt / 1e9, "unit": UNIT,
+        dt = reduce_max(dt, dist, dev)
+        e2e = {"value": job_throughput(step_bytes, args.e2e_steps, world, dt), "unit": UNIT,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": dt / args.e2e_steps * 1e3}
 

@@ -63,10 +63,18 @@ struct GqaCfg {
   static constexpr int VM_OFF = KM_OFF + (KPT ? kTile * MB : 0);
   static constexpr int KG_OFF = VM_OFF + (QUANT ? kTile * MB : 0);
   static constexpr int KG_ROWS = KPC ? kTile / GS : 0;
-  static constexpr int STAGE = KG_OFF + KG_ROWS * D * 8;
-  static constexpr int NST = STAGE >= 24576 ? 3 : 4;
-  static constexpr int Q_BYTES = 8 * D * 4;
-  static constexpr int SMEM = Q_BYTES + NST * STAGE;
+  // Quantised caches: a stage is 64 raw records (one bulk copy) followed by
+  // the tile's key-group metadata rows.  bf16 caches: planes filled by
+  // 16-byte copies with conflict-free swizzles.
+  static constexpr bool TMA = QUANT;
+  static constexpr int KG_OFF_T = kTile * REC;
+  static constexpr int STAGE = TMA ? KG_OFF_T + KG_ROWS * D * 8 : KG_OFF + KG_ROWS * D * 8;
+  static constexpr int NST = TMA ? (STAGE <= 13312 ? 4 : 3) : 2;
+  static constexpr int MIN_CTAS = BF ? 3 : (NST == 4 ? 4 : 3);
+  static constexpr int QSTR = D + 4;  // padded query row (floats): conflict-free head rows
+  static constexpr int Q_BYTES = 8 * QSTR * 4 + 2 * 8 * NG * 4;
+  static constexpr int BAR_OFF = Q_BYTES + NST * STAGE;
+  static constexpr int SMEM = BAR_OFF + (TMA ? 8 * NST : 0);
   static_assert(REC % 16 == 0, "records are 16-byte multiples");
   static_assert(!QUANT || (GS % 16 == 0 && D % GS == 0), "groups are whole k-steps");
   static_assert(4 * 8 * (D + 2) * 4 <= NST * STAGE, "merge scratch fits the stages");
@@ -88,12 +96,16 @@ __device__ __forceinline__ uint32_t nib_f16(uint32_t x, uint32_t mask) {
 }
 
 template <int BITS, int D, int KAX, int GS>
-__global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) {
+__global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
+    gqa_decode_kernel(const GqaDecodeArgs a) {
   using C = GqaCfg<BITS, D, KAX, GS>;
   constexpr bool BF = C::BF;
   constexpr int KS = C::KS, NG = C::NG;
   extern __shared__ __align__(128) uint8_t smem[];
-  float *q_s = reinterpret_cast<float *>(smem);
+  constexpr int QSTR = C::QSTR;
+  float *q_s = reinterpret_cast<float *>(smem);        // [8][QSTR]
+  float *qs_s = q_s + 8 * QSTR;                        // [8][NG] query sums per group
+  float *qo_s = qs_s + 8 * NG;                         // [8][NG] 1024-bias offsets
   uint8_t *stages = smem + C::Q_BYTES;
 
   const GqaView &v = a.v;
@@ -118,43 +130,58 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
       x = a.q_f32 ? static_cast<const float *>(a.q)[qi]
                   : bf16_to_f32(static_cast<const uint16_t *>(a.q)[qi]);
     }
-    q_s[e] = x;
+    q_s[h * QSTR + ch] = x;
   }
   __syncthreads();
+  // per-token key groups: query sums Qs and 1024-bias offsets Qoff of every
+  // (head, channel group), with the f16 values the score MMA actually uses;
+  // 128 / (8 NG) lanes per (head, group), reduced with shuffles.
+  if constexpr (C::KPT) {
+    constexpr int ITEMS = 8 * NG, LPI = 128 / ITEMS, CPL = GS / LPI;
+    const int item = tid / LPI, sub = tid % LPI;
+    const int h = item / NG, gi = item % NG;
+    const bool use_lo0 = a.q_f32 != 0;
+    float sq = 0.f, so = 0.f;
+#pragma unroll 4
+    for (int k = 0; k < CPL; ++k) {
+      const int ch = gi * GS + sub * CPL + k;
+      const bool hs = (BITS == 4) && ((ch & 15) >= 8);
+      const float x = q_s[h * QSTR + ch];
+      const float xs = hs ? x * 0.0625f : x;
+      float xe = __half2float(__float2half_rn(xs));
+      if (use_lo0) xe += __half2float(__float2half_rn(xs - xe));
+      sq += hs ? 16.f * xe : xe;
+      so += 1024.f * xe;
+    }
+#pragma unroll
+    for (int off = 1; off < LPI; off <<= 1) {
+      sq += __shfl_xor_sync(0xffffffffu, sq, off);
+      so += __shfl_xor_sync(0xffffffffu, so, off);
+    }
+    if (sub == 0) { qs_s[item] = sq; qo_s[item] = so; }
+    __syncthreads();
+  }
 
   // ---- query fragments (B operand of the score MMA), head n = g ----------
   uint32_t qb[KS][2], qbl[KS][2];
   if constexpr (!C::KPC) {
 #pragma unroll
     for (int js = 0; js < KS; ++js) {
-      const float *qh = q_s + g * D + 16 * js;
+      const float *qh = q_s + g * QSTR + 16 * js;
       float x2 = qh[2 * c + 8], x3 = qh[2 * c + 9];
       if (BITS == 4) { x2 *= 0.0625f; x3 *= 0.0625f; }
       split2<BF>(qh[2 * c], qh[2 * c + 1], qb[js][0], qbl[js][0]);
       split2<BF>(x2, x3, qb[js][1], qbl[js][1]);
     }
   }
-  // per-token key groups: query sums Qs and the 1024-bias offsets Qoff for
-  // the two heads (2c, 2c+1) of this lane's accumulator columns.
   float qs[NG][2], qoff[NG][2];
   if constexpr (C::KPT) {
 #pragma unroll
     for (int gi = 0; gi < NG; ++gi)
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh) {
-        const float *qh = q_s + (2 * c + hh) * D;
-        float sq = 0.f, so = 0.f;
-        for (int ch = gi * GS; ch < (gi + 1) * GS; ++ch) {
-          const bool hs = (BITS == 4) && ((ch & 15) >= 8);
-          const float xs = hs ? qh[ch] * 0.0625f : qh[ch];
-          const __half hi = __float2half_rn(xs);
-          float xe = __half2float(hi);
-          if (use_lo) xe += __half2float(__float2half_rn(xs - xe));
-          sq += hs ? 16.f * xe : xe;
-          so += 1024.f * xe;
-        }
-        qs[gi][hh] = sq;
-        qoff[gi][hh] = so;
+        qs[gi][hh] = qs_s[(2 * c + hh) * NG + gi];
+        qoff[gi][hh] = qo_s[(2 * c + hh) * NG + gi];
       }
   }
 
@@ -172,34 +199,53 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
   const int n_tiles = i1 > i0 ? (i1 - i0 + kTile - 1) / kTile : 0;
 
   // ---- producer: one tile of records into one stage ----------------------
-  auto issue = [&](int t, int s) {
+  // Thread tid copies chunk columns u = tid/8 + 16j of rows tid%8 + 8k.  All
+  // shared-memory swizzles depend on the row only through row % 8, so each
+  // (thread, column) has one destination offset and one plane stride, and a
+  // chunk costs two adds, a compare and the copy.
+  constexpr int NCOL = (C::CPR + 15) / 16;
+  const int crow = tid & 7, ccol = tid >> 3;
+  int cdst0[NCOL], cstr[NCOL];
+#pragma unroll
+  for (int j = 0; j < NCOL; ++j) {
+    const int u = ccol + 16 * j;
+    const int ub = 16 * u;
+    int off, str;
+    if (ub < C::KB) {
+      off = C::KP_OFF + crow * C::KSTR + 16 * kswz(C::KSWZ, crow, u);
+      str = C::KSTR;
+    } else if (ub < 2 * C::KB) {
+      off = C::VP_OFF + crow * C::VSTR + 16 * vswz(C::VSWZ, crow, u - C::KB / 16);
+      str = C::VSTR;
+    } else if (C::KPT && ub < 2 * C::KB + C::MB) {
+      off = C::KM_OFF + crow * C::MB + (ub - 2 * C::KB);
+      str = C::MB;
+    } else {
+      off = C::VM_OFF + crow * C::MB + (ub - 2 * C::KB - (C::KPT ? C::MB : 0));
+      str = C::MB;
+    }
+    cdst0[j] = (u < C::CPR) ? off : -1;
+    cstr[j] = 8 * str;
+  }
+  auto issue_cp = [&](int t, int s) {
     const int base = i0 + t * kTile;
     uint8_t *st = stages + s * C::STAGE;
-    for (int q = tid; q < kTile * C::CPR; q += 128) {
-      const int row = q / C::CPR, u = q - row * C::CPR;
-      const int item = base + row;
+#pragma unroll
+    for (int k = 0; k < kTile / 8; ++k) {
+      const int item = base + crow + 8 * k;
       bool valid = item < i1;
       int pos = item;
       if (a.gather && valid) {
         pos = kept[item];
         if (pos < 0 || pos >= len) {
           valid = false;
-          if (u == 0) set_err(a.err, 1);
+          if (ccol == 0) set_err(a.err, 1);
         }
       }
-      const uint8_t *src = rec + (size_t)(valid ? pos : 0) * C::REC + 16 * u;
-      uint8_t *dst;
-      const int ub = 16 * u;
-      if (ub < C::KB) {
-        dst = st + C::KP_OFF + row * C::KSTR + 16 * kswz(C::KSWZ, row, u);
-      } else if (ub < 2 * C::KB) {
-        dst = st + C::VP_OFF + row * C::VSTR + 16 * vswz(C::VSWZ, row, u - C::KB / 16);
-      } else if (C::KPT && ub < 2 * C::KB + C::MB) {
-        dst = st + C::KM_OFF + row * C::MB + (ub - 2 * C::KB);
-      } else {
-        dst = st + C::VM_OFF + row * C::MB + (ub - 2 * C::KB - (C::KPT ? C::MB : 0));
-      }
-      cp_async16(dst, src, valid);
+      const uint8_t *src = rec + (size_t)(valid ? pos : 0) * C::REC + 16 * ccol;
+#pragma unroll
+      for (int j = 0; j < NCOL; ++j)
+        if (cdst0[j] >= 0) cp_async16(st + cdst0[j] + k * cstr[j], src + 256 * j, valid);
     }
     if constexpr (C::KPC) {
       const int g0 = base / GS;
@@ -215,6 +261,112 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
     }
   };
 
+  // bulk-copy producer (quantised caches): one copy per tile, or one per
+  // kept record; rows that get no copy are zero-filled so stale bytes never
+  // reach the arithmetic.
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::BAR_OFF);
+  if constexpr (C::TMA) {
+    if (tid == 0) {
+#pragma unroll
+      for (int s = 0; s < C::NST; ++s) mbar_init(&bars[s], 1);
+      fence_mbar_init();
+    }
+    __syncthreads();
+  }
+  auto zero_rows = [&](uint8_t *st, int r_lo, int r_hi) {  // rows [r_lo, r_hi), all threads
+    uint4 *p = reinterpret_cast<uint4 *>(st + r_lo * C::REC);
+    const int n = (r_hi - r_lo) * (C::REC / 16);
+    for (int q = tid; q < n; q += 128) p[q] = make_uint4(0, 0, 0, 0);
+  };
+  auto issue_tma = [&](int t, int s) {
+    const int base = i0 + t * kTile;
+    uint8_t *st = stages + s * C::STAGE;
+    const int nrows = min(kTile, i1 - base);
+    int kgv = 0;  // complete key groups of this tile (per-channel keys)
+    if constexpr (C::KPC) kgv = max(0, min(C::KG_ROWS, len / GS - base / GS));
+    if (!a.gather) {
+      if (tid == 0) {
+        fence_proxy_async();
+        mbar_expect_tx(&bars[s], nrows * C::REC + kgv * D * 8);
+        bulk_g2s(st, rec + (size_t)base * C::REC, nrows * C::REC, &bars[s]);
+        if (C::KPC && kgv > 0)
+          bulk_g2s(st + C::KG_OFF_T, gmeta + (size_t)(base / GS) * D, kgv * D * 8, &bars[s]);
+      }
+      if (nrows < kTile) zero_rows(st, nrows, kTile);
+    } else {
+      if (warp == 0) {
+        int pos[2];
+        bool ok[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int row = lane + 32 * h;
+          ok[h] = row < nrows;
+          pos[h] = ok[h] ? kept[base + row] : 0;
+          if (ok[h] && (pos[h] < 0 || pos[h] >= len)) {
+            ok[h] = false;
+            set_err(a.err, 1);
+          }
+        }
+        const int nvalid = __popc(__ballot_sync(0xffffffffu, ok[0])) +
+                           __popc(__ballot_sync(0xffffffffu, ok[1]));
+        if (lane == 0) {
+          fence_proxy_async();
+          mbar_expect_tx(&bars[s], nvalid * C::REC);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int row = lane + 32 * h;
+          if (ok[h]) {
+            bulk_g2s(st + row * C::REC, rec + (size_t)pos[h] * C::REC, C::REC, &bars[s]);
+          } else {
+            uint4 *p = reinterpret_cast<uint4 *>(st + row * C::REC);
+#pragma unroll
+            for (int q = 0; q < C::REC / 16; ++q) p[q] = make_uint4(0, 0, 0, 0);
+          }
+        }
+      }
+    }
+  };
+  auto issue = [&](int t, int s) {
+    if constexpr (C::TMA)
+      issue_tma(t, s);
+    else
+      issue_cp(t, s);
+  };
+
+  // shared-memory addresses of the fragments (raw records or planes)
+  auto k_chunk = [&](const uint8_t *st, int t, int i) -> const uint8_t * {
+    if constexpr (C::TMA) return st + t * C::REC + 16 * (4 * i + c);
+    else return st + C::KP_OFF + t * C::KSTR + 16 * kswz(C::KSWZ, t, 4 * i + c);
+  };
+  auto k_half = [&](const uint8_t *st, int t) -> const uint8_t * {  // 8-byte lane segment
+    if constexpr (C::TMA) return st + t * C::REC + 8 * c;
+    else return st + C::KP_OFF + t * C::KSTR + 8 * c;
+  };
+  auto v_chunk = [&](const uint8_t *st, int t, int k) -> const uint8_t * {
+    const int u = g * (C::SV / 16) + k;
+    if constexpr (C::TMA) return st + t * C::REC + C::KB + 16 * u;
+    else return st + C::VP_OFF + t * C::VSTR + 16 * vswz(C::VSWZ, t, u);
+  };
+  auto v_small = [&](const uint8_t *st, int t) -> const uint8_t * {  // lane segment < 16 B
+    if constexpr (C::TMA) return st + t * C::REC + C::KB + C::SV * g;
+    else return st + C::VP_OFF + t * C::VSTR + C::SV * g;
+  };
+  auto km_row = [&](const uint8_t *st, int t) -> const float2 * {
+    if constexpr (C::TMA) return reinterpret_cast<const float2 *>(st + t * C::REC + 2 * C::KB);
+    else return reinterpret_cast<const float2 *>(st + C::KM_OFF + t * C::MB);
+  };
+  auto vm_row = [&](const uint8_t *st, int t) -> const float2 * {
+    if constexpr (C::TMA)
+      return reinterpret_cast<const float2 *>(st + t * C::REC + 2 * C::KB + (C::KPT ? C::MB : 0));
+    else return reinterpret_cast<const float2 *>(st + C::VM_OFF + t * C::MB);
+  };
+  auto kg_rows = [&](const uint8_t *st) -> const float2 * {
+    if constexpr (C::TMA) return reinterpret_cast<const float2 *>(st + C::KG_OFF_T);
+    else return reinterpret_cast<const float2 *>(st + C::KG_OFF);
+  };
+
   // ---- consumer: one warp's 16 rows of one stage --------------------------
   auto compute = [&](int t, int s) {
     const int base = i0 + t * kTile;
@@ -228,19 +380,17 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
       if (vB) { const int p = kept[base + tB]; vB = p >= 0 && p < len; }
     }
     float s4[4] = {0.f, 0.f, 0.f, 0.f};
-    const uint8_t *Kp = st + C::KP_OFF;
 
     // lane's K words for rows tA / tB
     auto load_k = [&](int t, uint32_t(&w)[C::NWK]) {
       if constexpr (C::SK >= 16) {
 #pragma unroll
         for (int i = 0; i < C::SK / 16; ++i) {
-          const uint4 x = *reinterpret_cast<const uint4 *>(Kp + t * C::KSTR +
-                                                           16 * kswz(C::KSWZ, t, 4 * i + c));
+          const uint4 x = *reinterpret_cast<const uint4 *>(k_chunk(st, t, i));
           w[4 * i] = x.x; w[4 * i + 1] = x.y; w[4 * i + 2] = x.z; w[4 * i + 3] = x.w;
         }
       } else {
-        const uint2 x = *reinterpret_cast<const uint2 *>(Kp + t * C::KSTR + 8 * c);
+        const uint2 x = *reinterpret_cast<const uint2 *>(k_half(st, t));
         w[0] = x.x; w[1] = x.y;
       }
     };
@@ -275,7 +425,7 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
           for (int ch = 0; ch < D; ++ch) {
             int by, hi;
             k_pos(ch, 16, D, &by, &hi);
-            d += q_s[h * D + ch] * bf16_to_f32(*reinterpret_cast<const uint16_t *>(row + by));
+            d += q_s[h * QSTR + ch] * bf16_to_f32(*reinterpret_cast<const uint16_t *>(row + by));
           }
         }
         s4[k] = d;
@@ -283,12 +433,12 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
     } else if constexpr (C::KPC) {
       // scale of each channel folded into the query for this group of
       // positions; zero point and 1024-bias enter as one per-head constant.
-      const float2 *kg = reinterpret_cast<const float2 *>(st + C::KG_OFF) + (r0 / GS) * D;
+      const float2 *kg = kg_rows(st) + (r0 / GS) * D;
       uint32_t pb[KS][2], pbl[KS][2];
       float zpart = 0.f, opart = 0.f;
 #pragma unroll
       for (int js = 0; js < KS; ++js) {
-        const float *qh = q_s + g * D + 16 * js;
+        const float *qh = q_s + g * QSTR + 16 * js;
         const float2 *sz = kg + 16 * js;
         float x[4];
         const int chs[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
@@ -341,8 +491,8 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
 #pragma unroll
         for (int k = 0; k < 4; ++k) s4[k] = d[k];
       } else {
-        const float2 *kmA = reinterpret_cast<const float2 *>(st + C::KM_OFF + tA * C::MB);
-        const float2 *kmB = reinterpret_cast<const float2 *>(st + C::KM_OFF + tB * C::MB);
+        const float2 *kmA = km_row(st, tA);
+        const float2 *kmB = km_row(st, tB);
         constexpr int JPG = GS / 16;  // k-steps per group
 #pragma unroll
         for (int gi = 0; gi < NG; ++gi) {
@@ -412,8 +562,8 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
       pf[0][0] = movmatrix_t(ht); pf[0][1] = movmatrix_t(hb);
       pf[0][2] = movmatrix_t(lt); pf[0][3] = movmatrix_t(lb);
     } else {
-      const float2 *vmA = reinterpret_cast<const float2 *>(st + C::VM_OFF + tA * C::MB);
-      const float2 *vmB = reinterpret_cast<const float2 *>(st + C::VM_OFF + tB * C::MB);
+      const float2 *vmA = vm_row(st, tA);
+      const float2 *vmB = vm_row(st, tB);
 #pragma unroll
       for (int gi = 0; gi < NG; ++gi) {
         const float2 mA = vmA[gi], mB = vmB[gi];
@@ -428,11 +578,9 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
     }
 
     // ---- value product: A = V^T from the lane's segments of 4 positions ----
-    const uint8_t *Vp = st + C::VP_OFF;
     const int T0 = r0 + 2 * c, T1 = T0 + 1, T2 = T0 + 8, T3 = T0 + 9;
     auto vload16 = [&](int t, int k) {  // k-th 16-byte chunk of lane g's segment
-      const int u = g * (C::SV / 16) + k;
-      return *reinterpret_cast<const uint4 *>(Vp + t * C::VSTR + 16 * vswz(C::VSWZ, t, u));
+      return *reinterpret_cast<const uint4 *>(v_chunk(st, t, k));
     };
     if constexpr (BITS == 16) {
       // one word per M-block: (row g, row g+8) of one position
@@ -465,10 +613,10 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
             w[i][4 * k] = x.x; w[i][4 * k + 1] = x.y; w[i][4 * k + 2] = x.z; w[i][4 * k + 3] = x.w;
           }
         } else if constexpr (C::SV == 8) {
-          const uint2 x = *reinterpret_cast<const uint2 *>(Vp + Ts[i] * C::VSTR + 8 * g);
+          const uint2 x = *reinterpret_cast<const uint2 *>(v_small(st, Ts[i]));
           w[i][0] = x.x; w[i][1] = x.y;
         } else {
-          w[i][0] = *reinterpret_cast<const uint32_t *>(Vp + Ts[i] * C::VSTR + 4 * g);
+          w[i][0] = *reinterpret_cast<const uint32_t *>(v_small(st, Ts[i]));
         }
       }
       const uint32_t k1024 = 0x64006400u;
@@ -516,21 +664,42 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
     }
   };
 
-  // ---- cp.async ring over the split's tiles --------------------------------
+  // ---- copy ring over the split's tiles -----------------------------------
 #pragma unroll
   for (int s = 0; s < C::NST - 1; ++s) {
     if (s < n_tiles) issue(s, s);
-    cp_async_commit();
+    if constexpr (!C::TMA) cp_async_commit();
   }
+  bool timed_out = false;
+  int t_stop = n_tiles;  // first tile not consumed
   for (int t = 0; t < n_tiles; ++t) {
-    cp_async_wait<C::NST - 2>();
-    __syncthreads();
+    bool ok = true;
+    if constexpr (C::TMA)
+      ok = mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22);
+    else
+      cp_async_wait<C::NST - 2>();
+    // every thread has finished tile t-1, and all agree whether a wait gave up
+    if (__syncthreads_or(!ok)) {
+      timed_out = true;
+      t_stop = t;
+      if (tid == 0) set_err(a.err, 8);
+      break;
+    }
     const int nt = t + C::NST - 1;
     if (nt < n_tiles) issue(nt, nt % C::NST);
-    cp_async_commit();
+    if constexpr (!C::TMA) cp_async_commit();
     compute(t, t % C::NST);
   }
-  cp_async_wait<0>();
+  if constexpr (C::TMA) {
+    if (timed_out) {
+      // let copies still in flight land (bounded) before the CTA leaves:
+      // tiles t_stop .. t_stop + NST - 2 were issued and not consumed
+      const int t_end = min(n_tiles, t_stop + C::NST - 1);
+      for (int u = t_stop; u < t_end; ++u) mbar_wait(&bars[u % C::NST], (u / C::NST) & 1, 1u << 20);
+    }
+  } else {
+    cp_async_wait<0>();
+  }
   __syncthreads();
 
   // ---- finish this warp's state ------------------------------------------
@@ -567,26 +736,28 @@ __global__ void __launch_bounds__(128) gqa_decode_kernel(const GqaDecodeArgs a) 
 
   // ---- merge the four warps; write output or split partial ---------------
   const size_t row0 = (size_t)b * a.Hq + (size_t)kvh * a.G;
-  for (int e = tid; e < a.G * RS; e += 128) {
-    const int h = e / RS, ch = e - h * RS;
+  for (int h = 0; h < a.G; ++h) {
     float M = -INFINITY;
 #pragma unroll
     for (int w = 0; w < 4; ++w) M = fmaxf(M, red[(w * 8 + h) * RS + D]);
-    float A = 0.f, L = 0.f;
-    if (M != -INFINITY) {
+    float wt[4], L = 0.f;
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        const float mw = red[(w * 8 + h) * RS + D];
-        const float sc = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-        L += sc * red[(w * 8 + h) * RS + D + 1];
-        if (ch < D) A += sc * red[(w * 8 + h) * RS + ch];
-      }
+    for (int w = 0; w < 4; ++w) {
+      const float mw = red[(w * 8 + h) * RS + D];
+      wt[w] = (mw == -INFINITY || M == -INFINITY) ? 0.f : exp2f(mw - M);
+      L += wt[w] * red[(w * 8 + h) * RS + D + 1];
     }
-    if (a.out) {
-      if (ch < D) a.out[(row0 + h) * D + ch] = (L > 0.f) ? A / L : 0.f;
-    } else {
-      float *pr = a.partial + ((size_t)split * gridDim.z * a.Hq + row0 + h) * RS;
-      pr[ch] = (ch < D) ? A : (ch == D ? M : L);
+    for (int ch = tid; ch < D; ch += 128) {
+      float A = 0.f;
+#pragma unroll
+      for (int w = 0; w < 4; ++w) A += wt[w] * red[(w * 8 + h) * RS + ch];
+      if (a.out) {
+        a.out[(row0 + h) * D + ch] = (L > 0.f) ? A / L : 0.f;
+      } else {
+        float *pr = a.partial + ((size_t)split * gridDim.z * a.Hq + row0 + h) * RS;
+        pr[ch] = A;
+        if (ch == 0) { pr[D] = M; pr[D + 1] = L; }
+      }
     }
   }
 }

@@ -204,8 +204,10 @@ kvk_status check_layer_index(const kvk_cache *c, int layer) {
   return KVK_OK;
 }
 
-// Split count that best fills the GPU: whole waves of CTAs and equal tile
-// counts per split, preferring fewer splits when two choices are within 1%.
+// Split count that best fills the GPU: whole waves of CTAs, equal tile
+// counts per split, and at least 16 tiles (1024 positions) per CTA so the
+// per-CTA query set-up and merge stay a small share of its work.  Among
+// choices within 1% the fewer splits win.
 int choose_splits(int units, int tiles, int slots, int max_splits) {
   if (tiles <= 1) return 1;
   const int smax = std::max(1, std::min(max_splits, tiles));
@@ -217,7 +219,8 @@ int choose_splits(int units, int tiles, int slots, int max_splits) {
     const double eff_w = waves / std::ceil(waves);
     const double per = (double)tiles / s;
     const double eff_t = per / std::ceil(per);
-    const double eff = eff_w * eff_t * (per < 2.0 ? 0.9 : 1.0);
+    const double eff_a = per >= 16.0 ? 1.0 : 0.75 + 0.25 * per / 16.0;
+    const double eff = eff_w * eff_t * eff_a;
     if (eff > best_eff * 1.01) {
       best_eff = eff;
       best = s;
