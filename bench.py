@@ -218,9 +218,14 @@ def main():
     ap.add_argument("--impl", default="kvk")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--profile-case", choices=["gqa", "mla"], default=None,
+                    help="small ncu case: decode launches only, no timing line")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
+        return
+    if args.profile_case:
+        profile_case(args.profile_case)
         return
 
     import torch
@@ -428,6 +433,45 @@ def main():
             "device_error": err,
         }
         print(json.dumps(rec))
+
+
+def profile_case(kind):
+    """The kernel-level ncu case.  gqa: one int4 g32 and one bf16 anchor at
+    the 14B step shape (B=32, 8 kv / 40 q heads, d_h 128, T=8192; 1.5 GB of
+    cache, both anchors larger than L2); each decode runs 3 times in the order
+    int4, bf16.  mla: one d=512 latent layer at B=64, T=4096 (302 MB)."""
+    import torch
+    from __graft_entry__ import build
+    build()
+    from paper_2609_37988_gb300 import workloads as W
+    from paper_2609_37988_gb300.cache import Cache, Layer
+    torch.cuda.set_device(0)
+    if kind == "gqa":
+        w = W.config(3)
+        layers = [Layer(bits=4, group=32), Layer(bits=16)]
+        c = Cache(n_layers=2, n_q_heads=40, n_kv_heads=8, head_dim=128, max_batch=32,
+                  max_ctx=8192, layers=layers)
+        for l in range(2):
+            k, v = W.kv_inputs(w, l, 0, 8192, device="cuda")
+            c.append(l, k, v)
+            del k, v
+        q = W.queries(w, 0, device="cuda")
+        for _ in range(3):
+            for l in range(2):
+                c.decode(l, q, w.sigma)
+    else:
+        w = W.config(4, n_layers=1)
+        w.layers[0]["width"] = 512
+        c = Cache(kind="mla", n_layers=1, n_q_heads=16, head_dim=128, latent_dim=512, rope_dim=64,
+                  max_batch=w.batch, max_ctx=w.context, layers=[Layer(bits=16, width=512)])
+        cl, kr = W.mla_inputs(w, 0, 0, w.context, device="cuda")
+        c.append(0, cl, kr)
+        wk, wv = W.mla_weights(w, 0, device="cuda")
+        qn, qp = W.mla_queries(w, 0, device="cuda")
+        for _ in range(3):
+            c.decode_mla(0, qn, qp, wk, wv, w.sigma)
+    torch.cuda.synchronize()
+    print(f"profile case {kind}: ok, device error {c.device_error()}")
 
 
 def _source_hash():
