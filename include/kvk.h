@@ -213,6 +213,30 @@ kvk_status kvk_decode_partial(kvk_cache *cache, int32_t layer, const void *q,
                               int32_t q_dtype, float softmax_scale, float *partials,
                               int32_t n_splits, kvk_stream stream);
 
+/* Decode attention exactly like kvk_decode_attention, for callers that
+ * cannot provide scratch device memory: for example a process whose device
+ * memory belongs to another allocator or is planned to a fixed budget, which
+ * may not call cudaMalloc to size a workspace for its largest split count.
+ * (The paper has no counterpart; this is a deployment convenience.)
+ *  - Allocates nothing and calls no allocating routine.  The split-K
+ *    partials go to one fixed buffer of 16 MiB (4,194,304 floats) compiled
+ *    into the library; every GPU that loads the library holds that buffer
+ *    until the process exits.
+ *  - A call needing more than n_splits * max_batch * n_q_heads *
+ *    (head_dim + 2) <= 4,194,304 floats returns KVK_ERR_CAPACITY and
+ *    enqueues nothing; pass fewer splits or use kvk_decode_attention.
+ *  - All calls on a device share the buffer, and it keeps the last call's
+ *    contents.  Each call writes every partial it later reads, so nothing
+ *    needs clearing, but calls that overlap on the GPU (different streams,
+ *    or different caches at once) race on it: order them.
+ *  - The first call on each device looks up the buffer's device address
+ *    (with that device current); make that first call before any stream
+ *    capture.
+ * Arguments, layouts and other errors as kvk_decode_attention. */
+kvk_status kvk_decode_attention_noalloc(kvk_cache *cache, int32_t layer, const void *q,
+                                        int32_t q_dtype, float softmax_scale, float *out,
+                                        int32_t n_splits, kvk_stream stream);
+
 /* Merge split partials in the format above:
  *   out[row] = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
  * partials device float [n_splits, n_rows, dim + 2]; out device float

@@ -63,6 +63,7 @@ _SIGS = {
     "kvk_decode_attention": [_P, _I, _P, _I, _F, _P, _I, _P],
     "kvk_decode_attention_mla": [_P, _I, _P, _P, _P, _P, _F, _P, _I, _P],
     "kvk_decode_partial": [_P, _I, _P, _I, _F, _P, _I, _P],
+    "kvk_decode_attention_noalloc": [_P, _I, _P, _I, _F, _P, _I, _P],
     "kvk_splitk_reduce": [_P, _I, _I, _I, _P, _P],
     "kvk_cost": [_P, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
                  ctypes.POINTER(ctypes.c_double)],

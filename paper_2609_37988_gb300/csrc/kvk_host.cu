@@ -532,6 +532,42 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   return KVK_OK;
 }
 
+}  // extern "C"
+
+// Records a failed CUDA call as the thread's last error (for noalloc.cu).
+kvk_status kvk_internal_cuda_error(cudaError_t e, const char *what) { return cuda_fail(e, what); }
+
+// Decode with the split-K partials in device memory the caller of this
+// function chose (`partial`, `partial_floats` floats) instead of the cache's
+// workspace.  Rejects a call whose partials would not fit.  Used by the
+// fixed-scratch entry point in noalloc.cu; not part of the C ABI.
+kvk_status kvk_internal_decode_with_partials(kvk_cache *c, int32_t layer, const void *q,
+                                             int32_t q_dtype, float scale, float *out,
+                                             int32_t n_splits, float *partial,
+                                             size_t partial_floats, kvk_stream stream) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->desc.kind != KVK_KIND_GQA) return fail(KVK_ERR_INVALID_ARG, "cache is not GQA");
+  if (!out || !aligned16(out)) return fail(KVK_ERR_INVALID_ARG, "null or misaligned out");
+  if (n_splits < 0 || n_splits > c->max_splits)
+    return fail(KVK_ERR_INVALID_ARG, "n_splits %d outside [0, %d]", n_splits, c->max_splits);
+  const int a = c->src[layer];
+  const int tiles = layer_tiles(c, a);
+  int ns = n_splits == 0 ? auto_splits(c, a) : n_splits;
+  ns = std::min(ns, tiles);
+  const size_t need = ns > 1 ? (size_t)ns * c->desc.max_batch * c->desc.n_q_heads *
+                                   ((size_t)c->desc.head_dim + 2)
+                             : 0;
+  if (need > partial_floats)
+    return fail(KVK_ERR_CAPACITY,
+                "layer %d: %d splits x %d rows need %zu partial floats; the fixed buffer "
+                "holds %zu (use fewer splits or kvk_decode_attention)",
+                layer, ns, c->desc.max_batch * c->desc.n_q_heads, need, partial_floats);
+  return gqa_decode_common(c, layer, q, q_dtype, scale, out, partial, ns, true, stream);
+}
+
+extern "C" {
+
 kvk_status kvk_decode_attention(kvk_cache *c, int32_t layer, const void *q, int32_t q_dtype,
                                 float softmax_scale, float *out, int32_t n_splits,
                                 kvk_stream stream) {
