@@ -125,6 +125,13 @@ __device__ __forceinline__ void ldmatrix_x2(uint32_t &r0, uint32_t &r1, const vo
                : "r"(smem_u32(p)));
 }
 
+// 2^x with the SFU (ex2.approx.ftz: relative error < 2^-22); -inf -> 0.
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // ---- packing -------------------------------------------------------------
 __device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
   __half2 h = __floats2half2_rn(lo, hi);

@@ -19,6 +19,12 @@ cudaError_t launch_gqa_decode(const GqaDecodeArgs &a, cudaStream_t st) {
   }
 }
 
+// positions per decode tile: 128 for per-token 4-bit keys, else 64
+int gqa_decode_tile(int bits, int D, int key_axis, int group) {
+  (void)D; (void)group;
+  return (bits == 4 && key_axis == 0) ? 128 : 64;
+}
+
 int gqa_decode_ctas_per_sm(int bits, int D, int key_axis, int group) {
   switch (bits) {
     case 16: return gqa_ctas_b16(D, key_axis, group);

@@ -62,15 +62,20 @@ struct GqaCfg {
   static constexpr int KM_OFF = VP_OFF + kTile * VSTR;
   static constexpr int VM_OFF = KM_OFF + (KPT ? kTile * MB : 0);
   static constexpr int KG_OFF = VM_OFF + (QUANT ? kTile * MB : 0);
+  // row blocks of 16 per warp and tile height: two blocks for per-token
+  // 4-bit keys (more independent work per warp, shared softmax reductions)
+  static constexpr int RB = (KPT && BITS == 4) ? 2 : 1;
+  static constexpr int TILE = 64 * RB;
   static constexpr int KG_ROWS = KPC ? kTile / GS : 0;
   // Quantised caches: a stage is 64 raw records (one bulk copy) followed by
   // the tile's key-group metadata rows.  bf16 caches: planes filled by
   // 16-byte copies with conflict-free swizzles.
   static constexpr bool TMA = QUANT;
-  static constexpr int KG_OFF_T = kTile * REC;
+  static constexpr int KG_OFF_T = TILE * REC;
   static constexpr int STAGE = TMA ? KG_OFF_T + KG_ROWS * D * 8 : KG_OFF + KG_ROWS * D * 8;
-  static constexpr int NST = TMA ? (STAGE <= 13312 ? 4 : 3) : 2;
-  static constexpr int MIN_CTAS = BF ? 3 : (NST == 4 ? 4 : 3);
+  static constexpr int NST = TMA ? (STAGE <= 13312 ? 4 : (STAGE <= 20480 ? 3 : 2)) : 2;
+  static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");
+  static constexpr int MIN_CTAS = (BF || NST != 4) ? 3 : 4;
   static constexpr int QSTR = D + 4;  // padded query row (floats): conflict-free head rows
   static constexpr int Q_BYTES = 8 * QSTR * 4 + 2 * 8 * NG * 4;
   static constexpr int BAR_OFF = Q_BYTES + NST * STAGE;
@@ -196,7 +201,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   const size_t slab = (size_t)b * v.Hkv + kvh;
   const uint8_t *rec = v.rec + slab * (size_t)v.cap * C::REC;
   const float2 *gmeta = C::KPC ? v.gmeta + slab * (size_t)(v.cap / GS) * D : nullptr;
-  const int n_tiles = i1 > i0 ? (i1 - i0 + kTile - 1) / kTile : 0;
+  const int n_tiles = i1 > i0 ? (i1 - i0 + C::TILE - 1) / C::TILE : 0;
 
   // ---- producer: one tile of records into one stage ----------------------
   // Thread tid copies chunk columns u = tid/8 + 16j of rows tid%8 + 8k.  All
@@ -279,9 +284,9 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     for (int q = tid; q < n; q += 128) p[q] = make_uint4(0, 0, 0, 0);
   };
   auto issue_tma = [&](int t, int s) {
-    const int base = i0 + t * kTile;
+    const int base = i0 + t * C::TILE;
     uint8_t *st = stages + s * C::STAGE;
-    const int nrows = min(kTile, i1 - base);
+    const int nrows = min(C::TILE, i1 - base);
     int kgv = 0;  // complete key groups of this tile (per-channel keys)
     if constexpr (C::KPC) kgv = max(0, min(C::KG_ROWS, len / GS - base / GS));
     if (!a.gather) {
@@ -292,13 +297,14 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
         if (C::KPC && kgv > 0)
           bulk_g2s(st + C::KG_OFF_T, gmeta + (size_t)(base / GS) * D, kgv * D * 8, &bars[s]);
       }
-      if (nrows < kTile) zero_rows(st, nrows, kTile);
+      if (nrows < C::TILE) zero_rows(st, nrows, C::TILE);
     } else {
       if (warp == 0) {
-        int pos[2];
-        bool ok[2];
+        constexpr int RPL = C::TILE / 32;  // rows per lane
+        int pos[RPL];
+        bool ok[RPL];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
+        for (int h = 0; h < RPL; ++h) {
           const int row = lane + 32 * h;
           ok[h] = row < nrows;
           pos[h] = ok[h] ? kept[base + row] : 0;
@@ -307,15 +313,16 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
             set_err(a.err, 1);
           }
         }
-        const int nvalid = __popc(__ballot_sync(0xffffffffu, ok[0])) +
-                           __popc(__ballot_sync(0xffffffffu, ok[1]));
+        int nvalid = 0;
+#pragma unroll
+        for (int h = 0; h < RPL; ++h) nvalid += __popc(__ballot_sync(0xffffffffu, ok[h]));
         if (lane == 0) {
           fence_proxy_async();
           mbar_expect_tx(&bars[s], nvalid * C::REC);
         }
         __syncwarp();
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
+        for (int h = 0; h < RPL; ++h) {
           const int row = lane + 32 * h;
           if (ok[h]) {
             bulk_g2s(st + row * C::REC, rec + (size_t)pos[h] * C::REC, C::REC, &bars[s]);
@@ -367,21 +374,15 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     else return reinterpret_cast<const float2 *>(st + C::KG_OFF);
   };
 
-  // ---- consumer: one warp's 16 rows of one stage --------------------------
+  // ---- consumer: one warp's RB blocks of 16 rows of one stage ------------
+  constexpr int RB = C::RB;
   auto compute = [&](int t, int s) {
-    const int base = i0 + t * kTile;
-    const int r0 = 16 * warp;
-    if (base + r0 >= i1) return;  // warp-uniform: no live row
+    const int base = i0 + t * C::TILE;
+    const int wr0 = 16 * RB * warp;
+    if (base + wr0 >= i1) return;  // warp-uniform: no live row
     const uint8_t *st = stages + s * C::STAGE;
-    const int tA = r0 + g, tB = tA + 8;
-    bool vA = base + tA < i1, vB = base + tB < i1;
-    if (a.gather) {
-      if (vA) { const int p = kept[base + tA]; vA = p >= 0 && p < len; }
-      if (vB) { const int p = kept[base + tB]; vB = p >= 0 && p < len; }
-    }
-    float s4[4] = {0.f, 0.f, 0.f, 0.f};
 
-    // lane's K words for rows tA / tB
+    // lane's K words of one row
     auto load_k = [&](int t, uint32_t(&w)[C::NWK]) {
       if constexpr (C::SK >= 16) {
 #pragma unroll
@@ -410,117 +411,139 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       }
     };
 
-    if (C::KPC && base + r0 >= Tq) {
-      // open per-channel key group: bf16 rows of the residual plane, plain
-      // fp32 dot products (at most group-1 positions per sequence).
-      const uint8_t *res = v.resid + slab * (size_t)GS * D * 2;
+    // ---- scores of each 16-row block (raw dot products, fp32) --------------
+    float s4[RB][4];
+    bool vA[RB], vB[RB];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int t = (k < 2 ? tA : tB);
-        const bool ok = (k < 2 ? vA : vB);
-        const int h = 2 * c + (k & 1);
-        float d = 0.f;
-        if (ok) {
-          const uint8_t *row = res + (size_t)((base + t) % GS) * D * 2;
-          for (int ch = 0; ch < D; ++ch) {
-            int by, hi;
-            k_pos(ch, 16, D, &by, &hi);
-            d += q_s[h * QSTR + ch] * bf16_to_f32(*reinterpret_cast<const uint16_t *>(row + by));
+    for (int rb = 0; rb < RB; ++rb) {
+      const int r0 = wr0 + 16 * rb;
+      const int tA = r0 + g, tB = tA + 8;
+      vA[rb] = base + tA < i1;
+      vB[rb] = base + tB < i1;
+      if (a.gather) {
+        if (vA[rb]) { const int p = kept[base + tA]; vA[rb] = p >= 0 && p < len; }
+        if (vB[rb]) { const int p = kept[base + tB]; vB[rb] = p >= 0 && p < len; }
+      }
+      s4[rb][0] = s4[rb][1] = s4[rb][2] = s4[rb][3] = 0.f;
+      if (base + r0 >= i1) continue;
+      if (C::KPC && base + r0 >= Tq) {
+        // open per-channel key group: bf16 rows of the residual plane, plain
+        // fp32 dot products (at most group-1 positions per sequence).
+        const uint8_t *res = v.resid + slab * (size_t)GS * D * 2;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int tt = (k < 2 ? tA : tB);
+          const bool ok = (k < 2 ? vA[rb] : vB[rb]);
+          const int h = 2 * c + (k & 1);
+          float d = 0.f;
+          if (ok) {
+            const uint8_t *row = res + (size_t)((base + tt) % GS) * D * 2;
+            for (int ch = 0; ch < D; ++ch) {
+              int by, hi;
+              k_pos(ch, 16, D, &by, &hi);
+              d += q_s[h * QSTR + ch] * bf16_to_f32(*reinterpret_cast<const uint16_t *>(row + by));
+            }
           }
+          s4[rb][k] = d;
         }
-        s4[k] = d;
-      }
-    } else if constexpr (C::KPC) {
-      // scale of each channel folded into the query for this group of
-      // positions; zero point and 1024-bias enter as one per-head constant.
-      const float2 *kg = kg_rows(st) + (r0 / GS) * D;
-      uint32_t pb[KS][2], pbl[KS][2];
-      float zpart = 0.f, opart = 0.f;
+      } else if constexpr (C::KPC) {
+        // scale of each channel folded into the query for this group of
+        // positions; zero point and 1024-bias enter as one per-head constant.
+        const float2 *kg = kg_rows(st) + (r0 / GS) * D;
+        uint32_t pb[KS][2], pbl[KS][2];
+        float zpart = 0.f, opart = 0.f;
 #pragma unroll
-      for (int js = 0; js < KS; ++js) {
-        const float *qh = q_s + g * QSTR + 16 * js;
-        const float2 *sz = kg + 16 * js;
-        float x[4];
-        const int chs[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+        for (int js = 0; js < KS; ++js) {
+          const float *qh = q_s + g * QSTR + 16 * js;
+          const float2 *sz = kg + 16 * js;
+          float x[4];
+          const int chs[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 m2 = sz[chs[e]];
-          zpart += qh[chs[e]] * m2.y;
-          x[e] = qh[chs[e]] * m2.x;
-          if (BITS == 4 && e >= 2) x[e] *= 0.0625f;
+          for (int e = 0; e < 4; ++e) {
+            const float2 m2 = sz[chs[e]];
+            zpart += qh[chs[e]] * m2.y;
+            x[e] = qh[chs[e]] * m2.x;
+            if (BITS == 4 && e >= 2) x[e] *= 0.0625f;
+          }
+          split2<false>(x[0], x[1], pb[js][0], pbl[js][0]);
+          split2<false>(x[2], x[3], pb[js][1], pbl[js][1]);
+          const float2 h0 = unpack2<false>(pb[js][0]), l0 = unpack2<false>(pbl[js][0]);
+          const float2 h1 = unpack2<false>(pb[js][1]), l1 = unpack2<false>(pbl[js][1]);
+          opart += 1024.f * ((h0.x + l0.x) + (h0.y + l0.y) + (h1.x + l1.x) + (h1.y + l1.y));
         }
-        split2<false>(x[0], x[1], pb[js][0], pbl[js][0]);
-        split2<false>(x[2], x[3], pb[js][1], pbl[js][1]);
-        const float2 h0 = unpack2<false>(pb[js][0]), l0 = unpack2<false>(pbl[js][0]);
-        const float2 h1 = unpack2<false>(pb[js][1]), l1 = unpack2<false>(pbl[js][1]);
-        opart += 1024.f * ((h0.x + l0.x) + (h0.y + l0.y) + (h1.x + l1.x) + (h1.y + l1.y));
-      }
-      zpart += __shfl_xor_sync(0xffffffffu, zpart, 1);
-      zpart += __shfl_xor_sync(0xffffffffu, zpart, 2);
-      opart += __shfl_xor_sync(0xffffffffu, opart, 1);
-      opart += __shfl_xor_sync(0xffffffffu, opart, 2);
-      const float corr = zpart - opart;  // head g
-      const float corr0 = __shfl_sync(0xffffffffu, corr, (2 * c) * 4);
-      const float corr1 = __shfl_sync(0xffffffffu, corr, (2 * c + 1) * 4);
-      uint32_t wa[C::NWK], wb[C::NWK];
-      load_k(tA, wa);
-      load_k(tB, wb);
-      float d[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int js = 0; js < KS; ++js) {
-        uint32_t a0, a1, a2, a3;
-        kfrag(wa, wb, js, a0, a1, a2, a3);
-        mma_f16(d, a0, a1, a2, a3, pb[js][0], pb[js][1]);
-        mma_f16(d, a0, a1, a2, a3, pbl[js][0], pbl[js][1]);
-      }
-      s4[0] = d[0] + corr0; s4[1] = d[1] + corr1;
-      s4[2] = d[2] + corr0; s4[3] = d[3] + corr1;
-    } else {
-      uint32_t wa[C::NWK], wb[C::NWK];
-      load_k(tA, wa);
-      load_k(tB, wb);
-      if constexpr (BF) {
-        float d[4] = {0.f, 0.f, 0.f, 0.f};
+        zpart += __shfl_xor_sync(0xffffffffu, zpart, 1);
+        zpart += __shfl_xor_sync(0xffffffffu, zpart, 2);
+        opart += __shfl_xor_sync(0xffffffffu, opart, 1);
+        opart += __shfl_xor_sync(0xffffffffu, opart, 2);
+        const float corr = zpart - opart;  // head g
+        const float corr0 = __shfl_sync(0xffffffffu, corr, (2 * c) * 4);
+        const float corr1 = __shfl_sync(0xffffffffu, corr, (2 * c + 1) * 4);
+        uint32_t wa[C::NWK], wb[C::NWK];
+        load_k(tA, wa);
+        load_k(tB, wb);
+        float d[4] = {corr0, corr1, corr0, corr1};
 #pragma unroll
         for (int js = 0; js < KS; ++js) {
           uint32_t a0, a1, a2, a3;
           kfrag(wa, wb, js, a0, a1, a2, a3);
-          mma_bf16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
-          if (use_lo) mma_bf16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
+          mma_f16(d, a0, a1, a2, a3, pb[js][0], pb[js][1]);
+          mma_f16(d, a0, a1, a2, a3, pbl[js][0], pbl[js][1]);
         }
 #pragma unroll
-        for (int k = 0; k < 4; ++k) s4[k] = d[k];
+        for (int k = 0; k < 4; ++k) s4[rb][k] = d[k];
       } else {
-        const float2 *kmA = km_row(st, tA);
-        const float2 *kmB = km_row(st, tB);
-        constexpr int JPG = GS / 16;  // k-steps per group
-#pragma unroll
-        for (int gi = 0; gi < NG; ++gi) {
+        uint32_t wa[C::NWK], wb[C::NWK];
+        load_k(tA, wa);
+        load_k(tB, wb);
+        if constexpr (BF) {
           float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int jj = 0; jj < JPG; ++jj) {
-            const int js = gi * JPG + jj;
+          for (int js = 0; js < KS; ++js) {
             uint32_t a0, a1, a2, a3;
             kfrag(wa, wb, js, a0, a1, a2, a3);
-            mma_f16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
-            if (use_lo) mma_f16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
+            mma_bf16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
+            if (use_lo) mma_bf16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
           }
-          const float2 mA = kmA[gi], mB = kmB[gi];
-          s4[0] += mA.x * (d[0] - qoff[gi][0]) + mA.y * qs[gi][0];
-          s4[1] += mA.x * (d[1] - qoff[gi][1]) + mA.y * qs[gi][1];
-          s4[2] += mB.x * (d[2] - qoff[gi][0]) + mB.y * qs[gi][0];
-          s4[3] += mB.x * (d[3] - qoff[gi][1]) + mB.y * qs[gi][1];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) s4[rb][k] = d[k];
+        } else {
+          const float2 *kmA = km_row(st, tA);
+          const float2 *kmB = km_row(st, tB);
+          constexpr int JPG = GS / 16;  // k-steps per group
+#pragma unroll
+          for (int gi = 0; gi < NG; ++gi) {
+            // the accumulator starts at -Qoff, so it ends at D' - Qoff
+            float d[4] = {-qoff[gi][0], -qoff[gi][1], -qoff[gi][0], -qoff[gi][1]};
+#pragma unroll
+            for (int jj = 0; jj < JPG; ++jj) {
+              const int js = gi * JPG + jj;
+              uint32_t a0, a1, a2, a3;
+              kfrag(wa, wb, js, a0, a1, a2, a3);
+              mma_f16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
+              if (use_lo) mma_f16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
+            }
+            const float2 mA = kmA[gi], mB = kmB[gi];
+            s4[rb][0] = fmaf(mA.x, d[0], fmaf(mA.y, qs[gi][0], s4[rb][0]));
+            s4[rb][1] = fmaf(mA.x, d[1], fmaf(mA.y, qs[gi][1], s4[rb][1]));
+            s4[rb][2] = fmaf(mB.x, d[2], fmaf(mB.y, qs[gi][0], s4[rb][2]));
+            s4[rb][3] = fmaf(mB.x, d[3], fmaf(mB.y, qs[gi][1], s4[rb][3]));
+          }
         }
       }
     }
 
-    // ---- online softmax (base-2 exponent, lazy rescaling) ------------------
-    float x[4];
-    x[0] = vA ? s4[0] * a.sig_log2 : -INFINITY;
-    x[1] = vA ? s4[1] * a.sig_log2 : -INFINITY;
-    x[2] = vB ? s4[2] * a.sig_log2 : -INFINITY;
-    x[3] = vB ? s4[3] * a.sig_log2 : -INFINITY;
-    float mt0 = fmaxf(x[0], x[2]), mt1 = fmaxf(x[1], x[3]);
+    // ---- online softmax over the warp's rows (base 2, lazy rescaling) ------
+    float p[RB][4];
+    float mt0 = -INFINITY, mt1 = -INFINITY;
+#pragma unroll
+    for (int rb = 0; rb < RB; ++rb) {
+      p[rb][0] = vA[rb] ? s4[rb][0] * a.sig_log2 : -INFINITY;
+      p[rb][1] = vA[rb] ? s4[rb][1] * a.sig_log2 : -INFINITY;
+      p[rb][2] = vB[rb] ? s4[rb][2] * a.sig_log2 : -INFINITY;
+      p[rb][3] = vB[rb] ? s4[rb][3] * a.sig_log2 : -INFINITY;
+      mt0 = fmaxf(mt0, fmaxf(p[rb][0], p[rb][2]));
+      mt1 = fmaxf(mt1, fmaxf(p[rb][1], p[rb][3]));
+    }
 #pragma unroll
     for (int off = 4; off < 32; off <<= 1) {
       mt0 = fmaxf(mt0, __shfl_xor_sync(0xffffffffu, mt0, off));
@@ -531,8 +554,8 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     const bool need = (mt0 > m_run[0] + 8.f) || (mt1 > m_run[1] + 8.f);
     if (__any_sync(0xffffffffu, need)) {
       const float n0 = fmaxf(m_run[0], mt0), n1 = fmaxf(m_run[1], mt1);
-      const float al0 = (n0 == -INFINITY) ? 1.f : exp2f(m_run[0] - n0);
-      const float al1 = (n1 == -INFINITY) ? 1.f : exp2f(m_run[1] - n1);
+      const float al0 = (n0 == -INFINITY) ? 1.f : fast_exp2(m_run[0] - n0);
+      const float al1 = (n1 == -INFINITY) ? 1.f : fast_exp2(m_run[1] - n1);
 #pragma unroll
       for (int m = 0; m < KS; ++m) {
         acc[m][0] *= al0; acc[m][2] *= al0;
@@ -543,122 +566,126 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       for (int gi = 0; gi < NG; ++gi) { zacc[gi][0] *= al0; zacc[gi][1] *= al1; }
       m_run[0] = n0; m_run[1] = n1;
     }
-    float p[4];
-    p[0] = (m_run[0] == -INFINITY) ? 0.f : exp2f(x[0] - m_run[0]);
-    p[1] = (m_run[1] == -INFINITY) ? 0.f : exp2f(x[1] - m_run[1]);
-    p[2] = (m_run[0] == -INFINITY) ? 0.f : exp2f(x[2] - m_run[0]);
-    p[3] = (m_run[1] == -INFINITY) ? 0.f : exp2f(x[3] - m_run[1]);
-    l_run[0] += p[0] + p[2];
-    l_run[1] += p[1] + p[3];
-
-    // ---- P^T fragments (B operand of the value MMA) ------------------------
-    // P' = p * scale per channel group (quantised) or P (bf16), split hi/lo,
-    // transposed from the score accumulator layout with movmatrix.
-    uint32_t pf[NG][4];
-    if constexpr (BF) {
-      uint32_t ht, lt, hb, lb;
-      split2<true>(p[0], p[1], ht, lt);
-      split2<true>(p[2], p[3], hb, lb);
-      pf[0][0] = movmatrix_t(ht); pf[0][1] = movmatrix_t(hb);
-      pf[0][2] = movmatrix_t(lt); pf[0][3] = movmatrix_t(lb);
-    } else {
-      const float2 *vmA = vm_row(st, tA);
-      const float2 *vmB = vm_row(st, tB);
+    {
+      const bool live0 = m_run[0] != -INFINITY, live1 = m_run[1] != -INFINITY;
 #pragma unroll
-      for (int gi = 0; gi < NG; ++gi) {
-        const float2 mA = vmA[gi], mB = vmB[gi];
-        uint32_t ht, lt, hb, lb;
-        split2<false>(p[0] * mA.x, p[1] * mA.x, ht, lt);
-        split2<false>(p[2] * mB.x, p[3] * mB.x, hb, lb);
-        pf[gi][0] = movmatrix_t(ht); pf[gi][1] = movmatrix_t(hb);
-        pf[gi][2] = movmatrix_t(lt); pf[gi][3] = movmatrix_t(lb);
-        zacc[gi][0] += p[0] * mA.y + p[2] * mB.y;
-        zacc[gi][1] += p[1] * mA.y + p[3] * mB.y;
+      for (int rb = 0; rb < RB; ++rb) {
+        p[rb][0] = live0 ? fast_exp2(p[rb][0] - m_run[0]) : 0.f;
+        p[rb][1] = live1 ? fast_exp2(p[rb][1] - m_run[1]) : 0.f;
+        p[rb][2] = live0 ? fast_exp2(p[rb][2] - m_run[0]) : 0.f;
+        p[rb][3] = live1 ? fast_exp2(p[rb][3] - m_run[1]) : 0.f;
+        l_run[0] += p[rb][0] + p[rb][2];
+        l_run[1] += p[rb][1] + p[rb][3];
       }
     }
 
-    // ---- value product: A = V^T from the lane's segments of 4 positions ----
-    const int T0 = r0 + 2 * c, T1 = T0 + 1, T2 = T0 + 8, T3 = T0 + 9;
-    auto vload16 = [&](int t, int k) {  // k-th 16-byte chunk of lane g's segment
-      return *reinterpret_cast<const uint4 *>(v_chunk(st, t, k));
-    };
+    // ---- value product: A = V^T from the lanes' segments of 4 positions ----
     if constexpr (BITS == 16) {
-      // one word per M-block: (row g, row g+8) of one position
 #pragma unroll
-      for (int k = 0; k < C::SV / 16; ++k) {
-        const uint4 w0 = vload16(T0, k), w1 = vload16(T1, k), w2 = vload16(T2, k),
-                    w3 = vload16(T3, k);
-        const uint32_t x0[4] = {w0.x, w0.y, w0.z, w0.w}, x1[4] = {w1.x, w1.y, w1.z, w1.w};
-        const uint32_t x2[4] = {w2.x, w2.y, w2.z, w2.w}, x3[4] = {w3.x, w3.y, w3.z, w3.w};
+      for (int rb = 0; rb < RB; ++rb) {
+        const int r0 = wr0 + 16 * rb;
+        if (base + r0 >= i1) continue;
+        // P^T fragments: P split hi/lo, transposed from the score layout
+        uint32_t pf[4];
+        {
+          uint32_t ht, lt, hb, lb;
+          split2<true>(p[rb][0], p[rb][1], ht, lt);
+          split2<true>(p[rb][2], p[rb][3], hb, lb);
+          pf[0] = movmatrix_t(ht); pf[1] = movmatrix_t(hb);
+          pf[2] = movmatrix_t(lt); pf[3] = movmatrix_t(lb);
+        }
+        const int T0 = r0 + 2 * c, T1 = T0 + 1, T2 = T0 + 8, T3 = T0 + 9;
+        // one word per M-block: (row g, row g+8) of one position
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int m = 4 * k + q;
-          const uint32_t a0 = __byte_perm(x0[q], x1[q], 0x5410);
-          const uint32_t a1 = __byte_perm(x0[q], x1[q], 0x7632);
-          const uint32_t a2 = __byte_perm(x2[q], x3[q], 0x5410);
-          const uint32_t a3 = __byte_perm(x2[q], x3[q], 0x7632);
-          mma_bf16(acc[m], a0, a1, a2, a3, pf[0][0], pf[0][1]);
-          mma_bf16(acc[m], a0, a1, a2, a3, pf[0][2], pf[0][3]);
+        for (int k = 0; k < C::SV / 16; ++k) {
+          const uint4 w0 = *reinterpret_cast<const uint4 *>(v_chunk(st, T0, k));
+          const uint4 w1 = *reinterpret_cast<const uint4 *>(v_chunk(st, T1, k));
+          const uint4 w2 = *reinterpret_cast<const uint4 *>(v_chunk(st, T2, k));
+          const uint4 w3 = *reinterpret_cast<const uint4 *>(v_chunk(st, T3, k));
+          const uint32_t x0[4] = {w0.x, w0.y, w0.z, w0.w}, x1[4] = {w1.x, w1.y, w1.z, w1.w};
+          const uint32_t x2[4] = {w2.x, w2.y, w2.z, w2.w}, x3[4] = {w3.x, w3.y, w3.z, w3.w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int m = 4 * k + q;
+            const uint32_t a0 = __byte_perm(x0[q], x1[q], 0x5410);
+            const uint32_t a1 = __byte_perm(x0[q], x1[q], 0x7632);
+            const uint32_t a2 = __byte_perm(x2[q], x3[q], 0x5410);
+            const uint32_t a3 = __byte_perm(x2[q], x3[q], 0x7632);
+            mma_bf16(acc[m], a0, a1, a2, a3, pf[0], pf[1]);
+            mma_bf16(acc[m], a0, a1, a2, a3, pf[2], pf[3]);
+          }
         }
       }
     } else {
-      uint32_t w[4][C::NWV];
-      const int Ts[4] = {T0, T1, T2, T3};
+      // lane g's value words of the 4 positions of each row block
+      uint32_t w[RB][4][C::NWV];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        if constexpr (C::SV >= 16) {
+      for (int rb = 0; rb < RB; ++rb) {
+        const int T0 = wr0 + 16 * rb + 2 * c;
+        const int Ts[4] = {T0, T0 + 1, T0 + 8, T0 + 9};
 #pragma unroll
-          for (int k = 0; k < C::SV / 16; ++k) {
-            const uint4 x = vload16(Ts[i], k);
-            w[i][4 * k] = x.x; w[i][4 * k + 1] = x.y; w[i][4 * k + 2] = x.z; w[i][4 * k + 3] = x.w;
+        for (int i = 0; i < 4; ++i) {
+          if constexpr (C::SV >= 16) {
+#pragma unroll
+            for (int k = 0; k < C::SV / 16; ++k) {
+              const uint4 x = *reinterpret_cast<const uint4 *>(v_chunk(st, Ts[i], k));
+              w[rb][i][4 * k] = x.x; w[rb][i][4 * k + 1] = x.y;
+              w[rb][i][4 * k + 2] = x.z; w[rb][i][4 * k + 3] = x.w;
+            }
+          } else if constexpr (C::SV == 8) {
+            const uint2 x = *reinterpret_cast<const uint2 *>(v_small(st, Ts[i]));
+            w[rb][i][0] = x.x; w[rb][i][1] = x.y;
+          } else {
+            w[rb][i][0] = *reinterpret_cast<const uint32_t *>(v_small(st, Ts[i]));
           }
-        } else if constexpr (C::SV == 8) {
-          const uint2 x = *reinterpret_cast<const uint2 *>(v_small(st, Ts[i]));
-          w[i][0] = x.x; w[i][1] = x.y;
-        } else {
-          w[i][0] = *reinterpret_cast<const uint32_t *>(v_small(st, Ts[i]));
         }
       }
       const uint32_t k1024 = 0x64006400u;
-      auto vmma = [&](int m, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3) {
-        a0 = hsub2_u32(a0, k1024); a1 = hsub2_u32(a1, k1024);
-        a2 = hsub2_u32(a2, k1024); a3 = hsub2_u32(a3, k1024);
+      uint32_t pf[RB][4];
+#pragma unroll
+      for (int m = 0; m < KS; ++m) {
         const int gi = (16 * m) / GS;
-        mma_f16(acc[m], a0, a1, a2, a3, pf[gi][0], pf[gi][1]);
-        mma_f16(acc[m], a0, a1, a2, a3, pf[gi][2], pf[gi][3]);
-      };
-      if constexpr (BITS == 8) {
-        // word k of a segment: M-blocks 2k (bytes 0,1) and 2k+1 (bytes 2,3)
+        if ((16 * m) % GS == 0) {
+          // P' = p * value scale of this channel group, split hi/lo and
+          // transposed; the zero points accumulate separately.
 #pragma unroll
-        for (int k = 0; k < C::NWV; ++k) {
-          const uint32_t X0 = __byte_perm(w[0][k], w[1][k], 0x5140);
-          const uint32_t X2 = __byte_perm(w[2][k], w[3][k], 0x5140);
-          const uint32_t Y0 = __byte_perm(w[0][k], w[1][k], 0x7362);
-          const uint32_t Y2 = __byte_perm(w[2][k], w[3][k], 0x7362);
-          vmma(2 * k, u8pair_f16(X0, 0x4140), u8pair_f16(X0, 0x4342), u8pair_f16(X2, 0x4140),
-               u8pair_f16(X2, 0x4342));
-          vmma(2 * k + 1, u8pair_f16(Y0, 0x4140), u8pair_f16(Y0, 0x4342),
-               u8pair_f16(Y2, 0x4140), u8pair_f16(Y2, 0x4342));
-        }
-      } else {
-        // word k of a segment: M-blocks 4k..4k+3, one byte each (row g low
-        // nibble, row g+8 high nibble -> 16x, undone at the end)
-#pragma unroll
-        for (int k = 0; k < C::NWV; ++k) {
-#pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            const uint32_t sel = hh ? 0x7632 : 0x5410;
-            uint32_t X0 = __byte_perm(w[0][k], w[1][k], sel);
-            uint32_t X2 = __byte_perm(w[2][k], w[3][k], sel);
-#pragma unroll
-            for (int q = 0; q < 2; ++q) {
-              const int m = 4 * k + 2 * hh + q;
-              vmma(m, nib_f16(X0, 0x000F000Fu), nib_f16(X0, 0x00F000F0u),
-                   nib_f16(X2, 0x000F000Fu), nib_f16(X2, 0x00F000F0u));
-              X0 >>= 8;
-              X2 >>= 8;
-            }
+          for (int rb = 0; rb < RB; ++rb) {
+            const int tA = wr0 + 16 * rb + g;
+            const float2 mA = vm_row(st, tA)[gi], mB = vm_row(st, tA + 8)[gi];
+            uint32_t ht, lt, hb, lb;
+            split2<false>(p[rb][0] * mA.x, p[rb][1] * mA.x, ht, lt);
+            split2<false>(p[rb][2] * mB.x, p[rb][3] * mB.x, hb, lb);
+            pf[rb][0] = movmatrix_t(ht); pf[rb][1] = movmatrix_t(hb);
+            pf[rb][2] = movmatrix_t(lt); pf[rb][3] = movmatrix_t(lb);
+            zacc[gi][0] = fmaf(p[rb][0], mA.y, fmaf(p[rb][2], mB.y, zacc[gi][0]));
+            zacc[gi][1] = fmaf(p[rb][1], mA.y, fmaf(p[rb][3], mB.y, zacc[gi][1]));
           }
+        }
+#pragma unroll
+        for (int rb = 0; rb < RB; ++rb) {
+          uint32_t a0, a1, a2, a3;
+          if constexpr (BITS == 8) {
+            // word m/2 of a segment: M-block m in bytes (0,1) or (2,3)
+            const int k = m >> 1;
+            const uint32_t sel = (m & 1) ? 0x7362 : 0x5140;
+            const uint32_t X0 = __byte_perm(w[rb][0][k], w[rb][1][k], sel);
+            const uint32_t X2 = __byte_perm(w[rb][2][k], w[rb][3][k], sel);
+            a0 = u8pair_f16(X0, 0x4140); a1 = u8pair_f16(X0, 0x4342);
+            a2 = u8pair_f16(X2, 0x4140); a3 = u8pair_f16(X2, 0x4342);
+          } else {
+            // word m/4: one byte per M-block (row g low nibble, row g+8 high
+            // nibble -> 16x, undone at the end)
+            const int k = m >> 2, hh = (m >> 1) & 1, sh = 8 * (m & 1);
+            const uint32_t sel = hh ? 0x7632 : 0x5410;
+            const uint32_t X0 = __byte_perm(w[rb][0][k], w[rb][1][k], sel) >> sh;
+            const uint32_t X2 = __byte_perm(w[rb][2][k], w[rb][3][k], sel) >> sh;
+            a0 = nib_f16(X0, 0x000F000Fu); a1 = nib_f16(X0, 0x00F000F0u);
+            a2 = nib_f16(X2, 0x000F000Fu); a3 = nib_f16(X2, 0x00F000F0u);
+          }
+          a0 = hsub2_u32(a0, k1024); a1 = hsub2_u32(a1, k1024);
+          a2 = hsub2_u32(a2, k1024); a3 = hsub2_u32(a3, k1024);
+          mma_f16(acc[m], a0, a1, a2, a3, pf[rb][0], pf[rb][1]);
+          mma_f16(acc[m], a0, a1, a2, a3, pf[rb][2], pf[rb][3]);
         }
       }
     }
@@ -775,6 +802,11 @@ cudaError_t launch_gqa_decode_t(const GqaDecodeArgs &a, cudaStream_t st) {
   dim3 grid(a.n_splits, a.v.Hkv, a.v.B);
   k<<<grid, 128, C::SMEM, st>>>(a);
   return cudaGetLastError();
+}
+
+template <int BITS, int D, int KAX, int GS>
+int gqa_tile_t() {
+  return GqaCfg<BITS, D, KAX, GS>::TILE;
 }
 
 template <int BITS, int D, int KAX, int GS>

@@ -45,6 +45,7 @@ struct GqaDecodeArgs {
 // (bits, D, key axis, q dtype) happens inside.
 cudaError_t launch_gqa_decode(const GqaDecodeArgs &a, cudaStream_t st);
 int gqa_decode_ctas_per_sm(int bits, int D, int key_axis, int group);
+int gqa_decode_tile(int bits, int D, int key_axis, int group);
 
 struct RewindArgs {
   int32_t *lens[64];

@@ -511,7 +511,10 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   args.G = c->desc.n_q_heads / c->desc.n_kv_heads;
   args.sig_log2 = scale * 1.4426950408889634f;
   args.n_splits = n_splits;
-  const int tps = (tiles + n_splits - 1) / n_splits;
+  // split boundaries fall on the kernel's tile height (64 or 128 positions)
+  const int kt = gqa_decode_tile(args.v.bits, args.v.D, args.v.key_axis, args.v.group);
+  const int per = kt / kTile;
+  const int tps = ((tiles + n_splits - 1) / n_splits + per - 1) / per * per;
   args.items_per_split = tps * kTile;
   args.err = c->err();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
