@@ -127,77 +127,8 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   const bool use_lo = a.q_f32 != 0;
   const int32_t *kept = v.kept_idx + (size_t)b * v.kept_cap;
 
-  for (int e = tid; e < 8 * D; e += 128) {
-    const int h = e / D, ch = e % D;
-    float x = 0.f;
-    if (h < a.G) {
-      const size_t qi = ((size_t)b * a.Hq + (size_t)kvh * a.G + h) * D + ch;
-      x = a.q_f32 ? static_cast<const float *>(a.q)[qi]
-                  : bf16_to_f32(static_cast<const uint16_t *>(a.q)[qi]);
-    }
-    q_s[h * QSTR + ch] = x;
-  }
-  __syncthreads();
-  // per-token key groups: query sums Qs and 1024-bias offsets Qoff of every
-  // (head, channel group), with the f16 values the score MMA actually uses;
-  // 128 / (8 NG) lanes per (head, group), reduced with shuffles.
-  if constexpr (C::KPT) {
-    constexpr int ITEMS = 8 * NG, LPI = 128 / ITEMS, CPL = GS / LPI;
-    const int item = tid / LPI, sub = tid % LPI;
-    const int h = item / NG, gi = item % NG;
-    const bool use_lo0 = a.q_f32 != 0;
-    float sq = 0.f, so = 0.f;
-#pragma unroll 4
-    for (int k = 0; k < CPL; ++k) {
-      const int ch = gi * GS + sub * CPL + k;
-      const bool hs = (BITS == 4) && ((ch & 15) >= 8);
-      const float x = q_s[h * QSTR + ch];
-      const float xs = hs ? x * 0.0625f : x;
-      float xe = __half2float(__float2half_rn(xs));
-      if (use_lo0) xe += __half2float(__float2half_rn(xs - xe));
-      sq += hs ? 16.f * xe : xe;
-      so += 1024.f * xe;
-    }
-#pragma unroll
-    for (int off = 1; off < LPI; off <<= 1) {
-      sq += __shfl_xor_sync(0xffffffffu, sq, off);
-      so += __shfl_xor_sync(0xffffffffu, so, off);
-    }
-    if (sub == 0) { qs_s[item] = sq; qo_s[item] = so; }
-    __syncthreads();
-  }
-
-  // ---- query fragments (B operand of the score MMA), head n = g ----------
-  uint32_t qb[KS][2], qbl[KS][2];
-  if constexpr (!C::KPC) {
-#pragma unroll
-    for (int js = 0; js < KS; ++js) {
-      const float *qh = q_s + g * QSTR + 16 * js;
-      float x2 = qh[2 * c + 8], x3 = qh[2 * c + 9];
-      if (BITS == 4) { x2 *= 0.0625f; x3 *= 0.0625f; }
-      split2<BF>(qh[2 * c], qh[2 * c + 1], qb[js][0], qbl[js][0]);
-      split2<BF>(x2, x3, qb[js][1], qbl[js][1]);
-    }
-  }
-  float qs[NG][2], qoff[NG][2];
-  if constexpr (C::KPT) {
-#pragma unroll
-    for (int gi = 0; gi < NG; ++gi)
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        qs[gi][hh] = qs_s[(2 * c + hh) * NG + gi];
-        qoff[gi][hh] = qo_s[(2 * c + hh) * NG + gi];
-      }
-  }
-
-  float acc[KS][4];
-#pragma unroll
-  for (int m = 0; m < KS; ++m) acc[m][0] = acc[m][1] = acc[m][2] = acc[m][3] = 0.f;
-  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-  float zacc[NG][2];
-#pragma unroll
-  for (int gi = 0; gi < NG; ++gi) zacc[gi][0] = zacc[gi][1] = 0.f;
-
+  // The copy producer comes first, so the first tiles are in flight while
+  // the query set-up below runs.
   const size_t slab = (size_t)b * v.Hkv + kvh;
   const uint8_t *rec = v.rec + slab * (size_t)v.cap * C::REC;
   const float2 *gmeta = C::KPC ? v.gmeta + slab * (size_t)(v.cap / GS) * D : nullptr;
@@ -341,6 +272,83 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     else
       issue_cp(t, s);
   };
+
+#pragma unroll
+  for (int s = 0; s < C::NST - 1; ++s) {
+    if (s < n_tiles) issue(s, s);
+    if constexpr (!C::TMA) cp_async_commit();
+  }
+
+  for (int e = tid; e < 8 * D; e += 128) {
+    const int h = e / D, ch = e % D;
+    float x = 0.f;
+    if (h < a.G) {
+      const size_t qi = ((size_t)b * a.Hq + (size_t)kvh * a.G + h) * D + ch;
+      x = a.q_f32 ? static_cast<const float *>(a.q)[qi]
+                  : bf16_to_f32(static_cast<const uint16_t *>(a.q)[qi]);
+    }
+    q_s[h * QSTR + ch] = x;
+  }
+  __syncthreads();
+  // per-token key groups: query sums Qs and 1024-bias offsets Qoff of every
+  // (head, channel group), with the f16 values the score MMA actually uses;
+  // 128 / (8 NG) lanes per (head, group), reduced with shuffles.
+  if constexpr (C::KPT) {
+    constexpr int ITEMS = 8 * NG, LPI = 128 / ITEMS, CPL = GS / LPI;
+    const int item = tid / LPI, sub = tid % LPI;
+    const int h = item / NG, gi = item % NG;
+    const bool use_lo0 = a.q_f32 != 0;
+    float sq = 0.f, so = 0.f;
+#pragma unroll 4
+    for (int k = 0; k < CPL; ++k) {
+      const int ch = gi * GS + sub * CPL + k;
+      const bool hs = (BITS == 4) && ((ch & 15) >= 8);
+      const float x = q_s[h * QSTR + ch];
+      const float xs = hs ? x * 0.0625f : x;
+      float xe = __half2float(__float2half_rn(xs));
+      if (use_lo0) xe += __half2float(__float2half_rn(xs - xe));
+      sq += hs ? 16.f * xe : xe;
+      so += 1024.f * xe;
+    }
+#pragma unroll
+    for (int off = 1; off < LPI; off <<= 1) {
+      sq += __shfl_xor_sync(0xffffffffu, sq, off);
+      so += __shfl_xor_sync(0xffffffffu, so, off);
+    }
+    if (sub == 0) { qs_s[item] = sq; qo_s[item] = so; }
+    __syncthreads();
+  }
+
+  // ---- query fragments (B operand of the score MMA), head n = g ----------
+  uint32_t qb[KS][2], qbl[KS][2];
+  if constexpr (!C::KPC) {
+#pragma unroll
+    for (int js = 0; js < KS; ++js) {
+      const float *qh = q_s + g * QSTR + 16 * js;
+      float x2 = qh[2 * c + 8], x3 = qh[2 * c + 9];
+      if (BITS == 4) { x2 *= 0.0625f; x3 *= 0.0625f; }
+      split2<BF>(qh[2 * c], qh[2 * c + 1], qb[js][0], qbl[js][0]);
+      split2<BF>(x2, x3, qb[js][1], qbl[js][1]);
+    }
+  }
+  float qs[NG][2], qoff[NG][2];
+  if constexpr (C::KPT) {
+#pragma unroll
+    for (int gi = 0; gi < NG; ++gi)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        qs[gi][hh] = qs_s[(2 * c + hh) * NG + gi];
+        qoff[gi][hh] = qo_s[(2 * c + hh) * NG + gi];
+      }
+  }
+
+  float acc[KS][4];
+#pragma unroll
+  for (int m = 0; m < KS; ++m) acc[m][0] = acc[m][1] = acc[m][2] = acc[m][3] = 0.f;
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float zacc[NG][2];
+#pragma unroll
+  for (int gi = 0; gi < NG; ++gi) zacc[gi][0] = zacc[gi][1] = 0.f;
 
   // shared-memory addresses of the fragments (raw records or planes)
   auto k_chunk = [&](const uint8_t *st, int t, int i) -> const uint8_t * {
@@ -692,11 +700,6 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   };
 
   // ---- copy ring over the split's tiles -----------------------------------
-#pragma unroll
-  for (int s = 0; s < C::NST - 1; ++s) {
-    if (s < n_tiles) issue(s, s);
-    if constexpr (!C::TMA) cp_async_commit();
-  }
   bool timed_out = false;
   int t_stop = n_tiles;  // first tile not consumed
   for (int t = 0; t < n_tiles; ++t) {
