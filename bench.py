@@ -66,6 +66,21 @@ def algorithmic_bytes(w, lens_after_append):
     return total, per_layer
 
 
+def algorithmic_bytes_mla(w, T):
+    """MLA step: every layer reads its latent cache [c[:d] | k^R] (bf16) at
+    length T, the absorbed/up-projection weight slices W_UK[:, :, :d] and
+    W_UV[:, :, :d], its queries, and writes its output."""
+    B, H = w.batch, w.n_q_heads
+    total, per_layer = 0, []
+    for l in range(w.n_layers):
+        d = w.layers[l]["width"]
+        cache = B * T * (d + w.rope_dim) * 2
+        per_layer.append(cache)
+        total += cache + 2 * H * w.head_dim * d * 2 + B * H * (w.head_dim + w.rope_dim) * 2 + \
+            B * H * w.head_dim * 4
+    return total, per_layer
+
+
 class Clocks:
     """nvidia-smi sampler running during the timed region."""
 
@@ -245,53 +260,76 @@ def main():
     from paper_2609_37988_gb300.cache import Cache, Layer
 
     w = W.config(args.config)
-    if w.kind != "gqa":
-        raise SystemExit("bench.py times the GQA workloads (1, 2, 3, 5)")
     T = w.context
-    pre = T - 1 if w.append_per_step else T
-    cache = Cache(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
-                  head_dim=w.head_dim, max_batch=w.batch, max_ctx=T, layers=[Layer(**a) for a in w.layers],
-                  max_splits=64, device=dev)
-    for a in w.anchors:
-        k, v = W.kv_inputs(w, a, 0, pre, device=dev)
-        cache.append(a, k, v)
-        del k, v
-    if w.keep:
-        import numpy as np
-        for a in w.anchors:
-            idx, n = W.kept_positions(w, a, np.full(w.batch, T), device=dev)
-            cache.set_kept(a, idx, n)
-    torch.cuda.synchronize()
-    qs = [W.queries(w, l, device=dev) for l in range(w.n_layers)]
-    outs = [torch.empty((w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
-            for _ in range(w.n_layers)]
-    new_kv = {}
-    if w.append_per_step:
-        for a in w.anchors:
-            new_kv[a] = W.kv_inputs(w, a, pre, T, device=dev)
     src = w.sources()
-
-    def step():
+    new_kv = {}
+    if w.kind == "mla":
+        cache = Cache(kind="mla", n_layers=w.n_layers, n_q_heads=w.n_q_heads, head_dim=w.head_dim,
+                      latent_dim=w.latent_dim, rope_dim=w.rope_dim, max_batch=w.batch, max_ctx=T,
+                      layers=[Layer(**a) for a in w.layers], max_splits=64, device=dev)
         for l in range(w.n_layers):
-            if l in new_kv:
-                cache.append(l, *new_kv[l])
-            cache.decode(l, qs[l], w.sigma, out=outs[l])
+            cl, kr = W.mla_inputs(w, l, 0, T, device=dev)
+            cache.append(l, cl, kr)
+            del cl, kr
+        mq = [W.mla_queries(w, l, device=dev) for l in range(w.n_layers)]
+        mw = [W.mla_weights(w, l, device=dev) for l in range(w.n_layers)]
+        qs = [torch.cat([a.flatten(), b.flatten()]) for a, b in mq]  # host copies for e2e
+        outs = [torch.empty((w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
+                for _ in range(w.n_layers)]
+
+        def layer_call(l, q_nope=None, q_pe=None):
+            qn, qp = (mq[l] if q_nope is None else (q_nope, q_pe))
+            cache.decode_mla(l, qn, qp, mw[l][0], mw[l][1], w.sigma, out=outs[l])
+
+        def step():
+            for l in range(w.n_layers):
+                layer_call(l)
+    else:
+        pre = T - 1 if w.append_per_step else T
+        cache = Cache(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
+                      head_dim=w.head_dim, max_batch=w.batch, max_ctx=T,
+                      layers=[Layer(**a) for a in w.layers], max_splits=64, device=dev)
+        for a in w.anchors:
+            k, v = W.kv_inputs(w, a, 0, pre, device=dev)
+            cache.append(a, k, v)
+            del k, v
+        if w.keep:
+            import numpy as np
+            for a in w.anchors:
+                idx, n = W.kept_positions(w, a, np.full(w.batch, T), device=dev)
+                cache.set_kept(a, idx, n)
+        qs = [W.queries(w, l, device=dev) for l in range(w.n_layers)]
+        outs = [torch.empty((w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
+                for _ in range(w.n_layers)]
         if w.append_per_step:
-            cache.rewind(1)
+            for a in w.anchors:
+                new_kv[a] = W.kv_inputs(w, a, pre, T, device=dev)
+
+        def step():
+            for l in range(w.n_layers):
+                if l in new_kv:
+                    cache.append(l, *new_kv[l])
+                cache.decode(l, qs[l], w.sigma, out=outs[l])
+            if w.append_per_step:
+                cache.rewind(1)
+    torch.cuda.synchronize()
 
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
         step()  # eager: sets kernel attributes, occupancy queries
         stream.synchronize()
-        splits = [cache.plan_splits(l) for l in range(w.n_layers)]
+        splits = [cache.plan_splits(l) if w.kind == "gqa" else 1 for l in range(w.n_layers)]
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=stream):
             step()
     torch.cuda.synchronize()
-    launches = sum(1 + (splits[l] > 1) for l in range(w.n_layers))
-    launches += len(new_kv) + (1 if w.append_per_step else 0)
-
-    step_bytes, per_layer = algorithmic_bytes(w, T)
+    if w.kind == "mla":
+        launches = 4 * w.n_layers  # absorb, latent decode, merge, up-projection
+        step_bytes, per_layer = algorithmic_bytes_mla(w, T)
+    else:
+        launches = sum(1 + (splits[l] > 1) for l in range(w.n_layers))
+        launches += len(new_kv) + (1 if w.append_per_step else 0)
+        step_bytes, per_layer = algorithmic_bytes(w, T)
 
     def barrier():
         if dist:
@@ -324,15 +362,21 @@ def main():
     with torch.cuda.stream(stream):
         for l in range(w.n_layers):
             a = src[l]
-            kind = "bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}"
+            if w.kind == "mla":
+                kind = f"mla_d{w.layers[l]['width']}"
+            else:
+                kind = "bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}"
             ns = splits[l]
-            part = torch.empty((max(ns, 2), w.batch * w.n_q_heads, w.head_dim + 2), device=dev)
+            if w.kind == "gqa":
+                part = torch.empty((max(ns, 2), w.batch * w.n_q_heads, w.head_dim + 2), device=dev)
             if l in new_kv:
                 cache.append(l, *new_kv[l])
             for r in range(reps):
                 s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 s0.record(stream)
-                if ns > 1:
+                if w.kind == "mla":
+                    layer_call(l)          # the whole MLA call (4 launches)
+                elif ns > 1:
                     cache.decode_partial(l, qs[l], w.sigma, ns, partials=part)
                 else:
                     cache.decode(l, qs[l], w.sigma, out=outs[l], n_splits=1)
@@ -364,7 +408,7 @@ def main():
 
     # ---- end to end through the public API, host buffers --------------------
     e2e = None
-    if args.e2e_steps > 0:
+    if args.e2e_steps > 0 and w.kind == "gqa":
         h_q = [q.cpu().pin_memory() for q in qs]
         h_kv = {a: (k.cpu().pin_memory(), v.cpu().pin_memory()) for a, (k, v) in new_kv.items()}
         h_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
@@ -401,7 +445,7 @@ def main():
 
     err = cache.device_error()
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and w.kind == "gqa":
         g, sample, cores = cpu_baseline(w)
         cpu = {"value": g, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
     clocks = clk.summary()
@@ -409,7 +453,10 @@ def main():
         rec = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "us_per_step": ms_step * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16/int4",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": ("bf16" if w.kind == "mla" else
+                      "/".join(sorted({("bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}")
+                                       for a in w.anchors}))),
             "data": "synthetic",
             "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "context": T,
                        "q_heads": w.n_q_heads, "kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
@@ -418,11 +465,14 @@ def main():
                                    "int8": sum(1 for a in w.anchors if w.layers[a]["bits"] == 8)},
                        "inheritors": w.n_layers - len(w.anchors),
                        "bytes_per_step": step_bytes, "cuda_graph": True,
-                       "l2": "inputs larger than L2 (each anchor >= 403 MB; step reads ~31 GB), no flush",
+                       "l2": (f"no flush; smallest per-layer read {min(per_layer) / 1e6:.0f} MB vs 126 MB L2"
+                              + (" (every layer's read exceeds L2)" if min(per_layer) > 126e6 else
+                                 " (some layers fit in L2; consecutive inheritors may hit it)")),
                        "parallelism": f"replicas x{world}"},
             "fraction_of_peak": value / hbm, "peak_gbs": hbm, "peak_kind": peak_kind,
             "fraction_of_nominal_8tbs": value / 8000.0,
-            "roofline": {"bound": "hbm", "kernel": f"gqa_decode ({dom})", "achieved": achieved,
+            "roofline": {"bound": "hbm", "kernel": (f"gqa_decode ({dom})" if w.kind == "gqa" else
+                                                   f"mla decode call ({dom})"), "achieved": achieved,
                          "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
                          "peak_source": f"MEASURED_PEAKS.json hbm_gbs ({peak_kind})"},
             "kernels": kernels,

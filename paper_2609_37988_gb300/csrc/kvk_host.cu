@@ -205,10 +205,11 @@ kvk_status check_layer_index(const kvk_cache *c, int layer) {
 }
 
 // Split count that best fills the GPU: whole waves of CTAs, equal tile
-// counts per split, and at least 16 tiles (1024 positions) per CTA so the
-// per-CTA query set-up and merge stay a small share of its work.  Among
-// choices within 1% the fewer splits win.
+// counts per split, and at least 16 64-position tiles per CTA so the
+// per-CTA query set-up and the split partials stay a small share of the
+// work.  Among choices within 1% the fewer splits win.
 int choose_splits(int units, int tiles, int slots, int max_splits) {
+  const double min_tiles = 16.0;
   if (tiles <= 1) return 1;
   const int smax = std::max(1, std::min(max_splits, tiles));
   int best = 1;
@@ -219,7 +220,7 @@ int choose_splits(int units, int tiles, int slots, int max_splits) {
     const double eff_w = waves / std::ceil(waves);
     const double per = (double)tiles / s;
     const double eff_t = per / std::ceil(per);
-    const double eff_a = per >= 16.0 ? 1.0 : 0.75 + 0.25 * per / 16.0;
+    const double eff_a = per >= min_tiles ? 1.0 : 0.75 + 0.25 * per / min_tiles;
     const double eff = eff_w * eff_t * eff_a;
     if (eff > best_eff * 1.01) {
       best_eff = eff;
@@ -249,7 +250,15 @@ int auto_splits(kvk_cache *c, int a) {
     }
   }
   const int units = mla ? c->desc.max_batch : c->desc.max_batch * c->desc.n_kv_heads;
-  return choose_splits(units, layer_tiles(c, a), c->sm_count * c->ctas[a], c->max_splits);
+  const int slots = c->sm_count * c->ctas[a];
+  if (mla) {
+    // Latent partials are as wide as the latent, and a second wave of these
+    // long CTAs costs more than it fills: as many splits as keep every CTA
+    // resident at once.
+    const int s = std::max(1, std::min(slots / std::max(1, units), c->max_splits));
+    return std::min(s, std::min(64, layer_tiles(c, a)));
+  }
+  return choose_splits(units, layer_tiles(c, a), slots, c->max_splits);
 }
 
 }  // namespace
@@ -617,7 +626,7 @@ kvk_status kvk_decode_attention_mla(kvk_cache *c, int32_t layer, const void *q_n
   args.v = c->mla_view(a);
   const int tiles = layer_tiles(c, a);
   if (n_splits == 0) n_splits = auto_splits(c, a);
-  n_splits = std::min(n_splits, tiles);
+  n_splits = std::min(std::min(n_splits, tiles), 64);
   args.q_nope = q_nope;
   args.q_pe = q_pe;
   args.w_uk = w_uk;

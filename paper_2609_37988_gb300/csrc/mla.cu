@@ -96,13 +96,6 @@ __global__ void __launch_bounds__(128)
         *reinterpret_cast<uint32_t *>(dst + W + kRope + i) = lo;
       }
     }
-    if (blockIdx.x == 0) {  // copy q_pe beside the hi half
-      for (int q = tid; q < 64 * kRope; q += 128) {
-        const int row = q / kRope, e = q % kRope;
-        const int b = b0 + row;
-        if (b < B) qlat[((size_t)b * H + h) * QROW + W + e] = q_pe[((size_t)b * H + h) * kRope + e];
-      }
-    }
     __syncthreads();
   }
 }
@@ -133,7 +126,8 @@ struct MlaCfg {
 
 template <int W>
 __global__ void __launch_bounds__(256)
-    mla_decode_kernel(const MlaView v, const uint16_t *__restrict__ qlat, int H, float sig_log2,
+    mla_decode_kernel(const MlaView v, const uint16_t *__restrict__ qlat,
+                      const uint16_t *__restrict__ q_pe, int H, float sig_log2,
                       int items_per_split, int n_splits, float *__restrict__ partial,
                       int32_t *err) {
   using C = MlaCfg<W>;
@@ -154,14 +148,19 @@ __global__ void __launch_bounds__(256)
   const int n_tiles = i1 > i0 ? (i1 - i0 + kTile - 1) / kTile : 0;
   const uint8_t *rec = v.rec + (size_t)b * v.cap * C::RB;
 
-  // absorbed query [hi | pe] and [lo] into shared memory, swizzled rows
+  // absorbed query [hi | pe] and [lo] into shared memory, swizzled rows;
+  // q_pe comes straight from the caller's tensor
   {
     constexpr int QROW = 2 * W + kRope;
     const uint16_t *qb = qlat + (size_t)b * H * QROW;
     for (int q = tid; q < kHeads * (C::QH_ROW / 16); q += 256) {
       const int h = q / (C::QH_ROW / 16), u = q % (C::QH_ROW / 16);
       uint4 x = make_uint4(0, 0, 0, 0);
-      if (h < H) x = *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + 8 * u);
+      if (h < H) {
+        x = (u < W / 8) ? *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + 8 * u)
+                        : *reinterpret_cast<const uint4 *>(q_pe + ((size_t)b * H + h) * kRope +
+                                                           8 * (u - W / 8));
+      }
       *reinterpret_cast<uint4 *>(qh_s + h * C::QH_ROW + 16 * swz8(h, u)) = x;
     }
     for (int q = tid; q < kHeads * (C::QL_ROW / 16); q += 256) {
@@ -208,28 +207,38 @@ __global__ void __launch_bounds__(256)
     const int base = i0 + t * kTile;
 
     // ---- scores: 16 positions x 8 heads per warp -------------------------
-    float d[4] = {0.f, 0.f, 0.f, 0.f};
+    // four independent accumulators (hi/lo x even/odd k-steps) so the MMA
+    // chain is not one long dependency
+    float dacc[4][4] = {};
     const int mat = lane >> 3, rr = lane & 7;
+    const int hrow = 8 * nb + rr;
 #pragma unroll 4
-    for (int ks = 0; ks < (W + kRope) / 16; ++ks) {
+    for (int ks = 0; ks < W / 16; ++ks) {
       uint32_t a0, a1, a2, a3;
       {
         const int row = 16 * mb + rr + ((mat & 1) ? 8 : 0);
         ldmatrix_x4(a0, a1, a2, a3, st + row * C::RB + 16 * swz8(row, 2 * ks + (mat >> 1)));
       }
-      const int hrow = 8 * nb + rr;
-      if (ks < W / 16) {
-        uint32_t b0, b1, b2, b3;  // hi (2 chunks) then lo (2 chunks)
-        const uint8_t *base_q = (mat < 2) ? qh_s + hrow * C::QH_ROW : ql_s + hrow * C::QL_ROW;
-        ldmatrix_x4(b0, b1, b2, b3, base_q + 16 * swz8(hrow, 2 * ks + (mat & 1)));
-        mma_bf16(d, a0, a1, a2, a3, b0, b1);
-        mma_bf16(d, a0, a1, a2, a3, b2, b3);
-      } else {
-        uint32_t b0, b1;
-        ldmatrix_x2(b0, b1, qh_s + hrow * C::QH_ROW + 16 * swz8(hrow, 2 * ks + (mat & 1)));
-        mma_bf16(d, a0, a1, a2, a3, b0, b1);
-      }
+      uint32_t b0, b1, b2, b3;  // hi (2 chunks) then lo (2 chunks)
+      const uint8_t *base_q = (mat < 2) ? qh_s + hrow * C::QH_ROW : ql_s + hrow * C::QL_ROW;
+      ldmatrix_x4(b0, b1, b2, b3, base_q + 16 * swz8(hrow, 2 * ks + (mat & 1)));
+      mma_bf16(dacc[(ks & 1) * 2], a0, a1, a2, a3, b0, b1);
+      mma_bf16(dacc[(ks & 1) * 2 + 1], a0, a1, a2, a3, b2, b3);
     }
+#pragma unroll
+    for (int ks = W / 16; ks < (W + kRope) / 16; ++ks) {
+      uint32_t a0, a1, a2, a3;
+      {
+        const int row = 16 * mb + rr + ((mat & 1) ? 8 : 0);
+        ldmatrix_x4(a0, a1, a2, a3, st + row * C::RB + 16 * swz8(row, 2 * ks + (mat >> 1)));
+      }
+      uint32_t b0, b1;
+      ldmatrix_x2(b0, b1, qh_s + hrow * C::QH_ROW + 16 * swz8(hrow, 2 * ks + (mat & 1)));
+      mma_bf16(dacc[ks & 3], a0, a1, a2, a3, b0, b1);
+    }
+    float d[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) d[k] = (dacc[0][k] + dacc[1][k]) + (dacc[2][k] + dacc[3][k]);
     const bool vA = base + 16 * mb + g < i1, vB = base + 16 * mb + g + 8 < i1;
     float x[4];
     x[0] = vA ? d[0] * sig_log2 : -INFINITY;
@@ -259,7 +268,7 @@ __global__ void __launch_bounds__(256)
                          fmaxf(tmax_s[2 * kHeads + h], tmax_s[3 * kHeads + h]));
         alpha[n2][hh] = 1.f;
         if (mt > m_run[n2][hh] + 8.f) {  // lazy: keep a stale max within 2^8
-          alpha[n2][hh] = (m_run[n2][hh] == -INFINITY) ? 0.f : exp2f(m_run[n2][hh] - mt);
+          alpha[n2][hh] = (m_run[n2][hh] == -INFINITY) ? 0.f : fast_exp2(m_run[n2][hh] - mt);
           m_run[n2][hh] = mt;
         }
       }
@@ -269,10 +278,10 @@ __global__ void __launch_bounds__(256)
       l_part[0] *= alpha[nb][0];
       l_part[1] *= alpha[nb][1];
       float p[4];
-      p[0] = (ma == -INFINITY) ? 0.f : exp2f(x[0] - ma);
-      p[1] = (mb2 == -INFINITY) ? 0.f : exp2f(x[1] - mb2);
-      p[2] = (ma == -INFINITY) ? 0.f : exp2f(x[2] - ma);
-      p[3] = (mb2 == -INFINITY) ? 0.f : exp2f(x[3] - mb2);
+      p[0] = (ma == -INFINITY) ? 0.f : fast_exp2(x[0] - ma);
+      p[1] = (mb2 == -INFINITY) ? 0.f : fast_exp2(x[1] - mb2);
+      p[2] = (ma == -INFINITY) ? 0.f : fast_exp2(x[2] - ma);
+      p[3] = (mb2 == -INFINITY) ? 0.f : fast_exp2(x[3] - mb2);
       l_part[0] += p[0] + p[2];
       l_part[1] += p[1] + p[3];
       uint32_t ht, lt, hb, lb;
@@ -368,74 +377,107 @@ __global__ void __launch_bounds__(256)
 }
 
 // ---------------------------------------------------------------------------
-// Up-projection: out[b,h,o] = sum_i o_lat[b,h,i] W_UV[h,o,i], i < d.
-// Per CTA one head and 16 outputs for 64 sequences: M = sequences,
-// N = outputs, K = d in chunks of 64 (o_lat split hi/lo bf16).
+// Split-K merge fused with the up-projection: out[b,h,o] = sum_i o_lat[b,h,i]
+// W_UV[h,o,i] with o_lat = merged latent output (LSE merge of the splits).
+// Per CTA one head and 16 sequences; 8 warps.  Phase 1 merges the 16 rows
+// (weights per split in shared memory, then many independent loads per
+// thread), writes o_lat split hi/lo bf16 to shared memory.  Phase 2: each
+// warp computes 16 sequences x 16 outputs, K = d, A by ldmatrix, B (W_UV
+// rows) read from global memory (it is shared by all sequence blocks, so it
+// stays in L2).
 template <int W>
-__global__ void __launch_bounds__(128)
-    mla_upv_kernel(const float *__restrict__ olat, const uint16_t *__restrict__ w_uv, int B,
-                   int H, int r, float *__restrict__ out) {
+__global__ void __launch_bounds__(256)
+    mla_merge_upv_kernel(const float *__restrict__ partial, int n_splits,
+                         const uint16_t *__restrict__ w_uv, int B, int H, int r,
+                         float *__restrict__ out) {
   constexpr int Dv = 128;
-  __shared__ __align__(16) uint16_t ah_s[64 * 64], al_s[64 * 64];  // [b][i] chunk
-  __shared__ __align__(16) uint16_t w_s[16 * 64];                   // [o][i] chunk
-  const int h = blockIdx.y, o0 = blockIdx.x * 16;
+  constexpr int OST = W + 8;  // padded o_lat row (bf16): conflict-free ldmatrix
+  __shared__ __align__(16) uint16_t oh_s[16 * OST], ol_s[16 * OST];
+  __shared__ float w_s[64 * 16];
+  __shared__ float linv_s[16];
+  const int h = blockIdx.x, b0 = blockIdx.y * 16;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c = lane & 3;
-  const int mat = lane >> 3, rr = lane & 7;
-  for (int b0 = 0; b0 < B; b0 += 64) {
-    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    for (int k0 = 0; k0 < W; k0 += 64) {
-      __syncthreads();
-      for (int q = tid; q < 64 * 32; q += 128) {  // 64 rows x 32 pairs
-        const int row = q / 32, pr = q % 32;
-        const int b = b0 + row;
-        float2 x = make_float2(0.f, 0.f);
-        if (b < B) x = *reinterpret_cast<const float2 *>(olat + ((size_t)b * H + h) * W + k0 + 2 * pr);
-        uint32_t hi, lo;
-        split2<true>(x.x, x.y, hi, lo);
-        const int u = pr / 4, wi = pr % 4;
-        reinterpret_cast<uint32_t *>(ah_s + row * 64 + 8 * swz8(row, u))[wi] = hi;
-        reinterpret_cast<uint32_t *>(al_s + row * 64 + 8 * swz8(row, u))[wi] = lo;
+  const size_t RS = (size_t)W + 2;
+  const size_t pstride = (size_t)B * H * RS;
+  if (tid < 16) {
+    const int b = b0 + tid;
+    float M = -INFINITY, L = 0.f;
+    if (b < B) {
+      const float *pr = partial + ((size_t)b * H + h) * RS;
+      for (int s = 0; s < n_splits; ++s) M = fmaxf(M, pr[s * pstride + W]);
+      for (int s = 0; s < n_splits; ++s) {
+        const float ms = pr[s * pstride + W];
+        const float wt = (ms == -INFINITY || M == -INFINITY) ? 0.f : exp2f(ms - M);
+        w_s[s * 16 + tid] = wt;
+        L += wt * pr[s * pstride + W + 1];
       }
-      for (int q = tid; q < 16 * 8; q += 128) {
-        const int o = q / 8, u = q % 8;
-        const uint4 x = *reinterpret_cast<const uint4 *>(w_uv + ((size_t)h * Dv + o0 + o) * r + k0 + 8 * u);
-        *reinterpret_cast<uint4 *>(w_s + o * 64 + 8 * swz8(o, u)) = x;
-      }
-      __syncthreads();
-#pragma unroll
-      for (int ks = 0; ks < 4; ++ks) {
-        const int row = 16 * warp + rr + ((mat & 1) ? 8 : 0);
-        const int ch = 2 * ks + (mat >> 1);
-        uint32_t a0, a1, a2, a3, l0, l1, l2, l3;
-        ldmatrix_x4(a0, a1, a2, a3, ah_s + row * 64 + 8 * swz8(row, ch));
-        ldmatrix_x4(l0, l1, l2, l3, al_s + row * 64 + 8 * swz8(row, ch));
-        uint32_t b0, b1, b2, b3;  // n-blocks 0 and 1 (outputs o0..o0+15)
-        const int orow = rr + ((mat >> 1) ? 8 : 0);
-        ldmatrix_x4(b0, b1, b2, b3, w_s + orow * 64 + 8 * swz8(orow, 2 * ks + (mat & 1)));
-        mma_bf16(acc[0], a0, a1, a2, a3, b0, b1);
-        mma_bf16(acc[0], l0, l1, l2, l3, b0, b1);
-        mma_bf16(acc[1], a0, a1, a2, a3, b2, b3);
-        mma_bf16(acc[1], l0, l1, l2, l3, b2, b3);
+    } else {
+      for (int s = 0; s < n_splits; ++s) w_s[s * 16 + tid] = 0.f;
+    }
+    linv_s[tid] = (L > 0.f) ? 1.f / L : 0.f;
+  }
+  __syncthreads();
+  for (int e = tid; e < 16 * (W / 2); e += 256) {
+    const int row = e / (W / 2), i = 2 * (e % (W / 2));
+    const int b = b0 + row;
+    float2 acc = make_float2(0.f, 0.f);
+    if (b < B) {
+      const float *pr = partial + ((size_t)b * H + h) * RS + i;
+#pragma unroll 8
+      for (int s = 0; s < n_splits; ++s) {
+        const float wt = w_s[s * 16 + row];
+        const float2 x = make_float2(pr[s * pstride], pr[s * pstride + 1]);
+        acc.x += wt * x.x;
+        acc.y += wt * x.y;
       }
     }
-#pragma unroll
-    for (int n = 0; n < 2; ++n)
-#pragma unroll
-      for (int hr = 0; hr < 2; ++hr) {
-        const int b = b0 + 16 * warp + g + 8 * hr;
-        if (b < B) {
-          float *dst = out + ((size_t)b * H + h) * Dv + o0 + 8 * n + 2 * c;
-          dst[0] = acc[n][2 * hr];
-          dst[1] = acc[n][2 * hr + 1];
-        }
-      }
+    const float li = linv_s[row];
+    uint32_t hi, lo;
+    split2<true>(acc.x * li, acc.y * li, hi, lo);
+    *reinterpret_cast<uint32_t *>(oh_s + row * OST + i) = hi;
+    *reinterpret_cast<uint32_t *>(ol_s + row * OST + i) = lo;
   }
+  __syncthreads();
+  // phase 2: warp -> outputs [16 warp, 16 warp + 16) as two n-blocks
+  const int mat = lane >> 3, rr = lane & 7;
+  float acc[2][4] = {};
+  const uint16_t *wrow0 = w_uv + ((size_t)h * Dv + 16 * warp + g) * r;
+  const uint16_t *wrow1 = wrow0 + (size_t)8 * r;
+#pragma unroll 4
+  for (int ks = 0; ks < W / 16; ++ks) {
+    uint32_t a0, a1, a2, a3, l0, l1, l2, l3;
+    const int row = rr + ((mat & 1) ? 8 : 0);
+    const int col = 16 * ks + 8 * (mat >> 1);
+    ldmatrix_x4(a0, a1, a2, a3, oh_s + row * OST + col);
+    ldmatrix_x4(l0, l1, l2, l3, ol_s + row * OST + col);
+    const int k0 = 16 * ks + 2 * c;
+    const uint32_t b00 = *reinterpret_cast<const uint32_t *>(wrow0 + k0);
+    const uint32_t b01 = *reinterpret_cast<const uint32_t *>(wrow0 + k0 + 8);
+    const uint32_t b10 = *reinterpret_cast<const uint32_t *>(wrow1 + k0);
+    const uint32_t b11 = *reinterpret_cast<const uint32_t *>(wrow1 + k0 + 8);
+    mma_bf16(acc[0], a0, a1, a2, a3, b00, b01);
+    mma_bf16(acc[0], l0, l1, l2, l3, b00, b01);
+    mma_bf16(acc[1], a0, a1, a2, a3, b10, b11);
+    mma_bf16(acc[1], l0, l1, l2, l3, b10, b11);
+  }
+#pragma unroll
+  for (int n = 0; n < 2; ++n)
+#pragma unroll
+    for (int hr = 0; hr < 2; ++hr) {
+      const int b = b0 + g + 8 * hr;
+      if (b < B) {
+        float *dst = out + ((size_t)b * H + h) * Dv + 16 * warp + 8 * n + 2 * c;
+        dst[0] = acc[n][2 * hr];
+        dst[1] = acc[n][2 * hr + 1];
+      }
+    }
 }
 
 template <int W>
 cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
   using C = MlaCfg<W>;
+  if (a.n_splits > 64) return cudaErrorInvalidValue;  // merge weights hold 64 splits
   const int B = a.v.B;
   mla_absorb_kernel<W><<<dim3(W / 64, a.H), 128, 0, st>>>(
       static_cast<const uint16_t *>(a.q_nope), static_cast<const uint16_t *>(a.q_pe),
@@ -447,12 +489,12 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  k<<<dim3(a.n_splits, B), 256, C::SMEM, st>>>(a.v, a.qlat, a.H, a.sig_log2, a.items_per_split,
+  k<<<dim3(a.n_splits, B), 256, C::SMEM, st>>>(a.v, a.qlat,
+                                                static_cast<const uint16_t *>(a.q_pe), a.H,
+                                                a.sig_log2, a.items_per_split,
                                                 a.n_splits, a.partial, a.err);
-  cudaError_t e = launch_splitk_merge(a.partial, a.n_splits, B * a.H, W, a.olat, st);
-  if (e != cudaSuccess) return e;
-  mla_upv_kernel<W><<<dim3(128 / 16, a.H), 128, 0, st>>>(
-      a.olat, static_cast<const uint16_t *>(a.w_uv), B, a.H, a.r, a.out);
+  mla_merge_upv_kernel<W><<<dim3(a.H, (B + 15) / 16), 256, 0, st>>>(
+      a.partial, a.n_splits, static_cast<const uint16_t *>(a.w_uv), B, a.H, a.r, a.out);
   return cudaGetLastError();
 }
 
