@@ -224,6 +224,92 @@ def run_reference(args):
 
 
 # ---------------------------------------------------------------------------
+def _layer_kind(w, l, src):
+    if w.kind == "mla":
+        return f"mla_d{w.layers[l]['width']}"
+    a = src[l]
+    return "bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}"
+
+
+def kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer, src, layer_call, dev,
+                     splitk_reduce, reps=5):
+    """Per-layer decode-kernel durations (ms) grouped by kind, with the
+    algorithmic bytes of each layer: ``{kind: [(ms, bytes), ...]}``."""
+    import torch
+    L = w.n_layers
+    parts = {}
+    if w.kind == "gqa":
+        for l in range(L):
+            if splits[l] > 1:
+                parts[l] = torch.empty((splits[l], w.batch * w.n_q_heads, w.head_dim + 2),
+                                       device=dev)
+
+    def run_layer(l):
+        if w.kind == "mla":
+            layer_call(l)  # the whole MLA call (4 launches)
+        elif splits[l] > 1:
+            cache.decode_partial(l, qs[l], w.sigma, splits[l], partials=parts[l])
+        else:
+            cache.decode(l, qs[l], w.sigma, out=outs[l], n_splits=1)
+
+    def merge(l):
+        if w.kind == "gqa" and splits[l] > 1:
+            splitk_reduce(parts[l], out=outs[l].view(-1, w.head_dim))
+
+    kt = {}
+    try:
+        evs = [(torch.cuda.Event(enable_timing=True, external=True),
+                torch.cuda.Event(enable_timing=True, external=True)) for _ in range(L)]
+
+        def tstep():
+            for l in range(L):
+                if l in new_kv:
+                    cache.append(l, *new_kv[l])
+                evs[l][0].record(stream)
+                run_layer(l)
+                evs[l][1].record(stream)
+                merge(l)
+            if w.append_per_step:
+                cache.rewind(1)
+
+        with torch.cuda.stream(stream):
+            tstep()
+            stream.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                tstep()
+            for r in range(reps + 1):
+                g.replay()
+                stream.synchronize()
+                if r == 0:
+                    continue
+                for l in range(L):
+                    kt.setdefault(_layer_kind(w, l, src), []).append(
+                        (evs[l][0].elapsed_time(evs[l][1]), per_layer[l]))
+        del g
+        return kt, "event nodes in a graph replay of the step"
+    except (TypeError, RuntimeError):
+        torch.cuda.synchronize()
+        kt = {}
+    with torch.cuda.stream(stream):
+        for l in range(L):
+            if l in new_kv:
+                cache.append(l, *new_kv[l])
+            for _ in range(reps):
+                s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                s0.record(stream)
+                run_layer(l)
+                s1.record(stream)
+                s1.synchronize()
+                kt.setdefault(_layer_kind(w, l, src), []).append((s0.elapsed_time(s1), per_layer[l]))
+            merge(l)
+        if w.append_per_step:
+            cache.rewind(1)
+        torch.cuda.synchronize()
+    return kt, "eager launches between events (includes host launch gaps)"
+
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -355,36 +441,15 @@ def main():
     value = job_throughput(step_bytes, args.steps, world, ms / 1e3)
 
     # ---- per-kernel durations (events on the launching stream) -------------
-    # decode kernel alone through kvk_decode_partial + kvk_splitk_reduce
+    # A replay of the same step, built from kvk_decode_partial + the split-K
+    # merge so that a pair of timing-event nodes brackets each layer's decode
+    # kernel inside the graph (no host launch gaps in the interval).  Falls
+    # back to eager launches bracketed by events where graph event nodes are
+    # not available.
     from paper_2609_37988_gb300.cache import splitk_reduce
-    kt = {}
-    reps = 5
-    with torch.cuda.stream(stream):
-        for l in range(w.n_layers):
-            a = src[l]
-            if w.kind == "mla":
-                kind = f"mla_d{w.layers[l]['width']}"
-            else:
-                kind = "bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}"
-            ns = splits[l]
-            if w.kind == "gqa":
-                part = torch.empty((max(ns, 2), w.batch * w.n_q_heads, w.head_dim + 2), device=dev)
-            if l in new_kv:
-                cache.append(l, *new_kv[l])
-            for r in range(reps):
-                s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                s0.record(stream)
-                if w.kind == "mla":
-                    layer_call(l)          # the whole MLA call (4 launches)
-                elif ns > 1:
-                    cache.decode_partial(l, qs[l], w.sigma, ns, partials=part)
-                else:
-                    cache.decode(l, qs[l], w.sigma, out=outs[l], n_splits=1)
-                s1.record(stream)
-                s1.synchronize()
-                kt.setdefault(kind, []).append((s0.elapsed_time(s1), per_layer[l]))
-        cache.rewind(1) if w.append_per_step else None
-        torch.cuda.synchronize()
+    kt, kernel_timing = kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer,
+                                         src, layer_call if w.kind == "mla" else None, dev,
+                                         splitk_reduce)
     hbm, peak_kind = peaks()
     totals = {k: sum(t for t, _ in v) for k, v in kt.items()}
     dom = max(totals, key=totals.get)
@@ -476,6 +541,7 @@ def main():
                          "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
                          "peak_source": f"MEASURED_PEAKS.json hbm_gbs ({peak_kind})"},
             "kernels": kernels,
+            "kernel_timing": kernel_timing,
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": launches * args.steps,

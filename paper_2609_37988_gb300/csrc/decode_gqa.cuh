@@ -79,7 +79,8 @@ struct GqaCfg {
   static constexpr int QSTR = D + 4;  // padded query row (floats): conflict-free head rows
   static constexpr int Q_BYTES = 8 * QSTR * 4 + 2 * 8 * NG * 4;
   static constexpr int BAR_OFF = Q_BYTES + NST * STAGE;
-  static constexpr int SMEM = BAR_OFF + (TMA ? 8 * NST : 0);
+  static constexpr int GMASK_OFF = BAR_OFF + (TMA ? 8 * NST : 0);
+  static constexpr int SMEM = GMASK_OFF + (TMA ? 16 * NST : 0);
   static_assert(REC % 16 == 0, "records are 16-byte multiples");
   static_assert(!QUANT || (GS % 16 == 0 && D % GS == 0), "groups are whole k-steps");
   static_assert(4 * 8 * (D + 2) * 4 <= NST * STAGE, "merge scratch fits the stages");
@@ -118,7 +119,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c = lane & 3;
   const int len = v.lens[b];
-  const int n_items = a.gather ? min(v.kept_n[b], v.kept_cap) : len;
+  // kept-position lists exist only with per-token key metadata or bf16
+  // caches (rejected by the host for per-channel keys)
+  const bool gather = !C::KPC && a.gather;
+  const int n_items = gather ? min(v.kept_n[b], v.kept_cap) : len;
   const int i0 = split * a.items_per_split;
   // the last split runs to the end, so a launch recorded for shorter
   // sequences (a replayed graph) still covers every position
@@ -171,7 +175,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       const int item = base + crow + 8 * k;
       bool valid = item < i1;
       int pos = item;
-      if (a.gather && valid) {
+      if (gather && valid) {
         pos = kept[item];
         if (pos < 0 || pos >= len) {
           valid = false;
@@ -209,6 +213,16 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     }
     __syncthreads();
   }
+  // gather: kept position of row (TILE/4) warp + lane of the next tile to
+  // issue, and per stage one row-validity word per warp
+  uint32_t *gmask = reinterpret_cast<uint32_t *>(smem + C::GMASK_OFF);
+  int gidx_next = -1;
+  if constexpr (C::TMA) {
+    if (gather) {
+      const int r = i0 + (C::TILE / 4) * warp + lane;
+      gidx_next = (lane < C::TILE / 4 && r < i1) ? kept[r] : -1;
+    }
+  }
   auto zero_rows = [&](uint8_t *st, int r_lo, int r_hi) {  // rows [r_lo, r_hi), all threads
     uint4 *p = reinterpret_cast<uint4 *>(st + r_lo * C::REC);
     const int n = (r_hi - r_lo) * (C::REC / 16);
@@ -220,7 +234,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     const int nrows = min(C::TILE, i1 - base);
     int kgv = 0;  // complete key groups of this tile (per-channel keys)
     if constexpr (C::KPC) kgv = max(0, min(C::KG_ROWS, len / GS - base / GS));
-    if (!a.gather) {
+    if (!gather) {
       if (tid == 0) {
         fence_proxy_async();
         mbar_expect_tx(&bars[s], nrows * C::REC + kgv * D * 8);
@@ -230,38 +244,35 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       }
       if (nrows < C::TILE) zero_rows(st, nrows, C::TILE);
     } else {
-      if (warp == 0) {
-        constexpr int RPL = C::TILE / 32;  // rows per lane
-        int pos[RPL];
-        bool ok[RPL];
-#pragma unroll
-        for (int h = 0; h < RPL; ++h) {
-          const int row = lane + 32 * h;
-          ok[h] = row < nrows;
-          pos[h] = ok[h] ? kept[base + row] : 0;
-          if (ok[h] && (pos[h] < 0 || pos[h] >= len)) {
-            ok[h] = false;
-            set_err(a.err, 1);
-          }
-        }
-        int nvalid = 0;
-#pragma unroll
-        for (int h = 0; h < RPL; ++h) nvalid += __popc(__ballot_sync(0xffffffffu, ok[h]));
-        if (lane == 0) {
-          fence_proxy_async();
-          mbar_expect_tx(&bars[s], nvalid * C::REC);
-        }
-        __syncwarp();
-#pragma unroll
-        for (int h = 0; h < RPL; ++h) {
-          const int row = lane + 32 * h;
-          if (ok[h]) {
-            bulk_g2s(st + row * C::REC, rec + (size_t)pos[h] * C::REC, C::REC, &bars[s]);
-          } else {
-            uint4 *p = reinterpret_cast<uint4 *>(st + row * C::REC);
-#pragma unroll
-            for (int q = 0; q < C::REC / 16; ++q) p[q] = make_uint4(0, 0, 0, 0);
-          }
+      // gather: warp w copies rows [RPW w, RPW (w+1)) of the tile with
+      // 16-byte copies.  Lane l holds the kept position of row RPW w + l,
+      // loaded one tile ahead (gidx_next) so that its latency hides behind
+      // the current tile's arithmetic; the warp's row-validity bits go to
+      // the stage's mask words, read by the consumer instead of the list.
+      // Rows without a valid kept position are zero-filled by the copy.
+      constexpr int CPRR = C::REC / 16;  // 16-byte chunks per record
+      constexpr int RPW = C::TILE / 4;   // rows per warp (<= 32)
+      const int myidx = gidx_next;
+      {
+        const int nrow = base + C::TILE + RPW * warp + lane;  // same row, next tile
+        gidx_next = (lane < RPW && nrow < i1) ? kept[nrow] : -1;
+      }
+      bool mine = lane < RPW && RPW * warp + lane < nrows;
+      if (mine && (myidx < 0 || myidx >= len)) {
+        mine = false;
+        set_err(a.err, 1);
+      }
+      const uint32_t vm = __ballot_sync(0xffffffffu, mine);
+      if (lane == 0) gmask[s * 4 + warp] = vm;
+      uint8_t *wst = st + RPW * warp * C::REC;
+#pragma unroll 3
+      for (int q0 = 0; q0 < RPW * CPRR; q0 += 32) {
+        const int q = q0 + lane, j = q / CPRR, u = q - j * CPRR;
+        const int pos = __shfl_sync(0xffffffffu, myidx, j & 31);
+        if (q < RPW * CPRR) {
+          const bool valid = (vm >> (j & 31)) & 1u;
+          cp_async16(wst + j * C::REC + 16 * u, rec + (size_t)(valid ? pos : 0) * C::REC + 16 * u,
+                     valid);
         }
       }
     }
@@ -273,10 +284,11 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       issue_cp(t, s);
   };
 
+  const bool use_cp = !C::TMA || gather;  // completion by cp.async groups
 #pragma unroll
   for (int s = 0; s < C::NST - 1; ++s) {
     if (s < n_tiles) issue(s, s);
-    if constexpr (!C::TMA) cp_async_commit();
+    if (use_cp) cp_async_commit();
   }
 
   for (int e = tid; e < 8 * D; e += 128) {
@@ -428,32 +440,46 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       const int tA = r0 + g, tB = tA + 8;
       vA[rb] = base + tA < i1;
       vB[rb] = base + tB < i1;
-      if (a.gather) {
+      if constexpr (C::TMA) {
+        if (gather) {
+          constexpr int RPW = C::TILE / 4;
+          vA[rb] = (gmask[s * 4 + tA / RPW] >> (tA % RPW)) & 1u;
+          vB[rb] = (gmask[s * 4 + tB / RPW] >> (tB % RPW)) & 1u;
+        }
+      } else if (gather) {
         if (vA[rb]) { const int p = kept[base + tA]; vA[rb] = p >= 0 && p < len; }
         if (vB[rb]) { const int p = kept[base + tB]; vB[rb] = p >= 0 && p < len; }
       }
       s4[rb][0] = s4[rb][1] = s4[rb][2] = s4[rb][3] = 0.f;
       if (base + r0 >= i1) continue;
       if (C::KPC && base + r0 >= Tq) {
-        // open per-channel key group: bf16 rows of the residual plane, plain
-        // fp32 dot products (at most group-1 positions per sequence).
+        // open per-channel key group (at most group-1 positions): bf16 rows
+        // of the residual plane, stored in the bf16 K fragment order, read
+        // from global memory straight into A fragments; the query enters as
+        // bf16 hi + lo fragments, fp32 accumulation.
         const uint8_t *res = v.resid + slab * (size_t)GS * D * 2;
+        const uint8_t *rowA = res + (size_t)((base + tA) % GS) * D * 2;
+        const uint8_t *rowB = res + (size_t)((base + tB) % GS) * D * 2;
+        float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int tt = (k < 2 ? tA : tB);
-          const bool ok = (k < 2 ? vA[rb] : vB[rb]);
-          const int h = 2 * c + (k & 1);
-          float d = 0.f;
-          if (ok) {
-            const uint8_t *row = res + (size_t)((base + tt) % GS) * D * 2;
-            for (int ch = 0; ch < D; ++ch) {
-              int by, hi;
-              k_pos(ch, 16, D, &by, &hi);
-              d += q_s[h * QSTR + ch] * bf16_to_f32(*reinterpret_cast<const uint16_t *>(row + by));
-            }
+        for (int i = 0; i < D / 32; ++i) {
+          const uint4 z = make_uint4(0, 0, 0, 0);
+          const uint4 xa = vA[rb] ? *reinterpret_cast<const uint4 *>(rowA + 16 * (4 * i + c)) : z;
+          const uint4 xb = vB[rb] ? *reinterpret_cast<const uint4 *>(rowB + 16 * (4 * i + c)) : z;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const float *qh = q_s + g * QSTR + 16 * (2 * i + h);
+            uint32_t b0, b0l, b1, b1l;
+            split2<true>(qh[2 * c], qh[2 * c + 1], b0, b0l);
+            split2<true>(qh[2 * c + 8], qh[2 * c + 9], b1, b1l);
+            const uint32_t a0 = h ? xa.z : xa.x, a2 = h ? xa.w : xa.y;
+            const uint32_t a1 = h ? xb.z : xb.x, a3 = h ? xb.w : xb.y;
+            mma_bf16(d, a0, a1, a2, a3, b0, b1);
+            mma_bf16(d, a0, a1, a2, a3, b0l, b1l);
           }
-          s4[rb][k] = d;
         }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) s4[rb][k] = d[k];
       } else if constexpr (C::KPC) {
         // scale of each channel folded into the query for this group of
         // positions; zero point and 1024-bias enter as one per-head constant.
@@ -704,10 +730,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   int t_stop = n_tiles;  // first tile not consumed
   for (int t = 0; t < n_tiles; ++t) {
     bool ok = true;
-    if constexpr (C::TMA)
-      ok = mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22);
-    else
+    if (use_cp)
       cp_async_wait<C::NST - 2>();
+    else
+      ok = mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22);
     // every thread has finished tile t-1, and all agree whether a wait gave up
     if (__syncthreads_or(!ok)) {
       timed_out = true;
@@ -717,10 +743,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     }
     const int nt = t + C::NST - 1;
     if (nt < n_tiles) issue(nt, nt % C::NST);
-    if constexpr (!C::TMA) cp_async_commit();
+    if (use_cp) cp_async_commit();
     compute(t, t % C::NST);
   }
-  if constexpr (C::TMA) {
+  if (!use_cp) {
     if (timed_out) {
       // let copies still in flight land (bounded) before the CTA leaves:
       // tiles t_stop .. t_stop + NST - 2 were issued and not consumed

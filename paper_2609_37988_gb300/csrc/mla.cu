@@ -378,26 +378,33 @@ __global__ void __launch_bounds__(256)
 
 // ---------------------------------------------------------------------------
 // Split-K merge fused with the up-projection: out[b,h,o] = sum_i o_lat[b,h,i]
-// W_UV[h,o,i] with o_lat = merged latent output (LSE merge of the splits).
-// Per CTA one head and 16 sequences; 8 warps.  Phase 1 merges the 16 rows
-// (weights per split in shared memory, then many independent loads per
-// thread), writes o_lat split hi/lo bf16 to shared memory.  Phase 2: each
-// warp computes 16 sequences x 16 outputs, K = d, A by ldmatrix, B (W_UV
-// rows) read from global memory (it is shared by all sequence blocks, so it
-// stays in L2).
+// W_UV[h,o,i] with o_lat the LSE merge of the splits' partials.  Grid (head,
+// 16-sequence block, quarter of the 128 outputs); 4 warps.  The CTA's 32
+// W_UV rows are prefetched into shared memory (cp.async) while phase 1
+// merges the 16 rows into o_lat (split hi/lo bf16, shared memory); phase 2:
+// warp w computes 16 sequences x 8 outputs over K = d on the tensor cores.
 template <int W>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(128)
     mla_merge_upv_kernel(const float *__restrict__ partial, int n_splits,
                          const uint16_t *__restrict__ w_uv, int B, int H, int r,
                          float *__restrict__ out) {
   constexpr int Dv = 128;
-  constexpr int OST = W + 8;  // padded o_lat row (bf16): conflict-free ldmatrix
-  __shared__ __align__(16) uint16_t oh_s[16 * OST], ol_s[16 * OST];
-  __shared__ float w_s[64 * 16];
-  __shared__ float linv_s[16];
-  const int h = blockIdx.x, b0 = blockIdx.y * 16;
+  constexpr int OST = W + 8;  // padded rows (bf16): conflict-free ldmatrix
+  extern __shared__ __align__(128) uint8_t dyn_smem[];
+  uint16_t *oh_s = reinterpret_cast<uint16_t *>(dyn_smem);  // [16][OST]
+  uint16_t *ol_s = oh_s + 16 * OST;                         // [16][OST]
+  uint16_t *w_s = ol_s + 16 * OST;                          // [32][OST]
+  float *wt_s = reinterpret_cast<float *>(w_s + 32 * OST);  // [64][16]
+  float *linv_s = wt_s + 64 * 16;                           // [16]
+  const int h = blockIdx.x, b0 = blockIdx.y * 16, o0 = blockIdx.z * 32;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c = lane & 3;
+  // prefetch this CTA's 32 rows of W_UV[h][:, :W]
+  for (int q = tid; q < 32 * (W / 8); q += 128) {
+    const int o = q / (W / 8), u = q % (W / 8);
+    cp_async16(w_s + o * OST + 8 * u, w_uv + ((size_t)h * Dv + o0 + o) * r + 8 * u, true);
+  }
+  cp_async_commit();
   const size_t RS = (size_t)W + 2;
   const size_t pstride = (size_t)B * H * RS;
   if (tid < 16) {
@@ -409,25 +416,25 @@ __global__ void __launch_bounds__(256)
       for (int s = 0; s < n_splits; ++s) {
         const float ms = pr[s * pstride + W];
         const float wt = (ms == -INFINITY || M == -INFINITY) ? 0.f : exp2f(ms - M);
-        w_s[s * 16 + tid] = wt;
+        wt_s[s * 16 + tid] = wt;
         L += wt * pr[s * pstride + W + 1];
       }
     } else {
-      for (int s = 0; s < n_splits; ++s) w_s[s * 16 + tid] = 0.f;
+      for (int s = 0; s < n_splits; ++s) wt_s[s * 16 + tid] = 0.f;
     }
     linv_s[tid] = (L > 0.f) ? 1.f / L : 0.f;
   }
   __syncthreads();
-  for (int e = tid; e < 16 * (W / 2); e += 256) {
+  for (int e = tid; e < 16 * (W / 2); e += 128) {
     const int row = e / (W / 2), i = 2 * (e % (W / 2));
     const int b = b0 + row;
     float2 acc = make_float2(0.f, 0.f);
     if (b < B) {
       const float *pr = partial + ((size_t)b * H + h) * RS + i;
-#pragma unroll 8
+#pragma unroll 4
       for (int s = 0; s < n_splits; ++s) {
-        const float wt = w_s[s * 16 + row];
-        const float2 x = make_float2(pr[s * pstride], pr[s * pstride + 1]);
+        const float wt = wt_s[s * 16 + row];
+        const float2 x = *reinterpret_cast<const float2 *>(pr + s * pstride);
         acc.x += wt * x.x;
         acc.y += wt * x.y;
       }
@@ -438,40 +445,30 @@ __global__ void __launch_bounds__(256)
     *reinterpret_cast<uint32_t *>(oh_s + row * OST + i) = hi;
     *reinterpret_cast<uint32_t *>(ol_s + row * OST + i) = lo;
   }
+  cp_async_wait<0>();
   __syncthreads();
-  // phase 2: warp -> outputs [16 warp, 16 warp + 16) as two n-blocks
   const int mat = lane >> 3, rr = lane & 7;
-  float acc[2][4] = {};
-  const uint16_t *wrow0 = w_uv + ((size_t)h * Dv + 16 * warp + g) * r;
-  const uint16_t *wrow1 = wrow0 + (size_t)8 * r;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 4
   for (int ks = 0; ks < W / 16; ++ks) {
-    uint32_t a0, a1, a2, a3, l0, l1, l2, l3;
+    uint32_t a0, a1, a2, a3, l0, l1, l2, l3, b0r, b1r;
     const int row = rr + ((mat & 1) ? 8 : 0);
     const int col = 16 * ks + 8 * (mat >> 1);
     ldmatrix_x4(a0, a1, a2, a3, oh_s + row * OST + col);
     ldmatrix_x4(l0, l1, l2, l3, ol_s + row * OST + col);
-    const int k0 = 16 * ks + 2 * c;
-    const uint32_t b00 = *reinterpret_cast<const uint32_t *>(wrow0 + k0);
-    const uint32_t b01 = *reinterpret_cast<const uint32_t *>(wrow0 + k0 + 8);
-    const uint32_t b10 = *reinterpret_cast<const uint32_t *>(wrow1 + k0);
-    const uint32_t b11 = *reinterpret_cast<const uint32_t *>(wrow1 + k0 + 8);
-    mma_bf16(acc[0], a0, a1, a2, a3, b00, b01);
-    mma_bf16(acc[0], l0, l1, l2, l3, b00, b01);
-    mma_bf16(acc[1], a0, a1, a2, a3, b10, b11);
-    mma_bf16(acc[1], l0, l1, l2, l3, b10, b11);
+    ldmatrix_x2(b0r, b1r, w_s + (8 * warp + rr) * OST + 16 * ks + 8 * (mat & 1));
+    mma_bf16(acc, a0, a1, a2, a3, b0r, b1r);
+    mma_bf16(acc2, l0, l1, l2, l3, b0r, b1r);
   }
 #pragma unroll
-  for (int n = 0; n < 2; ++n)
-#pragma unroll
-    for (int hr = 0; hr < 2; ++hr) {
-      const int b = b0 + g + 8 * hr;
-      if (b < B) {
-        float *dst = out + ((size_t)b * H + h) * Dv + 16 * warp + 8 * n + 2 * c;
-        dst[0] = acc[n][2 * hr];
-        dst[1] = acc[n][2 * hr + 1];
-      }
+  for (int hr = 0; hr < 2; ++hr) {
+    const int b = b0 + g + 8 * hr;
+    if (b < B) {
+      float *dst = out + ((size_t)b * H + h) * Dv + o0 + 8 * warp + 2 * c;
+      dst[0] = acc[2 * hr] + acc2[2 * hr];
+      dst[1] = acc[2 * hr + 1] + acc2[2 * hr + 1];
     }
+  }
 }
 
 template <int W>
@@ -493,7 +490,15 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
                                                 static_cast<const uint16_t *>(a.q_pe), a.H,
                                                 a.sig_log2, a.items_per_split,
                                                 a.n_splits, a.partial, a.err);
-  mla_merge_upv_kernel<W><<<dim3(a.H, (B + 15) / 16), 256, 0, st>>>(
+  constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (64 * 16 + 16) * 4;
+  static bool mu_attr = false;
+  if (!mu_attr) {
+    cudaError_t e2 = cudaFuncSetAttribute(mla_merge_upv_kernel<W>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, MU_SMEM);
+    if (e2 != cudaSuccess) return e2;
+    mu_attr = true;
+  }
+  mla_merge_upv_kernel<W><<<dim3(a.H, (B + 15) / 16, 4), 128, MU_SMEM, st>>>(
       a.partial, a.n_splits, static_cast<const uint16_t *>(a.w_uv), B, a.H, a.r, a.out);
   return cudaGetLastError();
 }
