@@ -17,10 +17,11 @@
 //   scores  S^T[16 pos x 8 heads] = K[16 x 16 ch] * Q^T, the G <= 8 query
 //           heads of the KV head share one read of every key byte;
 //   values  O^T[16 ch x 8 heads] += V^T[16 ch x 16 pos] * P^T.
-// Codes enter the MMA as exact f16 integers (the exponent-bias trick:
-// 0x6400 | c is the half 1024 + c).  Scale and zero stay fp32 and are
-// applied outside the MMA, so quantised operands lose nothing:
-//   keys, per-token groups:   s_t = sum_g sc_tg (D'_tg - Qoff_g) + z_tg Qs_g
+// Codes enter the MMA as exact f16 subnormals (the bit pattern c is the
+// half c * 2^-24; the factor 2^-24 is undone on the fp32 side).  Scale and
+// zero stay fp32 and are applied outside the MMA, so quantised operands lose
+// nothing:
+//   keys, per-token groups:   s_t = sum_g sc_tg D_tg + z_tg Qs_g
 //   keys, per-channel groups: scale folded into the query per group of
 //                             positions, zero term  sum_i q_i z_Gi
 //   values: P'_g = p * sc_tg per channel group (hi/lo f16 split), plus
@@ -93,13 +94,20 @@ __device__ __forceinline__ int vswz(int mode, int t, int u) {
   return u;
 }
 
-// f16 pair (1024 + lo, 1024 + hi) from two bytes picked by `sel` (PRMT).
+// Codes as f16 operands: a code c placed in the low bits of a zero f16 bit
+// pattern is the subnormal c * 2^-24, exact, and the tensor cores multiply
+// it exactly into fp32.  Every code-side product therefore carries a factor
+// 2^-24, undone once on the fp32 side (kCodeScale).
+constexpr float kCodeUnit = 5.9604644775390625e-8f;  // 2^-24
+constexpr float kCodeScale = 16777216.f;            // 2^24
+// f16 pair (c_lo, c_hi) * 2^-24 from two bytes picked by `sel` (PRMT; the
+// selector's other nibbles pick zero bytes).
 __device__ __forceinline__ uint32_t u8pair_f16(uint32_t x, uint32_t sel) {
-  return __byte_perm(x, 0x64646464u, sel);
+  return __byte_perm(x, 0u, sel);
 }
-__device__ __forceinline__ uint32_t nib_f16(uint32_t x, uint32_t mask) {
-  return (x & mask) | 0x64006400u;
-}
+// f16 pair of the nibbles under `mask` (low nibble: c * 2^-24, high nibble:
+// 16 c * 2^-24).
+__device__ __forceinline__ uint32_t nib_f16(uint32_t x, uint32_t mask) { return x & mask; }
 
 template <int BITS, int D, int KAX, int GS>
 __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
@@ -111,7 +119,6 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   constexpr int QSTR = C::QSTR;
   float *q_s = reinterpret_cast<float *>(smem);        // [8][QSTR]
   float *qs_s = q_s + 8 * QSTR;                        // [8][NG] query sums per group
-  float *qo_s = qs_s + 8 * NG;                         // [8][NG] 1024-bias offsets
   uint8_t *stages = smem + C::Q_BYTES;
 
   const GqaView &v = a.v;
@@ -302,15 +309,15 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     q_s[h * QSTR + ch] = x;
   }
   __syncthreads();
-  // per-token key groups: query sums Qs and 1024-bias offsets Qoff of every
-  // (head, channel group), with the f16 values the score MMA actually uses;
-  // 128 / (8 NG) lanes per (head, group), reduced with shuffles.
+  // per-token key groups: query sums Qs of every (head, channel group), of
+  // the f16 values the score MMA actually uses, times 2^-24 like the code
+  // products; 128 / (8 NG) lanes per (head, group), reduced with shuffles.
   if constexpr (C::KPT) {
     constexpr int ITEMS = 8 * NG, LPI = 128 / ITEMS, CPL = GS / LPI;
     const int item = tid / LPI, sub = tid % LPI;
     const int h = item / NG, gi = item % NG;
     const bool use_lo0 = a.q_f32 != 0;
-    float sq = 0.f, so = 0.f;
+    float sq = 0.f;
 #pragma unroll 4
     for (int k = 0; k < CPL; ++k) {
       const int ch = gi * GS + sub * CPL + k;
@@ -320,14 +327,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       float xe = __half2float(__float2half_rn(xs));
       if (use_lo0) xe += __half2float(__float2half_rn(xs - xe));
       sq += hs ? 16.f * xe : xe;
-      so += 1024.f * xe;
     }
 #pragma unroll
-    for (int off = 1; off < LPI; off <<= 1) {
-      sq += __shfl_xor_sync(0xffffffffu, sq, off);
-      so += __shfl_xor_sync(0xffffffffu, so, off);
-    }
-    if (sub == 0) { qs_s[item] = sq; qo_s[item] = so; }
+    for (int off = 1; off < LPI; off <<= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+    if (sub == 0) qs_s[item] = sq * kCodeUnit;
     __syncthreads();
   }
 
@@ -343,21 +346,23 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       split2<BF>(x2, x3, qb[js][1], qbl[js][1]);
     }
   }
-  float qs[NG][2], qoff[NG][2];
+  float qs[NG][2];
   if constexpr (C::KPT) {
 #pragma unroll
     for (int gi = 0; gi < NG; ++gi)
 #pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        qs[gi][hh] = qs_s[(2 * c + hh) * NG + gi];
-        qoff[gi][hh] = qo_s[(2 * c + hh) * NG + gi];
-      }
+      for (int hh = 0; hh < 2; ++hh) qs[gi][hh] = qs_s[(2 * c + hh) * NG + gi];
   }
+  // scores of quantised caches come out times 2^-24
+  const float sig = a.sig_log2 * (C::QUANT ? kCodeScale : 1.f);
 
   float acc[KS][4];
 #pragma unroll
   for (int m = 0; m < KS; ++m) acc[m][0] = acc[m][1] = acc[m][2] = acc[m][3] = 0.f;
-  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  // running maxima start finite, so that 2^(x - m) needs no guard: masked
+  // scores are -inf and give 0, and the first live tile replaces the start
+  // value (its rescale factor 2^(-1e30 - m) is 0)
+  float m_run[2] = {-1e30f, -1e30f}, l_run[2] = {0.f, 0.f};
   float zacc[NG][2];
 #pragma unroll
   for (int gi = 0; gi < NG; ++gi) zacc[gi][0] = zacc[gi][1] = 0.f;
@@ -479,13 +484,13 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           }
         }
 #pragma unroll
-        for (int k = 0; k < 4; ++k) s4[rb][k] = d[k];
+        for (int k = 0; k < 4; ++k) s4[rb][k] = d[k] * kCodeUnit;  // scores carry 2^-24
       } else if constexpr (C::KPC) {
         // scale of each channel folded into the query for this group of
-        // positions; zero point and 1024-bias enter as one per-head constant.
+        // positions; the zero points enter as one per-head constant.
         const float2 *kg = kg_rows(st) + (r0 / GS) * D;
         uint32_t pb[KS][2], pbl[KS][2];
-        float zpart = 0.f, opart = 0.f;
+        float zpart = 0.f;
 #pragma unroll
         for (int js = 0; js < KS; ++js) {
           const float *qh = q_s + g * QSTR + 16 * js;
@@ -501,15 +506,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           }
           split2<false>(x[0], x[1], pb[js][0], pbl[js][0]);
           split2<false>(x[2], x[3], pb[js][1], pbl[js][1]);
-          const float2 h0 = unpack2<false>(pb[js][0]), l0 = unpack2<false>(pbl[js][0]);
-          const float2 h1 = unpack2<false>(pb[js][1]), l1 = unpack2<false>(pbl[js][1]);
-          opart += 1024.f * ((h0.x + l0.x) + (h0.y + l0.y) + (h1.x + l1.x) + (h1.y + l1.y));
         }
         zpart += __shfl_xor_sync(0xffffffffu, zpart, 1);
         zpart += __shfl_xor_sync(0xffffffffu, zpart, 2);
-        opart += __shfl_xor_sync(0xffffffffu, opart, 1);
-        opart += __shfl_xor_sync(0xffffffffu, opart, 2);
-        const float corr = zpart - opart;  // head g
+        const float corr = zpart * kCodeUnit;  // head g, in the 2^-24 units of the MMA
         const float corr0 = __shfl_sync(0xffffffffu, corr, (2 * c) * 4);
         const float corr1 = __shfl_sync(0xffffffffu, corr, (2 * c + 1) * 4);
         uint32_t wa[C::NWK], wb[C::NWK];
@@ -546,8 +546,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           constexpr int JPG = GS / 16;  // k-steps per group
 #pragma unroll
           for (int gi = 0; gi < NG; ++gi) {
-            // the accumulator starts at -Qoff, so it ends at D' - Qoff
-            float d[4] = {-qoff[gi][0], -qoff[gi][1], -qoff[gi][0], -qoff[gi][1]};
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int jj = 0; jj < JPG; ++jj) {
               const int js = gi * JPG + jj;
@@ -571,25 +570,27 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     float mt0 = -INFINITY, mt1 = -INFINITY;
 #pragma unroll
     for (int rb = 0; rb < RB; ++rb) {
-      p[rb][0] = vA[rb] ? s4[rb][0] * a.sig_log2 : -INFINITY;
-      p[rb][1] = vA[rb] ? s4[rb][1] * a.sig_log2 : -INFINITY;
-      p[rb][2] = vB[rb] ? s4[rb][2] * a.sig_log2 : -INFINITY;
-      p[rb][3] = vB[rb] ? s4[rb][3] * a.sig_log2 : -INFINITY;
+      p[rb][0] = vA[rb] ? s4[rb][0] * sig : -INFINITY;
+      p[rb][1] = vA[rb] ? s4[rb][1] * sig : -INFINITY;
+      p[rb][2] = vB[rb] ? s4[rb][2] * sig : -INFINITY;
+      p[rb][3] = vB[rb] ? s4[rb][3] * sig : -INFINITY;
       mt0 = fmaxf(mt0, fmaxf(p[rb][0], p[rb][2]));
       mt1 = fmaxf(mt1, fmaxf(p[rb][1], p[rb][3]));
     }
-#pragma unroll
-    for (int off = 4; off < 32; off <<= 1) {
-      mt0 = fmaxf(mt0, __shfl_xor_sync(0xffffffffu, mt0, off));
-      mt1 = fmaxf(mt1, __shfl_xor_sync(0xffffffffu, mt1, off));
-    }
-    // Keep a stale maximum while the tile stays within 2^8 of it: the
-    // result is exact either way, and rescaling is skipped on most tiles.
+    // Keep a stale maximum while every score of the tile stays within 2^8
+    // of it: the result is exact either way.  One vote decides; only tiles
+    // that raise some lane's maximum reduce it over the row lanes and
+    // rescale.
     const bool need = (mt0 > m_run[0] + 8.f) || (mt1 > m_run[1] + 8.f);
     if (__any_sync(0xffffffffu, need)) {
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+        mt0 = fmaxf(mt0, __shfl_xor_sync(0xffffffffu, mt0, off));
+        mt1 = fmaxf(mt1, __shfl_xor_sync(0xffffffffu, mt1, off));
+      }
       const float n0 = fmaxf(m_run[0], mt0), n1 = fmaxf(m_run[1], mt1);
-      const float al0 = (n0 == -INFINITY) ? 1.f : fast_exp2(m_run[0] - n0);
-      const float al1 = (n1 == -INFINITY) ? 1.f : fast_exp2(m_run[1] - n1);
+      const float al0 = fast_exp2(m_run[0] - n0);
+      const float al1 = fast_exp2(m_run[1] - n1);
 #pragma unroll
       for (int m = 0; m < KS; ++m) {
         acc[m][0] *= al0; acc[m][2] *= al0;
@@ -601,13 +602,12 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       m_run[0] = n0; m_run[1] = n1;
     }
     {
-      const bool live0 = m_run[0] != -INFINITY, live1 = m_run[1] != -INFINITY;
 #pragma unroll
       for (int rb = 0; rb < RB; ++rb) {
-        p[rb][0] = live0 ? fast_exp2(p[rb][0] - m_run[0]) : 0.f;
-        p[rb][1] = live1 ? fast_exp2(p[rb][1] - m_run[1]) : 0.f;
-        p[rb][2] = live0 ? fast_exp2(p[rb][2] - m_run[0]) : 0.f;
-        p[rb][3] = live1 ? fast_exp2(p[rb][3] - m_run[1]) : 0.f;
+        p[rb][0] = fast_exp2(p[rb][0] - m_run[0]);
+        p[rb][1] = fast_exp2(p[rb][1] - m_run[1]);
+        p[rb][2] = fast_exp2(p[rb][2] - m_run[0]);
+        p[rb][3] = fast_exp2(p[rb][3] - m_run[1]);
         l_run[0] += p[rb][0] + p[rb][2];
         l_run[1] += p[rb][1] + p[rb][3];
       }
@@ -674,7 +674,6 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           }
         }
       }
-      const uint32_t k1024 = 0x64006400u;
       uint32_t pf[RB][4];
 #pragma unroll
       for (int m = 0; m < KS; ++m) {
@@ -709,15 +708,15 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           } else {
             // word m/4: one byte per M-block (row g low nibble, row g+8 high
             // nibble -> 16x, undone at the end)
-            const int k = m >> 2, hh = (m >> 1) & 1, sh = 8 * (m & 1);
-            const uint32_t sel = hh ? 0x7632 : 0x5410;
-            const uint32_t X0 = __byte_perm(w[rb][0][k], w[rb][1][k], sel) >> sh;
-            const uint32_t X2 = __byte_perm(w[rb][2][k], w[rb][3][k], sel) >> sh;
+            // byte b0 = 2 hh + (m & 1) of each position's word, the first
+            // position's to byte 0 and the second's to byte 2
+            const int k = m >> 2, b0 = 2 * ((m >> 1) & 1) + (m & 1), b2 = 4 + b0;
+            const uint32_t sel = b0 | (b0 << 4) | (b2 << 8) | (b2 << 12);
+            const uint32_t X0 = __byte_perm(w[rb][0][k], w[rb][1][k], sel);
+            const uint32_t X2 = __byte_perm(w[rb][2][k], w[rb][3][k], sel);
             a0 = nib_f16(X0, 0x000F000Fu); a1 = nib_f16(X0, 0x00F000F0u);
             a2 = nib_f16(X2, 0x000F000Fu); a3 = nib_f16(X2, 0x00F000F0u);
           }
-          a0 = hsub2_u32(a0, k1024); a1 = hsub2_u32(a1, k1024);
-          a2 = hsub2_u32(a2, k1024); a3 = hsub2_u32(a3, k1024);
           mma_f16(acc[m], a0, a1, a2, a3, pf[rb][0], pf[rb][1]);
           mma_f16(acc[m], a0, a1, a2, a3, pf[rb][2], pf[rb][3]);
         }
@@ -775,10 +774,11 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   for (int m = 0; m < KS; ++m) {
     const int ch0 = 16 * m + g, ch1 = ch0 + 8;
     const int gi = C::QUANT ? (16 * m) / GS : 0;
-    const float hs = (BITS == 4) ? 0.0625f : 1.f;
+    constexpr float vsc = C::QUANT ? kCodeScale : 1.f;  // value codes carry 2^-24
+    constexpr float hs = (BITS == 4) ? 0.0625f * vsc : vsc;
     const float z0 = C::QUANT ? zacc[gi][0] : 0.f, z1 = C::QUANT ? zacc[gi][1] : 0.f;
-    red[(warp * 8 + 2 * c) * RS + ch0] = acc[m][0] + z0;
-    red[(warp * 8 + 2 * c + 1) * RS + ch0] = acc[m][1] + z1;
+    red[(warp * 8 + 2 * c) * RS + ch0] = acc[m][0] * vsc + z0;
+    red[(warp * 8 + 2 * c + 1) * RS + ch0] = acc[m][1] * vsc + z1;
     red[(warp * 8 + 2 * c) * RS + ch1] = acc[m][2] * hs + z0;
     red[(warp * 8 + 2 * c + 1) * RS + ch1] = acc[m][3] * hs + z1;
   }
@@ -812,7 +812,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       } else {
         float *pr = a.partial + ((size_t)split * gridDim.z * a.Hq + row0 + h) * RS;
         pr[ch] = A;
-        if (ch == 0) { pr[D] = M; pr[D + 1] = L; }
+        if (ch == 0) { pr[D] = (L > 0.f) ? M : -INFINITY; pr[D + 1] = L; }
       }
     }
   }
