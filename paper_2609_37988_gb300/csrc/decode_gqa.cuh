@@ -544,8 +544,13 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           const float2 *kmA = km_row(st, tA);
           const float2 *kmB = km_row(st, tB);
           constexpr int JPG = GS / 16;  // k-steps per group
+          float4 qA, qB;  // (scale, zero) of groups 2j and 2j + 1: one 16-byte load
 #pragma unroll
           for (int gi = 0; gi < NG; ++gi) {
+            if ((gi & 1) == 0) {
+              qA = reinterpret_cast<const float4 *>(kmA)[gi >> 1];
+              qB = reinterpret_cast<const float4 *>(kmB)[gi >> 1];
+            }
             float d[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int jj = 0; jj < JPG; ++jj) {
@@ -555,7 +560,8 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
               mma_f16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
               if (use_lo) mma_f16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
             }
-            const float2 mA = kmA[gi], mB = kmB[gi];
+            const float2 mA = (gi & 1) ? make_float2(qA.z, qA.w) : make_float2(qA.x, qA.y);
+            const float2 mB = (gi & 1) ? make_float2(qB.z, qB.w) : make_float2(qB.x, qB.y);
             s4[rb][0] = fmaf(mA.x, d[0], fmaf(mA.y, qs[gi][0], s4[rb][0]));
             s4[rb][1] = fmaf(mA.x, d[1], fmaf(mA.y, qs[gi][1], s4[rb][1]));
             s4[rb][2] = fmaf(mB.x, d[2], fmaf(mB.y, qs[gi][0], s4[rb][2]));
@@ -675,6 +681,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
         }
       }
       uint32_t pf[RB][4];
+      float4 vA4[RB], vB4[RB];  // (scale, zero) of groups 2j, 2j + 1 of rows g, g + 8
 #pragma unroll
       for (int m = 0; m < KS; ++m) {
         const int gi = (16 * m) / GS;
@@ -684,7 +691,14 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
 #pragma unroll
           for (int rb = 0; rb < RB; ++rb) {
             const int tA = wr0 + 16 * rb + g;
-            const float2 mA = vm_row(st, tA)[gi], mB = vm_row(st, tA + 8)[gi];
+            if ((gi & 1) == 0) {
+              vA4[rb] = reinterpret_cast<const float4 *>(vm_row(st, tA))[gi >> 1];
+              vB4[rb] = reinterpret_cast<const float4 *>(vm_row(st, tA + 8))[gi >> 1];
+            }
+            const float2 mA = (gi & 1) ? make_float2(vA4[rb].z, vA4[rb].w)
+                                       : make_float2(vA4[rb].x, vA4[rb].y);
+            const float2 mB = (gi & 1) ? make_float2(vB4[rb].z, vB4[rb].w)
+                                       : make_float2(vB4[rb].x, vB4[rb].y);
             uint32_t ht, lt, hb, lb;
             split2<false>(p[rb][0] * mA.x, p[rb][1] * mA.x, ht, lt);
             split2<false>(p[rb][2] * mB.x, p[rb][3] * mB.x, hb, lb);
