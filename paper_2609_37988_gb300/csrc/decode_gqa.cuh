@@ -76,12 +76,14 @@ struct GqaCfg {
   static constexpr int STAGE = TMA ? KG_OFF_T + KG_ROWS * D * 8 : KG_OFF + KG_ROWS * D * 8;
   static constexpr int NST = TMA ? (STAGE <= 13312 ? 4 : (STAGE <= 20480 ? 3 : 2)) : 2;
   static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");
-  static constexpr int MIN_CTAS = (BF || NST != 4) ? 3 : 4;
   static constexpr int QSTR = D + 4;  // padded query row (floats): conflict-free head rows
   static constexpr int Q_BYTES = 8 * QSTR * 4 + 2 * 8 * NG * 4;
   static constexpr int BAR_OFF = Q_BYTES + NST * STAGE;
   static constexpr int GMASK_OFF = BAR_OFF + (TMA ? 8 * NST : 0);
   static constexpr int SMEM = GMASK_OFF + (TMA ? 16 * NST : 0);
+  // CTAs per SM the register budget is sized for: four where four fit in
+  // shared memory (228 KB per SM, 1 KB reserved per CTA), else three
+  static constexpr int MIN_CTAS = (!BF && 4 * (SMEM + 1024) <= 233472) ? 4 : 3;
   static_assert(REC % 16 == 0, "records are 16-byte multiples");
   static_assert(!QUANT || (GS % 16 == 0 && D % GS == 0), "groups are whole k-steps");
   static_assert(4 * 8 * (D + 2) * 4 <= NST * STAGE, "merge scratch fits the stages");
@@ -335,16 +337,32 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   }
 
   // ---- query fragments (B operand of the score MMA), head n = g ----------
-  uint32_t qb[KS][2], qbl[KS][2];
+  // Built once per CTA by warp 0 and kept in shared memory over the query
+  // rows (dead from here on): per k-step js, the 32 lanes' hi pairs at
+  // qf[64 js + lane] and lo pairs at qf[64 js + 32 + lane].
+  uint2 *qf = reinterpret_cast<uint2 *>(q_s);
   if constexpr (!C::KPC) {
+    static_assert(KS * 64 * 8 <= 8 * QSTR * 4, "query fragments fit the query rows");
+    uint32_t hb[KS][2], lb[KS][2];
+    if (warp == 0) {
 #pragma unroll
-    for (int js = 0; js < KS; ++js) {
-      const float *qh = q_s + g * QSTR + 16 * js;
-      float x2 = qh[2 * c + 8], x3 = qh[2 * c + 9];
-      if (BITS == 4) { x2 *= 0.0625f; x3 *= 0.0625f; }
-      split2<BF>(qh[2 * c], qh[2 * c + 1], qb[js][0], qbl[js][0]);
-      split2<BF>(x2, x3, qb[js][1], qbl[js][1]);
+      for (int js = 0; js < KS; ++js) {
+        const float *qh = q_s + g * QSTR + 16 * js;
+        float x2 = qh[2 * c + 8], x3 = qh[2 * c + 9];
+        if (BITS == 4) { x2 *= 0.0625f; x3 *= 0.0625f; }
+        split2<BF>(qh[2 * c], qh[2 * c + 1], hb[js][0], lb[js][0]);
+        split2<BF>(x2, x3, hb[js][1], lb[js][1]);
+      }
     }
+    __syncthreads();  // every read of the query rows is done
+    if (warp == 0) {
+#pragma unroll
+      for (int js = 0; js < KS; ++js) {
+        qf[64 * js + lane] = make_uint2(hb[js][0], hb[js][1]);
+        qf[64 * js + 32 + lane] = make_uint2(lb[js][0], lb[js][1]);
+      }
+    }
+    __syncthreads();
   }
   float qs[NG][2];
   if constexpr (C::KPT) {
@@ -535,8 +553,12 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           for (int js = 0; js < KS; ++js) {
             uint32_t a0, a1, a2, a3;
             kfrag(wa, wb, js, a0, a1, a2, a3);
-            mma_bf16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
-            if (use_lo) mma_bf16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
+            const uint2 qh = qf[64 * js + lane];
+            mma_bf16(d, a0, a1, a2, a3, qh.x, qh.y);
+            if (use_lo) {
+              const uint2 ql = qf[64 * js + 32 + lane];
+              mma_bf16(d, a0, a1, a2, a3, ql.x, ql.y);
+            }
           }
 #pragma unroll
           for (int k = 0; k < 4; ++k) s4[rb][k] = d[k];
@@ -557,8 +579,12 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
               const int js = gi * JPG + jj;
               uint32_t a0, a1, a2, a3;
               kfrag(wa, wb, js, a0, a1, a2, a3);
-              mma_f16(d, a0, a1, a2, a3, qb[js][0], qb[js][1]);
-              if (use_lo) mma_f16(d, a0, a1, a2, a3, qbl[js][0], qbl[js][1]);
+              const uint2 qh = qf[64 * js + lane];
+              mma_f16(d, a0, a1, a2, a3, qh.x, qh.y);
+              if (use_lo) {
+                const uint2 ql = qf[64 * js + 32 + lane];
+                mma_f16(d, a0, a1, a2, a3, ql.x, ql.y);
+              }
             }
             const float2 mA = (gi & 1) ? make_float2(qA.z, qA.w) : make_float2(qA.x, qA.y);
             const float2 mB = (gi & 1) ? make_float2(qB.z, qB.w) : make_float2(qB.x, qB.y);
