@@ -71,7 +71,7 @@ __device__ __forceinline__ void quant_lane(const float (&x)[E], int GS, int leve
 // so the global stores are whole 16-byte chunks.
 template <int D>
 __device__ void put_section(uint32_t *buf, int bits, bool is_k, const uint32_t (&val)[D / 32],
-                            int lane) {
+                            int t, int rec_bytes, int lane) {
   constexpr int E = D / 32;
   const int words = D * bits / 32;
   for (int w = lane; w < words; w += 32) buf[w] = 0;
@@ -83,7 +83,7 @@ __device__ void put_section(uint32_t *buf, int bits, bool is_k, const uint32_t (
     if (is_k)
       k_pos(ch, bits, D, &byte, &hi);
     else
-      v_pos(ch, bits, D, &byte, &hi);
+      v_pos(ch, bits, D, t, rec_bytes, &byte, &hi);
     uint32_t v = val[e];
     int shift = (byte & 3) * 8;
     if (bits == 4) shift += hi * 4;
@@ -135,7 +135,7 @@ __global__ void __launch_bounds__(128)
 #pragma unroll
           for (int e = 0; e < E; ++e) val[e] = f32_to_bf16_bits(xk[e]);
         }
-        put_section<D>(buf, kq ? v.bits : 16, true, val, lane);
+        put_section<D>(buf, kq ? v.bits : 16, true, val, t, L.rec, lane);
         const int kb = D * v.bits / 8;
         for (int q = lane; q < kb / 16; q += 32)
           reinterpret_cast<uint4 *>(rec + L.k_off)[q] = reinterpret_cast<uint4 *>(buf)[q];
@@ -154,7 +154,7 @@ __global__ void __launch_bounds__(128)
 #pragma unroll
           for (int e = 0; e < E; ++e) val[e] = f32_to_bf16_bits(xv[e]);
         }
-        put_section<D>(buf, v.bits, false, val, lane);
+        put_section<D>(buf, v.bits, false, val, t, L.rec, lane);
         const int vb = D * v.bits / 8;
         for (int q = lane; q < vb / 16; q += 32)
           reinterpret_cast<uint4 *>(rec + L.v_off)[q] = reinterpret_cast<uint4 *>(buf)[q];

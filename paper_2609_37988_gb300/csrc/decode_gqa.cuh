@@ -273,6 +273,9 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       }
       const uint32_t vm = __ballot_sync(0xffffffffu, mine);
       if (lane == 0) gmask[s * 4 + warp] = vm;
+      // value chunks are stored rotated by v_rot(position) and read rotated
+      // by v_rot(shared-memory row): chunk u of the record moves accordingly
+      constexpr int VC0 = C::KB / 16, NC = C::KB / 16;
       uint8_t *wst = st + RPW * warp * C::REC;
 #pragma unroll 3
       for (int q0 = 0; q0 < RPW * CPRR; q0 += 32) {
@@ -280,7 +283,11 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
         const int pos = __shfl_sync(0xffffffffu, myidx, j & 31);
         if (q < RPW * CPRR) {
           const bool valid = (vm >> (j & 31)) & 1u;
-          cp_async16(wst + j * C::REC + 16 * u, rec + (size_t)(valid ? pos : 0) * C::REC + 16 * u,
+          int ud = u;
+          if (u >= VC0 && u < VC0 + NC)
+            ud = VC0 + ((u - VC0 - v_rot(pos, C::REC, NC) + v_rot(RPW * warp + j, C::REC, NC)) &
+                        (NC - 1));
+          cp_async16(wst + j * C::REC + 16 * ud, rec + (size_t)(valid ? pos : 0) * C::REC + 16 * u,
                      valid);
         }
       }
@@ -398,10 +405,6 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     const int u = g * (C::SV / 16) + k;
     if constexpr (C::TMA) return st + t * C::REC + C::KB + 16 * u;
     else return st + C::VP_OFF + t * C::VSTR + 16 * vswz(C::VSWZ, t, u);
-  };
-  auto v_small = [&](const uint8_t *st, int t) -> const uint8_t * {  // lane segment < 16 B
-    if constexpr (C::TMA) return st + t * C::REC + C::KB + C::SV * g;
-    else return st + C::VP_OFF + t * C::VSTR + C::SV * g;
   };
   auto km_row = [&](const uint8_t *st, int t) -> const float2 * {
     if constexpr (C::TMA) return reinterpret_cast<const float2 *>(st + t * C::REC + 2 * C::KB);
@@ -683,27 +686,24 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
         }
       }
     } else {
-      // lane g's value words of the 4 positions of each row block
-      uint32_t w[RB][4][C::NWV];
+      // Value codes by ldmatrix.trans: matrix (j, k) is chunk k of the 8
+      // positions 16 rb + 8 j + i of the row block; lane (g, c) receives
+      // element g of positions 2c and 2c+1, i.e. its bytes of M-blocks
+      // (2k, 2k+1) (4-bit) or of M-block k (8-bit) for both positions.
+      // Chunks are stored rotated by v_rot(position) (conflict-free rows).
+      constexpr int NC = C::KB / 16;  // value chunks per record
+      uint32_t vw[RB][2 * NC];        // [rb][NC j + k]
 #pragma unroll
       for (int rb = 0; rb < RB; ++rb) {
-        const int T0 = wr0 + 16 * rb + 2 * c;
-        const int Ts[4] = {T0, T0 + 1, T0 + 8, T0 + 9};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          if constexpr (C::SV >= 16) {
-#pragma unroll
-            for (int k = 0; k < C::SV / 16; ++k) {
-              const uint4 x = *reinterpret_cast<const uint4 *>(v_chunk(st, Ts[i], k));
-              w[rb][i][4 * k] = x.x; w[rb][i][4 * k + 1] = x.y;
-              w[rb][i][4 * k + 2] = x.z; w[rb][i][4 * k + 3] = x.w;
-            }
-          } else if constexpr (C::SV == 8) {
-            const uint2 x = *reinterpret_cast<const uint2 *>(v_small(st, Ts[i]));
-            w[rb][i][0] = x.x; w[rb][i][1] = x.y;
-          } else {
-            w[rb][i][0] = *reinterpret_cast<const uint32_t *>(v_small(st, Ts[i]));
-          }
+        for (int q = 0; q < NC / 2; ++q) {
+          const int mi = 4 * q + (lane >> 3);  // this lane addresses matrix mi
+          const int j = mi / NC, k = mi % NC;
+          const int t = wr0 + 16 * rb + 8 * j + (lane & 7);
+          const uint8_t *src =
+              st + t * C::REC + C::KB + 16 * ((k + v_rot(t, C::REC, NC)) & (NC - 1));
+          ldmatrix_x4_t(vw[rb][4 * q], vw[rb][4 * q + 1], vw[rb][4 * q + 2], vw[rb][4 * q + 3],
+                        src);
         }
       }
       uint32_t pf[RB][4];
@@ -738,22 +738,15 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
         for (int rb = 0; rb < RB; ++rb) {
           uint32_t a0, a1, a2, a3;
           if constexpr (BITS == 8) {
-            // word m/2 of a segment: M-block m in bytes (0,1) or (2,3)
-            const int k = m >> 1;
-            const uint32_t sel = (m & 1) ? 0x7362 : 0x5140;
-            const uint32_t X0 = __byte_perm(w[rb][0][k], w[rb][1][k], sel);
-            const uint32_t X2 = __byte_perm(w[rb][2][k], w[rb][3][k], sel);
-            a0 = u8pair_f16(X0, 0x4140); a1 = u8pair_f16(X0, 0x4342);
-            a2 = u8pair_f16(X2, 0x4140); a3 = u8pair_f16(X2, 0x4342);
+            // bytes (row g, row g+8) of the two positions: (0, 2) and (1, 3)
+            const uint32_t X0 = vw[rb][m], X2 = vw[rb][NC + m];
+            a0 = u8pair_f16(X0, 0x4240); a1 = u8pair_f16(X0, 0x4341);
+            a2 = u8pair_f16(X2, 0x4240); a3 = u8pair_f16(X2, 0x4341);
           } else {
-            // word m/4: one byte per M-block (row g low nibble, row g+8 high
-            // nibble -> 16x, undone at the end)
-            // byte b0 = 2 hh + (m & 1) of each position's word, the first
-            // position's to byte 0 and the second's to byte 2
-            const int k = m >> 2, b0 = 2 * ((m >> 1) & 1) + (m & 1), b2 = 4 + b0;
-            const uint32_t sel = b0 | (b0 << 4) | (b2 << 8) | (b2 << 12);
-            const uint32_t X0 = __byte_perm(w[rb][0][k], w[rb][1][k], sel);
-            const uint32_t X2 = __byte_perm(w[rb][2][k], w[rb][3][k], sel);
+            // bytes 0 and 2 (even m) or 1 and 3 (odd m): row g in the low
+            // nibble, row g+8 in the high nibble (16x, undone at the end)
+            const int sh = 8 * (m & 1);
+            const uint32_t X0 = vw[rb][m >> 1] >> sh, X2 = vw[rb][NC + (m >> 1)] >> sh;
             a0 = nib_f16(X0, 0x000F000Fu); a1 = nib_f16(X0, 0x00F000F0u);
             a2 = nib_f16(X2, 0x000F000Fu); a3 = nib_f16(X2, 0x00F000F0u);
           }

@@ -28,7 +28,7 @@ __global__ void gqa_export_kernel(const GqaView v, uint8_t *k_out, uint8_t *v_ou
       if (!dst) continue;
       int byte, hi;
       if (kv)
-        v_pos(ch, v.bits, D, &byte, &hi);
+        v_pos(ch, v.bits, D, t, L.rec, &byte, &hi);
       else
         k_pos(ch, v.bits, D, &byte, &hi);
       const uint8_t *sec = rec + (kv ? L.v_off : L.k_off);

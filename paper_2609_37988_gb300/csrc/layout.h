@@ -33,10 +33,16 @@
 //      k-steps (2w, 2w+1) with nibbles ordered so that masking with
 //      0x000F000F / 0x00F000F0 (and again after >> 8) yields the f16 pairs of
 //      the a0 / a2 registers directly.
-//   V: channel ch -> M-block m = ch/16, row rr = ch%16, lane row g = rr%8,
-//      e = rr/8; lane g's segment (head_dim/8 elements) holds (m, e) at
-//      element 2m + e.  For 4-bit values byte m of lane g's segment holds row
-//      g in the low nibble and row g+8 in the high nibble.
+//   V, bf16: channel ch -> M-block m = ch/16, row rr = ch%16, lane row
+//      g = rr%8, e = rr/8; lane g's segment (head_dim/8 elements) holds
+//      (m, e) at element 2m + e.
+//   V, codes: laid out for ldmatrix.trans over 8 positions x 16 bytes: the
+//      16-bit element g of 16-byte chunk k is lane row g's pair of bytes for
+//      M-blocks (2k, 2k+1) (4-bit: byte 16k + 2g + (m%2) holds row g in the
+//      low nibble, row g+8 in the high nibble) or for M-block k (8-bit: byte
+//      16k + 2g + e).  The chunks of position t are rotated by v_rot(t), so
+//      that eight consecutive records' copies of one chunk fall in eight
+//      distinct 16-byte bank slots of shared memory.
 //
 // An MLA anchor stores [c[:width] | k^R] in bf16, natural order, one record
 // per (batch, position).
@@ -108,23 +114,34 @@ KVK_HD void k_pos(int ch, int bits, int D, int *byte, int *hi) {
   *byte = (seg >= 16) ? 16 * (4 * (bp >> 4) + c) + (bp & 15) : seg * c + bp;
 }
 
-// Position of channel `ch` inside the V section.
-KVK_HD void v_pos(int ch, int bits, int D, int *byte, int *hi) {
+// Chunk rotation of the V section of position t (records of rec_bytes, nc
+// 16-byte chunks, nc a power of two).  With R = rec_bytes / 16 the natural
+// bank slot of record t is R t mod 8: all distinct for odd R, period 4 for
+// R = 2 mod 4, period 2 for R = 4 mod 8, constant for R = 0 mod 8.
+KVK_HD int v_rot(int t, int rec_bytes, int nc) {
+  const int R = rec_bytes >> 4;
+  const int r = (R & 1) ? 0 : ((R & 3) == 2) ? (t >> 2) : ((R & 7) == 4) ? (t >> 1) : t;
+  return r & (nc - 1);
+}
+
+// Position of channel `ch` inside the V section of position t.
+KVK_HD void v_pos(int ch, int bits, int D, int t, int rec_bytes, int *byte, int *hi) {
   const int m = ch >> 4, rr = ch & 15;
   const int g = rr & 7, e = rr >> 3;
-  const int n = 2 * m + e;
-  const int seg = D * bits / 64;
-  int bp;
   *hi = 0;
   if (bits == 16) {
-    bp = 2 * n;
-  } else if (bits == 8) {
-    bp = n;
+    *byte = (D / 4) * g + 2 * (2 * m + e);
+    return;
+  }
+  int bl;  // logical byte
+  if (bits == 8) {
+    bl = 16 * m + 2 * g + e;
   } else {
-    bp = m;
+    bl = 16 * (m >> 1) + 2 * g + (m & 1);
     *hi = e;
   }
-  *byte = seg * g + bp;
+  const int nc = D * bits / 128;
+  *byte = 16 * (((bl >> 4) + v_rot(t, rec_bytes, nc)) & (nc - 1)) + (bl & 15);
 }
 
 KVK_HD int64_t align256(int64_t x) { return (x + 255) & ~(int64_t)255; }
