@@ -185,8 +185,9 @@ kvk_status kvk_set_kept(kvk_cache *cache, int32_t layer, const int32_t *idx,
  *   out[b,h,:] = sum_t softmax_t(scale * <q[b,h], k_t>) v_t
  * over the positions of sequence b (or its kept list), KV head h / G with
  * G = H_q / H_kv.  q: device [B, H_q, head_dim] in q_dtype; out: device
- * float [B, H_q, head_dim].  n_splits: context splits (0 = chosen from the
- * SM count), at most the max_splits given at creation. */
+ * float [B, H_q, head_dim].  softmax_scale: finite and > 0, else
+ * KVK_ERR_INVALID_ARG.  n_splits: context splits (0 = chosen from the SM
+ * count), at most the max_splits given at creation. */
 kvk_status kvk_decode_attention(kvk_cache *cache, int32_t layer, const void *q,
                                 int32_t q_dtype, float softmax_scale, float *out,
                                 int32_t n_splits, kvk_stream stream);
@@ -197,7 +198,7 @@ kvk_status kvk_decode_attention(kvk_cache *cache, int32_t layer, const void *q,
  *   out[b,h]  = W_UV[h][:, :d] sum_t softmax_t(s_t) c_t[:d]
  * q_nope device bf16 [B, H, head_dim]; q_pe device bf16 [B, H, rope_dim]
  * (post-RoPE); w_uk, w_uv device bf16 [H, head_dim, latent_dim]; out device
- * float [B, H, head_dim]. */
+ * float [B, H, head_dim].  softmax_scale: finite and > 0. */
 kvk_status kvk_decode_attention_mla(kvk_cache *cache, int32_t layer, const void *q_nope,
                                     const void *q_pe, const void *w_uk, const void *w_uv,
                                     float softmax_scale, float *out, int32_t n_splits,

@@ -111,7 +111,9 @@ __device__ __forceinline__ uint32_t u8pair_f16(uint32_t x, uint32_t sel) {
 // 16 c * 2^-24).
 __device__ __forceinline__ uint32_t nib_f16(uint32_t x, uint32_t mask) { return x & mask; }
 
-template <int BITS, int D, int KAX, int GS>
+// GATHER: the rows come from the anchor's kept-position list (compiled
+// separately so that the contiguous path carries none of its state).
+template <int BITS, int D, int KAX, int GS, bool GATHER>
 __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     gqa_decode_kernel(const GqaDecodeArgs a) {
   using C = GqaCfg<BITS, D, KAX, GS>;
@@ -130,7 +132,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   const int len = v.lens[b];
   // kept-position lists exist only with per-token key metadata or bf16
   // caches (rejected by the host for per-channel keys)
-  const bool gather = !C::KPC && a.gather;
+  constexpr bool gather = GATHER && !C::KPC;
   const int n_items = gather ? min(v.kept_n[b], v.kept_cap) : len;
   const int i0 = split * a.items_per_split;
   // the last split runs to the end, so a launch recorded for shorter
@@ -605,10 +607,12 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     float mt0 = -INFINITY, mt1 = -INFINITY;
 #pragma unroll
     for (int rb = 0; rb < RB; ++rb) {
-      p[rb][0] = vA[rb] ? s4[rb][0] * sig : -INFINITY;
-      p[rb][1] = vA[rb] ? s4[rb][1] * sig : -INFINITY;
-      p[rb][2] = vB[rb] ? s4[rb][2] * sig : -INFINITY;
-      p[rb][3] = vB[rb] ? s4[rb][3] * sig : -INFINITY;
+      // raw scores here; the scale (> 0, checked by the host) enters the
+      // maxima once and the exponent through one FMA
+      p[rb][0] = vA[rb] ? s4[rb][0] : -INFINITY;
+      p[rb][1] = vA[rb] ? s4[rb][1] : -INFINITY;
+      p[rb][2] = vB[rb] ? s4[rb][2] : -INFINITY;
+      p[rb][3] = vB[rb] ? s4[rb][3] : -INFINITY;
       mt0 = fmaxf(mt0, fmaxf(p[rb][0], p[rb][2]));
       mt1 = fmaxf(mt1, fmaxf(p[rb][1], p[rb][3]));
     }
@@ -616,6 +620,8 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     // of it: the result is exact either way.  One vote decides; only tiles
     // that raise some lane's maximum reduce it over the row lanes and
     // rescale.
+    mt0 *= sig;
+    mt1 *= sig;
     const bool need = (mt0 > m_run[0] + 8.f) || (mt1 > m_run[1] + 8.f);
     if (__any_sync(0xffffffffu, need)) {
 #pragma unroll
@@ -639,10 +645,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     {
 #pragma unroll
       for (int rb = 0; rb < RB; ++rb) {
-        p[rb][0] = fast_exp2(p[rb][0] - m_run[0]);
-        p[rb][1] = fast_exp2(p[rb][1] - m_run[1]);
-        p[rb][2] = fast_exp2(p[rb][2] - m_run[0]);
-        p[rb][3] = fast_exp2(p[rb][3] - m_run[1]);
+        p[rb][0] = fast_exp2(fmaf(p[rb][0], sig, -m_run[0]));
+        p[rb][1] = fast_exp2(fmaf(p[rb][1], sig, -m_run[1]));
+        p[rb][2] = fast_exp2(fmaf(p[rb][2], sig, -m_run[0]));
+        p[rb][3] = fast_exp2(fmaf(p[rb][3], sig, -m_run[1]));
         l_run[0] += p[rb][0] + p[rb][2];
         l_run[1] += p[rb][1] + p[rb][3];
       }
@@ -851,10 +857,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   }
 }
 
-template <int BITS, int D, int KAX, int GS>
-cudaError_t launch_gqa_decode_t(const GqaDecodeArgs &a, cudaStream_t st) {
+template <int BITS, int D, int KAX, int GS, bool GATHER>
+cudaError_t launch_gqa_decode_g(const GqaDecodeArgs &a, cudaStream_t st) {
   using C = GqaCfg<BITS, D, KAX, GS>;
-  auto k = gqa_decode_kernel<BITS, D, KAX, GS>;
+  auto k = gqa_decode_kernel<BITS, D, KAX, GS, GATHER>;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -867,6 +873,17 @@ cudaError_t launch_gqa_decode_t(const GqaDecodeArgs &a, cudaStream_t st) {
 }
 
 template <int BITS, int D, int KAX, int GS>
+cudaError_t launch_gqa_decode_t(const GqaDecodeArgs &a, cudaStream_t st) {
+  if constexpr (GqaCfg<BITS, D, KAX, GS>::KPC) {
+    if (a.gather) return cudaErrorInvalidValue;  // no kept lists with per-channel keys
+    return launch_gqa_decode_g<BITS, D, KAX, GS, false>(a, st);
+  } else {
+    return a.gather ? launch_gqa_decode_g<BITS, D, KAX, GS, true>(a, st)
+                    : launch_gqa_decode_g<BITS, D, KAX, GS, false>(a, st);
+  }
+}
+
+template <int BITS, int D, int KAX, int GS>
 int gqa_tile_t() {
   return GqaCfg<BITS, D, KAX, GS>::TILE;
 }
@@ -874,7 +891,7 @@ int gqa_tile_t() {
 template <int BITS, int D, int KAX, int GS>
 int gqa_ctas_per_sm_t() {
   using C = GqaCfg<BITS, D, KAX, GS>;
-  auto k = gqa_decode_kernel<BITS, D, KAX, GS>;
+  auto k = gqa_decode_kernel<BITS, D, KAX, GS, false>;
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   int n = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 128, C::SMEM) != cudaSuccess) n = 1;

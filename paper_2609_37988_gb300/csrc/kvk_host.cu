@@ -503,7 +503,8 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
     return fail(KVK_ERR_INVALID_ARG, "q_dtype must be F32 or BF16");
   if (n_splits < 0 || n_splits > c->max_splits)
     return fail(KVK_ERR_INVALID_ARG, "n_splits %d outside [0, %d]", n_splits, c->max_splits);
-  if (!std::isfinite(scale)) return fail(KVK_ERR_INVALID_ARG, "non-finite softmax scale");
+  if (!std::isfinite(scale) || !(scale > 0.f))
+    return fail(KVK_ERR_INVALID_ARG, "softmax scale must be finite and positive");
   const int a = c->src[layer];
   GqaDecodeArgs args;
   args.v = c->gqa_view(a);
@@ -621,6 +622,8 @@ kvk_status kvk_decode_attention_mla(kvk_cache *c, int32_t layer, const void *q_n
     return fail(KVK_ERR_INVALID_ARG, "null or misaligned MLA operand");
   if (n_splits < 0 || n_splits > c->max_splits)
     return fail(KVK_ERR_INVALID_ARG, "n_splits %d outside [0, %d]", n_splits, c->max_splits);
+  if (!std::isfinite(softmax_scale) || !(softmax_scale > 0.f))
+    return fail(KVK_ERR_INVALID_ARG, "softmax scale must be finite and positive");
   const int a = c->src[layer];
   MlaDecodeArgs args;
   args.v = c->mla_view(a);

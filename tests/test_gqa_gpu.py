@@ -128,6 +128,18 @@ def test_capacity_is_checked_on_the_host():
     assert c.lengths(0).cpu().tolist() == [90]
 
 
+def test_softmax_scale_must_be_positive():
+    from paper_2609_37988_gb300.cache import KVKError
+    c = _cache(1, 4, 1, 64, 64, [dict(bits=4, group=32)])
+    x = torch.zeros((1, 8, 1, 64), dtype=torch.bfloat16, device="cuda")
+    c.append(0, x, x)
+    q = torch.zeros((1, 4, 64), dtype=torch.bfloat16, device="cuda")
+    for bad in (0.0, -0.125, float("nan"), float("inf")):
+        with pytest.raises(KVKError, match="INVALID_ARG"):
+            c.decode(0, q, bad)
+    assert c.decode(0, q, 0.125).isfinite().all()
+
+
 @pytest.mark.parametrize("fmt", [dict(bits=4, group=32, key_axis="token"),
                                  dict(bits=8, group=64, key_axis="token"),
                                  dict(bits=16, group=64, key_axis="token")], ids=["int4", "int8", "bf16"])
