@@ -463,13 +463,17 @@ def main():
         b = sum(x for _, x in v) / len(v)
         kernels[k] = {"avg_us": round(d * 1e3, 2), "gbs": round(b / (d / 1e3) / 1e9, 1),
                       "frac": round(b / (d / 1e3) / 1e9 / hbm, 4)}
+    # DRAM bytes per launch of the dominant kernel from the committed ncu
+    # summary, used only while the decode sources still hash to the value
+    # recorded with it (null otherwise: the counters would be stale)
     traffic = None
     tf = os.path.join(ROOT, "profiles", "gqa_decode_traffic.json")
     if os.path.exists(tf):
         with open(tf) as f:
             tj = json.load(f)
-        if tj.get("kernel_kind") == dom and tj.get("source_hash") == _source_hash():
-            traffic = tj.get("bytes_per_launch_full")
+        ent = tj.get("kernels", {}).get(dom)
+        if ent and tj.get("source_hash") == _source_hash() and ent.get("workload") == w.name:
+            traffic = ent.get("bytes_per_launch")
 
     # ---- end to end through the public API, host buffers --------------------
     e2e = None
@@ -595,7 +599,7 @@ def _source_hash():
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2609_37988_gb300", "csrc")
     for n in sorted(os.listdir(d)):
-        if n.startswith("decode_gqa"):
+        if n.startswith("decode_gqa") or n in ("layout.h", "common.cuh", "kernels.h"):
             with open(os.path.join(d, n), "rb") as f:
                 h.update(f.read())
     return h.hexdigest()[:16]

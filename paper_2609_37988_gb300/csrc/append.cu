@@ -93,6 +93,65 @@ __device__ void put_section(uint32_t *buf, int bits, bool is_k, const uint32_t (
 }
 
 template <int D>
+__device__ __forceinline__ void load_row(const void *kin, const void *vin, int in_f32,
+                                         size_t ibase, int lane, float (&xk)[D / 32],
+                                         float (&xv)[D / 32]) {
+#pragma unroll
+  for (int e = 0; e < D / 32; ++e) {
+    xk[e] = load_in(kin, ibase + lane * (D / 32) + e, in_f32);
+    xv[e] = load_in(vin, ibase + lane * (D / 32) + e, in_f32);
+  }
+}
+
+// Quantises and writes one (sequence b, position t, KV head kvh) record from
+// the warp's inputs (lane holds channels [lane E, lane E + E)).
+template <int D>
+__device__ void append_row(const GqaView &v, const float (&xk)[D / 32], const float (&xv)[D / 32],
+                           int b, int kvh, int t, uint32_t *buf, int lane) {
+  constexpr int E = D / 32;
+  const RecLayout L = rec_layout(v.bits, D, v.group, v.key_axis);
+  uint8_t *rec = v.rec + (((size_t)b * v.Hkv + kvh) * v.cap + t) * L.rec;
+  const bool kq = v.bits != 16 && v.key_axis == 0;
+  const bool kres = v.bits != 16 && v.key_axis == 1;
+  // ---- K section ----
+  if (!kres) {
+    uint32_t val[E];
+    float sc = 0.f, zr = 0.f;
+    if (kq) {
+      quant_lane<E>(xk, v.group, (1 << v.bits) - 1, val, sc, zr);
+    } else {
+#pragma unroll
+      for (int e = 0; e < E; ++e) val[e] = f32_to_bf16_bits(xk[e]);
+    }
+    put_section<D>(buf, kq ? v.bits : 16, true, val, t, L.rec, lane);
+    const int kb = D * v.bits / 8;
+    for (int q = lane; q < kb / 16; q += 32)
+      reinterpret_cast<uint4 *>(rec + L.k_off)[q] = reinterpret_cast<uint4 *>(buf)[q];
+    if (kq && (lane * E) % v.group == 0)
+      reinterpret_cast<float2 *>(rec + L.km_off)[(lane * E) / v.group] = make_float2(sc, zr);
+    __syncwarp();
+  }
+  // ---- V section ----
+  {
+    uint32_t val[E];
+    float sc = 0.f, zr = 0.f;
+    const bool vq = v.bits != 16;
+    if (vq) {
+      quant_lane<E>(xv, v.group, (1 << v.bits) - 1, val, sc, zr);
+    } else {
+#pragma unroll
+      for (int e = 0; e < E; ++e) val[e] = f32_to_bf16_bits(xv[e]);
+    }
+    put_section<D>(buf, v.bits, false, val, t, L.rec, lane);
+    const int vb = D * v.bits / 8;
+    for (int q = lane; q < vb / 16; q += 32)
+      reinterpret_cast<uint4 *>(rec + L.v_off)[q] = reinterpret_cast<uint4 *>(buf)[q];
+    if (vq && (lane * E) % v.group == 0)
+      reinterpret_cast<float2 *>(rec + L.vm_off)[(lane * E) / v.group] = make_float2(sc, zr);
+  }
+}
+
+template <int D>
 __global__ void __launch_bounds__(128)
     gqa_append_rows(const GqaView v, const void *kin, const void *vin, int in_f32, int n_new,
                     const int32_t *n_per_seq, int32_t *err) {
@@ -113,54 +172,9 @@ __global__ void __launch_bounds__(128)
       ok = false;
     }
     if (ok) {
-      const size_t ibase = (((size_t)b * n_new + i) * v.Hkv + kvh) * D;
-      const RecLayout L = rec_layout(v.bits, D, v.group, v.key_axis);
-      uint8_t *rec = v.rec + (((size_t)b * v.Hkv + kvh) * v.cap + t) * L.rec;
-      uint32_t *buf = sbuf[warp];
       float xk[E], xv[E];
-#pragma unroll
-      for (int e = 0; e < E; ++e) {
-        xk[e] = load_in(kin, ibase + lane * E + e, in_f32);
-        xv[e] = load_in(vin, ibase + lane * E + e, in_f32);
-      }
-      const bool kq = v.bits != 16 && v.key_axis == 0;
-      const bool kres = v.bits != 16 && v.key_axis == 1;
-      // ---- K section ----
-      if (!kres) {
-        uint32_t val[E];
-        float sc = 0.f, zr = 0.f;
-        if (kq) {
-          quant_lane<E>(xk, v.group, (1 << v.bits) - 1, val, sc, zr);
-        } else {
-#pragma unroll
-          for (int e = 0; e < E; ++e) val[e] = f32_to_bf16_bits(xk[e]);
-        }
-        put_section<D>(buf, kq ? v.bits : 16, true, val, t, L.rec, lane);
-        const int kb = D * v.bits / 8;
-        for (int q = lane; q < kb / 16; q += 32)
-          reinterpret_cast<uint4 *>(rec + L.k_off)[q] = reinterpret_cast<uint4 *>(buf)[q];
-        if (kq && (lane * E) % v.group == 0)
-          reinterpret_cast<float2 *>(rec + L.km_off)[(lane * E) / v.group] = make_float2(sc, zr);
-        __syncwarp();
-      }
-      // ---- V section ----
-      {
-        uint32_t val[E];
-        float sc = 0.f, zr = 0.f;
-        const bool vq = v.bits != 16;
-        if (vq) {
-          quant_lane<E>(xv, v.group, (1 << v.bits) - 1, val, sc, zr);
-        } else {
-#pragma unroll
-          for (int e = 0; e < E; ++e) val[e] = f32_to_bf16_bits(xv[e]);
-        }
-        put_section<D>(buf, v.bits, false, val, t, L.rec, lane);
-        const int vb = D * v.bits / 8;
-        for (int q = lane; q < vb / 16; q += 32)
-          reinterpret_cast<uint4 *>(rec + L.v_off)[q] = reinterpret_cast<uint4 *>(buf)[q];
-        if (vq && (lane * E) % v.group == 0)
-          reinterpret_cast<float2 *>(rec + L.vm_off)[(lane * E) / v.group] = make_float2(sc, zr);
-      }
+      load_row<D>(kin, vin, in_f32, (((size_t)b * n_new + i) * v.Hkv + kvh) * D, lane, xk, xv);
+      append_row<D>(v, xk, xv, b, kvh, t, sbuf[warp], lane);
     }
   }
   // The last CTA advances the lengths (per-token layouts only; per-channel
@@ -181,6 +195,46 @@ __global__ void __launch_bounds__(128)
       if (threadIdx.x == 0) *v.counter = 0;
     }
   }
+}
+
+// Short appends (a decode step: n_new x H_kv <= 64 rows per sequence,
+// per-token layouts): one CTA of 8 warps per sequence.  The CTA reads the
+// length once while the warps' first input loads are in flight, writes all
+// rows of its sequence and then advances the length itself -- no other CTA
+// reads it, so no completion counter or fence is needed.
+template <int D>
+__global__ void __launch_bounds__(256)
+    gqa_append_seq(const GqaView v, const void *kin, const void *vin, int in_f32, int n_new,
+                   const int32_t *n_per_seq, int32_t *err) {
+  constexpr int E = D / 32;
+  __shared__ __align__(16) uint32_t sbuf[8][(2 * D * 2 + 2 * 64) / 4];
+  __shared__ int s_len, s_nb;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x;
+  const int rows = n_new * v.Hkv;
+  float xk[E], xv[E];
+  if (warp < rows)
+    load_row<D>(kin, vin, in_f32, ((size_t)b * n_new * v.Hkv + warp) * D, lane, xk, xv);
+  if (threadIdx.x == 0) {
+    s_nb = seq_count(n_per_seq, b, n_new, err);
+    s_len = v.lens[b];
+  }
+  __syncthreads();
+  const int len = s_len, nb = s_nb;
+  for (int r = warp; r < rows; r += 8) {
+    const int i = r / v.Hkv, kvh = r - i * v.Hkv;
+    if (r != warp)
+      load_row<D>(kin, vin, in_f32, ((size_t)b * n_new * v.Hkv + r) * D, lane, xk, xv);
+    if (i >= nb) continue;
+    const int t = len + i;
+    if (t >= v.cap) {
+      if (lane == 0) set_err(err, 2);
+      continue;
+    }
+    append_row<D>(v, xk, xv, b, kvh, t, sbuf[warp], lane);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) v.lens[b] = min((long long)len + nb, (long long)v.cap);
 }
 
 // Per-channel key groups completed by this append: one thread per
@@ -342,10 +396,16 @@ cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, i
     else
       gqa_append_kgroups<64><<<(unsigned)((thr + 127) / 128), 128, 0, st>>>(v, k, in_f32, n_new, n_per_seq, err, max_groups);
   }
-  if (v.D == 128)
+  if (!kpc && (size_t)n_new * v.Hkv <= 64) {
+    if (v.D == 128)
+      gqa_append_seq<128><<<v.B, 256, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
+    else
+      gqa_append_seq<64><<<v.B, 256, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
+  } else if (v.D == 128) {
     gqa_append_rows<128><<<blocks, 128, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
-  else
+  } else {
     gqa_append_rows<64><<<blocks, 128, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
+  }
   if (kpc) {
     if (v.D == 128)
       gqa_append_kresid<128><<<v.B, 128, 0, st>>>(v, k, in_f32, n_new, n_per_seq);

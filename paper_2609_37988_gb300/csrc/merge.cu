@@ -13,35 +13,71 @@
 namespace kvk {
 namespace {
 
+// One thread per output element: every load of the row's partials (the S
+// maxima, sums and this element's accumulators) is issued before any is
+// used, so the merge costs one memory round trip.  Rows per CTA: 128 / dim
+// (dim <= 128), else one row with a channel loop.
+template <int SB>
 __global__ void __launch_bounds__(128)
     splitk_merge_kernel(const float *__restrict__ P, int S, int n_rows, int dim,
                         float *__restrict__ out) {
-  const int row = blockIdx.x;
+  const int width = dim >= 128 ? 128 : dim;  // threads per row
+  const int rpc = 128 / width, r_in = (int)threadIdx.x / width;
+  const int row = blockIdx.x * rpc + r_in;
+  if (r_in >= rpc || row >= n_rows) return;
+  const int ch0 = (int)threadIdx.x % width;
   const size_t RS = (size_t)dim + 2;
-  __shared__ float w_s[256];
-  __shared__ float L_s;
-  if (threadIdx.x < 32) {
-    float M = -INFINITY;
-    for (int s = threadIdx.x; s < S; s += 32) M = fmaxf(M, P[((size_t)s * n_rows + row) * RS + dim]);
-    for (int off = 16; off; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    float L = 0.f;
-    for (int s = threadIdx.x; s < S; s += 32) {
-      const float *pr = P + ((size_t)s * n_rows + row) * RS;
-      const float ms = pr[dim];
-      const float w = (ms == -INFINITY || M == -INFINITY) ? 0.f : exp2f(ms - M);
-      w_s[s] = w;
-      L += w * pr[dim + 1];
-    }
-    for (int off = 16; off; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
-    if (threadIdx.x == 0) L_s = L;
+  const size_t SS = (size_t)n_rows * RS;  // split stride
+  const float *pr = P + (size_t)row * RS;
+  float m[SB], l[SB];
+#pragma unroll
+  for (int s = 0; s < SB; ++s) {
+    m[s] = s < S ? pr[s * SS + dim] : -INFINITY;
+    l[s] = s < S ? pr[s * SS + dim + 1] : 0.f;
   }
-  __syncthreads();
-  const float L = L_s;
-  for (int ch = threadIdx.x; ch < dim; ch += blockDim.x) {
-    float A = 0.f;
-    for (int s = 0; s < S; ++s) {
-      const float w = w_s[s];
-      if (w != 0.f) A += w * P[((size_t)s * n_rows + row) * RS + ch];
+  for (int ch = ch0; ch < dim; ch += 128) {
+    float x[SB];
+#pragma unroll
+    for (int s = 0; s < SB; ++s) x[s] = s < S ? pr[s * SS + ch] : 0.f;
+    float M = -INFINITY;
+#pragma unroll
+    for (int s = 0; s < SB; ++s) M = fmaxf(M, m[s]);
+    float L = 0.f, A = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int s = 0; s < SB; ++s) {
+        const float w = m[s] == -INFINITY ? 0.f : exp2f(m[s] - M);
+        L = fmaf(w, l[s], L);
+        A = fmaf(w, x[s], A);
+      }
+    }
+    out[(size_t)row * dim + ch] = (L > 0.f) ? A / L : 0.f;
+  }
+}
+
+// more than 16 splits: the same, with the split loop not unrolled
+__global__ void __launch_bounds__(128)
+    splitk_merge_kernel_n(const float *__restrict__ P, int S, int n_rows, int dim,
+                          float *__restrict__ out) {
+  const int width = dim >= 128 ? 128 : dim;  // threads per row
+  const int rpc = 128 / width, r_in = (int)threadIdx.x / width;
+  const int row = blockIdx.x * rpc + r_in;
+  if (r_in >= rpc || row >= n_rows) return;
+  const int ch0 = (int)threadIdx.x % width;
+  const size_t RS = (size_t)dim + 2;
+  const size_t SS = (size_t)n_rows * RS;
+  const float *pr = P + (size_t)row * RS;
+  float M = -INFINITY;
+  for (int s = 0; s < S; ++s) M = fmaxf(M, pr[s * SS + dim]);
+  for (int ch = ch0; ch < dim; ch += 128) {
+    float L = 0.f, A = 0.f;
+    if (M != -INFINITY) {
+      for (int s = 0; s < S; ++s) {
+        const float ms = pr[s * SS + dim];
+        const float w = ms == -INFINITY ? 0.f : exp2f(ms - M);
+        L = fmaf(w, pr[s * SS + dim + 1], L);
+        A = fmaf(w, pr[s * SS + ch], A);
+      }
     }
     out[(size_t)row * dim + ch] = (L > 0.f) ? A / L : 0.f;
   }
@@ -63,8 +99,16 @@ cudaError_t launch_rewind(const RewindArgs &a, cudaStream_t st) {
 
 cudaError_t launch_splitk_merge(const float *partials, int n_splits, int n_rows, int dim,
                                 float *out, cudaStream_t st) {
-  if (n_splits > 256) return cudaErrorInvalidValue;
-  splitk_merge_kernel<<<n_rows, 128, 0, st>>>(partials, n_splits, n_rows, dim, out);
+  if (n_splits < 1 || n_rows < 0 || dim < 1) return cudaErrorInvalidValue;
+  if (n_rows == 0) return cudaSuccess;
+  const int rpc = dim >= 128 ? 1 : 128 / dim;
+  const int grid = (n_rows + rpc - 1) / rpc;
+  if (n_splits <= 8)
+    splitk_merge_kernel<8><<<grid, 128, 0, st>>>(partials, n_splits, n_rows, dim, out);
+  else if (n_splits <= 16)
+    splitk_merge_kernel<16><<<grid, 128, 0, st>>>(partials, n_splits, n_rows, dim, out);
+  else
+    splitk_merge_kernel_n<<<grid, 128, 0, st>>>(partials, n_splits, n_rows, dim, out);
   return cudaGetLastError();
 }
 

@@ -191,6 +191,35 @@ def test_partials_and_reduce_equal_decode():
     assert torch.isinf(p[15, 16:, 128]).all() and (p[15, 16:, 129] == 0).all()
 
 
+@pytest.mark.parametrize("S,dim", [(1, 128), (5, 128), (8, 64), (9, 96), (16, 130), (17, 512),
+                                   (40, 128), (64, 32)])
+def test_splitk_reduce_matches_log_sum_exp(S, dim):
+    """The merge against the log-sum-exp identity in fp64, with empty splits
+    (m = -inf, l = 0) and rows whose splits are all empty."""
+    from paper_2609_37988_gb300.cache import splitk_reduce
+    rng = np.random.default_rng(S * 1000 + dim)
+    rows = 37
+    P = np.zeros((S, rows, dim + 2), np.float32)
+    P[:, :, :dim] = rng.normal(size=(S, rows, dim))
+    P[:, :, dim] = rng.normal(scale=6.0, size=(S, rows))
+    P[:, :, dim + 1] = rng.uniform(1.0, 50.0, size=(S, rows))
+    empty = rng.uniform(size=(S, rows)) < 0.3
+    empty[:, 5] = True  # a row with no positions at all
+    P[:, :, dim][empty] = -np.inf
+    P[:, :, dim + 1][empty] = 0.0
+    P[:, :, :dim][empty] = 0.0
+    got = splitk_reduce(torch.from_numpy(P).cuda()).cpu().numpy()
+    P64 = P.astype(np.float64)
+    m = P64[:, :, dim]
+    M = m.max(axis=0)
+    w = np.where(np.isinf(m), 0.0, np.exp2(m - np.where(np.isinf(M), 0.0, M)))
+    L = (w * P64[:, :, dim + 1]).sum(axis=0)
+    A = (w[:, :, None] * P64[:, :, :dim]).sum(axis=0)
+    want = np.where(L[:, None] > 0, A / np.where(L > 0, L, 1.0)[:, None], 0.0)
+    np.testing.assert_allclose(got, want, rtol=2e-6, atol=2e-6)
+    assert (got[5] == 0).all()
+
+
 def test_per_channel_keys_one_position_at_a_time():
     # the open group moves through the residual plane and is quantised when
     # it fills, exactly as a bulk append of the same positions
