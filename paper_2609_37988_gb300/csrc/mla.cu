@@ -407,41 +407,63 @@ __global__ void __launch_bounds__(128)
   cp_async_commit();
   const size_t RS = (size_t)W + 2;
   const size_t pstride = (size_t)B * H * RS;
-  if (tid < 16) {
-    const int b = b0 + tid;
-    float M = -INFINITY, L = 0.f;
+  // merge weights: every split's (m, l) of the 16 rows loaded at once
+  float *l_s = linv_s + 16;  // [64][16] split sums, then 1/L
+  for (int q = tid; q < n_splits * 16; q += 128) {
+    const int sp = q >> 4, row = q & 15, b = b0 + row;
+    float ms = -INFINITY, ls = 0.f;
     if (b < B) {
-      const float *pr = partial + ((size_t)b * H + h) * RS;
-      for (int s = 0; s < n_splits; ++s) M = fmaxf(M, pr[s * pstride + W]);
-      for (int s = 0; s < n_splits; ++s) {
-        const float ms = pr[s * pstride + W];
-        const float wt = (ms == -INFINITY || M == -INFINITY) ? 0.f : exp2f(ms - M);
-        wt_s[s * 16 + tid] = wt;
-        L += wt * pr[s * pstride + W + 1];
-      }
-    } else {
-      for (int s = 0; s < n_splits; ++s) wt_s[s * 16 + tid] = 0.f;
+      const float *pr = partial + sp * pstride + ((size_t)b * H + h) * RS;
+      ms = pr[W];
+      ls = pr[W + 1];
+    }
+    wt_s[q] = ms;
+    l_s[q] = ls;
+  }
+  __syncthreads();
+  if (tid < 16) {
+    float M = -INFINITY, L = 0.f;
+    for (int sp = 0; sp < n_splits; ++sp) M = fmaxf(M, wt_s[sp * 16 + tid]);
+    for (int sp = 0; sp < n_splits; ++sp) {
+      const float ms = wt_s[sp * 16 + tid];
+      const float wt = (ms == -INFINITY || M == -INFINITY) ? 0.f : exp2f(ms - M);
+      wt_s[sp * 16 + tid] = wt;
+      L += wt * l_s[sp * 16 + tid];
     }
     linv_s[tid] = (L > 0.f) ? 1.f / L : 0.f;
   }
   __syncthreads();
-  for (int e = tid; e < 16 * (W / 2); e += 128) {
-    const int row = e / (W / 2), i = 2 * (e % (W / 2));
-    const int b = b0 + row;
-    float2 acc = make_float2(0.f, 0.f);
-    if (b < B) {
-      const float *pr = partial + ((size_t)b * H + h) * RS + i;
-#pragma unroll 4
-      for (int s = 0; s < n_splits; ++s) {
-        const float wt = wt_s[s * 16 + row];
-        const float2 x = *reinterpret_cast<const float2 *>(pr + s * pstride);
-        acc.x += wt * x.x;
-        acc.y += wt * x.y;
-      }
+  // o_lat = sum_s w_s acc_s / L, (row, pair) elements of the 16 rows: each
+  // thread keeps its PER elements in registers and issues a split's loads
+  // together, one memory round trip per split
+  constexpr int PER = 16 * (W / 2) / 128;
+  float2 oacc[PER];
+#pragma unroll
+  for (int k = 0; k < PER; ++k) oacc[k] = make_float2(0.f, 0.f);
+  for (int sp = 0; sp < n_splits; ++sp) {
+    float2 x[PER];
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+      const int e = tid + 128 * k, row = e / (W / 2), i = 2 * (e % (W / 2));
+      const int b = b0 + row;
+      x[k] = b < B ? *reinterpret_cast<const float2 *>(partial + sp * pstride +
+                                                       ((size_t)b * H + h) * RS + i)
+                   : make_float2(0.f, 0.f);
     }
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+      const int row = (tid + 128 * k) / (W / 2);
+      const float wt = wt_s[sp * 16 + row];
+      oacc[k].x = fmaf(wt, x[k].x, oacc[k].x);
+      oacc[k].y = fmaf(wt, x[k].y, oacc[k].y);
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < PER; ++k) {
+    const int e = tid + 128 * k, row = e / (W / 2), i = 2 * (e % (W / 2));
     const float li = linv_s[row];
     uint32_t hi, lo;
-    split2<true>(acc.x * li, acc.y * li, hi, lo);
+    split2<true>(oacc[k].x * li, oacc[k].y * li, hi, lo);
     *reinterpret_cast<uint32_t *>(oh_s + row * OST + i) = hi;
     *reinterpret_cast<uint32_t *>(ol_s + row * OST + i) = lo;
   }
@@ -490,7 +512,7 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
                                                 static_cast<const uint16_t *>(a.q_pe), a.H,
                                                 a.sig_log2, a.items_per_split,
                                                 a.n_splits, a.partial, a.err);
-  constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (64 * 16 + 16) * 4;
+  constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
   static bool mu_attr = false;
   if (!mu_attr) {
     cudaError_t e2 = cudaFuncSetAttribute(mla_merge_upv_kernel<W>,
