@@ -319,7 +319,7 @@ def main():
     ap.add_argument("--impl", default="kvk")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--profile-case", choices=["gqa", "mla"], default=None,
+    ap.add_argument("--profile-case", choices=["gqa", "mla", "gather"], default=None,
                     help="small ncu case: decode launches only, no timing line")
     args = ap.parse_args()
     if args.impl == "reference":
@@ -559,7 +559,9 @@ def profile_case(kind):
     """The kernel-level ncu case.  gqa: one int4 g32 and one bf16 anchor at
     the 14B step shape (B=32, 8 kv / 40 q heads, d_h 128, T=8192; 1.5 GB of
     cache, both anchors larger than L2); each decode runs 3 times in the order
-    int4, bf16.  mla: one d=512 latent layer at B=64, T=4096 (302 MB)."""
+    int4, bf16.  mla: one d=512 latent layer at B=64, T=4096 (302 MB).
+    gather: one int4 g32 anchor at B=4, T=131072 with a kept list of T/8
+    positions per sequence (805 MB cache, 101 MB read per decode), 3 decodes."""
     import torch
     from __graft_entry__ import build
     build()
@@ -579,6 +581,20 @@ def profile_case(kind):
         for _ in range(3):
             for l in range(2):
                 c.decode(l, q, w.sigma)
+    elif kind == "gather":
+        import numpy as np
+        w = W.config(5, n_layers=1)
+        T = w.context
+        c = Cache(n_layers=1, n_q_heads=40, n_kv_heads=8, head_dim=128, max_batch=w.batch,
+                  max_ctx=T, layers=[Layer(bits=4, group=32, evict_capacity=w.keep)])
+        k, v = W.kv_inputs(w, 0, 0, T, device="cuda")
+        c.append(0, k, v)
+        del k, v
+        idx, n = W.kept_positions(w, 0, np.full(w.batch, T), device="cuda")
+        c.set_kept(0, idx, n)
+        q = W.queries(w, 0, device="cuda")
+        for _ in range(3):
+            c.decode(0, q, w.sigma)
     else:
         w = W.config(4, n_layers=1)
         w.layers[0]["width"] = 512

@@ -274,9 +274,10 @@ __global__ void __launch_bounds__(256)
       }
     // ---- weights of this warp's 16 positions -> P^T fragments -------------
     {
-      const float ma = m_run[nb][0], mb2 = m_run[nb][1];
-      l_part[0] *= alpha[nb][0];
-      l_part[1] *= alpha[nb][1];
+      // this warp's head block nb (selects, not indexing: no local memory)
+      const float ma = nb ? m_run[1][0] : m_run[0][0], mb2 = nb ? m_run[1][1] : m_run[0][1];
+      l_part[0] *= nb ? alpha[1][0] : alpha[0][0];
+      l_part[1] *= nb ? alpha[1][1] : alpha[0][1];
       float p[4];
       p[0] = (ma == -INFINITY) ? 0.f : fast_exp2(x[0] - ma);
       p[1] = (mb2 == -INFINITY) ? 0.f : fast_exp2(x[1] - mb2);
@@ -299,8 +300,9 @@ __global__ void __launch_bounds__(256)
       const int unit = warp + 8 * u;
       if (unit < C::UNITS) {
         const int un = unit & 1;
-        acc[u][0] *= alpha[un][0]; acc[u][2] *= alpha[un][0];
-        acc[u][1] *= alpha[un][1]; acc[u][3] *= alpha[un][1];
+        const float a0 = un ? alpha[1][0] : alpha[0][0], a1 = un ? alpha[1][1] : alpha[0][1];
+        acc[u][0] *= a0; acc[u][2] *= a0;
+        acc[u][1] *= a1; acc[u][3] *= a1;
       }
     }
     __syncthreads();
