@@ -28,75 +28,65 @@ constexpr int kHeads = 16;
 __device__ __forceinline__ int swz8(int row, int chunk) { return chunk ^ (row & 7); }
 
 // ---------------------------------------------------------------------------
-// Absorb: q_lat[b,h,i] = sum_j q_nope[b,h,j] W_UK[h,j,i], i < d.  Per CTA one
-// head and 64 latent coordinates for up to 64 sequences: M = sequences,
-// N = latent, K = Dn = 128.  Output qlat[b][h] = [hi(d) | pe(64) | lo(d)].
+// Absorb: q_lat[b,h,i] = sum_j q_nope[b,h,j] W_UK[h,j,i], i < d.  Grid
+// (64-coordinate block, head, 16-sequence block): M = 16 sequences, N = 64
+// latent coordinates (16 per warp), K = Dn = 128.  Small CTAs, many of them:
+// the operands arrive in one round trip.  Output qlat[b][h] =
+// [hi(d) | pe(64) | lo(d)].
 template <int W>
 __global__ void __launch_bounds__(128)
     mla_absorb_kernel(const uint16_t *__restrict__ q_nope, const uint16_t *__restrict__ q_pe,
                       const uint16_t *__restrict__ w_uk, int B, int H, int r,
                       uint16_t *__restrict__ qlat) {
   constexpr int Dn = 128;
-  __shared__ __align__(16) uint16_t a_s[64 * Dn];  // [b][j], swizzled 16B chunks
+  __shared__ __align__(16) uint16_t a_s[16 * Dn];  // [b][j], swizzled 16B chunks
   __shared__ __align__(16) uint16_t w_s[Dn * 64];  // [j][i], swizzled
-  const int h = blockIdx.y, i0 = blockIdx.x * 64;
+  const int h = blockIdx.y, i0 = blockIdx.x * 64, b0 = blockIdx.z * 16;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c = lane & 3;
   constexpr int QROW = 2 * W + kRope;
-  for (int b0 = 0; b0 < B; b0 += 64) {
-    // stage q_nope rows (64 sequences) and the W_UK slice
-    for (int q = tid; q < 64 * Dn / 8; q += 128) {
-      const int row = q / (Dn / 8), u = q % (Dn / 8);
-      const int b = b0 + row;
-      uint4 x = make_uint4(0, 0, 0, 0);
-      if (b < B) x = *reinterpret_cast<const uint4 *>(q_nope + ((size_t)b * H + h) * Dn + 8 * u);
-      *reinterpret_cast<uint4 *>(a_s + row * Dn + 8 * swz8(row, u)) = x;
+  for (int q = tid; q < 16 * Dn / 8; q += 128) {
+    const int row = q / (Dn / 8), u = q % (Dn / 8);
+    const int b = b0 + row;
+    uint4 x = make_uint4(0, 0, 0, 0);
+    if (b < B) x = *reinterpret_cast<const uint4 *>(q_nope + ((size_t)b * H + h) * Dn + 8 * u);
+    *reinterpret_cast<uint4 *>(a_s + row * Dn + 8 * swz8(row, u)) = x;
+  }
+  for (int q = tid; q < Dn * 8; q += 128) {
+    const int j = q / 8, u = q % 8;
+    const uint4 x = *reinterpret_cast<const uint4 *>(w_uk + ((size_t)h * Dn + j) * r + i0 + 8 * u);
+    *reinterpret_cast<uint4 *>(w_s + j * 64 + 8 * swz8(j, u)) = x;
+  }
+  __syncthreads();
+  float acc[2][4] = {};
+  const int mat = lane >> 3, rr = lane & 7;
+#pragma unroll
+  for (int ks = 0; ks < Dn / 16; ++ks) {
+    uint32_t a0, a1, a2, a3, b0r, b1r, b2r, b3r;
+    {
+      const int row = rr + ((mat & 1) ? 8 : 0);
+      ldmatrix_x4(a0, a1, a2, a3, a_s + row * Dn + 8 * swz8(row, 2 * ks + (mat >> 1)));
     }
-    for (int q = tid; q < Dn * 8; q += 128) {
-      const int j = q / 8, u = q % 8;
-      const uint4 x = *reinterpret_cast<const uint4 *>(w_uk + ((size_t)h * Dn + j) * r + i0 + 8 * u);
-      *reinterpret_cast<uint4 *>(w_s + j * 64 + 8 * swz8(j, u)) = x;
+    {
+      const int j = 16 * ks + rr + ((mat & 1) ? 8 : 0);
+      ldmatrix_x4_t(b0r, b1r, b2r, b3r, w_s + j * 64 + 8 * swz8(j, 2 * warp + (mat >> 1)));
     }
-    __syncthreads();
-    float acc[8][4];
+    mma_bf16(acc[0], a0, a1, a2, a3, b0r, b1r);
+    mma_bf16(acc[1], a0, a1, a2, a3, b2r, b3r);
+  }
 #pragma unroll
-    for (int n = 0; n < 8; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
-    const int mrow = 16 * warp;
+  for (int n = 0; n < 2; ++n) {
+    const int i = i0 + 16 * warp + 8 * n + 2 * c;
 #pragma unroll
-    for (int ks = 0; ks < Dn / 16; ++ks) {
-      uint32_t a0, a1, a2, a3;
-      {
-        const int mat = lane >> 3, rr = lane & 7;
-        const int row = mrow + rr + ((mat & 1) ? 8 : 0);
-        const int ch = 2 * ks + (mat >> 1);
-        ldmatrix_x4(a0, a1, a2, a3, a_s + row * Dn + 8 * swz8(row, ch));
-      }
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {  // two n-blocks per ldmatrix.x4.trans
-        uint32_t b0, b1, b2, b3;
-        const int mat = lane >> 3, rr = lane & 7;
-        const int j = 16 * ks + rr + ((mat & 1) ? 8 : 0);
-        const int ch = 2 * np + (mat >> 1);
-        ldmatrix_x4_t(b0, b1, b2, b3, w_s + j * 64 + 8 * swz8(j, ch));
-        mma_bf16(acc[2 * np], a0, a1, a2, a3, b0, b1);
-        mma_bf16(acc[2 * np + 1], a0, a1, a2, a3, b2, b3);
-      }
+    for (int hr = 0; hr < 2; ++hr) {
+      const int b = b0 + g + 8 * hr;
+      if (b >= B) continue;
+      uint32_t hi, lo;
+      split2<true>(acc[n][2 * hr], acc[n][2 * hr + 1], hi, lo);
+      uint16_t *dst = qlat + ((size_t)b * H + h) * QROW;
+      *reinterpret_cast<uint32_t *>(dst + i) = hi;
+      *reinterpret_cast<uint32_t *>(dst + W + kRope + i) = lo;
     }
-#pragma unroll
-    for (int n = 0; n < 8; ++n) {
-      const int i = i0 + 8 * n + 2 * c;
-#pragma unroll
-      for (int hr = 0; hr < 2; ++hr) {
-        const int b = b0 + mrow + g + 8 * hr;
-        if (b >= B) continue;
-        uint32_t hi, lo;
-        split2<true>(acc[n][2 * hr], acc[n][2 * hr + 1], hi, lo);
-        uint16_t *dst = qlat + ((size_t)b * H + h) * QROW;
-        *reinterpret_cast<uint32_t *>(dst + i) = hi;
-        *reinterpret_cast<uint32_t *>(dst + W + kRope + i) = lo;
-      }
-    }
-    __syncthreads();
   }
 }
 
@@ -439,25 +429,36 @@ __global__ void __launch_bounds__(128)
   // thread keeps its PER elements in registers and issues a split's loads
   // together, one memory round trip per split
   constexpr int PER = 16 * (W / 2) / 128;
+  constexpr int SG = PER >= 16 ? 1 : 16 / PER;  // splits whose loads are in flight together
   float2 oacc[PER];
 #pragma unroll
   for (int k = 0; k < PER; ++k) oacc[k] = make_float2(0.f, 0.f);
-  for (int sp = 0; sp < n_splits; ++sp) {
-    float2 x[PER];
+  for (int sp0 = 0; sp0 < n_splits; sp0 += SG) {
+    float2 x[SG][PER];
 #pragma unroll
-    for (int k = 0; k < PER; ++k) {
-      const int e = tid + 128 * k, row = e / (W / 2), i = 2 * (e % (W / 2));
-      const int b = b0 + row;
-      x[k] = b < B ? *reinterpret_cast<const float2 *>(partial + sp * pstride +
-                                                       ((size_t)b * H + h) * RS + i)
-                   : make_float2(0.f, 0.f);
+    for (int g2 = 0; g2 < SG; ++g2) {
+      const int sp = sp0 + g2;
+#pragma unroll
+      for (int k = 0; k < PER; ++k) {
+        const int e = tid + 128 * k, row = e / (W / 2), i = 2 * (e % (W / 2));
+        const int b = b0 + row;
+        x[g2][k] = (sp < n_splits && b < B)
+                       ? *reinterpret_cast<const float2 *>(partial + sp * pstride +
+                                                           ((size_t)b * H + h) * RS + i)
+                       : make_float2(0.f, 0.f);
+      }
     }
 #pragma unroll
-    for (int k = 0; k < PER; ++k) {
-      const int row = (tid + 128 * k) / (W / 2);
-      const float wt = wt_s[sp * 16 + row];
-      oacc[k].x = fmaf(wt, x[k].x, oacc[k].x);
-      oacc[k].y = fmaf(wt, x[k].y, oacc[k].y);
+    for (int g2 = 0; g2 < SG; ++g2) {
+      const int sp = sp0 + g2;
+      if (sp >= n_splits) break;
+#pragma unroll
+      for (int k = 0; k < PER; ++k) {
+        const int row = (tid + 128 * k) / (W / 2);
+        const float wt = wt_s[sp * 16 + row];
+        oacc[k].x = fmaf(wt, x[g2][k].x, oacc[k].x);
+        oacc[k].y = fmaf(wt, x[g2][k].y, oacc[k].y);
+      }
     }
   }
 #pragma unroll
@@ -500,7 +501,7 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
   using C = MlaCfg<W>;
   if (a.n_splits > 64) return cudaErrorInvalidValue;  // merge weights hold 64 splits
   const int B = a.v.B;
-  mla_absorb_kernel<W><<<dim3(W / 64, a.H), 128, 0, st>>>(
+  mla_absorb_kernel<W><<<dim3(W / 64, a.H, (B + 15) / 16), 128, 0, st>>>(
       static_cast<const uint16_t *>(a.q_nope), static_cast<const uint16_t *>(a.q_pe),
       static_cast<const uint16_t *>(a.w_uk), B, a.H, a.r, a.qlat);
   auto k = mla_decode_kernel<W>;
