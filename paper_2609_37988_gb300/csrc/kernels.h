@@ -84,8 +84,12 @@ struct MlaDecodeArgs {
   float *olat;         // [B, H, width]
   float *out;          // [B, H, Dv]
   int32_t *err;
+  const void *tmap;    // host copy of the anchor's 128-byte tensor map (mla_make_tmap)
 };
 cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st);
+// Encodes the decode kernel's tensor map of an MLA anchor into `out` (128
+// bytes, 64-byte aligned).
+cudaError_t mla_make_tmap(void *out, const MlaView &v);
 int mla_decode_ctas_per_sm(int width);
 
 }  // namespace kvk

@@ -154,6 +154,10 @@ struct kvk_cache {
   int sm_count;
   int device;
   std::vector<int> ctas;  // per layer, decode CTAs per SM (0 = not queried)
+  struct alignas(64) Tmap {
+    uint8_t bytes[128];
+  };
+  std::vector<Tmap> tmap;  // per MLA anchor, the decode kernel's tensor map
 
   GqaView gqa_view(int l) const {
     const ArenaLayout &A = lay[l];
@@ -353,6 +357,17 @@ kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg
   if (e != cudaSuccess) {
     delete c;
     return cuda_fail(e, "querying the device");
+  }
+  if (desc->kind == KVK_KIND_MLA) {
+    c->tmap.resize(desc->n_layers);
+    for (int l = 0; l < desc->n_layers; ++l) {
+      if (cfg[l].inherit) continue;
+      e = mla_make_tmap(c->tmap[l].bytes, c->mla_view(l));
+      if (e != cudaSuccess) {
+        delete c;
+        return cuda_fail(e, "encoding the tensor map of an MLA anchor");
+      }
+    }
   }
   *out = c;
   return KVK_OK;
@@ -627,6 +642,7 @@ kvk_status kvk_decode_attention_mla(kvk_cache *c, int32_t layer, const void *q_n
   const int a = c->src[layer];
   MlaDecodeArgs args;
   args.v = c->mla_view(a);
+  args.tmap = c->tmap[a].bytes;
   const int tiles = layer_tiles(c, a);
   if (n_splits == 0) n_splits = auto_splits(c, a);
   n_splits = std::min(std::min(n_splits, tiles), 64);

@@ -15,6 +15,8 @@
 // hi + lo bf16 halves, so products keep ~16 significant bits.
 #include <math.h>
 
+#include <cuda.h>  // CUtensorMap and its enums (the encoder is reached through the runtime)
+
 #include "common.cuh"
 #include "kernels.h"
 #include "layout.h"
@@ -91,281 +93,480 @@ __global__ void __launch_bounds__(128)
 }
 
 // ---------------------------------------------------------------------------
-// Latent split-K decode.  Grid (split, sequence); 8 warps.  Tile = 64
-// positions of [c[:W] | k^R] streamed through a cp.async ring.
-//   score phase: warp (mb, nb) = (warp/2, warp%2): 16 positions x 8 heads,
-//                K = W (q_lat hi and lo) + 64 (q_pe);
-//   value phase: warp w owns (16 latent rows x 8 heads) units w, w+8, ...
-//                of O^T[W x 16], K = the tile's 64 positions (P hi and lo).
-template <int W>
-struct MlaCfg {
-  static constexpr int RB = (W + kRope) * 2;      // record bytes
-  static constexpr int NCH = RB / 16;             // 16-byte chunks per record
-  static constexpr int STAGE = kTile * RB;
-  static constexpr int NST = W >= 512 ? 2 : (W >= 256 ? 3 : 4);
-  static constexpr int QH_ROW = (W + kRope) * 2;  // bytes: hi q_lat | q_pe
-  static constexpr int QL_ROW = W * 2;            // bytes: lo q_lat
-  static constexpr int Q_BYTES = kHeads * (QH_ROW + QL_ROW);
-  static constexpr int P_BYTES = 4 * 2 * 4 * 32 * 4;
-  static constexpr int X_BYTES = 4 * kHeads * 4 * 2;  // tile maxima, row sums
-  static constexpr int SMEM = Q_BYTES + P_BYTES + X_BYTES + NST * STAGE;
-  static constexpr int UNITS = W / 8;              // (16 rows x 8 heads) value units
-  static constexpr int UPW = (UNITS + 7) / 8;      // units per warp
-  static_assert(NCH % 8 == 0, "swizzle needs 8-chunk multiples");
-};
+// Latent split-K decode on the 5th-generation tensor cores.  Grid (split,
+// sequence); 6 warps: warps 0-3 run the softmax and the epilogue, warp 4
+// issues the UMMAs, warp 5 the TMA copies.  Tiles of TR positions of
+// [c[:W] | k^R] (TR = 48 for W = 512, so that three stages fit, else 64).
+//
+// Shared memory per stage: the tile as (W + 64)/64 boxes of TR positions x
+// 64 coordinates, each box TR rows of 128 bytes in the 128-byte swizzled
+// layout, written by TMA tensor copies (one per box, completing on the
+// stage's mbarrier).  The same bytes serve both products:
+//   scores  S[pos x 32] = C[pos x (W+64)] [Q_hi ; Q_lo]^T
+//           (UMMA M=64 (rows past TR are ignored), N=32: columns 0-15 are
+//           the heads' q_lat hi (+ q_pe) parts, 16-31 their q_lat lo parts;
+//           A = the tile K-major);
+//   values  O^T[W x 32] += C^T[W x TR pos] [P_hi | P_lo]
+//           (UMMA M=128 latent rows (64 for W = 64), N = 16 heads hi + 16
+//           heads lo, A = the tile read MN-major); O = columns h + 16+h.
+// Score rows come back with tcgen05.ld (M=64 accumulator: row r in TMEM
+// lane 32 (r/16) + r%16), so lane r%16 of softmax warp r/16 owns position r:
+// its 16 scores stay in registers; the online softmax is base 2 with a stale
+// maximum kept within 2^8 (one vote per tile; maxima are reduced only when
+// one rises).  The weights go hi/lo in bf16 into the P operand; O stays in
+// TMEM until the end (rescaled in place on the rare tiles that raise a
+// maximum).  The MMA warp keeps the tensor core fed: scores(t) goes out as
+// soon as tile t has landed, values(t-1) as soon as P(t-1) is written; the
+// copy warp refills a stage as soon as the values that read it completed.
+// Every wait is bounded (an abort flag stops the other role); the CTA frees
+// its TMEM on every path.
+// positions per decode tile (and rows of a TMA box) for kept width w
+__host__ __device__ constexpr int mla_tile_rows(int w) { return w == 512 ? 48 : 64; }
 
 template <int W>
-__global__ void __launch_bounds__(256)
-    mla_decode_kernel(const MlaView v, const uint16_t *__restrict__ qlat,
-                      const uint16_t *__restrict__ q_pe, int H, float sig_log2,
-                      int items_per_split, int n_splits, float *__restrict__ partial,
+struct MlaCfg {
+  static constexpr int TR = mla_tile_rows(W);         // positions per tile
+  static constexpr int KH = W + kRope;                // hi extent: latent + rope
+  static constexpr int BOXES = KH / 64;               // 64-coordinate boxes per tile
+  static constexpr int BOX = TR * 128;                // bytes per box
+  static constexpr int STAGE = BOXES * BOX;
+  static constexpr int NST = 3;
+  static constexpr int QB = 32 * KH * 2;              // [Q_hi ; Q_lo] operand (32 rows)
+  static constexpr int PB = 4 * 1024;                 // [P_hi | P_lo] operand, 4 column blocks
+  static constexpr int OFF_Q = NST * STAGE;
+  static constexpr int OFF_P = OFF_Q + QB;            // two buffers
+  static constexpr int OFF_RED = OFF_P + 2 * PB;      // float [4][16] maxima, [4][16] sums
+  static constexpr int OFF_BAR = OFF_RED + 512;       // full[NST], sbar[2], pbar[2], obar[NST], dbar
+  static constexpr int NBAR = 2 * NST + 5;
+  static constexpr int OFF_TB = OFF_BAR + 8 * NBAR;   // TMEM base address, abort flag
+  static constexpr int SMEM = OFF_TB + 16 + 1024;     // + slack to align the base to 1024
+  static constexpr int MV = W >= 128 ? 128 : 64;      // value UMMA M
+  static constexpr int MB = W / MV;                   // value M-blocks
+  static constexpr int OCOLS = 32 * MB;               // TMEM columns of O
+  static constexpr int SCOLS = 64;                    // two 32-column S buffers
+  static constexpr int TCOLS = OCOLS + SCOLS <= 128 ? 128 : 256;
+  static_assert(KH % 64 == 0 && W % 64 == 0, "whole boxes");
+  static_assert(TR % 16 == 0 && TR <= 64, "tile rows");
+  static_assert(OCOLS + SCOLS <= TCOLS, "TMEM columns");
+  static_assert(SMEM <= 232448, "shared memory");
+};
+
+// shared-memory matrix descriptor (sm_100 format): start, leading and
+// stride byte offsets (>> 4), version 1, layout (0 = none, 2 = 128B swizzle)
+__device__ __forceinline__ uint64_t umma_desc(uint32_t addr, uint32_t lbo, uint32_t sbo,
+                                              uint32_t layout) {
+  return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | ((uint64_t)1 << 46) |
+         ((uint64_t)(layout & 7) << 61);
+}
+// instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B
+__host__ __device__ constexpr uint32_t umma_idesc(int M, int N, bool a_mn, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) |
+         ((b_mn ? 1u : 0u) << 16) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t da, uint64_t db, uint32_t idesc,
+                                         bool accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(da), "l"(db), "r"(idesc), "r"(accumulate ? 1 : 0)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t *bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// 16 consecutive TMEM columns of this warp's 32 lanes
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+// 2-D TMA tile load (x = coordinate, y = row) completing on `bar`
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *tmap, int x, int y,
+                                            uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Waits for a barrier phase, at most `limit` polls, giving up early when the
+// CTA's abort flag is set; false when it gave up.
+__device__ __forceinline__ bool mbar_wait_or_abort(uint64_t *bar, uint32_t parity, uint32_t limit,
+                                                   const volatile int *abort_flag) {
+  const uint32_t a = smem_u32(bar);
+  for (uint32_t i = 0; i < limit; ++i) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(a), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if ((i & 63) == 63 && *abort_flag) return false;
+  }
+  return false;
+}
+// barrier over the four softmax warps (named barrier 1, 128 threads); the
+// reduction form returns whether any thread passed true
+__device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+__device__ __forceinline__ bool softmax_sync_or(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 128, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u)
+      : "memory");
+  return r != 0;
+}
+
+template <int W>
+__global__ void __launch_bounds__(192, 1)
+    mla_decode_kernel(const __grid_constant__ CUtensorMap tmap, const MlaView v,
+                      const uint16_t *__restrict__ qlat, const uint16_t *__restrict__ q_pe, int H,
+                      float sig, int items_per_split, int n_splits, float *__restrict__ partial,
                       int32_t *err) {
   using C = MlaCfg<W>;
-  extern __shared__ __align__(128) uint8_t smem[];
-  uint8_t *qh_s = smem;
-  uint8_t *ql_s = smem + kHeads * C::QH_ROW;
-  uint32_t *p_s = reinterpret_cast<uint32_t *>(smem + C::Q_BYTES);
-  float *tmax_s = reinterpret_cast<float *>(smem + C::Q_BYTES + C::P_BYTES);  // [4][16]
-  float *lsum_s = tmax_s + 4 * kHeads;                                         // [4][16]
-  uint8_t *stages = smem + C::Q_BYTES + C::P_BYTES + C::X_BYTES;
+  constexpr int TR = C::TR;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  // full[s]: tile landed in stage s; sbar[i]: scores of a tile with parity i
+  // done; pbar[i]: its weights written (4 arrivals); obar[s]: the values of
+  // the tile in stage s done; dbar: everything done
+  uint64_t *full = reinterpret_cast<uint64_t *>(sm + C::OFF_BAR);
+  uint64_t *sbar = full + C::NST, *pbar = sbar + 2, *obar = pbar + 2, *dbar = obar + C::NST;
+  uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + C::OFF_TB);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + C::OFF_TB + 4);
+  float *red = reinterpret_cast<float *>(sm + C::OFF_RED);  // [4 warps][16]
+  float *lsum = red + 4 * kHeads;                           // [4 warps][16]
+  uint8_t *q_s = sm + C::OFF_Q;
 
   const int split = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int g = lane >> 2, c = lane & 3;
   const int len = v.lens[b];
   const int i0 = split * items_per_split;
   const int i1 = (split == n_splits - 1) ? len : min(i0 + items_per_split, len);
-  const int n_tiles = i1 > i0 ? (i1 - i0 + kTile - 1) / kTile : 0;
-  const uint8_t *rec = v.rec + (size_t)b * v.cap * C::RB;
+  const int n_tiles = i1 > i0 ? (i1 - i0 + TR - 1) / TR : 0;
+  const int row0 = b * (int)v.cap + i0;  // tensor-map row of the split's first position
+  constexpr uint32_t kLimit = 1u << 22;
 
-  // absorbed query [hi | pe] and [lo] into shared memory, swizzled rows;
-  // q_pe comes straight from the caller's tensor
+  if (tid == 0) {
+    for (int i = 0; i < C::NBAR; ++i) {
+      const bool pb = i >= C::NST + 2 && i < C::NST + 4;
+      mbar_init(&full[i], pb ? 4 : 1);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 4) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tbase)),
+                 "r"(C::TCOLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  // query operand, K-major core layout: row n, coordinate k at
+  // (n/8) SBO + (k/8) 128 + (n%8) 16 + (k%8) 2 with SBO = (W+64)/8 128.
+  // Rows 0-15: [q_lat hi | q_pe] of head n; rows 16-31: [q_lat lo | 0] of
+  // head n-16.
   {
-    constexpr int QROW = 2 * W + kRope;
+    constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (unused 64) | lo(W)]
     const uint16_t *qb = qlat + (size_t)b * H * QROW;
-    for (int q = tid; q < kHeads * (C::QH_ROW / 16); q += 256) {
-      const int h = q / (C::QH_ROW / 16), u = q % (C::QH_ROW / 16);
+    for (int q = tid; q < 32 * (C::KH / 8); q += 192) {
+      const int n = q / (C::KH / 8), c = q % (C::KH / 8);
+      const int h = n & 15;
       uint4 x = make_uint4(0, 0, 0, 0);
       if (h < H) {
-        x = (u < W / 8) ? *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + 8 * u)
-                        : *reinterpret_cast<const uint4 *>(q_pe + ((size_t)b * H + h) * kRope +
-                                                           8 * (u - W / 8));
+        if (n < 16)
+          x = *reinterpret_cast<const uint4 *>(c < W / 8 ? qb + (size_t)h * QROW + 8 * c
+                                                         : q_pe + ((size_t)b * H + h) * kRope + 8 * (c - W / 8));
+        else if (c < W / 8)
+          x = *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + C::KH + 8 * c);
       }
-      *reinterpret_cast<uint4 *>(qh_s + h * C::QH_ROW + 16 * swz8(h, u)) = x;
-    }
-    for (int q = tid; q < kHeads * (C::QL_ROW / 16); q += 256) {
-      const int h = q / (C::QL_ROW / 16), u = q % (C::QL_ROW / 16);
-      uint4 x = make_uint4(0, 0, 0, 0);
-      if (h < H) x = *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + W + kRope + 8 * u);
-      *reinterpret_cast<uint4 *>(ql_s + h * C::QL_ROW + 16 * swz8(h, u)) = x;
+      *reinterpret_cast<uint4 *>(q_s + (n / 8) * (C::KH / 8 * 128) + c * 128 + (n % 8) * 16) = x;
     }
   }
-
-  auto issue = [&](int t, int s) {
-    const int base = i0 + t * kTile;
-    uint8_t *st = stages + s * C::STAGE;
-    for (int q = tid; q < kTile * C::NCH; q += 256) {
-      const int row = q / C::NCH, u = q - row * C::NCH;
-      const int item = base + row;
-      const bool valid = item < i1;
-      const uint8_t *src = rec + (size_t)(valid ? item : 0) * C::RB + 16 * u;
-      cp_async16(st + row * C::RB + 16 * swz8(row, u), src, valid);
-    }
-  };
-
-  const int mb = warp >> 1, nb = warp & 1;
-  float m_run[2][2] = {{-INFINITY, -INFINITY}, {-INFINITY, -INFINITY}};  // [nb][hh]
-  float l_part[2] = {0.f, 0.f};  // this warp's rows, heads nb*8 + 2c + hh
-  float acc[C::UPW][4];
-#pragma unroll
-  for (int u = 0; u < C::UPW; ++u) acc[u][0] = acc[u][1] = acc[u][2] = acc[u][3] = 0.f;
-
-#pragma unroll
-  for (int s = 0; s < C::NST - 1; ++s) {
-    if (s < n_tiles) issue(s, s);
-    cp_async_commit();
-  }
-  for (int t = 0; t < n_tiles; ++t) {
-    cp_async_wait<C::NST - 2>();
-    __syncthreads();
-    {
-      const int nt = t + C::NST - 1;
-      if (nt < n_tiles) issue(nt, nt % C::NST);
-      cp_async_commit();
-    }
-    const uint8_t *st = stages + (t % C::NST) * C::STAGE;
-    const int base = i0 + t * kTile;
-
-    // ---- scores: 16 positions x 8 heads per warp -------------------------
-    // four independent accumulators (hi/lo x even/odd k-steps) so the MMA
-    // chain is not one long dependency
-    float dacc[4][4] = {};
-    const int mat = lane >> 3, rr = lane & 7;
-    const int hrow = 8 * nb + rr;
-#pragma unroll 4
-    for (int ks = 0; ks < W / 16; ++ks) {
-      uint32_t a0, a1, a2, a3;
-      {
-        const int row = 16 * mb + rr + ((mat & 1) ? 8 : 0);
-        ldmatrix_x4(a0, a1, a2, a3, st + row * C::RB + 16 * swz8(row, 2 * ks + (mat >> 1)));
-      }
-      uint32_t b0, b1, b2, b3;  // hi (2 chunks) then lo (2 chunks)
-      const uint8_t *base_q = (mat < 2) ? qh_s + hrow * C::QH_ROW : ql_s + hrow * C::QL_ROW;
-      ldmatrix_x4(b0, b1, b2, b3, base_q + 16 * swz8(hrow, 2 * ks + (mat & 1)));
-      mma_bf16(dacc[(ks & 1) * 2], a0, a1, a2, a3, b0, b1);
-      mma_bf16(dacc[(ks & 1) * 2 + 1], a0, a1, a2, a3, b2, b3);
-    }
-#pragma unroll
-    for (int ks = W / 16; ks < (W + kRope) / 16; ++ks) {
-      uint32_t a0, a1, a2, a3;
-      {
-        const int row = 16 * mb + rr + ((mat & 1) ? 8 : 0);
-        ldmatrix_x4(a0, a1, a2, a3, st + row * C::RB + 16 * swz8(row, 2 * ks + (mat >> 1)));
-      }
-      uint32_t b0, b1;
-      ldmatrix_x2(b0, b1, qh_s + hrow * C::QH_ROW + 16 * swz8(hrow, 2 * ks + (mat & 1)));
-      mma_bf16(dacc[ks & 3], a0, a1, a2, a3, b0, b1);
-    }
-    float d[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) d[k] = (dacc[0][k] + dacc[1][k]) + (dacc[2][k] + dacc[3][k]);
-    const bool vA = base + 16 * mb + g < i1, vB = base + 16 * mb + g + 8 < i1;
-    float x[4];
-    x[0] = vA ? d[0] * sig_log2 : -INFINITY;
-    x[1] = vA ? d[1] * sig_log2 : -INFINITY;
-    x[2] = vB ? d[2] * sig_log2 : -INFINITY;
-    x[3] = vB ? d[3] * sig_log2 : -INFINITY;
-    float mt0 = fmaxf(x[0], x[2]), mt1 = fmaxf(x[1], x[3]);
-#pragma unroll
-    for (int off = 4; off < 32; off <<= 1) {
-      mt0 = fmaxf(mt0, __shfl_xor_sync(0xffffffffu, mt0, off));
-      mt1 = fmaxf(mt1, __shfl_xor_sync(0xffffffffu, mt1, off));
-    }
-    if (g == 0) {
-      tmax_s[mb * kHeads + 8 * nb + 2 * c] = mt0;
-      tmax_s[mb * kHeads + 8 * nb + 2 * c + 1] = mt1;
-    }
-    __syncthreads();
-
-    // ---- running maxima: every thread derives the same values -------------
-    float alpha[2][2];
-#pragma unroll
-    for (int n2 = 0; n2 < 2; ++n2)
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const int h = 8 * n2 + 2 * c + hh;
-        float mt = fmaxf(fmaxf(tmax_s[h], tmax_s[kHeads + h]),
-                         fmaxf(tmax_s[2 * kHeads + h], tmax_s[3 * kHeads + h]));
-        alpha[n2][hh] = 1.f;
-        if (mt > m_run[n2][hh] + 8.f) {  // lazy: keep a stale max within 2^8
-          alpha[n2][hh] = (m_run[n2][hh] == -INFINITY) ? 0.f : fast_exp2(m_run[n2][hh] - mt);
-          m_run[n2][hh] = mt;
-        }
-      }
-    // ---- weights of this warp's 16 positions -> P^T fragments -------------
-    {
-      // this warp's head block nb (selects, not indexing: no local memory)
-      const float ma = nb ? m_run[1][0] : m_run[0][0], mb2 = nb ? m_run[1][1] : m_run[0][1];
-      l_part[0] *= nb ? alpha[1][0] : alpha[0][0];
-      l_part[1] *= nb ? alpha[1][1] : alpha[0][1];
-      float p[4];
-      p[0] = (ma == -INFINITY) ? 0.f : fast_exp2(x[0] - ma);
-      p[1] = (mb2 == -INFINITY) ? 0.f : fast_exp2(x[1] - mb2);
-      p[2] = (ma == -INFINITY) ? 0.f : fast_exp2(x[2] - ma);
-      p[3] = (mb2 == -INFINITY) ? 0.f : fast_exp2(x[3] - mb2);
-      l_part[0] += p[0] + p[2];
-      l_part[1] += p[1] + p[3];
-      uint32_t ht, lt, hb, lb;
-      split2<true>(p[0], p[1], ht, lt);
-      split2<true>(p[2], p[3], hb, lb);
-      uint32_t *pf = p_s + ((mb * 2 + nb) * 4) * 32;
-      pf[0 * 32 + lane] = movmatrix_t(ht);
-      pf[1 * 32 + lane] = movmatrix_t(hb);
-      pf[2 * 32 + lane] = movmatrix_t(lt);
-      pf[3 * 32 + lane] = movmatrix_t(lb);
-    }
-    // rescale the value accumulators of this warp's units
-#pragma unroll
-    for (int u = 0; u < C::UPW; ++u) {
-      const int unit = warp + 8 * u;
-      if (unit < C::UNITS) {
-        const int un = unit & 1;
-        const float a0 = un ? alpha[1][0] : alpha[0][0], a1 = un ? alpha[1][1] : alpha[0][1];
-        acc[u][0] *= a0; acc[u][2] *= a0;
-        acc[u][1] *= a1; acc[u][3] *= a1;
-      }
-    }
-    __syncthreads();
-
-    // ---- values: O^T[16 latent x 8 heads] += C^T[16 x 64 pos] P^T -----------
-#pragma unroll
-    for (int u = 0; u < C::UPW; ++u) {
-      const int unit = warp + 8 * u;
-      if (unit < C::UNITS) {
-        const int mblk = unit >> 1, un = unit & 1;
-#pragma unroll
-        for (int kb = 0; kb < 4; ++kb) {
-          uint32_t a0, a1, a2, a3;
-          const int row = 16 * kb + rr + ((mat >> 1) ? 8 : 0);
-          ldmatrix_x4_t(a0, a1, a2, a3, st + row * C::RB + 16 * swz8(row, 2 * mblk + (mat & 1)));
-          const uint32_t *pf = p_s + ((kb * 2 + un) * 4) * 32;
-          mma_bf16(acc[u], a0, a1, a2, a3, pf[lane], pf[32 + lane]);
-          mma_bf16(acc[u], a0, a1, a2, a3, pf[64 + lane], pf[96 + lane]);
-        }
-      }
-    }
-  }
-  cp_async_wait<0>();
+  fence_proxy_async();
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tbase;
+  const uint32_t t_o = tmem, t_s = tmem + C::OCOLS;  // O columns, then two S buffers
+  auto stage = [&](int s) { return sm + s * C::STAGE; };
+  auto pbuf = [&](int ps) { return sm + C::OFF_P + ps * C::PB; };
+  bool failed = false;
 
-  // ---- row sums across the four position blocks ----------------------------
-#pragma unroll
-  for (int off = 4; off < 32; off <<= 1) {
-    l_part[0] += __shfl_xor_sync(0xffffffffu, l_part[0], off);
-    l_part[1] += __shfl_xor_sync(0xffffffffu, l_part[1], off);
-  }
-  if (g == 0) {
-    lsum_s[mb * kHeads + 8 * nb + 2 * c] = l_part[0];
-    lsum_s[mb * kHeads + 8 * nb + 2 * c + 1] = l_part[1];
-  }
-  __syncthreads();
-
-  const size_t RS = (size_t)W + 2;
-  const size_t prow0 = ((size_t)split * v.B + b) * H;
-#pragma unroll
-  for (int u = 0; u < C::UPW; ++u) {
-    const int unit = warp + 8 * u;
-    if (unit < C::UNITS) {
-      const int mblk = unit >> 1, un = unit & 1;
-      const int r0 = 16 * mblk + g;
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const int h = 8 * un + 2 * c + hh;
-        if (h < H) {
-          float *pr = partial + (prow0 + h) * RS;
-          pr[r0] = acc[u][hh];
-          pr[r0 + 8] = acc[u][2 + hh];
+  if (warp == 5) {
+    // ======================= copy warp ====================================
+    int issued = 0;
+    if (lane == 0) {
+      for (; issued < n_tiles; ++issued) {
+        const int s = issued % C::NST;
+        // the stage's previous tile was read by its values
+        if (issued >= C::NST &&
+            !mbar_wait_or_abort(&obar[s], ((issued - C::NST) / C::NST) & 1, kLimit, abort_flag)) {
+          *abort_flag = 1;
+          set_err(err, 8);
+          break;
         }
+        fence_proxy_async();
+        mbar_expect_tx(&full[s], C::STAGE);
+#pragma unroll
+        for (int j = 0; j < C::BOXES; ++j)
+          tma_load_2d(stage(s) + j * C::BOX, &tmap, 64 * j, row0 + issued * TR, &full[s]);
+      }
+      // the last copies land before the CTA leaves (bounded; done at once
+      // when they were consumed)
+      for (int u = max(0, issued - C::NST); u < issued; ++u)
+        mbar_wait(&full[u % C::NST], (u / C::NST) & 1, kLimit);
+    }
+    __syncwarp();
+  } else if (warp == 4) {
+    // ======================= MMA warp =====================================
+    constexpr uint32_t ID_S = umma_idesc(64, 32, false, false);
+    constexpr uint32_t ID_V = umma_idesc(C::MV, 32, true, true);
+    auto issue_values = [&](int t) {  // lane 0: O^T[:, hi | lo] += C^T [P_hi | P_lo]
+      tc_fence_after();
+      const uint64_t da = umma_desc(smem_u32(stage(t % C::NST)), C::BOX, 1024, 2);
+      const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, 1024, 0);
+#pragma unroll
+      for (int ks = 0; ks < TR / 16; ++ks)
+#pragma unroll
+        for (int mb = 0; mb < C::MB; ++mb)
+          umma_f16(t_o + 32 * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
+                   dp + (uint64_t)(ks * 16), ID_V, t > 0 || ks > 0);
+      umma_commit(&obar[t % C::NST]);
+    };
+    for (int t = 0; t < n_tiles && !failed; ++t) {
+      const int s = t % C::NST;
+      bool ok = mbar_wait_or_abort(&full[s], (t / C::NST) & 1, kLimit, abort_flag);
+      // rows past the split's end: zero them (the cache may hold anything)
+      const int nval = min(TR, i1 - (i0 + t * TR));
+      if (ok && nval < TR) {
+        for (int q = lane; q < C::BOXES * (TR - nval) * 8; q += 32) {
+          const int j = q / ((TR - nval) * 8), rem = q % ((TR - nval) * 8);
+          const int r = nval + rem / 8, u = rem % 8;
+          *reinterpret_cast<uint4 *>(stage(s) + j * C::BOX + r * 128 + 16 * u) = make_uint4(0, 0, 0, 0);
+        }
+        fence_proxy_async();
+        __syncwarp();
+      }
+      // the S buffer of tile t was read by softmax(t-2)
+      if (ok && t >= 2) ok = mbar_wait_or_abort(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag);
+      if (ok && lane == 0) {  // scores(t) -> S[t & 1]
+        tc_fence_after();
+        const uint64_t dc = umma_desc(smem_u32(stage(s)), 16, 1024, 2);
+        const uint64_t dq = umma_desc(smem_u32(q_s), 128, C::KH / 8 * 128, 0);
+#pragma unroll
+        for (int ks = 0; ks < C::KH / 16; ++ks)
+          umma_f16(t_s + 32 * (t & 1), dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
+                   dq + (uint64_t)(ks * 16), ID_S, ks > 0);
+        umma_commit(&sbar[t & 1]);
+      }
+      if (ok && t >= 1) {  // values(t-1) once P(t-1) is written
+        ok = mbar_wait_or_abort(&pbar[(t - 1) & 1], ((t - 1) >> 1) & 1, kLimit, abort_flag);
+        if (ok && lane == 0) issue_values(t - 1);
+      }
+      failed = !__all_sync(0xffffffffu, ok);
+    }
+    if (!failed && n_tiles > 0) {
+      const int t = n_tiles - 1;
+      const bool ok = mbar_wait_or_abort(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
+      if (ok && lane == 0) issue_values(t);
+      failed = !__all_sync(0xffffffffu, ok);
+    }
+    if (failed && lane == 0) {
+      *abort_flag = 1;
+      set_err(err, 8);
+    }
+    // every UMMA lands before the CTA leaves (bounded)
+    if (lane == 0) {
+      umma_commit(dbar);
+      mbar_wait(dbar, 0, kLimit);
+    }
+    __syncwarp();
+  } else {
+    // ======================= softmax warps ================================
+    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+    const int prow = 16 * warp + lane;  // this lane's tile position (lanes 0-15)
+    float m_run[kHeads], l_part[kHeads];
+#pragma unroll
+    for (int h = 0; h < kHeads; ++h) { m_run[h] = -1e30f; l_part[h] = 0.f; }
+    for (int t = 0; t < n_tiles; ++t) {
+      const int base = i0 + t * TR, nval = min(TR, i1 - base);
+      bool ok = mbar_wait_or_abort(&sbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
+      // P buffer (t & 1) was read by values(t-2)
+      if (ok && t >= 2)
+        ok = mbar_wait_or_abort(&obar[(t - 2) % C::NST], ((t - 2) / C::NST) & 1, kLimit, abort_flag);
+      if (softmax_sync_or(!ok)) { failed = true; break; }
+      tc_fence_after();
+      float x[kHeads];
+      {
+        float lo[16];
+        tmem_ld16(t_s + 32 * (t & 1) + lane_off, x);
+        tmem_ld16(t_s + 32 * (t & 1) + 16 + lane_off, lo);
+        const bool live = lane < 16 && prow < nval;
+#pragma unroll
+        for (int h = 0; h < kHeads; ++h) x[h] = live ? x[h] + lo[h] : -INFINITY;
+      }
+      bool need = false;
+#pragma unroll
+      for (int h = 0; h < kHeads; ++h) need |= x[h] * sig > m_run[h] + 8.f;
+      if (softmax_sync_or(need)) {
+        // new maxima: reduce over the 16 rows of each warp, then the 4 warps
+#pragma unroll
+        for (int h = 0; h < kHeads; ++h) {
+          float mx = x[h];
+#pragma unroll
+          for (int off = 1; off < 16; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+          if (lane == 0) red[warp * kHeads + h] = mx;
+        }
+        softmax_sync();
+        float alpha[kHeads];
+        bool any = false;
+#pragma unroll
+        for (int h = 0; h < kHeads; ++h) {
+          const float mt =
+              fmaxf(fmaxf(red[h], red[kHeads + h]), fmaxf(red[2 * kHeads + h], red[3 * kHeads + h])) * sig;
+          alpha[h] = 1.f;
+          if (mt > m_run[h] + 8.f) {  // stale maximum kept while within 2^8
+            alpha[h] = fast_exp2(m_run[h] - mt);
+            m_run[h] = mt;
+            any = true;
+          }
+          l_part[h] *= alpha[h];
+        }
+        if (t >= 1 && any) {
+          // O holds values up to t-1: wait for them, scale per head in TMEM
+          ok = mbar_wait_or_abort(&obar[(t - 1) % C::NST], ((t - 1) / C::NST) & 1, kLimit, abort_flag);
+          if (softmax_sync_or(!ok)) { failed = true; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int mb = 0; mb < C::MB; ++mb)
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+              float o[16];
+              tmem_ld16(t_o + 32 * mb + 16 * half + lane_off, o);
+#pragma unroll
+              for (int h = 0; h < 16; ++h) o[h] *= alpha[h];
+              tmem_st16(t_o + 32 * mb + 16 * half + lane_off, o);
+            }
+        }
+        softmax_sync();  // `red` is reused by the next vote
+      }
+      // weights hi/lo in bf16 into the MN-major P operand: position k, column
+      // n (0-15 hi, 16-31 lo) at (k/8) 128 + (n/8) 1024 + (k%8) 16 + (n%8) 2
+      if (lane < 16 && prow < TR) {
+        uint32_t hw[8], lw[8];
+#pragma unroll
+        for (int h = 0; h < kHeads; h += 2) {
+          const float p0 = fast_exp2(fmaf(x[h], sig, -m_run[h]));
+          const float p1 = fast_exp2(fmaf(x[h + 1], sig, -m_run[h + 1]));
+          l_part[h] += p0;
+          l_part[h + 1] += p1;
+          split2<true>(p0, p1, hw[h / 2], lw[h / 2]);
+        }
+        uint8_t *pp = pbuf(t & 1) + (prow / 8) * 128 + (prow % 8) * 16;
+        *reinterpret_cast<uint4 *>(pp) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *reinterpret_cast<uint4 *>(pp + 1024) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+        *reinterpret_cast<uint4 *>(pp + 2048) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        *reinterpret_cast<uint4 *>(pp + 3072) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&pbar[t & 1]);  // one of the four arrivals
+    }
+    // ---- partial of this split: O^T columns h + 16+h, m, l ------------------
+    if (!failed && n_tiles > 0) {
+      const int t = n_tiles - 1;
+      const bool ok = mbar_wait_or_abort(&obar[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag);
+      failed = softmax_sync_or(!ok);
+    }
+    if (failed && tid == 0) {
+      *abort_flag = 1;
+      set_err(err, 8);
+    }
+    if (!failed) {
+      tc_fence_after();
+      const size_t RS = (size_t)W + 2;
+      const size_t prow_base = ((size_t)split * v.B + b) * H;
+#pragma unroll
+      for (int h = 0; h < kHeads; ++h) {
+        float sum = l_part[h];
+#pragma unroll
+        for (int off = 1; off < 16; off <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+        if (lane == 0) lsum[warp * kHeads + h] = sum;
+      }
+#pragma unroll
+      for (int mb = 0; mb < C::MB; ++mb) {
+        float o[16];
+        if (n_tiles > 0) {
+          float lo[16];
+          tmem_ld16(t_o + 32 * mb + lane_off, o);
+          tmem_ld16(t_o + 32 * mb + 16 + lane_off, lo);
+#pragma unroll
+          for (int h = 0; h < 16; ++h) o[h] += lo[h];
+        } else {
+#pragma unroll
+          for (int h = 0; h < 16; ++h) o[h] = 0.f;
+        }
+        // latent row of this lane: M=128 blocks use every lane; the M=64
+        // block (W = 64) holds row 16 warp + lane in lanes 0-15
+        const int r = C::MV == 128 ? 128 * mb + 32 * warp + lane : 16 * warp + lane;
+        if (C::MV == 128 || lane < 16) {
+#pragma unroll
+          for (int h = 0; h < kHeads; ++h)
+            if (h < H) partial[(prow_base + h) * RS + r] = o[h];
+        }
+      }
+      softmax_sync();
+      if (tid < H) {
+        const float L = lsum[tid] + lsum[kHeads + tid] + lsum[2 * kHeads + tid] + lsum[3 * kHeads + tid];
+        float mh = m_run[0];
+#pragma unroll
+        for (int h = 1; h < kHeads; ++h) mh = (tid == h) ? m_run[h] : mh;
+        float *pr = partial + (prow_base + tid) * RS;
+        pr[W] = (L > 0.f) ? mh : -INFINITY;
+        pr[W + 1] = L;
       }
     }
   }
-  // publish m and l: lane (g == 0, c) of warp 0 holds m for heads 2c+hh and
-  // 8+2c+hh (all threads agree on m_run).
-  if (warp == 0 && g == 0) {
-#pragma unroll
-    for (int n2 = 0; n2 < 2; ++n2)
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const int h = 8 * n2 + 2 * c + hh;
-        if (h < H) {
-          float *pr = partial + (prow0 + h) * RS;
-          pr[W] = m_run[n2][hh];
-          pr[W + 1] = lsum_s[h] + lsum_s[kHeads + h] + lsum_s[2 * kHeads + h] +
-                      lsum_s[3 * kHeads + h];
-        }
-      }
-  }
-  (void)err;
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TCOLS)
+                 : "memory");
 }
 
 // ---------------------------------------------------------------------------
@@ -511,10 +712,10 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  k<<<dim3(a.n_splits, B), 256, C::SMEM, st>>>(a.v, a.qlat,
-                                                static_cast<const uint16_t *>(a.q_pe), a.H,
-                                                a.sig_log2, a.items_per_split,
-                                                a.n_splits, a.partial, a.err);
+  k<<<dim3(a.n_splits, B), 192, C::SMEM, st>>>(*static_cast<const CUtensorMap *>(a.tmap), a.v,
+                                                a.qlat, static_cast<const uint16_t *>(a.q_pe),
+                                                a.H, a.sig_log2, a.items_per_split, a.n_splits,
+                                                a.partial, a.err);
   constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
   static bool mu_attr = false;
   if (!mu_attr) {
@@ -534,13 +735,45 @@ int mla_ctas_t() {
   auto k = mla_decode_kernel<W>;
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 256, C::SMEM) != cudaSuccess) n = 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 192, C::SMEM) != cudaSuccess) n = 1;
   return n > 0 ? n : 1;
 }
 
 }  // namespace
 
+// Tensor map of an MLA anchor's records for the decode kernel: a 2-D view
+// [B cap rows x (width + rope) bf16], boxes of 64 x 64 with the 128-byte
+// swizzle (the UMMA operand layout).  The encoder is the driver's
+// cuTensorMapEncodeTiled, reached through the runtime's entry-point query so
+// the library links the static runtime only.
+cudaError_t mla_make_tmap(void *out, const MlaView &v) {
+  using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                              const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                              const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                              CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+  static Encode encode = nullptr;
+  if (!encode) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    const cudaError_t e =
+        cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess) return e;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+    encode = reinterpret_cast<Encode>(fn);
+  }
+  const cuuint64_t dims[2] = {(cuuint64_t)(v.width + v.rope), (cuuint64_t)v.B * (cuuint64_t)v.cap};
+  const cuuint64_t strides[1] = {(cuuint64_t)v.rec_bytes};
+  const cuuint32_t box[2] = {64, (cuuint32_t)mla_tile_rows(v.width)};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = encode(static_cast<CUtensorMap *>(out), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                            v.rec, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st) {
+  if (!a.tmap) return cudaErrorInvalidValue;
   switch (a.v.width) {
     case 512: return launch_mla_t<512>(a, st);
     case 256: return launch_mla_t<256>(a, st);
