@@ -302,19 +302,19 @@ __global__ void __launch_bounds__(192, 1)
   {
     constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (unused 64) | lo(W)]
     const uint16_t *qb = qlat + (size_t)b * H * QROW;
-    for (int q = tid; q < 32 * (C::KH / 8); q += 192) {
+    for (int q = tid; q < 32 * (C::KH / 8); q += 192) {  // 16-byte cp.async, zero-filled
       const int n = q / (C::KH / 8), c = q % (C::KH / 8);
       const int h = n & 15;
-      uint4 x = make_uint4(0, 0, 0, 0);
-      if (h < H) {
-        if (n < 16)
-          x = *reinterpret_cast<const uint4 *>(c < W / 8 ? qb + (size_t)h * QROW + 8 * c
-                                                         : q_pe + ((size_t)b * H + h) * kRope + 8 * (c - W / 8));
-        else if (c < W / 8)
-          x = *reinterpret_cast<const uint4 *>(qb + (size_t)h * QROW + C::KH + 8 * c);
-      }
-      *reinterpret_cast<uint4 *>(q_s + (n / 8) * (C::KH / 8 * 128) + c * 128 + (n % 8) * 16) = x;
+      const uint16_t *src = qb;
+      const bool valid = h < H && (n < 16 || c < W / 8);
+      if (valid)
+        src = n >= 16     ? qb + (size_t)h * QROW + C::KH + 8 * c
+              : c < W / 8 ? qb + (size_t)h * QROW + 8 * c
+                          : q_pe + ((size_t)b * H + h) * kRope + 8 * (c - W / 8);
+      cp_async16(q_s + (n / 8) * (C::KH / 8 * 128) + c * 128 + (n % 8) * 16, src, valid);
     }
+    cp_async_commit();
+    cp_async_wait<0>();
   }
   fence_proxy_async();
   tc_fence_before();
