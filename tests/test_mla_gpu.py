@@ -75,3 +75,29 @@ def test_mla_depth_sharing_and_batch_over_64():
     ref = oatt.mla_decode_unabsorbed(f32(qn[sel]), f32(qp[sel]), f32(c[sel]), f32(kr[sel]), f32(wk),
                                      f32(wv), 256, [100] * 4, sigma)
     assert_close(f32(a[sel]), ref, what="mla B=70")
+
+
+@pytest.mark.parametrize("width", [512, 64])
+def test_mla_fewer_heads_empty_sequence_many_splits(width):
+    """H < 16 (padded head rows of the tensor-core operands), a sequence with
+    no positions (its output is 0), a 1-position sequence, and more splits
+    than tiles (empty splits merge away)."""
+    B, r, H = 3, 512, 5
+    lens = np.array([0, 1, 200])
+    c_ = _mla_cache(B, 256, [width], H=H, max_splits=16)
+    c, kr = _inputs(B, 200, r, 40 + width)
+    c_.append(0, c.cuda(), kr.cuda(), n_per_seq=torch.tensor(lens, dtype=torch.int32, device="cuda"))
+    wk, wv = _weights(H, r, 13)
+    g = torch.Generator().manual_seed(17)
+    qn = torch.randn((B, H, 128), generator=g).to(torch.bfloat16)
+    qp = torch.randn((B, H, 64), generator=g).to(torch.bfloat16)
+    sigma = 1.0 / math.sqrt(128 + 64)
+    sel = [1, 2]
+    ref = oatt.mla_decode_unabsorbed(f32(qn[sel]), f32(qp[sel]), f32(c[sel]), f32(kr[sel]), f32(wk),
+                                     f32(wv), width, lens[sel], sigma)
+    for ns in (0, 7, 16):
+        out = c_.decode_mla(0, qn.cuda(), qp.cuda(), wk.cuda(), wv.cuda(), sigma, n_splits=ns)
+        assert torch.isfinite(out).all()
+        assert (out[0] == 0).all()
+        assert_close(f32(out[sel]), ref, what=f"mla H=5 d={width} splits={ns}")
+    assert c_.device_error() == 0
