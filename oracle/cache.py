@@ -19,21 +19,28 @@ from . import quant
 from .attention import gqa_decode, resolve_sources
 
 
-def anchor_state(k, v, lens, bits, group=None, key_axis="token", value_axis="token"):
+def anchor_state(k, v, lens, bits, group=None, key_axis="token", value_axis="token",
+                 scheme="grouped"):
     """Stored and dequantised state of one GQA anchor.
 
     k, v : ``[B, H_kv, T, D]`` values as written (float32-exact)
     lens : ``[B]`` tokens written per sequence
+    scheme : ``"grouped"`` (asymmetric, scale and zero per group) or
+             ``"symmetric"`` (the paper's per-vector quantiser: one bf16
+             scale per token-head row of keys and of values, Appendix C.3)
     Returns a dict with ``k_hat``/``v_hat`` (float64, zero past ``lens``) and,
     for quantised layers, the stored ``k_codes``, ``k_scale``, ``k_zero``,
     ``v_codes``, ``v_scale``, ``v_zero`` and (per-channel keys)
     ``k_residual``; per-channel entries are lists indexed by sequence because
-    each sequence's group count depends on its own length.
+    each sequence's group count depends on its own length.  The symmetric
+    scheme stores signed ``k_codes``/``v_codes`` and ``k_scale``/``v_scale``
+    of shape ``[B, H_kv, T]``, no zeros.
     """
     k = np.asarray(k, np.float32)
     v = np.asarray(v, np.float32)
     B, H, T, D = k.shape
-    st = {"bits": bits, "group": group, "key_axis": key_axis, "value_axis": value_axis}
+    st = {"bits": bits, "group": group, "key_axis": key_axis, "value_axis": value_axis,
+          "scheme": scheme}
     k_hat = np.zeros(k.shape, np.float64)
     v_hat = np.zeros(v.shape, np.float64)
     if bits == 16:
@@ -43,6 +50,19 @@ def anchor_state(k, v, lens, bits, group=None, key_axis="token", value_axis="tok
             v_hat[b, :, :n] = v[b, :, :n]
         st.update(k_hat=k_hat, v_hat=v_hat)
         return st
+    if scheme == "symmetric":
+        kc, ks = quant.quantise_symmetric(k, bits)
+        vc, vs = quant.quantise_symmetric(v, bits)
+        kh = quant.dequantise_symmetric(kc, ks)
+        vh = quant.dequantise_symmetric(vc, vs)
+        for b in range(B):
+            n = int(lens[b])
+            k_hat[b, :, :n] = kh[b, :, :n]
+            v_hat[b, :, :n] = vh[b, :, :n]
+        st.update(k_codes=kc, k_scale=ks, v_codes=vc, v_scale=vs, k_hat=k_hat, v_hat=v_hat)
+        return st
+    if scheme != "grouped":
+        raise ValueError(f"unknown quantisation scheme {scheme!r}")
     if value_axis != "token":
         raise ValueError("values are quantised per token")
     vc, vs, vz = quant.quantise_per_token(v, bits, group)

@@ -28,9 +28,20 @@ full-precision window).
 
 Symmetric per-vector quantiser
 ------------------------------
-Appendix C.3, the scheme the paper trains with: ``q = 2^(b-1) - 1``,
+Appendix C.3, the scheme the paper trains with: one scale per stored vector
+(a 128-element token-head row), no zero point, ``q = 2^(b-1) - 1``,
 ``s = max|x| / q``, ``code = clip(round(x / s), -q, q)``, dequantise as
-``code * s``.  Same float32 op discipline; half-to-even rounding.
+``code * s``.  The caption of Tab. realized_bits fixes the stored scale as
+one bf16 per row; the paper does not say whether the codes are computed
+with the scale before or after that rounding.  The reading used here (and by
+the CUDA path) computes them with the stored scale, so that dequantisation
+uses exactly the scale the codes were made for:
+
+    s32  = f32( max|x| / q )            one binary32 division
+    s    = bf16(s32)                    round to nearest even
+    code = clip( rint( f32(x / s) ), -q, q )
+
+A zero vector stores scale 0 and codes 0.
 """
 from __future__ import annotations
 
@@ -124,22 +135,42 @@ def dequantise_per_channel(codes, scale, zero, group: int, residual=None) -> np.
     return out
 
 
+def round_bf16(x) -> np.ndarray:
+    """float32 -> nearest bfloat16 (ties to even), returned as float32.
+
+    Integer arithmetic on the binary32 pattern: adding 0x7FFF plus the lowest
+    kept bit and truncating the low 16 bits rounds to nearest, ties to even,
+    for every finite value (subnormals included)."""
+    u = np.asarray(x, dtype=F32).view(np.uint32).astype(np.uint64)
+    r = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
+    return r.astype(np.uint32).view(F32)
+
+
+def sym_levels(bits: int) -> int:
+    """q = 2^(b-1) - 1 of the symmetric quantiser (b = 2, 4 or 8)."""
+    if bits not in (2, 4, 8):
+        raise ValueError(f"symmetric quantiser supports 2, 4 or 8 bits, got {bits}")
+    return (1 << (bits - 1)) - 1
+
+
 def quantise_symmetric(x: np.ndarray, bits: int):
     """Paper's symmetric per-vector quantiser along the last axis.
 
     Returns ``(codes int8, scale f32)``; ``codes`` lie in ``[-q, q]`` with
-    ``q = 2^(bits-1) - 1``.  A zero vector stores scale 0 and codes 0.
+    ``q = 2^(bits-1) - 1``; ``scale`` holds bf16 values (the stored scale).
+    A zero vector stores scale 0 and codes 0.
     """
     x = np.asarray(x, dtype=F32)
-    q = F32((1 << (bits - 1)) - 1)
+    q = F32(sym_levels(bits))
     amax = np.abs(x).max(axis=-1)
-    s = (amax / q).astype(F32)
+    s = round_bf16((amax / q).astype(F32))       # one f32 division, then bf16
     safe = np.where(s == 0, F32(1), s).astype(F32)
-    r = (x / safe[..., None]).astype(F32)
+    r = (x / safe[..., None]).astype(F32)         # one f32 division
     codes = np.clip(np.rint(r), -q, q)
     codes = np.where(s[..., None] == 0, F32(0), codes)
     return codes.astype(np.int8), s
 
 
 def dequantise_symmetric(codes, scale) -> np.ndarray:
+    """float64 ``code * scale`` (one scale per vector of the last axis)."""
     return np.asarray(codes, np.float64) * np.asarray(scale, np.float64)[..., None]

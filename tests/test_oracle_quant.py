@@ -110,3 +110,97 @@ def test_symmetric_two_bits_has_three_levels():
     assert (np.abs(c4[np.arange(100), i]) == 7).all()
     err = np.abs(quant.dequantise_symmetric(c4, s4) - x).max(1)
     assert (err <= 0.5 * s4 + 1e-6).all()
+
+
+def test_round_bf16_matches_torch():
+    # the bit-pattern rounding against torch's own float32 -> bfloat16
+    # conversion (round to nearest even), on random values, exact ties with
+    # an even and an odd kept bit, subnormals and large magnitudes
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(5)
+    u = rng.integers(0, 0x7F000000, 20000, dtype=np.uint64).astype(np.uint32)
+    ties = (rng.integers(0, 0x7F00, 2000, dtype=np.uint64).astype(np.uint32) << 16) | 0x8000
+    sub = rng.integers(1, 0x007FFFFF, 2000, dtype=np.uint64).astype(np.uint32)
+    bits = np.concatenate([u, ties, sub])
+    x = np.concatenate([bits, bits | 0x80000000]).view(F32)
+    ref = torch.from_numpy(x.copy()).to(torch.bfloat16).float().numpy()
+    got = quant.round_bf16(x)
+    assert (got.view(np.uint32) == ref.view(np.uint32)).all()
+
+
+def _round_binary(v, p):
+    """Nearest binary floating-point value with p significant bits to the
+    exact rational v (ties to even), as a Fraction; normal range only."""
+    from fractions import Fraction
+    if v == 0:
+        return Fraction(0)
+    sign = -1 if v < 0 else 1
+    a = abs(v)
+    e = 0
+    while a >= 2:
+        a /= 2
+        e += 1
+    while a < 1:
+        a *= 2
+        e -= 1
+    m = a * (1 << (p - 1))                  # in [2^(p-1), 2^p)
+    n = round(m)                            # Fraction.__round__: ties to even
+    return sign * Fraction(n, 1 << (p - 1)) * (Fraction(2) ** e)
+
+
+def _brute_symmetric(vals, bits):
+    # exact rationals, each binary32 step rounded to 24 bits, the scale to 8
+    from fractions import Fraction
+    q = (1 << (bits - 1)) - 1
+    xs = [Fraction(float(F32(v))) for v in vals]
+    amax = max(abs(x) for x in xs)
+    if amax == 0:
+        return [0] * len(xs), 0.0
+    s = _round_binary(_round_binary(amax / q, 24), 8)
+    codes = [int(max(-q, min(q, round(_round_binary(x / s, 24))))) for x in xs]
+    return codes, float(s)
+
+
+@pytest.mark.parametrize("bits", [2, 4, 8])
+def test_symmetric_brute_force(bits):
+    rng = np.random.default_rng(40 + bits)
+    for trial in range(40):
+        n = int(rng.integers(1, 9))
+        x = (rng.standard_normal(n) * 2.0 ** rng.integers(-6, 6)).astype(F32)
+        if trial % 5 == 0:
+            x = np.round(x * 4) / 4           # dyadic values: exact ties occur
+        c, s = quant.quantise_symmetric(x, bits)
+        bc, bs = _brute_symmetric(x, bits)
+        assert c.tolist() == bc and float(s) == bs, (x, c, s, bc, bs)
+
+
+def test_symmetric_worked_examples():
+    # b = 2 (q = 1): max|x| = 1 gives s = 1, codes rint(x)
+    c, s = quant.quantise_symmetric(np.array([1.0, -0.4, 0.6, 0.2], F32), 2)
+    assert float(s) == 1.0 and c.tolist() == [1, 0, 1, 0]
+    # b = 4 (q = 7), s = 1: rint is half to even (-3.5 -> -4, 2.5 -> 2)
+    c, s = quant.quantise_symmetric(np.array([7.0, -3.5, 2.5, 0.49], F32), 4)
+    assert float(s) == 1.0 and c.tolist() == [7, -4, 2, 0]
+    # b = 4, max|x| = 1: 1/7 stored in bf16 is 0.142578125 (8 significant
+    # bits, rounded down), and 0.5 / 0.142578125 = 3.507 -> 4; with the
+    # unrounded float32 scale the same element would give 3
+    c, s = quant.quantise_symmetric(np.array([1.0, 0.5], F32), 4)
+    assert float(s) == 0.142578125 and c.tolist() == [7, 4]
+    # a zero vector stores scale 0 and codes 0
+    c, s = quant.quantise_symmetric(np.zeros(128, F32), 8)
+    assert float(s) == 0.0 and (c == 0).all()
+
+
+def test_symmetric_anchor_state():
+    from oracle import cache as ocache
+    rng = np.random.default_rng(9)
+    k = rng.standard_normal((2, 3, 10, 128)).astype(F32)
+    v = rng.standard_normal((2, 3, 10, 128)).astype(F32)
+    lens = [10, 4]
+    st = ocache.anchor_state(k, v, lens, 4, scheme="symmetric")
+    assert st["k_codes"].dtype == np.int8 and st["k_scale"].shape == (2, 3, 10)
+    for b, n in enumerate(lens):
+        for x, name in ((k, "k"), (v, "v")):
+            err = np.abs(st[name + "_hat"][b, :, :n] - x[b, :, :n]).max(-1)
+            assert (err <= 0.5 * st[name + "_scale"][b, :, :n] + 1e-6).all()
+            assert (st[name + "_hat"][b, :, n:] == 0).all()
