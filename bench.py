@@ -55,7 +55,12 @@ def algorithmic_bytes(w, lens_after_append):
     per_layer = []
     for l in range(w.n_layers):
         a = w.layers[src[l]]
-        rec = 4 * D if a["bits"] == 16 else 2 * D * a["bits"] // 8 + 2 * 8 * D // a["group"]
+        if a["bits"] == 16:
+            rec = 4 * D
+        elif a.get("scheme") == "symmetric":
+            rec = 2 * D * a["bits"] // 8 + 2 * 2      # codes + two bf16 scales
+        else:
+            rec = 2 * D * a["bits"] // 8 + 2 * 8 * D // a["group"]
         n = w.keep if w.keep else lens_after_append
         cache = B * H * n * rec
         qo = B * w.n_q_heads * D * (2 + 4)
@@ -172,6 +177,8 @@ def cpu_baseline(w, seconds=12.0):
         q = W.queries(w, a)[0, :G].float().numpy()
         if bits == 16:
             units.append((bits, q, kk, vv, None))
+        elif w.layers[a].get("scheme") == "symmetric":
+            units.append((bits, q, oq.quantise_symmetric(kk, bits), oq.quantise_symmetric(vv, bits), 0))
         else:
             g = w.layers[a]["group"]
             units.append((bits, q, oq.quantise_per_token(kk, bits, g), oq.quantise_per_token(vv, bits, g), g))
@@ -183,6 +190,10 @@ def cpu_baseline(w, seconds=12.0):
             if bits == 16:
                 kh, vh = kq, vq
                 nbytes += T * 4 * D
+            elif g == 0:  # symmetric: codes + one bf16 scale per row
+                kh = oq.dequantise_symmetric(*kq)
+                vh = oq.dequantise_symmetric(*vq)
+                nbytes += T * (2 * D * bits // 8 + 4)
             else:
                 kh = oq.dequantise_per_token(*kq, g)
                 vh = oq.dequantise_per_token(*vq, g)
@@ -204,7 +215,7 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2609_37988_gb300 import workloads as W
-    w = W.config(args.config)
+    w = W.config(args.config, sym_bits=args.sym_bits)
     per = max(2.0, 60.0 / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):
         cpu_baseline(w, seconds=min(per, 3.0))
@@ -227,8 +238,10 @@ def run_reference(args):
 def _layer_kind(w, l, src):
     if w.kind == "mla":
         return f"mla_d{w.layers[l]['width']}"
-    a = src[l]
-    return "bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}"
+    a = w.layers[src[l]]
+    if a["bits"] == 16:
+        return "bf16"
+    return f"{'sym' if a.get('scheme') == 'symmetric' else 'int'}{a['bits']}"
 
 
 def kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer, src, layer_call, dev,
@@ -319,7 +332,10 @@ def main():
     ap.add_argument("--impl", default="kvk")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--profile-case", choices=["gqa", "mla", "gather"], default=None,
+    ap.add_argument("--sym-bits", type=int, choices=[8, 4, 2], default=None,
+                    help="store the quantised anchors with the symmetric per-vector "
+                         "quantiser at this bit-width")
+    ap.add_argument("--profile-case", choices=["gqa", "mla", "gather", "sym"], default=None,
                     help="small ncu case: decode launches only, no timing line")
     args = ap.parse_args()
     if args.impl == "reference":
@@ -345,7 +361,7 @@ def main():
     from paper_2609_37988_gb300 import workloads as W
     from paper_2609_37988_gb300.cache import Cache, Layer
 
-    w = W.config(args.config)
+    w = W.config(args.config, sym_bits=args.sym_bits)
     T = w.context
     src = w.sources()
     new_kv = {}
@@ -524,14 +540,12 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms_step, "us_per_step": ms_step * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": ("bf16" if w.kind == "mla" else
-                      "/".join(sorted({("bf16" if w.layers[a]["bits"] == 16 else f"int{w.layers[a]['bits']}")
-                                       for a in w.anchors}))),
+                      "/".join(sorted({_layer_kind(w, a, src) for a in w.anchors}))),
             "data": "synthetic",
             "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "context": T,
                        "q_heads": w.n_q_heads, "kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
-                       "anchors": {"bf16": sum(1 for a in w.anchors if w.layers[a]["bits"] == 16),
-                                   "int4": sum(1 for a in w.anchors if w.layers[a]["bits"] == 4),
-                                   "int8": sum(1 for a in w.anchors if w.layers[a]["bits"] == 8)},
+                       "anchors": {k: sum(1 for a in w.anchors if _layer_kind(w, a, src) == k)
+                                   for k in sorted({_layer_kind(w, a, src) for a in w.anchors})},
                        "inheritors": w.n_layers - len(w.anchors),
                        "bytes_per_step": step_bytes, "cuda_graph": True,
                        "l2": (f"no flush; smallest per-layer read {min(per_layer) / 1e6:.0f} MB vs 126 MB L2"
@@ -561,7 +575,9 @@ def profile_case(kind):
     cache, both anchors larger than L2); each decode runs 3 times in the order
     int4, bf16.  mla: one d=512 latent layer at B=64, T=4096 (302 MB).
     gather: one int4 g32 anchor at B=4, T=131072 with a kept list of T/8
-    positions per sequence (805 MB cache, 101 MB read per decode), 3 decodes."""
+    positions per sequence (805 MB cache, 101 MB read per decode), 3 decodes.
+    sym: one symmetric anchor of each bit-width (8, 4, 2) at the 14B step
+    shape (2.2 GB of cache), each decoded 3 times."""
     import torch
     from __graft_entry__ import build
     build()
@@ -580,6 +596,20 @@ def profile_case(kind):
         q = W.queries(w, 0, device="cuda")
         for _ in range(3):
             for l in range(2):
+                c.decode(l, q, w.sigma)
+    elif kind == "sym":
+        # one anchor of each symmetric bit-width at the 14B step shape
+        w = W.config(3)
+        layers = [Layer(bits=b, scheme="symmetric") for b in (8, 4, 2)]
+        c = Cache(n_layers=3, n_q_heads=40, n_kv_heads=8, head_dim=128, max_batch=32,
+                  max_ctx=8192, layers=layers)
+        for l in range(3):
+            k, v = W.kv_inputs(w, l, 0, 8192, device="cuda")
+            c.append(l, k, v)
+            del k, v
+        q = W.queries(w, 0, device="cuda")
+        for _ in range(3):
+            for l in range(3):
                 c.decode(l, q, w.sigma)
     elif kind == "gather":
         import numpy as np

@@ -7,9 +7,11 @@
  *
  *   depth      a layer owns a cache (an "anchor") or inherits the nearest
  *              anchor before it and reads it with its own query (Sec. 2.1);
- *   precision  a cache is stored at 16, 8 or 4 bits (Sec. 2.1; grouped
- *              asymmetric quantiser of Appendix C.3 with a scale and a zero
- *              point per group);
+ *   precision  a cache is stored at 16, 8, 4 or 2 bits (Sec. 2.1) with
+ *              either quantiser of Appendix C.3: the grouped asymmetric one
+ *              (a scale and a zero point per group of channels or
+ *              positions) or the paper's symmetric per-vector one (one bf16
+ *              scale per token-head row, codes in [-q, q], q = 2^(b-1) - 1);
  *   rank       an MLA latent truncated to its first d coordinates plus the
  *              post-RoPE positional key (Sec. 2.1, Appendix C.2).
  *
@@ -60,6 +62,7 @@ typedef enum {
 
 enum { KVK_KIND_GQA = 0, KVK_KIND_MLA = 1 };
 enum { KVK_AXIS_TOKEN = 0, KVK_AXIS_CHANNEL = 1 };
+enum { KVK_QUANT_GROUPED = 0, KVK_QUANT_SYMMETRIC = 1 };
 enum { KVK_DTYPE_F32 = 0, KVK_DTYPE_BF16 = 1 };
 
 /* Device error word values (kvk_get_device_error). */
@@ -88,11 +91,18 @@ typedef struct {
 } kvk_model_desc;
 
 /* One plan action (Sec. 2.2).  inherit=1 is the depth action; otherwise the
- * layer owns a cache at `bits` (16 = bf16, 8 or 4 = grouped quantiser with
- * `group` elements per scale/zero pair) and, for MLA, keeps the first
- * `width` latent coordinates (truncate on write, Appendix C.2).  key_axis
- * selects per-token groups (g channels of one token) or per-channel groups
- * (g positions of one channel, KIVI keys); values are per-token.
+ * layer owns a cache at `bits` (16 = bf16; 8, 4 or 2 = quantised codes) and,
+ * for MLA, keeps the first `width` latent coordinates (truncate on write,
+ * Appendix C.2).
+ *  scheme KVK_QUANT_GROUPED: `group` elements per fp32 (scale, zero) pair;
+ *    key_axis selects per-token groups (g channels of one token) or
+ *    per-channel groups (g positions of one channel, KIVI keys); values are
+ *    per-token.  This build: bits 8 or 4, group 32 or 64.
+ *  scheme KVK_QUANT_SYMMETRIC: the paper's quantiser (Appendix C.3): one
+ *    bf16 scale s = max|x| / q per token-head row of keys and of values,
+ *    codes clip(rint(x / s), -q, q) with q = 2^(b-1) - 1 (three levels at
+ *    two bits), x = code * s; `group` is ignored and both axes must be
+ *    KVK_AXIS_TOKEN.  This build: GQA, head_dim 128, bits 8, 4 or 2.
  * evict_capacity > 0 reserves a kept-position list of that length per
  * sequence (eviction composed with compression, Sec. 3.3). */
 typedef struct {
@@ -103,6 +113,7 @@ typedef struct {
   int32_t value_axis;
   int32_t width;
   int32_t evict_capacity;
+  int32_t scheme;      /* KVK_QUANT_GROUPED or KVK_QUANT_SYMMETRIC */
 } kvk_layer_cfg;
 
 typedef struct kvk_cache kvk_cache;
@@ -110,9 +121,11 @@ typedef struct kvk_cache kvk_cache;
 /* Validate a plan and report the device bytes each layer's arena needs
  * (0 for inheritors).  arena_bytes: host array of n_layers entries.
  * Errors: INVALID_ARG, INVALID_CONFIG (layer 0 inherits, bits not in
- * {16,8,4}, group not dividing head_dim, MLA width not in r/8..r), and
- * UNSUPPORTED for valid plans outside this build (2-bit codes, per-channel
- * values, head_dim other than 64/128, per-channel keys with eviction). */
+ * {16,8,4,2}, unknown scheme, group not dividing head_dim for the grouped
+ * scheme, a per-channel axis with the symmetric scheme, MLA width not in
+ * r/8..r), and UNSUPPORTED for valid plans outside this build (grouped 2-bit
+ * codes, per-channel values, head_dim other than 64/128, the symmetric
+ * scheme with head_dim 64 or on MLA, per-channel keys with eviction). */
 kvk_status kvk_cache_plan(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
                           size_t *arena_bytes);
 
@@ -248,7 +261,8 @@ kvk_status kvk_splitk_reduce(const float *partials, int32_t n_splits, int32_t n_
 /* Cost accounting of the cache's plan.
  *  bits_per_token_model: sum over layers of eq. (cost), in bits per token;
  *  bytes_per_token_stored: bytes this build stores per token, summed over
- *      anchors, including fp32 scale/zero metadata (Tab. realized_bits
+ *      anchors, including the quantisers' metadata (fp32 scale/zero pairs,
+ *      or two bf16 scales per row for the symmetric scheme; Tab. realized_bits
  *      counts metadata the same way);
  *  rho: eq. (compression) against the bf16 GQA cache of the same geometry
  *      (for MLA, n_kv_heads * head_dim = latent_dim is used as C0's width,
@@ -272,6 +286,9 @@ kvk_status kvk_plan_cost(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
  *              per-channel keys: k_scale, k_zero float [B, H_kv, T/g, D] and
  *              k_residual bf16 [B, H_kv, g, D] (positions of the open group,
  *              row = position mod g).
+ *  symmetric:  k_out, v_out int8 codes in [-q, q] [B, H_kv, T, D];
+ *              k_scale, v_scale float [B, H_kv, T] (the stored bf16 scales,
+ *              widened); k_zero, v_zero, k_residual unused.
  *  MLA:        k_out bf16 [B, T, width] latent, v_out bf16 [B, T, rope_dim].
  * Any pointer the format does not use may be NULL. */
 kvk_status kvk_export_layer(const kvk_cache *cache, int32_t layer, void *k_out, void *v_out,

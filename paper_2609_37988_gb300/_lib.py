@@ -20,6 +20,7 @@ STATUS_NAMES = {
 }
 KIND_GQA, KIND_MLA = 0, 1
 AXIS_TOKEN, AXIS_CHANNEL = 0, 1
+QUANT_GROUPED, QUANT_SYMMETRIC = 0, 1
 DTYPE_F32, DTYPE_BF16 = 0, 1
 
 
@@ -31,7 +32,8 @@ class ModelDesc(ctypes.Structure):
 
 class LayerCfg(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
-        "inherit", "bits", "group", "key_axis", "value_axis", "width", "evict_capacity")]
+        "inherit", "bits", "group", "key_axis", "value_axis", "width", "evict_capacity",
+        "scheme")]
 
 
 class KVKError(RuntimeError):

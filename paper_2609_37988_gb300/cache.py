@@ -14,7 +14,7 @@ import torch
 
 from . import _lib
 from ._lib import (AXIS_CHANNEL, AXIS_TOKEN, DTYPE_BF16, DTYPE_F32, KIND_GQA, KIND_MLA,
-                   KVKError, LayerCfg, ModelDesc, check, load)
+                   QUANT_GROUPED, QUANT_SYMMETRIC, KVKError, LayerCfg, ModelDesc, check, load)
 
 __all__ = ["Layer", "Cache", "splitk_reduce", "KVKError"]
 
@@ -22,20 +22,25 @@ __all__ = ["Layer", "Cache", "splitk_reduce", "KVKError"]
 @dataclass
 class Layer:
     """One plan action.  ``inherit=True`` is the depth action; otherwise a
-    cache at ``bits`` (16, 8, 4) with quantisation ``group`` and key axis
-    ``"token"``/``"channel"``, MLA kept ``width``, optional eviction list
-    capacity."""
+    cache at ``bits`` (16, 8, 4, 2) quantised with ``scheme`` ``"grouped"``
+    (asymmetric, ``group`` elements per scale/zero pair, key axis
+    ``"token"``/``"channel"``) or ``"symmetric"`` (one bf16 scale per
+    token-head row), MLA kept ``width``, optional eviction list capacity."""
     inherit: bool = False
     bits: int = 16
     group: int = 64
     key_axis: str = "token"
     width: int = 0
     evict_capacity: int = 0
+    scheme: str = "grouped"
 
     def to_c(self) -> LayerCfg:
+        if self.scheme not in ("grouped", "symmetric"):
+            raise ValueError(f"unknown quantisation scheme {self.scheme!r}")
         return LayerCfg(int(self.inherit), self.bits, self.group,
                         AXIS_CHANNEL if self.key_axis == "channel" else AXIS_TOKEN,
-                        AXIS_TOKEN, self.width, self.evict_capacity)
+                        AXIS_TOKEN, self.width, self.evict_capacity,
+                        QUANT_SYMMETRIC if self.scheme == "symmetric" else QUANT_GROUPED)
 
 
 def _ptr(t):
@@ -204,6 +209,15 @@ class Cache:
             res["v"] = torch.empty((B, H, T, D), dtype=torch.bfloat16, device=dev)
             check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["k"]), _ptr(res["v"]),
                                             None, None, None, None, None, _stream(stream)))
+            return res
+        if L.scheme == "symmetric":
+            res["k_codes"] = torch.empty((B, H, T, D), dtype=torch.int8, device=dev)
+            res["v_codes"] = torch.empty((B, H, T, D), dtype=torch.int8, device=dev)
+            res["k_scale"] = torch.empty((B, H, T), dtype=torch.float32, device=dev)
+            res["v_scale"] = torch.empty((B, H, T), dtype=torch.float32, device=dev)
+            check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["k_codes"]),
+                                            _ptr(res["v_codes"]), _ptr(res["k_scale"]), None,
+                                            _ptr(res["v_scale"]), None, None, _stream(stream)))
             return res
         g = L.group
         res["k_codes"] = torch.empty((B, H, T, D), dtype=torch.uint8, device=dev)

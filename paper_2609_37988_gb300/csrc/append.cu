@@ -67,6 +67,64 @@ __device__ __forceinline__ void quant_lane(const float (&x)[E], int GS, int leve
   zr = mn;
 }
 
+// Symmetric per-vector quantiser (Appendix C.3) of one warp's row, lane
+// holding E channels: s = bf16(max|x| / q) (one binary32 division, then
+// round to nearest even), code = clip(rint(x / s), -q, q) with the stored
+// scale, returned offset by q (u = code + q).  A zero row stores s = 0 and
+// code 0.  Returns the bf16 bits of s.
+template <int E>
+__device__ __forceinline__ uint16_t quant_sym_lane(const float (&x)[E], int bits,
+                                                   uint32_t (&u)[E]) {
+  float am = 0.f;
+#pragma unroll
+  for (int e = 0; e < E; ++e) am = fmaxf(am, fabsf(x[e]));
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, off));
+  const float q = (float)sym_levels(bits);
+  const uint16_t sb = f32_to_bf16_bits(__fdiv_rn(am, q));
+  const float s = bf16_to_f32(sb);
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    float r = 0.f;
+    if (s != 0.f) r = fminf(fmaxf(rintf(__fdiv_rn(x[e], s)), -q), q);
+    u[e] = (uint32_t)(int)(r + q);
+  }
+  return sb;
+}
+
+// Symmetric record of (sequence b, position t, KV head kvh): both sections
+// assembled in the per-warp buffer in physical (rotated) order, stored as
+// whole 16-byte chunks; the two scales go to the scale plane.
+template <int D>
+__device__ void append_row_sym(const GqaView &v, const float (&xk)[D / 32],
+                               const float (&xv)[D / 32], int b, int kvh, int t, uint32_t *buf,
+                               int lane) {
+  constexpr int E = D / 32;
+  const int rb = v.rec_bytes;
+  const int kb = D * v.bits / 8;
+  const size_t row = ((size_t)b * v.Hkv + kvh) * v.cap + t;
+  uint32_t uk[E], uv[E];
+  const uint32_t sk = quant_sym_lane<E>(xk, v.bits, uk);
+  const uint32_t sv = quant_sym_lane<E>(xv, v.bits, uv);
+  for (int w = lane; w < rb / 4; w += 32) buf[w] = 0;
+  __syncwarp();
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int ch = lane * E + e;
+    const int lk = sym_k_bit(ch, v.bits, D);
+    const int pk = 8 * sym_phys(lk >> 3, t, rb) + (lk & 7);
+    atomicOr(buf + (pk >> 5), uk[e] << (pk & 31));
+    const int lv = sym_v_bit(ch, v.bits, D) + 8 * kb;
+    const int pv = 8 * sym_phys(lv >> 3, t, rb) + (lv & 7);
+    atomicOr(buf + (pv >> 5), uv[e] << (pv & 31));
+  }
+  __syncwarp();
+  uint4 *rec = reinterpret_cast<uint4 *>(v.rec + row * rb);
+  for (int q = lane; q < rb / 16; q += 32) rec[q] = reinterpret_cast<const uint4 *>(buf)[q];
+  if (lane == 0) v.scales[row] = sk | (sv << 16);
+  __syncwarp();
+}
+
 // Writes one section (K or V) of a record through a per-warp shared buffer
 // so the global stores are whole 16-byte chunks.
 template <int D>
@@ -109,6 +167,10 @@ template <int D>
 __device__ void append_row(const GqaView &v, const float (&xk)[D / 32], const float (&xv)[D / 32],
                            int b, int kvh, int t, uint32_t *buf, int lane) {
   constexpr int E = D / 32;
+  if (v.scheme == kSchemeSym) {
+    append_row_sym<D>(v, xk, xv, b, kvh, t, buf, lane);
+    return;
+  }
   const RecLayout L = rec_layout(v.bits, D, v.group, v.key_axis);
   uint8_t *rec = v.rec + (((size_t)b * v.Hkv + kvh) * v.cap + t) * L.rec;
   const bool kq = v.bits != 16 && v.key_axis == 0;

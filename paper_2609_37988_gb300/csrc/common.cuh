@@ -22,6 +22,13 @@ __device__ __forceinline__ void cp_async16(void *dst, const void *src, bool vali
                "l"(src), "r"(n)
                : "memory");
 }
+// Copies 4 bytes (both addresses 4-byte aligned), or zero-fills.
+__device__ __forceinline__ void cp_async4(void *dst, const void *src, bool valid) {
+  const int n = valid ? 4 : 0;
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(smem_u32(dst)), "l"(src),
+               "r"(n)
+               : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() {
   asm volatile("cp.async.commit_group;\n" ::: "memory");
 }

@@ -28,6 +28,13 @@
 //           sum_t p_t z_tg added once at the end.
 // bf16 caches multiply bf16 operands directly; P is split into hi + lo
 // bf16 halves so the value product keeps ~16 significant bits.
+// The symmetric per-vector scheme (KAX == kKaxSym; the paper's quantiser,
+// Appendix C.3) is the per-token case with one group per row: codes stored
+// as u = code + q, so x = s u - q s, i.e. scale s and zero -q s, with the
+// bf16 scales streamed from the anchor's scale plane beside the records.
+// 2-bit codes (this scheme only) enter the MMA like 4-bit ones, as masked
+// fields of a word at weights 4^e that the query (keys) or the final
+// accumulator scale (values) undoes.
 #pragma once
 #include <math.h>
 
@@ -37,16 +44,20 @@
 
 namespace kvk {
 
+// key-axis template value of the symmetric per-vector scheme
+constexpr int kKaxSym = 2;
+
 template <int BITS, int D, int KAX, int GS>
 struct GqaCfg {
   static constexpr bool BF = (BITS == 16);
   static constexpr bool QUANT = !BF;
-  static constexpr bool KPT = QUANT && KAX == 0;  // per-token key meta in record
+  static constexpr bool SYM = QUANT && KAX == kKaxSym;  // scales in the scale plane
+  static constexpr bool KPT = QUANT && (KAX == 0 || SYM);  // per-token key groups
   static constexpr bool KPC = QUANT && KAX == 1;  // per-channel key groups
   static constexpr int KS = D / 16;               // k-steps (= value M-blocks)
   static constexpr int NG = QUANT ? D / GS : 1;   // channel groups per row
   static constexpr int KB = D * BITS / 8;         // K (and V) section bytes
-  static constexpr int MB = QUANT ? ((NG * 8 + 15) & ~15) : 0;
+  static constexpr int MB = (QUANT && !SYM) ? ((NG * 8 + 15) & ~15) : 0;
   static constexpr int REC = 2 * KB + (KPT ? MB : 0) + (QUANT ? MB : 0);
   static constexpr int CPR = REC / 16;            // 16-byte chunks per record
   static constexpr int SK = KB / 4;               // bytes of one lane's K segment
@@ -65,15 +76,19 @@ struct GqaCfg {
   static constexpr int KG_OFF = VM_OFF + (QUANT ? kTile * MB : 0);
   // row blocks of 16 per warp and tile height: two blocks for per-token
   // 4-bit keys (more independent work per warp, shared softmax reductions)
-  static constexpr int RB = (KPT && BITS == 4) ? 2 : 1;
+  static constexpr int RB = (KPT && BITS <= 4) ? 2 : 1;
   static constexpr int TILE = 64 * RB;
   static constexpr int KG_ROWS = KPC ? kTile / GS : 0;
+  static constexpr int NCH = REC / 16;            // 16-byte chunks per record
+  static constexpr float QL = SYM ? (float)((1 << (BITS - 1)) - 1) : 0.f;  // symmetric q
   // Quantised caches: a stage is 64 raw records (one bulk copy) followed by
   // the tile's key-group metadata rows.  bf16 caches: planes filled by
   // 16-byte copies with conflict-free swizzles.
   static constexpr bool TMA = QUANT;
   static constexpr int KG_OFF_T = TILE * REC;
-  static constexpr int STAGE = TMA ? KG_OFF_T + KG_ROWS * D * 8 : KG_OFF + KG_ROWS * D * 8;
+  static constexpr int SC_OFF_T = TILE * REC;     // symmetric: one scale word per row
+  static constexpr int STAGE = TMA ? KG_OFF_T + KG_ROWS * D * 8 + (SYM ? TILE * 4 : 0)
+                                   : KG_OFF + KG_ROWS * D * 8;
   static constexpr int NST = TMA ? (STAGE <= 13312 ? 4 : (STAGE <= 20480 ? 3 : 2)) : 2;
   static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");
   static constexpr int QSTR = D + 4;  // padded query row (floats): conflict-free head rows
@@ -85,6 +100,8 @@ struct GqaCfg {
   // shared memory (228 KB per SM, 1 KB reserved per CTA), else three
   static constexpr int MIN_CTAS = (!BF && 4 * (SMEM + 1024) <= 233472) ? 4 : 3;
   static_assert(REC % 16 == 0, "records are 16-byte multiples");
+  static_assert(BITS != 2 || SYM, "2-bit codes exist for the symmetric scheme only");
+  static_assert(!SYM || (D == 128 && GS == D), "symmetric rows are 128 channels, one group");
   static_assert(!QUANT || (GS % 16 == 0 && D % GS == 0), "groups are whole k-steps");
   static_assert(4 * 8 * (D + 2) * 4 <= NST * STAGE, "merge scratch fits the stages");
 };
@@ -110,6 +127,22 @@ __device__ __forceinline__ uint32_t u8pair_f16(uint32_t x, uint32_t sel) {
 // f16 pair of the nibbles under `mask` (low nibble: c * 2^-24, high nibble:
 // 16 c * 2^-24).
 __device__ __forceinline__ uint32_t nib_f16(uint32_t x, uint32_t mask) { return x & mask; }
+
+// The key code of channel ch enters the score MMA at weight 4^e (the query
+// fragment of that channel carries 4^-e): 4-bit codes in a high nibble
+// (slots 8..15 of a k-step) e = 2; 2-bit codes e = 2 (k-step mod 2) +
+// (slot >= 8); else e = 0.  key_weight(ch, s) = 4^(s e), s = +1 or -1,
+// built from its exponent bits (exact, no division).
+template <int BITS>
+__device__ __forceinline__ int key_weight_exp(int ch) {
+  if constexpr (BITS == 4) return ((ch & 15) >= 8) ? 2 : 0;
+  if constexpr (BITS == 2) return 2 * ((ch >> 4) & 1) + ((ch & 15) >= 8);
+  return 0;
+}
+template <int BITS>
+__device__ __forceinline__ float key_weight(int ch, int sgn) {
+  return __int_as_float((127 + 2 * sgn * key_weight_exp<BITS>(ch)) << 23);
+}
 
 // GATHER: the rows come from the anchor's kept-position list (compiled
 // separately so that the contiguous path carries none of its state).
@@ -147,6 +180,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   const size_t slab = (size_t)b * v.Hkv + kvh;
   const uint8_t *rec = v.rec + slab * (size_t)v.cap * C::REC;
   const float2 *gmeta = C::KPC ? v.gmeta + slab * (size_t)(v.cap / GS) * D : nullptr;
+  const uint32_t *scl = C::SYM ? v.scales + slab * (size_t)v.cap : nullptr;
   const int n_tiles = i1 > i0 ? (i1 - i0 + C::TILE - 1) / C::TILE : 0;
 
   // ---- producer: one tile of records into one stage ----------------------
@@ -247,11 +281,15 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     if constexpr (C::KPC) kgv = max(0, min(C::KG_ROWS, len / GS - base / GS));
     if (!gather) {
       if (tid == 0) {
+        // symmetric scales: whole 16-byte groups of 4 words (the slab's
+        // capacity is a multiple of 64 positions, so they stay inside it)
+        const int scb = C::SYM ? ((nrows + 3) & ~3) * 4 : 0;
         fence_proxy_async();
-        mbar_expect_tx(&bars[s], nrows * C::REC + kgv * D * 8);
+        mbar_expect_tx(&bars[s], nrows * C::REC + kgv * D * 8 + scb);
         bulk_g2s(st, rec + (size_t)base * C::REC, nrows * C::REC, &bars[s]);
         if (C::KPC && kgv > 0)
           bulk_g2s(st + C::KG_OFF_T, gmeta + (size_t)(base / GS) * D, kgv * D * 8, &bars[s]);
+        if (C::SYM) bulk_g2s(st + C::SC_OFF_T, scl + base, scb, &bars[s]);
       }
       if (nrows < C::TILE) zero_rows(st, nrows, C::TILE);
     } else {
@@ -275,8 +313,9 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       }
       const uint32_t vm = __ballot_sync(0xffffffffu, mine);
       if (lane == 0) gmask[s * 4 + warp] = vm;
-      // value chunks are stored rotated by v_rot(position) and read rotated
-      // by v_rot(shared-memory row): chunk u of the record moves accordingly
+      // value chunks (grouped) or whole records (symmetric) are stored
+      // rotated by the position and read rotated by the shared-memory row:
+      // chunk u of the record moves accordingly
       constexpr int VC0 = C::KB / 16, NC = C::KB / 16;
       uint8_t *wst = st + RPW * warp * C::REC;
 #pragma unroll 3
@@ -286,12 +325,18 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
         if (q < RPW * CPRR) {
           const bool valid = (vm >> (j & 31)) & 1u;
           int ud = u;
-          if (u >= VC0 && u < VC0 + NC)
+          if constexpr (C::SYM)
+            ud = (u - sym_rot(pos, C::NCH) + sym_rot(RPW * warp + j, C::NCH)) & (C::NCH - 1);
+          else if (u >= VC0 && u < VC0 + NC)
             ud = VC0 + ((u - VC0 - v_rot(pos, C::REC, NC) + v_rot(RPW * warp + j, C::REC, NC)) &
                         (NC - 1));
           cp_async16(wst + j * C::REC + 16 * ud, rec + (size_t)(valid ? pos : 0) * C::REC + 16 * u,
                      valid);
         }
+      }
+      if constexpr (C::SYM) {
+        if (lane < RPW)
+          cp_async4(st + C::SC_OFF_T + 4 * (RPW * warp + lane), scl + (mine ? myidx : 0), mine);
       }
     }
   };
@@ -332,12 +377,12 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
 #pragma unroll 4
     for (int k = 0; k < CPL; ++k) {
       const int ch = gi * GS + sub * CPL + k;
-      const bool hs = (BITS == 4) && ((ch & 15) >= 8);
+      const float w = key_weight<BITS>(ch, 1);  // a power of two: exact scaling
       const float x = q_s[h * QSTR + ch];
-      const float xs = hs ? x * 0.0625f : x;
+      const float xs = x * key_weight<BITS>(ch, -1);
       float xe = __half2float(__float2half_rn(xs));
       if (use_lo0) xe += __half2float(__float2half_rn(xs - xe));
-      sq += hs ? 16.f * xe : xe;
+      sq += w * xe;
     }
 #pragma unroll
     for (int off = 1; off < LPI; off <<= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
@@ -357,10 +402,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
 #pragma unroll
       for (int js = 0; js < KS; ++js) {
         const float *qh = q_s + g * QSTR + 16 * js;
-        float x2 = qh[2 * c + 8], x3 = qh[2 * c + 9];
-        if (BITS == 4) { x2 *= 0.0625f; x3 *= 0.0625f; }
-        split2<BF>(qh[2 * c], qh[2 * c + 1], hb[js][0], lb[js][0]);
-        split2<BF>(x2, x3, hb[js][1], lb[js][1]);
+        // inverse code weights of this lane's channels (powers of two)
+        const float w0 = key_weight<BITS>(16 * js, -1), w1 = key_weight<BITS>(16 * js + 8, -1);
+        split2<BF>(qh[2 * c] * w0, qh[2 * c + 1] * w0, hb[js][0], lb[js][0]);
+        split2<BF>(qh[2 * c + 8] * w1, qh[2 * c + 9] * w1, hb[js][1], lb[js][1]);
       }
     }
     __syncthreads();  // every read of the query rows is done
@@ -394,14 +439,26 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
 #pragma unroll
   for (int gi = 0; gi < NG; ++gi) zacc[gi][0] = zacc[gi][1] = 0.f;
 
-  // shared-memory addresses of the fragments (raw records or planes)
+  // shared-memory addresses of the fragments (raw records or planes).
+  // Symmetric records are rotated as a whole by sym_rot(row); the rows a
+  // lane reads for keys are g and g + 8 of a 16-row block, so the rotation
+  // is one per lane.
+  const int krot = C::SYM ? sym_rot(g, C::NCH) : 0;
   auto k_chunk = [&](const uint8_t *st, int t, int i) -> const uint8_t * {
-    if constexpr (C::TMA) return st + t * C::REC + 16 * (4 * i + c);
+    if constexpr (C::SYM) return st + t * C::REC + 16 * ((4 * i + c + krot) & (C::NCH - 1));
+    else if constexpr (C::TMA) return st + t * C::REC + 16 * (4 * i + c);
     else return st + C::KP_OFF + t * C::KSTR + 16 * kswz(C::KSWZ, t, 4 * i + c);
   };
   auto k_half = [&](const uint8_t *st, int t) -> const uint8_t * {  // 8-byte lane segment
-    if constexpr (C::TMA) return st + t * C::REC + 8 * c;
+    if constexpr (C::SYM)
+      return st + t * C::REC + 16 * (((c >> 1) + krot) & (C::NCH - 1)) + 8 * (c & 1);
+    else if constexpr (C::TMA) return st + t * C::REC + 8 * c;
     else return st + C::KP_OFF + t * C::KSTR + 8 * c;
+  };
+  // symmetric scales of shared-memory row t: (K scale, V scale)
+  auto sc_pair = [&](const uint8_t *st, int t) -> float2 {
+    const uint32_t w = reinterpret_cast<const uint32_t *>(st + C::SC_OFF_T)[t];
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
   };
   auto v_chunk = [&](const uint8_t *st, int t, int k) -> const uint8_t * {
     const int u = g * (C::SV / 16) + k;
@@ -451,6 +508,13 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       } else if constexpr (BITS == 8) {
         a0 = u8pair_f16(wa[js], 0x4140); a2 = u8pair_f16(wa[js], 0x4342);
         a1 = u8pair_f16(wb[js], 0x4140); a3 = u8pair_f16(wb[js], 0x4342);
+      } else if constexpr (BITS == 2) {
+        // k-step js: byte (js/2) % 2 of each half, fields 2 (js % 2) + {0, 1}
+        const int sh = (js & 2) * 4;
+        const uint32_t xa = wa[js >> 2] >> sh, xb = wb[js >> 2] >> sh;
+        const uint32_t m0 = 0x00030003u << (4 * (js & 1)), m2 = 0x000C000Cu << (4 * (js & 1));
+        a0 = xa & m0; a2 = xa & m2;
+        a1 = xb & m0; a3 = xb & m2;
       } else {
         const int sh = (js & 1) * 8;
         const uint32_t xa = wa[js >> 1] >> sh, xb = wb[js >> 1] >> sh;
@@ -572,9 +636,14 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           const float2 *kmB = km_row(st, tB);
           constexpr int JPG = GS / 16;  // k-steps per group
           float4 qA, qB;  // (scale, zero) of groups 2j and 2j + 1: one 16-byte load
+          if constexpr (C::SYM) {  // one group: scale s, zero -q s
+            const float kA = sc_pair(st, tA).x, kB = sc_pair(st, tB).x;
+            qA = make_float4(kA, -C::QL * kA, 0.f, 0.f);
+            qB = make_float4(kB, -C::QL * kB, 0.f, 0.f);
+          }
 #pragma unroll
           for (int gi = 0; gi < NG; ++gi) {
-            if ((gi & 1) == 0) {
+            if (!C::SYM && (gi & 1) == 0) {
               qA = reinterpret_cast<const float4 *>(kmA)[gi >> 1];
               qB = reinterpret_cast<const float4 *>(kmB)[gi >> 1];
             }
@@ -707,7 +776,8 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
           const int j = mi / NC, k = mi % NC;
           const int t = wr0 + 16 * rb + 8 * j + (lane & 7);
           const uint8_t *src =
-              st + t * C::REC + C::KB + 16 * ((k + v_rot(t, C::REC, NC)) & (NC - 1));
+              C::SYM ? st + t * C::REC + 16 * ((NC + k + sym_rot(t, C::NCH)) & (C::NCH - 1))
+                     : st + t * C::REC + C::KB + 16 * ((k + v_rot(t, C::REC, NC)) & (NC - 1));
           ldmatrix_x4_t(vw[rb][4 * q], vw[rb][4 * q + 1], vw[rb][4 * q + 2], vw[rb][4 * q + 3],
                         src);
         }
@@ -723,7 +793,14 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
 #pragma unroll
           for (int rb = 0; rb < RB; ++rb) {
             const int tA = wr0 + 16 * rb + g;
-            if ((gi & 1) == 0) {
+            if constexpr (C::SYM) {
+              // rows without a position have p = 0 but possibly a stale
+              // scale word: their scale becomes 0 (0 * NaN would poison)
+              const float sA = vA[rb] ? sc_pair(st, tA).y : 0.f;
+              const float sB = vB[rb] ? sc_pair(st, tA + 8).y : 0.f;
+              vA4[rb] = make_float4(sA, -C::QL * sA, 0.f, 0.f);
+              vB4[rb] = make_float4(sB, -C::QL * sB, 0.f, 0.f);
+            } else if ((gi & 1) == 0) {
               vA4[rb] = reinterpret_cast<const float4 *>(vm_row(st, tA))[gi >> 1];
               vB4[rb] = reinterpret_cast<const float4 *>(vm_row(st, tA + 8))[gi >> 1];
             }
@@ -748,6 +825,14 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
             const uint32_t X0 = vw[rb][m], X2 = vw[rb][NC + m];
             a0 = u8pair_f16(X0, 0x4240); a1 = u8pair_f16(X0, 0x4341);
             a2 = u8pair_f16(X2, 0x4240); a3 = u8pair_f16(X2, 0x4341);
+          } else if constexpr (BITS == 2) {
+            // byte (m/2) % 2 of each half, field 2 (m % 2) (row g) and
+            // 2 (m % 2) + 1 (row g+8): weights 4^(2 (m%2)) and 4^(2 (m%2) + 1)
+            const int sh = (m & 2) * 4;
+            const uint32_t X0 = vw[rb][m >> 2] >> sh, X2 = vw[rb][NC + (m >> 2)] >> sh;
+            const uint32_t mg = 0x00030003u << (4 * (m & 1)), mh = 0x000C000Cu << (4 * (m & 1));
+            a0 = X0 & mg; a1 = X0 & mh;
+            a2 = X2 & mg; a3 = X2 & mh;
           } else {
             // bytes 0 and 2 (even m) or 1 and 3 (odd m): row g in the low
             // nibble, row g+8 in the high nibble (16x, undone at the end)
@@ -814,10 +899,13 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     const int ch0 = 16 * m + g, ch1 = ch0 + 8;
     const int gi = C::QUANT ? (16 * m) / GS : 0;
     constexpr float vsc = C::QUANT ? kCodeScale : 1.f;  // value codes carry 2^-24
-    constexpr float hs = (BITS == 4) ? 0.0625f * vsc : vsc;
+    // code weights of rows g and g+8 of M-block m, undone here
+    const float ls = (BITS == 2 && (m & 1)) ? 0.0625f * vsc : vsc;
+    const float hs = (BITS == 4) ? 0.0625f * vsc
+                   : (BITS == 2) ? ((m & 1) ? 0.015625f * vsc : 0.25f * vsc) : vsc;
     const float z0 = C::QUANT ? zacc[gi][0] : 0.f, z1 = C::QUANT ? zacc[gi][1] : 0.f;
-    red[(warp * 8 + 2 * c) * RS + ch0] = acc[m][0] * vsc + z0;
-    red[(warp * 8 + 2 * c + 1) * RS + ch0] = acc[m][1] * vsc + z1;
+    red[(warp * 8 + 2 * c) * RS + ch0] = acc[m][0] * ls + z0;
+    red[(warp * 8 + 2 * c + 1) * RS + ch0] = acc[m][1] * ls + z1;
     red[(warp * 8 + 2 * c) * RS + ch1] = acc[m][2] * hs + z0;
     red[(warp * 8 + 2 * c + 1) * RS + ch1] = acc[m][3] * hs + z1;
   }

@@ -22,6 +22,25 @@ __global__ void gqa_export_kernel(const GqaView v, uint8_t *k_out, uint8_t *v_ou
     const size_t row = id / D;  // (slab, t)
     const int t = (int)(row % max_ctx);
     const size_t slab = row / max_ctx;
+    if (v.scheme == kSchemeSym) {
+      // signed codes in [-q, q] and the two bf16 scales, widened
+      const uint8_t *rec = v.rec + (slab * v.cap + t) * v.rec_bytes;
+      const int q = sym_levels(v.bits), mask = (1 << v.bits) - 1;
+      for (int kv = 0; kv < 2; ++kv) {
+        uint8_t *dst = kv ? v_out : k_out;
+        if (!dst) continue;
+        const int lb = kv ? sym_v_bit(ch, v.bits, D) + D * v.bits : sym_k_bit(ch, v.bits, D);
+        const int pb = sym_phys(lb >> 3, t, v.rec_bytes);
+        const int u = (rec[pb] >> (lb & 7)) & mask;
+        dst[id] = (uint8_t)(int8_t)(u - q);
+      }
+      if (ch == 0) {
+        const uint32_t w = v.scales[slab * v.cap + t];
+        if (k_scale) k_scale[row] = bf16_to_f32((uint16_t)(w & 0xffffu));
+        if (v_scale) v_scale[row] = bf16_to_f32((uint16_t)(w >> 16));
+      }
+      continue;
+    }
     const uint8_t *rec = v.rec + (slab * v.cap + t) * L.rec;
     for (int kv = 0; kv < 2; ++kv) {
       uint8_t *dst = kv ? v_out : k_out;

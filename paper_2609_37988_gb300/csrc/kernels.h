@@ -14,9 +14,11 @@ struct GqaView {
   int32_t *counter;    // append completion counter
   int32_t *kept_n;     // [B]
   int32_t *kept_idx;   // [B * kept_cap]
+  uint32_t *scales;    // symmetric scheme: bf16 (K, V) scale pair per (slab, position)
   int64_t cap;         // positions per slab
   int kept_cap;
   int B, Hkv, D, bits, group, key_axis, rec_bytes;
+  int scheme;          // kSchemeGrouped or kSchemeSym
 };
 
 struct MlaView {
@@ -44,8 +46,8 @@ struct GqaDecodeArgs {
 // Returns cudaSuccess or the launch error.  Template dispatch on
 // (bits, D, key axis, q dtype) happens inside.
 cudaError_t launch_gqa_decode(const GqaDecodeArgs &a, cudaStream_t st);
-int gqa_decode_ctas_per_sm(int bits, int D, int key_axis, int group);
-int gqa_decode_tile(int bits, int D, int key_axis, int group);
+int gqa_decode_ctas_per_sm(int bits, int D, int key_axis, int group, int scheme);
+int gqa_decode_tile(int bits, int D, int key_axis, int group, int scheme);
 
 struct RewindArgs {
   int32_t *lens[64];

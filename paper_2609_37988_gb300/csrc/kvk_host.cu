@@ -73,6 +73,8 @@ kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
     if (l == 0) return fail(KVK_ERR_INVALID_CONFIG, "layer 0 must own a cache (it inherits)");
     return KVK_OK;
   }
+  if (c->scheme != KVK_QUANT_GROUPED && c->scheme != KVK_QUANT_SYMMETRIC)
+    return fail(KVK_ERR_INVALID_CONFIG, "layer %d: unknown quantisation scheme %d", l, c->scheme);
   if (d->kind == KVK_KIND_MLA) {
     if (c->bits != 16 && c->bits != 8 && c->bits != 4 && c->bits != 2)
       return fail(KVK_ERR_INVALID_CONFIG, "layer %d: bits %d not in {16, 8, 4, 2}", l, c->bits);
@@ -89,12 +91,21 @@ kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
   }
   if (c->bits != 16 && c->bits != 8 && c->bits != 4 && c->bits != 2)
     return fail(KVK_ERR_INVALID_CONFIG, "layer %d: bits %d not in {16, 8, 4, 2}", l, c->bits);
-  if (c->bits != 16) {
+  if (c->bits != 16 && c->scheme == KVK_QUANT_SYMMETRIC) {
+    // one scale per token-head row (Appendix C.3): both axes per token
+    if (c->key_axis != KVK_AXIS_TOKEN || c->value_axis != KVK_AXIS_TOKEN)
+      return fail(KVK_ERR_INVALID_CONFIG,
+                  "layer %d: the symmetric scheme scales whole token-head rows", l);
+    if (need_support && d->head_dim != 128)
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: symmetric scheme with head_dim %d (this build: 128)",
+                  l, d->head_dim);
+  } else if (c->bits != 16) {
     if (c->group <= 0 || d->head_dim % c->group)
       return fail(KVK_ERR_INVALID_CONFIG, "layer %d: group %d must divide head_dim", l, c->group);
     if (!need_support) return KVK_OK;
     if (c->bits == 2)
-      return fail(KVK_ERR_UNSUPPORTED, "layer %d: 2-bit codes are not in this build", l);
+      return fail(KVK_ERR_UNSUPPORTED,
+                  "layer %d: grouped 2-bit codes are not in this build (the symmetric scheme has them)", l);
     if (c->group != 32 && c->group != 64)
       return fail(KVK_ERR_UNSUPPORTED, "layer %d: group %d (this build: 32, 64)", l, c->group);
     if (c->value_axis != KVK_AXIS_TOKEN)
@@ -109,11 +120,21 @@ kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
   return KVK_OK;
 }
 
+// Internal scheme and group of a layer: bf16 layers count as grouped with a
+// nominal group of 64; symmetric layers scale whole rows (group = head_dim).
+int layer_scheme(const kvk_layer_cfg *c) {
+  return (c->bits != 16 && c->scheme == KVK_QUANT_SYMMETRIC) ? kSchemeSym : kSchemeGrouped;
+}
+int layer_group(const kvk_model_desc *d, const kvk_layer_cfg *c) {
+  if (c->bits == 16) return 64;
+  return layer_scheme(c) == kSchemeSym ? d->head_dim : c->group;
+}
+
 ArenaLayout layer_layout(const kvk_model_desc *d, const kvk_layer_cfg *c) {
   const bool mla = d->kind == KVK_KIND_MLA;
   return arena_layout(mla ? 1 : 0, d->max_batch, mla ? 1 : d->n_kv_heads, d->max_ctx, d->head_dim,
-                      c->bits, c->bits == 16 ? 64 : c->group, c->key_axis, c->evict_capacity,
-                      c->width, d->rope_dim);
+                      c->bits, layer_group(d, c), c->key_axis, c->evict_capacity, c->width,
+                      d->rope_dim, layer_scheme(c));
 }
 
 struct WsLayout {
@@ -167,6 +188,7 @@ struct kvk_cache {
     v.rec = a + A.rec;
     v.gmeta = A.gmeta >= 0 ? reinterpret_cast<float2 *>(a + A.gmeta) : nullptr;
     v.resid = A.resid >= 0 ? a + A.resid : nullptr;
+    v.scales = A.scales >= 0 ? reinterpret_cast<uint32_t *>(a + A.scales) : nullptr;
     v.lens = reinterpret_cast<int32_t *>(a + A.lens);
     v.counter = reinterpret_cast<int32_t *>(a + A.counter);
     v.kept_n = reinterpret_cast<int32_t *>(a + A.kept_n);
@@ -177,9 +199,10 @@ struct kvk_cache {
     v.Hkv = desc.n_kv_heads;
     v.D = desc.head_dim;
     v.bits = c.bits;
-    v.group = c.bits == 16 ? 64 : c.group;
+    v.group = layer_group(&desc, &c);
     v.key_axis = c.bits == 16 ? 0 : c.key_axis;
     v.rec_bytes = A.rec_bytes;
+    v.scheme = layer_scheme(&c);
     return v;
   }
   MlaView mla_view(int l) const {
@@ -250,7 +273,7 @@ int auto_splits(kvk_cache *c, int a) {
     } else {
       const kvk_layer_cfg &L = c->cfg[a];
       c->ctas[a] = gqa_decode_ctas_per_sm(L.bits, c->desc.head_dim, L.bits == 16 ? 0 : L.key_axis,
-                                          L.bits == 16 ? 64 : L.group);
+                                          layer_group(&c->desc, &L), layer_scheme(&L));
     }
   }
   const int units = mla ? c->desc.max_batch : c->desc.max_batch * c->desc.n_kv_heads;
@@ -537,7 +560,8 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   args.sig_log2 = scale * 1.4426950408889634f;
   args.n_splits = n_splits;
   // split boundaries fall on the kernel's tile height (64 or 128 positions)
-  const int kt = gqa_decode_tile(args.v.bits, args.v.D, args.v.key_axis, args.v.group);
+  const int kt =
+      gqa_decode_tile(args.v.bits, args.v.D, args.v.key_axis, args.v.group, args.v.scheme);
   const int per = kt / kTile;
   const int tps = ((tiles + n_splits - 1) / n_splits + per - 1) / per * per;
   args.items_per_split = tps * kTile;
@@ -689,6 +713,9 @@ kvk_status kvk_plan_cost(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
       double per;
       if (a.bits == 16) {
         per = 4.0 * d.head_dim;
+      } else if (a.scheme == KVK_QUANT_SYMMETRIC) {
+        // codes + one bf16 scale per row, K and V
+        per = 2.0 * d.head_dim * a.bits / 8.0 + 2.0 * 2.0;
       } else {
         // codes + one fp32 (scale, zero) pair per group, K and V
         per = 2.0 * d.head_dim * a.bits / 8.0 + 2.0 * 8.0 * d.head_dim / a.group;

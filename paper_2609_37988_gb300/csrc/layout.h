@@ -44,6 +44,29 @@
 //      that eight consecutive records' copies of one chunk fall in eight
 //      distinct 16-byte bank slots of shared memory.
 //
+// Symmetric per-vector scheme (the paper's own quantiser, Appendix C.3: one
+// bf16 scale per token-head row, no zero point, codes in [-q, q] with
+// q = 2^(b-1) - 1, b = 2, 4 or 8).  Codes are stored offset by q (u = code +
+// q, unsigned) in the same fragment orders as above, 2-bit codes as below.
+// The record holds only [K section | V section]; the two bf16 scales of a
+// (position, KV head) sit in a scale plane [slab][cap] as one 32-bit word
+// (K scale in the low half, V scale in the high half).  The record's 16-byte
+// chunks are rotated as a whole: logical chunk u of position t sits at chunk
+// (u + sym_rot(t)) mod nch.  With 64-byte records (2-bit) the rotation is
+// (t/2) mod 4, with 128- or 256-byte records t mod 8; either way the key
+// fragments of eight consecutive positions and the ldmatrix rows of one value
+// chunk fall on distinct shared-memory bank slots.
+//
+//   2-bit K: lane c's segment is 8 bytes (two 32-bit words); word w holds
+//      k-steps 4w..4w+3.  In each 16-bit half (low half: slots 2c and 2c+8,
+//      high half: 2c+1 and 2c+9) byte jj/2 of k-step jj = j % 4 holds four
+//      2-bit fields: field 2 (jj % 2) + a for a = 0 (a0 register) or 1 (a2),
+//      so a mask of 0x00030003 << (4 (jj % 2)) (a0) or 0x000C000C << ...
+//      (a2), after >> 8 for jj >= 2, yields the f16 pair at weight 4^field.
+//   2-bit V: the 16-bit element g of 16-byte chunk k holds lane row g's
+//      fields of M-blocks 4k..4k+3: byte (m/2) % 2, field 2 (m % 2) + e for
+//      row g + 8e.
+//
 // An MLA anchor stores [c[:width] | k^R] in bf16, natural order, one record
 // per (batch, position).
 #pragma once
@@ -58,6 +81,10 @@
 namespace kvk {
 
 constexpr int kTile = 64;  // positions per decode tile
+
+// quantisation schemes of a GQA anchor
+constexpr int kSchemeGrouped = 0;    // asymmetric, (scale, zero) per group
+constexpr int kSchemeSym = 1;        // symmetric, one bf16 scale per row
 
 KVK_HD int sec_bytes(int bits, int D) { return D * bits / 8; }
 KVK_HD int meta_bytes(int D, int g) { return (((D / g) * 8) + 15) & ~15; }
@@ -144,6 +171,41 @@ KVK_HD void v_pos(int ch, int bits, int D, int t, int rec_bytes, int *byte, int 
   *byte = 16 * (((bl >> 4) + v_rot(t, rec_bytes, nc)) & (nc - 1)) + (bl & 15);
 }
 
+// ---- symmetric per-vector records ------------------------------------------
+KVK_HD int sym_levels(int bits) { return (1 << (bits - 1)) - 1; }
+KVK_HD int sym_rec_bytes(int bits, int D) { return 2 * sec_bytes(bits, D); }
+KVK_HD int sym_rot(int t, int nch) { return nch == 4 ? ((t >> 1) & 3) : (t & 7); }
+
+// Logical bit offset of channel `ch` inside the K section (before rotation).
+KVK_HD int sym_k_bit(int ch, int bits, int D) {
+  if (bits == 2) {
+    const int j = ch >> 4, s = ch & 15;
+    const int c = (s & 7) >> 1;
+    const int r = (s & 1) | ((s >> 3) << 1);
+    const int w = j >> 2, jj = j & 3, h = r & 1, a = r >> 1;
+    return 64 * c + 32 * w + 16 * h + 8 * (jj >> 1) + 2 * (2 * (jj & 1) + a);
+  }
+  int byte, hi;
+  k_pos(ch, bits, D, &byte, &hi);
+  return 8 * byte + 4 * hi;
+}
+
+// Logical bit offset of channel `ch` inside the V section (before rotation).
+KVK_HD int sym_v_bit(int ch, int bits, int D) {
+  const int m = ch >> 4, rr = ch & 15;
+  const int g = rr & 7, e = rr >> 3;
+  if (bits == 2) return 8 * (16 * (m >> 2) + 2 * g + ((m >> 1) & 1)) + 2 * (2 * (m & 1) + e);
+  if (bits == 8) return 8 * (16 * m + 2 * g + e);
+  (void)D;
+  return 8 * (16 * (m >> 1) + 2 * g + (m & 1)) + 4 * e;
+}
+
+// Physical byte of logical record byte `lb` of position t.
+KVK_HD int sym_phys(int lb, int t, int rec_bytes) {
+  const int nch = rec_bytes >> 4;
+  return 16 * (((lb >> 4) + sym_rot(t, nch)) & (nch - 1)) + (lb & 15);
+}
+
 KVK_HD int64_t align256(int64_t x) { return (x + 255) & ~(int64_t)255; }
 
 // Offsets inside one anchor's arena.
@@ -155,6 +217,7 @@ struct ArenaLayout {
   int64_t rec;       // records
   int64_t gmeta;     // float2 [B*Hkv][cap/g][D] (per-channel keys)
   int64_t resid;     // bf16 K rows [B*Hkv][g][D] (per-channel keys)
+  int64_t scales;    // uint32 [B*Hkv][cap] bf16 (K, V) scales (symmetric scheme)
   int64_t total;
   int64_t cap;       // positions per slab (max_ctx rounded up to kTile)
   int rec_bytes;
@@ -162,7 +225,8 @@ struct ArenaLayout {
 
 // mla: records are [B][cap][(width + rope) * 2 bytes]; kv heads = 1.
 KVK_HD ArenaLayout arena_layout(int mla, int B, int Hkv, int max_ctx, int D, int bits,
-                                int g, int key_axis, int kept_cap, int width, int rope) {
+                                int g, int key_axis, int kept_cap, int width, int rope,
+                                int scheme = kSchemeGrouped) {
   ArenaLayout A;
   A.cap = ((int64_t)max_ctx + kTile - 1) / kTile * kTile;
   int64_t off = 0;
@@ -175,9 +239,16 @@ KVK_HD ArenaLayout arena_layout(int mla, int B, int Hkv, int max_ctx, int D, int
   A.kept_idx = off;
   off = align256(off + 4 * (int64_t)B * kept_cap);
   A.rec = off;
+  A.scales = -1;
   if (mla) {
     A.rec_bytes = (width + rope) * 2;
     off = align256(off + (int64_t)B * A.cap * A.rec_bytes);
+    A.gmeta = A.resid = -1;
+  } else if (bits != 16 && scheme == kSchemeSym) {
+    A.rec_bytes = sym_rec_bytes(bits, D);
+    off = align256(off + (int64_t)B * Hkv * A.cap * A.rec_bytes);
+    A.scales = off;
+    off = align256(off + (int64_t)B * Hkv * A.cap * 4);
     A.gmeta = A.resid = -1;
   } else {
     A.rec_bytes = rec_layout(bits, D, g, key_axis).rec;

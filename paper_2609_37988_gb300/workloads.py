@@ -30,6 +30,7 @@ Five workloads (``config(n)``):
 from __future__ import annotations
 
 import math
+import re
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -46,7 +47,7 @@ class Workload:
     head_dim: int
     batch: int
     context: int                   # positions read per step
-    layers: list                   # per-layer dicts (inherit, bits, group, key_axis, width, evict_capacity)
+    layers: list                   # per-layer dicts (inherit, bits, group, key_axis, width, evict_capacity, scheme)
     sigma: float
     q_dtype: torch.dtype
     kv_dtype: torch.dtype
@@ -70,15 +71,19 @@ class Workload:
         return src
 
 
-def _layer(inherit=False, bits=16, group=64, key_axis="token", width=0, evict_capacity=0):
+def _layer(inherit=False, bits=16, group=64, key_axis="token", width=0, evict_capacity=0,
+           scheme="grouped"):
     return dict(inherit=inherit, bits=bits, group=group, key_axis=key_axis, width=width,
-                evict_capacity=evict_capacity)
+                evict_capacity=evict_capacity, scheme=scheme)
 
 
 def config(n: int, seed: int = None, *, batch: int = None, context: int = None,
-           n_layers: int = None) -> Workload:
+           n_layers: int = None, sym_bits: int = None) -> Workload:
     """Workload ``n`` (1..5).  ``batch``/``context``/``n_layers`` shrink it
-    for oracle-sized tests while keeping the per-layer draws."""
+    for oracle-sized tests while keeping the per-layer draws.  ``sym_bits``
+    (8, 4 or 2) stores every quantised anchor with the paper's symmetric
+    per-vector quantiser at that bit-width instead (per-token rows; the
+    plan, shapes and inputs are otherwise unchanged)."""
     seed = n if seed is None else seed
     rng = np.random.default_rng(seed)
     if n == 1:
@@ -125,6 +130,16 @@ def config(n: int, seed: int = None, *, batch: int = None, context: int = None,
                      layers, 1.0 / math.sqrt(128), torch.bfloat16, torch.bfloat16, seed, keep=T // 8)
     else:
         raise ValueError(f"no workload {n}")
+    if sym_bits is not None:
+        if sym_bits not in (8, 4, 2) or w.kind != "gqa" or w.head_dim != 128:
+            raise ValueError("symmetric anchors: 8, 4 or 2 bits on a head_dim-128 GQA workload")
+        for a in w.layers:
+            if not a["inherit"] and a["bits"] != 16:
+                a.update(bits=sym_bits, scheme="symmetric", key_axis="token")
+        if re.search(r"int\d", w.name):
+            w.name = re.sub(r"int\d", f"sym{sym_bits}", w.name)
+        else:
+            w.name += f"-sym{sym_bits}"
     if batch is not None:
         w.batch = batch
     if n_layers is not None:

@@ -50,6 +50,8 @@ def oracle_state(k_bthd, v_bthd, lens, cfg):
     buffered in bf16 by the cache, so fp32 key inputs are rounded to bf16
     first (bf16 inputs are unchanged)."""
     k = to_bhtd(k_bthd)
+    if cfg["bits"] != 16 and cfg.get("scheme", "grouped") == "symmetric":
+        return ocache.anchor_state(k, to_bhtd(v_bthd), lens, cfg["bits"], scheme="symmetric")
     if cfg["bits"] != 16 and cfg["key_axis"] == "channel":
         k = torch.from_numpy(k).to(torch.bfloat16).float().numpy()
     if cfg["bits"] == 16:
@@ -68,6 +70,13 @@ def check_codes(exp: dict, st: dict, lens, cfg):
         if cfg["bits"] == 16:
             k = exp["k"][b, :, :n].float().cpu().numpy()
             np.testing.assert_array_equal(k, st["k_hat"][b, :, :n].astype(np.float32))
+            continue
+        if cfg.get("scheme", "grouped") == "symmetric":
+            for x in ("k", "v"):
+                np.testing.assert_array_equal(exp[x + "_codes"][b, :, :n].cpu().numpy(),
+                                              st[x + "_codes"][b, :, :n])
+                np.testing.assert_array_equal(exp[x + "_scale"][b, :, :n].cpu().numpy(),
+                                              st[x + "_scale"][b, :, :n])
             continue
         g = cfg["group"]
         np.testing.assert_array_equal(exp["v_codes"][b, :, :n].cpu().numpy(), st["v_codes"][b, :, :n])

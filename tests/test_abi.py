@@ -120,3 +120,48 @@ def test_plan_cost_matches_oracle_and_paper(lib):
                max_batch=1, max_ctx=64)
     narrow = _plan_cost(lib, m5, _plan(lib, *([(0, 16, 0, 0, 0, 64, 0)] * 48)))
     assert narrow[0] == 48 * (64 + 64) * 16
+
+
+# symmetric per-vector scheme: (inherit, bits, group, key_axis, value_axis,
+# width, evict_capacity, scheme)
+def _sym(bits, key_axis=0, value_axis=0, evict=0):
+    return (0, bits, 0, key_axis, value_axis, 0, evict, 1)
+
+
+def test_symmetric_plan_validation(lib):
+    d = _desc(lib)
+    ok, sizes = _plan_status(lib, d, _plan(lib, _sym(2), _sym(4), INH, _sym(8, evict=100)))
+    assert ok == 0 and sizes[2] == 0
+    # a per-channel axis contradicts one scale per token-head row
+    assert _plan_status(lib, d, _plan(lib, _sym(4, key_axis=1), BF16, BF16, BF16))[0] == 2
+    assert _plan_status(lib, d, _plan(lib, _sym(4, value_axis=1), BF16, BF16, BF16))[0] == 2
+    # unknown scheme; 3 bits
+    assert _plan_status(lib, d, _plan(lib, (0, 4, 32, 0, 0, 0, 0, 2), BF16, BF16, BF16))[0] == 2
+    assert _plan_status(lib, d, _plan(lib, _sym(3), BF16, BF16, BF16))[0] == 2
+    # head_dim 64 and MLA latents are outside this build
+    assert _plan_status(lib, _desc(lib, head_dim=64), _plan(lib, _sym(4), BF16, BF16, BF16))[0] == 5
+    m = _desc(lib, kind=1, n_layers=1, n_q_heads=16, head_dim=128, latent_dim=512, rope_dim=64)
+    assert _plan_status(lib, m, _plan(lib, (0, 4, 0, 0, 0, 512, 0, 1)))[0] == 5
+    # grouped 2-bit stays unsupported, and says where 2-bit codes are
+    assert _plan_status(lib, d, _plan(lib, BF16, (0, 2, 32, 0, 0, 0, 0, 0), BF16, BF16))[0] == 5
+    assert "symmetric" in lib.load().kvk_last_error().decode()
+
+
+def test_symmetric_arena_and_cost(lib):
+    from oracle import cost
+    # per (position, kv head): codes of K and V (2 * 128 b / 8 bytes), plus
+    # one 4-byte scale word in the scale plane
+    B, H, T = 3, 2, 640
+    d = _desc(lib, n_layers=3, max_batch=B, max_ctx=T)
+    ok, sizes = _plan_status(lib, d, _plan(lib, _sym(8), _sym(4), _sym(2)))
+    assert ok == 0
+    for s, rec in zip(sizes, (256, 128, 64)):
+        assert B * H * T * (rec + 4) <= s <= B * H * T * (rec + 4) + 4096
+    # stored bits per element = b + 16/128 (Tab. realized_bits, "ours")
+    for bits in (8, 4, 2):
+        d1 = _desc(lib, n_layers=1, n_kv_heads=8, n_q_heads=40, max_batch=1, max_ctx=64)
+        b, stored, rho = _plan_cost(lib, d1, _plan(lib, _sym(bits)))
+        assert b == 2 * 8 * 128 * bits                    # eq. (cost): metadata-free
+        per_elem = stored * 8 / (2 * 8 * 128)
+        assert per_elem == pytest.approx(cost.bits_per_element_symmetric(bits))
+        assert rho == pytest.approx(16 / bits)
