@@ -217,6 +217,8 @@ template <int D>
 __global__ void __launch_bounds__(128)
     gqa_append_rows(const GqaView v, const void *kin, const void *vin, int in_f32, int n_new,
                     const int32_t *n_per_seq, int32_t *err) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int E = D / 32;
   __shared__ __align__(16) uint32_t sbuf[4][(2 * D * 2 + 2 * 64) / 4];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -268,6 +270,8 @@ template <int D>
 __global__ void __launch_bounds__(256)
     gqa_append_seq(const GqaView v, const void *kin, const void *vin, int in_f32, int n_new,
                    const int32_t *n_per_seq, int32_t *err) {
+  pdl_wait();
+  pdl_trigger();
   constexpr int E = D / 32;
   __shared__ __align__(16) uint32_t sbuf[8][(2 * D * 2 + 2 * 64) / 4];
   __shared__ int s_len, s_nb;
@@ -305,6 +309,8 @@ template <int D>
 __global__ void __launch_bounds__(128)
     gqa_append_kgroups(const GqaView v, const void *kin, int in_f32, int n_new,
                        const int32_t *n_per_seq, int32_t *err, int max_groups) {
+  pdl_wait();
+  pdl_trigger();
   const int pairs = D / 2;
   const size_t id = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   const size_t total = (size_t)v.B * v.Hkv * max_groups * pairs;
@@ -380,6 +386,8 @@ template <int D>
 __global__ void __launch_bounds__(128)
     gqa_append_kresid(const GqaView v, const void *kin, int in_f32, int n_new,
                       const int32_t *n_per_seq) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.x;
   const int GS = v.group;
   const int nb = seq_count(n_per_seq, b, n_new, nullptr);
@@ -406,6 +414,8 @@ __global__ void __launch_bounds__(128)
 __global__ void __launch_bounds__(128)
     mla_append_rows(const MlaView v, const uint16_t *c, const uint16_t *kr, int latent, int n_new,
                     const int32_t *n_per_seq, int32_t *err) {
+  pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const size_t wid = (size_t)blockIdx.x * 4 + warp;
   if (wid < (size_t)v.B * n_new) {
@@ -449,42 +459,37 @@ cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, i
   const size_t rows = (size_t)v.B * n_new * v.Hkv;
   const unsigned blocks = (unsigned)((rows + 3) / 4);
   const bool kpc = v.bits != 16 && v.key_axis == 1;
+  const bool d128 = v.D == 128;
+  cudaError_t e = cudaSuccess;
   if (kpc) {
     // groups first (they read residual rows the open group may overwrite)
     const int max_groups = (n_new + v.group - 1) / v.group + 1;
     const size_t thr = (size_t)v.B * v.Hkv * max_groups * (v.D / 2);
-    if (v.D == 128)
-      gqa_append_kgroups<128><<<(unsigned)((thr + 127) / 128), 128, 0, st>>>(v, k, in_f32, n_new, n_per_seq, err, max_groups);
-    else
-      gqa_append_kgroups<64><<<(unsigned)((thr + 127) / 128), 128, 0, st>>>(v, k, in_f32, n_new, n_per_seq, err, max_groups);
+    const dim3 grid((unsigned)((thr + 127) / 128));
+    e = launch_pdl(d128 ? gqa_append_kgroups<128> : gqa_append_kgroups<64>, grid, dim3(128), 0, st,
+                   v, k, in_f32, n_new, n_per_seq, err, max_groups);
   }
-  if (!kpc && (size_t)n_new * v.Hkv <= 64) {
-    if (v.D == 128)
-      gqa_append_seq<128><<<v.B, 256, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
+  if (e == cudaSuccess) {
+    if (!kpc && (size_t)n_new * v.Hkv <= 64)
+      e = launch_pdl(d128 ? gqa_append_seq<128> : gqa_append_seq<64>, dim3(v.B), dim3(256), 0, st,
+                     v, k, vv, in_f32, n_new, n_per_seq, err);
     else
-      gqa_append_seq<64><<<v.B, 256, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
-  } else if (v.D == 128) {
-    gqa_append_rows<128><<<blocks, 128, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
-  } else {
-    gqa_append_rows<64><<<blocks, 128, 0, st>>>(v, k, vv, in_f32, n_new, n_per_seq, err);
+      e = launch_pdl(d128 ? gqa_append_rows<128> : gqa_append_rows<64>, dim3(blocks), dim3(128), 0,
+                     st, v, k, vv, in_f32, n_new, n_per_seq, err);
   }
-  if (kpc) {
-    if (v.D == 128)
-      gqa_append_kresid<128><<<v.B, 128, 0, st>>>(v, k, in_f32, n_new, n_per_seq);
-    else
-      gqa_append_kresid<64><<<v.B, 128, 0, st>>>(v, k, in_f32, n_new, n_per_seq);
-  }
-  return cudaGetLastError();
+  if (e == cudaSuccess && kpc)
+    e = launch_pdl(d128 ? gqa_append_kresid<128> : gqa_append_kresid<64>, dim3(v.B), dim3(128), 0,
+                   st, v, k, in_f32, n_new, n_per_seq);
+  return e;
 }
 
 cudaError_t launch_mla_append(const MlaView &v, const void *c, const void *kr, int latent,
                               int n_new, const int32_t *n_per_seq, int32_t *err,
                               cudaStream_t st) {
   const size_t rows = (size_t)v.B * n_new;
-  mla_append_rows<<<(unsigned)((rows + 3) / 4), 128, 0, st>>>(
-      v, static_cast<const uint16_t *>(c), static_cast<const uint16_t *>(kr), latent, n_new,
-      n_per_seq, err);
-  return cudaGetLastError();
+  return launch_pdl(mla_append_rows, dim3((unsigned)((rows + 3) / 4)), dim3(128), 0, st, v,
+                    static_cast<const uint16_t *>(c), static_cast<const uint16_t *>(kr), latent,
+                    n_new, n_per_seq, err);
 }
 
 }  // namespace kvk

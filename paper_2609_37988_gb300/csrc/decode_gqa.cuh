@@ -149,6 +149,7 @@ __device__ __forceinline__ float key_weight(int ch, int sgn) {
 template <int BITS, int D, int KAX, int GS, bool GATHER>
 __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     gqa_decode_kernel(const GqaDecodeArgs a) {
+  pdl_wait();
   using C = GqaCfg<BITS, D, KAX, GS>;
   constexpr bool BF = C::BF;
   constexpr int KS = C::KS, NG = C::NG;
@@ -647,19 +648,26 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
               qA = reinterpret_cast<const float4 *>(kmA)[gi >> 1];
               qB = reinterpret_cast<const float4 *>(kmB)[gi >> 1];
             }
-            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            // long groups accumulate alternate k-steps in two chains
+            constexpr int NCHAIN = JPG >= 4 ? 2 : 1;
+            float dd[NCHAIN][4];
+#pragma unroll
+            for (int h = 0; h < NCHAIN; ++h) dd[h][0] = dd[h][1] = dd[h][2] = dd[h][3] = 0.f;
 #pragma unroll
             for (int jj = 0; jj < JPG; ++jj) {
               const int js = gi * JPG + jj;
               uint32_t a0, a1, a2, a3;
               kfrag(wa, wb, js, a0, a1, a2, a3);
               const uint2 qh = qf[64 * js + lane];
-              mma_f16(d, a0, a1, a2, a3, qh.x, qh.y);
+              mma_f16(dd[jj % NCHAIN], a0, a1, a2, a3, qh.x, qh.y);
               if (use_lo) {
                 const uint2 ql = qf[64 * js + 32 + lane];
-                mma_f16(d, a0, a1, a2, a3, ql.x, ql.y);
+                mma_f16(dd[jj % NCHAIN], a0, a1, a2, a3, ql.x, ql.y);
               }
             }
+            float d[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) d[k] = NCHAIN == 2 ? dd[0][k] + dd[NCHAIN - 1][k] : dd[0][k];
             const float2 mA = (gi & 1) ? make_float2(qA.z, qA.w) : make_float2(qA.x, qA.y);
             const float2 mB = (gi & 1) ? make_float2(qB.z, qB.w) : make_float2(qB.x, qB.y);
             s4[rb][0] = fmaf(mA.x, d[0], fmaf(mA.y, qs[gi][0], s4[rb][0]));
@@ -784,10 +792,13 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       }
       uint32_t pf[RB][4];
       float4 vA4[RB], vB4[RB];  // (scale, zero) of groups 2j, 2j + 1 of rows g, g + 8
+      // M-blocks in pairs (groups span whole pairs): the four MMAs of a
+      // pair and row block alternate between the two accumulators
+      static_assert(GS % 32 == 0, "value groups cover whole M-block pairs");
 #pragma unroll
-      for (int m = 0; m < KS; ++m) {
-        const int gi = (16 * m) / GS;
-        if ((16 * m) % GS == 0) {
+      for (int m0 = 0; m0 < KS; m0 += 2) {
+        const int gi = (16 * m0) / GS;
+        if ((16 * m0) % GS == 0) {
           // P' = p * value scale of this channel group, split hi/lo and
           // transposed; the zero points accumulate separately.
 #pragma unroll
@@ -819,30 +830,39 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
         }
 #pragma unroll
         for (int rb = 0; rb < RB; ++rb) {
-          uint32_t a0, a1, a2, a3;
-          if constexpr (BITS == 8) {
-            // bytes (row g, row g+8) of the two positions: (0, 2) and (1, 3)
-            const uint32_t X0 = vw[rb][m], X2 = vw[rb][NC + m];
-            a0 = u8pair_f16(X0, 0x4240); a1 = u8pair_f16(X0, 0x4341);
-            a2 = u8pair_f16(X2, 0x4240); a3 = u8pair_f16(X2, 0x4341);
-          } else if constexpr (BITS == 2) {
-            // byte (m/2) % 2 of each half, field 2 (m % 2) (row g) and
-            // 2 (m % 2) + 1 (row g+8): weights 4^(2 (m%2)) and 4^(2 (m%2) + 1)
-            const int sh = (m & 2) * 4;
-            const uint32_t X0 = vw[rb][m >> 2] >> sh, X2 = vw[rb][NC + (m >> 2)] >> sh;
-            const uint32_t mg = 0x00030003u << (4 * (m & 1)), mh = 0x000C000Cu << (4 * (m & 1));
-            a0 = X0 & mg; a1 = X0 & mh;
-            a2 = X2 & mg; a3 = X2 & mh;
-          } else {
-            // bytes 0 and 2 (even m) or 1 and 3 (odd m): row g in the low
-            // nibble, row g+8 in the high nibble (16x, undone at the end)
-            const int sh = 8 * (m & 1);
-            const uint32_t X0 = vw[rb][m >> 1] >> sh, X2 = vw[rb][NC + (m >> 1)] >> sh;
-            a0 = nib_f16(X0, 0x000F000Fu); a1 = nib_f16(X0, 0x00F000F0u);
-            a2 = nib_f16(X2, 0x000F000Fu); a3 = nib_f16(X2, 0x00F000F0u);
+          uint32_t af[2][4];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int m = m0 + u;
+            uint32_t &a0 = af[u][0], &a1 = af[u][1], &a2 = af[u][2], &a3 = af[u][3];
+            if constexpr (BITS == 8) {
+              // bytes (row g, row g+8) of the two positions: (0, 2) and (1, 3)
+              const uint32_t X0 = vw[rb][m], X2 = vw[rb][NC + m];
+              a0 = u8pair_f16(X0, 0x4240); a1 = u8pair_f16(X0, 0x4341);
+              a2 = u8pair_f16(X2, 0x4240); a3 = u8pair_f16(X2, 0x4341);
+            } else if constexpr (BITS == 2) {
+              // byte (m/2) % 2 of each half, field 2 (m % 2) (row g) and
+              // 2 (m % 2) + 1 (row g+8): weights 4^(2 (m%2)) and 4^(2 (m%2) + 1)
+              const int sh = (m & 2) * 4;
+              const uint32_t X0 = vw[rb][m >> 2] >> sh, X2 = vw[rb][NC + (m >> 2)] >> sh;
+              const uint32_t mg = 0x00030003u << (4 * (m & 1)), mh = 0x000C000Cu << (4 * (m & 1));
+              a0 = X0 & mg; a1 = X0 & mh;
+              a2 = X2 & mg; a3 = X2 & mh;
+            } else {
+              // bytes 0 and 2 (even m) or 1 and 3 (odd m): row g in the low
+              // nibble, row g+8 in the high nibble (16x, undone at the end)
+              const int sh = 8 * (m & 1);
+              const uint32_t X0 = vw[rb][m >> 1] >> sh, X2 = vw[rb][NC + (m >> 1)] >> sh;
+              a0 = nib_f16(X0, 0x000F000Fu); a1 = nib_f16(X0, 0x00F000F0u);
+              a2 = nib_f16(X2, 0x000F000Fu); a3 = nib_f16(X2, 0x00F000F0u);
+            }
           }
-          mma_f16(acc[m], a0, a1, a2, a3, pf[rb][0], pf[rb][1]);
-          mma_f16(acc[m], a0, a1, a2, a3, pf[rb][2], pf[rb][3]);
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int u = 0; u < 2; ++u)
+              mma_f16(acc[m0 + u], af[u][0], af[u][1], af[u][2], af[u][3], pf[rb][2 * h],
+                      pf[rb][2 * h + 1]);
         }
       }
     }
@@ -880,6 +900,8 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     cp_async_wait<0>();
   }
   __syncthreads();
+
+  pdl_trigger();  // the next kernel may be scheduled as this grid retires
 
   // ---- finish this warp's state ------------------------------------------
 #pragma unroll
@@ -956,8 +978,7 @@ cudaError_t launch_gqa_decode_g(const GqaDecodeArgs &a, cudaStream_t st) {
     attr_set = true;
   }
   dim3 grid(a.n_splits, a.v.Hkv, a.v.B);
-  k<<<grid, 128, C::SMEM, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k, grid, dim3(128), C::SMEM, st, a);
 }
 
 template <int BITS, int D, int KAX, int GS>

@@ -21,6 +21,8 @@ template <int SB>
 __global__ void __launch_bounds__(128)
     splitk_merge_kernel(const float *__restrict__ P, int S, int n_rows, int dim,
                         float *__restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   const int width = dim >= 128 ? 128 : dim;  // threads per row
   const int rpc = 128 / width, r_in = (int)threadIdx.x / width;
   const int row = blockIdx.x * rpc + r_in;
@@ -59,6 +61,8 @@ __global__ void __launch_bounds__(128)
 __global__ void __launch_bounds__(128)
     splitk_merge_kernel_n(const float *__restrict__ P, int S, int n_rows, int dim,
                           float *__restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   const int width = dim >= 128 ? 128 : dim;  // threads per row
   const int rpc = 128 / width, r_in = (int)threadIdx.x / width;
   const int row = blockIdx.x * rpc + r_in;
@@ -84,6 +88,8 @@ __global__ void __launch_bounds__(128)
 }
 
 __global__ void rewind_kernel(const RewindArgs a) {
+  pdl_wait();
+  pdl_trigger();
   for (int i = threadIdx.x; i < a.n_anchors * a.B; i += blockDim.x) {
     int32_t *l = a.lens[i / a.B] + (i % a.B);
     *l = max(0, *l - a.n);
@@ -93,8 +99,7 @@ __global__ void rewind_kernel(const RewindArgs a) {
 }  // namespace
 
 cudaError_t launch_rewind(const RewindArgs &a, cudaStream_t st) {
-  rewind_kernel<<<1, 256, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(rewind_kernel, dim3(1), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_splitk_merge(const float *partials, int n_splits, int n_rows, int dim,
@@ -104,12 +109,11 @@ cudaError_t launch_splitk_merge(const float *partials, int n_splits, int n_rows,
   const int rpc = dim >= 128 ? 1 : 128 / dim;
   const int grid = (n_rows + rpc - 1) / rpc;
   if (n_splits <= 8)
-    splitk_merge_kernel<8><<<grid, 128, 0, st>>>(partials, n_splits, n_rows, dim, out);
+    return launch_pdl(splitk_merge_kernel<8>, grid, dim3(128), 0, st, partials, n_splits, n_rows, dim, out);
   else if (n_splits <= 16)
-    splitk_merge_kernel<16><<<grid, 128, 0, st>>>(partials, n_splits, n_rows, dim, out);
+    return launch_pdl(splitk_merge_kernel<16>, grid, dim3(128), 0, st, partials, n_splits, n_rows, dim, out);
   else
-    splitk_merge_kernel_n<<<grid, 128, 0, st>>>(partials, n_splits, n_rows, dim, out);
-  return cudaGetLastError();
+    return launch_pdl(splitk_merge_kernel_n, grid, dim3(128), 0, st, partials, n_splits, n_rows, dim, out);
 }
 
 }  // namespace kvk

@@ -40,6 +40,7 @@ __global__ void __launch_bounds__(128)
     mla_absorb_kernel(const uint16_t *__restrict__ q_nope, const uint16_t *__restrict__ q_pe,
                       const uint16_t *__restrict__ w_uk, int B, int H, int r,
                       uint16_t *__restrict__ qlat) {
+  pdl_wait();
   constexpr int Dn = 128;
   __shared__ __align__(16) uint16_t a_s[16 * Dn];  // [b][j], swizzled 16B chunks
   __shared__ __align__(16) uint16_t w_s[Dn * 64];  // [j][i], swizzled
@@ -47,18 +48,23 @@ __global__ void __launch_bounds__(128)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c = lane & 3;
   constexpr int QROW = 2 * W + kRope;
+  // every operand chunk in flight at once (asynchronous 16-byte copies;
+  // rows past the batch are zero-filled)
+#pragma unroll
   for (int q = tid; q < 16 * Dn / 8; q += 128) {
     const int row = q / (Dn / 8), u = q % (Dn / 8);
     const int b = b0 + row;
-    uint4 x = make_uint4(0, 0, 0, 0);
-    if (b < B) x = *reinterpret_cast<const uint4 *>(q_nope + ((size_t)b * H + h) * Dn + 8 * u);
-    *reinterpret_cast<uint4 *>(a_s + row * Dn + 8 * swz8(row, u)) = x;
+    cp_async16(a_s + row * Dn + 8 * swz8(row, u),
+               q_nope + ((size_t)(b < B ? b : 0) * H + h) * Dn + 8 * u, b < B);
   }
+#pragma unroll
   for (int q = tid; q < Dn * 8; q += 128) {
     const int j = q / 8, u = q % 8;
-    const uint4 x = *reinterpret_cast<const uint4 *>(w_uk + ((size_t)h * Dn + j) * r + i0 + 8 * u);
-    *reinterpret_cast<uint4 *>(w_s + j * 64 + 8 * swz8(j, u)) = x;
+    cp_async16(w_s + j * 64 + 8 * swz8(j, u), w_uk + ((size_t)h * Dn + j) * r + i0 + 8 * u, true);
   }
+  cp_async_commit();
+  cp_async_wait<0>();
+  pdl_trigger();
   __syncthreads();
   float acc[2][4] = {};
   const int mat = lane >> 3, rr = lane & 7;
@@ -256,6 +262,7 @@ __global__ void __launch_bounds__(192, 1)
                       const uint16_t *__restrict__ qlat, const uint16_t *__restrict__ q_pe, int H,
                       float sig, int items_per_split, int n_splits, float *__restrict__ partial,
                       int32_t *err) {
+  pdl_wait();
   using C = MlaCfg<W>;
   constexpr int TR = C::TR;
   extern __shared__ uint8_t smem_raw[];
@@ -351,6 +358,7 @@ __global__ void __launch_bounds__(192, 1)
         mbar_wait(&full[u % C::NST], (u / C::NST) & 1, kLimit);
     }
     __syncwarp();
+    pdl_trigger();
   } else if (warp == 4) {
     // ======================= MMA warp =====================================
     constexpr uint32_t ID_S = umma_idesc(64, 32, false, false);
@@ -415,6 +423,7 @@ __global__ void __launch_bounds__(192, 1)
       mbar_wait(dbar, 0, kLimit);
     }
     __syncwarp();
+    pdl_trigger();
   } else {
     // ======================= softmax warps ================================
     const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
@@ -507,6 +516,7 @@ __global__ void __launch_bounds__(192, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&pbar[t & 1]);  // one of the four arrivals
     }
+    pdl_trigger();
     // ---- partial of this split: O^T columns h + 16+h, m, l ------------------
     if (!failed && n_tiles > 0) {
       const int t = n_tiles - 1;
@@ -581,6 +591,7 @@ __global__ void __launch_bounds__(128)
     mla_merge_upv_kernel(const float *__restrict__ partial, int n_splits,
                          const uint16_t *__restrict__ w_uv, int B, int H, int r,
                          float *__restrict__ out) {
+  pdl_wait();
   constexpr int Dv = 128;
   constexpr int OST = W + 8;  // padded rows (bf16): conflict-free ldmatrix
   extern __shared__ __align__(128) uint8_t dyn_smem[];
@@ -672,6 +683,7 @@ __global__ void __launch_bounds__(128)
     *reinterpret_cast<uint32_t *>(ol_s + row * OST + i) = lo;
   }
   cp_async_wait<0>();
+  pdl_trigger();
   __syncthreads();
   const int mat = lane >> 3, rr = lane & 7;
   float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};
@@ -702,31 +714,31 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
   using C = MlaCfg<W>;
   if (a.n_splits > 64) return cudaErrorInvalidValue;  // merge weights hold 64 splits
   const int B = a.v.B;
-  mla_absorb_kernel<W><<<dim3(W / 64, a.H, (B + 15) / 16), 128, 0, st>>>(
-      static_cast<const uint16_t *>(a.q_nope), static_cast<const uint16_t *>(a.q_pe),
-      static_cast<const uint16_t *>(a.w_uk), B, a.H, a.r, a.qlat);
   auto k = mla_decode_kernel<W>;
+  constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(mla_merge_upv_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               MU_SMEM);
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  k<<<dim3(a.n_splits, B), 192, C::SMEM, st>>>(*static_cast<const CUtensorMap *>(a.tmap), a.v,
-                                                a.qlat, static_cast<const uint16_t *>(a.q_pe),
-                                                a.H, a.sig_log2, a.items_per_split, a.n_splits,
-                                                a.partial, a.err);
-  constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
-  static bool mu_attr = false;
-  if (!mu_attr) {
-    cudaError_t e2 = cudaFuncSetAttribute(mla_merge_upv_kernel<W>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize, MU_SMEM);
-    if (e2 != cudaSuccess) return e2;
-    mu_attr = true;
-  }
-  mla_merge_upv_kernel<W><<<dim3(a.H, (B + 15) / 16, 4), 128, MU_SMEM, st>>>(
-      a.partial, a.n_splits, static_cast<const uint16_t *>(a.w_uv), B, a.H, a.r, a.out);
-  return cudaGetLastError();
+  cudaError_t e = launch_pdl(mla_absorb_kernel<W>, dim3(W / 64, a.H, (B + 15) / 16), dim3(128), 0,
+                             st, static_cast<const uint16_t *>(a.q_nope),
+                             static_cast<const uint16_t *>(a.q_pe),
+                             static_cast<const uint16_t *>(a.w_uk), B, a.H, a.r, a.qlat);
+  if (e == cudaSuccess)
+    e = launch_pdl(k, dim3(a.n_splits, B), dim3(192), C::SMEM, st,
+                   *static_cast<const CUtensorMap *>(a.tmap), a.v,
+                   static_cast<const uint16_t *>(a.qlat), static_cast<const uint16_t *>(a.q_pe),
+                   a.H, a.sig_log2, a.items_per_split, a.n_splits, a.partial, a.err);
+  if (e == cudaSuccess)
+    e = launch_pdl(mla_merge_upv_kernel<W>, dim3(a.H, (B + 15) / 16, 4), dim3(128), MU_SMEM, st,
+                   static_cast<const float *>(a.partial), a.n_splits,
+                   static_cast<const uint16_t *>(a.w_uv), B, a.H, a.r, a.out);
+  return e;
 }
 
 template <int W>
