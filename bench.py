@@ -335,7 +335,7 @@ def main():
     ap.add_argument("--sym-bits", type=int, choices=[8, 4, 2], default=None,
                     help="store the quantised anchors with the symmetric per-vector "
                          "quantiser at this bit-width")
-    ap.add_argument("--profile-case", choices=["gqa", "mla", "gather", "sym"], default=None,
+    ap.add_argument("--profile-case", choices=["gqa", "mla", "mla64", "gather", "sym"], default=None,
                     help="small ncu case: decode launches only, no timing line")
     args = ap.parse_args()
     if args.impl == "reference":
@@ -573,7 +573,8 @@ def profile_case(kind):
     """The kernel-level ncu case.  gqa: one int4 g32 and one bf16 anchor at
     the 14B step shape (B=32, 8 kv / 40 q heads, d_h 128, T=8192; 1.5 GB of
     cache, both anchors larger than L2); each decode runs 3 times in the order
-    int4, bf16.  mla: one d=512 latent layer at B=64, T=4096 (302 MB).
+    int4, bf16.  mla / mla64: one d=512 (302 MB) / d=64 (67 MB) latent layer
+    at B=64, T=4096.
     gather: one int4 g32 anchor at B=4, T=131072 with a kept list of T/8
     positions per sequence (805 MB cache, 101 MB read per decode), 3 decodes.
     sym: one symmetric anchor of each bit-width (8, 4, 2) at the 14B step
@@ -626,10 +627,11 @@ def profile_case(kind):
         for _ in range(3):
             c.decode(0, q, w.sigma)
     else:
+        width = 64 if kind == "mla64" else 512
         w = W.config(4, n_layers=1)
-        w.layers[0]["width"] = 512
+        w.layers[0]["width"] = width
         c = Cache(kind="mla", n_layers=1, n_q_heads=16, head_dim=128, latent_dim=512, rope_dim=64,
-                  max_batch=w.batch, max_ctx=w.context, layers=[Layer(bits=16, width=512)])
+                  max_batch=w.batch, max_ctx=w.context, layers=[Layer(bits=16, width=width)])
         cl, kr = W.mla_inputs(w, 0, 0, w.context, device="cuda")
         c.append(0, cl, kr)
         wk, wv = W.mla_weights(w, 0, device="cuda")

@@ -15,6 +15,8 @@
 // hi + lo bf16 halves, so products keep ~16 significant bits.
 #include <math.h>
 
+#include <algorithm>
+
 #include <cuda.h>  // CUtensorMap and its enums (the encoder is reached through the runtime)
 
 #include "common.cuh"
@@ -709,6 +711,20 @@ __global__ void __launch_bounds__(128)
   }
 }
 
+// Kernel attributes of the latent decode: its dynamic shared memory, and the
+// largest shared-memory carveout (with no preference the occupancy query
+// sizes the carveout for one CTA per SM, although two CTAs of the narrower
+// widths fit).
+template <int W>
+cudaError_t mla_decode_attrs() {
+  auto k = mla_decode_kernel<W>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, MlaCfg<W>::SMEM);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
+  return e;
+}
+
 template <int W>
 cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
   using C = MlaCfg<W>;
@@ -718,7 +734,7 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
   constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e = mla_decode_attrs<W>();
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(mla_merge_upv_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                MU_SMEM);
@@ -741,13 +757,29 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
   return e;
 }
 
+// Latent decode CTAs that fit on one SM, from the kernel's registers and
+// shared memory and its TMEM columns (the runtime's occupancy query answers
+// one for this kernel at any size, while two CTAs of the narrower widths do
+// run side by side).
 template <int W>
 int mla_ctas_t() {
   using C = MlaCfg<W>;
   auto k = mla_decode_kernel<W>;
-  cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-  int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 192, C::SMEM) != cudaSuccess) n = 1;
+  if (mla_decode_attrs<W>() != cudaSuccess) return 1;
+  cudaFuncAttributes fa;
+  int dev = 0, smem_sm = 0, regs_sm = 0, resv = 0;
+  if (cudaFuncGetAttributes(&fa, k) != cudaSuccess || cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&resv, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess)
+    return 1;
+  const int warp_regs = (fa.numRegs * 32 + 255) / 256 * 256;  // allocation unit: 256
+  const int by_regs = regs_sm / (6 * warp_regs);
+  const int by_smem = smem_sm / (C::SMEM + resv);
+  const int by_tmem = 512 / C::TCOLS;
+  const int n = std::min(std::min(by_regs, by_smem), std::min(by_tmem, 2048 / 192));
   return n > 0 ? n : 1;
 }
 
