@@ -335,7 +335,8 @@ def main():
     ap.add_argument("--sym-bits", type=int, choices=[8, 4, 2], default=None,
                     help="store the quantised anchors with the symmetric per-vector "
                          "quantiser at this bit-width")
-    ap.add_argument("--profile-case", choices=["gqa", "mla", "mla64", "gather", "sym"], default=None,
+    ap.add_argument("--profile-case", choices=["gqa", "kpc", "mla", "mla64", "gather", "sym"],
+                    default=None,
                     help="small ncu case: decode launches only, no timing line")
     args = ap.parse_args()
     if args.impl == "reference":
@@ -578,7 +579,9 @@ def profile_case(kind):
     gather: one int4 g32 anchor at B=4, T=131072 with a kept list of T/8
     positions per sequence (805 MB cache, 101 MB read per decode), 3 decodes.
     sym: one symmetric anchor of each bit-width (8, 4, 2) at the 14B step
-    shape (2.2 GB of cache), each decoded 3 times."""
+    shape (2.2 GB of cache), each decoded 3 times.  kpc: per-channel keys at
+    the 7B step shape, one int4 g32 and one int8 g64 anchor (250 MB), 3
+    decodes each."""
     import torch
     from __graft_entry__ import build
     build()
@@ -592,6 +595,23 @@ def profile_case(kind):
                   max_ctx=8192, layers=layers)
         for l in range(2):
             k, v = W.kv_inputs(w, l, 0, 8192, device="cuda")
+            c.append(l, k, v)
+            del k, v
+        q = W.queries(w, 0, device="cuda")
+        for _ in range(3):
+            for l in range(2):
+                c.decode(l, q, w.sigma)
+    elif kind == "kpc":
+        # per-channel keys at the 7B step shape: one int4 g32 and one int8
+        # g64 anchor (B=16, 4 kv / 28 q heads, T=8192)
+        w = W.config(2)
+        layers = [Layer(bits=4, group=32, key_axis="channel"),
+                  Layer(bits=8, group=64, key_axis="channel")]
+        c = Cache(n_layers=2, n_q_heads=28, n_kv_heads=4, head_dim=128, max_batch=16,
+                  max_ctx=8192, layers=layers)
+        a0 = w.anchors[0]
+        for l in range(2):
+            k, v = W.kv_inputs(w, a0, 0, 8192, device="cuda")
             c.append(l, k, v)
             del k, v
         q = W.queries(w, 0, device="cuda")

@@ -89,17 +89,29 @@ struct GqaCfg {
   static constexpr int SC_OFF_T = TILE * REC;     // symmetric: one scale word per row
   static constexpr int STAGE = TMA ? KG_OFF_T + KG_ROWS * D * 8 + (SYM ? TILE * 4 : 0)
                                    : KG_OFF + KG_ROWS * D * 8;
-  static constexpr int NST = TMA ? (STAGE <= 13312 ? 4 : (STAGE <= 20480 ? 3 : 2)) : 2;
-  static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");
   static constexpr int QSTR = D + 4;  // padded query row (floats): conflict-free head rows
   static constexpr int Q_BYTES = 8 * QSTR * 4 + 2 * 8 * NG * 4;
+  // per-channel keys: the query folded with each group's scales, once per
+  // tile, in the score MMA's fragment order ([KG_ROWS][KS][32] x 16 bytes),
+  // and the zero-point terms per warp ([4][KG_ROWS][8] floats)
+  static constexpr int FOLD_BYTES = KPC ? KG_ROWS * KS * 32 * 16 : 0;
+  static constexpr int ZRED_BYTES = KPC ? 4 * KG_ROWS * 8 * 4 : 0;
+  // stages: four where they and the rest fit four CTAs per SM (57 KB each),
+  // else three or two by stage size
+  static constexpr int FIXED = Q_BYTES + FOLD_BYTES + ZRED_BYTES + 24 * 4;
+  static constexpr int NST = !TMA ? 2
+                             : KPC ? (FIXED + 4 * STAGE <= 57344 ? 4 : (FIXED + 3 * STAGE <= 57344 ? 3 : (STAGE <= 20480 ? 3 : 2)))
+                                   : (STAGE <= 13312 ? 4 : (STAGE <= 20480 ? 3 : 2));
+  static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");
   static constexpr int BAR_OFF = Q_BYTES + NST * STAGE;
   static constexpr int GMASK_OFF = BAR_OFF + (TMA ? 8 * NST : 0);
-  static constexpr int SMEM = GMASK_OFF + (TMA ? 16 * NST : 0);
+  static constexpr int FOLD_OFF = (GMASK_OFF + (TMA ? 16 * NST : 0) + 15) & ~15;  // 16-byte stores
+  static constexpr int SMEM = FOLD_OFF + FOLD_BYTES + ZRED_BYTES;
   // CTAs per SM the register budget is sized for: four where four fit in
   // shared memory (228 KB per SM, 1 KB reserved per CTA), else three
   static constexpr int MIN_CTAS = (!BF && 4 * (SMEM + 1024) <= 233472) ? 4 : 3;
   static_assert(REC % 16 == 0, "records are 16-byte multiples");
+  static_assert(Q_BYTES % 16 == 0 && STAGE % 16 == 0 && FOLD_OFF % 16 == 0, "16-byte aligned regions");
   static_assert(BITS != 2 || SYM, "2-bit codes exist for the symmetric scheme only");
   static_assert(!SYM || (D == 128 && GS == D), "symmetric rows are 128 channels, one group");
   static_assert(!QUANT || (GS % 16 == 0 && D % GS == 0), "groups are whole k-steps");
@@ -480,6 +492,50 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     else return reinterpret_cast<const float2 *>(st + C::KG_OFF);
   };
 
+  // ---- per-channel keys: the query folded with the key scales -------------
+  // For each group slot of the tile, head n's query times the group's
+  // per-channel scales, split hi/lo f16 in the B-fragment order of the score
+  // MMA (k-step js, lane), plus each warp's share of sum_ch q[n][ch]
+  // zero[ch].  Built once per tile by all threads (every block of a group
+  // reads it) instead of by every warp for its own block.  Slots of groups
+  // that are not complete hold garbage that no block reads (those rows are
+  // scored from the bf16 residual).
+  uint4 *fold = reinterpret_cast<uint4 *>(smem + C::FOLD_OFF);
+  float *zred = reinterpret_cast<float *>(smem + C::FOLD_OFF + C::FOLD_BYTES);
+  auto fold_query = [&](int s) {
+    static_assert(!C::KPC || KS % 4 == 0, "k-steps split evenly over the four warps");
+    const float2 *kg0 = kg_rows(stages + s * C::STAGE);
+    float zp[C::KPC ? C::KG_ROWS : 1];
+#pragma unroll
+    for (int gs = 0; gs < (C::KPC ? C::KG_ROWS : 1); ++gs) zp[gs] = 0.f;
+#pragma unroll
+    for (int k = 0; k < C::KG_ROWS * KS / 4; ++k) {
+      const int gs = (4 * k) / KS, js = warp + (4 * k) % KS;
+      const float *qh = q_s + g * QSTR + 16 * js;
+      const float2 *sz = kg0 + gs * D + 16 * js;
+      float x[4];
+      const int chs[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 m2 = sz[chs[e]];
+        zp[gs] += qh[chs[e]] * m2.y;
+        x[e] = qh[chs[e]] * m2.x;
+        if (BITS == 4 && e >= 2) x[e] *= 0.0625f;
+      }
+      uint32_t h0, l0, h1, l1;
+      split2<false>(x[0], x[1], h0, l0);
+      split2<false>(x[2], x[3], h1, l1);
+      fold[(gs * KS + js) * 32 + lane] = make_uint4(h0, h1, l0, l1);
+    }
+#pragma unroll
+    for (int gs = 0; gs < (C::KPC ? C::KG_ROWS : 1); ++gs) {
+      float z = zp[gs];
+      z += __shfl_xor_sync(0xffffffffu, z, 1);
+      z += __shfl_xor_sync(0xffffffffu, z, 2);
+      if (c == 0 && C::KPC) zred[(warp * C::KG_ROWS + gs) * 8 + g] = z;
+    }
+  };
+
   // ---- consumer: one warp's RB blocks of 16 rows of one stage ------------
   constexpr int RB = C::RB;
   auto compute = [&](int t, int s) {
@@ -574,45 +630,34 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
 #pragma unroll
         for (int k = 0; k < 4; ++k) s4[rb][k] = d[k] * kCodeUnit;  // scores carry 2^-24
       } else if constexpr (C::KPC) {
-        // scale of each channel folded into the query for this group of
-        // positions; the zero points enter as one per-head constant.
-        const float2 *kg = kg_rows(st) + (r0 / GS) * D;
-        uint32_t pb[KS][2], pbl[KS][2];
-        float zpart = 0.f;
+        // the query folded with this group's per-channel scales (built for
+        // the tile by fold_query), the zero points entering as one per-head
+        // constant in the 2^-24 units of the MMA
+        const int gs = r0 / GS;
+        const uint4 *fg = fold + gs * KS * 32 + lane;
+        float2 z2 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int js = 0; js < KS; ++js) {
-          const float *qh = q_s + g * QSTR + 16 * js;
-          const float2 *sz = kg + 16 * js;
-          float x[4];
-          const int chs[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 m2 = sz[chs[e]];
-            zpart += qh[chs[e]] * m2.y;
-            x[e] = qh[chs[e]] * m2.x;
-            if (BITS == 4 && e >= 2) x[e] *= 0.0625f;
-          }
-          split2<false>(x[0], x[1], pb[js][0], pbl[js][0]);
-          split2<false>(x[2], x[3], pb[js][1], pbl[js][1]);
+        for (int w = 0; w < 4; ++w) {
+          const float2 zw = *reinterpret_cast<const float2 *>(zred + (w * C::KG_ROWS + gs) * 8 + 2 * c);
+          z2.x += zw.x;
+          z2.y += zw.y;
         }
-        zpart += __shfl_xor_sync(0xffffffffu, zpart, 1);
-        zpart += __shfl_xor_sync(0xffffffffu, zpart, 2);
-        const float corr = zpart * kCodeUnit;  // head g, in the 2^-24 units of the MMA
-        const float corr0 = __shfl_sync(0xffffffffu, corr, (2 * c) * 4);
-        const float corr1 = __shfl_sync(0xffffffffu, corr, (2 * c + 1) * 4);
+        const float corr0 = z2.x * kCodeUnit, corr1 = z2.y * kCodeUnit;
         uint32_t wa[C::NWK], wb[C::NWK];
         load_k(tA, wa);
         load_k(tB, wb);
-        float d[4] = {corr0, corr1, corr0, corr1};
+        // hi and lo products in two accumulator chains
+        float d[4] = {corr0, corr1, corr0, corr1}, dl[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int js = 0; js < KS; ++js) {
           uint32_t a0, a1, a2, a3;
           kfrag(wa, wb, js, a0, a1, a2, a3);
-          mma_f16(d, a0, a1, a2, a3, pb[js][0], pb[js][1]);
-          mma_f16(d, a0, a1, a2, a3, pbl[js][0], pbl[js][1]);
+          const uint4 f = fg[js * 32];
+          mma_f16(d, a0, a1, a2, a3, f.x, f.y);
+          mma_f16(dl, a0, a1, a2, a3, f.z, f.w);
         }
 #pragma unroll
-        for (int k = 0; k < 4; ++k) s4[rb][k] = d[k];
+        for (int k = 0; k < 4; ++k) s4[rb][k] = d[k] + dl[k];
       } else {
         uint32_t wa[C::NWK], wb[C::NWK];
         load_k(tA, wa);
@@ -887,6 +932,10 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     const int nt = t + C::NST - 1;
     if (nt < n_tiles) issue(nt, nt % C::NST);
     if (use_cp) cp_async_commit();
+    if constexpr (C::KPC) {
+      fold_query(t % C::NST);
+      __syncthreads();
+    }
     compute(t, t % C::NST);
   }
   if (!use_cp) {
