@@ -264,7 +264,6 @@ __global__ void __launch_bounds__(192, 1)
                       const uint16_t *__restrict__ qlat, const uint16_t *__restrict__ q_pe, int H,
                       float sig, int items_per_split, int n_splits, float *__restrict__ partial,
                       int32_t *err) {
-  pdl_wait();
   using C = MlaCfg<W>;
   constexpr int TR = C::TR;
   extern __shared__ uint8_t smem_raw[];
@@ -304,14 +303,22 @@ __global__ void __launch_bounds__(192, 1)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  // query operand, K-major core layout: row n, coordinate k at
+  tc_fence_before();
+  __syncthreads();  // barriers initialised, TMEM address published
+  tc_fence_after();
+  // The copy warp streams the cache at once: this kernel's CTAs start only
+  // after every CTA of the absorb kernel passed its own wait for the work
+  // enqueued before the call (which wrote the cache and the lengths).  The
+  // other warps wait for the absorb itself before reading its q_lat.
+  // Query operand, K-major core layout: row n, coordinate k at
   // (n/8) SBO + (k/8) 128 + (n%8) 16 + (k%8) 2 with SBO = (W+64)/8 128.
   // Rows 0-15: [q_lat hi | q_pe] of head n; rows 16-31: [q_lat lo | 0] of
   // head n-16.
-  {
+  if (warp != 5) {
+    pdl_wait();
     constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (unused 64) | lo(W)]
     const uint16_t *qb = qlat + (size_t)b * H * QROW;
-    for (int q = tid; q < 32 * (C::KH / 8); q += 192) {  // 16-byte cp.async, zero-filled
+    for (int q = tid; q < 32 * (C::KH / 8); q += 160) {  // 16-byte cp.async, zero-filled
       const int n = q / (C::KH / 8), c = q % (C::KH / 8);
       const int h = n & 15;
       const uint16_t *src = qb;
@@ -324,11 +331,11 @@ __global__ void __launch_bounds__(192, 1)
     }
     cp_async_commit();
     cp_async_wait<0>();
+    fence_proxy_async();
+    tc_fence_before();
+    asm volatile("bar.sync 2, 160;" ::: "memory");  // warps 0-4: the query is staged
+    tc_fence_after();
   }
-  fence_proxy_async();
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
   const uint32_t tmem = *tbase;
   const uint32_t t_o = tmem, t_s = tmem + C::OCOLS;  // O columns, then two S buffers
   auto stage = [&](int s) { return sm + s * C::STAGE; };
@@ -593,7 +600,6 @@ __global__ void __launch_bounds__(128)
     mla_merge_upv_kernel(const float *__restrict__ partial, int n_splits,
                          const uint16_t *__restrict__ w_uv, int B, int H, int r,
                          float *__restrict__ out) {
-  pdl_wait();
   constexpr int Dv = 128;
   constexpr int OST = W + 8;  // padded rows (bf16): conflict-free ldmatrix
   extern __shared__ __align__(128) uint8_t dyn_smem[];
@@ -605,12 +611,17 @@ __global__ void __launch_bounds__(128)
   const int h = blockIdx.x, b0 = blockIdx.y * 16, o0 = blockIdx.z * 32;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c = lane & 3;
-  // prefetch this CTA's 32 rows of W_UV[h][:, :W]
+  // prefetch this CTA's 32 rows of W_UV[h][:, :W].  Issued before the wait
+  // for the decode kernel: this kernel's CTAs start only after the decode's
+  // CTAs passed their own wait, which followed the absorb, whose CTAs in turn
+  // waited for everything the caller enqueued before the call; the partials,
+  // the decode's output, are read after the wait.
   for (int q = tid; q < 32 * (W / 8); q += 128) {
     const int o = q / (W / 8), u = q % (W / 8);
     cp_async16(w_s + o * OST + 8 * u, w_uv + ((size_t)h * Dv + o0 + o) * r + 8 * u, true);
   }
   cp_async_commit();
+  pdl_wait();
   const size_t RS = (size_t)W + 2;
   const size_t pstride = (size_t)B * H * RS;
   // merge weights: every split's (m, l) of the 16 rows loaded at once
