@@ -495,30 +495,55 @@ def main():
     # ---- end to end through the public API, host buffers --------------------
     e2e = None
     if args.e2e_steps > 0 and w.kind == "gqa":
-        h_q = [q.cpu().pin_memory() for q in qs]
-        h_kv = {a: (k.cpu().pin_memory(), v.cpu().pin_memory()) for a, (k, v) in new_kv.items()}
-        h_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
-        d_q = [torch.empty_like(q) for q in qs]
-        d_kv = {a: (torch.empty_like(k), torch.empty_like(v)) for a, (k, v) in new_kv.items()}
-        h2d = sum(q.numel() * q.element_size() for q in h_q) + \
-            sum(k.numel() * k.element_size() * 2 for k, _ in h_kv.values())
-        d2h = sum(o.numel() * o.element_size() for o in h_out)
+        # one pinned host buffer and one device buffer per kind of tensor, so
+        # that a step's inputs arrive in two copies and its outputs leave in one
+        # (per-layer copies cost more in fixed latency than in bytes)
+        h_q_all = torch.stack([q.cpu() for q in qs]).pin_memory()
+        d_q_all = torch.empty_like(h_q_all, device=dev)
+        d_q = list(d_q_all.unbind(0))
+        kv_layers = sorted(new_kv)
+        h_kv_all = (torch.stack([t for a in kv_layers for t in new_kv[a]]).cpu().pin_memory()
+                    if kv_layers else None)
+        d_kv_all = torch.empty_like(h_kv_all, device=dev) if kv_layers else None
+        d_kv = {a: (d_kv_all[2 * i], d_kv_all[2 * i + 1]) for i, a in enumerate(kv_layers)}
+        e_out_all = torch.empty((w.n_layers,) + tuple(outs[0].shape), dtype=outs[0].dtype, device=dev)
+        e_outs = list(e_out_all.unbind(0))
+        h_out_all = torch.empty(e_out_all.shape, dtype=e_out_all.dtype).pin_memory()
+        h2d = h_q_all.numel() * h_q_all.element_size() + \
+            (h_kv_all.numel() * h_kv_all.element_size() if kv_layers else 0)
+        d2h = h_out_all.numel() * h_out_all.element_size()
+        e2e_mode = "eager"
         with torch.cuda.stream(stream):
-            def e2e_step():
-                for l in range(w.n_layers):
-                    d_q[l].copy_(h_q[l], non_blocking=True)
-                for a in d_kv:
-                    d_kv[a][0].copy_(h_kv[a][0], non_blocking=True)
-                    d_kv[a][1].copy_(h_kv[a][1], non_blocking=True)
+            def e2e_body():
+                d_q_all.copy_(h_q_all, non_blocking=True)
+                if kv_layers:
+                    d_kv_all.copy_(h_kv_all, non_blocking=True)
                 for l in range(w.n_layers):
                     if l in d_kv:
                         cache.append(l, *d_kv[l])
-                    cache.decode(l, d_q[l], w.sigma, out=outs[l])
-                    h_out[l].copy_(outs[l], non_blocking=True)
+                    cache.decode(l, d_q[l], w.sigma, out=e_outs[l])
+                h_out_all.copy_(e_out_all, non_blocking=True)
                 if w.append_per_step:
                     cache.rewind(1)
+
+            def e2e_step():
+                e2e_body()
                 stream.synchronize()
             e2e_step()
+            # the same API calls and pinned-host copies recorded once as a CUDA
+            # graph: every replay copies the step's inputs in and its outputs out
+            try:
+                g_e2e = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g_e2e, stream=stream):
+                    e2e_body()
+
+                def e2e_step():
+                    g_e2e.replay()
+                    stream.synchronize()
+                e2e_step()
+                e2e_mode = "cuda graph of the API calls and host copies"
+            except Exception:  # capture unsupported: stay eager
+                torch.cuda.synchronize()
             barrier()
             t0 = time.perf_counter()
             for _ in range(args.e2e_steps):
@@ -526,7 +551,7 @@ def main():
             dt = time.perf_counter() - t0
         dt = reduce_max(dt, dist, dev)
         e2e = {"value": job_throughput(step_bytes, args.e2e_steps, world, dt), "unit": UNIT,
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "launch": e2e_mode,
                "ms_per_step": dt / args.e2e_steps * 1e3}
 
     err = cache.device_error()
