@@ -58,7 +58,8 @@ def gqa_decode(q, k_hat, v_hat, lens, sigma, kept=None):
     lens   : ``[B]`` valid positions per sequence
     sigma  : softmax scale
     kept   : optional list (per sequence) of position arrays to read instead
-             of ``0..lens[b]-1``
+             of ``0..lens[b]-1``; an entry may instead be a list of arrays,
+             one per KV head (per-head kept lists)
     Returns ``[B, H_q, D]`` float64.
     """
     q = np.asarray(q, np.float64)
@@ -69,11 +70,15 @@ def gqa_decode(q, k_hat, v_hat, lens, sigma, kept=None):
     G = Hq // Hkv
     out = np.zeros((B, Hq, D), np.float64)
     for b in range(B):
-        pos = np.arange(int(lens[b])) if kept is None else np.asarray(kept[b], np.int64)
-        if pos.size == 0:
-            continue
+        per_head = kept is not None and isinstance(kept[b], (list, tuple))
         for h in range(Hq):
             j = h // G
+            if kept is None:
+                pos = np.arange(int(lens[b]))
+            else:
+                pos = np.asarray(kept[b][j] if per_head else kept[b], np.int64)
+            if pos.size == 0:
+                continue
             K = np.asarray(k_hat[b, j, pos], np.float64)
             V = np.asarray(v_hat[b, j, pos], np.float64)
             p = softmax_weights(sigma * (K @ q[b, h]))
