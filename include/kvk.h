@@ -189,9 +189,51 @@ kvk_status kvk_decode_plan_splits(kvk_cache *cache, int32_t layer, int32_t *n_sp
  * idx device int32 [B, evict_capacity] sorted ascending, n_kept device
  * int32[B] <= evict_capacity.  Decode then reads only those positions; an
  * entry past the sequence length sets KVK_DEVERR_KEPT_RANGE and is skipped.
- * n_kept == NULL clears the list (all positions are read again). */
+ * The list is shared by the sequence's KV heads (kvk_evict_window installs
+ * per-head lists).  n_kept == NULL clears the lists (all positions are read
+ * again). */
 kvk_status kvk_set_kept(kvk_cache *cache, int32_t layer, const int32_t *idx,
                         const int32_t *n_kept, kvk_stream stream);
+
+/* Attention-scored eviction composed with the compressed cache (Sec. 3.3;
+ * the paper's evictors sum attention over a 32-query observation window).
+ * For every sequence b and KV head j of anchor `layer`, each position t
+ * before the last n_win gets the attention mass that the window's queries of
+ * the heads of j put on it,
+ *   vote[b,j,t] = sum_{w < n_win} sum_{h in group j}
+ *                 softmax_{u <= p_w}(softmax_scale <q[b,w,h], k_u>)[t],
+ * p_w = len_b - n_win + w (window query w sits at position p_w and sees the
+ * positions up to itself; keys dequantised from the cache).  The budget -
+ * n_win largest votes (equal votes: the smaller position first) and the
+ * window become the kept list of (b, j), sorted; a sequence of at most
+ * `budget` positions keeps all of them.  The lists are installed as the
+ * anchor's kept lists, one per (sequence, KV head): decode then reads, for
+ * KV head j of sequence b, only its own list, until kvk_set_kept replaces or
+ * clears it.
+ *  q_win:   device [B, n_win, H_q, head_dim] in q_dtype, post-RoPE, the
+ *           queries of each sequence's last n_win positions; 1 <= n_win <= 256;
+ *  budget:  n_win <= budget <= evict_capacity;
+ *  scratch: device, 256-byte aligned, at least kvk_evict_scratch_size bytes.
+ *           Once the stream reaches the end of the call it starts with the
+ *           votes: float32 vote[b,j,t] at index (b H_kv + j) C + t, C =
+ *           max_ctx rounded up to a multiple of 64, for t < len_b - n_win of
+ *           the sequences longer than `budget` (the rest unspecified).
+ * Errors: INHERITED_LAYER (evict on the anchor), INVALID_CONFIG
+ * (evict_capacity 0), UNSUPPORTED (MLA, grouped per-channel keys),
+ * INVALID_ARG. */
+kvk_status kvk_evict_scratch_size(const kvk_cache *cache, int32_t layer, int32_t n_win,
+                                  size_t *scratch_bytes);
+kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, int32_t q_dtype,
+                            int32_t n_win, float softmax_scale, int32_t budget, void *scratch,
+                            size_t scratch_bytes, kvk_stream stream);
+
+/* Copy anchor `layer`'s kept lists out, device to device, on `stream`.
+ * *per_head (host) = -1: no list installed (nothing copied); 0: lists per
+ * sequence, idx [B, evict_capacity], n_kept [B]; 1: lists per (sequence, KV
+ * head), idx [B, H_kv, evict_capacity], n_kept [B, H_kv].  idx and n_kept
+ * are device buffers of at least the per-head sizes. */
+kvk_status kvk_export_kept(const kvk_cache *cache, int32_t layer, int32_t *idx, int32_t *n_kept,
+                           int32_t *per_head, kvk_stream stream);
 
 /* GQA decode attention of `layer` with its own query (inheritors read their
  * source anchor, Sec. 2.1):

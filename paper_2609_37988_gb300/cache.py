@@ -150,6 +150,50 @@ class Cache:
             _need(idx, "idx"); _need(n_kept, "n_kept")
         check(self.lib.kvk_set_kept(self.handle, layer, _ptr(idx), _ptr(n_kept), _stream(stream)))
 
+    def evict_window(self, layer: int, q_win: torch.Tensor, scale: float, budget: int,
+                     stream=None):
+        """Attention-scored eviction: ``q_win`` ``[B, n_win, H_q, head_dim]``,
+        the queries of each sequence's last ``n_win`` positions; installs
+        per-(sequence, KV head) kept lists of ``budget`` positions.  Returns
+        the votes, a float32 view ``[max_batch, H_kv, C]`` of the scratch
+        (valid before each window of the sequences longer than ``budget``,
+        once the stream has run the call)."""
+        _need(q_win, "q_win")
+        d = self.desc
+        if q_win.dim() != 4 or (q_win.shape[0], q_win.shape[2], q_win.shape[3]) != (
+                d.max_batch, d.n_q_heads, d.head_dim):
+            raise ValueError("q_win must be [max_batch, n_win, n_q_heads, head_dim]")
+        n_win = q_win.shape[1]
+        nbytes = ctypes.c_size_t()
+        check(self.lib.kvk_evict_scratch_size(self.handle, layer, n_win, ctypes.byref(nbytes)))
+        scratch = torch.empty(nbytes.value, dtype=torch.uint8, device=self.device)
+        check(self.lib.kvk_evict_window(self.handle, layer, _ptr(q_win), _dtype_code(q_win), n_win,
+                                        float(scale), budget, _ptr(scratch), nbytes.value,
+                                        _stream(stream)))
+        self._evict_scratch = scratch  # kept alive until the stream is done with it
+        C = (d.max_ctx + 63) // 64 * 64
+        return scratch[: 4 * d.max_batch * d.n_kv_heads * C].view(torch.float32).view(
+            d.max_batch, d.n_kv_heads, C)
+
+    def kept_lists(self, layer: int, stream=None):
+        """Installed kept lists: ``(idx, n, per_head)`` device tensors shaped
+        per head ``[B, H_kv, cap]`` / ``[B, H_kv]`` (or per sequence), or
+        ``None`` when no list is installed."""
+        d = self.desc
+        cap = self.layers[layer].evict_capacity
+        idx = torch.empty((d.max_batch, d.n_kv_heads, max(cap, 1)), dtype=torch.int32,
+                          device=self.device)
+        n = torch.empty((d.max_batch, d.n_kv_heads), dtype=torch.int32, device=self.device)
+        ph = ctypes.c_int32()
+        check(self.lib.kvk_export_kept(self.handle, layer, _ptr(idx), _ptr(n), ctypes.byref(ph),
+                                       _stream(stream)))
+        if ph.value < 0:
+            return None
+        if ph.value == 0:
+            flat_i = idx.view(-1)[: d.max_batch * cap].view(d.max_batch, cap)
+            return flat_i, n.view(-1)[: d.max_batch].clone(), False
+        return idx, n, True
+
     def rewind(self, n: int, stream=None):
         """Drop the last ``n`` positions of every sequence of every anchor."""
         check(self.lib.kvk_rewind(self.handle, n, _stream(stream)))

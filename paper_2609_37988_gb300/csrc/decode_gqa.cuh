@@ -179,14 +179,15 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   // kept-position lists exist only with per-token key metadata or bf16
   // caches (rejected by the host for per-channel keys)
   constexpr bool gather = GATHER && !C::KPC;
-  const int n_items = gather ? min(v.kept_n[b], v.kept_cap) : len;
+  const int kunit = v.kept_per_head ? b * v.Hkv + blockIdx.y : b;  // whose kept list
+  const int n_items = gather ? min(v.kept_n[kunit], v.kept_cap) : len;
   const int i0 = split * a.items_per_split;
   // the last split runs to the end, so a launch recorded for shorter
   // sequences (a replayed graph) still covers every position
   const int i1 = (split == a.n_splits - 1) ? n_items : min(i0 + a.items_per_split, n_items);
   const int Tq = C::KPC ? (len / GS) * GS : len;  // positions held as codes
   const bool use_lo = a.q_f32 != 0;
-  const int32_t *kept = v.kept_idx + (size_t)b * v.kept_cap;
+  const int32_t *kept = v.kept_idx + (size_t)kunit * v.kept_cap;
 
   // The copy producer comes first, so the first tiles are in flight while
   // the query set-up below runs.

@@ -12,11 +12,12 @@ struct GqaView {
   uint8_t *resid;      // per-channel key residual plane, or null
   int32_t *lens;       // [B]
   int32_t *counter;    // append completion counter
-  int32_t *kept_n;     // [B]
-  int32_t *kept_idx;   // [B * kept_cap]
+  int32_t *kept_n;     // [B] (shared by the kv heads) or [B * Hkv] (per head)
+  int32_t *kept_idx;   // [B * kept_cap] or [B * Hkv * kept_cap]
   uint32_t *scales;    // symmetric scheme: bf16 (K, V) scale pair per (slab, position)
   int64_t cap;         // positions per slab
   int kept_cap;
+  int kept_per_head;   // kept lists per (sequence, kv head) instead of per sequence
   int B, Hkv, D, bits, group, key_axis, rec_bytes;
   int scheme;          // kSchemeGrouped or kSchemeSym
 };
@@ -65,6 +66,25 @@ cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, i
 cudaError_t launch_mla_append(const MlaView &v, const void *c, const void *kr, int latent,
                               int n_new, const int32_t *n_per_seq, int32_t *err,
                               cudaStream_t st);
+
+// Window-vote eviction of one GQA anchor (evict.cu): votes of the positions
+// before the last n_win, top budget - n_win of them and the window written
+// as per-(sequence, kv head) kept lists into the anchor's arena.  scratch:
+// float votes [B * Hkv * cap] then float2 row statistics
+// [B * Hkv * rows * tiles] with rows = n_win * G, tiles = cap / 128.
+struct EvictArgs {
+  GqaView v;
+  const void *q;       // [B, n_win, Hq, D]
+  int q_f32;
+  int Hq, G, n_win, budget;
+  float sig_log2;      // softmax scale * log2(e)
+  int n_tiles;         // 128-position tiles launched per (sequence, kv head)
+  float *votes;
+  float2 *stats;
+  int32_t *err;
+};
+cudaError_t launch_gqa_evict(const EvictArgs &a, cudaStream_t st);
+constexpr int kEvictTile = 128;
 
 cudaError_t launch_gqa_export(const GqaView &v, void *k_out, void *v_out, float *k_scale,
                               float *k_zero, float *v_scale, float *v_zero, void *k_resid,

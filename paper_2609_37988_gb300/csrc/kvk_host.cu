@@ -195,6 +195,7 @@ struct kvk_cache {
     v.kept_idx = reinterpret_cast<int32_t *>(a + A.kept_idx);
     v.cap = A.cap;
     v.kept_cap = c.evict_capacity;
+    v.kept_per_head = kept_on[l] == 2;
     v.B = desc.max_batch;
     v.Hkv = desc.n_kv_heads;
     v.D = desc.head_dim;
@@ -527,6 +528,105 @@ kvk_status kvk_set_kept(kvk_cache *c, int32_t layer, const int32_t *idx, const i
     e = cudaMemcpyAsync(c->arena[layer] + A.kept_n, n_kept, B * 4, cudaMemcpyDeviceToDevice, st);
   if (e != cudaSuccess) return cuda_fail(e, "copying the kept list");
   c->kept_on[layer] = 1;
+  return KVK_OK;
+}
+
+namespace {
+struct EvictScratch {
+  size_t votes, stats, total;
+  int n_tiles;
+};
+EvictScratch evict_scratch(const kvk_cache *c, int layer, int n_win) {
+  EvictScratch e;
+  const size_t units = (size_t)c->desc.max_batch * c->desc.n_kv_heads;
+  const size_t cap = (size_t)c->lay[layer].cap;
+  const size_t R = (size_t)n_win * (c->desc.n_q_heads / c->desc.n_kv_heads);
+  e.n_tiles = (int)((cap + kEvictTile - 1) / kEvictTile);
+  e.votes = align256((int64_t)(units * cap * 4));
+  e.stats = align256((int64_t)((units * R * e.n_tiles + units * R) * 8));
+  e.total = e.votes + e.stats;
+  return e;
+}
+
+kvk_status check_evict(const kvk_cache *c, int32_t layer, int32_t n_win) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->desc.kind != KVK_KIND_GQA) return fail(KVK_ERR_UNSUPPORTED, "eviction scoring on an MLA cache");
+  const kvk_layer_cfg &L = c->cfg[layer];
+  if (L.inherit)
+    return fail(KVK_ERR_INHERITED_LAYER, "layer %d inherits; evict on layer %d", layer, c->src[layer]);
+  if (L.evict_capacity <= 0) return fail(KVK_ERR_INVALID_CONFIG, "layer %d has evict_capacity 0", layer);
+  if (L.bits != 16 && L.key_axis == KVK_AXIS_CHANNEL && L.scheme != KVK_QUANT_SYMMETRIC)
+    return fail(KVK_ERR_UNSUPPORTED, "layer %d: eviction with per-channel keys", layer);
+  if (n_win < 1 || n_win > 256) return fail(KVK_ERR_INVALID_ARG, "n_win %d outside [1, 256]", n_win);
+  return KVK_OK;
+}
+}  // namespace
+
+kvk_status kvk_evict_scratch_size(const kvk_cache *c, int32_t layer, int32_t n_win, size_t *bytes) {
+  kvk_status s = check_evict(c, layer, n_win);
+  if (s) return s;
+  if (!bytes) return fail(KVK_ERR_INVALID_ARG, "null output");
+  *bytes = evict_scratch(c, layer, n_win).total;
+  return KVK_OK;
+}
+
+kvk_status kvk_evict_window(kvk_cache *c, int32_t layer, const void *q_win, int32_t q_dtype,
+                            int32_t n_win, float softmax_scale, int32_t budget, void *scratch,
+                            size_t scratch_bytes, kvk_stream stream) {
+  kvk_status s = check_evict(c, layer, n_win);
+  if (s) return s;
+  const kvk_layer_cfg &L = c->cfg[layer];
+  if (budget < n_win || budget > L.evict_capacity)
+    return fail(KVK_ERR_INVALID_ARG, "budget %d outside [n_win %d, evict_capacity %d]", budget, n_win,
+                L.evict_capacity);
+  if (!q_win || !aligned16(q_win)) return fail(KVK_ERR_INVALID_ARG, "null or misaligned q_win");
+  if (q_dtype != KVK_DTYPE_F32 && q_dtype != KVK_DTYPE_BF16)
+    return fail(KVK_ERR_INVALID_ARG, "q_dtype must be F32 or BF16");
+  if (!std::isfinite(softmax_scale) || !(softmax_scale > 0.f))
+    return fail(KVK_ERR_INVALID_ARG, "softmax scale must be finite and positive");
+  const EvictScratch es = evict_scratch(c, layer, n_win);
+  if (!scratch || (reinterpret_cast<uintptr_t>(scratch) & 255u) || scratch_bytes < es.total)
+    return fail(KVK_ERR_INVALID_ARG, "scratch null, not 256-byte aligned or smaller than %zu bytes",
+                es.total);
+  EvictArgs a;
+  a.v = c->gqa_view(layer);
+  a.v.kept_per_head = 1;
+  a.q = q_win;
+  a.q_f32 = q_dtype == KVK_DTYPE_F32;
+  a.Hq = c->desc.n_q_heads;
+  a.G = c->desc.n_q_heads / c->desc.n_kv_heads;
+  a.n_win = n_win;
+  a.budget = budget;
+  a.sig_log2 = softmax_scale * 1.4426950408889634f;
+  a.n_tiles = es.n_tiles;
+  a.votes = static_cast<float *>(scratch);
+  a.stats = reinterpret_cast<float2 *>(static_cast<uint8_t *>(scratch) + es.votes);
+  a.err = c->err();
+  cudaError_t e = launch_gqa_evict(a, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "eviction launch");
+  c->kept_on[layer] = 2;  // per-(sequence, kv head) lists from now on
+  return KVK_OK;
+}
+
+kvk_status kvk_export_kept(const kvk_cache *c, int32_t layer, int32_t *idx, int32_t *n_kept,
+                           int32_t *per_head, kvk_stream stream) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->cfg[layer].inherit)
+    return fail(KVK_ERR_INHERITED_LAYER, "layer %d inherits layer %d's lists", layer, c->src[layer]);
+  if (!idx || !n_kept || !per_head) return fail(KVK_ERR_INVALID_ARG, "null output");
+  const int cap = c->cfg[layer].evict_capacity;
+  *per_head = c->kept_on[layer] == 2 ? 1 : (c->kept_on[layer] == 1 ? 0 : -1);
+  if (cap <= 0 || c->kept_on[layer] == 0) return KVK_OK;
+  const size_t units = (size_t)c->desc.max_batch * (c->kept_on[layer] == 2 ? c->desc.n_kv_heads : 1);
+  const ArenaLayout &A = c->lay[layer];
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemcpyAsync(idx, c->arena[layer] + A.kept_idx, units * cap * 4,
+                                  cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(n_kept, c->arena[layer] + A.kept_n, units * 4, cudaMemcpyDeviceToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(e, "copying the kept lists");
   return KVK_OK;
 }
 

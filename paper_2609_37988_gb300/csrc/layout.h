@@ -212,8 +212,8 @@ KVK_HD int64_t align256(int64_t x) { return (x + 255) & ~(int64_t)255; }
 struct ArenaLayout {
   int64_t lens;      // int32[B]
   int64_t counter;   // int32 (append completion counter)
-  int64_t kept_n;    // int32[B]
-  int64_t kept_idx;  // int32[B * kept_cap]
+  int64_t kept_n;    // int32[B * Hkv]: per sequence, or per (sequence, kv head)
+  int64_t kept_idx;  // int32[B * Hkv * kept_cap]
   int64_t rec;       // records
   int64_t gmeta;     // float2 [B*Hkv][cap/g][D] (per-channel keys)
   int64_t resid;     // bf16 K rows [B*Hkv][g][D] (per-channel keys)
@@ -235,9 +235,9 @@ KVK_HD ArenaLayout arena_layout(int mla, int B, int Hkv, int max_ctx, int D, int
   A.counter = off;
   off = align256(off + 4);
   A.kept_n = off;
-  off = align256(off + 4 * (int64_t)B);
+  off = align256(off + 4 * (int64_t)B * Hkv);
   A.kept_idx = off;
-  off = align256(off + 4 * (int64_t)B * kept_cap);
+  off = align256(off + 4 * (int64_t)B * Hkv * kept_cap);
   A.rec = off;
   A.scales = -1;
   if (mla) {
