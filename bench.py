@@ -335,15 +335,22 @@ def main():
     ap.add_argument("--sym-bits", type=int, choices=[8, 4, 2], default=None,
                     help="store the quantised anchors with the symmetric per-vector "
                          "quantiser at this bit-width")
-    ap.add_argument("--profile-case", choices=["gqa", "kpc", "mla", "mla64", "gather", "sym"],
+    ap.add_argument("--profile-case",
+                    choices=["gqa", "kpc", "mla", "mla64", "gather", "sym", "evict", "evict-small"],
                     default=None,
-                    help="small ncu case: decode launches only, no timing line")
+                    help="small ncu case: decode (or eviction) launches only, no timing line")
+    ap.add_argument("--evict", action="store_true",
+                    help="time the window-vote evictor at the long-context 14B shape instead "
+                         "of the decode step (one JSON line of its own)")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
         return
     if args.profile_case:
         profile_case(args.profile_case)
+        return
+    if args.evict:
+        evict_bench(args)
         return
 
     import torch
@@ -595,6 +602,96 @@ def main():
         print(json.dumps(rec))
 
 
+EVICT_WINDOW = 32
+
+
+def evict_flops(lens, n_win, G, H_kv, D, budget):
+    """Algorithmic FLOPs of one eviction call: every window query row scores
+    its causal range once (2 D per score); sequences within the budget do
+    nothing."""
+    total = 0
+    for L in lens:
+        if L <= budget:
+            continue
+        P = L - n_win
+        total += H_kv * G * sum(P + w + 1 for w in range(n_win)) * 2 * D
+    return total
+
+
+def alu_peak_tflops(sm_count, sm_mhz):
+    """FP32 FMA peak: 128 FP32 lanes per SM, 2 FLOP per FMA, at ``sm_mhz``."""
+    return sm_count * 128 * 2 * sm_mhz * 1e6 / 1e12
+
+
+def _evict_setup(B, T, dev):
+    import torch
+    from paper_2609_37988_gb300 import workloads as W
+    from paper_2609_37988_gb300.cache import Cache, Layer
+    w = W.config(5, n_layers=1, batch=B, context=T)
+    c = Cache(n_layers=1, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads, head_dim=w.head_dim,
+              max_batch=w.batch, max_ctx=T,
+              layers=[Layer(bits=4, group=32, evict_capacity=w.keep)], device=dev)
+    for b0 in range(0, T, 16384):
+        k, v = W.kv_inputs(w, 0, b0, min(T, b0 + 16384), device=dev)
+        c.append(0, k.contiguous(), v.contiguous())
+        del k, v
+    q = W.window_queries(w, 0, EVICT_WINDOW, device=dev)
+    torch.cuda.synchronize()
+    return w, c, q
+
+
+def evict_bench(args):
+    """The window-vote evictor (Sec. 3.3) at the long-context 14B shape: one
+    int4 g32 anchor, B=4, 8 KV / 40 q heads, d_h 128, 131072 cached
+    positions, a 32-query window, budget T/8.  Each call scores the window
+    against the whole cache, merges the softmax statistics, votes and selects;
+    timed with CUDA events on the launching stream (inputs: the 0.8 GB cache
+    and the 2.7 GB score buffer, both larger than L2)."""
+    import torch
+    from __graft_entry__ import build
+    build()
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    w, c, q = _evict_setup(4, 131072, dev)
+    budget = w.keep
+    for _ in range(max(3, args.warmup)):
+        c.evict_window(0, q, w.sigma, budget)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    with Clocks(0) as clk:
+        torch.cuda.synchronize()
+        for s, e in ev:
+            s.record(stream)
+            c.evict_window(0, q, w.sigma, budget)
+            e.record(stream)
+        torch.cuda.synchronize()
+    ms = [s.elapsed_time(e) for s, e in ev]
+    assert c.device_error() == 0
+    clocks = clk.summary()
+    lens = [w.context] * w.batch
+    G = w.n_q_heads // w.n_kv_heads
+    flops = evict_flops(lens, EVICT_WINDOW, G, w.n_kv_heads, w.head_dim, budget)
+    mean_ms = statistics.mean(ms)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    max_mhz = (clocks or {}).get("sm_max_mhz") or 2070.0
+    peak = alu_peak_tflops(sms, max_mhz)
+    achieved = flops / (mean_ms * 1e-3) / 1e12
+    line = {"metric": "window-vote eviction: ms per call, FP32 TFLOP/s of the score contraction",
+            "value": round(mean_ms, 4), "unit": "ms", "higher_is_better": False,
+            "steps": args.steps, "warmup": max(3, args.warmup), "n_gpus": 1,
+            "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "qwen2.5-14b-b4-t131072-int4g32 one anchor, window 32, "
+                                   f"budget {budget}", "l2": "inputs larger than L2"},
+            "roofline": {"bound": "alu", "achieved": round(achieved, 2), "peak": round(peak, 1),
+                         "unit": "TFLOP/s", "frac": round(achieved / peak, 3), "traffic": None,
+                         "peak_source": f"{sms} SMs x 128 FP32 lanes x 2 x {max_mhz:.0f} MHz"},
+            "ms_min": round(min(ms), 4), "ms_max": round(max(ms), 4),
+            "gpu_launches": 4 * args.steps, "clocks": clocks}
+    print(json.dumps(line))
+
+
 def profile_case(kind):
     """The kernel-level ncu case.  gqa: one int4 g32 and one bf16 anchor at
     the 14B step shape (B=32, 8 kv / 40 q heads, d_h 128, T=8192; 1.5 GB of
@@ -657,6 +754,13 @@ def profile_case(kind):
         for _ in range(3):
             for l in range(3):
                 c.decode(l, q, w.sigma)
+    elif kind in ("evict", "evict-small"):
+        # the evictor at the long-context 14B shape, or a 1-sequence, 32768-position
+        # case (70 MB of cache, 168 MB of scores) for multi-pass captures
+        B, T = (4, 131072) if kind == "evict" else (1, 32768)
+        w, c, q = _evict_setup(B, T, torch.device("cuda", 0))
+        for _ in range(3):
+            c.evict_window(0, q, w.sigma, w.keep)
     elif kind == "gather":
         import numpy as np
         w = W.config(5, n_layers=1)

@@ -10,12 +10,14 @@
 // with x = scale log2(e) <q_{w,h}, k_t> on the dequantised key and (M, L)
 // the row's maximum and sum over its causal range.  The budget - n_win
 // largest votes (ties: the smaller position) and the window become the
-// anchor's kept list for (b, j), sorted.  Four launches: row statistics per
-// 128-position tile, their merge per row, the votes, the selection.
+// anchor's kept list for (b, j), sorted.  Four launches: scores and row
+// statistics per 128-position tile, the statistics merged per row, the votes
+// (streaming the stored scores), the selection.
 //
 // The scores run on the CUDA cores in fp32: the evictor runs once per
 // prefill, not per decode step, and fp32 dot products keep the votes within
-// ~1e-6 of the fp64 definition.
+// ~1e-6 of the fp64 definition.  Storing the scores (R x 4 bytes per
+// position) costs less than computing them twice (R x D products).
 #include <math.h>
 
 #include "common.cuh"
@@ -25,8 +27,7 @@
 namespace kvk {
 namespace {
 
-constexpr int kT = kEvictTile;  // positions per CTA (one per thread)
-constexpr int kRC = 32;         // query rows per chunk
+constexpr int kT = kEvictTile;  // positions per scoring tile
 
 // Dequantised channel ch of the key of position t from its record (the
 // scale word of the symmetric scheme passed in).
@@ -52,142 +53,169 @@ __device__ __forceinline__ float key_elem(const GqaView &v, const RecLayout &L, 
   return fmaf((float)code, m.x, m.y);
 }
 
-// Shared memory of the two scoring passes: dequantised keys [kT][D + 4]
-// (rows padded by 16 bytes: the 16-byte loads of eight consecutive threads,
-// one row each, fall in distinct banks), the query rows of one chunk
-// [kRC][D], the tile's raw records.
+// Scores of one 128-position tile against every window query row of its
+// (sequence, KV head): X[r][t] = sig_log2 <q_r, k_t>, an fp32 contraction of
+// [R x D] by [D x 128] on the CUDA cores, register-tiled: thread (tx, ty)
+// holds rows ty*4 .. ty*4+3 of a 64-row chunk against positions tx*4 ..
+// tx*4+3 and 64 + tx*4 .. 64 + tx*4+3 of the tile (32 products per pair of
+// key loads and one query load).  The dequantised keys sit channel-major in
+// shared memory [D][128], the chunk's query rows [D][64].  Each row's
+// (max, sum 2^(x - max)) over the tile's positions in its causal range goes
+// to the per-tile statistics, and the scores of the positions before the
+// window go to the score buffer, which the vote pass streams instead of
+// recomputing them.
+constexpr int kRC = 64;        // window query rows per chunk
+constexpr int kThreads = 256;  // 16 position groups x 16 row groups
+
 template <int D>
-constexpr int evict_kstride() { return D + 4; }
-template <int D>
-constexpr int evict_smem(int rec_bytes) {
-  return kT * evict_kstride<D>() * 4 + kRC * D * 4 + kT * rec_bytes;
+constexpr int evict_smem() {
+  return (D * kT + D * kRC) * 4;
 }
 
-// VOTES = false: row statistics (M, L) of this tile per window query row;
-// VOTES = true: the tile's votes from the merged statistics.
-template <int D, bool VOTES>
-__global__ void __launch_bounds__(kT) evict_pass_kernel(const EvictArgs a) {
+template <int D>
+__global__ void __launch_bounds__(kThreads, 2) evict_scores_kernel(const EvictArgs a) {
   pdl_wait();
-  pdl_trigger();
   const GqaView &v = a.v;
   const int tile = blockIdx.x, j = blockIdx.y, b = blockIdx.z;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tid = threadIdx.x;
   const int len = v.lens[b];
-  if (len <= a.budget) return;  // the sequence keeps every position
-  const int P = len - a.n_win;
   const int t0 = tile * kT;
-  if (t0 >= (VOTES ? P : len)) return;
+  if (len <= a.budget || t0 >= len) {  // the sequence keeps everything / tile past the end
+    pdl_trigger();
+    return;
+  }
+  const int P = len - a.n_win;
   const int unit = b * v.Hkv + j;
   const int R = a.n_win * a.G;
-  extern __shared__ __align__(16) uint8_t smem[];
-  float *kf = reinterpret_cast<float *>(smem);
-  constexpr int KS = evict_kstride<D>();
-  float *qs = kf + kT * KS;
-  uint8_t *recs = reinterpret_cast<uint8_t *>(qs + kRC * D);
-
-  // the tile's records (contiguous in the slab), then one key row per thread
+  extern __shared__ __align__(16) float evict_sm[];
+  float *kt = evict_sm;          // [D][kT]
+  float *qt = evict_sm + D * kT; // [D][kRC]
   const size_t slab = (size_t)b * v.Hkv + j;
-  const int nrow = min(kT, len - t0);
   {
-    const uint4 *src = reinterpret_cast<const uint4 *>(v.rec + (slab * v.cap + t0) * v.rec_bytes);
-    uint4 *dst = reinterpret_cast<uint4 *>(recs);
-    const int n = nrow * v.rec_bytes / 16;
-    for (int q = tid; q < n; q += kT) dst[q] = src[q];
-  }
-  __syncthreads();
-  const int t = t0 + tid;
-  const bool live = tid < nrow;
-  if (live) {
+    // two threads per position, half of the channels each
+    const int p = tid & (kT - 1), half = tid / kT;
+    const int t = t0 + p;
+    const bool live = t < len;
     const RecLayout L = rec_layout(v.bits, D, v.group, v.key_axis);
-    const uint8_t *rec = recs + tid * v.rec_bytes;
-    const uint32_t sw = v.scheme == kSchemeSym ? v.scales[slab * v.cap + t] : 0u;
-    for (int ch = 0; ch < D; ++ch) kf[tid * KS + ch] = key_elem(v, L, rec, t, sw, ch);
+    const uint8_t *rec = v.rec + (slab * v.cap + (live ? t : t0)) * v.rec_bytes;
+    const uint32_t sw = (live && v.scheme == kSchemeSym) ? v.scales[slab * v.cap + t] : 0u;
+    for (int ch = half * (D / 2); ch < (half + 1) * (D / 2); ++ch)
+      kt[ch * kT + p] = live ? key_elem(v, L, rec, t, sw, ch) : 0.f;
   }
-  float vote = 0.f;
-  float2 *stats = a.stats + (size_t)unit * R * a.n_tiles;          // [R][n_tiles]
-  const float2 *fin = a.stats + (size_t)gridDim.z * v.Hkv * R * a.n_tiles + (size_t)unit * R;
+  const int tx = tid & 15, ty = tid >> 4;
+  float2 *stats = a.stats + (size_t)unit * R * a.n_tiles;
+  float *scores = a.scores + (size_t)unit * R * a.sc_stride;
   for (int rc0 = 0; rc0 < R; rc0 += kRC) {
-    const int nr = min(kRC, R - rc0);
-    __syncthreads();  // the previous chunk's rows are consumed (and the keys are written)
-    for (int e = tid; e < kRC * D; e += kT) {  // rows past the last are zero
-      const int rr = e / D, ch = e % D;
-      const int r = rc0 + rr, w = r / a.G, h = j * a.G + r % a.G;
-      const size_t qi = (((size_t)b * a.n_win + w) * a.Hq + h) * D + ch;
-      qs[rr * D + ch] = rr >= nr ? 0.f
-                        : a.q_f32 ? static_cast<const float *>(a.q)[qi]
-                                  : bf16_to_f32(static_cast<const uint16_t *>(a.q)[qi]);
-    }
-    __syncthreads();
-    // x[rr] = <q_rr, k_t>: eight key channels in registers against every
-    // row's eight (broadcast) query channels
-    float x[kRC];
-#pragma unroll
-    for (int rr = 0; rr < kRC; ++rr) x[rr] = 0.f;
-    if (live) {
-      const float *kr = kf + tid * KS;
-#pragma unroll 1
-      for (int c0 = 0; c0 < D; c0 += 8) {
-        const float4 k0 = *reinterpret_cast<const float4 *>(kr + c0);
-        const float4 k1 = *reinterpret_cast<const float4 *>(kr + c0 + 4);
-#pragma unroll
-        for (int rr = 0; rr < kRC; ++rr) {
-          const float4 q0 = *reinterpret_cast<const float4 *>(qs + rr * D + c0);
-          const float4 q1 = *reinterpret_cast<const float4 *>(qs + rr * D + c0 + 4);
-          float s = x[rr];
-          s = fmaf(k0.x, q0.x, s); s = fmaf(k0.y, q0.y, s);
-          s = fmaf(k0.z, q0.z, s); s = fmaf(k0.w, q0.w, s);
-          s = fmaf(k1.x, q1.x, s); s = fmaf(k1.y, q1.y, s);
-          s = fmaf(k1.z, q1.z, s); s = fmaf(k1.w, q1.w, s);
-          x[rr] = s;
+    __syncthreads();  // keys written; the previous chunk's query rows consumed
+    // the chunk's query rows, channel-major (rows past R are zero)
+    for (int e = tid; e < kRC * (D / 4); e += kThreads) {
+      const int rr = e & (kRC - 1), c4 = e / kRC;
+      const int r = rc0 + rr;
+      float4 x4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (r < R) {
+        const int w = r / a.G, h = j * a.G + r % a.G;
+        const size_t qi = (((size_t)b * a.n_win + w) * a.Hq + h) * D + 4 * c4;
+        if (a.q_f32) {
+          x4 = *reinterpret_cast<const float4 *>(static_cast<const float *>(a.q) + qi);
+        } else {
+          const uint2 u = *reinterpret_cast<const uint2 *>(static_cast<const uint16_t *>(a.q) + qi);
+          x4 = make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u),
+                           __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xFFFF0000u));
         }
       }
+      qt[(4 * c4 + 0) * kRC + rr] = x4.x;
+      qt[(4 * c4 + 1) * kRC + rr] = x4.y;
+      qt[(4 * c4 + 2) * kRC + rr] = x4.z;
+      qt[(4 * c4 + 3) * kRC + rr] = x4.w;
+    }
+    __syncthreads();
+    float acc[4][8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int c = 0; c < 8; ++c) acc[i][c] = 0.f;
+#pragma unroll 4
+    for (int k = 0; k < D; ++k) {
+      const float4 k0 = *reinterpret_cast<const float4 *>(kt + k * kT + tx * 4);
+      const float4 k1 = *reinterpret_cast<const float4 *>(kt + k * kT + 64 + tx * 4);
+      const float4 q4 = *reinterpret_cast<const float4 *>(qt + k * kRC + ty * 4);
+      const float kk[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
+      const float qq[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int c = 0; c < 8; ++c) acc[i][c] = fmaf(qq[i], kk[c], acc[i][c]);
     }
 #pragma unroll
-    for (int rr = 0; rr < kRC; ++rr) x[rr] *= a.sig_log2;
-    if constexpr (VOTES) {
-      // positions before the window: every window query sees them
+    for (int i = 0; i < 4; ++i) {
+      const int r = rc0 + ty * 4 + i;
+      const int last = P + r / a.G;  // the last position row r sees
+      float m = -INFINITY;
 #pragma unroll
-      for (int rr = 0; rr < kRC; ++rr) {
-        if (rr >= nr) break;
-        const float2 ml = fin[rc0 + rr];
-        if (live && t < P && ml.y > 0.f) vote += exp2f(x[rr] - ml.x) / ml.y;
+      for (int c = 0; c < 8; ++c) {
+        const int t = t0 + (c >> 2) * 64 + tx * 4 + (c & 3);
+        acc[i][c] *= a.sig_log2;
+        if (t <= last) m = fmaxf(m, acc[i][c]);
       }
-    } else {
-      // per row: maximum and sum over this tile's positions in its causal
-      // range (block reductions over the 128 threads)
-      __shared__ float red[4][kRC];
-      __shared__ float rowm[kRC];
 #pragma unroll
-      for (int rr = 0; rr < kRC; ++rr) {
-        const int w = (rc0 + rr) / a.G;
-        const bool ok = live && rr < nr && t <= P + w;
-        float m = ok ? x[rr] : -INFINITY;
+      for (int off = 8; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+      float l = 0.f;
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-        if (lane == 0) red[warp][rr] = m;
+      for (int c = 0; c < 8; ++c) {
+        const int t = t0 + (c >> 2) * 64 + tx * 4 + (c & 3);
+        if (t <= last) l += exp2f(acc[i][c] - m);  // m is finite: this row sees t
       }
-      __syncthreads();
-      if (tid < kRC) rowm[tid] = fmaxf(fmaxf(red[0][tid], red[1][tid]), fmaxf(red[2][tid], red[3][tid]));
-      __syncthreads();
 #pragma unroll
-      for (int rr = 0; rr < kRC; ++rr) {
-        const int w = (rc0 + rr) / a.G;
-        const bool ok = live && rr < nr && t <= P + w;
-        const float m = rowm[rr];
-        float l = (ok && m != -INFINITY) ? exp2f(x[rr] - m) : 0.f;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
-        if (lane == 0) red[warp][rr] = l;
+      for (int off = 8; off > 0; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
+      if (r < R) {
+        if (tx == 0) stats[(size_t)r * a.n_tiles + tile] = make_float2(m, l);
+        float *row = scores + (size_t)r * a.sc_stride + t0 + tx * 4;
+        if (t0 + tx * 4 < P) *reinterpret_cast<float4 *>(row) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+        if (t0 + 64 + tx * 4 < P)
+          *reinterpret_cast<float4 *>(row + 64) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
       }
-      __syncthreads();
-      if (tid < nr)
-        stats[(size_t)(rc0 + tid) * a.n_tiles + tile] =
-            make_float2(rowm[tid], red[0][tid] + red[1][tid] + red[2][tid] + red[3][tid]);
     }
   }
-  if constexpr (VOTES) {
-    if (live && t < P) a.votes[(size_t)unit * v.cap + t] = vote;
+  pdl_trigger();
+}
+
+// Votes of 256 positions before the window: sum over the rows of
+// 2^(x - M - log2 L) with the rows' merged statistics, streaming the scores.
+constexpr int kVoteT = 256;
+constexpr int kVoteRows = 1024;  // merged statistics staged per round
+
+__global__ void __launch_bounds__(kVoteT) evict_votes_kernel(const EvictArgs a) {
+  pdl_wait();
+  const GqaView &v = a.v;
+  const int j = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
+  const int len = v.lens[b];
+  const int P = len - a.n_win;
+  const int t = blockIdx.x * kVoteT + tid;
+  if (len <= a.budget || (int)blockIdx.x * kVoteT >= P) {
+    pdl_trigger();
+    return;
   }
+  const int unit = b * v.Hkv + j;
+  const int R = a.n_win * a.G;
+  const float2 *fin = a.stats + (size_t)gridDim.z * v.Hkv * R * a.n_tiles + (size_t)unit * R;
+  const float *x = a.scores + (size_t)unit * R * a.sc_stride + t;
+  __shared__ float norm[kVoteRows];
+  float vote = 0.f;
+  for (int r0 = 0; r0 < R; r0 += kVoteRows) {
+    const int nr = min(kVoteRows, R - r0);
+    __syncthreads();
+    for (int i = tid; i < nr; i += kVoteT) {
+      const float2 ml = fin[r0 + i];
+      norm[i] = ml.x + log2f(ml.y);
+    }
+    __syncthreads();
+    if (t < P) {
+#pragma unroll 8
+      for (int r = 0; r < nr; ++r) vote += exp2f(x[(size_t)(r0 + r) * a.sc_stride] - norm[r]);
+    }
+  }
+  if (t < P) a.votes[(size_t)unit * v.cap + t] = vote;
+  pdl_trigger();
 }
 
 // Merged (M, L) of every window query row over its tiles.
@@ -317,20 +345,18 @@ __global__ void __launch_bounds__(1024) evict_select_kernel(const EvictArgs a) {
 
 template <int D>
 cudaError_t launch_evict_d(const EvictArgs &a, cudaStream_t st) {
-  const int smem = evict_smem<D>(a.v.rec_bytes);
-  cudaError_t e = cudaFuncSetAttribute(evict_pass_kernel<D, false>,
+  constexpr int smem = evict_smem<D>();
+  cudaError_t e = cudaFuncSetAttribute(evict_scores_kernel<D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(evict_pass_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem);
   if (e != cudaSuccess) return e;
-  const dim3 grid(a.n_tiles, a.v.Hkv, a.v.B);
-  e = launch_pdl(evict_pass_kernel<D, false>, grid, dim3(kT), smem, st, a);
+  e = launch_pdl(evict_scores_kernel<D>, dim3(a.n_tiles, a.v.Hkv, a.v.B), dim3(kThreads), smem, st, a);
   if (e == cudaSuccess) {
     const int rows = a.v.B * a.v.Hkv * a.n_win * a.G;
     e = launch_pdl(evict_merge_stats_kernel, dim3((rows + 127) / 128), dim3(128), 0, st, a);
   }
-  if (e == cudaSuccess) e = launch_pdl(evict_pass_kernel<D, true>, grid, dim3(kT), smem, st, a);
+  if (e == cudaSuccess)
+    e = launch_pdl(evict_votes_kernel, dim3((a.v.cap + kVoteT - 1) / kVoteT, a.v.Hkv, a.v.B),
+                   dim3(kVoteT), 0, st, a);
   if (e == cudaSuccess)
     e = launch_pdl(evict_select_kernel, dim3(a.v.Hkv, a.v.B), dim3(1024), 0, st, a);
   return e;

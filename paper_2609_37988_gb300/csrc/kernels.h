@@ -79,8 +79,10 @@ struct EvictArgs {
   int Hq, G, n_win, budget;
   float sig_log2;      // softmax scale * log2(e)
   int n_tiles;         // 128-position tiles launched per (sequence, kv head)
-  float *votes;
-  float2 *stats;
+  int sc_stride;       // n_tiles * kEvictTile: row stride of the scores
+  float *votes;        // [B * Hkv][cap]
+  float2 *stats;       // [B * Hkv][R][n_tiles] per-tile (max, sum), then [B * Hkv][R] merged
+  float *scores;       // [B * Hkv][R][sc_stride] scaled scores (log2 domain)
   int32_t *err;
 };
 cudaError_t launch_gqa_evict(const EvictArgs &a, cudaStream_t st);

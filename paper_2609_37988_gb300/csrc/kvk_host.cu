@@ -533,7 +533,7 @@ kvk_status kvk_set_kept(kvk_cache *c, int32_t layer, const int32_t *idx, const i
 
 namespace {
 struct EvictScratch {
-  size_t votes, stats, total;
+  size_t votes, stats, scores, total;  // region sizes: votes, statistics, scores
   int n_tiles;
 };
 EvictScratch evict_scratch(const kvk_cache *c, int layer, int n_win) {
@@ -544,7 +544,8 @@ EvictScratch evict_scratch(const kvk_cache *c, int layer, int n_win) {
   e.n_tiles = (int)((cap + kEvictTile - 1) / kEvictTile);
   e.votes = align256((int64_t)(units * cap * 4));
   e.stats = align256((int64_t)((units * R * e.n_tiles + units * R) * 8));
-  e.total = e.votes + e.stats;
+  e.scores = align256((int64_t)(units * R * e.n_tiles * kEvictTile * 4));
+  e.total = e.votes + e.stats + e.scores;
   return e;
 }
 
@@ -600,8 +601,10 @@ kvk_status kvk_evict_window(kvk_cache *c, int32_t layer, const void *q_win, int3
   a.budget = budget;
   a.sig_log2 = softmax_scale * 1.4426950408889634f;
   a.n_tiles = es.n_tiles;
+  a.sc_stride = es.n_tiles * kEvictTile;
   a.votes = static_cast<float *>(scratch);
   a.stats = reinterpret_cast<float2 *>(static_cast<uint8_t *>(scratch) + es.votes);
+  a.scores = reinterpret_cast<float *>(static_cast<uint8_t *>(scratch) + es.votes + es.stats);
   a.err = c->err();
   cudaError_t e = launch_gqa_evict(a, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "eviction launch");

@@ -198,6 +198,13 @@ def queries(w: Workload, layer: int, step: int = 0, device="cpu") -> torch.Tenso
                  dtype=w.q_dtype, device=device)
 
 
+def window_queries(w: Workload, layer: int, n_win: int, device="cpu") -> torch.Tensor:
+    """Queries of each sequence's last ``n_win`` positions (the eviction
+    observation window) ``[B, n_win, H_q, D]``."""
+    return randn((w.batch, n_win, w.n_q_heads, w.head_dim), w.seed, layer, 10,
+                 dtype=w.q_dtype, device=device)
+
+
 def kept_positions(w: Workload, layer: int, lens, device="cpu"):
     """Sorted uniform samples of ``w.keep`` positions per sequence:
     (idx ``[B, keep]`` int32, n_kept ``[B]`` int32)."""

@@ -220,3 +220,40 @@ def test_evict_rejections():
     with pytest.raises(KVKError):
         c.evict_window(0, q, 0.0, 16)
     assert c.kept_lists(0) is None      # nothing was installed
+
+
+@pytest.mark.slow
+def test_evict_full_size_sampled():
+    """The bench's eviction call (14B long-context shape: B=4, 8 KV / 40 q
+    heads, 131072 positions, int4 g32, window 32, budget T/8) with the bench's
+    inputs; two (sequence, KV head) units checked against the oracle: every
+    vote, and the kept list up to near-ties at the cut."""
+    import bench
+    from paper_2609_37988_gb300 import workloads as W
+    w, c, q = bench._evict_setup(4, 131072, torch.device("cuda", 0))
+    budget, n_win = w.keep, bench.EVICT_WINDOW
+    G = w.n_q_heads // w.n_kv_heads
+    votes = f32(c.evict_window(0, q, w.sigma, budget))
+    idx, n, _ = c.kept_lists(0)
+    idx, n = idx.cpu().numpy(), n.cpu().numpy()
+    assert c.device_error() == 0
+    T = w.context
+    P = T - n_win
+    cfg = w.layers[0]
+    for b, j in ((0, 0), (3, 7)):
+        # the bench's inputs (drawn on the device), this unit's keys only
+        k = torch.cat([W.kv_inputs(w, 0, b0, min(T, b0 + 16384), device="cuda")[0]
+                       [b:b + 1, :, j:j + 1].cpu() for b0 in range(0, T, 16384)], 1)
+        st = oracle_state(f32(k), f32(k), np.array([T]), cfg)
+        qb = f32(q[b, :, j * G:(j + 1) * G])
+        ov = oev.window_votes(qb, st["k_hat"][0], T, w.sigma, 0, G)
+        gv = votes[b, j, :P]
+        err = np.abs(gv - ov)
+        assert (err <= VOTE_RTOL * ov + VOTE_ATOL).all(), f"unit ({b},{j}): vote error {err.max():.3e}"
+        assert int(n[b, j]) == budget
+        sel = idx[b, j, :budget]
+        np.testing.assert_array_equal(sel[-n_win:], np.arange(P, T))
+        want = set(oev.select(ov, budget - n_win).tolist())
+        kth = np.sort(ov)[::-1][budget - n_win - 1]
+        for t in set(sel[:-n_win].tolist()) ^ want:
+            assert abs(ov[t] - kth) <= 4 * (VOTE_RTOL * kth + VOTE_ATOL), (b, j, t)
