@@ -20,9 +20,12 @@
 // position) costs less than computing them twice (R x D products).
 #include <math.h>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "layout.h"
+#include "umma.cuh"
 
 namespace kvk {
 namespace {
@@ -197,7 +200,7 @@ __global__ void __launch_bounds__(kVoteT) evict_votes_kernel(const EvictArgs a) 
   }
   const int unit = b * v.Hkv + j;
   const int R = a.n_win * a.G;
-  const float2 *fin = a.stats + (size_t)gridDim.z * v.Hkv * R * a.n_tiles + (size_t)unit * R;
+  const float2 *fin = a.fin + (size_t)unit * R;
   const float *x = a.scores + (size_t)unit * R * a.sc_stride + t;
   __shared__ float norm[kVoteRows];
   float vote = 0.f;
@@ -219,27 +222,35 @@ __global__ void __launch_bounds__(kVoteT) evict_votes_kernel(const EvictArgs a) 
 }
 
 // Merged (M, L) of every window query row over its tiles.
-__global__ void __launch_bounds__(128) evict_merge_stats_kernel(const EvictArgs a) {
+// One warp per (unit, row): lanes stride over the row's tile entries
+// (coalesced), then warp reductions of the maximum and of the rescaled sums.
+constexpr int kMergeWarps = 8;
+__global__ void __launch_bounds__(32 * kMergeWarps) evict_merge_stats_kernel(const EvictArgs a) {
   pdl_wait();
   pdl_trigger();
   const GqaView &v = a.v;
   const int R = a.n_win * a.G;
   const int units = v.B * v.Hkv;
-  const int id = blockIdx.x * blockDim.x + threadIdx.x;
+  const int id = blockIdx.x * kMergeWarps + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (id >= units * R) return;
   const int unit = id / R, r = id % R, b = unit / v.Hkv;
   const int len = v.lens[b];
   if (len <= a.budget) return;
-  const int nt = min((len + kT - 1) / kT, a.n_tiles);
-  const float2 *st = a.stats + ((size_t)unit * R + r) * a.n_tiles;
+  const int nt = min((len + kT - 1) / kT, a.n_tiles) * a.stat_sub;
+  const float2 *st = a.stats + ((size_t)unit * R + r) * a.n_tiles * a.stat_sub;
   float M = -INFINITY;
-  for (int i = 0; i < nt; ++i) M = fmaxf(M, st[i].x);
+  for (int i = lane; i < nt; i += 32) M = fmaxf(M, st[i].x);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
   float L = 0.f;
   if (M != -INFINITY)
-    for (int i = 0; i < nt; ++i)
-      if (st[i].x != -INFINITY) L += st[i].y * exp2f(st[i].x - M);
-  float2 *fin = a.stats + (size_t)units * R * a.n_tiles;
-  fin[id] = make_float2(M, L);
+    for (int i = lane; i < nt; i += 32) {
+      const float2 e = st[i];
+      if (e.x != -INFINITY) L += e.y * exp2f(e.x - M);
+    }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
+  if (lane == 0) a.fin[id] = make_float2(M, L);
 }
 
 // Block-wide exclusive scan of one int per thread (1024 threads); returns the
@@ -269,6 +280,20 @@ __device__ __forceinline__ int block_scan_1024(int x, int *wsum, int *total) {
   const int r = wsum[warp] + inc - x;
   __syncthreads();  // wsum is reused by the next scan
   return r;
+}
+
+// keys t0 .. t0+7 (zero past n); t0 is a multiple of 8 and the array
+// 32-byte aligned
+__device__ __forceinline__ void load8(const uint32_t *key, int t0, int n, uint32_t (&kk)[8]) {
+  if (t0 + 8 <= n) {
+    const uint4 u0 = *reinterpret_cast<const uint4 *>(key + t0);
+    const uint4 u1 = *reinterpret_cast<const uint4 *>(key + t0 + 4);
+    kk[0] = u0.x; kk[1] = u0.y; kk[2] = u0.z; kk[3] = u0.w;
+    kk[4] = u1.x; kk[5] = u1.y; kk[6] = u1.z; kk[7] = u1.w;
+  } else {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) kk[u] = t0 + u < n ? key[t0 + u] : 0u;
+  }
 }
 
 // Kept list of one (sequence, kv head): the budget - n_win largest votes by
@@ -302,9 +327,25 @@ __global__ void __launch_bounds__(1024) evict_select_kernel(const EvictArgs a) {
       const int shift = 24 - 8 * pass;
       for (int d = tid; d < 256; d += 1024) hist[d] = 0;
       __syncthreads();
-      for (int t = tid; t < P; t += 1024) {
-        const uint32_t kk = key[t];
-        if ((kk & mask) == prefix) atomicAdd(&hist[(kk >> shift) & 255], 1);
+      // votes of similar size share their leading bytes, so most lanes of a
+      // warp hit the bin of lane 0: those are counted with one atomic, the
+      // others one by one.  Eight consecutive votes per thread per round
+      // keep eight loads in flight.
+      for (int c0 = 0; c0 < P; c0 += 8 * 1024) {
+        uint32_t kk[8];
+        load8(key, c0 + 8 * tid, P, kk);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const bool hit = c0 + 8 * tid + u < P && (kk[u] & mask) == prefix;
+          const uint32_t bin = hit ? (kk[u] >> shift) & 255 : 256u;
+          const uint32_t bin0 = __shfl_sync(0xffffffffu, bin, 0);
+          const uint32_t same = __ballot_sync(0xffffffffu, bin == bin0);
+          if (bin == bin0) {
+            if ((threadIdx.x & 31) == 0 && bin0 < 256u) atomicAdd(&hist[bin0], __popc(same));
+          } else if (hit) {
+            atomicAdd(&hist[bin], 1);
+          }
+        }
       }
       __syncthreads();
       if (tid == 0) {
@@ -324,23 +365,602 @@ __global__ void __launch_bounds__(1024) evict_select_kernel(const EvictArgs a) {
     }
   }
   // positions above the threshold key, and the first `rank` equal to it
+  // (one scan of the packed counts: greater in the high half, equal in the
+  // low half; a taken position's slot is the greater ones before it plus
+  // the equal ones before it, at most `rank`)
   const uint32_t theta = prefix;
-  int eq_carry = 0, out_carry = 0;
-  for (int c0 = 0; c0 < P && k > 0; c0 += 1024) {
-    const int t = c0 + tid;
-    const uint32_t kk = t < P ? key[t] : 0u;
-    const bool gt = t < P && kk > theta, eq = t < P && kk == theta;
-    const int eq_before = eq_carry + block_scan_1024(eq ? 1 : 0, wsum, &s_total);
-    const int eq_tot = s_total;
-    const bool take = gt || (eq && eq_before < rank);
-    const int pos = out_carry + block_scan_1024(take ? 1 : 0, wsum, &s_total);
-    const int take_tot = s_total;
-    if (take && pos < k) out[pos] = t;
-    eq_carry += eq_tot;
-    out_carry += take_tot;
+  int gt_carry = 0, eq_carry = 0;
+  for (int c0 = 0; c0 < P && k > 0; c0 += 8 * 1024) {
+    const int tb = c0 + 8 * tid;  // this thread's eight consecutive positions
+    uint32_t kk[8];
+    load8(key, tb, P, kk);
+    int ngt = 0, neq = 0;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      ngt += tb + u < P && kk[u] > theta;
+      neq += tb + u < P && kk[u] == theta;
+    }
+    const int ex = block_scan_1024((ngt << 16) | neq, wsum, &s_total);
+    const int tot = s_total;
+    int gt_before = gt_carry + (ex >> 16), eq_before = eq_carry + (ex & 0xFFFF);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const bool gt = tb + u < P && kk[u] > theta, eq = tb + u < P && kk[u] == theta;
+      const int pos = gt_before + min(eq_before, rank);
+      if ((gt || (eq && eq_before < rank)) && pos < k) out[pos] = tb + u;
+      gt_before += gt;
+      eq_before += eq;
+    }
+    gt_carry += tot >> 16;
+    eq_carry += tot & 0xFFFF;
   }
   for (int i = tid; i < a.n_win; i += 1024) out[k + i] = P + i;
   if (tid == 0) v.kept_n[unit] = a.budget;
+}
+
+// ---------------------------------------------------------------------------
+// Tensor-core scoring (tcgen05; head_dim 128, at most 256 window rows).
+//
+// The scores of a 128-position tile are one UMMA chain over K = 128
+// channels.  The dequantised keys, split into bf16 hi + lo, and the window
+// query rows (split likewise when they arrive in fp32; bf16 queries have no
+// lo part) sit in shared memory in the K-major 128-byte-swizzled layout
+// (two 64-channel boxes of 128-byte rows, 16-byte chunk c of row r stored at
+// chunk c ^ (r & 7)).  hi*hi + hi*lo + lo*hi keeps ~16 significant bits of
+// each factor (the dropped lo*lo term is below 2^-16 of the product); the
+// tensor cores accumulate in fp32 in TMEM.
+//  * statistics pass: A = query rows (M = 128 per chunk), B = keys (N = 128
+//    positions): TMEM lane = row, so each thread reduces its row over the
+//    positions without shuffles (two entries per tile and row, one per
+//    64-position half);
+//  * vote pass: A = keys (M = 128 positions), B = query rows (N = R rounded
+//    up to 16): TMEM lane = position, so each thread sums its position's
+//    weights over the rows.
+// The vote pass recomputes the scores: on the tensor cores that is cheaper
+// than a round trip through HBM.  A CTA (one per SM) walks a contiguous range
+// of (unit, tile) items; with two key stages the keys of the next item are
+// dequantised while the tensor cores run the current one, and the epilogue
+// of an item reads one TMEM buffer while the next item's chain fills the
+// other.  Query rows past R are zero; in the statistics pass the last row
+// chunk may read rows past the query buffer (lanes that are never used).
+constexpr int kTcWorkers = 256;              // dequantise and run the epilogues
+constexpr int kTcThreads = kTcWorkers + 32;  // + the MMA warp
+
+// barrier 1 over the worker warps (the MMA warp runs on its own)
+__device__ __forceinline__ void workers_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+__device__ __forceinline__ bool workers_sync_or(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 256, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u)
+      : "memory");
+  return r != 0;
+}
+
+// 16-byte chunks of a head_dim-128 K section per key format
+__host__ __device__ constexpr int TcFmtKs16(int fmt) {
+  return fmt == 0 ? 16 : (fmt == 1 || fmt == 3) ? 8 : (fmt == 2 || fmt == 4) ? 4 : 2;
+}
+
+struct TcPlan {
+  int items_per_cta, n_items;
+  int R16, nch, q_lo, k_lo, nst, nstg, fmt;  // nst key stages, nstg staging buffers
+  int kb_nch, kb_stride, stg_bytes;  // staged 16-byte chunks per position, their stride
+  int stage, off_q, off_ql, off_k, off_stg, off_norm, off_pv, off_bar, smem;
+};
+
+// key formats of the tensor-core dequantiser
+enum { kFmtBf16 = 0, kFmtG8, kFmtG4, kFmtS8, kFmtS4, kFmtS2 };
+
+template <int FMT>
+struct TcFmt {
+  static constexpr int BITS = FMT == kFmtBf16                   ? 16
+                              : (FMT == kFmtG8 || FMT == kFmtS8) ? 8
+                              : (FMT == kFmtG4 || FMT == kFmtS4) ? 4
+                                                                 : 2;
+  static constexpr bool SYM = FMT >= kFmtS8;
+  static constexpr int KS = 128 * BITS / 8;  // K-section bytes
+};
+
+// hi (and lo) bf16 words of 8 channels -> one swizzled 16-byte chunk of row
+// `row` holding channels ch0 .. ch0 + 7 (box stride `box` bytes)
+__device__ __forceinline__ void put_chunk(uint8_t *buf, int row, int ch0, int box, uint4 w) {
+  const int off = (ch0 >> 6) * box + row * 128 + ((((ch0 & 63) >> 3) ^ (row & 7)) << 4);
+  *reinterpret_cast<uint4 *>(buf + off) = w;
+}
+__device__ __forceinline__ void put8(uint8_t *hi, uint8_t *lo, bool with_lo, int row, int ch0,
+                                     int box, const float (&x)[8]) {
+  uint32_t h[4], l[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) split2<true>(x[2 * i], x[2 * i + 1], h[i], l[i]);
+  put_chunk(hi, row, ch0, box, make_uint4(h[0], h[1], h[2], h[3]));
+  if (with_lo) put_chunk(lo, row, ch0, box, make_uint4(l[0], l[1], l[2], l[3]));
+}
+// exact float of a small unsigned integer (< 2^23) on the FMA/ALU pipes
+__device__ __forceinline__ float u2f(uint32_t u) {
+  return __uint_as_float(0x4B000000u | u) - 8388608.f;
+}
+
+// Channels H*64 .. H*64+63 of one position's key, from its staged bundle
+// (K section in logical order, then the group metadata or the symmetric
+// scale word), dequantised into the key stage (hi, and lo unless bf16).
+template <int FMT, int H>
+__device__ __forceinline__ void tc_dequant_half(const uint8_t *bundle, int row, int group,
+                                                uint8_t *kh, uint8_t *kl) {
+  using F = TcFmt<FMT>;
+  constexpr int D = 128, KBOX = 128 * 128;
+  uint32_t w[F::KS / 4];
+#pragma unroll
+  for (int c = 0; c < F::KS / 16; ++c) {
+    const uint4 u = *reinterpret_cast<const uint4 *>(bundle + 16 * c);
+    w[4 * c] = u.x; w[4 * c + 1] = u.y; w[4 * c + 2] = u.z; w[4 * c + 3] = u.w;
+  }
+  if constexpr (F::BITS == 16) {
+    static_assert(!F::SYM, "bf16 keys carry no scale");
+    // bf16 keys are exact: gather them into channel order, no lo part
+#pragma unroll
+    for (int cc = 0; cc < 8; ++cc) {
+      const int ch0 = H * 64 + 8 * cc;
+      uint32_t o[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        int b0, b1, h0, h1;
+        k_pos(ch0 + 2 * i, 16, D, &b0, &h0);
+        k_pos(ch0 + 2 * i + 1, 16, D, &b1, &h1);
+        const uint32_t sel = (uint32_t)((b0 & 3) | (((b0 & 3) + 1) << 4) | ((4 + (b1 & 3)) << 8) |
+                                        ((5 + (b1 & 3)) << 12));
+        o[i] = __byte_perm(w[b0 >> 2], w[b1 >> 2], sel);
+      }
+      put_chunk(kh, row, ch0, KBOX, make_uint4(o[0], o[1], o[2], o[3]));
+    }
+  } else {
+    constexpr int QL = (1 << (F::BITS - 1)) - 1;  // symmetric code offset
+    const float sym_s = F::SYM ? __uint_as_float(*reinterpret_cast<const uint32_t *>(bundle + F::KS) << 16)
+                               : 0.f;
+#pragma unroll
+    for (int cc = 0; cc < 8; ++cc) {
+      const int ch0 = H * 64 + 8 * cc;
+      float2 m = make_float2(0.f, 0.f);
+      if constexpr (!F::SYM) m = *reinterpret_cast<const float2 *>(bundle + F::KS + 8 * (ch0 / group));
+      float x[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int ch = ch0 + i;
+        if constexpr (F::SYM) {
+          const int lb = sym_k_bit(ch, F::BITS, D);
+          const uint32_t u = (w[lb >> 5] >> (lb & 31)) & ((1u << F::BITS) - 1u);
+          x[i] = sym_s * (u2f(u) - (float)QL);
+        } else {
+          int byte, hi;
+          k_pos(ch, F::BITS, D, &byte, &hi);
+          const int sh = 8 * (byte & 3) + (F::BITS == 4 && hi ? 4 : 0);
+          const uint32_t u = (w[byte >> 2] >> sh) & ((1u << F::BITS) - 1u);
+          x[i] = fmaf(u2f(u), m.x, m.y);
+        }
+      }
+      put8(kh, kl, true, row, ch0, KBOX, x);
+    }
+  }
+}
+
+template <int FMT>
+__device__ __forceinline__ void tc_dequant(const uint8_t *bundle, int row, int half, int group,
+                                           uint8_t *kh, uint8_t *kl) {
+  if (half == 0)
+    tc_dequant_half<FMT, 0>(bundle, row, group, kh, kl);
+  else
+    tc_dequant_half<FMT, 1>(bundle, row, group, kh, kl);
+}
+
+template <bool VOTES>
+__global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs a, const TcPlan p) {
+  extern __shared__ uint8_t evict_tc_raw[];
+  uint8_t *sm = evict_tc_raw + ((1024u - (smem_u32(evict_tc_raw) & 1023u)) & 1023u);
+  // bar[0], [1]: the chain of TMEM buffer 0 / 1 done; [2]: drain; [3], [4]:
+  // the keys of an even / odd item staged (one arrival per worker warp)
+  uint64_t *bar = reinterpret_cast<uint64_t *>(sm + p.off_bar);
+  uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + 40);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + 44);
+  float *norm = reinterpret_cast<float *>(sm + p.off_norm);
+  float *pv = reinterpret_cast<float *>(sm + p.off_pv);
+  uint8_t *qh = sm + p.off_q, *ql = sm + p.off_ql;
+  const GqaView &v = a.v;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int R = a.n_win * a.G;
+  constexpr uint32_t kLimit = 1u << 22;
+  constexpr int D = 128;
+  constexpr int KBOX = 128 * 128;  // bytes of one 64-channel box of a 128-row key tile
+
+  if (tid == 0) {
+    for (int i = 0; i < 5; ++i) mbar_init(&bar[i], i < 3 ? 1 : kTcWorkers / 32);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  pdl_wait();  // the cache, lengths and (vote pass) merged statistics are complete
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tbase)),
+                 "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tbase;
+
+  const int it0 = blockIdx.x * p.items_per_cta;
+  const int it1 = min(it0 + p.items_per_cta, p.n_items);
+  const int quarter = warp & 3, half = warp >> 2;
+  const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+  uint32_t phases = 0u;  // bit tb: parity of TMEM buffer tb's next completion
+  bool failed = false;
+
+  auto valid = [&](int it) {
+    const int len = v.lens[(it / a.n_tiles) / v.Hkv];
+    const int t0 = (it % a.n_tiles) * kT;
+    return len > a.budget && t0 < (VOTES ? len - a.n_win : len);
+  };
+  auto next_valid = [&](int it) {
+    while (it < it1 && !valid(it)) ++it;
+    return it;
+  };
+
+  // query rows of `unit` (and, for the votes, the rows' log-normalisers;
+  // +inf for the padding rows, whose weights are then 0)
+  auto load_q = [&](int unit) {
+    const int b = unit / v.Hkv, j = unit % v.Hkv;
+    const int box = p.R16 * 128;
+    for (int e = tid; e < p.R16 * (D / 8); e += kTcWorkers) {
+      const int r = e >> 4, c8 = e & 15;
+      float x[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] = 0.f;
+      if (r < R) {
+        const int w = r / a.G, h = j * a.G + r % a.G;
+        const size_t qi = (((size_t)b * a.n_win + w) * a.Hq + h) * D + 8 * c8;
+        if (a.q_f32) {
+          const float4 u0 = *reinterpret_cast<const float4 *>(static_cast<const float *>(a.q) + qi);
+          const float4 u1 = *reinterpret_cast<const float4 *>(static_cast<const float *>(a.q) + qi + 4);
+          x[0] = u0.x; x[1] = u0.y; x[2] = u0.z; x[3] = u0.w;
+          x[4] = u1.x; x[5] = u1.y; x[6] = u1.z; x[7] = u1.w;
+        } else {
+          const uint4 u = *reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(a.q) + qi);
+          const uint32_t ww[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            x[2 * i] = __uint_as_float(ww[i] << 16);
+            x[2 * i + 1] = __uint_as_float(ww[i] & 0xFFFF0000u);
+          }
+        }
+      }
+      put8(qh, ql, p.q_lo != 0, r, 8 * c8, box, x);
+    }
+    if constexpr (VOTES) {
+      for (int r = tid; r < p.R16; r += kTcWorkers) {
+        if (r < R) {
+          const float2 f = a.fin[(size_t)unit * R + r];
+          norm[r] = f.x + log2f(f.y);
+        } else {
+          norm[r] = INFINITY;
+        }
+      }
+    }
+    fence_proxy_async();
+    workers_sync();
+  };
+
+  // asynchronous copy of the K bundles of item `it` (K section in logical
+  // order, then the group metadata or the symmetric scale word) into staging
+  // buffer g; one commit group per call
+  auto stage_copy = [&](int it, int g) {
+    const int unit = it / a.n_tiles, t0 = (it % a.n_tiles) * kT;
+    const int len = v.lens[unit / v.Hkv];
+    uint8_t *dst0 = sm + p.off_stg + g * p.stg_bytes;
+    const int NC = p.kb_nch;
+    const int ks16 = TcFmtKs16(p.fmt);
+    const bool sym = p.fmt >= kFmtS8;
+    const int nrec = v.rec_bytes >> 4;
+    const int km = ks16 * 32;  // grouped: key metadata follows the K and V sections
+    const uint8_t *base = v.rec + (size_t)unit * v.cap * v.rec_bytes;
+    for (int e = tid; e < kT * NC; e += kTcWorkers) {
+      const int pos = e / NC, c = e - pos * NC;
+      const int t = t0 + pos;
+      const bool ok = t < len;
+      const int so = sym ? 16 * ((c + sym_rot(t, nrec)) & (nrec - 1)) : c < ks16 ? 16 * c : km + 16 * (c - ks16);
+      cp_async16(dst0 + pos * p.kb_stride + 16 * c, base + (size_t)(ok ? t : t0) * v.rec_bytes + so, ok);
+    }
+    if (sym)
+      for (int pos = tid; pos < kT; pos += kTcWorkers) {
+        const int t = t0 + pos;
+        const bool ok = t < len;
+        cp_async4(dst0 + pos * p.kb_stride + 16 * ks16,
+                  v.scales + (size_t)unit * v.cap + (ok ? t : t0), ok);
+      }
+    cp_async_commit();
+  };
+
+  // dequantised keys of the item staged in buffer g into key stage s
+  auto dequant = [&](int g, int s) {
+    const int pidx = tid & 127, hf = tid >> 7;
+    const uint8_t *bundle = sm + p.off_stg + g * p.stg_bytes + pidx * p.kb_stride;
+    uint8_t *kh = sm + p.off_k + s * p.stage, *kl = kh + 2 * KBOX;
+    switch (p.fmt) {
+      case kFmtBf16: tc_dequant<kFmtBf16>(bundle, pidx, hf, v.group, kh, kl); break;
+      case kFmtG8: tc_dequant<kFmtG8>(bundle, pidx, hf, v.group, kh, kl); break;
+      case kFmtG4: tc_dequant<kFmtG4>(bundle, pidx, hf, v.group, kh, kl); break;
+      case kFmtS8: tc_dequant<kFmtS8>(bundle, pidx, hf, v.group, kh, kl); break;
+      case kFmtS4: tc_dequant<kFmtS4>(bundle, pidx, hf, v.group, kh, kl); break;
+      default: tc_dequant<kFmtS2>(bundle, pidx, hf, v.group, kh, kl); break;
+    }
+  };
+
+  // one MMA chain for the tile in key stage s into TMEM buffer tb (thread 0)
+  auto issue = [&](int s, int tb) {
+    tc_fence_after();
+    const uint32_t kh = smem_u32(sm + p.off_k + s * p.stage), kl = kh + 2 * KBOX;
+    const uint32_t qa = smem_u32(qh), qb = smem_u32(ql);
+    const uint32_t qbox = (uint32_t)p.R16 * 128;
+    const uint32_t d0 = tmem + 256u * tb;
+    auto dsc = [](uint32_t addr) { return umma_desc(addr, 16, 1024, 2); };
+    if constexpr (!VOTES) {
+      const uint32_t id = umma_idesc(128, 128, false, false);
+      for (int c = 0; c < p.nch; ++c) {
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t ko = (ks >> 2) * KBOX + (ks & 3) * 32;
+          const uint32_t qo = (ks >> 2) * qbox + c * 16384 + (ks & 3) * 32;
+          umma_f16(d0 + 128 * c, dsc(qa + qo), dsc(kh + ko), id, ks > 0);
+          if (p.k_lo) umma_f16(d0 + 128 * c, dsc(qa + qo), dsc(kl + ko), id, true);
+          if (p.q_lo) umma_f16(d0 + 128 * c, dsc(qb + qo), dsc(kh + ko), id, true);
+        }
+      }
+    } else {
+      const uint32_t id = umma_idesc(128, p.R16, false, false);
+#pragma unroll
+      for (int ks = 0; ks < D / 16; ++ks) {
+        const uint32_t ko = (ks >> 2) * KBOX + (ks & 3) * 32;
+        const uint32_t qo = (ks >> 2) * qbox + (ks & 3) * 32;
+        umma_f16(d0, dsc(kh + ko), dsc(qa + qo), id, ks > 0);
+        if (p.k_lo) umma_f16(d0, dsc(kl + ko), dsc(qa + qo), id, true);
+        if (p.q_lo) umma_f16(d0, dsc(kh + ko), dsc(qb + qo), id, true);
+      }
+    }
+    umma_commit(&bar[tb]);
+  };
+
+  // epilogue of item `it` from TMEM buffer tb
+  auto epilogue = [&](int it, int tb) {
+    const int unit = it / a.n_tiles, tile = it % a.n_tiles;
+    const int len = v.lens[unit / v.Hkv];
+    const int P = len - a.n_win;
+    const int t0 = tile * kT;
+    const float sg = a.sig_log2;
+    if constexpr (!VOTES) {
+      float2 *st = a.stats + (size_t)unit * R * (2 * a.n_tiles);
+      for (int c = 0; c < p.nch; ++c) {
+        if (128 * c + 32 * quarter >= R) continue;  // the warp's rows are all padding
+        const int r = 128 * c + 32 * quarter + lane;
+        const int last = P + r / a.G;  // the last position row r sees
+        float y[64];
+        const uint32_t ta = tmem + 256u * tb + 128 * c + 64 * half + lane_off;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          float z[16];
+          tmem_ld16(ta + 16 * q, z);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) y[16 * q + i] = z[i];
+        }
+        const int tb0 = t0 + 64 * half;
+        const int nv = min(64, last - tb0 + 1);  // positions of the half row r sees
+        float m = -INFINITY, l = 0.f;
+        if (nv >= 64) {
+#pragma unroll
+          for (int i = 0; i < 64; ++i) m = fmaxf(m, y[i]);
+          const float ms = m * sg;
+#pragma unroll
+          for (int i = 0; i < 64; ++i) l += fast_exp2(fmaf(y[i], sg, -ms));
+          m = ms;
+        } else if (nv > 0) {
+#pragma unroll
+          for (int i = 0; i < 64; ++i)
+            if (i < nv) m = fmaxf(m, y[i]);
+          const float ms = m * sg;
+#pragma unroll
+          for (int i = 0; i < 64; ++i)
+            if (i < nv) l += fast_exp2(fmaf(y[i], sg, -ms));
+          m = ms;
+        }
+        if (r < R) st[(size_t)r * (2 * a.n_tiles) + 2 * tile + half] = make_float2(m, l);
+      }
+    } else {
+      const int pos = 32 * quarter + lane, t = t0 + pos;
+      const int n16 = p.R16 / 16, h0 = (n16 + 1) / 2;
+      const int bk0 = half ? h0 : 0, bk1 = half ? n16 : h0;
+      float vote = 0.f;
+      for (int bk = bk0; bk < bk1; ++bk) {
+        float y[16];
+        tmem_ld16(tmem + 256u * tb + 16 * bk + lane_off, y);
+        const float4 *nr = reinterpret_cast<const float4 *>(norm + 16 * bk);
+#pragma unroll
+        for (int i4 = 0; i4 < 4; ++i4) {
+          const float4 c4 = nr[i4];
+          vote += fast_exp2(fmaf(y[4 * i4], sg, -c4.x));
+          vote += fast_exp2(fmaf(y[4 * i4 + 1], sg, -c4.y));
+          vote += fast_exp2(fmaf(y[4 * i4 + 2], sg, -c4.z));
+          vote += fast_exp2(fmaf(y[4 * i4 + 3], sg, -c4.w));
+        }
+      }
+      if (half) pv[pos] = vote;
+      workers_sync();
+      if (!half && t < P) a.votes[(size_t)unit * v.cap + t] = vote + pv[pos];
+    }
+  };
+
+  // waits for the chain in TMEM buffer tb, runs its epilogue, frees the buffers
+  auto finish = [&](int it, int tb) -> bool {
+    const bool ok = mbar_wait_or_abort(&bar[tb], (phases >> tb) & 1u, kLimit, abort_flag);
+    phases ^= 1u << tb;
+    if (workers_sync_or(!ok)) return false;
+    tc_fence_after();
+    epilogue(it, tb);
+    tc_fence_before();
+    workers_sync();
+    return true;
+  };
+
+  if (warp == kTcWorkers / 32) {
+    // ======================= MMA warp =====================================
+    // the same item sequence as the workers; each chain once its keys are staged
+    int kk = 0;
+    for (int it = next_valid(it0); it < it1; it = next_valid(it + 1), ++kk) {
+      if (!mbar_wait_or_abort(&bar[3 + (kk & 1)], (kk >> 1) & 1, kLimit, abort_flag)) {
+        if (lane == 0) *abort_flag = 1;
+        break;
+      }
+      if (lane == 0) issue(kk % p.nst, kk & 1);
+      __syncwarp();
+    }
+    // every chain issued lands before TMEM is released (bounded)
+    if (lane == 0 && kk > 0) {
+      umma_commit(&bar[2]);
+      mbar_wait(&bar[2], 0, kLimit);
+    }
+    __syncwarp();
+  } else {
+    // ======================= workers ======================================
+    int cur_unit = -1, pend = -1, pend_tb = 0, k = 0;
+    int it = next_valid(it0);
+    if (it < it1) stage_copy(it, 0);
+    while (it < it1 && !failed) {
+      const int unit = it / a.n_tiles;
+      const int nxt = next_valid(it + 1);
+      if (p.nstg == 2) {
+        if (nxt < it1)
+          stage_copy(nxt, (k + 1) & 1);  // overwrites the staging of item k - 1, already dequantised
+        else
+          cp_async_commit();  // an empty group keeps the wait count below uniform
+      }
+      if (unit != cur_unit) {
+        if (pend >= 0) {
+          failed = !finish(pend, pend_tb);
+          pend = -1;
+          if (failed) break;
+        }
+        load_q(unit);
+        cur_unit = unit;
+      }
+      if (p.nst == 1 && pend >= 0) {  // the single key stage must be free
+        failed = !finish(pend, pend_tb);
+        pend = -1;
+        if (failed) break;
+      }
+      if (p.nstg == 2)
+        cp_async_wait<1>();  // this item's bundles landed (the next item's may be in flight)
+      else
+        cp_async_wait<0>();
+      workers_sync();
+      dequant(p.nstg == 2 ? (k & 1) : 0, k % p.nst);
+      fence_proxy_async();  // the keys, written here, are read by the tensor cores
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar[3 + (k & 1)]);
+      if (p.nstg == 1 && nxt < it1) {  // the staging is consumed once every worker is done
+        workers_sync();
+        stage_copy(nxt, 0);
+      }
+      if (pend >= 0) {
+        failed = !finish(pend, pend_tb);
+        if (failed) break;
+      }
+      pend = it; pend_tb = k & 1;
+      ++k;
+      it = nxt;
+    }
+    if (!failed && pend >= 0) failed = !finish(pend, pend_tb);
+    cp_async_wait<0>();  // no copy outlives the CTA
+    if (failed) {
+      *abort_flag = 1;
+      if (tid == 0) set_err(a.err, 8);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512)
+                 : "memory");
+  pdl_trigger();
+}
+
+// Shared-memory plan of the tensor-core kernels: the query rows first (hi,
+// then lo), so that the statistics pass's reads past the last query row
+// (at most 112 rows of 128 bytes per box) stay inside the key stages that
+// follow; two key stages when they fit, else one; two staging buffers of
+// the K bundles.  Bundle strides are odd multiples of 16 bytes, so the
+// 16-byte loads of eight consecutive positions fall in distinct banks.
+TcPlan tc_plan(const EvictArgs &a, int sms) {
+  TcPlan p;
+  const int R = a.n_win * a.G;
+  p.R16 = (R + 15) / 16 * 16;
+  p.nch = (p.R16 + 127) / 128;
+  p.q_lo = a.q_f32 ? 1 : 0;
+  p.k_lo = a.v.bits != 16 ? 1 : 0;
+  p.fmt = a.v.bits == 16 ? kFmtBf16
+          : a.v.scheme == kSchemeSym ? (a.v.bits == 8 ? kFmtS8 : a.v.bits == 4 ? kFmtS4 : kFmtS2)
+                                     : (a.v.bits == 8 ? kFmtG8 : kFmtG4);
+  const int ks16 = TcFmtKs16(p.fmt);
+  const int extra = a.v.bits == 16 ? 0 : a.v.scheme == kSchemeSym ? 1 : meta_bytes(128, a.v.group) / 16;
+  p.kb_nch = ks16 + (a.v.scheme == kSchemeSym ? 0 : extra);  // the scale word is copied apart
+  const int kb = ks16 + extra;
+  p.kb_stride = 16 * (kb % 2 ? kb : kb + 1);
+  p.stg_bytes = kT * p.kb_stride;
+  p.stage = p.k_lo ? 4 * 128 * 128 : 2 * 128 * 128;
+  p.off_q = 0;
+  p.off_ql = p.R16 * 256;
+  const int qbytes = p.R16 * 256 * (p.q_lo ? 2 : 1);
+  p.off_k = (qbytes + 1023) / 1024 * 1024;
+  auto fits = [&](int nst, int nstg) {
+    return p.off_k + nst * p.stage + nstg * p.stg_bytes + 256 * 4 + 128 * 4 + 64 + 1024 <= 232448;
+  };
+  p.nst = fits(2, 2) ? 2 : 1;
+  p.nstg = fits(p.nst, 2) ? 2 : 1;
+  p.off_stg = p.off_k + p.nst * p.stage;
+  p.off_norm = p.off_stg + p.nstg * p.stg_bytes;
+  p.off_pv = p.off_norm + 256 * 4;
+  p.off_bar = p.off_pv + 128 * 4;
+  p.smem = p.off_bar + 64 + 1024;  // + alignment of the base to 1024 bytes
+  p.n_items = a.v.B * a.v.Hkv * a.n_tiles;
+  const int grid = std::max(1, std::min(p.n_items, sms));
+  p.items_per_cta = (p.n_items + grid - 1) / grid;
+  return p;
+}
+
+cudaError_t launch_evict_tc(const EvictArgs &a, cudaStream_t st) {
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+  }
+  const TcPlan p = tc_plan(a, sms);
+  cudaError_t e = cudaFuncSetAttribute(evict_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       p.smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(evict_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((p.n_items + p.items_per_cta - 1) / p.items_per_cta);
+  e = launch_pdl(evict_tc_kernel<false>, grid, dim3(kTcThreads), p.smem, st, a, p);
+  if (e == cudaSuccess) {
+    const int rows = a.v.B * a.v.Hkv * a.n_win * a.G;
+    e = launch_pdl(evict_merge_stats_kernel, dim3((rows + kMergeWarps - 1) / kMergeWarps),
+                   dim3(32 * kMergeWarps), 0, st, a);
+  }
+  if (e == cudaSuccess) e = launch_pdl(evict_tc_kernel<true>, grid, dim3(kTcThreads), p.smem, st, a, p);
+  if (e == cudaSuccess)
+    e = launch_pdl(evict_select_kernel, dim3(a.v.Hkv, a.v.B), dim3(1024), 0, st, a);
+  return e;
 }
 
 template <int D>
@@ -352,7 +972,8 @@ cudaError_t launch_evict_d(const EvictArgs &a, cudaStream_t st) {
   e = launch_pdl(evict_scores_kernel<D>, dim3(a.n_tiles, a.v.Hkv, a.v.B), dim3(kThreads), smem, st, a);
   if (e == cudaSuccess) {
     const int rows = a.v.B * a.v.Hkv * a.n_win * a.G;
-    e = launch_pdl(evict_merge_stats_kernel, dim3((rows + 127) / 128), dim3(128), 0, st, a);
+    e = launch_pdl(evict_merge_stats_kernel, dim3((rows + kMergeWarps - 1) / kMergeWarps),
+                   dim3(32 * kMergeWarps), 0, st, a);
   }
   if (e == cudaSuccess)
     e = launch_pdl(evict_votes_kernel, dim3((a.v.cap + kVoteT - 1) / kVoteT, a.v.Hkv, a.v.B),
@@ -365,6 +986,7 @@ cudaError_t launch_evict_d(const EvictArgs &a, cudaStream_t st) {
 }  // namespace
 
 cudaError_t launch_gqa_evict(const EvictArgs &a, cudaStream_t st) {
+  if (evict_uses_tc(a.v.D, a.n_win * a.G)) return launch_evict_tc(a, st);
   switch (a.v.D) {
     case 128: return launch_evict_d<128>(a, st);
     case 64: return launch_evict_d<64>(a, st);

@@ -80,13 +80,19 @@ struct EvictArgs {
   float sig_log2;      // softmax scale * log2(e)
   int n_tiles;         // 128-position tiles launched per (sequence, kv head)
   int sc_stride;       // n_tiles * kEvictTile: row stride of the scores
+  int stat_sub;        // statistics entries per tile and row (1 or 2)
   float *votes;        // [B * Hkv][cap]
-  float2 *stats;       // [B * Hkv][R][n_tiles] per-tile (max, sum), then [B * Hkv][R] merged
+  float2 *stats;       // [B * Hkv][R][n_tiles * stat_sub] per-tile (max, sum)
+  float2 *fin;         // [B * Hkv][R] merged (max, sum)
   float *scores;       // [B * Hkv][R][sc_stride] scaled scores (log2 domain)
   int32_t *err;
 };
 cudaError_t launch_gqa_evict(const EvictArgs &a, cudaStream_t st);
 constexpr int kEvictTile = 128;
+// Whether the evictor scores on the tensor cores (head_dim 128, at most 256
+// window query rows per KV head); otherwise it scores on the CUDA cores and
+// stores the scores.
+inline bool evict_uses_tc(int D, int R) { return D == 128 && R >= 1 && R <= 256; }
 
 cudaError_t launch_gqa_export(const GqaView &v, void *k_out, void *v_out, float *k_scale,
                               float *k_zero, float *v_scale, float *v_zero, void *k_resid,
