@@ -765,9 +765,9 @@ def profile_case(kind):
             for l in range(3):
                 c.decode(l, q, w.sigma)
     elif kind in ("evict", "evict-small"):
-        # the evictor at the long-context 14B shape, or a 1-sequence, 32768-position
-        # case (70 MB of cache, 168 MB of scores) for multi-pass captures
-        B, T = (4, 131072) if kind == "evict" else (1, 32768)
+        # the evictor at the long-context 14B shape, or its one-sequence slice
+        # (B=1: 168 MB of cache, a quarter of the items) for multi-pass captures
+        B, T = (4, 131072) if kind == "evict" else (1, 131072)
         w, c, q = _evict_setup(B, T, torch.device("cuda", 0))
         for _ in range(3):
             c.evict_window(0, q, w.sigma, w.keep)

@@ -423,15 +423,16 @@ __global__ void __launch_bounds__(1024) evict_select_kernel(const EvictArgs a) {
 // of an item reads one TMEM buffer while the next item's chain fills the
 // other.  Query rows past R are zero; in the statistics pass the last row
 // chunk may read rows past the query buffer (lanes that are never used).
-constexpr int kTcWorkers = 256;              // dequantise and run the epilogues
+constexpr int kTcWorkers = 512;              // dequantise and run the epilogues
 constexpr int kTcThreads = kTcWorkers + 32;  // + the MMA warp
+static_assert(kEvictStatSub == kTcWorkers / 128, "one statistics entry per worker column slice");
 
 // barrier 1 over the worker warps (the MMA warp runs on its own)
-__device__ __forceinline__ void workers_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+__device__ __forceinline__ void workers_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 __device__ __forceinline__ bool workers_sync_or(bool v) {
   uint32_t r;
   asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 256, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 512, p;\n selp.u32 %0, 1, 0, q;\n}\n"
       : "=r"(r)
       : "r"(v ? 1u : 0u)
       : "memory");
@@ -447,6 +448,7 @@ struct TcPlan {
   int items_per_cta, n_items;
   int R16, nch, q_lo, k_lo, nst, nstg, fmt;  // nst key stages, nstg staging buffers
   int kb_nch, kb_stride, stg_bytes;  // staged 16-byte chunks per position, their stride
+  int nc_magic;                      // ceil(2^16 / kb_nch): e / kb_nch = (e nc_magic) >> 16 here
   int stage, off_q, off_ql, off_k, off_stg, off_norm, off_pv, off_bar, smem;
 };
 
@@ -482,75 +484,91 @@ __device__ __forceinline__ float u2f(uint32_t u) {
   return __uint_as_float(0x4B000000u | u) - 8388608.f;
 }
 
-// Channels H*64 .. H*64+63 of one position's key, from its staged bundle
+// Channels 32 qc .. 32 qc + 31 of one position's key, from its staged bundle
 // (K section in logical order, then the group metadata or the symmetric
 // scale word), dequantised into the key stage (hi, and lo unless bf16).
-template <int FMT, int H>
-__device__ __forceinline__ void tc_dequant_half(const uint8_t *bundle, int row, int group,
-                                                uint8_t *kh, uint8_t *kl) {
+// Every layout places quarter qc at a fixed offset from quarter 0 with the
+// same pattern (bf16: +64 bytes per quarter; 8-bit: +64 (qc >> 1) + 8 (qc &
+// 1) bytes; 4-bit: +4 qc bytes; 2-bit: +32 (qc >> 1) + 8 (qc & 1) bits), so
+// the quarter's words are loaded at a run-time offset and the channels are
+// picked out at the compile-time positions of quarter 0.
+template <int FMT>
+__device__ __forceinline__ void tc_dequant(const uint8_t *bundle, int row, int qc, int gshift,
+                                           uint8_t *kh, uint8_t *kl) {
   using F = TcFmt<FMT>;
   constexpr int D = 128, KBOX = 128 * 128;
-  uint32_t w[F::KS / 4];
-#pragma unroll
-  for (int c = 0; c < F::KS / 16; ++c) {
-    const uint4 u = *reinterpret_cast<const uint4 *>(bundle + 16 * c);
-    w[4 * c] = u.x; w[4 * c + 1] = u.y; w[4 * c + 2] = u.z; w[4 * c + 3] = u.w;
-  }
+  const uint32_t *bw = reinterpret_cast<const uint32_t *>(bundle);
   if constexpr (F::BITS == 16) {
-    static_assert(!F::SYM, "bf16 keys carry no scale");
+    static_assert(!F::SYM && F::KS == 256, "bf16 keys: 256 bytes, no scale");
     // bf16 keys are exact: gather them into channel order, no lo part
+    uint32_t w[16];
 #pragma unroll
-    for (int cc = 0; cc < 8; ++cc) {
-      const int ch0 = H * 64 + 8 * cc;
+    for (int c = 0; c < 4; ++c) {
+      const uint4 u = reinterpret_cast<const uint4 *>(bundle)[4 * qc + c];
+      w[4 * c] = u.x; w[4 * c + 1] = u.y; w[4 * c + 2] = u.z; w[4 * c + 3] = u.w;
+    }
+#pragma unroll
+    for (int cc = 0; cc < 4; ++cc) {
       uint32_t o[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         int b0, b1, h0, h1;
-        k_pos(ch0 + 2 * i, 16, D, &b0, &h0);
-        k_pos(ch0 + 2 * i + 1, 16, D, &b1, &h1);
+        k_pos(8 * cc + 2 * i, 16, D, &b0, &h0);
+        k_pos(8 * cc + 2 * i + 1, 16, D, &b1, &h1);
         const uint32_t sel = (uint32_t)((b0 & 3) | (((b0 & 3) + 1) << 4) | ((4 + (b1 & 3)) << 8) |
                                         ((5 + (b1 & 3)) << 12));
         o[i] = __byte_perm(w[b0 >> 2], w[b1 >> 2], sel);
       }
-      put_chunk(kh, row, ch0, KBOX, make_uint4(o[0], o[1], o[2], o[3]));
+      put_chunk(kh, row, 32 * qc + 8 * cc, KBOX, make_uint4(o[0], o[1], o[2], o[3]));
     }
   } else {
     constexpr int QL = (1 << (F::BITS - 1)) - 1;  // symmetric code offset
+    // the quarter's words; channel l of quarter 0 sits in word W(l) at bit S(l)
+    constexpr int NW = F::BITS == 8 ? 8 : 4;
+    uint32_t w[NW];
+    if constexpr (F::BITS == 8) {
+      const int ob = 16 * (qc >> 1) + 2 * (qc & 1);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const uint2 u = *reinterpret_cast<const uint2 *>(bw + 4 * c + ob);
+        w[2 * c] = u.x; w[2 * c + 1] = u.y;
+      }
+    } else if constexpr (F::BITS == 4) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) w[c] = bw[4 * c + qc];
+    } else {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) w[c] = bw[2 * c + (qc >> 1)] >> (8 * (qc & 1));
+    }
     const float sym_s = F::SYM ? __uint_as_float(*reinterpret_cast<const uint32_t *>(bundle + F::KS) << 16)
                                : 0.f;
+    // groups of 32 or 64 channels: the quarter lies in one group
+    float2 m = make_float2(0.f, 0.f);
+    if constexpr (!F::SYM) m = *reinterpret_cast<const float2 *>(bundle + F::KS + 8 * ((32 * qc) >> gshift));
 #pragma unroll
-    for (int cc = 0; cc < 8; ++cc) {
-      const int ch0 = H * 64 + 8 * cc;
-      float2 m = make_float2(0.f, 0.f);
-      if constexpr (!F::SYM) m = *reinterpret_cast<const float2 *>(bundle + F::KS + 8 * (ch0 / group));
+    for (int cc = 0; cc < 4; ++cc) {
+      const int ch0 = 32 * qc + 8 * cc;
       float x[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const int ch = ch0 + i;
-        if constexpr (F::SYM) {
-          const int lb = sym_k_bit(ch, F::BITS, D);
-          const uint32_t u = (w[lb >> 5] >> (lb & 31)) & ((1u << F::BITS) - 1u);
-          x[i] = sym_s * (u2f(u) - (float)QL);
+        const int l = 8 * cc + i;  // channel of quarter 0
+        int wi, sh;
+        if constexpr (F::BITS == 2) {
+          const int bit = sym_k_bit(l, 2, D);
+          wi = bit >> 6;
+          sh = bit & 63;
         } else {
           int byte, hi;
-          k_pos(ch, F::BITS, D, &byte, &hi);
-          const int sh = 8 * (byte & 3) + (F::BITS == 4 && hi ? 4 : 0);
-          const uint32_t u = (w[byte >> 2] >> sh) & ((1u << F::BITS) - 1u);
-          x[i] = fmaf(u2f(u), m.x, m.y);
+          k_pos(l, F::BITS, D, &byte, &hi);
+          wi = F::BITS == 8 ? 2 * (byte >> 4) + ((byte & 15) >> 2) : byte >> 4;
+          sh = 8 * (byte & 3) + 4 * hi;
         }
+        const uint32_t u = (w[wi] >> sh) & ((1u << F::BITS) - 1u);
+        x[i] = F::SYM ? sym_s * (u2f(u) - (float)QL) : fmaf(u2f(u), m.x, m.y);
       }
       put8(kh, kl, true, row, ch0, KBOX, x);
     }
   }
-}
-
-template <int FMT>
-__device__ __forceinline__ void tc_dequant(const uint8_t *bundle, int row, int half, int group,
-                                           uint8_t *kh, uint8_t *kl) {
-  if (half == 0)
-    tc_dequant_half<FMT, 0>(bundle, row, group, kh, kl);
-  else
-    tc_dequant_half<FMT, 1>(bundle, row, group, kh, kl);
 }
 
 template <bool VOTES>
@@ -569,6 +587,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int R = a.n_win * a.G;
   constexpr uint32_t kLimit = 1u << 22;
+  constexpr uint32_t kSleepyLimit = 1u << 20;  // polls of up to 2 us each
   constexpr int D = 128;
   constexpr int KBOX = 128 * 128;  // bytes of one 64-channel box of a 128-row key tile
 
@@ -592,19 +611,51 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
 
   const int it0 = blockIdx.x * p.items_per_cta;
   const int it1 = min(it0 + p.items_per_cta, p.n_items);
-  const int quarter = warp & 3, half = warp >> 2;
+  // worker warp w reads TMEM lanes 32 (w % 4) .. + 31; slice = w / 4
+  const int quarter = warp & 3, slice = warp >> 2;
   const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
   uint32_t phases = 0u;  // bit tb: parity of TMEM buffer tb's next completion
   bool failed = false;
 
-  auto valid = [&](int it) {
-    const int len = v.lens[(it / a.n_tiles) / v.Hkv];
-    const int t0 = (it % a.n_tiles) * kT;
-    return len > a.budget && t0 < (VOTES ? len - a.n_win : len);
+  const int gshift = v.group == 64 ? 6 : 5;  // grouped layers: groups of 32 or 64 channels
+  // rows of this thread in the statistics epilogue, divided by G (the row's
+  // window query), once
+  int rdiv[2];
+#pragma unroll
+  for (int c = 0; c < 2; ++c) rdiv[c] = (128 * c + 32 * quarter + lane) / a.G;
+  // (unit, tile) of item `it` and the unit's length, advanced without divisions
+  struct Cursor {
+    int it, unit, tile, len;
   };
-  auto next_valid = [&](int it) {
-    while (it < it1 && !valid(it)) ++it;
-    return it;
+  const int units = v.B * v.Hkv;
+  auto at = [&](int it) {
+    Cursor c;
+    c.it = it;
+    c.unit = it / a.n_tiles;
+    c.tile = it - c.unit * a.n_tiles;
+    c.len = c.unit < units ? v.lens[c.unit / v.Hkv] : 0;
+    return c;
+  };
+  auto next_valid = [&](Cursor c) {  // c or the first valid item after it (c.it == it1: none)
+    while (c.it < it1) {
+      if (c.len > a.budget && c.tile * kT < (VOTES ? c.len - a.n_win : c.len)) break;
+      // an invalid item has no valid successor in its unit: on to the next unit
+      c.it += a.n_tiles - c.tile;
+      c.tile = 0;
+      ++c.unit;
+      c.len = c.unit < units ? v.lens[c.unit / v.Hkv] : 0;
+    }
+    c.it = min(c.it, it1);
+    return c;
+  };
+  auto after = [&](Cursor c) {  // the item after c
+    ++c.it;
+    if (++c.tile == a.n_tiles) {
+      c.tile = 0;
+      ++c.unit;
+      c.len = c.unit < units ? v.lens[c.unit / v.Hkv] : 0;
+    }
+    return c;
   };
 
   // query rows of `unit` (and, for the votes, the rows' log-normalisers;
@@ -654,9 +705,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
   // asynchronous copy of the K bundles of item `it` (K section in logical
   // order, then the group metadata or the symmetric scale word) into staging
   // buffer g; one commit group per call
-  auto stage_copy = [&](int it, int g) {
-    const int unit = it / a.n_tiles, t0 = (it % a.n_tiles) * kT;
-    const int len = v.lens[unit / v.Hkv];
+  auto stage_copy = [&](const Cursor &cu, int g) {
+    const int unit = cu.unit, t0 = cu.tile * kT, len = cu.len;
     uint8_t *dst0 = sm + p.off_stg + g * p.stg_bytes;
     const int NC = p.kb_nch;
     const int ks16 = TcFmtKs16(p.fmt);
@@ -665,7 +715,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
     const int km = ks16 * 32;  // grouped: key metadata follows the K and V sections
     const uint8_t *base = v.rec + (size_t)unit * v.cap * v.rec_bytes;
     for (int e = tid; e < kT * NC; e += kTcWorkers) {
-      const int pos = e / NC, c = e - pos * NC;
+      const int pos = (e * p.nc_magic) >> 16, c = e - pos * NC;
       const int t = t0 + pos;
       const bool ok = t < len;
       const int so = sym ? 16 * ((c + sym_rot(t, nrec)) & (nrec - 1)) : c < ks16 ? 16 * c : km + 16 * (c - ks16);
@@ -683,16 +733,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
 
   // dequantised keys of the item staged in buffer g into key stage s
   auto dequant = [&](int g, int s) {
-    const int pidx = tid & 127, hf = tid >> 7;
+    const int pidx = tid & 127, hf = tid >> 7;  // position, channel quarter
     const uint8_t *bundle = sm + p.off_stg + g * p.stg_bytes + pidx * p.kb_stride;
     uint8_t *kh = sm + p.off_k + s * p.stage, *kl = kh + 2 * KBOX;
     switch (p.fmt) {
-      case kFmtBf16: tc_dequant<kFmtBf16>(bundle, pidx, hf, v.group, kh, kl); break;
-      case kFmtG8: tc_dequant<kFmtG8>(bundle, pidx, hf, v.group, kh, kl); break;
-      case kFmtG4: tc_dequant<kFmtG4>(bundle, pidx, hf, v.group, kh, kl); break;
-      case kFmtS8: tc_dequant<kFmtS8>(bundle, pidx, hf, v.group, kh, kl); break;
-      case kFmtS4: tc_dequant<kFmtS4>(bundle, pidx, hf, v.group, kh, kl); break;
-      default: tc_dequant<kFmtS2>(bundle, pidx, hf, v.group, kh, kl); break;
+      case kFmtBf16: tc_dequant<kFmtBf16>(bundle, pidx, hf, gshift, kh, kl); break;
+      case kFmtG8: tc_dequant<kFmtG8>(bundle, pidx, hf, gshift, kh, kl); break;
+      case kFmtG4: tc_dequant<kFmtG4>(bundle, pidx, hf, gshift, kh, kl); break;
+      case kFmtS8: tc_dequant<kFmtS8>(bundle, pidx, hf, gshift, kh, kl); break;
+      case kFmtS4: tc_dequant<kFmtS4>(bundle, pidx, hf, gshift, kh, kl); break;
+      default: tc_dequant<kFmtS2>(bundle, pidx, hf, gshift, kh, kl); break;
     }
   };
 
@@ -731,54 +781,56 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
   };
 
   // epilogue of item `it` from TMEM buffer tb
-  auto epilogue = [&](int it, int tb) {
-    const int unit = it / a.n_tiles, tile = it % a.n_tiles;
-    const int len = v.lens[unit / v.Hkv];
+  auto epilogue = [&](const Cursor &cu, int tb) {
+    const int unit = cu.unit, tile = cu.tile, len = cu.len;
     const int P = len - a.n_win;
     const int t0 = tile * kT;
     const float sg = a.sig_log2;
     if constexpr (!VOTES) {
-      float2 *st = a.stats + (size_t)unit * R * (2 * a.n_tiles);
+      float2 *st = a.stats + (size_t)unit * R * (kEvictStatSub * a.n_tiles);
       for (int c = 0; c < p.nch; ++c) {
         if (128 * c + 32 * quarter >= R) continue;  // the warp's rows are all padding
         const int r = 128 * c + 32 * quarter + lane;
-        const int last = P + r / a.G;  // the last position row r sees
-        float y[64];
-        const uint32_t ta = tmem + 256u * tb + 128 * c + 64 * half + lane_off;
+        const int last = P + (c == 0 ? rdiv[0] : rdiv[1]);  // the last position row r sees
+        float y[32];
+        const uint32_t ta = tmem + 256u * tb + 128 * c + 32 * slice + lane_off;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < 2; ++q) {
           float z[16];
           tmem_ld16(ta + 16 * q, z);
 #pragma unroll
           for (int i = 0; i < 16; ++i) y[16 * q + i] = z[i];
         }
-        const int tb0 = t0 + 64 * half;
-        const int nv = min(64, last - tb0 + 1);  // positions of the half row r sees
+        const int tb0 = t0 + 32 * slice;
+        const int nv = min(32, last - tb0 + 1);  // positions of the slice row r sees
         float m = -INFINITY, l = 0.f;
-        if (nv >= 64) {
+        if (nv >= 32) {  // four independent chains each
+          float mm[4] = {y[0], y[1], y[2], y[3]}, ll[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int i = 0; i < 64; ++i) m = fmaxf(m, y[i]);
-          const float ms = m * sg;
+          for (int i = 4; i < 32; ++i) mm[i & 3] = fmaxf(mm[i & 3], y[i]);
+          const float ms = fmaxf(fmaxf(mm[0], mm[1]), fmaxf(mm[2], mm[3])) * sg;
 #pragma unroll
-          for (int i = 0; i < 64; ++i) l += fast_exp2(fmaf(y[i], sg, -ms));
+          for (int i = 0; i < 32; ++i) ll[i & 3] += fast_exp2(fmaf(y[i], sg, -ms));
           m = ms;
+          l = (ll[0] + ll[1]) + (ll[2] + ll[3]);
         } else if (nv > 0) {
 #pragma unroll
-          for (int i = 0; i < 64; ++i)
+          for (int i = 0; i < 32; ++i)
             if (i < nv) m = fmaxf(m, y[i]);
           const float ms = m * sg;
 #pragma unroll
-          for (int i = 0; i < 64; ++i)
+          for (int i = 0; i < 32; ++i)
             if (i < nv) l += fast_exp2(fmaf(y[i], sg, -ms));
           m = ms;
         }
-        if (r < R) st[(size_t)r * (2 * a.n_tiles) + 2 * tile + half] = make_float2(m, l);
+        if (r < R)
+          st[(size_t)r * (kEvictStatSub * a.n_tiles) + kEvictStatSub * tile + slice] = make_float2(m, l);
       }
     } else {
       const int pos = 32 * quarter + lane, t = t0 + pos;
-      const int n16 = p.R16 / 16, h0 = (n16 + 1) / 2;
-      const int bk0 = half ? h0 : 0, bk1 = half ? n16 : h0;
-      float vote = 0.f;
+      const int n16 = p.R16 / 16, per = (n16 + 3) / 4;
+      const int bk0 = min(n16, slice * per), bk1 = min(n16, bk0 + per);
+      float vv[4] = {0.f, 0.f, 0.f, 0.f};  // four independent chains
       for (int bk = bk0; bk < bk1; ++bk) {
         float y[16];
         tmem_ld16(tmem + 256u * tb + 16 * bk + lane_off, y);
@@ -786,21 +838,22 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
 #pragma unroll
         for (int i4 = 0; i4 < 4; ++i4) {
           const float4 c4 = nr[i4];
-          vote += fast_exp2(fmaf(y[4 * i4], sg, -c4.x));
-          vote += fast_exp2(fmaf(y[4 * i4 + 1], sg, -c4.y));
-          vote += fast_exp2(fmaf(y[4 * i4 + 2], sg, -c4.z));
-          vote += fast_exp2(fmaf(y[4 * i4 + 3], sg, -c4.w));
+          vv[0] += fast_exp2(fmaf(y[4 * i4], sg, -c4.x));
+          vv[1] += fast_exp2(fmaf(y[4 * i4 + 1], sg, -c4.y));
+          vv[2] += fast_exp2(fmaf(y[4 * i4 + 2], sg, -c4.z));
+          vv[3] += fast_exp2(fmaf(y[4 * i4 + 3], sg, -c4.w));
         }
       }
-      if (half) pv[pos] = vote;
+      const float vote = (vv[0] + vv[1]) + (vv[2] + vv[3]);
+      if (slice) pv[(slice - 1) * 128 + pos] = vote;
       workers_sync();
-      if (!half && t < P) a.votes[(size_t)unit * v.cap + t] = vote + pv[pos];
+      if (!slice && t < P) a.votes[(size_t)unit * v.cap + t] = vote + pv[pos] + pv[128 + pos] + pv[256 + pos];
     }
   };
 
   // waits for the chain in TMEM buffer tb, runs its epilogue, frees the buffers
-  auto finish = [&](int it, int tb) -> bool {
-    const bool ok = mbar_wait_or_abort(&bar[tb], (phases >> tb) & 1u, kLimit, abort_flag);
+  auto finish = [&](const Cursor &it, int tb) -> bool {
+    const bool ok = mbar_wait_sleepy(&bar[tb], (phases >> tb) & 1u, kSleepyLimit, abort_flag, 2000);
     phases ^= 1u << tb;
     if (workers_sync_or(!ok)) return false;
     tc_fence_after();
@@ -814,8 +867,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
     // ======================= MMA warp =====================================
     // the same item sequence as the workers; each chain once its keys are staged
     int kk = 0;
-    for (int it = next_valid(it0); it < it1; it = next_valid(it + 1), ++kk) {
-      if (!mbar_wait_or_abort(&bar[3 + (kk & 1)], (kk >> 1) & 1, kLimit, abort_flag)) {
+    for (Cursor cu = next_valid(at(it0)); cu.it < it1; cu = next_valid(after(cu)), ++kk) {
+      if (!mbar_wait_sleepy(&bar[3 + (kk & 1)], (kk >> 1) & 1, kSleepyLimit, abort_flag, 2000)) {
         if (lane == 0) *abort_flag = 1;
         break;
       }
@@ -830,30 +883,32 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
     __syncwarp();
   } else {
     // ======================= workers ======================================
-    int cur_unit = -1, pend = -1, pend_tb = 0, k = 0;
-    int it = next_valid(it0);
-    if (it < it1) stage_copy(it, 0);
-    while (it < it1 && !failed) {
-      const int unit = it / a.n_tiles;
-      const int nxt = next_valid(it + 1);
+    int cur_unit = -1, pend_tb = 0, k = 0;
+    bool has_pend = false;
+    Cursor pend;
+    Cursor it = next_valid(at(it0));
+    if (it.it < it1) stage_copy(it, 0);
+    while (it.it < it1 && !failed) {
+      const int unit = it.unit;
+      const Cursor nxt = next_valid(after(it));
       if (p.nstg == 2) {
-        if (nxt < it1)
+        if (nxt.it < it1)
           stage_copy(nxt, (k + 1) & 1);  // overwrites the staging of item k - 1, already dequantised
         else
           cp_async_commit();  // an empty group keeps the wait count below uniform
       }
       if (unit != cur_unit) {
-        if (pend >= 0) {
+        if (has_pend) {
           failed = !finish(pend, pend_tb);
-          pend = -1;
+          has_pend = false;
           if (failed) break;
         }
         load_q(unit);
         cur_unit = unit;
       }
-      if (p.nst == 1 && pend >= 0) {  // the single key stage must be free
+      if (p.nst == 1 && has_pend) {  // the single key stage must be free
         failed = !finish(pend, pend_tb);
-        pend = -1;
+        has_pend = false;
         if (failed) break;
       }
       if (p.nstg == 2)
@@ -865,19 +920,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
       fence_proxy_async();  // the keys, written here, are read by the tensor cores
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar[3 + (k & 1)]);
-      if (p.nstg == 1 && nxt < it1) {  // the staging is consumed once every worker is done
+      if (p.nstg == 1 && nxt.it < it1) {  // the staging is consumed once every worker is done
         workers_sync();
         stage_copy(nxt, 0);
       }
-      if (pend >= 0) {
+      if (has_pend) {
         failed = !finish(pend, pend_tb);
         if (failed) break;
       }
-      pend = it; pend_tb = k & 1;
+      pend = it; pend_tb = k & 1; has_pend = true;
       ++k;
       it = nxt;
     }
-    if (!failed && pend >= 0) failed = !finish(pend, pend_tb);
+    if (!failed && has_pend) failed = !finish(pend, pend_tb);
     cp_async_wait<0>();  // no copy outlives the CTA
     if (failed) {
       *abort_flag = 1;
@@ -914,6 +969,7 @@ TcPlan tc_plan(const EvictArgs &a, int sms) {
   p.kb_nch = ks16 + (a.v.scheme == kSchemeSym ? 0 : extra);  // the scale word is copied apart
   const int kb = ks16 + extra;
   p.kb_stride = 16 * (kb % 2 ? kb : kb + 1);
+  p.nc_magic = (65536 + p.kb_nch - 1) / p.kb_nch;
   p.stg_bytes = kT * p.kb_stride;
   p.stage = p.k_lo ? 4 * 128 * 128 : 2 * 128 * 128;
   p.off_q = 0;
@@ -921,14 +977,14 @@ TcPlan tc_plan(const EvictArgs &a, int sms) {
   const int qbytes = p.R16 * 256 * (p.q_lo ? 2 : 1);
   p.off_k = (qbytes + 1023) / 1024 * 1024;
   auto fits = [&](int nst, int nstg) {
-    return p.off_k + nst * p.stage + nstg * p.stg_bytes + 256 * 4 + 128 * 4 + 64 + 1024 <= 232448;
+    return p.off_k + nst * p.stage + nstg * p.stg_bytes + 256 * 4 + 3 * 128 * 4 + 64 + 1024 <= 232448;
   };
   p.nst = fits(2, 2) ? 2 : 1;
   p.nstg = fits(p.nst, 2) ? 2 : 1;
   p.off_stg = p.off_k + p.nst * p.stage;
   p.off_norm = p.off_stg + p.nstg * p.stg_bytes;
   p.off_pv = p.off_norm + 256 * 4;
-  p.off_bar = p.off_pv + 128 * 4;
+  p.off_bar = p.off_pv + 3 * 128 * 4;
   p.smem = p.off_bar + 64 + 1024;  // + alignment of the base to 1024 bytes
   p.n_items = a.v.B * a.v.Hkv * a.n_tiles;
   const int grid = std::max(1, std::min(p.n_items, sms));

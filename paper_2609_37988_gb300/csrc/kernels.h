@@ -80,7 +80,7 @@ struct EvictArgs {
   float sig_log2;      // softmax scale * log2(e)
   int n_tiles;         // 128-position tiles launched per (sequence, kv head)
   int sc_stride;       // n_tiles * kEvictTile: row stride of the scores
-  int stat_sub;        // statistics entries per tile and row (1 or 2)
+  int stat_sub;        // statistics entries per tile and row (1 or kEvictStatSub)
   float *votes;        // [B * Hkv][cap]
   float2 *stats;       // [B * Hkv][R][n_tiles * stat_sub] per-tile (max, sum)
   float2 *fin;         // [B * Hkv][R] merged (max, sum)
@@ -89,6 +89,7 @@ struct EvictArgs {
 };
 cudaError_t launch_gqa_evict(const EvictArgs &a, cudaStream_t st);
 constexpr int kEvictTile = 128;
+constexpr int kEvictStatSub = 4;  // statistics entries per tile and row, at most
 // Whether the evictor scores on the tensor cores (head_dim 128, at most 256
 // window query rows per KV head); otherwise it scores on the CUDA cores and
 // stores the scores.

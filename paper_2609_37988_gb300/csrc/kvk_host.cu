@@ -543,7 +543,7 @@ EvictScratch evict_scratch(const kvk_cache *c, int layer, int n_win) {
   const size_t R = (size_t)n_win * (c->desc.n_q_heads / c->desc.n_kv_heads);
   e.n_tiles = (int)((cap + kEvictTile - 1) / kEvictTile);
   e.votes = align256((int64_t)(units * cap * 4));
-  e.stats = align256((int64_t)((units * R * 2 * e.n_tiles + units * R) * 8));
+  e.stats = align256((int64_t)((units * R * kEvictStatSub * e.n_tiles + units * R) * 8));
   e.scores = evict_uses_tc(c->desc.head_dim, (int)R)
                  ? 0
                  : align256((int64_t)(units * R * e.n_tiles * kEvictTile * 4));
@@ -604,10 +604,11 @@ kvk_status kvk_evict_window(kvk_cache *c, int32_t layer, const void *q_win, int3
   a.sig_log2 = softmax_scale * 1.4426950408889634f;
   a.n_tiles = es.n_tiles;
   a.sc_stride = es.n_tiles * kEvictTile;
-  a.stat_sub = evict_uses_tc(c->desc.head_dim, n_win * a.G) ? 2 : 1;
+  a.stat_sub = evict_uses_tc(c->desc.head_dim, n_win * a.G) ? kEvictStatSub : 1;
   a.votes = static_cast<float *>(scratch);
   a.stats = reinterpret_cast<float2 *>(static_cast<uint8_t *>(scratch) + es.votes);
-  a.fin = a.stats + (size_t)c->desc.max_batch * c->desc.n_kv_heads * n_win * a.G * 2 * es.n_tiles;
+  a.fin = a.stats + (size_t)c->desc.max_batch * c->desc.n_kv_heads * n_win * a.G * kEvictStatSub *
+                        es.n_tiles;
   a.scores = es.scores ? reinterpret_cast<float *>(static_cast<uint8_t *>(scratch) + es.votes + es.stats)
                        : nullptr;
   a.err = c->err();

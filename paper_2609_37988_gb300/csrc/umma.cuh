@@ -86,4 +86,22 @@ __device__ __forceinline__ bool mbar_wait_or_abort(uint64_t *bar, uint32_t parit
   }
   return false;
 }
+// As mbar_wait_or_abort, each poll suspending the thread for up to
+// `hint_ns` nanoseconds while the phase is incomplete (it resumes as soon as
+// the phase completes), so a waiting warp issues few instructions.
+__device__ __forceinline__ bool mbar_wait_sleepy(uint64_t *bar, uint32_t parity, uint32_t limit,
+                                                 const volatile int *abort_flag, uint32_t hint_ns) {
+  const uint32_t a = smem_u32(bar);
+  for (uint32_t i = 0; i < limit; ++i) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(a), "r"(parity), "r"(hint_ns)
+        : "memory");
+    if (ok) return true;
+    if ((i & 7) == 7 && *abort_flag) return false;
+  }
+  return false;
+}
 }  // namespace kvk
