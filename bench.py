@@ -209,6 +209,43 @@ def cpu_baseline(w, seconds=12.0):
     return nbytes / dt / 1e9, sample, cores
 
 
+def cpu_baseline_mla(w, seconds=12.0):
+    """The oracle's unabsorbed MLA decode (as it stands) on one sequence of
+    the widest and of the narrowest latent layer of the workload (inputs
+    drawn for a batch of one).  Bytes counted as on the GPU: the sequence's
+    latent cache [c[:d] | k^R] in bf16.  Returns (GB/s, sample text, cores)."""
+    from oracle import attention as oatt
+    from paper_2609_37988_gb300 import workloads as W
+
+    w1 = W.config(4, batch=1)
+    T = w1.context
+    widths = {}
+    for l, a in enumerate(w1.layers):
+        widths.setdefault(a["width"], l)
+    units = []
+    for d in sorted({max(widths), min(widths)}):
+        l = widths[d]
+        cl, kr = W.mla_inputs(w1, l, 0, T)
+        wk, wv = W.mla_weights(w1, l)
+        qn, qp = W.mla_queries(w1, l)
+        units.append((d, qn.float().numpy(), qp.float().numpy(), cl.float().numpy(),
+                      kr.float().numpy(), wk.float().numpy(), wv.float().numpy()))
+    nbytes, n = 0, 0
+    t0 = time.perf_counter()
+    while True:
+        for d, qn, qp, cl, kr, wk, wv in units:
+            oatt.mla_decode_unabsorbed(qn, qp, cl, kr, wk, wv, d, [T], w1.sigma)
+            nbytes += T * (d + w1.rope_dim) * 2
+        n += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0))
+    sample = (f"{n} passes over one sequence of a d={max(widths)} and a d={min(widths)} latent "
+              f"layer, {T} positions, {w1.n_q_heads} heads (unabsorbed oracle)")
+    return nbytes / dt / 1e9, sample, cores
+
+
 def run_reference(args):
     """--impl reference: the oracle as it stands, on the host cores."""
     rank = int(os.environ.get("RANK", "0"))
@@ -216,12 +253,13 @@ def run_reference(args):
         return
     from paper_2609_37988_gb300 import workloads as W
     w = W.config(args.config, sym_bits=args.sym_bits)
+    base = cpu_baseline if w.kind == "gqa" else cpu_baseline_mla
     per = max(2.0, 60.0 / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):
-        cpu_baseline(w, seconds=min(per, 3.0))
+        base(w, seconds=min(per, 3.0))
     vals = []
     for _ in range(args.steps):
-        g, sample, cores = cpu_baseline(w, seconds=per)
+        g, sample, cores = base(w, seconds=per)
         vals.append(g)
     v = statistics.median(vals)
     print(json.dumps({
@@ -501,10 +539,30 @@ def main():
 
     # ---- end to end through the public API, host buffers --------------------
     e2e = None
-    if args.e2e_steps > 0 and w.kind == "gqa":
+    if args.e2e_steps > 0:
         # one pinned host buffer and one device buffer per kind of tensor, so
         # that a step's inputs arrive in two copies and its outputs leave in one
         # (per-layer copies cost more in fixed latency than in bytes)
+        e_out_all = torch.empty((w.n_layers,) + tuple(outs[0].shape), dtype=outs[0].dtype, device=dev)
+        e_outs = list(e_out_all.unbind(0))
+        h_out_all = torch.empty(e_out_all.shape, dtype=e_out_all.dtype).pin_memory()
+        d2h = h_out_all.numel() * h_out_all.element_size()
+        if w.kind == "mla":
+            # the step's inputs are every layer's q_nope and q_pe; the
+            # up-projection weights are model parameters, resident
+            h_qn = torch.stack([a for a, _ in mq]).cpu().pin_memory()
+            h_qp = torch.stack([b for _, b in mq]).cpu().pin_memory()
+            d_qn = torch.empty_like(h_qn, device=dev)
+            d_qp = torch.empty_like(h_qp, device=dev)
+            h2d = h_qn.numel() * h_qn.element_size() + h_qp.numel() * h_qp.element_size()
+
+            def e2e_body():
+                d_qn.copy_(h_qn, non_blocking=True)
+                d_qp.copy_(h_qp, non_blocking=True)
+                for l in range(w.n_layers):
+                    cache.decode_mla(l, d_qn[l], d_qp[l], mw[l][0], mw[l][1], w.sigma, out=e_outs[l])
+                h_out_all.copy_(e_out_all, non_blocking=True)
+    if args.e2e_steps > 0 and w.kind == "gqa":
         h_q_all = torch.stack([q.cpu() for q in qs]).pin_memory()
         d_q_all = torch.empty_like(h_q_all, device=dev)
         d_q = list(d_q_all.unbind(0))
@@ -513,26 +571,23 @@ def main():
                     if kv_layers else None)
         d_kv_all = torch.empty_like(h_kv_all, device=dev) if kv_layers else None
         d_kv = {a: (d_kv_all[2 * i], d_kv_all[2 * i + 1]) for i, a in enumerate(kv_layers)}
-        e_out_all = torch.empty((w.n_layers,) + tuple(outs[0].shape), dtype=outs[0].dtype, device=dev)
-        e_outs = list(e_out_all.unbind(0))
-        h_out_all = torch.empty(e_out_all.shape, dtype=e_out_all.dtype).pin_memory()
         h2d = h_q_all.numel() * h_q_all.element_size() + \
             (h_kv_all.numel() * h_kv_all.element_size() if kv_layers else 0)
-        d2h = h_out_all.numel() * h_out_all.element_size()
+
+        def e2e_body():
+            d_q_all.copy_(h_q_all, non_blocking=True)
+            if kv_layers:
+                d_kv_all.copy_(h_kv_all, non_blocking=True)
+            for l in range(w.n_layers):
+                if l in d_kv:
+                    cache.append(l, *d_kv[l])
+                cache.decode(l, d_q[l], w.sigma, out=e_outs[l])
+            h_out_all.copy_(e_out_all, non_blocking=True)
+            if w.append_per_step:
+                cache.rewind(1)
+    if args.e2e_steps > 0:
         e2e_mode = "eager"
         with torch.cuda.stream(stream):
-            def e2e_body():
-                d_q_all.copy_(h_q_all, non_blocking=True)
-                if kv_layers:
-                    d_kv_all.copy_(h_kv_all, non_blocking=True)
-                for l in range(w.n_layers):
-                    if l in d_kv:
-                        cache.append(l, *d_kv[l])
-                    cache.decode(l, d_q[l], w.sigma, out=e_outs[l])
-                h_out_all.copy_(e_out_all, non_blocking=True)
-                if w.append_per_step:
-                    cache.rewind(1)
-
             def e2e_step():
                 e2e_body()
                 stream.synchronize()
@@ -563,8 +618,8 @@ def main():
 
     err = cache.device_error()
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and w.kind == "gqa":
-        g, sample, cores = cpu_baseline(w)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        g, sample, cores = cpu_baseline(w) if w.kind == "gqa" else cpu_baseline_mla(w)
         cpu = {"value": g, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
     clocks = clk.summary()
     if rank == 0:
