@@ -12,7 +12,7 @@ Modules
 -------
 quant      grouped asymmetric quantiser (fp32 op sequence), dequantisation
            (fp64), the paper's symmetric per-vector quantiser (Appendix C.3).
-attention  layer -> source resolution (Sec. 2.1, depth axis), GQA decode
+attention  layer -> source resolution (Sec. 2.1, depth axis), GQA decode and causal chunk (prefill) attention
            attention over dequantised caches, kept-position gather, MLA
            decode in the unabsorbed form (Appendix C.2).
 evict      the attention-scored evictor composed with the cache (Sec. 3.3):

@@ -11,6 +11,13 @@ Everything here runs in float64 on already-dequantised caches.
   positions the layer reads, output ``sum_t p_t v_t``.  With a kept-position
   list (eviction composed with compression, Sec. 3.3) only the listed
   positions are read.
+* ``gqa_prefill`` -- attention of a chunk of new queries over the
+  compressed cache: the chunk is the last ``C`` positions of each sequence
+  (already written to the cache), and query ``i`` at position
+  ``len - C + i`` attends causally to positions ``0 .. len - C + i`` of the
+  dequantised cache (the other side of the step the paper times as
+  pre-fill, Sec. 5: the cache holds the compressed keys and values the
+  decode steps then read).  Queries before position 0 give zeros.
 * ``mla_decode_unabsorbed`` -- Appendix C.2: the MLA cache holds the latent
   ``c`` truncated to its first ``d`` coordinates and the post-RoPE positional
   key ``k^R`` shared by all heads.  Head ``h`` reconstructs its content key
@@ -83,6 +90,37 @@ def gqa_decode(q, k_hat, v_hat, lens, sigma, kept=None):
             V = np.asarray(v_hat[b, j, pos], np.float64)
             p = softmax_weights(sigma * (K @ q[b, h]))
             out[b, h] = p @ V
+    return out
+
+
+def gqa_prefill(q, k_hat, v_hat, lens, sigma):
+    """Causal chunk attention over a GQA cache.
+
+    q      : ``[B, C, H_q, D]`` the queries of each sequence's last ``C``
+             positions
+    k_hat  : ``[B, H_kv, T, D]`` dequantised keys, v_hat likewise
+    lens   : ``[B]`` positions held (the chunk included)
+    Returns ``[B, C, H_q, D]`` float64.
+    """
+    q = np.asarray(q, np.float64)
+    B, C, Hq, D = q.shape
+    Hkv = k_hat.shape[1]
+    if Hq % Hkv:
+        raise ValueError("H_q must be a multiple of H_kv")
+    G = Hq // Hkv
+    out = np.zeros((B, C, Hq, D), np.float64)
+    for b in range(B):
+        L = int(lens[b])
+        for i in range(C):
+            p = L - C + i  # position of query i
+            if p < 0:
+                continue
+            for h in range(Hq):
+                j = h // G
+                K = np.asarray(k_hat[b, j, :p + 1], np.float64)
+                V = np.asarray(v_hat[b, j, :p + 1], np.float64)
+                w = softmax_weights(sigma * (K @ q[b, i, h]))
+                out[b, i, h] = w @ V
     return out
 
 

@@ -150,3 +150,69 @@ def test_plan_inheritors_read_source_and_full_precision_is_plain_attention():
     kh = quant.dequantise_per_channel(st[2]["k_codes"][1], st[2]["k_scale"][1], st[2]["k_zero"][1], 32,
                                       st[2]["k_residual"][1])
     np.testing.assert_allclose(st[2]["k_hat"][1, :, :33], kh, atol=0)
+
+
+# ---- chunk (prefill) attention ----------------------------------------------
+def _brute_prefill(q, K, V, lens, sigma):
+    B, C, Hq, D = q.shape
+    G = Hq // K.shape[1]
+    out = np.zeros(q.shape, np.float64)
+    for b in range(B):
+        for i in range(C):
+            p = int(lens[b]) - C + i
+            if p < 0:
+                continue
+            for h in range(Hq):
+                j = h // G
+                sc = [sigma * sum(float(q[b, i, h, c]) * float(K[b, j, t, c]) for c in range(D))
+                      for t in range(p + 1)]
+                m = max(sc)
+                w = [math.exp(x - m) for x in sc]
+                tot = sum(w)
+                for c in range(D):
+                    out[b, i, h, c] = sum(w[t] * float(V[b, j, t, c]) for t in range(p + 1)) / tot
+    return out
+
+
+def test_prefill_matches_brute_force():
+    rng = np.random.default_rng(3)
+    B, C, Hq, Hkv, T, D = 2, 4, 4, 2, 9, 3
+    q = rng.standard_normal((B, C, Hq, D))
+    K = rng.standard_normal((B, Hkv, T, D))
+    V = rng.standard_normal((B, Hkv, T, D))
+    lens = [9, 3]  # sequence 1: the first query sits before position 0
+    got = attention.gqa_prefill(q, K, V, lens, 0.7)
+    np.testing.assert_allclose(got, _brute_prefill(q, K, V, lens, 0.7), rtol=1e-12, atol=1e-12)
+    assert (got[1, 0] == 0).all()
+
+
+def test_prefill_matches_library_causal_sdpa():
+    # torch's scaled_dot_product_attention with an explicit causal mask whose
+    # diagonal is shifted by the cached prefix, in float64
+    rng = np.random.default_rng(4)
+    B, C, Hq, Hkv, T, D = 1, 6, 6, 3, 20, 8
+    q = rng.standard_normal((B, C, Hq, D))
+    K = rng.standard_normal((B, Hkv, T, D))
+    V = rng.standard_normal((B, Hkv, T, D))
+    G = Hq // Hkv
+    qt = torch.from_numpy(q).permute(0, 2, 1, 3)                      # [B, Hq, C, D]
+    kt = torch.from_numpy(K).repeat_interleave(G, dim=1)               # [B, Hq, T, D]
+    vt = torch.from_numpy(V).repeat_interleave(G, dim=1)
+    mask = torch.arange(T)[None, :] <= (T - C + torch.arange(C))[:, None]
+    ref = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask, scale=0.3)
+    got = attention.gqa_prefill(q, K, V, [T], 0.3)
+    np.testing.assert_allclose(got, ref.permute(0, 2, 1, 3).numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_prefill_first_position_returns_its_value_and_last_query_is_decode():
+    rng = np.random.default_rng(5)
+    B, C, Hq, Hkv, D = 1, 5, 4, 1, 6
+    q = rng.standard_normal((B, C, Hq, D))
+    K = rng.standard_normal((B, Hkv, C, D))
+    V = rng.standard_normal((B, Hkv, C, D))
+    got = attention.gqa_prefill(q, K, V, [C], 1.0)
+    # the chunk is the whole sequence: query 0 sees only position 0
+    np.testing.assert_array_equal(got[0, 0], np.broadcast_to(V[0, 0, 0], (Hq, D)))
+    # the last query sees every position: one decode step
+    np.testing.assert_allclose(got[:, -1], attention.gqa_decode(q[:, -1], K, V, [C], 1.0),
+                               rtol=1e-13, atol=1e-13)
