@@ -227,6 +227,27 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
                             int32_t n_win, float softmax_scale, int32_t budget, void *scratch,
                             size_t scratch_bytes, kvk_stream stream);
 
+/* Causal chunk attention (pre-fill) of `layer` over its compressed cache
+ * (Sec. 5 times pre-fill over compressed caches): the chunk is the last n_q
+ * positions of every sequence, already written with kvk_append; query i of
+ * sequence b sits at position len_b - n_q + i and attends to positions
+ * 0 .. len_b - n_q + i of the dequantised stored keys and values (the ones
+ * decode reads), with its own query heads (an inheriting layer reads its
+ * anchor).  Queries before position 0 (len_b < n_q) give zeros.  Kept lists
+ * are not used: pre-fill reads every position.
+ *  q:       device [B, n_q, H_q, head_dim] in q_dtype (post-RoPE);
+ *  out:     device float32 [B, n_q, H_q, head_dim];
+ *  scratch: device, 256-byte aligned, at least kvk_prefill_scratch_size
+ *           bytes (per-row softmax statistics).
+ * Errors: UNSUPPORTED (MLA, head_dim != 128, grouped per-channel keys),
+ * INVALID_ARG (n_q outside [1, max_ctx], null or misaligned pointers,
+ * scale not finite and positive, scratch too small). */
+kvk_status kvk_prefill_scratch_size(const kvk_cache *cache, int32_t layer, int32_t n_q,
+                                    size_t *scratch_bytes);
+kvk_status kvk_prefill_attention(kvk_cache *cache, int32_t layer, const void *q, int32_t q_dtype,
+                                 int32_t n_q, float softmax_scale, float *out, void *scratch,
+                                 size_t scratch_bytes, kvk_stream stream);
+
 /* Copy anchor `layer`'s kept lists out, device to device, on `stream`.
  * *per_head (host) = -1: no list installed (nothing copied); 0: lists per
  * sequence, idx [B, evict_capacity], n_kept [B]; 1: lists per (sequence, KV

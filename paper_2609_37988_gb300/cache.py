@@ -175,6 +175,27 @@ class Cache:
         return scratch[: 4 * d.max_batch * d.n_kv_heads * C].view(torch.float32).view(
             d.max_batch, d.n_kv_heads, C)
 
+    def prefill(self, layer: int, q: torch.Tensor, scale: float, out: torch.Tensor = None,
+                stream=None) -> torch.Tensor:
+        """Causal chunk attention of ``q`` ``[B, n_q, H_q, head_dim]``, the
+        queries of each sequence's last ``n_q`` positions (appended first),
+        over the compressed cache; returns float32 ``[B, n_q, H_q, head_dim]``."""
+        _need(q, "q")
+        d = self.desc
+        if q.dim() != 4 or (q.shape[0], q.shape[2], q.shape[3]) != (d.max_batch, d.n_q_heads, d.head_dim):
+            raise ValueError("q must be [max_batch, n_q, n_q_heads, head_dim]")
+        n_q = q.shape[1]
+        if out is None:
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        nbytes = ctypes.c_size_t()
+        check(self.lib.kvk_prefill_scratch_size(self.handle, layer, n_q, ctypes.byref(nbytes)))
+        scratch = torch.empty(nbytes.value, dtype=torch.uint8, device=self.device)
+        check(self.lib.kvk_prefill_attention(self.handle, layer, _ptr(q), _dtype_code(q), n_q,
+                                             float(scale), _ptr(out), _ptr(scratch), nbytes.value,
+                                             _stream(stream)))
+        self._prefill_scratch = scratch  # kept alive until the stream is done with it
+        return out
+
     def kept_lists(self, layer: int, stream=None):
         """Installed kept lists: ``(idx, n, per_head)`` device tensors shaped
         per head ``[B, H_kv, cap]`` / ``[B, H_kv]`` (or per sequence), or

@@ -26,6 +26,7 @@
 #include "kernels.h"
 #include "layout.h"
 #include "umma.cuh"
+#include "window_tc.cuh"
 
 namespace kvk {
 namespace {
@@ -427,23 +428,6 @@ constexpr int kTcWorkers = 512;              // dequantise and run the epilogues
 constexpr int kTcThreads = kTcWorkers + 32;  // + the MMA warp
 static_assert(kEvictStatSub == kTcWorkers / 128, "one statistics entry per worker column slice");
 
-// barrier 1 over the worker warps (the MMA warp runs on its own)
-__device__ __forceinline__ void workers_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
-__device__ __forceinline__ bool workers_sync_or(bool v) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 512, p;\n selp.u32 %0, 1, 0, q;\n}\n"
-      : "=r"(r)
-      : "r"(v ? 1u : 0u)
-      : "memory");
-  return r != 0;
-}
-
-// 16-byte chunks of a head_dim-128 K section per key format
-__host__ __device__ constexpr int TcFmtKs16(int fmt) {
-  return fmt == 0 ? 16 : (fmt == 1 || fmt == 3) ? 8 : (fmt == 2 || fmt == 4) ? 4 : 2;
-}
-
 struct TcPlan {
   int items_per_cta, n_items;
   int R16, nch, q_lo, k_lo, nst, nstg, fmt;  // nst key stages, nstg staging buffers
@@ -451,125 +435,6 @@ struct TcPlan {
   int nc_magic;                      // ceil(2^16 / kb_nch): e / kb_nch = (e nc_magic) >> 16 here
   int stage, off_q, off_ql, off_k, off_stg, off_norm, off_pv, off_bar, smem;
 };
-
-// key formats of the tensor-core dequantiser
-enum { kFmtBf16 = 0, kFmtG8, kFmtG4, kFmtS8, kFmtS4, kFmtS2 };
-
-template <int FMT>
-struct TcFmt {
-  static constexpr int BITS = FMT == kFmtBf16                   ? 16
-                              : (FMT == kFmtG8 || FMT == kFmtS8) ? 8
-                              : (FMT == kFmtG4 || FMT == kFmtS4) ? 4
-                                                                 : 2;
-  static constexpr bool SYM = FMT >= kFmtS8;
-  static constexpr int KS = 128 * BITS / 8;  // K-section bytes
-};
-
-// hi (and lo) bf16 words of 8 channels -> one swizzled 16-byte chunk of row
-// `row` holding channels ch0 .. ch0 + 7 (box stride `box` bytes)
-__device__ __forceinline__ void put_chunk(uint8_t *buf, int row, int ch0, int box, uint4 w) {
-  const int off = (ch0 >> 6) * box + row * 128 + ((((ch0 & 63) >> 3) ^ (row & 7)) << 4);
-  *reinterpret_cast<uint4 *>(buf + off) = w;
-}
-__device__ __forceinline__ void put8(uint8_t *hi, uint8_t *lo, bool with_lo, int row, int ch0,
-                                     int box, const float (&x)[8]) {
-  uint32_t h[4], l[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) split2<true>(x[2 * i], x[2 * i + 1], h[i], l[i]);
-  put_chunk(hi, row, ch0, box, make_uint4(h[0], h[1], h[2], h[3]));
-  if (with_lo) put_chunk(lo, row, ch0, box, make_uint4(l[0], l[1], l[2], l[3]));
-}
-// exact float of a small unsigned integer (< 2^23) on the FMA/ALU pipes
-__device__ __forceinline__ float u2f(uint32_t u) {
-  return __uint_as_float(0x4B000000u | u) - 8388608.f;
-}
-
-// Channels 32 qc .. 32 qc + 31 of one position's key, from its staged bundle
-// (K section in logical order, then the group metadata or the symmetric
-// scale word), dequantised into the key stage (hi, and lo unless bf16).
-// Every layout places quarter qc at a fixed offset from quarter 0 with the
-// same pattern (bf16: +64 bytes per quarter; 8-bit: +64 (qc >> 1) + 8 (qc &
-// 1) bytes; 4-bit: +4 qc bytes; 2-bit: +32 (qc >> 1) + 8 (qc & 1) bits), so
-// the quarter's words are loaded at a run-time offset and the channels are
-// picked out at the compile-time positions of quarter 0.
-template <int FMT>
-__device__ __forceinline__ void tc_dequant(const uint8_t *bundle, int row, int qc, int gshift,
-                                           uint8_t *kh, uint8_t *kl) {
-  using F = TcFmt<FMT>;
-  constexpr int D = 128, KBOX = 128 * 128;
-  const uint32_t *bw = reinterpret_cast<const uint32_t *>(bundle);
-  if constexpr (F::BITS == 16) {
-    static_assert(!F::SYM && F::KS == 256, "bf16 keys: 256 bytes, no scale");
-    // bf16 keys are exact: gather them into channel order, no lo part
-    uint32_t w[16];
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const uint4 u = reinterpret_cast<const uint4 *>(bundle)[4 * qc + c];
-      w[4 * c] = u.x; w[4 * c + 1] = u.y; w[4 * c + 2] = u.z; w[4 * c + 3] = u.w;
-    }
-#pragma unroll
-    for (int cc = 0; cc < 4; ++cc) {
-      uint32_t o[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        int b0, b1, h0, h1;
-        k_pos(8 * cc + 2 * i, 16, D, &b0, &h0);
-        k_pos(8 * cc + 2 * i + 1, 16, D, &b1, &h1);
-        const uint32_t sel = (uint32_t)((b0 & 3) | (((b0 & 3) + 1) << 4) | ((4 + (b1 & 3)) << 8) |
-                                        ((5 + (b1 & 3)) << 12));
-        o[i] = __byte_perm(w[b0 >> 2], w[b1 >> 2], sel);
-      }
-      put_chunk(kh, row, 32 * qc + 8 * cc, KBOX, make_uint4(o[0], o[1], o[2], o[3]));
-    }
-  } else {
-    constexpr int QL = (1 << (F::BITS - 1)) - 1;  // symmetric code offset
-    // the quarter's words; channel l of quarter 0 sits in word W(l) at bit S(l)
-    constexpr int NW = F::BITS == 8 ? 8 : 4;
-    uint32_t w[NW];
-    if constexpr (F::BITS == 8) {
-      const int ob = 16 * (qc >> 1) + 2 * (qc & 1);
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const uint2 u = *reinterpret_cast<const uint2 *>(bw + 4 * c + ob);
-        w[2 * c] = u.x; w[2 * c + 1] = u.y;
-      }
-    } else if constexpr (F::BITS == 4) {
-#pragma unroll
-      for (int c = 0; c < 4; ++c) w[c] = bw[4 * c + qc];
-    } else {
-#pragma unroll
-      for (int c = 0; c < 4; ++c) w[c] = bw[2 * c + (qc >> 1)] >> (8 * (qc & 1));
-    }
-    const float sym_s = F::SYM ? __uint_as_float(*reinterpret_cast<const uint32_t *>(bundle + F::KS) << 16)
-                               : 0.f;
-    // groups of 32 or 64 channels: the quarter lies in one group
-    float2 m = make_float2(0.f, 0.f);
-    if constexpr (!F::SYM) m = *reinterpret_cast<const float2 *>(bundle + F::KS + 8 * ((32 * qc) >> gshift));
-#pragma unroll
-    for (int cc = 0; cc < 4; ++cc) {
-      const int ch0 = 32 * qc + 8 * cc;
-      float x[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int l = 8 * cc + i;  // channel of quarter 0
-        int wi, sh;
-        if constexpr (F::BITS == 2) {
-          const int bit = sym_k_bit(l, 2, D);
-          wi = bit >> 6;
-          sh = bit & 63;
-        } else {
-          int byte, hi;
-          k_pos(l, F::BITS, D, &byte, &hi);
-          wi = F::BITS == 8 ? 2 * (byte >> 4) + ((byte & 15) >> 2) : byte >> 4;
-          sh = 8 * (byte & 3) + 4 * hi;
-        }
-        const uint32_t u = (w[wi] >> sh) & ((1u << F::BITS) - 1u);
-        x[i] = F::SYM ? sym_s * (u2f(u) - (float)QL) : fmaf(u2f(u), m.x, m.y);
-      }
-      put8(kh, kl, true, row, ch0, KBOX, x);
-    }
-  }
-}
 
 template <bool VOTES>
 __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs a, const TcPlan p) {
@@ -699,7 +564,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
       }
     }
     fence_proxy_async();
-    workers_sync();
+    workers_sync<kTcWorkers>();
   };
 
   // asynchronous copy of the K bundles of item `it` (K section in logical
@@ -737,12 +602,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
     const uint8_t *bundle = sm + p.off_stg + g * p.stg_bytes + pidx * p.kb_stride;
     uint8_t *kh = sm + p.off_k + s * p.stage, *kl = kh + 2 * KBOX;
     switch (p.fmt) {
-      case kFmtBf16: tc_dequant<kFmtBf16>(bundle, pidx, hf, gshift, kh, kl); break;
-      case kFmtG8: tc_dequant<kFmtG8>(bundle, pidx, hf, gshift, kh, kl); break;
-      case kFmtG4: tc_dequant<kFmtG4>(bundle, pidx, hf, gshift, kh, kl); break;
-      case kFmtS8: tc_dequant<kFmtS8>(bundle, pidx, hf, gshift, kh, kl); break;
-      case kFmtS4: tc_dequant<kFmtS4>(bundle, pidx, hf, gshift, kh, kl); break;
-      default: tc_dequant<kFmtS2>(bundle, pidx, hf, gshift, kh, kl); break;
+      case kFmtBf16: tc_dequant<kFmtBf16>(bundle, bundle + TcFmtKs16(kFmtBf16) * 16, pidx, hf, gshift, kh, kl); break;
+      case kFmtG8: tc_dequant<kFmtG8>(bundle, bundle + TcFmtKs16(kFmtG8) * 16, pidx, hf, gshift, kh, kl); break;
+      case kFmtG4: tc_dequant<kFmtG4>(bundle, bundle + TcFmtKs16(kFmtG4) * 16, pidx, hf, gshift, kh, kl); break;
+      case kFmtS8: tc_dequant<kFmtS8>(bundle, bundle + TcFmtKs16(kFmtS8) * 16, pidx, hf, gshift, kh, kl); break;
+      case kFmtS4: tc_dequant<kFmtS4>(bundle, bundle + TcFmtKs16(kFmtS4) * 16, pidx, hf, gshift, kh, kl); break;
+      default: tc_dequant<kFmtS2>(bundle, bundle + TcFmtKs16(kFmtS2) * 16, pidx, hf, gshift, kh, kl); break;
     }
   };
 
@@ -846,7 +711,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
       }
       const float vote = (vv[0] + vv[1]) + (vv[2] + vv[3]);
       if (slice) pv[(slice - 1) * 128 + pos] = vote;
-      workers_sync();
+      workers_sync<kTcWorkers>();
       if (!slice && t < P) a.votes[(size_t)unit * v.cap + t] = vote + pv[pos] + pv[128 + pos] + pv[256 + pos];
     }
   };
@@ -855,11 +720,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
   auto finish = [&](const Cursor &it, int tb) -> bool {
     const bool ok = mbar_wait_sleepy(&bar[tb], (phases >> tb) & 1u, kSleepyLimit, abort_flag, 2000);
     phases ^= 1u << tb;
-    if (workers_sync_or(!ok)) return false;
+    if (workers_sync_or<kTcWorkers>(!ok)) return false;
     tc_fence_after();
     epilogue(it, tb);
     tc_fence_before();
-    workers_sync();
+    workers_sync<kTcWorkers>();
     return true;
   };
 
@@ -915,13 +780,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) evict_tc_kernel(const EvictArgs
         cp_async_wait<1>();  // this item's bundles landed (the next item's may be in flight)
       else
         cp_async_wait<0>();
-      workers_sync();
+      workers_sync<kTcWorkers>();
       dequant(p.nstg == 2 ? (k & 1) : 0, k % p.nst);
       fence_proxy_async();  // the keys, written here, are read by the tensor cores
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar[3 + (k & 1)]);
       if (p.nstg == 1 && nxt.it < it1) {  // the staging is consumed once every worker is done
-        workers_sync();
+        workers_sync<kTcWorkers>();
         stage_copy(nxt, 0);
       }
       if (has_pend) {

@@ -88,6 +88,20 @@ struct EvictArgs {
   int32_t *err;
 };
 cudaError_t launch_gqa_evict(const EvictArgs &a, cudaStream_t st);
+
+// Causal chunk attention (prefill) over a GQA anchor, head_dim 128.
+struct PfArgs {
+  GqaView v;
+  const void *q;       // [B, n_q, Hq, D]
+  int q_f32;
+  int Hq, G, n_q;
+  float sig_log2;      // softmax scale * log2(e)
+  float2 *stats;       // [B * Hkv][n_q * G] (max, sum) per row
+  float *out;          // [B, n_q, Hq, D]
+  int32_t *err;
+};
+cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st);
+bool prefill_plan_fits(const PfArgs &a);
 constexpr int kEvictTile = 128;
 constexpr int kEvictStatSub = 4;  // statistics entries per tile and row, at most
 // Whether the evictor scores on the tensor cores (head_dim 128, at most 256

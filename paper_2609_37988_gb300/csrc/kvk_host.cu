@@ -635,6 +635,64 @@ kvk_status kvk_evict_window(kvk_cache *c, int32_t layer, const void *q_win, int3
   return KVK_OK;
 }
 
+namespace {
+kvk_status check_prefill(const kvk_cache *c, int32_t layer, int32_t n_q) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->desc.kind != KVK_KIND_GQA) return fail(KVK_ERR_UNSUPPORTED, "pre-fill on an MLA cache");
+  if (c->desc.head_dim != 128) return fail(KVK_ERR_UNSUPPORTED, "pre-fill needs head_dim 128");
+  const kvk_layer_cfg &L = c->cfg[c->src[layer]];
+  if (L.bits != 16 && L.key_axis == KVK_AXIS_CHANNEL && L.scheme != KVK_QUANT_SYMMETRIC)
+    return fail(KVK_ERR_UNSUPPORTED, "pre-fill over per-channel key groups");
+  if (n_q < 1 || n_q > c->desc.max_ctx)
+    return fail(KVK_ERR_INVALID_ARG, "n_q %d outside [1, max_ctx]", n_q);
+  return KVK_OK;
+}
+size_t prefill_scratch(const kvk_cache *c, int32_t n_q) {
+  const size_t rows = (size_t)c->desc.max_batch * c->desc.n_q_heads * n_q;  // units x n_q G
+  return (size_t)align256((int64_t)(rows * 8));
+}
+}  // namespace
+
+kvk_status kvk_prefill_scratch_size(const kvk_cache *c, int32_t layer, int32_t n_q, size_t *bytes) {
+  kvk_status s = check_prefill(c, layer, n_q);
+  if (s) return s;
+  if (!bytes) return fail(KVK_ERR_INVALID_ARG, "null output");
+  *bytes = prefill_scratch(c, n_q);
+  return KVK_OK;
+}
+
+kvk_status kvk_prefill_attention(kvk_cache *c, int32_t layer, const void *q, int32_t q_dtype, int32_t n_q,
+                                 float softmax_scale, float *out, void *scratch, size_t scratch_bytes,
+                                 kvk_stream stream) {
+  kvk_status s = check_prefill(c, layer, n_q);
+  if (s) return s;
+  if (!q || !aligned16(q)) return fail(KVK_ERR_INVALID_ARG, "null or misaligned q");
+  if (!out || !aligned16(out)) return fail(KVK_ERR_INVALID_ARG, "null or misaligned out");
+  if (q_dtype != KVK_DTYPE_F32 && q_dtype != KVK_DTYPE_BF16)
+    return fail(KVK_ERR_INVALID_ARG, "q_dtype must be F32 or BF16");
+  if (!std::isfinite(softmax_scale) || !(softmax_scale > 0.f))
+    return fail(KVK_ERR_INVALID_ARG, "softmax scale must be finite and positive");
+  const size_t need = prefill_scratch(c, n_q);
+  if (!scratch || (reinterpret_cast<uintptr_t>(scratch) & 255u) || scratch_bytes < need)
+    return fail(KVK_ERR_INVALID_ARG, "scratch null, not 256-byte aligned or smaller than %zu bytes", need);
+  PfArgs a;
+  a.v = c->gqa_view(c->src[layer]);
+  a.q = q;
+  a.q_f32 = q_dtype == KVK_DTYPE_F32;
+  a.Hq = c->desc.n_q_heads;
+  a.G = c->desc.n_q_heads / c->desc.n_kv_heads;
+  a.n_q = n_q;
+  a.sig_log2 = softmax_scale * 1.4426950408889634f;
+  a.stats = static_cast<float2 *>(scratch);
+  a.out = out;
+  a.err = c->err();
+  if (!prefill_plan_fits(a)) return fail(KVK_ERR_UNSUPPORTED, "pre-fill plan does not fit shared memory");
+  cudaError_t e = launch_gqa_prefill(a, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "pre-fill launch");
+  return KVK_OK;
+}
+
 kvk_status kvk_export_kept(const kvk_cache *c, int32_t layer, int32_t *idx, int32_t *n_kept,
                            int32_t *per_head, kvk_stream stream) {
   kvk_status s = check_layer_index(c, layer);
