@@ -374,9 +374,13 @@ def main():
                     help="store the quantised anchors with the symmetric per-vector "
                          "quantiser at this bit-width")
     ap.add_argument("--profile-case",
-                    choices=["gqa", "kpc", "mla", "mla64", "gather", "sym", "evict", "evict-small"],
+                    choices=["gqa", "kpc", "mla", "mla64", "gather", "sym", "evict", "evict-small",
+                             "prefill", "prefill-small"],
                     default=None,
                     help="small ncu case: decode (or eviction) launches only, no timing line")
+    ap.add_argument("--prefill", action="store_true",
+                    help="time causal chunk attention (pre-fill) over one compressed 14B anchor "
+                         "instead of the decode step (one JSON line of its own)")
     ap.add_argument("--evict", action="store_true",
                     help="time the window-vote evictor at the long-context 14B shape instead "
                          "of the decode step (one JSON line of its own)")
@@ -389,6 +393,9 @@ def main():
         return
     if args.evict:
         evict_bench(args)
+        return
+    if args.prefill:
+        prefill_bench(args)
         return
 
     import torch
@@ -757,6 +764,87 @@ def evict_bench(args):
     print(json.dumps(line))
 
 
+PREFILL_CHUNK = 2048
+
+
+def prefill_flops(lens, n_q, Hq, D):
+    """Algorithmic FLOPs of one pre-fill call: every query scores and weights
+    its causal range once (2 D for the score, 2 D for the value product)."""
+    total = 0
+    for L in lens:
+        for i in range(n_q):
+            p = L - n_q + i
+            if p >= 0:
+                total += (p + 1) * Hq * 4 * D
+    return total
+
+
+def _prefill_setup(B, T, n_q, dev, bits=4):
+    import torch
+    from paper_2609_37988_gb300 import workloads as W
+    from paper_2609_37988_gb300.cache import Cache, Layer
+    w = W.config(3, n_layers=1, batch=B, context=T)
+    layer = Layer(bits=bits, group=32) if bits != 16 else Layer(bits=16)
+    c = Cache(n_layers=1, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads, head_dim=w.head_dim,
+              max_batch=B, max_ctx=T, layers=[layer], device=dev)
+    for b0 in range(0, T, 4096):
+        k, v = W.kv_inputs(w, 0, b0, min(T, b0 + 4096), device=dev)
+        c.append(0, k.contiguous(), v.contiguous())
+        del k, v
+    q = W.randn((B, n_q, w.n_q_heads, w.head_dim), w.seed, 0, 11, dtype=torch.bfloat16, device=dev)
+    torch.cuda.synchronize()
+    return w, c, q
+
+
+def prefill_bench(args):
+    """Pre-fill over one compressed anchor at the 14B shape: int4 g32, B=4
+    sequences of 8192 positions, the last 2048 of which are the chunk (the
+    last chunk of a chunked pre-fill: 6144 cached positions before it);
+    40 q / 8 KV heads, head_dim 128, bf16 queries.  CUDA events on the
+    launching stream, inputs (0.8 GB of cache) larger than L2."""
+    import torch
+    from __graft_entry__ import build
+    build()
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    B, T = 4, 8192
+    w, c, q = _prefill_setup(B, T, PREFILL_CHUNK, dev)
+    out = torch.empty(q.shape, dtype=torch.float32, device=dev)
+    for _ in range(max(3, args.warmup)):
+        c.prefill(0, q, w.sigma, out=out)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    with Clocks(0) as clk:
+        torch.cuda.synchronize()
+        for s0, e0 in ev:
+            s0.record(stream)
+            c.prefill(0, q, w.sigma, out=out)
+            e0.record(stream)
+        torch.cuda.synchronize()
+    ms = [s0.elapsed_time(e0) for s0, e0 in ev]
+    assert c.device_error() == 0
+    flops = prefill_flops([T] * B, PREFILL_CHUNK, w.n_q_heads, w.head_dim)
+    mean_ms = statistics.mean(ms)
+    achieved = flops / (mean_ms * 1e-3) / 1e12
+    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+        peak = float(json.load(f)["bf16_tflops"])
+    line = {"metric": "pre-fill over a compressed anchor: ms per call, TFLOP/s of the attention",
+            "value": round(mean_ms, 4), "unit": "ms", "higher_is_better": False,
+            "steps": args.steps, "warmup": max(3, args.warmup), "n_gpus": 1,
+            "dtype": "bf16x2 (hi/lo) in, f32 accumulate", "data": "synthetic",
+            "config": {"workload": f"qwen2.5-14b-b{B}-t{T} int4g32 anchor, chunk {PREFILL_CHUNK}",
+                       "l2": "inputs larger than L2"},
+            "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": round(peak, 1),
+                         "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
+                         "peak_source": "measured bf16 dense (burst)",
+                         "work": f"scores and value products counted once ({flops / 1e9:.1f} GFLOP)"},
+            "ms_min": round(min(ms), 4), "ms_max": round(max(ms), 4),
+            "gpu_launches": 2 * args.steps, "clocks": clk.summary()}
+    print(json.dumps(line))
+
+
 def profile_case(kind):
     """The kernel-level ncu case.  gqa: one int4 g32 and one bf16 anchor at
     the 14B step shape (B=32, 8 kv / 40 q heads, d_h 128, T=8192; 1.5 GB of
@@ -826,6 +914,13 @@ def profile_case(kind):
         w, c, q = _evict_setup(B, T, torch.device("cuda", 0))
         for _ in range(3):
             c.evict_window(0, q, w.sigma, w.keep)
+    elif kind in ("prefill", "prefill-small"):
+        # pre-fill at the 14B shape (B=4, T=8192, chunk 2048), or one sequence
+        # of 4096 positions with a 1024-query chunk for multi-pass captures
+        B, T, n = (4, 8192, PREFILL_CHUNK) if kind == "prefill" else (1, 4096, 1024)
+        w, c, q = _prefill_setup(B, T, n, torch.device("cuda", 0))
+        for _ in range(3):
+            c.prefill(0, q, w.sigma)
     elif kind == "gather":
         import numpy as np
         w = W.config(5, n_layers=1)

@@ -98,6 +98,7 @@ struct PfArgs {
   float sig_log2;      // softmax scale * log2(e)
   float2 *stats;       // [B * Hkv][n_q * G] (max, sum) per row
   float *out;          // [B, n_q, Hq, D]
+  int *counter;        // two job counters (statistics, output), zeroed by the launch
   int32_t *err;
 };
 cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st);

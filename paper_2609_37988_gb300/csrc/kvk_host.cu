@@ -650,7 +650,7 @@ kvk_status check_prefill(const kvk_cache *c, int32_t layer, int32_t n_q) {
 }
 size_t prefill_scratch(const kvk_cache *c, int32_t n_q) {
   const size_t rows = (size_t)c->desc.max_batch * c->desc.n_q_heads * n_q;  // units x n_q G
-  return (size_t)align256((int64_t)(rows * 8));
+  return (size_t)align256((int64_t)(rows * 8)) + 256;  // + the job counters
 }
 }  // namespace
 
@@ -685,6 +685,7 @@ kvk_status kvk_prefill_attention(kvk_cache *c, int32_t layer, const void *q, int
   a.n_q = n_q;
   a.sig_log2 = softmax_scale * 1.4426950408889634f;
   a.stats = static_cast<float2 *>(scratch);
+  a.counter = reinterpret_cast<int *>(static_cast<uint8_t *>(scratch) + need - 256);
   a.out = out;
   a.err = c->err();
   if (!prefill_plan_fits(a)) return fail(KVK_ERR_UNSUPPORTED, "pre-fill plan does not fit shared memory");

@@ -42,7 +42,7 @@ constexpr int kPfRows = 128;  // rows per job
 constexpr int kQBox = kPfRows * 128;  // one 64-channel box of the job's query rows
 
 struct PfPlan {
-  int n_rb, n_jobs, jobs_per_cta;
+  int n_rb, n_jobs, grid;
   int q_lo, k_lo, fmt, gshift;
   int ks16, nrec, ncopy;  // K-section chunks, record chunks, chunks staged per position
   uint32_t nc_magic;      // ceil(2^32 / ncopy): e / ncopy = umulhi(e, nc_magic)
@@ -70,6 +70,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + p.off_bar);
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + 56);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + 60);
+  volatile int *s_job = reinterpret_cast<volatile int *>(sm + p.off_bar + 64);
   float *norm = reinterpret_cast<float *>(sm + p.off_norm);  // [128] log-normaliser per job row
   float2 *red = reinterpret_cast<float2 *>(sm + p.off_red);  // [4][128] slice statistics
   uint8_t *qh = sm, *ql = sm + p.off_ql;
@@ -102,16 +103,28 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   // at 64 (k & 1), O^T at 128
   const uint32_t t_o = tmem + 128;
 
-  const int j0 = blockIdx.x * p.jobs_per_cta;
-  const int j1 = min(j0 + p.jobs_per_cta, p.n_jobs);
+  // Jobs are handed out one at a time from a counter (the longest row
+  // blocks first), so CTAs finish together although jobs differ in length.
+  // Every thread of the CTA takes part in each hand-out; a CTA that gave up
+  // keeps taking jobs (and skips them) until none is left, so no barrier
+  // waits for threads that left.
+  const int units = v.B * v.Hkv;
+  int *counter = a.counter + (OUT ? 1 : 0);
+  auto next_job = [&]() -> int {
+    asm volatile("bar.sync 2, %0;" ::"n"(kPfThreads) : "memory");  // the previous id is read
+    if (tid == 0) *s_job = atomicAdd(counter, 1);
+    asm volatile("bar.sync 2, %0;" ::"n"(kPfThreads) : "memory");
+    return *s_job;
+  };
 
   struct Job {
     int unit, b, j, r0, nr, len, n_t;
   };
   auto job_at = [&](int job) {
     Job J;
-    J.unit = job / p.n_rb;
-    const int rb = job - J.unit * p.n_rb;
+    const int step = job / units;
+    J.unit = job - step * units;
+    const int rb = p.n_rb - 1 - step;
     J.b = J.unit / v.Hkv;
     J.j = J.unit - J.b * v.Hkv;
     J.r0 = rb * kPfRows;
@@ -159,7 +172,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     };
     int kk = 0;
     bool ok = true;
-    for (int job = j0; job < j1 && ok; ++job) {
+    for (int job = next_job(); job < p.n_jobs; job = next_job()) {
+      if (!ok) continue;
       const Job J = job_at(job);
       for (int k = 0; k < J.n_t && ok; ++k, ++kk) {
         // with one stage the previous tile's values are read before the
@@ -178,6 +192,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         }
         __syncwarp();
       }
+      if (!ok && lane == 0) *abort_flag = 1;
       if constexpr (OUT) {
         if (ok && J.n_t > 0) {
           ok = mbar_wait_sleepy(&bar[4], (kk - 1) & 1, kLimit, abort_flag, 2000);
@@ -271,15 +286,17 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         } else {
           so = cl;
         }
-        cp_async16(dst0 + pos * p.b_stride + 16 * cl, base + (size_t)(ok ? t : t0) * v.rec_bytes + 16 * so,
-                   ok);
+        // output pass: the whole logical record; statistics: K section and
+        // key metadata back to back
+        cp_async16(dst0 + pos * p.b_stride + 16 * (OUT ? cl : c),
+                   base + (size_t)(ok ? t : t0) * v.rec_bytes + 16 * so, ok);
       }
       if (sym)
         for (int pos = tid; pos < TT; pos += kPfWorkers) {
           const int t = t0 + pos;
           const bool ok = t < J.len;
-          cp_async4(dst0 + pos * p.b_stride + v.rec_bytes, v.scales + (size_t)J.unit * v.cap + (ok ? t : t0),
-                    ok);
+          cp_async4(dst0 + pos * p.b_stride + (OUT ? v.rec_bytes : 16 * p.ks16),
+                    v.scales + (size_t)J.unit * v.cap + (ok ? t : t0), ok);
         }
       cp_async_commit();
     };
@@ -294,7 +311,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       const int mb = (p.nrec * 16 - 2 * ks) / 2;  // grouped: bytes of one metadata block
       const bool sym = p.fmt >= kFmtS8;
       if (part < 4) {
-        const uint8_t *kmeta = sym ? bundle + v.rec_bytes : bundle + 2 * ks;
+        const uint8_t *kmeta = !OUT ? bundle + ks : sym ? bundle + v.rec_bytes : bundle + 2 * ks;
         switch (p.fmt) {
           case kFmtBf16: tc_dequant<kFmtBf16, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
           case kFmtG8: tc_dequant<kFmtG8, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
@@ -322,7 +339,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     };
 
     int kk = 0;
-    for (int job = j0; job < j1 && !failed; ++job) {
+    for (int job = next_job(); job < p.n_jobs; job = next_job()) {
+      if (failed) continue;
       const Job J = job_at(job);
       const int base = J.len - a.n_q;  // position of chunk query 0
       load_q(J);
@@ -332,31 +350,43 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       const int last = base + (J.r0 + rl) / a.G;  // the last position the row sees
       const bool warp_live = 32 * quarter < J.nr;
       float m_run = -INFINITY, l_run = 0.f;  // statistics: this slice's running pair
-      if (J.n_t > 0) stage_copy(J, 0, kk & (p.nstg - 1));
-      for (int k = 0; k < J.n_t && !failed; ++k, ++kk) {
+      const bool pipe = p.nst == 2;
+      // Stage tile kn (tile counter kkn): its records have landed; the values
+      // the stage held are read (the value product of tile kkn - nst);
+      // dequantised and announced to the MMA warp.  With two stages the next
+      // tile is staged before this tile's scores are awaited, so that the
+      // dequantisation overlaps the score product.
+      auto stage_tile = [&](int kn, int kkn) -> bool {
         if (p.nstg == 2) {
-          if (k + 1 < J.n_t)
-            stage_copy(J, k + 1, (kk + 1) & 1);  // the staging of tile kk - 1, consumed
+          if (kn + 1 < J.n_t)
+            stage_copy(J, kn + 1, (kkn + 1) & 1);  // the staging of tile kkn - 1, consumed
           else
-            cp_async_commit();
-        }
-        if (OUT && p.nst == 1 && k > 0 && !wait_pv(kk - 1)) failed = true;  // the one stage is free
-        if (p.nstg == 2)
+            cp_async_commit();  // keeps the wait count uniform
           cp_async_wait<1>();
-        else
+        } else {
           cp_async_wait<0>();
-        if (workers_sync_or<kPfWorkers>(failed)) { failed = true; break; }
-        if (OUT || part < 4) dequant(kk & (p.nstg - 1), kk % p.nst);
+        }
+        const bool ok = OUT ? wait_pv(kkn - p.nst) : true;
+        if (workers_sync_or<kPfWorkers>(!ok)) return false;
+        if (OUT || part < 4) dequant(kkn & (p.nstg - 1), kkn % p.nst);
         fence_proxy_async();  // the stage, written here, is read by the tensor cores
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bar[kk & 1]);
-        if (p.nstg == 1 && k + 1 < J.n_t) {
-          workers_sync<kPfWorkers>();
-          stage_copy(J, k + 1, 0);
+        if (lane == 0) mbar_arrive(&bar[kkn & 1]);
+        if (p.nstg == 1 && kn + 1 < J.n_t) {
+          workers_sync<kPfWorkers>();  // the one staging buffer is consumed
+          stage_copy(J, kn + 1, 0);
         }
-        // scores of this tile
+        return true;
+      };
+      if (J.n_t > 0) {
+        stage_copy(J, 0, kk & (p.nstg - 1));
+        if (!stage_tile(0, kk)) failed = true;
+      }
+      for (int k = 0; k < J.n_t && !failed; ++k, ++kk) {
+        if (pipe && k + 1 < J.n_t && !stage_tile(k + 1, kk + 1)) { failed = true; break; }
+        // scores of this tile; output pass: the P buffer is free
         bool ok = mbar_wait_sleepy(&bar[2 + (kk & 1)], (kk >> 1) & 1, kLimit, abort_flag, 2000);
-        if (OUT && ok && k > 0) ok = wait_pv(kk - 1);  // the P buffer is free
+        if (OUT && ok) ok = wait_pv(kk - 1);
         if (workers_sync_or<kPfWorkers>(!ok)) { failed = true; break; }
         tc_fence_after();
         const int t0 = k * TT;
@@ -408,9 +438,14 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         tc_fence_before();
         __syncwarp();
         if (OUT && lane == 0) mbar_arrive(&bar[4]);
-        if (!OUT) workers_sync<kPfWorkers>();  // the score buffer is free for tile kk + 2
+        // one stage: the next tile after this one's epilogue (and, in the
+        // output pass, its value product)
+        if (!pipe && k + 1 < J.n_t && !stage_tile(k + 1, kk + 1)) { failed = true; break; }
       }
-      if (failed) break;
+      if (failed) {
+        *abort_flag = 1;
+        continue;
+      }
       if constexpr (!OUT) {
         // the four slices' pairs of each row, combined
         red[slice * kPfRows + rl] = make_float2(m_run, l_run);
@@ -434,7 +469,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         float o[32];
         if (J.n_t > 0) {
           if (!wait_pv(kk - 1)) failed = true;
-          if (workers_sync_or<kPfWorkers>(failed)) { failed = true; break; }
+          if (workers_sync_or<kPfWorkers>(failed)) { failed = true; *abort_flag = 1; continue; }
           tc_fence_after();
           float z[16];
           tmem_ld16(t_o + 32 * slice + lane_off, z);
@@ -497,7 +532,7 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   const int kmeta16 = (p.fmt == kFmtBf16 || sym) ? 0 : (p.nrec - 2 * p.ks16) / 2;
   p.ncopy = out ? p.nrec : p.ks16 + kmeta16;
   p.nc_magic = (uint32_t)((0x100000000ull + p.ncopy - 1) / p.ncopy);
-  const int bchunks = p.nrec + (sym ? 1 : 0);
+  const int bchunks = (out ? p.nrec : p.ncopy) + (sym ? 1 : 0);
   p.b_stride = 16 * (bchunks % 2 ? bchunks : bchunks + 1);
   p.stg_bytes = TT * p.b_stride;
   const int kbox = TT * 128;
@@ -506,7 +541,7 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   const int qbytes = kPfRows * 256 * (p.q_lo ? 2 : 1);
   p.off_k = (qbytes + 1023) / 1024 * 1024;
   const int pbytes = out ? 2 * kPfRows * 128 : 0;
-  const int tail = pbytes + kPfRows * 4 + 4 * kPfRows * 8 + 64 + 1024;
+  const int tail = pbytes + kPfRows * 4 + 4 * kPfRows * 8 + 128 + 1024;
   auto fits = [&](int nst, int nstg) { return p.off_k + nst * p.stage + nstg * p.stg_bytes + tail <= 232448; };
   p.nst = fits(2, 1) ? 2 : 1;
   p.nstg = fits(p.nst, 2) ? 2 : 1;
@@ -515,9 +550,8 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   p.off_norm = p.off_p + pbytes;
   p.off_red = p.off_norm + kPfRows * 4;
   p.off_bar = p.off_red + 4 * kPfRows * 8;
-  p.smem = p.off_bar + 64 + 1024;
-  const int grid = std::max(1, std::min(p.n_jobs, sms));
-  p.jobs_per_cta = (p.n_jobs + grid - 1) / grid;
+  p.smem = p.off_bar + 128 + 1024;
+  p.grid = std::max(1, std::min(p.n_jobs, sms));
   return p;
 }
 
@@ -542,11 +576,11 @@ cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st) {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, po.smem);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(prefill_kernel<false>, dim3((ps.n_jobs + ps.jobs_per_cta - 1) / ps.jobs_per_cta),
-                 dim3(kPfThreads), ps.smem, st, a, ps);
+  e = cudaMemsetAsync(a.counter, 0, 2 * sizeof(int), st);  // the job counters
   if (e == cudaSuccess)
-    e = launch_pdl(prefill_kernel<true>, dim3((po.n_jobs + po.jobs_per_cta - 1) / po.jobs_per_cta),
-                   dim3(kPfThreads), po.smem, st, a, po);
+    e = launch_pdl(prefill_kernel<false>, dim3(ps.grid), dim3(kPfThreads), ps.smem, st, a, ps);
+  if (e == cudaSuccess)
+    e = launch_pdl(prefill_kernel<true>, dim3(po.grid), dim3(kPfThreads), po.smem, st, a, po);
   return e;
 }
 
