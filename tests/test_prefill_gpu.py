@@ -119,3 +119,28 @@ def test_prefill_rejections():
               max_batch=1, max_ctx=64, layers=[Layer(bits=16, width=512)])
     with pytest.raises((KVKError, ValueError)):
         m.prefill(0, torch.zeros((1, 4, 16, 128), dtype=torch.bfloat16, device="cuda"), 0.1)
+
+
+@pytest.mark.slow
+def test_prefill_full_size_sampled():
+    """The bench's pre-fill call (14B shape: int4 g32 anchor, B=4 x 8192
+    positions, 40 q / 8 KV heads, a 2048-query chunk) with the bench's
+    inputs; sampled queries of the first and last sequence against the
+    oracle (each one a decode over its causal prefix)."""
+    import bench
+    from paper_2609_37988_gb300 import workloads as W
+    B, T, n_q = 4, 8192, bench.PREFILL_CHUNK
+    w, c, q = bench._prefill_setup(B, T, n_q, torch.device("cuda", 0))
+    out = f32(c.prefill(0, q, w.sigma))
+    assert c.device_error() == 0
+    fmt = dict(bits=4, group=32, key_axis="token")
+    for b in (0, B - 1):
+        k = torch.cat([W.kv_inputs(w, 0, t0, min(T, t0 + 4096), device="cuda")[0][b:b + 1].cpu()
+                       for t0 in range(0, T, 4096)], 1)
+        v = torch.cat([W.kv_inputs(w, 0, t0, min(T, t0 + 4096), device="cuda")[1][b:b + 1].cpu()
+                       for t0 in range(0, T, 4096)], 1)
+        st = oracle_state(f32(k), f32(v), np.array([T]), fmt)
+        for i in (0, 1, 777, n_q - 2, n_q - 1):
+            p = T - n_q + i
+            ref = oatt.gqa_decode(f32(q[b:b + 1, i]), st["k_hat"], st["v_hat"], [p + 1], w.sigma)
+            assert_close(out[b:b + 1, i], ref, what=f"sequence {b} query {i}")
