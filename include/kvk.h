@@ -238,7 +238,9 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
  *  q:       device [B, n_q, H_q, head_dim] in q_dtype (post-RoPE);
  *  out:     device float32 [B, n_q, H_q, head_dim];
  *  scratch: device, 256-byte aligned, at least kvk_prefill_scratch_size
- *           bytes (per-row softmax statistics).
+ *           bytes: per-row softmax statistics and the anchor's cache
+ *           dequantised once into the products' operand layout (1 KB per
+ *           position and KV head for quantised anchors, 512 B for bf16).
  * Errors: UNSUPPORTED (MLA, head_dim != 128, grouped per-channel keys),
  * INVALID_ARG (n_q outside [1, max_ctx], null or misaligned pointers,
  * scale not finite and positive, scratch too small). */

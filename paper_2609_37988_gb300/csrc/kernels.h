@@ -99,10 +99,12 @@ struct PfArgs {
   float2 *stats;       // [B * Hkv][n_q * G] (max, sum) per row
   float *out;          // [B, n_q, Hq, D]
   int *counter;        // two job counters (statistics, output), zeroed by the launch
+  uint8_t *tiles;      // [B * Hkv][cap / 64] expanded tiles of prefill_tile_bytes(bits)
   int32_t *err;
 };
 cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st);
 bool prefill_plan_fits(const PfArgs &a);
+size_t prefill_tile_bytes(int bits);
 constexpr int kEvictTile = 128;
 constexpr int kEvictStatSub = 4;  // statistics entries per tile and row, at most
 // Whether the evictor scores on the tensor cores (head_dim 128, at most 256

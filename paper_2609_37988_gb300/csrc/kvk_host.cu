@@ -648,9 +648,21 @@ kvk_status check_prefill(const kvk_cache *c, int32_t layer, int32_t n_q) {
     return fail(KVK_ERR_INVALID_ARG, "n_q %d outside [1, max_ctx]", n_q);
   return KVK_OK;
 }
-size_t prefill_scratch(const kvk_cache *c, int32_t n_q) {
+// Pre-fill scratch: the rows' statistics, the two job counters, then the
+// expanded tiles (every 64-position tile of every unit, dequantised once).
+struct PrefillScratch {
+  size_t stats, counters, tiles, total;
+};
+PrefillScratch prefill_scratch(const kvk_cache *c, int32_t layer, int32_t n_q) {
+  PrefillScratch p;
+  const int a = c->src[layer];
   const size_t rows = (size_t)c->desc.max_batch * c->desc.n_q_heads * n_q;  // units x n_q G
-  return (size_t)align256((int64_t)(rows * 8)) + 256;  // + the job counters
+  p.stats = 0;
+  p.counters = (size_t)align256((int64_t)(rows * 8));
+  p.tiles = (size_t)((p.counters + 256 + 1023) & ~(size_t)1023);
+  const size_t units = (size_t)c->desc.max_batch * c->desc.n_kv_heads;
+  p.total = p.tiles + units * (size_t)(c->lay[a].cap / 64) * prefill_tile_bytes(c->cfg[a].bits);
+  return p;
 }
 }  // namespace
 
@@ -658,7 +670,7 @@ kvk_status kvk_prefill_scratch_size(const kvk_cache *c, int32_t layer, int32_t n
   kvk_status s = check_prefill(c, layer, n_q);
   if (s) return s;
   if (!bytes) return fail(KVK_ERR_INVALID_ARG, "null output");
-  *bytes = prefill_scratch(c, n_q);
+  *bytes = prefill_scratch(c, layer, n_q).total;
   return KVK_OK;
 }
 
@@ -673,9 +685,10 @@ kvk_status kvk_prefill_attention(kvk_cache *c, int32_t layer, const void *q, int
     return fail(KVK_ERR_INVALID_ARG, "q_dtype must be F32 or BF16");
   if (!std::isfinite(softmax_scale) || !(softmax_scale > 0.f))
     return fail(KVK_ERR_INVALID_ARG, "softmax scale must be finite and positive");
-  const size_t need = prefill_scratch(c, n_q);
-  if (!scratch || (reinterpret_cast<uintptr_t>(scratch) & 255u) || scratch_bytes < need)
-    return fail(KVK_ERR_INVALID_ARG, "scratch null, not 256-byte aligned or smaller than %zu bytes", need);
+  const PrefillScratch ps = prefill_scratch(c, layer, n_q);
+  if (!scratch || (reinterpret_cast<uintptr_t>(scratch) & 255u) || scratch_bytes < ps.total)
+    return fail(KVK_ERR_INVALID_ARG, "scratch null, not 256-byte aligned or smaller than %zu bytes",
+                ps.total);
   PfArgs a;
   a.v = c->gqa_view(c->src[layer]);
   a.q = q;
@@ -685,7 +698,8 @@ kvk_status kvk_prefill_attention(kvk_cache *c, int32_t layer, const void *q, int
   a.n_q = n_q;
   a.sig_log2 = softmax_scale * 1.4426950408889634f;
   a.stats = static_cast<float2 *>(scratch);
-  a.counter = reinterpret_cast<int *>(static_cast<uint8_t *>(scratch) + need - 256);
+  a.counter = reinterpret_cast<int *>(static_cast<uint8_t *>(scratch) + ps.counters);
+  a.tiles = static_cast<uint8_t *>(scratch) + ps.tiles;
   a.out = out;
   a.err = c->err();
   if (!prefill_plan_fits(a)) return fail(KVK_ERR_UNSUPPORTED, "pre-fill plan does not fit shared memory");

@@ -8,21 +8,24 @@
 // Rows: row r = i G + h of a (sequence, KV head) unit is chunk query i and
 // head h of the KV head's group; query i sits at position len - n_q + i and
 // sees positions 0 .. len - n_q + i.  A job is 128 consecutive rows of one
-// unit.  Two kernels over jobs, one persistent CTA per SM (16 worker warps,
-// one MMA warp):
+// unit.  Three launches:
+//  * expand: every 64-position tile of the cache is dequantised once into
+//    the layout the products read (bf16 hi and lo halves, K-major
+//    128-byte-swizzled boxes), in caller scratch;
 //  * statistics: per row, the maximum M and the sum L of 2^(x - M) of its
 //    scaled scores x = sigma log2(e) <q, k> over its causal range, online
-//    over 128-position tiles (S = Q K^T with TMEM lane = row, so a thread
-//    updates its row's running pair);
-//  * output: per 64-position tile, S = Q K^T, P = 2^(x - M - log2 L) (zero
-//    past the row's limit) into shared memory, O^T += V^T P^T; after the last
-//    tile O^T (TMEM lane = channel) is written out.  The normalisers being
-//    final, the output pass never rescales O.
-// Keys and values are dequantised into bf16 hi + lo halves in the K-major
-// 128-byte-swizzled layout (rows = positions); the value MMA reads the value
-// tile as an MN-major operand of that same layout.  Products are
-// hi*hi + hi*lo + lo*hi (no lo part for bf16 caches or bf16 queries), fp32
-// accumulation in TMEM.
+//    over the tiles (S = Q K^T with TMEM lane = row);
+//  * outputs: per tile, S = Q K^T, P = 2^(x - M - log2 L) (zero past the
+//    row's limit) into shared memory, O^T += V^T P^T (the value tile read as
+//    an MN-major operand); after the job's last tile O^T (TMEM lane =
+//    channel) is written out.  The normalisers being final, O is never
+//    rescaled.
+// The two attention kernels run one persistent CTA per SM with three roles:
+// a copy warp brings each job's tiles in with bulk copies, an MMA warp
+// issues the tcgen05 products, 16 worker warps run the epilogues.  Products
+// are hi*hi + hi*lo + lo*hi (no lo part for bf16 caches or bf16 queries),
+// fp32 accumulation in TMEM.  Jobs are handed out from a counter, the
+// longest row blocks first.
 #include <math.h>
 
 #include <algorithm>
@@ -37,40 +40,126 @@ namespace kvk {
 namespace {
 
 constexpr int kPfWorkers = 512;
-constexpr int kPfThreads = kPfWorkers + 32;
-constexpr int kPfRows = 128;  // rows per job
-constexpr int kQBox = kPfRows * 128;  // one 64-channel box of the job's query rows
+constexpr int kPfThreads = kPfWorkers + 64;  // + the MMA warp and the copy warp
+constexpr int kPfRows = 128;                 // rows per job
+constexpr int kQBox = kPfRows * 128;         // one 64-channel box of the job's query rows
+constexpr int kPfT = 64;                     // positions per tile
+constexpr int kPfBox = kPfT * 128;           // one 64-channel box of a tile (8 KB)
 
 struct PfPlan {
-  int n_rb, n_jobs, grid;
+  int n_rb, n_jobs, grid, n_t64;
   int q_lo, k_lo, fmt, gshift;
-  int ks16, nrec, ncopy;  // K-section chunks, record chunks, chunks staged per position
-  uint32_t nc_magic;      // ceil(2^32 / ncopy): e / ncopy = umulhi(e, nc_magic)
-  int b_stride, stg_bytes, stage, nst, nstg;
-  int off_ql, off_k, off_stg, off_p, off_norm, off_red, off_bar, smem;
+  int ks16, nrec;
+  uint32_t nc_magic;  // expand: ceil(2^32 / nrec), e / nrec = umulhi(e, nc_magic)
+  int b_stride;       // expand: staged record stride (odd multiple of 16 bytes)
+  int kbytes, tbytes; // a tile's keys (hi, lo); the whole tile (keys, values)
+  int ns;             // key (and value) stages of the attention kernels
+  int off_ql, off_k, off_v, off_p, off_norm, off_red, off_bar, smem, smem_x;
 };
 
 // Tiles a job reads: positions up to that of the job's last row.
-__device__ __forceinline__ int pf_tiles(int len, int n_q, int G, int r_last, int tt) {
+__device__ __forceinline__ int pf_tiles(int len, int n_q, int G, int r_last) {
   const int p_max = len - n_q + r_last / G;
-  return p_max >= 0 ? p_max / tt + 1 : 0;
+  return p_max >= 0 ? p_max / kPfT + 1 : 0;
+}
+
+// Expand: the keys and values of one 64-position tile of one unit, staged
+// raw (rotations undone), dequantised per (position, channel quarter) into
+// [K hi | K lo | V hi | V lo] (8 KB boxes; no lo halves for bf16 caches)
+// and stored for every job of the unit to copy.  Positions past the length
+// are zero.
+__global__ void __launch_bounds__(kPfWorkers) prefill_expand_kernel(const PfArgs a, const PfPlan p) {
+  extern __shared__ uint8_t pf_raw[];
+  uint8_t *sm = pf_raw + ((1024u - (smem_u32(pf_raw) & 1023u)) & 1023u);
+  const GqaView &v = a.v;
+  const int tile = blockIdx.x, unit = blockIdx.y, tid = threadIdx.x;
+  pdl_wait();
+  const int len = v.lens[unit / v.Hkv];
+  const int t0 = tile * kPfT;
+  if (t0 >= len) {
+    pdl_trigger();
+    return;
+  }
+  uint8_t *stg = sm + p.tbytes;
+  const uint8_t *base = v.rec + (size_t)unit * v.cap * v.rec_bytes;
+  const bool sym = p.fmt >= kFmtS8, bf = p.fmt == kFmtBf16;
+  for (int e = tid; e < kPfT * p.nrec; e += kPfWorkers) {
+    const int pos = (int)__umulhi((uint32_t)e, p.nc_magic), c = e - pos * p.nrec;
+    const int t = t0 + pos;
+    const bool ok = t < len;
+    int so;
+    if (sym)
+      so = (c + sym_rot(t, p.nrec)) & (p.nrec - 1);
+    else if (!bf && c >= p.ks16 && c < 2 * p.ks16)
+      so = p.ks16 + ((c - p.ks16 + v_rot(t, v.rec_bytes, p.ks16)) & (p.ks16 - 1));
+    else
+      so = c;
+    cp_async16(stg + pos * p.b_stride + 16 * c, base + (size_t)(ok ? t : t0) * v.rec_bytes + 16 * so, ok);
+  }
+  if (sym)
+    for (int pos = tid; pos < kPfT; pos += kPfWorkers) {
+      const int t = t0 + pos;
+      const bool ok = t < len;
+      cp_async4(stg + pos * p.b_stride + v.rec_bytes, v.scales + (size_t)unit * v.cap + (ok ? t : t0), ok);
+    }
+  cp_async_commit();
+  cp_async_wait<0>();
+  __syncthreads();
+  // threads [0, 256): key quarters; [256, 512): value quarters
+  const int pidx = tid & (kPfT - 1), part = tid / kPfT;
+  const uint8_t *bundle = stg + pidx * p.b_stride;
+  const int ks = 16 * p.ks16;
+  const int mb = (p.nrec * 16 - 2 * ks) / 2;  // grouped: one metadata block
+  uint8_t *kh = sm, *kl = sm + 2 * kPfBox;
+  if (part < 4) {
+    const uint8_t *kmeta = sym ? bundle + v.rec_bytes : bundle + 2 * ks;
+    switch (p.fmt) {
+      case kFmtBf16: tc_dequant<kFmtBf16, kPfBox>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
+      case kFmtG8: tc_dequant<kFmtG8, kPfBox>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
+      case kFmtG4: tc_dequant<kFmtG4, kPfBox>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
+      case kFmtS8: tc_dequant<kFmtS8, kPfBox>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
+      case kFmtS4: tc_dequant<kFmtS4, kPfBox>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
+      default: tc_dequant<kFmtS2, kPfBox>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
+    }
+  } else {
+    const int qc = part - 4;
+    uint8_t *vh = sm + p.kbytes, *vl = vh + 2 * kPfBox;
+    const uint8_t *vsec = bundle + ks, *vmeta = bundle + 2 * ks + mb;
+    const float svs =
+        sym ? __uint_as_float(*reinterpret_cast<const uint32_t *>(bundle + v.rec_bytes) & 0xFFFF0000u) : 0.f;
+    switch (p.fmt) {
+      case kFmtBf16: tc_dequant_v<kFmtBf16, kPfBox>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
+      case kFmtG8: tc_dequant_v<kFmtG8, kPfBox>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
+      case kFmtG4: tc_dequant_v<kFmtG4, kPfBox>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
+      case kFmtS8: tc_dequant_v<kFmtS8, kPfBox>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
+      case kFmtS4: tc_dequant_v<kFmtS4, kPfBox>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
+      default: tc_dequant_v<kFmtS2, kPfBox>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
+    }
+  }
+  __syncthreads();
+  uint4 *dst = reinterpret_cast<uint4 *>(a.tiles + ((size_t)unit * p.n_t64 + tile) * p.tbytes);
+  const uint4 *src = reinterpret_cast<const uint4 *>(sm);
+  for (int i = tid; i < p.tbytes / 16; i += kPfWorkers) dst[i] = src[i];
+  pdl_trigger();
 }
 
 template <bool OUT>
 __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, const PfPlan p) {
-  constexpr int TT = OUT ? 64 : 128;     // positions per tile
-  constexpr int KBOX = TT * 128;         // one 64-channel box of a key (value) tile
   constexpr int D = 128;
   constexpr uint32_t kLimit = 1u << 20;  // polls of up to 2 us each
   extern __shared__ uint8_t pf_raw[];
   uint8_t *sm = pf_raw + ((1024u - (smem_u32(pf_raw) & 1023u)) & 1023u);
-  // bar: [0], [1] keys (and values) of an even / odd tile staged (16
-  // arrivals); [2], [3] scores of an even / odd tile done; [4] P of a tile
-  // written (16 arrivals); [5] its value product done; [6] drain
+  // barriers: kfull[3] keys of a stage landed, kfree[3] its score product
+  // done, vfull[3] / vfree[3] the same for values, sdone[2] scores of an
+  // even / odd tile done, epi the workers' epilogue of a tile done (16
+  // arrivals), pvdone a value product done, qready the job's query rows
+  // staged (16 arrivals), drain
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + p.off_bar);
-  uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + 56);
-  volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + 60);
-  volatile int *s_job = reinterpret_cast<volatile int *>(sm + p.off_bar + 64);
+  uint64_t *kfull = bar, *kfree = bar + 3, *vfull = bar + 6, *vfree = bar + 9, *sdone = bar + 12;
+  uint64_t *epi = bar + 14, *pvdone = bar + 15, *qready = bar + 16, *drain = bar + 17;
+  uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + 144);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + 148);
+  volatile int *s_job = reinterpret_cast<volatile int *>(sm + p.off_bar + 152);
   float *norm = reinterpret_cast<float *>(sm + p.off_norm);  // [128] log-normaliser per job row
   float2 *red = reinterpret_cast<float2 *>(sm + p.off_red);  // [4][128] slice statistics
   uint8_t *qh = sm, *ql = sm + p.off_ql;
@@ -81,13 +170,14 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   const int quarter = warp & 3, slice = warp >> 2;
   const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
   const float sg = a.sig_log2;
+  const int vbytes = p.tbytes - p.kbytes;
 
   if (tid == 0) {
-    for (int i = 0; i < 7; ++i) mbar_init(&bar[i], (i == 0 || i == 1 || i == 4) ? kPfWorkers / 32 : 1);
+    for (int i = 0; i < 18; ++i) mbar_init(&bar[i], (i == 14 || i == 16) ? kPfWorkers / 32 : 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  pdl_wait();
+  pdl_wait();  // the expanded tiles, lengths and (output pass) statistics are complete
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(tbase)),
@@ -99,13 +189,12 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tbase;
-  // TMEM: statistics: scores of tile k at column 128 (k & 1); output: scores
-  // at 64 (k & 1), O^T at 128
+  // TMEM: scores of tile k at column 64 (k & 1); output pass: O^T at 128
   const uint32_t t_o = tmem + 128;
 
   // Jobs are handed out one at a time from a counter (the longest row
   // blocks first), so CTAs finish together although jobs differ in length.
-  // Every thread of the CTA takes part in each hand-out; a CTA that gave up
+  // Every thread of the CTA takes part in each hand-out; a role that gave up
   // keeps taking jobs (and skips them) until none is left, so no barrier
   // waits for threads that left.
   const int units = v.B * v.Hkv;
@@ -116,7 +205,6 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     asm volatile("bar.sync 2, %0;" ::"n"(kPfThreads) : "memory");
     return *s_job;
   };
-
   struct Job {
     int unit, b, j, r0, nr, len, n_t;
   };
@@ -130,98 +218,144 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     J.r0 = rb * kPfRows;
     J.nr = min(kPfRows, R - J.r0);
     J.len = v.lens[J.b];
-    J.n_t = pf_tiles(J.len, a.n_q, a.G, J.r0 + J.nr - 1, TT);
+    J.n_t = pf_tiles(J.len, a.n_q, a.G, J.r0 + J.nr - 1);
     return J;
   };
+  auto sleepy = [&](uint64_t *b, uint32_t parity) {
+    return mbar_wait_sleepy(b, parity, kLimit, abort_flag, 2000);
+  };
 
-  if (warp == kPfWorkers / 32) {
+  if (warp == kPfWorkers / 32 + 1) {
+    // ======================= copy warp ====================================
+    // lane 0 copies each tile's keys (and values) into the next stage once
+    // the products that read the stage's previous tile are done
+    int kk = 0;
+    bool ok = true;
+    for (int job = next_job(); job < p.n_jobs; job = next_job()) {
+      if (ok && lane == 0) {
+        const Job J = job_at(job);
+        const uint8_t *src0 = a.tiles + (size_t)J.unit * p.n_t64 * p.tbytes;
+        for (int k = 0; k < J.n_t && ok; ++k, ++kk) {
+          const int s = kk % p.ns, u = kk / p.ns;
+          if (u > 0) ok = sleepy(&kfree[s], (u - 1) & 1);
+          if (ok) {
+            fence_proxy_async();
+            mbar_expect_tx(&kfull[s], p.kbytes);
+            bulk_g2s(sm + p.off_k + s * p.kbytes, src0 + (size_t)k * p.tbytes, p.kbytes, &kfull[s]);
+          }
+          if (OUT && ok) {
+            if (u > 0) ok = sleepy(&vfree[s], (u - 1) & 1);
+            if (ok) {
+              mbar_expect_tx(&vfull[s], vbytes);
+              bulk_g2s(sm + p.off_v + s * vbytes, src0 + (size_t)k * p.tbytes + p.kbytes, vbytes, &vfull[s]);
+            }
+          }
+        }
+        if (!ok) *abort_flag = 1;
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+    }
+    // the last copies land before the CTA leaves (bounded; at once when
+    // they were consumed)
+    if (lane == 0)
+      for (int c = max(0, kk - p.ns); c < kk; ++c) {
+        mbar_wait(&kfull[c % p.ns], (c / p.ns) & 1, 1u << 22);
+        if (OUT) mbar_wait(&vfull[c % p.ns], (c / p.ns) & 1, 1u << 22);
+      }
+    __syncwarp();
+  } else if (warp == kPfWorkers / 32) {
     // ======================= MMA warp =====================================
     auto dsc = [](uint32_t addr) { return umma_desc(addr, 16, 1024, 2); };
     const uint32_t qa = smem_u32(qh), qb = smem_u32(ql);
-    auto issue_s = [&](int kk) {  // S = Q K^T of the tile in stage kk % nst
+    auto issue_s = [&](int kk, int s) {  // S = Q K^T of the tile in key stage s
       tc_fence_after();
-      const uint32_t kh = smem_u32(sm + p.off_k + (kk % p.nst) * p.stage), kl = kh + 2 * KBOX;
-      const uint32_t d0 = OUT ? tmem + 64u * (kk & 1) : tmem + 128u * (kk & 1);
-      constexpr uint32_t id = umma_idesc(128, TT, false, false);
+      const uint32_t kh = smem_u32(sm + p.off_k + s * p.kbytes), kl = kh + 2 * kPfBox;
+      const uint32_t d0 = tmem + 64u * (kk & 1);
+      constexpr uint32_t id = umma_idesc(128, kPfT, false, false);
 #pragma unroll
       for (int ks = 0; ks < D / 16; ++ks) {
-        const uint32_t ko = (ks >> 2) * KBOX + (ks & 3) * 32;
+        const uint32_t ko = (ks >> 2) * kPfBox + (ks & 3) * 32;
         const uint32_t qo = (ks >> 2) * kQBox + (ks & 3) * 32;
         umma_f16(d0, dsc(qa + qo), dsc(kh + ko), id, ks > 0);
         if (p.k_lo) umma_f16(d0, dsc(qa + qo), dsc(kl + ko), id, true);
         if (p.q_lo) umma_f16(d0, dsc(qb + qo), dsc(kh + ko), id, true);
       }
-      umma_commit(&bar[2 + (kk & 1)]);
+      umma_commit(&sdone[kk & 1]);
+      umma_commit(&kfree[s]);
     };
-    auto issue_pv = [&](int kk, bool acc) {  // O^T += V^T P^T of tile kk
+    auto issue_pv = [&](int s, bool acc) {  // O^T += V^T P^T, values in stage s
       tc_fence_after();
-      const uint32_t vh = smem_u32(sm + p.off_k + (kk % p.nst) * p.stage) + 2 * (p.k_lo ? 2 : 1) * KBOX;
-      const uint32_t vl = vh + 2 * KBOX;
+      const uint32_t vh = smem_u32(sm + p.off_v + s * vbytes), vl = vh + 2 * kPfBox;
       const uint32_t pa = smem_u32(ph), pb = smem_u32(pl);
       constexpr uint32_t id = umma_idesc(128, kPfRows, true, false);
 #pragma unroll
-      for (int ks = 0; ks < TT / 16; ++ks) {
-        // values MN-major: channels in 64-wide boxes KBOX apart, 16 positions per k-step
-        const uint64_t va = umma_desc(vh + ks * 2048, KBOX, 1024, 2);
-        const uint64_t vb = umma_desc(vl + ks * 2048, KBOX, 1024, 2);
+      for (int ks = 0; ks < kPfT / 16; ++ks) {
+        // values MN-major: channels in 64-wide boxes kPfBox apart, 16 positions per k-step
+        const uint64_t va = umma_desc(vh + ks * 2048, kPfBox, 1024, 2);
+        const uint64_t vb = umma_desc(vl + ks * 2048, kPfBox, 1024, 2);
         umma_f16(t_o, va, dsc(pa + ks * 32), id, acc || ks > 0);
         if (p.k_lo) umma_f16(t_o, vb, dsc(pa + ks * 32), id, true);
         umma_f16(t_o, va, dsc(pb + ks * 32), id, true);
       }
-      umma_commit(&bar[5]);
+      umma_commit(pvdone);
+      umma_commit(&vfree[s]);
     };
-    int kk = 0;
+    uint32_t epi_seen = 0;  // epilogues this warp has waited for
+    auto wait_epi = [&](int c) -> bool {
+      bool ok = true;
+      while (ok && (int)epi_seen <= c) {
+        ok = sleepy(epi, epi_seen & 1);
+        ++epi_seen;
+      }
+      return ok;
+    };
+    auto pv = [&](int c, bool acc) -> bool {  // value product of tile c once its P is written
+      const int s = c % p.ns;
+      bool ok = wait_epi(c);
+      if (ok) ok = sleepy(&vfull[s], (c / p.ns) & 1);
+      if (ok) issue_pv(s, acc);
+      return ok;
+    };
+    int kk = 0, njob = 0;
     bool ok = true;
     for (int job = next_job(); job < p.n_jobs; job = next_job()) {
-      if (!ok) continue;
-      const Job J = job_at(job);
-      for (int k = 0; k < J.n_t && ok; ++k, ++kk) {
-        // with one stage the previous tile's values are read before the
-        // workers overwrite them with this tile; with two, this tile's scores
-        // go first so that they overlap the previous tile's P
-        const bool pv_first = OUT && p.nst == 1;
-        if (pv_first && k > 0) {
-          ok = mbar_wait_sleepy(&bar[4], (kk - 1) & 1, kLimit, abort_flag, 2000);
-          if (ok && lane == 0) issue_pv(kk - 1, k > 1);
+      if (ok && lane == 0) {
+        const Job J = job_at(job);
+        ok = sleepy(qready, njob & 1);  // this job's query rows are staged
+        ++njob;
+        for (int k = 0; k < J.n_t && ok; ++k, ++kk) {
+          const int s = kk % p.ns;
+          if (kk >= 2) ok = wait_epi(kk - 2);  // the score buffer of tile kk - 2 is read
+          if (ok) ok = sleepy(&kfull[s], (kk / p.ns) & 1);
+          if (ok) issue_s(kk, s);
+          if (OUT && ok && k > 0) ok = pv(kk - 1, k > 1);
         }
-        if (ok) ok = mbar_wait_sleepy(&bar[kk & 1], (kk >> 1) & 1, kLimit, abort_flag, 2000);
-        if (ok && lane == 0) issue_s(kk);
-        if (OUT && !pv_first && ok && k > 0) {
-          ok = mbar_wait_sleepy(&bar[4], (kk - 1) & 1, kLimit, abort_flag, 2000);
-          if (ok && lane == 0) issue_pv(kk - 1, k > 1);
-        }
-        __syncwarp();
+        if (OUT && ok && J.n_t > 0) ok = pv(kk - 1, J.n_t > 1);
+        // every epilogue of the job is awaited before the next job: a wait
+        // that fell two phases behind the barrier would read the wrong parity
+        if (ok && J.n_t > 0) ok = wait_epi(kk - 1);
+        if (!ok) *abort_flag = 1;
       }
-      if (!ok && lane == 0) *abort_flag = 1;
-      if constexpr (OUT) {
-        if (ok && J.n_t > 0) {
-          ok = mbar_wait_sleepy(&bar[4], (kk - 1) & 1, kLimit, abort_flag, 2000);
-          if (ok && lane == 0) issue_pv(kk - 1, J.n_t > 1);
-          __syncwarp();
-        }
-      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
     }
-    if (!ok && lane == 0) *abort_flag = 1;
-    // every MMA this warp issued lands before TMEM is released (bounded)
+    // every product issued lands before TMEM is released (bounded)
     if (lane == 0 && kk > 0) {
-      umma_commit(&bar[6]);
-      mbar_wait(&bar[6], 0, 1u << 22);
+      umma_commit(drain);
+      mbar_wait(drain, 0, 1u << 22);
     }
     __syncwarp();
   } else {
     // ======================= workers ======================================
-    const int pidx = tid & (TT - 1), part = tid / TT;  // staging/dequant: position, part
     bool failed = false;
     uint32_t pv_seen = 0;  // value products whose completion the workers have waited for
-    auto wait_pv = [&](int kk) -> bool {  // completion of tile kk's value product
+    auto wait_pv = [&](int c) -> bool {  // completion of tile c's value product
       bool ok = true;
-      while (ok && (int)pv_seen <= kk) {
-        ok = mbar_wait_sleepy(&bar[5], pv_seen & 1, kLimit, abort_flag, 2000);
+      while (ok && (int)pv_seen <= c) {
+        ok = sleepy(pvdone, pv_seen & 1);
         ++pv_seen;
       }
       return ok;
     };
-
     // query rows r0 .. r0 + 127 of the unit (zero past R); output pass: the
     // rows' log-normalisers (+inf for rows that see no position)
     auto load_q = [&](const Job &J) {
@@ -261,81 +395,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
           norm[rl] = nv;
         }
       }
-      fence_proxy_async();
+      fence_proxy_async();  // the rows, written here, are read by the tensor cores
       workers_sync<kPfWorkers>();
-    };
-
-    // asynchronous copy of tile k's records (rotation undone; statistics:
-    // the K section and key metadata only) into staging buffer g
-    auto stage_copy = [&](const Job &J, int k, int g) {
-      const int t0 = k * TT;
-      uint8_t *dst0 = sm + p.off_stg + g * p.stg_bytes;
-      const uint8_t *base = v.rec + (size_t)J.unit * v.cap * v.rec_bytes;
-      const bool sym = p.fmt >= kFmtS8, bf = p.fmt == kFmtBf16;
-      for (int e = tid; e < TT * p.ncopy; e += kPfWorkers) {
-        const int pos = (int)__umulhi((uint32_t)e, p.nc_magic), c = e - pos * p.ncopy;
-        const int t = t0 + pos;
-        const bool ok = t < J.len;
-        // logical chunk cl of the record, and where it is stored
-        const int cl = OUT ? c : (c < p.ks16 ? c : 2 * p.ks16 + (c - p.ks16));
-        int so;
-        if (sym) {
-          so = (cl + sym_rot(t, p.nrec)) & (p.nrec - 1);
-        } else if (!bf && cl >= p.ks16 && cl < 2 * p.ks16) {
-          so = p.ks16 + ((cl - p.ks16 + v_rot(t, v.rec_bytes, p.ks16)) & (p.ks16 - 1));
-        } else {
-          so = cl;
-        }
-        // output pass: the whole logical record; statistics: K section and
-        // key metadata back to back
-        cp_async16(dst0 + pos * p.b_stride + 16 * (OUT ? cl : c),
-                   base + (size_t)(ok ? t : t0) * v.rec_bytes + 16 * so, ok);
-      }
-      if (sym)
-        for (int pos = tid; pos < TT; pos += kPfWorkers) {
-          const int t = t0 + pos;
-          const bool ok = t < J.len;
-          cp_async4(dst0 + pos * p.b_stride + (OUT ? v.rec_bytes : 16 * p.ks16),
-                    v.scales + (size_t)J.unit * v.cap + (ok ? t : t0), ok);
-        }
-      cp_async_commit();
-    };
-
-    // dequantised keys (and values) of the tile staged in buffer g into
-    // stage s: threads [0, 4 TT) the keys by (position, channel quarter),
-    // the output pass's other threads the values
-    auto dequant = [&](int g, int s) {
-      const uint8_t *bundle = sm + p.off_stg + g * p.stg_bytes + pidx * p.b_stride;
-      uint8_t *kh = sm + p.off_k + s * p.stage, *kl = kh + 2 * KBOX;
-      const int ks = 16 * p.ks16;  // K-section bytes
-      const int mb = (p.nrec * 16 - 2 * ks) / 2;  // grouped: bytes of one metadata block
-      const bool sym = p.fmt >= kFmtS8;
-      if (part < 4) {
-        const uint8_t *kmeta = !OUT ? bundle + ks : sym ? bundle + v.rec_bytes : bundle + 2 * ks;
-        switch (p.fmt) {
-          case kFmtBf16: tc_dequant<kFmtBf16, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
-          case kFmtG8: tc_dequant<kFmtG8, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
-          case kFmtG4: tc_dequant<kFmtG4, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
-          case kFmtS8: tc_dequant<kFmtS8, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
-          case kFmtS4: tc_dequant<kFmtS4, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
-          default: tc_dequant<kFmtS2, KBOX>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
-        }
-      } else if constexpr (OUT) {
-        const int qc = part - 4;
-        uint8_t *vh = kh + 2 * (p.k_lo ? 2 : 1) * KBOX, *vl = vh + 2 * KBOX;
-        const uint8_t *vsec = bundle + ks;
-        const uint8_t *vmeta = bundle + 2 * ks + mb;
-        const float svs =
-            sym ? __uint_as_float(*reinterpret_cast<const uint32_t *>(bundle + v.rec_bytes) & 0xFFFF0000u) : 0.f;
-        switch (p.fmt) {
-          case kFmtBf16: tc_dequant_v<kFmtBf16, KBOX>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
-          case kFmtG8: tc_dequant_v<kFmtG8, KBOX>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
-          case kFmtG4: tc_dequant_v<kFmtG4, KBOX>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
-          case kFmtS8: tc_dequant_v<kFmtS8, KBOX>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
-          case kFmtS4: tc_dequant_v<kFmtS4, KBOX>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
-          default: tc_dequant_v<kFmtS2, KBOX>(vsec, vmeta, svs, pidx, qc, p.gshift, vh, vl); break;
-        }
-      }
     };
 
     int kk = 0;
@@ -344,76 +405,40 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       const Job J = job_at(job);
       const int base = J.len - a.n_q;  // position of chunk query 0
       load_q(J);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(qready);
       // this thread's row of the job in the score epilogues
       const int rl = 32 * quarter + lane;
       const bool row_live = rl < J.nr;
       const int last = base + (J.r0 + rl) / a.G;  // the last position the row sees
       const bool warp_live = 32 * quarter < J.nr;
       float m_run = -INFINITY, l_run = 0.f;  // statistics: this slice's running pair
-      const bool pipe = p.nst == 2;
-      // Stage tile kn (tile counter kkn): its records have landed; the values
-      // the stage held are read (the value product of tile kkn - nst);
-      // dequantised and announced to the MMA warp.  With two stages the next
-      // tile is staged before this tile's scores are awaited, so that the
-      // dequantisation overlaps the score product.
-      auto stage_tile = [&](int kn, int kkn) -> bool {
-        if (p.nstg == 2) {
-          if (kn + 1 < J.n_t)
-            stage_copy(J, kn + 1, (kkn + 1) & 1);  // the staging of tile kkn - 1, consumed
-          else
-            cp_async_commit();  // keeps the wait count uniform
-          cp_async_wait<1>();
-        } else {
-          cp_async_wait<0>();
-        }
-        const bool ok = OUT ? wait_pv(kkn - p.nst) : true;
-        if (workers_sync_or<kPfWorkers>(!ok)) return false;
-        if (OUT || part < 4) dequant(kkn & (p.nstg - 1), kkn % p.nst);
-        fence_proxy_async();  // the stage, written here, is read by the tensor cores
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bar[kkn & 1]);
-        if (p.nstg == 1 && kn + 1 < J.n_t) {
-          workers_sync<kPfWorkers>();  // the one staging buffer is consumed
-          stage_copy(J, kn + 1, 0);
-        }
-        return true;
-      };
-      if (J.n_t > 0) {
-        stage_copy(J, 0, kk & (p.nstg - 1));
-        if (!stage_tile(0, kk)) failed = true;
-      }
-      for (int k = 0; k < J.n_t && !failed; ++k, ++kk) {
-        if (pipe && k + 1 < J.n_t && !stage_tile(k + 1, kk + 1)) { failed = true; break; }
+      for (int k = 0; k < J.n_t; ++k, ++kk) {
         // scores of this tile; output pass: the P buffer is free
-        bool ok = mbar_wait_sleepy(&bar[2 + (kk & 1)], (kk >> 1) & 1, kLimit, abort_flag, 2000);
+        bool ok = sleepy(&sdone[kk & 1], (kk >> 1) & 1);
         if (OUT && ok) ok = wait_pv(kk - 1);
-        if (workers_sync_or<kPfWorkers>(!ok)) { failed = true; break; }
+        if (workers_sync_or<kPfWorkers>(!ok)) {
+          failed = true;
+          *abort_flag = 1;
+          break;
+        }
         tc_fence_after();
-        const int t0 = k * TT;
+        const int tb = k * kPfT + 16 * slice;  // first position of this thread's slice
         if constexpr (!OUT) {
-          // online (max, sum) of this row over the slice's 32 positions
+          // online (max, sum) of this row over the slice's 16 positions
           if (warp_live) {
-            float y[32];
-            const uint32_t ta = tmem + 128u * (kk & 1) + 32 * slice + lane_off;
-            {
-              float z[16];
-              tmem_ld16(ta, z);
-#pragma unroll
-              for (int i = 0; i < 16; ++i) y[i] = z[i];
-              tmem_ld16(ta + 16, z);
-#pragma unroll
-              for (int i = 0; i < 16; ++i) y[16 + i] = z[i];
-            }
-            const int nv = min(32, last - (t0 + 32 * slice) + 1);
+            float y[16];
+            tmem_ld16(tmem + 64u * (kk & 1) + 16 * slice + lane_off, y);
+            const int nv = min(16, last - tb + 1);
             if (row_live && nv > 0) {
               float mm = -INFINITY;
 #pragma unroll
-              for (int i = 0; i < 32; ++i)
+              for (int i = 0; i < 16; ++i)
                 if (i < nv) mm = fmaxf(mm, y[i]);
               const float mn = fmaxf(m_run, mm * sg);
               float ll[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-              for (int i = 0; i < 32; ++i)
+              for (int i = 0; i < 16; ++i)
                 if (i < nv) ll[i & 3] += fast_exp2(fmaf(y[i], sg, -mn));
               l_run = l_run * fast_exp2(m_run - mn) + ((ll[0] + ll[1]) + (ll[2] + ll[3]));
               m_run = mn;
@@ -424,7 +449,6 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
           float y[16];
           tmem_ld16(tmem + 64u * (kk & 1) + 16 * slice + lane_off, y);
           const float c = norm[rl];
-          const int tb = t0 + 16 * slice;
           float x0[8], x1[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
@@ -437,15 +461,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         }
         tc_fence_before();
         __syncwarp();
-        if (OUT && lane == 0) mbar_arrive(&bar[4]);
-        // one stage: the next tile after this one's epilogue (and, in the
-        // output pass, its value product)
-        if (!pipe && k + 1 < J.n_t && !stage_tile(k + 1, kk + 1)) { failed = true; break; }
+        if (lane == 0) mbar_arrive(epi);
       }
-      if (failed) {
-        *abort_flag = 1;
-        continue;
-      }
+      if (failed) continue;
       if constexpr (!OUT) {
         // the four slices' pairs of each row, combined
         red[slice * kPfRows + rl] = make_float2(m_run, l_run);
@@ -468,8 +486,12 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         // O^T: lane = channel 32 quarter + lane, columns = the job's rows
         float o[32];
         if (J.n_t > 0) {
-          if (!wait_pv(kk - 1)) failed = true;
-          if (workers_sync_or<kPfWorkers>(failed)) { failed = true; *abort_flag = 1; continue; }
+          const bool ok = wait_pv(kk - 1);
+          if (workers_sync_or<kPfWorkers>(!ok)) {
+            failed = true;
+            *abort_flag = 1;
+            continue;
+          }
           tc_fence_after();
           float z[16];
           tmem_ld16(t_o + 32 * slice + lane_off, z);
@@ -496,11 +518,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         workers_sync<kPfWorkers>();  // O^T read before the next job's first value product
       }
     }
-    cp_async_wait<0>();  // no copy outlives the CTA
-    if (failed) {
-      *abort_flag = 1;
-      if (tid == 0) set_err(a.err, 8);
-    }
+    if (failed && tid == 0) set_err(a.err, 8);
   }
   tc_fence_before();
   __syncthreads();
@@ -511,15 +529,16 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   pdl_trigger();
 }
 
-// Shared-memory plan: the job's query rows (hi, then lo), the key (and
-// value) stages, the staging buffers of raw records (strides odd multiples
-// of 16 bytes), P (output pass), normalisers and slice statistics, barriers.
+// Shared-memory plan.  Attention kernels: the job's query rows (hi, then
+// lo), the key stages, the value stages and P (output pass), normalisers,
+// slice statistics (statistics pass), barriers; as many stages (up to three)
+// as fit.  Expand kernel: one tile and its staged records.
 PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   PfPlan p;
   const int R = a.n_q * a.G;
-  const int TT = out ? 64 : 128;
   p.n_rb = (R + kPfRows - 1) / kPfRows;
   p.n_jobs = a.v.B * a.v.Hkv * p.n_rb;
+  p.n_t64 = a.v.cap / kPfT;
   p.q_lo = a.q_f32 ? 1 : 0;
   p.k_lo = a.v.bits != 16 ? 1 : 0;
   p.fmt = a.v.bits == 16 ? kFmtBf16
@@ -528,38 +547,39 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   p.gshift = a.v.group == 64 ? 6 : 5;
   p.ks16 = TcFmtKs16(p.fmt);
   p.nrec = a.v.rec_bytes / 16;
+  p.nc_magic = (uint32_t)((0x100000000ull + p.nrec - 1) / p.nrec);
   const bool sym = p.fmt >= kFmtS8;
-  const int kmeta16 = (p.fmt == kFmtBf16 || sym) ? 0 : (p.nrec - 2 * p.ks16) / 2;
-  p.ncopy = out ? p.nrec : p.ks16 + kmeta16;
-  p.nc_magic = (uint32_t)((0x100000000ull + p.ncopy - 1) / p.ncopy);
-  const int bchunks = (out ? p.nrec : p.ncopy) + (sym ? 1 : 0);
+  const int bchunks = p.nrec + (sym ? 1 : 0);
   p.b_stride = 16 * (bchunks % 2 ? bchunks : bchunks + 1);
-  p.stg_bytes = TT * p.b_stride;
-  const int kbox = TT * 128;
-  p.stage = 2 * kbox * ((p.k_lo ? 2 : 1) * (out ? 2 : 1));
+  p.kbytes = 2 * kPfBox * (p.k_lo ? 2 : 1);
+  p.tbytes = 2 * p.kbytes;
+  p.smem_x = p.tbytes + kPfT * p.b_stride + 1024;
   p.off_ql = kPfRows * 256;
   const int qbytes = kPfRows * 256 * (p.q_lo ? 2 : 1);
   p.off_k = (qbytes + 1023) / 1024 * 1024;
+  const int vb = out ? p.tbytes - p.kbytes : 0;
   const int pbytes = out ? 2 * kPfRows * 128 : 0;
-  const int tail = pbytes + kPfRows * 4 + 4 * kPfRows * 8 + 128 + 1024;
-  auto fits = [&](int nst, int nstg) { return p.off_k + nst * p.stage + nstg * p.stg_bytes + tail <= 232448; };
-  p.nst = fits(2, 1) ? 2 : 1;
-  p.nstg = fits(p.nst, 2) ? 2 : 1;
-  p.off_stg = p.off_k + p.nst * p.stage;
-  p.off_p = (p.off_stg + p.nstg * p.stg_bytes + 1023) / 1024 * 1024;
+  const int nbytes = out ? kPfRows * 4 : 0;
+  const int rbytes = out ? 0 : 4 * kPfRows * 8;
+  auto total = [&](int ns) { return p.off_k + ns * (p.kbytes + vb) + pbytes + nbytes + rbytes + 256 + 1024; };
+  p.ns = total(3) <= 232448 ? 3 : total(2) <= 232448 ? 2 : 1;
+  p.off_v = p.off_k + p.ns * p.kbytes;
+  p.off_p = p.off_v + p.ns * vb;
   p.off_norm = p.off_p + pbytes;
-  p.off_red = p.off_norm + kPfRows * 4;
-  p.off_bar = p.off_red + 4 * kPfRows * 8;
-  p.smem = p.off_bar + 128 + 1024;
+  p.off_red = p.off_norm + nbytes;
+  p.off_bar = p.off_red + rbytes;
+  p.smem = p.off_bar + 256 + 1024;  // + alignment of the base to 1024 bytes
   p.grid = std::max(1, std::min(p.n_jobs, sms));
   return p;
 }
 
 }  // namespace
 
+size_t prefill_tile_bytes(int bits) { return (size_t)2 * 2 * kPfBox * (bits != 16 ? 2 : 1); }
+
 bool prefill_plan_fits(const PfArgs &a) {
   const PfPlan s = pf_plan(a, false, 1), o = pf_plan(a, true, 1);
-  return s.smem <= 232448 && o.smem <= 232448;
+  return s.smem <= 232448 && o.smem <= 232448 && o.ns >= 2;
 }
 
 cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st) {
@@ -571,12 +591,17 @@ cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
   }
   const PfPlan ps = pf_plan(a, false, sms), po = pf_plan(a, true, sms);
-  cudaError_t e = cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       ps.smem);
+  cudaError_t e = cudaFuncSetAttribute(prefill_expand_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       ps.smem_x);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, ps.smem);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, po.smem);
   if (e != cudaSuccess) return e;
   e = cudaMemsetAsync(a.counter, 0, 2 * sizeof(int), st);  // the job counters
+  if (e == cudaSuccess)
+    e = launch_pdl(prefill_expand_kernel, dim3(ps.n_t64, a.v.B * a.v.Hkv), dim3(kPfWorkers), ps.smem_x, st,
+                   a, ps);
   if (e == cudaSuccess)
     e = launch_pdl(prefill_kernel<false>, dim3(ps.grid), dim3(kPfThreads), ps.smem, st, a, ps);
   if (e == cudaSuccess)
