@@ -42,9 +42,10 @@ namespace {
 constexpr int kPfWorkers = 512;
 constexpr int kPfThreads = kPfWorkers + 64;  // + the MMA warp and the copy warp
 constexpr int kPfRows = 128;                 // rows per job
-constexpr int kQBox = kPfRows * 128;         // one 64-channel box of the job's query rows
 constexpr int kPfT = 64;                     // positions per tile
 constexpr int kPfBox = kPfT * 128;           // one 64-channel box of a tile (8 KB)
+constexpr int kPfMaxStages = 6;              // key (and value) stages at most
+constexpr int kPfBarBytes = 320;             // barriers and the CTA's shared words
 
 struct PfPlan {
   int n_rb, n_jobs, grid, n_t64;
@@ -54,7 +55,8 @@ struct PfPlan {
   int b_stride;       // expand: staged record stride (odd multiple of 16 bytes)
   int kbytes, tbytes; // a tile's keys (hi, lo); the whole tile (keys, values)
   int ns;             // key (and value) stages of the attention kernels
-  int off_ql, off_k, off_v, off_p, off_norm, off_red, off_bar, smem, smem_x;
+  int band;           // units per band of the job order
+  int off_v, off_norm, off_red, off_bar, smem, smem_x;  // key stages at offset 0
 };
 
 // Tiles a job reads: positions up to that of the job's last row.
@@ -143,27 +145,62 @@ __global__ void __launch_bounds__(kPfWorkers) prefill_expand_kernel(const PfArgs
   pdl_trigger();
 }
 
+// S = Q K^T of one tile into TMEM columns d0.., Q (bf16 pairs, hi then lo
+// 64 columns on) from TMEM at t_q, the keys (hi, then lo 2 boxes on) K-major
+// in shared memory at kh: 16 channels per k-step.
+template <bool KLO, bool QLO>
+__device__ __forceinline__ void pf_issue_scores(uint32_t d0, uint32_t t_q, uint32_t kh) {
+  constexpr uint32_t id = umma_idesc(128, kPfT, false, false);
+  constexpr uint32_t hi = umma_desc_hi_sw128(1024);
+  const uint32_t lo_h = umma_desc_lo(kh, 16), lo_l = lo_h + (2 * kPfBox >> 4);
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    const uint32_t ko = ((ks >> 2) * kPfBox + (ks & 3) * 32) >> 4;
+    umma_f16_ts_w(d0, t_q + 8 * ks, lo_h + ko, hi, id, ks > 0);
+    if (KLO) umma_f16_ts_w(d0, t_q + 8 * ks, lo_l + ko, hi, id, true);
+    if (QLO) umma_f16_ts_w(d0, t_q + 64 + 8 * ks, lo_h + ko, hi, id, true);
+  }
+}
+// O += P V of one tile: P (bf16 pairs, hi then lo 32 columns on) from TMEM
+// at pa, the values (hi, then lo 2 boxes on) MN-major in shared memory at vh
+// (64-channel boxes kPfBox apart), 16 positions per k-step.
+template <bool KLO>
+__device__ __forceinline__ void pf_issue_values(uint32_t t_o, uint32_t pa, uint32_t vh, bool acc) {
+  constexpr uint32_t id = umma_idesc(128, 128, false, true);
+  constexpr uint32_t hi = umma_desc_hi_sw128(1024);
+  const uint32_t lo_h = umma_desc_lo(vh, kPfBox), lo_l = lo_h + (2 * kPfBox >> 4);
+#pragma unroll
+  for (int ks = 0; ks < kPfT / 16; ++ks) {
+    umma_f16_ts_w(t_o, pa + 8 * ks, lo_h + 128 * ks, hi, id, acc || ks > 0);
+    if (KLO) umma_f16_ts_w(t_o, pa + 8 * ks, lo_l + 128 * ks, hi, id, true);
+    umma_f16_ts_w(t_o, pa + 32 + 8 * ks, lo_h + 128 * ks, hi, id, true);
+  }
+}
+
 template <bool OUT>
 __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, const PfPlan p) {
   constexpr int D = 128;
   constexpr uint32_t kLimit = 1u << 20;  // polls of up to 2 us each
   extern __shared__ uint8_t pf_raw[];
   uint8_t *sm = pf_raw + ((1024u - (smem_u32(pf_raw) & 1023u)) & 1023u);
-  // barriers: kfull[3] keys of a stage landed, kfree[3] its score product
-  // done, vfull[3] / vfree[3] the same for values, sdone[2] scores of an
-  // even / odd tile done, epi the workers' epilogue of a tile done (16
-  // arrivals), pvdone a value product done, qready the job's query rows
-  // staged (16 arrivals), drain
+  // barriers: kfull[6] keys of a stage landed, kfree[6] its score product
+  // done, vfull[6] / vfree[6] the same for values; per tile parity: sdone[2]
+  // scores done, epi[2] the workers' epilogue done (16 arrivals), pvdone[2]
+  // value product done; qready the job's query rows staged (16 arrivals),
+  // drain.  A barrier per parity completes every other tile, and the next
+  // completion of one always depends on the wait for its previous one, so
+  // no wait can fall two phases behind.
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + p.off_bar);
-  uint64_t *kfull = bar, *kfree = bar + 3, *vfull = bar + 6, *vfree = bar + 9, *sdone = bar + 12;
-  uint64_t *epi = bar + 14, *pvdone = bar + 15, *qready = bar + 16, *drain = bar + 17;
-  uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + 144);
-  volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + 148);
-  volatile int *s_job = reinterpret_cast<volatile int *>(sm + p.off_bar + 152);
+  constexpr int S6 = kPfMaxStages;
+  uint64_t *kfull = bar, *kfree = bar + S6, *vfull = bar + 2 * S6, *vfree = bar + 3 * S6;
+  uint64_t *sdone = bar + 4 * S6, *epi = sdone + 2, *pvdone = sdone + 4, *qready = sdone + 6, *drain = sdone + 7;
+  constexpr int kBars = 4 * S6 + 8;
+  static_assert(kBars * 8 + 12 <= kPfBarBytes, "barrier region");
+  uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + kBars * 8);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + kBars * 8 + 4);
+  volatile int *s_job = reinterpret_cast<volatile int *>(sm + p.off_bar + kBars * 8 + 8);
   float *norm = reinterpret_cast<float *>(sm + p.off_norm);  // [128] log-normaliser per job row
   float2 *red = reinterpret_cast<float2 *>(sm + p.off_red);  // [4][128] slice statistics
-  uint8_t *qh = sm, *ql = sm + p.off_ql;
-  uint8_t *ph = sm + p.off_p, *pl = ph + kPfRows * 128;
   const GqaView &v = a.v;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int R = a.n_q * a.G;
@@ -173,15 +210,19 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   const int vbytes = p.tbytes - p.kbytes;
 
   if (tid == 0) {
-    for (int i = 0; i < 18; ++i) mbar_init(&bar[i], (i == 14 || i == 16) ? kPfWorkers / 32 : 1);
+    for (int i = 0; i < kBars; ++i) {
+      uint64_t *b = &bar[i];
+      mbar_init(b, (b == epi || b == epi + 1 || b == qready) ? kPfWorkers / 32 : 1);
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
   pdl_wait();  // the expanded tiles, lengths and (output pass) statistics are complete
+  constexpr uint32_t kCols = OUT ? 512 : 256;
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(tbase)),
-                 "r"(256)
+                 "n"(kCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -189,11 +230,19 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tbase;
-  // TMEM: scores of tile k at column 64 (k & 1); output pass: O^T at 128
+  // TMEM columns (lane = the job's row in every region): scores of tile k
+  // at 64 (k & 1), fp32; the job's query rows as bf16 pairs (hi 64 columns,
+  // then lo), the A operand of the score products; output pass: O at 128
+  // (fp32, 128 channels) and P of tile k at 256 + 64 (k & 1) (bf16 pairs,
+  // hi 32 columns, then lo), the A operand of the value products.
   const uint32_t t_o = tmem + 128;
+  const uint32_t t_q = tmem + (OUT ? 384 : 128);
+  auto t_p = [&](int k) { return tmem + 256 + 64 * (k & 1); };
 
-  // Jobs are handed out one at a time from a counter (the longest row
-  // blocks first), so CTAs finish together although jobs differ in length.
+  // Jobs are handed out one at a time from a counter, so CTAs finish
+  // together although jobs differ in length.  Order: bands of p.band units
+  // (whose tiles the band's jobs share in L2), in each band the longest row
+  // blocks first.
   // Every thread of the CTA takes part in each hand-out; a role that gave up
   // keeps taking jobs (and skips them) until none is left, so no barrier
   // waits for threads that left.
@@ -210,8 +259,11 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   };
   auto job_at = [&](int job) {
     Job J;
-    const int step = job / units;
-    J.unit = job - step * units;
+    const int per = p.band * p.n_rb;
+    const int g = job / per, w = job - g * per;
+    const int ub = min(p.band, units - g * p.band);  // units in this band
+    const int step = w / ub;
+    J.unit = g * p.band + (w - step * ub);
     const int rb = p.n_rb - 1 - step;
     J.b = J.unit / v.Hkv;
     J.j = J.unit - J.b * v.Hkv;
@@ -241,7 +293,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
           if (ok) {
             fence_proxy_async();
             mbar_expect_tx(&kfull[s], p.kbytes);
-            bulk_g2s(sm + p.off_k + s * p.kbytes, src0 + (size_t)k * p.tbytes, p.kbytes, &kfull[s]);
+            bulk_g2s(sm + s * p.kbytes, src0 + (size_t)k * p.tbytes, p.kbytes, &kfull[s]);
           }
           if (OUT && ok) {
             if (u > 0) ok = sleepy(&vfree[s], (u - 1) & 1);
@@ -265,55 +317,35 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     __syncwarp();
   } else if (warp == kPfWorkers / 32) {
     // ======================= MMA warp =====================================
-    auto dsc = [](uint32_t addr) { return umma_desc(addr, 16, 1024, 2); };
-    const uint32_t qa = smem_u32(qh), qb = smem_u32(ql);
     auto issue_s = [&](int kk, int s) {  // S = Q K^T of the tile in key stage s
       tc_fence_after();
-      const uint32_t kh = smem_u32(sm + p.off_k + s * p.kbytes), kl = kh + 2 * kPfBox;
-      const uint32_t d0 = tmem + 64u * (kk & 1);
-      constexpr uint32_t id = umma_idesc(128, kPfT, false, false);
-#pragma unroll
-      for (int ks = 0; ks < D / 16; ++ks) {
-        const uint32_t ko = (ks >> 2) * kPfBox + (ks & 3) * 32;
-        const uint32_t qo = (ks >> 2) * kQBox + (ks & 3) * 32;
-        umma_f16(d0, dsc(qa + qo), dsc(kh + ko), id, ks > 0);
-        if (p.k_lo) umma_f16(d0, dsc(qa + qo), dsc(kl + ko), id, true);
-        if (p.q_lo) umma_f16(d0, dsc(qb + qo), dsc(kh + ko), id, true);
+      const uint32_t kh = smem_u32(sm + s * p.kbytes), d0 = tmem + 64u * (kk & 1);
+      if (p.k_lo) {
+        if (p.q_lo) pf_issue_scores<true, true>(d0, t_q, kh);
+        else pf_issue_scores<true, false>(d0, t_q, kh);
+      } else {
+        if (p.q_lo) pf_issue_scores<false, true>(d0, t_q, kh);
+        else pf_issue_scores<false, false>(d0, t_q, kh);
       }
       umma_commit(&sdone[kk & 1]);
       umma_commit(&kfree[s]);
     };
-    auto issue_pv = [&](int s, bool acc) {  // O^T += V^T P^T, values in stage s
+    auto issue_pv = [&](int c, int s, bool acc) {  // O += P V of tile c, values in stage s
       tc_fence_after();
-      const uint32_t vh = smem_u32(sm + p.off_v + s * vbytes), vl = vh + 2 * kPfBox;
-      const uint32_t pa = smem_u32(ph), pb = smem_u32(pl);
-      constexpr uint32_t id = umma_idesc(128, kPfRows, true, false);
-#pragma unroll
-      for (int ks = 0; ks < kPfT / 16; ++ks) {
-        // values MN-major: channels in 64-wide boxes kPfBox apart, 16 positions per k-step
-        const uint64_t va = umma_desc(vh + ks * 2048, kPfBox, 1024, 2);
-        const uint64_t vb = umma_desc(vl + ks * 2048, kPfBox, 1024, 2);
-        umma_f16(t_o, va, dsc(pa + ks * 32), id, acc || ks > 0);
-        if (p.k_lo) umma_f16(t_o, vb, dsc(pa + ks * 32), id, true);
-        umma_f16(t_o, va, dsc(pb + ks * 32), id, true);
-      }
-      umma_commit(pvdone);
+      const uint32_t vh = smem_u32(sm + p.off_v + s * vbytes);
+      if (p.k_lo) pf_issue_values<true>(t_o, t_p(c), vh, acc);
+      else pf_issue_values<false>(t_o, t_p(c), vh, acc);
+      umma_commit(&pvdone[c & 1]);
       umma_commit(&vfree[s]);
     };
-    uint32_t epi_seen = 0;  // epilogues this warp has waited for
-    auto wait_epi = [&](int c) -> bool {
-      bool ok = true;
-      while (ok && (int)epi_seen <= c) {
-        ok = sleepy(epi, epi_seen & 1);
-        ++epi_seen;
-      }
-      return ok;
+    auto wait_epi = [&](int c) -> bool {  // the workers' epilogue of tile c
+      return c < 0 || sleepy(&epi[c & 1], (c >> 1) & 1);
     };
     auto pv = [&](int c, bool acc) -> bool {  // value product of tile c once its P is written
       const int s = c % p.ns;
       bool ok = wait_epi(c);
       if (ok) ok = sleepy(&vfull[s], (c / p.ns) & 1);
-      if (ok) issue_pv(s, acc);
+      if (ok) issue_pv(c, s, acc);
       return ok;
     };
     int kk = 0, njob = 0;
@@ -347,55 +379,59 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   } else {
     // ======================= workers ======================================
     bool failed = false;
-    uint32_t pv_seen = 0;  // value products whose completion the workers have waited for
     auto wait_pv = [&](int c) -> bool {  // completion of tile c's value product
-      bool ok = true;
-      while (ok && (int)pv_seen <= c) {
-        ok = sleepy(pvdone, pv_seen & 1);
-        ++pv_seen;
-      }
-      return ok;
+      return c < 0 || sleepy(&pvdone[c & 1], (c >> 1) & 1);
     };
-    // query rows r0 .. r0 + 127 of the unit (zero past R); output pass: the
-    // rows' log-normalisers (+inf for rows that see no position)
+    // query rows r0 .. r0 + 127 of the unit (zero past R) into TMEM, this
+    // thread's row and quarter of the channels; output pass: the rows'
+    // log-normalisers (+inf for rows that see no position)
     auto load_q = [&](const Job &J) {
-      for (int e = tid; e < kPfRows * (D / 8); e += kPfWorkers) {
-        const int rl = e >> 4, c8 = e & 15;
-        const int r = J.r0 + rl;
-        float x[8];
+      const int rl = 32 * quarter + lane;
+      float x[32];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) x[i] = 0.f;
-        if (rl < J.nr) {
-          const int qi = r / a.G, h = J.j * a.G + (r - qi * a.G);
-          const size_t off = (((size_t)J.b * a.n_q + qi) * a.Hq + h) * D + 8 * c8;
-          if (a.q_f32) {
-            const float4 u0 = *reinterpret_cast<const float4 *>(static_cast<const float *>(a.q) + off);
-            const float4 u1 = *reinterpret_cast<const float4 *>(static_cast<const float *>(a.q) + off + 4);
-            x[0] = u0.x; x[1] = u0.y; x[2] = u0.z; x[3] = u0.w;
-            x[4] = u1.x; x[5] = u1.y; x[6] = u1.z; x[7] = u1.w;
-          } else {
-            const uint4 u = *reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(a.q) + off);
+      for (int i = 0; i < 32; ++i) x[i] = 0.f;
+      if (rl < J.nr) {
+        const int r = J.r0 + rl;
+        const int qi = r / a.G, h = J.j * a.G + (r - qi * a.G);
+        const size_t off = (((size_t)J.b * a.n_q + qi) * a.Hq + h) * D + 32 * slice;
+        if (a.q_f32) {
+          const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(a.q) + off);
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const float4 u = src[c];
+            x[4 * c] = u.x; x[4 * c + 1] = u.y; x[4 * c + 2] = u.z; x[4 * c + 3] = u.w;
+          }
+        } else {
+          const uint4 *src = reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(a.q) + off);
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const uint4 u = src[c];
             const uint32_t ww[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-              x[2 * i] = __uint_as_float(ww[i] << 16);
-              x[2 * i + 1] = __uint_as_float(ww[i] & 0xFFFF0000u);
+              x[8 * c + 2 * i] = __uint_as_float(ww[i] << 16);
+              x[8 * c + 2 * i + 1] = __uint_as_float(ww[i] & 0xFFFF0000u);
             }
           }
         }
-        put8(qh, ql, p.q_lo != 0, rl, 8 * c8, kQBox, x);
       }
+      uint32_t hw[16], lw[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) split2<true>(x[2 * i], x[2 * i + 1], hw[i], lw[i]);
+      tmem_st16_nw(t_q + 16 * slice + lane_off, hw);
+      if (p.q_lo) tmem_st16_nw(t_q + 64 + 16 * slice + lane_off, lw);
       if constexpr (OUT) {
-        for (int rl = tid; rl < kPfRows; rl += kPfWorkers) {
+        for (int r2 = tid; r2 < kPfRows; r2 += kPfWorkers) {
           float nv = INFINITY;
-          if (rl < J.nr) {
-            const float2 f = a.stats[(size_t)J.unit * R + J.r0 + rl];
+          if (r2 < J.nr) {
+            const float2 f = a.stats[(size_t)J.unit * R + J.r0 + r2];
             if (f.y > 0.f) nv = f.x + log2f(f.y);
           }
-          norm[rl] = nv;
+          norm[r2] = nv;
         }
       }
-      fence_proxy_async();  // the rows, written here, are read by the tensor cores
+      tmem_wait_st();
+      tc_fence_before();  // the rows, stored here, are read by the tensor cores
       workers_sync<kPfWorkers>();
     };
 
@@ -414,9 +450,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       const bool warp_live = 32 * quarter < J.nr;
       float m_run = -INFINITY, l_run = 0.f;  // statistics: this slice's running pair
       for (int k = 0; k < J.n_t; ++k, ++kk) {
-        // scores of this tile; output pass: the P buffer is free
+        // scores of this tile; output pass: its P buffer is free
         bool ok = sleepy(&sdone[kk & 1], (kk >> 1) & 1);
-        if (OUT && ok) ok = wait_pv(kk - 1);
+        if (OUT && ok) ok = wait_pv(kk - 2);  // its P buffer is free
         if (workers_sync_or<kPfWorkers>(!ok)) {
           failed = true;
           *abort_flag = 1;
@@ -455,13 +491,21 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
             x0[i] = tb + i <= last ? fast_exp2(fmaf(y[i], sg, -c)) : 0.f;
             x1[i] = tb + 8 + i <= last ? fast_exp2(fmaf(y[8 + i], sg, -c)) : 0.f;
           }
-          put8(ph, pl, true, rl, 16 * slice, kPfRows * 128, x0);
-          put8(ph, pl, true, rl, 16 * slice + 8, kPfRows * 128, x1);
-          fence_proxy_async();  // P, written here, is read by the tensor cores
+          // positions 16 slice .. 16 slice + 15 of the tile: 8 columns of
+          // bf16 pairs (hi), the same 32 columns on (lo)
+          uint32_t hw[8], lw[8];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            split2<true>(x0[2 * i], x0[2 * i + 1], hw[i], lw[i]);
+            split2<true>(x1[2 * i], x1[2 * i + 1], hw[4 + i], lw[4 + i]);
+          }
+          tmem_st8_nw(t_p(kk) + 8 * slice + lane_off, hw);
+          tmem_st8_nw(t_p(kk) + 32 + 8 * slice + lane_off, lw);
+          tmem_wait_st();
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(epi);
+        if (lane == 0) mbar_arrive(&epi[kk & 1]);
       }
       if (failed) continue;
       if constexpr (!OUT) {
@@ -483,7 +527,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         }
         workers_sync<kPfWorkers>();
       } else {
-        // O^T: lane = channel 32 quarter + lane, columns = the job's rows
+        // O: lane = the job's row, 32 channels per slice
         float o[32];
         if (J.n_t > 0) {
           const bool ok = wait_pv(kk - 1);
@@ -504,18 +548,15 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
 #pragma unroll
           for (int i = 0; i < 32; ++i) o[i] = 0.f;
         }
-        const int d = 32 * quarter + lane;
+        if (row_live) {
+          const int r = J.r0 + rl;
+          const int qi = r / a.G, h = J.j * a.G + (r - qi * a.G);
+          float4 *dst = reinterpret_cast<float4 *>(a.out + (((size_t)J.b * a.n_q + qi) * a.Hq + h) * D + 32 * slice);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int rr = 32 * slice + i;
-          if (rr < J.nr) {
-            const int r = J.r0 + rr;
-            const int qi = r / a.G, h = J.j * a.G + (r - qi * a.G);
-            a.out[(((size_t)J.b * a.n_q + qi) * a.Hq + h) * D + d] = o[i];
-          }
+          for (int c = 0; c < 8; ++c) dst[c] = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
         }
         tc_fence_before();
-        workers_sync<kPfWorkers>();  // O^T read before the next job's first value product
+        workers_sync<kPfWorkers>();  // O read before the next job's first value product
       }
     }
     if (failed && tid == 0) set_err(a.err, 8);
@@ -524,7 +565,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   __syncthreads();
   tc_fence_after();
   if (warp == 0)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(kCols)
                  : "memory");
   pdl_trigger();
 }
@@ -554,21 +595,26 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   p.kbytes = 2 * kPfBox * (p.k_lo ? 2 : 1);
   p.tbytes = 2 * p.kbytes;
   p.smem_x = p.tbytes + kPfT * p.b_stride + 1024;
-  p.off_ql = kPfRows * 256;
-  const int qbytes = kPfRows * 256 * (p.q_lo ? 2 : 1);
-  p.off_k = (qbytes + 1023) / 1024 * 1024;
   const int vb = out ? p.tbytes - p.kbytes : 0;
-  const int pbytes = out ? 2 * kPfRows * 128 : 0;
   const int nbytes = out ? kPfRows * 4 : 0;
   const int rbytes = out ? 0 : 4 * kPfRows * 8;
-  auto total = [&](int ns) { return p.off_k + ns * (p.kbytes + vb) + pbytes + nbytes + rbytes + 256 + 1024; };
-  p.ns = total(3) <= 232448 ? 3 : total(2) <= 232448 ? 2 : 1;
-  p.off_v = p.off_k + p.ns * p.kbytes;
-  p.off_p = p.off_v + p.ns * vb;
-  p.off_norm = p.off_p + pbytes;
+  // the most key (and value) stages that fit; query rows and P live in TMEM
+  p.ns = 1;
+  for (int ns = kPfMaxStages; ns >= 1; --ns)
+    if (ns * (p.kbytes + vb) + nbytes + rbytes + kPfBarBytes + 1024 <= 232448) {
+      p.ns = ns;
+      break;
+    }
+  // bands of units whose tiles take up to 32 MB (L2 holds two bands)
+  const long long unit_bytes = (long long)p.n_t64 * (out ? p.tbytes : p.kbytes);
+  p.band = (int)std::max(1LL, std::min<long long>(a.v.B * a.v.Hkv, (32LL << 20) / std::max(1LL, unit_bytes)));
+  p.off_v = p.ns * p.kbytes;
+  p.off_norm = p.off_v + p.ns * vb;
   p.off_red = p.off_norm + nbytes;
   p.off_bar = p.off_red + rbytes;
-  p.smem = p.off_bar + 256 + 1024;  // + alignment of the base to 1024 bytes
+  // + alignment of the base to 1024 bytes; at least half the SM's shared
+  // memory, so that one CTA (holding its TMEM columns) runs per SM
+  p.smem = std::max(p.off_bar + kPfBarBytes + 1024, 116 * 1024);
   p.grid = std::max(1, std::min(p.n_jobs, sms));
   return p;
 }
