@@ -40,7 +40,7 @@ namespace kvk {
 namespace {
 
 constexpr int kPfWorkers = 512;
-constexpr int kPfThreads = kPfWorkers + 96;  // + two MMA warps and the copy warp
+constexpr int kPfThreads = kPfWorkers + 128;  // + three MMA warps and the copy warp
 constexpr int kPfRows = 128;                 // rows per job
 constexpr int kPfT = 64;                     // positions per tile
 constexpr int kPfBox = kPfT * 128;           // one 64-channel box of a tile (8 KB)
@@ -187,14 +187,14 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   // done, vfull[6] / vfree[6] the same for values; per tile parity: sdone[2]
   // scores done, epi[2] the workers' epilogue done (16 arrivals), pvdone[2]
   // value product done; qready the job's query rows staged (16 arrivals),
-  // drain[2] (one per MMA warp).  A barrier per parity completes every other tile, and the next
+  // drain[3] (one per MMA warp).  A barrier per parity completes every other tile, and the next
   // completion of one always depends on the wait for its previous one, so
   // no wait can fall two phases behind.
   uint64_t *bar = reinterpret_cast<uint64_t *>(sm + p.off_bar);
   constexpr int S6 = kPfMaxStages;
   uint64_t *kfull = bar, *kfree = bar + S6, *vfull = bar + 2 * S6, *vfree = bar + 3 * S6;
   uint64_t *sdone = bar + 4 * S6, *epi = sdone + 2, *pvdone = sdone + 4, *qready = sdone + 6, *drain = sdone + 7;
-  constexpr int kBars = 4 * S6 + 9;
+  constexpr int kBars = 4 * S6 + 10;
   static_assert(kBars * 8 + 12 <= kPfBarBytes, "barrier region");
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + kBars * 8);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + kBars * 8 + 4);
@@ -317,14 +317,14 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         if (OUT) mbar_wait(&vfull[c % p.ns], (c / p.ns) & 1, 1u << 22);
       }
     __syncwarp();
-  } else if (warp == kPfWorkers / 32 || warp == kPfWorkers / 32 + 2) {
+  } else if (warp >= kPfWorkers / 32) {
     // ======================= MMA warps ====================================
     // Each warp's lane 0 issues a stream of products (one thread issues at
-    // most one product per ~45 cycles, so two streams keep the tensor cores
-    // busy): warp 16 the score products (statistics pass: of the even
-    // tiles), warp 18 the value products (statistics pass: the odd tiles'
-    // scores).  A commit covers the products its own thread issued.
-    const int role = warp == kPfWorkers / 32 ? 0 : 1;
+    // most one product per ~45 cycles, so several streams keep the tensor
+    // cores busy): warps 16 and 18 the score products of the even and the
+    // odd tiles, warp 19 (output pass) the value products.  A commit covers
+    // the products its own thread issued.
+    const int role = warp == kPfWorkers / 32 ? 0 : warp == kPfWorkers / 32 + 2 ? 1 : 2;
     auto issue_s = [&](int kk, int s) {  // S = Q K^T of the tile in key stage s
       tc_fence_after();
       const uint32_t kh = smem_u32(sm + s * p.kbytes), d0 = tmem + 64u * (kk & 1);
@@ -356,10 +356,11 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       if (ok) issue_pv(c, s, acc);
       return ok;
     };
-    // Barrier phases: epi[c & 1] completes for tile c + 2 only after S(c + 2)
-    // was issued, and S(c + 2) is issued after its warp waited for epi(c);
-    // the value warp waits for epi(c) before PV(c), which the workers await
-    // before the epilogue of c + 2.  So no wait falls two phases behind.
+    // Barrier phases: a score warp waits for epi(c) (its parity's previous
+    // phase) before S(c + 2), and epi[c & 1] completes for tile c + 2 only
+    // after S(c + 2); the value warp waits for every epi(c) in order before
+    // PV(c), which the workers await before the epilogue of c + 2.  So every
+    // wait is for the phase after the one its warp last saw.
     int kk = 0, njob = 0, issued = 0;
     bool ok = true;
     for (int job = next_job(); job < p.n_jobs; job = next_job()) {
@@ -369,13 +370,13 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         ok = sleepy(qready, njob & 1);
         ++njob;
         for (int k = 0; k < J.n_t && ok; ++k, ++kk) {
-          if (OUT ? role == 0 : (kk & 1) == role) {
+          if ((kk & 1) == role) {
             const int s = kk % p.ns;
             if (kk >= 2) ok = wait_epi(kk - 2);  // the score buffer of tile kk - 2 is read
             if (ok) ok = sleepy(&kfull[s], (kk / p.ns) & 1);
             if (ok) issue_s(kk, s);
             ++issued;
-          } else if (OUT) {
+          } else if (OUT && role == 2) {
             ok = pv(kk, k > 0);
             ++issued;
           }
@@ -387,7 +388,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     // every product this warp issued lands before TMEM is released (bounded)
     if (lane == 0 && issued > 0) {
       umma_commit(&drain[role]);
-      mbar_wait(&drain[role], 0, 1u << 22);
+      mbar_wait(&drain[role], 0, 1u << 22);  // drain[0..2]
     }
     __syncwarp();
   } else {
