@@ -482,15 +482,24 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
             tmem_ld16(tmem + 64u * (kk & 1) + 16 * slice + lane_off, y);
             const int nv = min(16, last - tb + 1);
             if (row_live && nv > 0) {
-              float mm = -INFINITY;
+              float ll[4] = {0.f, 0.f, 0.f, 0.f}, mn;
+              if (nv == 16) {  // the whole slice is in the row's range (most tiles)
+                float mm[4];
 #pragma unroll
-              for (int i = 0; i < 16; ++i)
-                if (i < nv) mm = fmaxf(mm, y[i]);
-              const float mn = fmaxf(m_run, mm * sg);
-              float ll[4] = {0.f, 0.f, 0.f, 0.f};
+                for (int i = 0; i < 4; ++i) mm[i] = fmaxf(fmaxf(y[i], y[4 + i]), fmaxf(y[8 + i], y[12 + i]));
+                mn = fmaxf(m_run, fmaxf(fmaxf(mm[0], mm[1]), fmaxf(mm[2], mm[3])) * sg);
 #pragma unroll
-              for (int i = 0; i < 16; ++i)
-                if (i < nv) ll[i & 3] += fast_exp2(fmaf(y[i], sg, -mn));
+                for (int i = 0; i < 16; ++i) ll[i & 3] += fast_exp2(fmaf(y[i], sg, -mn));
+              } else {
+                float mm = -INFINITY;
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                  if (i < nv) mm = fmaxf(mm, y[i]);
+                mn = fmaxf(m_run, mm * sg);
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                  if (i < nv) ll[i & 3] += fast_exp2(fmaf(y[i], sg, -mn));
+              }
               l_run = l_run * fast_exp2(m_run - mn) + ((ll[0] + ll[1]) + (ll[2] + ll[3]));
               m_run = mn;
             }
@@ -501,10 +510,18 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
           tmem_ld16(tmem + 64u * (kk & 1) + 16 * slice + lane_off, y);
           const float c = norm[rl];
           float x0[8], x1[8];
+          if (tb + 15 <= last) {  // the whole slice is in the row's range (most tiles)
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            x0[i] = tb + i <= last ? fast_exp2(fmaf(y[i], sg, -c)) : 0.f;
-            x1[i] = tb + 8 + i <= last ? fast_exp2(fmaf(y[8 + i], sg, -c)) : 0.f;
+            for (int i = 0; i < 8; ++i) {
+              x0[i] = fast_exp2(fmaf(y[i], sg, -c));
+              x1[i] = fast_exp2(fmaf(y[8 + i], sg, -c));
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              x0[i] = tb + i <= last ? fast_exp2(fmaf(y[i], sg, -c)) : 0.f;
+              x1[i] = tb + 8 + i <= last ? fast_exp2(fmaf(y[8 + i], sg, -c)) : 0.f;
+            }
           }
           // positions 16 slice .. 16 slice + 15 of the tile: 8 columns of
           // bf16 pairs (hi), the same 32 columns on (lo)
