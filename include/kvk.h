@@ -235,8 +235,9 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
  * decode reads), with its own query heads (an inheriting layer reads its
  * anchor).  Queries before position 0 (len_b < n_q) give zeros.  Kept lists
  * are not used: pre-fill reads every position.
- *  q:       device [B, n_q, H_q, head_dim] in q_dtype (post-RoPE);
- *  out:     device float32 [B, n_q, H_q, head_dim];
+ *  q:       device [B, n_q, H_q, head_dim] in q_dtype (post-RoPE),
+ *           16-byte aligned;
+ *  out:     device float32 [B, n_q, H_q, head_dim], 16-byte aligned;
  *  scratch: device, 256-byte aligned, at least kvk_prefill_scratch_size
  *           bytes: per-row softmax statistics and the anchor's cache
  *           dequantised once into the products' operand layout (1 KB per

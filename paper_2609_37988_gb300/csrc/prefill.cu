@@ -16,16 +16,19 @@
 //    scaled scores x = sigma log2(e) <q, k> over its causal range, online
 //    over the tiles (S = Q K^T with TMEM lane = row);
 //  * outputs: per tile, S = Q K^T, P = 2^(x - M - log2 L) (zero past the
-//    row's limit) into shared memory, O^T += V^T P^T (the value tile read as
-//    an MN-major operand); after the job's last tile O^T (TMEM lane =
-//    channel) is written out.  The normalisers being final, O is never
-//    rescaled.
-// The two attention kernels run one persistent CTA per SM with three roles:
-// a copy warp brings each job's tiles in with bulk copies, an MMA warp
-// issues the tcgen05 products, 16 worker warps run the epilogues.  Products
-// are hi*hi + hi*lo + lo*hi (no lo part for bf16 caches or bf16 queries),
-// fp32 accumulation in TMEM.  Jobs are handed out from a counter, the
-// longest row blocks first.
+//    row's limit) as bf16 hi and lo pairs into TMEM, O += P V (P the A
+//    operand from TMEM, the value tile an MN-major B operand); after the
+//    job's last tile O (TMEM lane = row) is written out.  The normalisers
+//    being final, O is never rescaled.
+// The two attention kernels run one persistent CTA per SM: a copy warp
+// brings each job's tiles in with bulk copies, three MMA warps issue the
+// tcgen05 products (one thread issues at most one product per ~45 cycles:
+// the scores of even and of odd tiles, and the value products, are three
+// streams), 16 worker warps stage the query rows into TMEM (the A operand
+// of the score products) and run the epilogues.  Products are hi*hi +
+// hi*lo + lo*hi (no lo part for bf16 caches or bf16 queries), fp32
+// accumulation in TMEM.  Jobs are handed out from a counter in bands of
+// units whose tiles stay in L2, the longest row blocks first.
 #include <math.h>
 
 #include <algorithm>
