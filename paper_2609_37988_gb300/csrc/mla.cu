@@ -145,8 +145,8 @@ struct MlaCfg {
   static constexpr int OFF_Q = NST * STAGE;
   static constexpr int OFF_P = OFF_Q + QB;            // two buffers
   static constexpr int OFF_RED = OFF_P + 2 * PB;      // float [4][16] maxima, [4][16] sums
-  static constexpr int OFF_BAR = OFF_RED + 512;       // full[NST], sbar[2], pbar[2], obar[NST], dbar
-  static constexpr int NBAR = 2 * NST + 5;
+  static constexpr int OFF_BAR = OFF_RED + 512;       // full[NST], sbar[2], pbar[2], obar[NST], dbar[2]
+  static constexpr int NBAR = 2 * NST + 6;
   static constexpr int OFF_TB = OFF_BAR + 8 * NBAR;   // TMEM base address, abort flag
   static constexpr int SMEM = OFF_TB + 16 + 1024;     // + slack to align the base to 1024
   static constexpr int MV = W >= 128 ? 128 : 64;      // value UMMA M
@@ -183,8 +183,13 @@ __device__ __forceinline__ bool softmax_sync_or(bool v) {
   return r != 0;
 }
 
+// warps: 0-3 softmax, 4 score products, 5 copies, 6 value products (one
+// thread issues at most one tcgen05 product per ~45 cycles: the two product
+// streams come from two warps)
+constexpr int kMlaThreads = 224;
+
 template <int W>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kMlaThreads, 1)
     mla_decode_kernel(const __grid_constant__ CUtensorMap tmap, const MlaView v,
                       const uint16_t *__restrict__ qlat, const uint16_t *__restrict__ q_pe, int H,
                       float sig, int items_per_split, int n_splits, float *__restrict__ partial,
@@ -195,7 +200,7 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   // full[s]: tile landed in stage s; sbar[i]: scores of a tile with parity i
   // done; pbar[i]: its weights written (4 arrivals); obar[s]: the values of
-  // the tile in stage s done; dbar: everything done
+  // the tile in stage s done; dbar[2]: everything each MMA warp issued done
   uint64_t *full = reinterpret_cast<uint64_t *>(sm + C::OFF_BAR);
   uint64_t *sbar = full + C::NST, *pbar = sbar + 2, *obar = pbar + 2, *dbar = obar + C::NST;
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + C::OFF_TB);
@@ -239,7 +244,7 @@ __global__ void __launch_bounds__(192, 1)
   // (n/8) SBO + (k/8) 128 + (n%8) 16 + (k%8) 2 with SBO = (W+64)/8 128.
   // Rows 0-15: [q_lat hi | q_pe] of head n; rows 16-31: [q_lat lo | 0] of
   // head n-16.
-  if (warp != 5) {
+  if (warp < 5) {
     pdl_wait();
     constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (unused 64) | lo(W)]
     const uint16_t *qb = qlat + (size_t)b * H * QROW;
@@ -294,21 +299,8 @@ __global__ void __launch_bounds__(192, 1)
     __syncwarp();
     pdl_trigger();
   } else if (warp == 4) {
-    // ======================= MMA warp =====================================
+    // ======================= score warp ===================================
     constexpr uint32_t ID_S = umma_idesc(64, 32, false, false);
-    constexpr uint32_t ID_V = umma_idesc(C::MV, 32, true, true);
-    auto issue_values = [&](int t) {  // lane 0: O^T[:, hi | lo] += C^T [P_hi | P_lo]
-      tc_fence_after();
-      const uint64_t da = umma_desc(smem_u32(stage(t % C::NST)), C::BOX, 1024, 2);
-      const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, 1024, 0);
-#pragma unroll
-      for (int ks = 0; ks < TR / 16; ++ks)
-#pragma unroll
-        for (int mb = 0; mb < C::MB; ++mb)
-          umma_f16(t_o + 32 * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
-                   dp + (uint64_t)(ks * 16), ID_V, t > 0 || ks > 0);
-      umma_commit(&obar[t % C::NST]);
-    };
     for (int t = 0; t < n_tiles && !failed; ++t) {
       const int s = t % C::NST;
       bool ok = mbar_wait_or_abort(&full[s], (t / C::NST) & 1, kLimit, abort_flag);
@@ -335,26 +327,47 @@ __global__ void __launch_bounds__(192, 1)
                    dq + (uint64_t)(ks * 16), ID_S, ks > 0);
         umma_commit(&sbar[t & 1]);
       }
-      if (ok && t >= 1) {  // values(t-1) once P(t-1) is written
-        ok = mbar_wait_or_abort(&pbar[(t - 1) & 1], ((t - 1) >> 1) & 1, kLimit, abort_flag);
-        if (ok && lane == 0) issue_values(t - 1);
-      }
-      failed = !__all_sync(0xffffffffu, ok);
-    }
-    if (!failed && n_tiles > 0) {
-      const int t = n_tiles - 1;
-      const bool ok = mbar_wait_or_abort(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
-      if (ok && lane == 0) issue_values(t);
       failed = !__all_sync(0xffffffffu, ok);
     }
     if (failed && lane == 0) {
       *abort_flag = 1;
       set_err(err, 8);
     }
-    // every UMMA lands before the CTA leaves (bounded)
+    // every UMMA this warp issued lands before the CTA leaves (bounded)
     if (lane == 0) {
-      umma_commit(dbar);
-      mbar_wait(dbar, 0, kLimit);
+      umma_commit(&dbar[0]);
+      mbar_wait(&dbar[0], 0, kLimit);
+    }
+    __syncwarp();
+    pdl_trigger();
+  } else if (warp == 6) {
+    // ======================= value warp ===================================
+    // values(t) once P(t) is written; it waits for every pbar phase in
+    // order, and pbar(t + 2) needs obar(t), committed after values(t)
+    constexpr uint32_t ID_V = umma_idesc(C::MV, 32, true, true);
+    for (int t = 0; t < n_tiles && !failed; ++t) {
+      const bool ok = mbar_wait_or_abort(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
+      if (ok && lane == 0) {  // O^T[:, hi | lo] += C^T [P_hi | P_lo]
+        tc_fence_after();
+        const uint64_t da = umma_desc(smem_u32(stage(t % C::NST)), C::BOX, 1024, 2);
+        const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, 1024, 0);
+#pragma unroll
+        for (int ks = 0; ks < TR / 16; ++ks)
+#pragma unroll
+          for (int mb = 0; mb < C::MB; ++mb)
+            umma_f16(t_o + 32 * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
+                     dp + (uint64_t)(ks * 16), ID_V, t > 0 || ks > 0);
+        umma_commit(&obar[t % C::NST]);
+      }
+      failed = !__all_sync(0xffffffffu, ok);
+    }
+    if (failed && lane == 0) {
+      *abort_flag = 1;
+      set_err(err, 8);
+    }
+    if (lane == 0) {
+      umma_commit(&dbar[1]);
+      mbar_wait(&dbar[1], 0, kLimit);
     }
     __syncwarp();
     pdl_trigger();
@@ -682,7 +695,7 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
                              static_cast<const uint16_t *>(a.q_pe),
                              static_cast<const uint16_t *>(a.w_uk), B, a.H, a.r, a.qlat);
   if (e == cudaSuccess)
-    e = launch_pdl(k, dim3(a.n_splits, B), dim3(192), C::SMEM, st,
+    e = launch_pdl(k, dim3(a.n_splits, B), dim3(kMlaThreads), C::SMEM, st,
                    *static_cast<const CUtensorMap *>(a.tmap), a.v,
                    static_cast<const uint16_t *>(a.qlat), static_cast<const uint16_t *>(a.q_pe),
                    a.H, a.sig_log2, a.items_per_split, a.n_splits, a.partial, a.err);
@@ -712,10 +725,10 @@ int mla_ctas_t() {
       cudaDeviceGetAttribute(&resv, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess)
     return 1;
   const int warp_regs = (fa.numRegs * 32 + 255) / 256 * 256;  // allocation unit: 256
-  const int by_regs = regs_sm / (6 * warp_regs);
+  const int by_regs = regs_sm / (kMlaThreads / 32 * warp_regs);
   const int by_smem = smem_sm / (C::SMEM + resv);
   const int by_tmem = 512 / C::TCOLS;
-  const int n = std::min(std::min(by_regs, by_smem), std::min(by_tmem, 2048 / 192));
+  const int n = std::min(std::min(by_regs, by_smem), std::min(by_tmem, 2048 / kMlaThreads));
   return n > 0 ? n : 1;
 }
 
