@@ -145,8 +145,8 @@ struct MlaCfg {
   static constexpr int OFF_Q = NST * STAGE;
   static constexpr int OFF_P = OFF_Q + QB;            // two buffers
   static constexpr int OFF_RED = OFF_P + 2 * PB;      // float [4][16] maxima, [4][16] sums
-  static constexpr int OFF_BAR = OFF_RED + 512;       // full[NST], sbar[2], pbar[2], obar[NST], dbar[2]
-  static constexpr int NBAR = 2 * NST + 6;
+  static constexpr int OFF_BAR = OFF_RED + 512;       // full[NST], sbar[2], pbar[2], obar[NST], dbar[3]
+  static constexpr int NBAR = 2 * NST + 7;
   static constexpr int OFF_TB = OFF_BAR + 8 * NBAR;   // TMEM base address, abort flag
   static constexpr int SMEM = OFF_TB + 16 + 1024;     // + slack to align the base to 1024
   static constexpr int MV = W >= 128 ? 128 : 64;      // value UMMA M
@@ -183,10 +183,10 @@ __device__ __forceinline__ bool softmax_sync_or(bool v) {
   return r != 0;
 }
 
-// warps: 0-3 softmax, 4 score products, 5 copies, 6 value products (one
-// thread issues at most one tcgen05 product per ~45 cycles: the two product
-// streams come from two warps)
-constexpr int kMlaThreads = 224;
+// warps: 0-3 softmax, 4 and 7 the score products of even and odd tiles, 5
+// copies, 6 value products (one thread issues at most one tcgen05 product
+// per ~45 cycles: the products come as three streams)
+constexpr int kMlaThreads = 256;
 
 template <int W>
 __global__ void __launch_bounds__(kMlaThreads, 1)
@@ -200,7 +200,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
   uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   // full[s]: tile landed in stage s; sbar[i]: scores of a tile with parity i
   // done; pbar[i]: its weights written (4 arrivals); obar[s]: the values of
-  // the tile in stage s done; dbar[2]: everything each MMA warp issued done
+  // the tile in stage s done; dbar[3]: everything each MMA warp issued done
   uint64_t *full = reinterpret_cast<uint64_t *>(sm + C::OFF_BAR);
   uint64_t *sbar = full + C::NST, *pbar = sbar + 2, *obar = pbar + 2, *dbar = obar + C::NST;
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + C::OFF_TB);
@@ -244,11 +244,12 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
   // (n/8) SBO + (k/8) 128 + (n%8) 16 + (k%8) 2 with SBO = (W+64)/8 128.
   // Rows 0-15: [q_lat hi | q_pe] of head n; rows 16-31: [q_lat lo | 0] of
   // head n-16.
-  if (warp < 5) {
+  if (warp < 5 || warp == 7) {
     pdl_wait();
     constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (unused 64) | lo(W)]
     const uint16_t *qb = qlat + (size_t)b * H * QROW;
-    for (int q = tid; q < 32 * (C::KH / 8); q += 160) {  // 16-byte cp.async, zero-filled
+    // warps 0-4 stage it; the second score warp only waits for it
+    for (int q = tid; warp < 5 && q < 32 * (C::KH / 8); q += 160) {  // 16-byte cp.async, zero-filled
       const int n = q / (C::KH / 8), c = q % (C::KH / 8);
       const int h = n & 15;
       const uint16_t *src = qb;
@@ -263,7 +264,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     cp_async_wait<0>();
     fence_proxy_async();
     tc_fence_before();
-    asm volatile("bar.sync 2, 160;" ::: "memory");  // warps 0-4: the query is staged
+    asm volatile("bar.sync 2, 192;" ::: "memory");  // warps 0-4 and 7: the query is staged
     tc_fence_after();
   }
   const uint32_t tmem = *tbase;
@@ -298,12 +299,20 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     }
     __syncwarp();
     pdl_trigger();
-  } else if (warp == 4) {
-    // ======================= score warp ===================================
+  } else if (warp == 4 || warp == 7) {
+    // ======================= score warps ==================================
+    // warp 4 the even tiles, warp 7 the odd ones.  Before tile t a warp
+    // waits for softmax(t-2) (its S buffer is free), which follows softmax
+    // of every earlier tile, hence the landing of the stage's previous tile
+    // (t - NST <= t - 2): its wait for full[t % NST] is then for the phase
+    // right after the last completed one.
+    const int role = warp == 4 ? 0 : 1;
     constexpr uint32_t ID_S = umma_idesc(64, 32, false, false);
-    for (int t = 0; t < n_tiles && !failed; ++t) {
+    for (int t = role; t < n_tiles && !failed; t += 2) {
       const int s = t % C::NST;
-      bool ok = mbar_wait_or_abort(&full[s], (t / C::NST) & 1, kLimit, abort_flag);
+      bool ok = true;
+      if (t >= 2) ok = mbar_wait_or_abort(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag);
+      if (ok) ok = mbar_wait_or_abort(&full[s], (t / C::NST) & 1, kLimit, abort_flag);
       // rows past the split's end: zero them (the cache may hold anything)
       const int nval = min(TR, i1 - (i0 + t * TR));
       if (ok && nval < TR) {
@@ -315,8 +324,6 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         fence_proxy_async();
         __syncwarp();
       }
-      // the S buffer of tile t was read by softmax(t-2)
-      if (ok && t >= 2) ok = mbar_wait_or_abort(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag);
       if (ok && lane == 0) {  // scores(t) -> S[t & 1]
         tc_fence_after();
         const uint64_t dc = umma_desc(smem_u32(stage(s)), 16, 1024, 2);
@@ -335,8 +342,8 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     }
     // every UMMA this warp issued lands before the CTA leaves (bounded)
     if (lane == 0) {
-      umma_commit(&dbar[0]);
-      mbar_wait(&dbar[0], 0, kLimit);
+      umma_commit(&dbar[2 * role]);
+      mbar_wait(&dbar[2 * role], 0, kLimit);
     }
     __syncwarp();
     pdl_trigger();
