@@ -57,7 +57,8 @@ struct PfPlan {
   uint32_t nc_magic;  // expand: ceil(2^32 / nrec), e / nrec = umulhi(e, nc_magic)
   int b_stride;       // expand: staged record stride (odd multiple of 16 bytes)
   int kbytes, tbytes; // a tile's keys (hi, lo); the whole tile (keys, values)
-  int ns;             // key (and value) stages of the attention kernels
+  int ns;             // key stages of the attention kernels
+  int nv;             // value stages (output pass)
   int band;           // units per band of the job order
   int off_v, off_norm, off_red, off_bar, smem, smem_x;  // key stages at offset 0
 };
@@ -301,10 +302,11 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
             bulk_g2s(sm + s * p.kbytes, src0 + (size_t)k * p.tbytes, p.kbytes, &kfull[s]);
           }
           if (OUT && ok) {
-            if (u > 0) ok = sleepy(&vfree[s], (u - 1) & 1);
+            const int sv = kk % p.nv, uv = kk / p.nv;
+            if (uv > 0) ok = sleepy(&vfree[sv], (uv - 1) & 1);
             if (ok) {
-              mbar_expect_tx(&vfull[s], vbytes);
-              bulk_g2s(sm + p.off_v + s * vbytes, src0 + (size_t)k * p.tbytes + p.kbytes, vbytes, &vfull[s]);
+              mbar_expect_tx(&vfull[sv], vbytes);
+              bulk_g2s(sm + p.off_v + sv * vbytes, src0 + (size_t)k * p.tbytes + p.kbytes, vbytes, &vfull[sv]);
             }
           }
         }
@@ -315,9 +317,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     // the last copies land before the CTA leaves (bounded; at once when
     // they were consumed)
     if (lane == 0)
-      for (int c = max(0, kk - p.ns); c < kk; ++c) {
-        mbar_wait(&kfull[c % p.ns], (c / p.ns) & 1, 1u << 22);
-        if (OUT) mbar_wait(&vfull[c % p.ns], (c / p.ns) & 1, 1u << 22);
+      for (int c = max(0, kk - max(p.ns, p.nv)); c < kk; ++c) {
+        if (c >= kk - p.ns) mbar_wait(&kfull[c % p.ns], (c / p.ns) & 1, 1u << 22);
+        if (OUT && c >= kk - p.nv) mbar_wait(&vfull[c % p.nv], (c / p.nv) & 1, 1u << 22);
       }
     __syncwarp();
   } else if (warp >= kPfWorkers / 32) {
@@ -353,9 +355,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       return c < 0 || sleepy(&epi[c & 1], (c >> 1) & 1);
     };
     auto pv = [&](int c, bool acc) -> bool {  // value product of tile c once its P is written
-      const int s = c % p.ns;
+      const int s = c % p.nv;
       bool ok = wait_epi(c);
-      if (ok) ok = sleepy(&vfull[s], (c / p.ns) & 1);
+      if (ok) ok = sleepy(&vfull[s], (c / p.nv) & 1);
       if (ok) issue_pv(c, s, acc);
       return ok;
     };
@@ -633,18 +635,25 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   const int vb = out ? p.tbytes - p.kbytes : 0;
   const int nbytes = out ? kPfRows * 4 : 0;
   const int rbytes = out ? 0 : 4 * kPfRows * 8;
-  // the most key (and value) stages that fit; query rows and P live in TMEM
-  p.ns = 1;
-  for (int ns = kPfMaxStages; ns >= 1; --ns)
-    if (ns * (p.kbytes + vb) + nbytes + rbytes + kPfBarBytes + 1024 <= 232448) {
-      p.ns = ns;
-      break;
-    }
+  // the most stages that fit (query rows and P live in TMEM).  Output
+  // pass: value tiles wait for the value product three tiles back, key
+  // tiles only for the score product, so values get the larger share
+  // (int4: 2 key and 5 value stages of 32 KB); keys keep at least two
+  // (a score warp's wait for the stage it skipped relies on ns >= 2).
+  const int avail = 232448 - (nbytes + rbytes + kPfBarBytes + 1024);
+  if (!out) {
+    p.ns = std::max(1, std::min(kPfMaxStages, avail / p.kbytes));
+    p.nv = 1;
+  } else {
+    const int T = avail / p.kbytes;  // key and value tiles are the same size
+    p.ns = std::min(kPfMaxStages, std::max(2, T / 3));
+    p.nv = std::max(1, std::min(kPfMaxStages, T - p.ns));
+  }
   // bands of units whose tiles take up to 32 MB (L2 holds two bands)
   const long long unit_bytes = (long long)p.n_t64 * (out ? p.tbytes : p.kbytes);
   p.band = (int)std::max(1LL, std::min<long long>(a.v.B * a.v.Hkv, (32LL << 20) / std::max(1LL, unit_bytes)));
   p.off_v = p.ns * p.kbytes;
-  p.off_norm = p.off_v + p.ns * vb;
+  p.off_norm = p.off_v + p.nv * vb;
   p.off_red = p.off_norm + nbytes;
   p.off_bar = p.off_red + rbytes;
   // + alignment of the base to 1024 bytes; at least half the SM's shared
@@ -660,7 +669,7 @@ size_t prefill_tile_bytes(int bits) { return (size_t)2 * 2 * kPfBox * (bits != 1
 
 bool prefill_plan_fits(const PfArgs &a) {
   const PfPlan s = pf_plan(a, false, 1), o = pf_plan(a, true, 1);
-  return s.smem <= 232448 && o.smem <= 232448 && o.ns >= 2;
+  return s.smem <= 232448 && o.smem <= 232448 && o.ns >= 2 && o.nv >= 2;
 }
 
 cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st) {
