@@ -55,7 +55,7 @@ typedef enum {
   KVK_ERR_INVALID_CONFIG = 2,  /* plan rejected (e.g. layer 0 inherits)      */
   KVK_ERR_INHERITED_LAYER = 3, /* write to a layer that owns no cache        */
   KVK_ERR_CAPACITY = 4,        /* append would pass max_ctx                  */
-  KVK_ERR_UNSUPPORTED = 5,     /* valid request this build does not handle   */
+  KVK_ERR_UNSUPPORTED = 5,     /* valid request this library does not handle */
   KVK_ERR_CUDA = 6,            /* a CUDA runtime call failed                 */
   KVK_ERR_DEVICE = 7           /* the device error word was set              */
 } kvk_status;
@@ -97,12 +97,12 @@ typedef struct {
  *  scheme KVK_QUANT_GROUPED: `group` elements per fp32 (scale, zero) pair;
  *    key_axis selects per-token groups (g channels of one token) or
  *    per-channel groups (g positions of one channel, KIVI keys); values are
- *    per-token.  This build: bits 8 or 4, group 32 or 64.
+ *    per-token.  This library: bits 8 or 4, group 32 or 64.
  *  scheme KVK_QUANT_SYMMETRIC: the paper's quantiser (Appendix C.3): one
  *    bf16 scale s = max|x| / q per token-head row of keys and of values,
  *    codes clip(rint(x / s), -q, q) with q = 2^(b-1) - 1 (three levels at
  *    two bits), x = code * s; `group` is ignored and both axes must be
- *    KVK_AXIS_TOKEN.  This build: GQA, head_dim 128, bits 8, 4 or 2.
+ *    KVK_AXIS_TOKEN.  This library: GQA, head_dim 128, bits 8, 4 or 2.
  * evict_capacity > 0 reserves a kept-position list of that length per
  * sequence (eviction composed with compression, Sec. 3.3). */
 typedef struct {
@@ -123,7 +123,7 @@ typedef struct kvk_cache kvk_cache;
  * Errors: INVALID_ARG, INVALID_CONFIG (layer 0 inherits, bits not in
  * {16,8,4,2}, unknown scheme, group not dividing head_dim for the grouped
  * scheme, a per-channel axis with the symmetric scheme, MLA width not in
- * r/8..r), and UNSUPPORTED for valid plans outside this build (grouped 2-bit
+ * r/8..r), and UNSUPPORTED for valid plans outside this library (grouped 2-bit
  * codes, per-channel values, head_dim other than 64/128, the symmetric
  * scheme with head_dim 64 or on MLA, per-channel keys with eviction). */
 kvk_status kvk_cache_plan(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
@@ -326,7 +326,7 @@ kvk_status kvk_splitk_reduce(const float *partials, int32_t n_splits, int32_t n_
 
 /* Cost accounting of the cache's plan.
  *  bits_per_token_model: sum over layers of eq. (cost), in bits per token;
- *  bytes_per_token_stored: bytes this build stores per token, summed over
+ *  bytes_per_token_stored: bytes this library stores per token, summed over
  *      anchors, including the quantisers' metadata (fp32 scale/zero pairs,
  *      or two bf16 scales per row for the symmetric scheme; Tab. realized_bits
  *      counts metadata the same way);

@@ -91,5 +91,5 @@ def bits_per_element_grouped(b: int, g: int, meta_bits: int = 32,
 
 def bytes_per_row_grouped(d_h: int, b: int, g: int, meta_bytes_per_group: int = 8) -> int:
     """Stored bytes of one quantised (token, head) row: codes + fp32 scale and
-    zero per group (the layout this build stores)."""
+    zero per group (the layout the library stores)."""
     return d_h * b // 8 + (d_h // g) * meta_bytes_per_group

@@ -53,7 +53,7 @@ kvk_status check_desc(const kvk_model_desc *d, bool need_support = true) {
       return fail(KVK_ERR_INVALID_ARG, "n_q_heads must be a positive multiple of n_kv_heads");
     if (d->head_dim <= 0) return fail(KVK_ERR_INVALID_ARG, "head_dim must be positive");
     if (need_support && d->head_dim != 64 && d->head_dim != 128)
-      return fail(KVK_ERR_UNSUPPORTED, "head_dim %d (this build supports 64 and 128)", d->head_dim);
+      return fail(KVK_ERR_UNSUPPORTED, "head_dim %d (supported: 64 and 128)", d->head_dim);
     if (need_support && d->n_q_heads / d->n_kv_heads > 8)
       return fail(KVK_ERR_UNSUPPORTED, "more than 8 query heads per KV head");
   } else {
@@ -79,12 +79,12 @@ kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
     if (c->bits != 16 && c->bits != 8 && c->bits != 4 && c->bits != 2)
       return fail(KVK_ERR_INVALID_CONFIG, "layer %d: bits %d not in {16, 8, 4, 2}", l, c->bits);
     if (need_support && c->bits != 16)
-      return fail(KVK_ERR_UNSUPPORTED, "layer %d: quantised MLA latents are not in this build", l);
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: quantised MLA latents are not supported", l);
     const int r = d->latent_dim;
     if (c->width != r && c->width != r / 2 && c->width != r / 4 && c->width != r / 8)
       return fail(KVK_ERR_INVALID_CONFIG, "layer %d: width %d not in {r/8, r/4, r/2, r}", l, c->width);
     if (need_support && c->width != 64 && c->width != 128 && c->width != 256 && c->width != 512)
-      return fail(KVK_ERR_UNSUPPORTED, "layer %d: width %d (this build: 64..512)", l, c->width);
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: width %d (supported: 64..512)", l, c->width);
     if (need_support && c->evict_capacity)
       return fail(KVK_ERR_UNSUPPORTED, "layer %d: eviction lists on MLA layers", l);
     return KVK_OK;
@@ -97,7 +97,7 @@ kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
       return fail(KVK_ERR_INVALID_CONFIG,
                   "layer %d: the symmetric scheme scales whole token-head rows", l);
     if (need_support && d->head_dim != 128)
-      return fail(KVK_ERR_UNSUPPORTED, "layer %d: symmetric scheme with head_dim %d (this build: 128)",
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: symmetric scheme with head_dim %d (supported: 128)",
                   l, d->head_dim);
   } else if (c->bits != 16) {
     if (c->group <= 0 || d->head_dim % c->group)
@@ -105,9 +105,9 @@ kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
     if (!need_support) return KVK_OK;
     if (c->bits == 2)
       return fail(KVK_ERR_UNSUPPORTED,
-                  "layer %d: grouped 2-bit codes are not in this build (the symmetric scheme has them)", l);
+                  "layer %d: grouped 2-bit codes are not supported (the symmetric scheme has them)", l);
     if (c->group != 32 && c->group != 64)
-      return fail(KVK_ERR_UNSUPPORTED, "layer %d: group %d (this build: 32, 64)", l, c->group);
+      return fail(KVK_ERR_UNSUPPORTED, "layer %d: group %d (supported: 32, 64)", l, c->group);
     if (c->value_axis != KVK_AXIS_TOKEN)
       return fail(KVK_ERR_UNSUPPORTED, "layer %d: values are quantised per token", l);
     if (c->key_axis != KVK_AXIS_TOKEN && c->key_axis != KVK_AXIS_CHANNEL)

@@ -138,7 +138,7 @@ def test_symmetric_plan_validation(lib):
     # unknown scheme; 3 bits
     assert _plan_status(lib, d, _plan(lib, (0, 4, 32, 0, 0, 0, 0, 2), BF16, BF16, BF16))[0] == 2
     assert _plan_status(lib, d, _plan(lib, _sym(3), BF16, BF16, BF16))[0] == 2
-    # head_dim 64 and MLA latents are outside this build
+    # head_dim 64 and MLA latents are outside what the library supports
     assert _plan_status(lib, _desc(lib, head_dim=64), _plan(lib, _sym(4), BF16, BF16, BF16))[0] == 5
     m = _desc(lib, kind=1, n_layers=1, n_q_heads=16, head_dim=128, latent_dim=512, rope_dim=64)
     assert _plan_status(lib, m, _plan(lib, (0, 4, 0, 0, 0, 512, 0, 1)))[0] == 5
