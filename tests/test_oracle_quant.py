@@ -204,3 +204,96 @@ def test_symmetric_anchor_state():
             err = np.abs(st[name + "_hat"][b, :, :n] - x[b, :, :n]).max(-1)
             assert (err <= 0.5 * st[name + "_scale"][b, :, :n] + 1e-6).all()
             assert (st[name + "_hat"][b, :, n:] == 0).all()
+
+
+# ---- dequantisers: pinned against scalar loops over (position, channel) ----
+# A group index taken as i % n_groups instead of i // g (np.tile for
+# np.repeat), a scale/zero swap or a per-channel group indexed by channel
+# instead of by position fails these: every group gets its own scale and zero.
+
+@pytest.mark.parametrize("group", [32, 64])
+def test_dequantise_per_token_matches_scalar_loop(group):
+    rng = np.random.default_rng(100 + group)
+    D = 128
+    n_g = D // group
+    codes = rng.integers(0, 16, (2, 3, D), dtype=np.uint8)
+    scale = rng.uniform(0.1, 2.0, (2, 3, n_g)).astype(F32)
+    zero = rng.uniform(-3.0, 3.0, (2, 3, n_g)).astype(F32)
+    got = quant.dequantise_per_token(codes, scale, zero, group)
+    assert got.shape == (2, 3, D) and got.dtype == np.float64
+    for idx in np.ndindex(2, 3):
+        for i in range(D):
+            want = float(codes[idx][i]) * float(scale[idx][i // group]) + float(zero[idx][i // group])
+            assert got[idx][i] == want, (idx, i)
+
+
+@pytest.mark.parametrize("bits,group", [(8, 64), (4, 32), (4, 64), (2, 32)])
+def test_per_token_roundtrip_through_dequantiser(bits, group):
+    # |x - dequant(quant(x))| <= scale/2 of the element's own group (plus
+    # binary32 slack), through the two library functions
+    rng = np.random.default_rng(bits * 1000 + group)
+    x = (rng.standard_normal((4, 2, 9, 128)) * rng.lognormal(0, 1, (1, 1, 1, 128))).astype(F32)
+    c, s, z = quant.quantise_per_token(x, bits, group)
+    xh = quant.dequantise_per_token(c, s, z, group)
+    slack = 8 * np.finfo(np.float32).eps * np.abs(x).max()
+    for i in range(128):
+        bound = 0.5 * s[..., i // group].astype(np.float64) + slack
+        assert (np.abs(xh[..., i] - x[..., i]) <= bound).all(), i
+
+
+def test_dequantise_per_channel_matches_scalar_loop():
+    rng = np.random.default_rng(12)
+    g, nG, D, R = 32, 3, 8, 5
+    codes = rng.integers(0, 256, (2, nG * g, D), dtype=np.uint8)
+    scale = rng.uniform(0.1, 2.0, (2, nG, D)).astype(F32)
+    zero = rng.uniform(-3.0, 3.0, (2, nG, D)).astype(F32)
+    resid = rng.standard_normal((2, R, D)).astype(F32)
+    got = quant.dequantise_per_channel(codes, scale, zero, g, resid)
+    assert got.shape == (2, nG * g + R, D)
+    for h in range(2):
+        for t in range(nG * g):
+            for ch in range(D):
+                want = float(codes[h, t, ch]) * float(scale[h, t // g, ch]) + float(zero[h, t // g, ch])
+                assert got[h, t, ch] == want, (h, t, ch)
+        for t in range(R):
+            assert (got[h, nG * g + t] == resid[h, t].astype(np.float64)).all()
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_per_channel_roundtrip_through_dequantiser(bits):
+    rng = np.random.default_rng(60 + bits)
+    g, T, D = 32, 100, 16          # three full groups + 4 residual positions
+    x = (rng.standard_normal((T, D)) * rng.lognormal(0, 1, (1, D))).astype(F32)
+    c, s, z, r = quant.quantise_per_channel(x, bits, g)
+    xh = quant.dequantise_per_channel(c, s, z, g, r)
+    slack = 8 * np.finfo(np.float32).eps * np.abs(x).max()
+    for t in range(96):
+        bound = 0.5 * s[t // g].astype(np.float64) + slack
+        assert (np.abs(xh[t] - x[t]) <= bound).all(), t
+    assert (xh[96:] == x[96:]).all()
+
+
+@pytest.mark.parametrize("bits,group", [(8, 64), (4, 32)])
+def test_grouped_per_token_anchor_state_matches_brute_force(bits, group):
+    # the anchor state the grouped per-token workloads use, element by
+    # element from the scalar quantiser of _brute_group: codes, scales,
+    # zeros and x_hat = code * scale + zero, zeros past each length
+    from oracle import cache as ocache
+    rng = np.random.default_rng(bits + group)
+    B, H, T, D = 2, 2, 6, 128
+    k = rng.standard_normal((B, H, T, D)).astype(F32)
+    v = (rng.standard_normal((B, H, T, D)) * 3.0).astype(F32)
+    lens = [6, 3]
+    st = ocache.anchor_state(k, v, lens, bits, group)
+    for name, x in (("k", k), ("v", v)):
+        for b in range(B):
+            for h in range(H):
+                for t in range(T):
+                    for gi in range(D // group):
+                        bc, bs, bz = _brute_group(list(x[b, h, t, gi * group:(gi + 1) * group]), bits)
+                        assert list(st[name + "_codes"][b, h, t, gi * group:(gi + 1) * group]) == bc
+                        assert st[name + "_scale"][b, h, t, gi] == bs
+                        assert st[name + "_zero"][b, h, t, gi] == bz
+                        for i in range(group):
+                            want = float(bc[i]) * float(bs) + float(bz) if t < lens[b] else 0.0
+                            assert st[name + "_hat"][b, h, t, gi * group + i] == want
