@@ -100,14 +100,24 @@ class Clocks:
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index),
-                 "--query-gpu=clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "--query-gpu=timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
                  "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
                  "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "10"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            # the timed region starts once the sampler is producing rows
+            t0 = time.perf_counter()
+            while time.perf_counter() - t0 < 10.0 and self.proc.poll() is None:
+                if os.path.getsize(self.path) > 0:
+                    break
+                time.sleep(0.01)
         except Exception:
             self.proc = None
         return self
+
+    def mark(self, which):
+        """Host wall-clock time of the start or end of the timed region."""
+        setattr(self, "t_" + which, time.time())
 
     def __exit__(self, *exc):
         if self.proc:
@@ -120,13 +130,24 @@ class Clocks:
     def summary(self):
         if not self.proc or not self.path:
             return None
+        import datetime
         rows = []
         with open(self.path) as f:
             for line in f:
                 parts = [x.strip() for x in line.split(",")]
-                if len(parts) >= 8:
-                    rows.append(parts)
+                if len(parts) >= 9:
+                    try:
+                        ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                    except ValueError:
+                        ts = None
+                    rows.append((ts, parts[1:]))
         os.unlink(self.path)
+        # rows sampled inside the timed region (all rows if none carry a
+        # usable time stamp or the region was too short to hold one)
+        t0, t1 = getattr(self, "t_start", None), getattr(self, "t_end", None)
+        inside = [r for ts, r in rows if ts is not None and t0 is not None and t1 is not None
+                  and t0 <= ts <= t1]
+        rows = inside or [r for _, r in rows]
         if not rows:
             return None
         sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
@@ -134,7 +155,8 @@ class Clocks:
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({n for r in rows for n, v in zip(names, r[4:8]) if v.lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None,
-                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows),
+                "samples_in_timed_region": len(inside), "interval_ms": 10}
 
 
 def reduce_max(x: float, dist=None, device=None) -> float:
@@ -498,12 +520,14 @@ def main():
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with Clocks(local) as clk:
             torch.cuda.synchronize()
+            clk.mark("start")
             e0.record(stream)
             for _ in range(args.steps):
                 graph.replay()
             e1.record(stream)
             e1.synchronize()
             torch.cuda.synchronize()
+            clk.mark("end")
         barrier()
     ms = reduce_max(e0.elapsed_time(e1), dist, dev)
     ms_step = ms / args.steps
@@ -703,7 +727,7 @@ def _evict_setup(B, T, dev):
 
 
 def evict_bench(args):
-    """The window-vote evictor (Sec. 3.3) at the long-context 14B shape: one
+    """The window-vote evictor (Sec. 3.4) at the long-context 14B shape: one
     int4 g32 anchor, B=4, 8 KV / 40 q heads, d_h 128, 131072 cached
     positions, a 32-query window, budget T/8.  Each call scores the window
     against the whole cache, merges the softmax statistics, votes and selects;
@@ -724,11 +748,13 @@ def evict_bench(args):
           for _ in range(args.steps)]
     with Clocks(0) as clk:
         torch.cuda.synchronize()
+        clk.mark("start")
         for s, e in ev:
             s.record(stream)
             c.evict_window(0, q, w.sigma, budget)
             e.record(stream)
         torch.cuda.synchronize()
+        clk.mark("end")
     ms = [s.elapsed_time(e) for s, e in ev]
     assert c.device_error() == 0
     clocks = clk.summary()
@@ -818,11 +844,13 @@ def prefill_bench(args):
           for _ in range(args.steps)]
     with Clocks(0) as clk:
         torch.cuda.synchronize()
+        clk.mark("start")
         for s0, e0 in ev:
             s0.record(stream)
             c.prefill(0, q, w.sigma, out=out)
             e0.record(stream)
         torch.cuda.synchronize()
+        clk.mark("end")
     ms = [s0.elapsed_time(e0) for s0, e0 in ev]
     assert c.device_error() == 0
     flops = prefill_flops([T] * B, PREFILL_CHUNK, w.n_q_heads, w.head_dim)

@@ -54,7 +54,9 @@ typedef enum {
   KVK_ERR_INVALID_ARG = 1,     /* null pointer, bad size, misaligned buffer  */
   KVK_ERR_INVALID_CONFIG = 2,  /* plan rejected (e.g. layer 0 inherits)      */
   KVK_ERR_INHERITED_LAYER = 3, /* write to a layer that owns no cache        */
-  KVK_ERR_CAPACITY = 4,        /* append would pass max_ctx                  */
+  KVK_ERR_CAPACITY = 4,        /* append would pass max_ctx, or a noalloc
+                                  decode needs more partials than its fixed
+                                  buffer holds                               */
   KVK_ERR_UNSUPPORTED = 5,     /* valid request this library does not handle */
   KVK_ERR_CUDA = 6,            /* a CUDA runtime call failed                 */
   KVK_ERR_DEVICE = 7           /* the device error word was set              */
@@ -104,7 +106,7 @@ typedef struct {
  *    two bits), x = code * s; `group` is ignored and both axes must be
  *    KVK_AXIS_TOKEN.  This library: GQA, head_dim 128, bits 8, 4 or 2.
  * evict_capacity > 0 reserves a kept-position list of that length per
- * sequence (eviction composed with compression, Sec. 3.3). */
+ * sequence (eviction composed with compression, Sec. 3.4). */
 typedef struct {
   int32_t inherit;
   int32_t bits;
@@ -185,7 +187,7 @@ kvk_status kvk_rewind(kvk_cache *cache, int32_t n, kvk_stream stream);
  * on the anchor's lengths and on the SM count). */
 kvk_status kvk_decode_plan_splits(kvk_cache *cache, int32_t layer, int32_t *n_splits);
 
-/* Install the kept-position list of anchor `layer` (eviction, Sec. 3.3):
+/* Install the kept-position list of anchor `layer` (eviction, Sec. 3.4):
  * idx device int32 [B, evict_capacity] sorted ascending, n_kept device
  * int32[B] <= evict_capacity.  Decode then reads only those positions; an
  * entry past the sequence length sets KVK_DEVERR_KEPT_RANGE and is skipped.
@@ -195,7 +197,7 @@ kvk_status kvk_decode_plan_splits(kvk_cache *cache, int32_t layer, int32_t *n_sp
 kvk_status kvk_set_kept(kvk_cache *cache, int32_t layer, const int32_t *idx,
                         const int32_t *n_kept, kvk_stream stream);
 
-/* Attention-scored eviction composed with the compressed cache (Sec. 3.3;
+/* Attention-scored eviction composed with the compressed cache (Sec. 3.4;
  * the paper's evictors sum attention over a 32-query observation window).
  * For every sequence b and KV head j of anchor `layer`, each position t
  * before the last n_win gets the attention mass that the window's queries of
@@ -228,7 +230,7 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
                             size_t scratch_bytes, kvk_stream stream);
 
 /* Causal chunk attention (pre-fill) of `layer` over its compressed cache
- * (Sec. 5 times pre-fill over compressed caches): the chunk is the last n_q
+ * (Sec. 4 times pre-fill over compressed caches): the chunk is the last n_q
  * positions of every sequence, already written with kvk_append; query i of
  * sequence b sits at position len_b - n_q + i and attends to positions
  * 0 .. len_b - n_q + i of the dequantised stored keys and values (the ones
@@ -302,9 +304,15 @@ kvk_status kvk_decode_partial(kvk_cache *cache, int32_t layer, const void *q,
  *    partials go to one fixed buffer of 16 MiB (4,194,304 floats) compiled
  *    into the library; every GPU that loads the library holds that buffer
  *    until the process exits.
- *  - A call needing more than n_splits * max_batch * n_q_heads *
- *    (head_dim + 2) <= 4,194,304 floats returns KVK_ERR_CAPACITY and
- *    enqueues nothing; pass fewer splits or use kvk_decode_attention.
+ *  - The partials take S * max_batch * n_q_heads * (head_dim + 2) floats,
+ *    where S is the split count the call actually uses: n_splits, or the
+ *    automatic count when n_splits is 0, in either case capped at the number
+ *    of 64-position tiles of the context; a call that resolves to one split
+ *    writes its output directly and needs no partials.  A call needing more
+ *    than 4,194,304 floats returns KVK_ERR_CAPACITY and enqueues nothing;
+ *    pass fewer splits or use kvk_decode_attention.
+ *  - The cache's device must be the current device (the buffer is per
+ *    device); otherwise KVK_ERR_INVALID_ARG and nothing is enqueued.
  *  - All calls on a device share the buffer, and it keeps the last call's
  *    contents.  Each call writes every partial it later reads, so nothing
  *    needs clearing, but calls that overlap on the GPU (different streams,
@@ -362,7 +370,8 @@ kvk_status kvk_export_layer(const kvk_cache *cache, int32_t layer, void *k_out, 
                             void *k_residual, kvk_stream stream);
 
 /* Synchronise `stream`, read the device error word into *code and clear it.
- * Returns KVK_ERR_DEVICE if the word was non-zero. */
+ * Returns KVK_ERR_DEVICE if the word was non-zero.  After a
+ * KVK_DEVERR_TIMEOUT the outputs of the affected calls are unspecified. */
 kvk_status kvk_get_device_error(kvk_cache *cache, kvk_stream stream, int32_t *code);
 
 const char *kvk_status_string(kvk_status s);

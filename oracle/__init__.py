@@ -15,7 +15,7 @@ quant      grouped asymmetric quantiser (fp32 op sequence), dequantisation
 attention  layer -> source resolution (Sec. 2.1, depth axis), GQA decode and causal chunk (prefill) attention
            attention over dequantised caches, kept-position gather, MLA
            decode in the unabsorbed form (Appendix C.2).
-evict      the attention-scored evictor composed with the cache (Sec. 3.3):
+evict      the attention-scored evictor composed with the cache (Sec. 3.4):
            votes summed over an observation window of queries, top
            positions per (sequence, KV head), kept lists.
 cost       eq. (cost), eq. (compression), eq. (action space), eq. (range) and

@@ -9,14 +9,14 @@ Everything here runs in float64 on already-dequantised caches.
   query head: query head ``h`` reads KV head ``h // G`` (contiguous groups of
   ``G = H_q / H_kv``), scores ``s_t = sigma * <q_h, k_t>``, softmax over the
   positions the layer reads, output ``sum_t p_t v_t``.  With a kept-position
-  list (eviction composed with compression, Sec. 3.3) only the listed
+  list (eviction composed with compression, Sec. 3.4) only the listed
   positions are read.
 * ``gqa_prefill`` -- attention of a chunk of new queries over the
   compressed cache: the chunk is the last ``C`` positions of each sequence
   (already written to the cache), and query ``i`` at position
   ``len - C + i`` attends causally to positions ``0 .. len - C + i`` of the
   dequantised cache (the other side of the step the paper times as
-  pre-fill, Sec. 5: the cache holds the compressed keys and values the
+  pre-fill, Sec. 4: the cache holds the compressed keys and values the
   decode steps then read).  Queries before position 0 give zeros.
 * ``mla_decode_unabsorbed`` -- Appendix C.2: the MLA cache holds the latent
   ``c`` truncated to its first ``d`` coordinates and the post-RoPE positional

@@ -1,7 +1,7 @@
 """Oracle of the attention-scored evictor (test infrastructure; see
 ``oracle/__init__.py``).
 
-Sec. 3.3 composes token eviction with the cache plan: an evictor runs on
+Sec. 3.4 composes token eviction with the cache plan: an evictor runs on
 the same (compressed) cache and the reduction factors multiply.  The
 evictors the paper runs (SnapKV and its relatives, Appendix "Eviction
 implementations") score positions by summing attention over a 32-query

@@ -4,7 +4,7 @@ Grouped asymmetric quantiser
 ----------------------------
 Appendix C.3 of the paper describes it in one sentence: a scale and a zero
 point per group of ``g`` elements, using all ``2^b`` levels (the KIVI / MLX
-grouped scheme it benchmarks in Sec. 5).  The paper gives no formula, so the
+grouped scheme it benchmarks in Sec. 4).  The paper gives no formula, so the
 reading used here (and by the CUDA path) is the usual one:
 
     mn    = min(x)            zero  = mn

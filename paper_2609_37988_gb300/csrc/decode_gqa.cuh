@@ -3,7 +3,7 @@
 // Computes, for every query head h of sequence b (Sec. 2.1 GQA; the depth
 // axis only changes which anchor is read):
 //     out[b,h] = sum_t softmax_t(sigma <q[b,h], k_t>) v_t ,  k_t/v_t of KV head h/G
-// over the positions of b (or its kept list, Sec. 3.3), with k_t and v_t
+// over the positions of b (or its kept list, Sec. 3.4), with k_t and v_t
 // dequantised on the fly (grouped asymmetric codes, Appendix C.3).
 //
 // Grid (split, kv head, batch); 4 warps per CTA; each CTA streams its
@@ -368,15 +368,33 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     if (use_cp) cp_async_commit();
   }
 
-  for (int e = tid; e < 8 * D; e += 128) {
-    const int h = e / D, ch = e % D;
-    float x = 0.f;
+  // the query rows: eight consecutive channels per thread, read with 16-byte
+  // loads issued together (one memory round trip); heads past G are zero
+  if (tid * 8 < 8 * D) {
+    const int h = (tid * 8) / D, ch = (tid * 8) % D;
+    float x[8];
     if (h < a.G) {
       const size_t qi = ((size_t)b * a.Hq + (size_t)kvh * a.G + h) * D + ch;
-      x = a.q_f32 ? static_cast<const float *>(a.q)[qi]
-                  : bf16_to_f32(static_cast<const uint16_t *>(a.q)[qi]);
+      if (a.q_f32) {
+        const float4 *qp = reinterpret_cast<const float4 *>(static_cast<const float *>(a.q) + qi);
+        const float4 x0 = qp[0], x1 = qp[1];
+        x[0] = x0.x; x[1] = x0.y; x[2] = x0.z; x[3] = x0.w;
+        x[4] = x1.x; x[5] = x1.y; x[6] = x1.z; x[7] = x1.w;
+      } else {
+        const uint4 w = *reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(a.q) + qi);
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          x[2 * i] = __uint_as_float(ws[i] << 16);
+          x[2 * i + 1] = __uint_as_float(ws[i] & 0xffff0000u);
+        }
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) x[i] = 0.f;
     }
-    q_s[h * QSTR + ch] = x;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) q_s[h * QSTR + ch + i] = x[i];
   }
   __syncthreads();
   // per-token key groups: query sums Qs of every (head, channel group), of
@@ -917,37 +935,67 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   // ---- copy ring over the split's tiles -----------------------------------
   bool timed_out = false;
   int t_stop = n_tiles;  // first tile not consumed
-  for (int t = 0; t < n_tiles; ++t) {
+  // Bulk-copy ring (quantised, contiguous, per-token keys): the stage that
+  // tile t - 1 used is refilled as soon as every warp has finished it,
+  // before tile t is awaited, so NST copies are in flight during each wait.
+  // The barrier at the top of an iteration both frees that stage and lets
+  // all threads agree whether a wait of the previous iteration gave up
+  // (a warp whose wait gave up skips that tile's arithmetic).
+  constexpr bool kEarly = C::TMA && !gather && !C::KPC;
+  if constexpr (kEarly) {
     bool ok = true;
-    if (use_cp)
-      cp_async_wait<C::NST - 2>();
-    else
-      ok = mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22);
-    // every thread has finished tile t-1, and all agree whether a wait gave up
-    if (__syncthreads_or(!ok)) {
+    int t_fail = -1;
+    for (int t = 0; t < n_tiles; ++t) {
+      if (__syncthreads_or(!ok)) {
+        t_fail = t - 1;
+        break;
+      }
+      const int nt = t + C::NST - 1;
+      if (nt < n_tiles) issue(nt, nt % C::NST);
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22));
+      if (ok) compute(t, t % C::NST);
+    }
+    if (t_fail < 0 && __syncthreads_or(!ok)) t_fail = n_tiles - 1;
+    if (t_fail >= 0) {
       timed_out = true;
-      t_stop = t;
       if (tid == 0) set_err(a.err, 8);
-      break;
-    }
-    const int nt = t + C::NST - 1;
-    if (nt < n_tiles) issue(nt, nt % C::NST);
-    if (use_cp) cp_async_commit();
-    if constexpr (C::KPC) {
-      fold_query(t % C::NST);
-      __syncthreads();
-    }
-    compute(t, t % C::NST);
-  }
-  if (!use_cp) {
-    if (timed_out) {
-      // let copies still in flight land (bounded) before the CTA leaves:
-      // tiles t_stop .. t_stop + NST - 2 were issued and not consumed
-      const int t_end = min(n_tiles, t_stop + C::NST - 1);
-      for (int u = t_stop; u < t_end; ++u) mbar_wait(&bars[u % C::NST], (u / C::NST) & 1, 1u << 20);
+      // tiles t_fail .. t_fail + NST - 1 were issued: let them land (bounded)
+      const int t_end = min(n_tiles, t_fail + C::NST);
+      for (int u = t_fail; u < t_end; ++u) mbar_wait(&bars[u % C::NST], (u / C::NST) & 1, 1u << 20);
     }
   } else {
-    cp_async_wait<0>();
+    for (int t = 0; t < n_tiles; ++t) {
+      bool ok = true;
+      if (use_cp)
+        cp_async_wait<C::NST - 2>();
+      else
+        ok = mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22);
+      // every thread has finished tile t-1, and all agree whether a wait gave up
+      if (__syncthreads_or(!ok)) {
+        timed_out = true;
+        t_stop = t;
+        if (tid == 0) set_err(a.err, 8);
+        break;
+      }
+      const int nt = t + C::NST - 1;
+      if (nt < n_tiles) issue(nt, nt % C::NST);
+      if (use_cp) cp_async_commit();
+      if constexpr (C::KPC) {
+        fold_query(t % C::NST);
+        __syncthreads();
+      }
+      compute(t, t % C::NST);
+    }
+    if (!use_cp) {
+      if (timed_out) {
+        // let copies still in flight land (bounded) before the CTA leaves:
+        // tiles t_stop .. t_stop + NST - 2 were issued and not consumed
+        const int t_end = min(n_tiles, t_stop + C::NST - 1);
+        for (int u = t_stop; u < t_end; ++u) mbar_wait(&bars[u % C::NST], (u / C::NST) & 1, 1u << 20);
+      }
+    } else {
+      cp_async_wait<0>();
+    }
   }
   __syncthreads();
 

@@ -1,5 +1,5 @@
 // evict.cu -- window-vote eviction composed with a compressed GQA cache
-// (Sec. 3.3: an evictor runs on the same cache and the reduction factors
+// (Sec. 3.4: an evictor runs on the same cache and the reduction factors
 // multiply; the evictors sum attention over an observation window of the
 // last queries, Appendix "Eviction implementations").
 //

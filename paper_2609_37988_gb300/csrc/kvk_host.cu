@@ -788,6 +788,20 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
 // Records a failed CUDA call as the thread's last error (for noalloc.cu).
 kvk_status kvk_internal_cuda_error(cudaError_t e, const char *what) { return cuda_fail(e, what); }
 
+// INVALID_ARG unless the calling thread's current device is the one the cache
+// was created on (for noalloc.cu, whose fixed buffer is per device).
+kvk_status kvk_internal_check_current_device(const kvk_cache *c) {
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
+  int dev = -1;
+  const cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "querying the current device");
+  if (dev != c->device)
+    return fail(KVK_ERR_INVALID_ARG,
+                "current device %d is not the cache's device %d: make the cache's device current",
+                dev, c->device);
+  return KVK_OK;
+}
+
 // Decode with the split-K partials in device memory the caller of this
 // function chose (`partial`, `partial_floats` floats) instead of the cache's
 // workspace.  Rejects a call whose partials would not fit.  Used by the

@@ -10,9 +10,12 @@
 //     out   = W_UV[h][:, :d] o_lat                          (up-projection)
 // All heads of a sequence share the latent, so every cache byte is read once
 // for all H heads and both contractions are dense enough for the tensor
-// cores (mma.m16n8k16, bf16 operands, fp32 accumulate).  fp32 operands that
-// must enter a bf16 MMA (q_lat, softmax weights, o_lat) are split into
-// hi + lo bf16 halves, so products keep ~16 significant bits.
+// cores: the latent decode issues tcgen05.mma (operands staged by TMA tensor
+// copies in shared memory, accumulators in TMEM); the small absorb and the
+// merge + up-projection use mma.m16n8k16.  bf16 operands, fp32 accumulate;
+// fp32 operands that must enter a bf16 product (q_lat, softmax weights,
+// o_lat) are split into hi + lo bf16 halves, so products keep ~16
+// significant bits.
 #include <math.h>
 
 #include <algorithm>

@@ -22,6 +22,7 @@
 
 // host side of this library (kvk_host.cu)
 kvk_status kvk_internal_cuda_error(cudaError_t e, const char *what);
+kvk_status kvk_internal_check_current_device(const kvk_cache *c);
 kvk_status kvk_internal_decode_with_partials(kvk_cache *c, int32_t layer, const void *q,
                                              int32_t q_dtype, float scale, float *out,
                                              int32_t n_splits, float *partial,
@@ -61,6 +62,10 @@ extern "C" kvk_status kvk_decode_attention_noalloc(kvk_cache *cache, int32_t lay
                                                    const void *q, int32_t q_dtype,
                                                    float softmax_scale, float *out,
                                                    int32_t n_splits, kvk_stream stream) {
+  // The buffer looked up below belongs to the current device; the cache's
+  // arenas to the device it was created on.  Refuse a mismatch up front.
+  const kvk_status ds = kvk_internal_check_current_device(cache);
+  if (ds != KVK_OK) return ds;
   float *scratch = nullptr;
   const cudaError_t e = scratch_for_current_device(&scratch);
   if (e != cudaSuccess) return kvk_internal_cuda_error(e, "looking up the fixed scratch buffer");

@@ -1,7 +1,7 @@
 // prefill.cu -- causal chunk attention over a compressed GQA cache
 // (head_dim 128) on the tensor cores: the queries of each sequence's last n_q
 // positions attend to the dequantised cache up to their own position (the
-// pre-fill the paper times over compressed caches, Sec. 5; the chunk's keys
+// pre-fill the paper times over compressed caches, Sec. 4; the chunk's keys
 // and values are written with kvk_append first, so the chunk reads the same
 // stored keys and values the decode steps then read).
 //

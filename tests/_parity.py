@@ -7,6 +7,8 @@ oracle.
 """
 from __future__ import annotations
 
+import os
+
 import numpy as np
 import torch
 
@@ -27,6 +29,10 @@ def assert_close(got, ref, max_abs=MAX_ABS, rel_l2=REL_L2, what=""):
     err = np.abs(got - ref).max() if got.size else 0.0
     den = np.linalg.norm(ref)
     rel = np.linalg.norm(got - ref) / den if den > 0 else np.linalg.norm(got)
+    log = os.environ.get("KVK_PARITY_LOG")
+    if log:  # optional record of every comparison's errors (one line each)
+        with open(log, "a") as f:
+            f.write(f"{what}\t{err:.3e}\t{rel:.3e}\n")
     assert err <= max_abs and rel <= rel_l2, f"{what}: max-abs {err:.3e}, rel-L2 {rel:.3e}"
     return err, rel
 

@@ -91,14 +91,35 @@ def test_mla_workload_reduced():
         assert_close(f32(out), ref, what=f"mla layer {l} d={d}")
 
 
+def _one_anchor_of_each_kind(w):
+    """The workload cut to the first anchor of each storage kind (bits,
+    quantiser, key axis), each followed by an inheritor, in layer order; the
+    per-layer input scales follow their anchors."""
+    picked = {}
+    for a in w.anchors:
+        cfg = w.layers[a]
+        picked.setdefault((cfg["bits"], cfg["scheme"], cfg["key_axis"]), a)
+    layers, scale = [], {}
+    for a in sorted(picked.values()):
+        if a in w.kv_scale:
+            scale[len(layers)] = w.kv_scale[a]
+        layers.append(dict(w.layers[a]))
+        layers.append(dict(w.layers[a], inherit=True))
+    w.layers, w.n_layers, w.kv_scale = layers, len(layers), scale
+    return w
+
+
 @pytest.mark.slow
-@pytest.mark.parametrize("n", [2, 3, 5])
-def test_full_size_sampled(n):
-    """Full geometry, first anchors only (memory and time), sampled rows."""
-    w = W.config(n)
-    keep_layers = w.anchors[:2]
-    last = keep_layers[-1]
-    w = W.config(n, n_layers=last + 1 + (1 if last + 1 < w.n_layers and w.layers[last + 1]["inherit"] else 0))
+@pytest.mark.parametrize("n,sym", [(2, None), (3, None), (5, None), (3, 8), (3, 4), (3, 2)],
+                         ids=["cfg2", "cfg3", "cfg5", "cfg3-sym8", "cfg3-sym4", "cfg3-sym2"])
+def test_full_size_sampled(n, sym):
+    """Full geometry (batch, context, heads, the bench's automatic split
+    count), one anchor of every storage kind the workload holds (and an
+    inheritor reading it), sampled sequences against the oracle."""
+    w = _one_anchor_of_each_kind(W.config(n, sym_bits=sym))
+    if sym is not None:  # the bf16 anchors are covered by the cfg3 case
+        w.layers = [a for a in w.layers if a["bits"] != 16]
+        w.n_layers = len(w.layers)
     _run_gqa(w, check_rows=[0, w.batch - 1])
 
 

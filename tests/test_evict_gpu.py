@@ -1,5 +1,5 @@
 """GPU parity of the window-vote evictor composed with the compressed cache
-(Sec. 3.3; Appendix, eviction implementations: votes summed over an
+(Sec. 3.4; Appendix, eviction implementations: votes summed over an
 observation window of queries), through the C ABI.
 
 The votes are compared with the fp64 oracle on the same dequantised keys;
@@ -160,7 +160,7 @@ def test_evict_then_decode_per_head(fmt):
 
 def test_evict_equal_votes_keep_smaller_positions():
     # every key the same: every vote is equal, so the first budget - n_win
-    # positions are kept (Sec. 3.3 reading: ties go to the smaller position)
+    # positions are kept (Sec. 3.4 reading: ties go to the smaller position)
     B, Hkv, G, D = 2, 1, 3, 64
     c = _cache(B, G, Hkv, D, 600, [dict(bits=8, group=64, key_axis="token", evict_capacity=128)])
     k = torch.full((B, 500, Hkv, D), 0.25, dtype=torch.bfloat16, device="cuda")

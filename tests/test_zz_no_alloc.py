@@ -1,9 +1,10 @@
 """kvk_decode_attention_noalloc: the decode entry point for callers that
 cannot provide scratch device memory.  Its split-K partials live in a fixed
-buffer inside the library; these checks call it through the C ABI and
-compare it with kvk_decode_attention on two calls in a row (the second call
-reuses a buffer still holding the first call's partials), and check that a
-request too large for the buffer is refused before anything runs.
+buffer inside the library; these checks call it through the C ABI on two
+calls in a row (the second call reuses a buffer still holding the first
+call's partials) and compare each result with the fp64 oracle on the same
+inputs and with kvk_decode_attention, and check that a request too large for
+the buffer is refused before anything runs.
 
 Kept in a file of its own, collected last."""
 import ctypes
@@ -13,9 +14,13 @@ import numpy as np
 import pytest
 import torch
 
-from _parity import assert_close
+from _parity import assert_close, f32, gqa_expected, oracle_state
 
 pytestmark = pytest.mark.gpu
+
+B, HQ, HKV, D, T = 3, 10, 2, 128, 1500
+LENS = [T, T // 2, 77]
+CFGS = [dict(bits=4, group=32, key_axis="token"), dict(bits=16, group=64, key_axis="token")]
 
 
 def _noalloc(cache, layer, q, scale, out, n_splits):
@@ -28,31 +33,36 @@ def _noalloc(cache, layer, q, scale, out, n_splits):
                                             n_splits, stream)
 
 
-def _cache_with_data(B=3, Hq=10, Hkv=2, D=128, T=1500, seed=0):
+def _cache_with_data(seed=0):
     from paper_2609_37988_gb300.cache import Cache, Layer
-    c = Cache(n_layers=2, n_q_heads=Hq, n_kv_heads=Hkv, head_dim=D, max_batch=B, max_ctx=T,
+    c = Cache(n_layers=2, n_q_heads=HQ, n_kv_heads=HKV, head_dim=D, max_batch=B, max_ctx=T,
               layers=[Layer(bits=4, group=32), Layer(bits=16)], max_splits=64)
     g = torch.Generator().manual_seed(seed)
+    states = []
     for l in range(2):
-        k = torch.randn((B, T, Hkv, D), generator=g).to(torch.bfloat16).cuda()
-        v = torch.randn((B, T, Hkv, D), generator=g).to(torch.bfloat16).cuda()
-        c.append(l, k, v, n_per_seq=torch.tensor([T, T // 2, 77], dtype=torch.int32, device="cuda"))
-    return c
+        k = torch.randn((B, T, HKV, D), generator=g).to(torch.bfloat16)
+        v = torch.randn((B, T, HKV, D), generator=g).to(torch.bfloat16)
+        c.append(l, k.cuda(), v.cuda(), n_per_seq=torch.tensor(LENS, dtype=torch.int32, device="cuda"))
+        states.append(oracle_state(f32(k), f32(v), LENS, CFGS[l]))
+    return c, states
 
 
-def test_matches_decode_on_two_calls_in_a_row():
-    c = _cache_with_data()
-    scale = 1.0 / math.sqrt(128)
+def test_matches_oracle_and_decode_on_two_calls_in_a_row():
+    c, states = _cache_with_data()
+    scale = 1.0 / math.sqrt(D)
     g = torch.Generator().manual_seed(1)
-    calls = [(0, torch.randn((3, 10, 128), generator=g).to(torch.bfloat16), 0),
-             (1, torch.randn((3, 10, 128), generator=g).to(torch.float32), 5)]
+    calls = [(0, torch.randn((B, HQ, D), generator=g).to(torch.bfloat16), 0),
+             (1, torch.randn((B, HQ, D), generator=g).to(torch.float32), 5)]
     for layer, q, ns in calls:
+        expected = gqa_expected(q, states[layer], LENS, scale)
         q = q.cuda()
-        ref = c.decode(layer, q, scale, n_splits=ns)
-        out = torch.full_like(ref, float("nan"))
+        out = torch.full((B, HQ, D), float("nan"), device="cuda")
         assert _noalloc(c, layer, q, scale, out, ns) == 0
         torch.cuda.synchronize()
-        assert_close(out.cpu().numpy(), ref.cpu().numpy(), what=f"noalloc layer {layer}")
+        assert_close(out.cpu().numpy(), expected, what=f"noalloc layer {layer} vs oracle")
+        ref = c.decode(layer, q, scale, n_splits=ns)
+        torch.cuda.synchronize()
+        assert_close(out.cpu().numpy(), ref.cpu().numpy(), what=f"noalloc layer {layer} vs decode")
     assert c.device_error() == 0
 
 
