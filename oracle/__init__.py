@@ -21,7 +21,9 @@ evict      the attention-scored evictor composed with the cache (Sec. 3.4):
 cost       eq. (cost), eq. (compression), eq. (action space), eq. (range) and
            the metadata-inclusive storage accounting of Tab. realized_bits.
 cache      whole-plan reference: builds every anchor's stored state from a
-           per-layer plan and computes every layer's decode output.
+           per-layer plan (GQA anchors, and MLA anchors whose kept latent
+           and positional key are stored as quantised vectors) and computes
+           every layer's decode output.
 
 Parity status: every function here is pinned by a ``-m "not gpu"`` test
 (``tests/test_oracle_*.py``) against closed forms, the paper's printed

@@ -110,3 +110,53 @@ def plan_outputs(owns, states, queries, lens, sigma, kept=None):
         kp = None if kept is None else kept.get(s)
         outs.append(gqa_decode(queries[l], st["k_hat"], st["v_hat"], lens[s], sigma, kp))
     return outs
+
+
+def mla_anchor_state(c, k_r, lens, width, bits, scheme="symmetric"):
+    """Stored and dequantised state of one MLA anchor (all three axes: the
+    latent truncated to its first ``width`` coordinates, Appendix C.2, and
+    stored with a quantiser of Appendix C.3).
+
+    c   : ``[B, T, >= width]`` latents as written (bf16-exact values)
+    k_r : ``[B, T, d_R]`` post-RoPE positional keys
+    Every position stores two vectors, the kept latent ``c[:width]`` and the
+    positional key, each quantised as ONE vector:
+
+    * ``"symmetric"`` (the paper's quantiser, bits 8/4/2): one bf16 scale per
+      vector, signed codes in ``[-q, q]``;
+    * ``"grouped"`` (asymmetric, bits 8/4): one float32 (scale, zero) pair
+      per vector, the group spanning the whole vector.
+
+    ``bits == 16`` stores the bf16 values (no codes).  Returns a dict with
+    ``c_hat`` ``[B, T, width]`` and ``kr_hat`` ``[B, T, d_R]`` (float64,
+    zero past each length) and, when quantised, ``c_codes``, ``c_scale``,
+    ``kr_codes``, ``kr_scale`` (+ ``c_zero``, ``kr_zero`` for the grouped
+    scheme), codes ``[B, T, n]`` and metadata ``[B, T]``.
+    """
+    c = np.asarray(c, np.float32)[:, :, :width]
+    k_r = np.asarray(k_r, np.float32)
+    B, T, _ = c.shape
+    st = {"bits": bits, "scheme": scheme, "width": width}
+    if bits == 16:
+        c_hat, kr_hat = c.astype(np.float64), k_r.astype(np.float64)
+    elif scheme == "symmetric":
+        cc, cs = quant.quantise_symmetric(c, bits)
+        rc, rs = quant.quantise_symmetric(k_r, bits)
+        st.update(c_codes=cc, c_scale=cs, kr_codes=rc, kr_scale=rs)
+        c_hat, kr_hat = quant.dequantise_symmetric(cc, cs), quant.dequantise_symmetric(rc, rs)
+    elif scheme == "grouped":
+        cc, cs, cz = quant.quantise_groups(c, bits)
+        rc, rs, rz = quant.quantise_groups(k_r, bits)
+        st.update(c_codes=cc, c_scale=cs, c_zero=cz, kr_codes=rc, kr_scale=rs, kr_zero=rz)
+        c_hat = quant.dequantise_per_token(cc, cs[..., None], cz[..., None], width)
+        kr_hat = quant.dequantise_per_token(rc, rs[..., None], rz[..., None], k_r.shape[-1])
+    else:
+        raise ValueError(f"unknown quantisation scheme {scheme!r}")
+    c_hat = np.array(c_hat, np.float64)
+    kr_hat = np.array(kr_hat, np.float64)
+    for b in range(B):
+        n = int(lens[b])
+        c_hat[b, n:] = 0.0
+        kr_hat[b, n:] = 0.0
+    st.update(c_hat=c_hat, kr_hat=kr_hat)
+    return st
