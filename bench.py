@@ -71,15 +71,26 @@ def algorithmic_bytes(w, lens_after_append):
     return total, per_layer
 
 
+def mla_position_bytes(w, l):
+    """Stored bytes of one position of MLA layer l: [c[:d] | k^R] in bf16,
+    or their codes plus the two vectors' scales (and zeros)."""
+    a = w.layers[l]
+    n = a["width"] + w.rope_dim
+    if a["bits"] == 16:
+        return 2 * n
+    return n * a["bits"] // 8 + (4 if a.get("scheme") == "symmetric" else 16)
+
+
 def algorithmic_bytes_mla(w, T):
-    """MLA step: every layer reads its latent cache [c[:d] | k^R] (bf16) at
-    length T, the absorbed/up-projection weight slices W_UK[:, :, :d] and
-    W_UV[:, :, :d], its queries, and writes its output."""
+    """MLA step: every layer reads its latent cache [c[:d] | k^R] at length
+    T (bf16, or codes and per-position metadata), the absorbed /
+    up-projection weight slices W_UK[:, :, :d] and W_UV[:, :, :d], its
+    queries, and writes its output."""
     B, H = w.batch, w.n_q_heads
     total, per_layer = 0, []
     for l in range(w.n_layers):
         d = w.layers[l]["width"]
-        cache = B * T * (d + w.rope_dim) * 2
+        cache = B * T * mla_position_bytes(w, l)
         per_layer.append(cache)
         total += cache + 2 * H * w.head_dim * d * 2 + B * H * (w.head_dim + w.rope_dim) * 2 + \
             B * H * w.head_dim * 4
@@ -239,7 +250,8 @@ def cpu_baseline_mla(w, seconds=12.0):
     from oracle import attention as oatt
     from paper_2609_37988_gb300 import workloads as W
 
-    w1 = W.config(4, batch=1)
+    w1 = W.config(4, batch=1, mla_bits=w.layers[0]["bits"] if w.layers[0]["bits"] != 16 else None,
+                  mla_scheme=w.layers[0].get("scheme", "symmetric"))
     T = w1.context
     widths = {}
     for l, a in enumerate(w1.layers):
@@ -250,14 +262,19 @@ def cpu_baseline_mla(w, seconds=12.0):
         cl, kr = W.mla_inputs(w1, l, 0, T)
         wk, wv = W.mla_weights(w1, l)
         qn, qp = W.mla_queries(w1, l)
-        units.append((d, qn.float().numpy(), qp.float().numpy(), cl.float().numpy(),
-                      kr.float().numpy(), wk.float().numpy(), wv.float().numpy()))
+        cl, kr = cl.float().numpy(), kr.float().numpy()
+        if w1.layers[l]["bits"] != 16:  # the oracle's stored state (outside the timed loop)
+            from oracle import cache as ocache
+            st = ocache.mla_anchor_state(cl, kr, [T], d, w1.layers[l]["bits"], w1.layers[l]["scheme"])
+            cl, kr = st["c_hat"], st["kr_hat"]
+        units.append((l, d, qn.float().numpy(), qp.float().numpy(), cl, kr, wk.float().numpy(),
+                      wv.float().numpy()))
     nbytes, n = 0, 0
     t0 = time.perf_counter()
     while True:
-        for d, qn, qp, cl, kr, wk, wv in units:
+        for l, d, qn, qp, cl, kr, wk, wv in units:
             oatt.mla_decode_unabsorbed(qn, qp, cl, kr, wk, wv, d, [T], w1.sigma)
-            nbytes += T * (d + w1.rope_dim) * 2
+            nbytes += T * mla_position_bytes(w1, l)
         n += 1
         if time.perf_counter() - t0 >= seconds:
             break
@@ -274,7 +291,8 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2609_37988_gb300 import workloads as W
-    w = W.config(args.config, sym_bits=args.sym_bits)
+    w = W.config(args.config, sym_bits=args.sym_bits, mla_bits=args.mla_bits,
+                 mla_scheme=args.mla_scheme)
     base = cpu_baseline if w.kind == "gqa" else cpu_baseline_mla
     per = max(2.0, 60.0 / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):
@@ -297,7 +315,9 @@ def run_reference(args):
 # ---------------------------------------------------------------------------
 def _layer_kind(w, l, src):
     if w.kind == "mla":
-        return f"mla_d{w.layers[l]['width']}"
+        a = w.layers[l]
+        q = "" if a["bits"] == 16 else f"_{'sym' if a.get('scheme') == 'symmetric' else 'int'}{a['bits']}"
+        return f"mla_d{a['width']}{q}"
     a = w.layers[src[l]]
     if a["bits"] == 16:
         return "bf16"
@@ -392,6 +412,10 @@ def main():
     ap.add_argument("--impl", default="kvk")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--mla-bits", type=int, choices=[8, 4, 2], default=None,
+                    help="MLA workload (--config 4): store every latent layer quantised at this "
+                         "bit-width (the kept latent and k^R one vector each)")
+    ap.add_argument("--mla-scheme", choices=["symmetric", "grouped"], default="symmetric")
     ap.add_argument("--sym-bits", type=int, choices=[8, 4, 2], default=None,
                     help="store the quantised anchors with the symmetric per-vector "
                          "quantiser at this bit-width")
@@ -436,7 +460,8 @@ def main():
     from paper_2609_37988_gb300 import workloads as W
     from paper_2609_37988_gb300.cache import Cache, Layer
 
-    w = W.config(args.config, sym_bits=args.sym_bits)
+    w = W.config(args.config, sym_bits=args.sym_bits, mla_bits=args.mla_bits,
+                 mla_scheme=args.mla_scheme)
     T = w.context
     src = w.sources()
     new_kv = {}
@@ -658,7 +683,8 @@ def main():
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "us_per_step": ms_step * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": ("bf16" if w.kind == "mla" else
+            "dtype": ("/".join(sorted({_layer_kind(w, l, src) for l in range(w.n_layers)}))
+                      if w.kind == "mla" else
                       "/".join(sorted({_layer_kind(w, a, src) for a in w.anchors}))),
             "data": "synthetic",
             "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "context": T,

@@ -105,6 +105,14 @@ typedef struct {
  *    codes clip(rint(x / s), -q, q) with q = 2^(b-1) - 1 (three levels at
  *    two bits), x = code * s; `group` is ignored and both axes must be
  *    KVK_AXIS_TOKEN.  This library: GQA, head_dim 128, bits 8, 4 or 2.
+ *  MLA layers at 8, 4 or 2 bits (all three axes at once): each position's
+ *    kept latent c[:width] and its positional key k^R are each quantised as
+ *    ONE vector, with one bf16 scale (symmetric; 8/4/2 bits) or one fp32
+ *    (scale, zero) pair (grouped, the group spanning the vector; 8/4 bits);
+ *    `group` and the axes are ignored.  Decode feeds the codes to the
+ *    tensor cores as exact f16 values with the value weights p * s rounded
+ *    to f16 hi + lo, so p * s (p <= 256) must stay below 65504: latent
+ *    scales below 255.
  * evict_capacity > 0 reserves a kept-position list of that length per
  * sequence (eviction composed with compression, Sec. 3.4). */
 typedef struct {
@@ -127,13 +135,13 @@ typedef struct kvk_cache kvk_cache;
  * scheme, a per-channel axis with the symmetric scheme, MLA width not in
  * r/8..r), and UNSUPPORTED for valid plans outside this library (grouped 2-bit
  * codes, per-channel values, head_dim other than 64/128, the symmetric
- * scheme with head_dim 64 or on MLA, per-channel keys with eviction). */
+ * scheme with GQA head_dim 64, per-channel keys with eviction). */
 kvk_status kvk_cache_plan(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
                           size_t *arena_bytes);
 
 /* Device workspace bytes for a cache whose decode calls use at most
  * max_splits context splits.  Holds the device error word, split-K partials,
- * the absorbed MLA query and per-unit merge counters. */
+ * and the absorbed MLA query. */
 kvk_status kvk_workspace_size(const kvk_model_desc *desc, int32_t max_splits,
                               size_t *ws_bytes);
 
@@ -364,6 +372,11 @@ kvk_status kvk_plan_cost(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
  *              k_scale, v_scale float [B, H_kv, T] (the stored bf16 scales,
  *              widened); k_zero, v_zero, k_residual unused.
  *  MLA:        k_out bf16 [B, T, width] latent, v_out bf16 [B, T, rope_dim].
+ *  quantised MLA: k_out, v_out codes [B, T, width] (latent) and
+ *              [B, T, rope_dim] (k^R), one byte each (int8 in [-q, q] for
+ *              the symmetric scheme, uint8 for the grouped one); k_scale,
+ *              k_zero float [B, T] of the latent vectors, v_scale, v_zero of
+ *              the k^R vectors (zeros 0 for the symmetric scheme).
  * Any pointer the format does not use may be NULL. */
 kvk_status kvk_export_layer(const kvk_cache *cache, int32_t layer, void *k_out, void *v_out,
                             float *k_scale, float *k_zero, float *v_scale, float *v_zero,

@@ -263,10 +263,23 @@ class Cache:
         dev = self.device
         res = {}
         if self.kind == "mla":
-            res["c"] = torch.empty((B, T, L.width), dtype=torch.bfloat16, device=dev)
-            res["k_r"] = torch.empty((B, T, d.rope_dim), dtype=torch.bfloat16, device=dev)
-            check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["c"]), _ptr(res["k_r"]),
-                                            None, None, None, None, None, _stream(stream)))
+            if L.bits == 16:
+                res["c"] = torch.empty((B, T, L.width), dtype=torch.bfloat16, device=dev)
+                res["k_r"] = torch.empty((B, T, d.rope_dim), dtype=torch.bfloat16, device=dev)
+                check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["c"]), _ptr(res["k_r"]),
+                                                None, None, None, None, None, _stream(stream)))
+                return res
+            # quantised latents: codes (signed for the symmetric scheme) and
+            # per-position scales (and zeros) of the latent and of k^R
+            ct = torch.int8 if L.scheme == "symmetric" else torch.uint8
+            res["c_codes"] = torch.empty((B, T, L.width), dtype=ct, device=dev)
+            res["kr_codes"] = torch.empty((B, T, d.rope_dim), dtype=ct, device=dev)
+            for k in ("c_scale", "c_zero", "kr_scale", "kr_zero"):
+                res[k] = torch.empty((B, T), dtype=torch.float32, device=dev)
+            check(self.lib.kvk_export_layer(self.handle, layer, _ptr(res["c_codes"]),
+                                            _ptr(res["kr_codes"]), _ptr(res["c_scale"]),
+                                            _ptr(res["c_zero"]), _ptr(res["kr_scale"]),
+                                            _ptr(res["kr_zero"]), None, _stream(stream)))
             return res
         H, D = d.n_kv_heads, d.head_dim
         if L.bits == 16:

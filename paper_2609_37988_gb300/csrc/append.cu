@@ -451,6 +451,94 @@ __global__ void __launch_bounds__(128)
   }
 }
 
+// Quantised MLA append (the layout in layout.h): one warp per (sequence,
+// new position); the kept latent c[:W] and the positional key are each
+// quantised as one vector (symmetric: one bf16 scale; grouped: one fp32
+// scale and zero), codes staged in shared memory and stored chunk by chunk.
+template <int W>
+__global__ void __launch_bounds__(128)
+    mla_append_q(const MlaView v, const uint16_t *c, const uint16_t *kr, int latent, int n_new,
+                 const int32_t *n_per_seq, int32_t *err) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int R = 64, KH = W + R, EC = W / 32, ER = R / 32;
+  __shared__ uint8_t buf[4][KH];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const size_t wid = (size_t)blockIdx.x * 4 + warp;
+  if (wid < (size_t)v.B * n_new) {
+    const int i = (int)(wid % n_new), b = (int)(wid / n_new);
+    const int nb = seq_count(n_per_seq, b, n_new, err);
+    const int t = v.lens[b] + i;
+    bool ok = i < nb;
+    if (ok && t >= v.cap) {
+      if (lane == 0) set_err(err, 2);
+      ok = false;
+    }
+    if (ok) {
+      const uint16_t *cs = c + ((size_t)b * n_new + i) * latent;
+      const uint16_t *ks = kr + ((size_t)b * n_new + i) * R;
+      float xc[EC], xr[ER];
+#pragma unroll
+      for (int e = 0; e < EC; ++e) xc[e] = bf16_to_f32(cs[lane + 32 * e]);
+#pragma unroll
+      for (int e = 0; e < ER; ++e) xr[e] = bf16_to_f32(ks[lane + 32 * e]);
+      uint32_t uc[EC], ur[ER];
+      if (v.scheme == kSchemeSym) {
+        const uint16_t sc = quant_sym_lane<EC>(xc, v.bits, uc);
+        const uint16_t sr = quant_sym_lane<ER>(xr, v.bits, ur);
+        if (lane == 0)
+          reinterpret_cast<uint32_t *>(v.meta)[(size_t)b * v.cap + t] = (uint32_t)sc | ((uint32_t)sr << 16);
+      } else {
+        const int lev = (1 << v.bits) - 1;
+        float sc, zc, sr, zr;
+        quant_lane<EC>(xc, W, lev, uc, sc, zc);
+        quant_lane<ER>(xr, R, lev, ur, sr, zr);
+        if (lane == 0)
+          reinterpret_cast<float4 *>(v.meta)[(size_t)b * v.cap + t] = make_float4(sc, zc, sr, zr);
+      }
+#pragma unroll
+      for (int e = 0; e < EC; ++e) buf[warp][lane + 32 * e] = (uint8_t)uc[e];
+#pragma unroll
+      for (int e = 0; e < ER; ++e) buf[warp][W + lane + 32 * e] = (uint8_t)ur[e];
+      __syncwarp();
+      uint8_t *rec = v.rec + ((size_t)b * v.cap + t) * v.rec_bytes;
+      for (int j = lane; j < KH / 8; j += 32) {
+        const uint8_t *cd = buf[warp] + 8 * j;
+        if (v.bits == 8) {
+          uint2 w;
+          w.x = cd[0] | (cd[1] << 8) | (cd[2] << 16) | ((uint32_t)cd[3] << 24);
+          w.y = cd[4] | (cd[5] << 8) | (cd[6] << 16) | ((uint32_t)cd[7] << 24);
+          reinterpret_cast<uint2 *>(rec)[j] = w;
+        } else if (v.bits == 4) {
+          uint32_t w = 0;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) w |= (uint32_t)cd[k] << mla_q_bit(k, 4);
+          reinterpret_cast<uint32_t *>(rec)[j] = w;
+        } else {
+          uint32_t w = 0;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) w |= (uint32_t)cd[k] << mla_q_bit(k, 2);
+          reinterpret_cast<uint16_t *>(rec)[j] = (uint16_t)w;
+        }
+      }
+    }
+  }
+  __syncthreads();
+  __shared__ int last;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    last = (atomicAdd(v.counter, 1) == (int)gridDim.x - 1);
+  }
+  __syncthreads();
+  if (last) {
+    for (int b = threadIdx.x; b < v.B; b += blockDim.x) {
+      const int nb = seq_count(n_per_seq, b, n_new, nullptr);
+      v.lens[b] = min((long long)v.lens[b] + nb, (long long)v.cap);
+    }
+    if (threadIdx.x == 0) *v.counter = 0;
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, int in_f32,
@@ -487,9 +575,19 @@ cudaError_t launch_mla_append(const MlaView &v, const void *c, const void *kr, i
                               int n_new, const int32_t *n_per_seq, int32_t *err,
                               cudaStream_t st) {
   const size_t rows = (size_t)v.B * n_new;
-  return launch_pdl(mla_append_rows, dim3((unsigned)((rows + 3) / 4)), dim3(128), 0, st, v,
-                    static_cast<const uint16_t *>(c), static_cast<const uint16_t *>(kr), latent,
-                    n_new, n_per_seq, err);
+  const dim3 grid((unsigned)((rows + 3) / 4));
+  const uint16_t *cc = static_cast<const uint16_t *>(c), *kk = static_cast<const uint16_t *>(kr);
+  if (v.bits != 16) {
+    if (v.rope != 64) return cudaErrorInvalidValue;
+    switch (v.width) {
+      case 512: return launch_pdl(mla_append_q<512>, grid, dim3(128), 0, st, v, cc, kk, latent, n_new, n_per_seq, err);
+      case 256: return launch_pdl(mla_append_q<256>, grid, dim3(128), 0, st, v, cc, kk, latent, n_new, n_per_seq, err);
+      case 128: return launch_pdl(mla_append_q<128>, grid, dim3(128), 0, st, v, cc, kk, latent, n_new, n_per_seq, err);
+      case 64: return launch_pdl(mla_append_q<64>, grid, dim3(128), 0, st, v, cc, kk, latent, n_new, n_per_seq, err);
+      default: return cudaErrorInvalidValue;
+    }
+  }
+  return launch_pdl(mla_append_rows, grid, dim3(128), 0, st, v, cc, kk, latent, n_new, n_per_seq, err);
 }
 
 }  // namespace kvk

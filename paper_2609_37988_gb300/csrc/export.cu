@@ -120,6 +120,54 @@ __global__ void mla_export_kernel(const MlaView v, uint16_t *c_out, uint16_t *kr
   }
 }
 
+// Quantised MLA anchor: codes of the latent [B, T, width] and of k^R [B, T,
+// rope] (signed codes for the symmetric scheme, unsigned for the grouped
+// one), one byte each, and the per-position scales (and zeros).
+__global__ void mla_export_q_kernel(const MlaView v, uint8_t *c_out, uint8_t *kr_out,
+                                    float *c_scale, float *c_zero, float *kr_scale, float *kr_zero,
+                                    int max_ctx) {
+  const int KH = v.width + v.rope;
+  const int off = v.scheme == kSchemeSym ? sym_levels(v.bits) : 0;
+  const size_t total = (size_t)v.B * max_ctx * KH;
+  for (size_t id = (size_t)blockIdx.x * blockDim.x + threadIdx.x; id < total;
+       id += (size_t)gridDim.x * blockDim.x) {
+    const int k = (int)(id % KH);
+    const size_t row = id / KH;
+    const int t = (int)(row % max_ctx);
+    const size_t b = row / max_ctx;
+    const size_t pos = b * v.cap + t;
+    const uint8_t *rec = v.rec + pos * v.rec_bytes;
+    uint32_t chunk;
+    if (v.bits == 8) chunk = reinterpret_cast<const uint32_t *>(rec)[(k >> 3) * 2 + ((k & 7) >> 2)] >>
+                             (8 * (k & 3));
+    else if (v.bits == 4) chunk = reinterpret_cast<const uint32_t *>(rec)[k >> 3] >> mla_q_bit(k & 7, 4);
+    else chunk = (uint32_t)reinterpret_cast<const uint16_t *>(rec)[k >> 3] >> mla_q_bit(k & 7, 2);
+    const int u = (int)(chunk & ((1u << v.bits) - 1));
+    const uint8_t code = (uint8_t)(int8_t)(u - off);
+    if (k < v.width) {
+      if (c_out) c_out[row * v.width + k] = code;
+    } else if (kr_out) {
+      kr_out[row * v.rope + (k - v.width)] = code;
+    }
+    if (k == 0) {
+      float sc, zc, sr, zr;
+      if (v.scheme == kSchemeSym) {
+        const uint32_t w = reinterpret_cast<const uint32_t *>(v.meta)[pos];
+        sc = __uint_as_float(w << 16);
+        sr = __uint_as_float(w & 0xffff0000u);
+        zc = zr = 0.f;
+      } else {
+        const float4 m = reinterpret_cast<const float4 *>(v.meta)[pos];
+        sc = m.x; zc = m.y; sr = m.z; zr = m.w;
+      }
+      if (c_scale) c_scale[row] = sc;
+      if (c_zero) c_zero[row] = zc;
+      if (kr_scale) kr_scale[row] = sr;
+      if (kr_zero) kr_zero[row] = zr;
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_gqa_export(const GqaView &v, void *k_out, void *v_out, float *k_scale,
@@ -134,10 +182,16 @@ cudaError_t launch_gqa_export(const GqaView &v, void *k_out, void *v_out, float 
   return cudaGetLastError();
 }
 
-cudaError_t launch_mla_export(const MlaView &v, void *c_out, void *kr_out, int max_ctx,
+cudaError_t launch_mla_export(const MlaView &v, void *c_out, void *kr_out, float *c_scale,
+                              float *c_zero, float *kr_scale, float *kr_zero, int max_ctx,
                               cudaStream_t st) {
-  mla_export_kernel<<<1024, 256, 0, st>>>(v, static_cast<uint16_t *>(c_out),
-                                          static_cast<uint16_t *>(kr_out), max_ctx);
+  if (v.bits != 16)
+    mla_export_q_kernel<<<1024, 256, 0, st>>>(v, static_cast<uint8_t *>(c_out),
+                                              static_cast<uint8_t *>(kr_out), c_scale, c_zero,
+                                              kr_scale, kr_zero, max_ctx);
+  else
+    mla_export_kernel<<<1024, 256, 0, st>>>(v, static_cast<uint16_t *>(c_out),
+                                            static_cast<uint16_t *>(kr_out), max_ctx);
   return cudaGetLastError();
 }
 

@@ -23,11 +23,14 @@ struct GqaView {
 };
 
 struct MlaView {
-  uint8_t *rec;        // [B][cap][(width + rope) bf16]
+  uint8_t *rec;        // [B][cap][(width + rope) bf16], or quantised codes (layout.h)
+  uint8_t *meta;       // quantised: per-position scales (and zeros) plane, else null
   int32_t *lens;
   int32_t *counter;
   int64_t cap;
   int B, width, rope, rec_bytes;
+  int bits;            // 16, or 8 / 4 / 2 for quantised latents
+  int scheme;          // kSchemeGrouped or kSchemeSym (quantised latents)
 };
 
 struct GqaDecodeArgs {
@@ -115,7 +118,8 @@ inline bool evict_uses_tc(int D, int R) { return D == 128 && R >= 1 && R <= 256;
 cudaError_t launch_gqa_export(const GqaView &v, void *k_out, void *v_out, float *k_scale,
                               float *k_zero, float *v_scale, float *v_zero, void *k_resid,
                               int max_ctx, cudaStream_t st);
-cudaError_t launch_mla_export(const MlaView &v, void *c_out, void *kr_out, int max_ctx,
+cudaError_t launch_mla_export(const MlaView &v, void *c_out, void *kr_out, float *c_scale,
+                              float *c_zero, float *kr_scale, float *kr_zero, int max_ctx,
                               cudaStream_t st);
 
 struct MlaDecodeArgs {
@@ -135,9 +139,11 @@ struct MlaDecodeArgs {
   const void *tmap;    // host copy of the anchor's 128-byte tensor map (mla_make_tmap)
 };
 cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st);
+// the same for an anchor of quantised latents (mla_q.cu; one CTA per SM)
+cudaError_t launch_mla_decode_q(const MlaDecodeArgs &a, cudaStream_t st);
 // Encodes the decode kernel's tensor map of an MLA anchor into `out` (128
 // bytes, 64-byte aligned).
 cudaError_t mla_make_tmap(void *out, const MlaView &v);
-int mla_decode_ctas_per_sm(int width);
+int mla_decode_ctas_per_sm(int width, int bits = 16);
 
 }  // namespace kvk

@@ -78,8 +78,11 @@ kvk_status check_layer(const kvk_model_desc *d, const kvk_layer_cfg *c, int l,
   if (d->kind == KVK_KIND_MLA) {
     if (c->bits != 16 && c->bits != 8 && c->bits != 4 && c->bits != 2)
       return fail(KVK_ERR_INVALID_CONFIG, "layer %d: bits %d not in {16, 8, 4, 2}", l, c->bits);
-    if (need_support && c->bits != 16)
-      return fail(KVK_ERR_UNSUPPORTED, "layer %d: quantised MLA latents are not supported", l);
+    // quantised latents: the kept latent and k^R are each one vector
+    // (symmetric: 8/4/2 bits; grouped: 8/4 bits, the group spanning the vector)
+    if (need_support && c->bits == 2 && c->scheme == KVK_QUANT_GROUPED)
+      return fail(KVK_ERR_UNSUPPORTED,
+                  "layer %d: grouped 2-bit latents are not supported (the symmetric scheme has them)", l);
     const int r = d->latent_dim;
     if (c->width != r && c->width != r / 2 && c->width != r / 4 && c->width != r / 8)
       return fail(KVK_ERR_INVALID_CONFIG, "layer %d: width %d not in {r/8, r/4, r/2, r}", l, c->width);
@@ -211,6 +214,9 @@ struct kvk_cache {
     uint8_t *a = arena[l];
     MlaView v;
     v.rec = a + A.rec;
+    v.meta = A.scales >= 0 ? a + A.scales : nullptr;
+    v.bits = cfg[l].bits;
+    v.scheme = layer_scheme(&cfg[l]);
     v.lens = reinterpret_cast<int32_t *>(a + A.lens);
     v.counter = reinterpret_cast<int32_t *>(a + A.counter);
     v.cap = A.cap;
@@ -284,7 +290,7 @@ int auto_splits(kvk_cache *c, int a) {
   const bool mla = c->desc.kind == KVK_KIND_MLA;
   if (!c->ctas[a]) {
     if (mla) {
-      c->ctas[a] = mla_decode_ctas_per_sm(c->cfg[a].width);
+      c->ctas[a] = mla_decode_ctas_per_sm(c->cfg[a].width, c->cfg[a].bits);
     } else {
       const kvk_layer_cfg &L = c->cfg[a];
       c->ctas[a] = gqa_decode_ctas_per_sm(L.bits, c->desc.head_dim, L.bits == 16 ? 0 : L.key_axis,
@@ -402,7 +408,7 @@ kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg
   if (desc->kind == KVK_KIND_MLA) {
     c->tmap.resize(desc->n_layers);
     for (int l = 0; l < desc->n_layers; ++l) {
-      if (cfg[l].inherit) continue;
+      if (cfg[l].inherit || cfg[l].bits != 16) continue;  // quantised tiles use bulk copies
       e = mla_make_tmap(c->tmap[l].bytes, c->mla_view(l));
       if (e != cudaSuccess) {
         delete c;
@@ -920,7 +926,10 @@ kvk_status kvk_plan_cost(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
     if (a.inherit) continue;  // eq. (cost): inheriting costs nothing
     if (mla) {
       bits += (double)(a.width + d.rope_dim) * a.bits;
-      bytes += (double)(a.width + d.rope_dim) * a.bits / 8.0;
+      // codes, plus per position the two vectors' metadata: a bf16 scale
+      // each (symmetric) or an fp32 scale and zero each (grouped)
+      bytes += (double)(a.width + d.rope_dim) * a.bits / 8.0 +
+               (a.bits == 16 ? 0.0 : (a.scheme == KVK_QUANT_SYMMETRIC ? 4.0 : 16.0));
     } else {
       bits += 2.0 * d.n_kv_heads * d.head_dim * a.bits;
       double per;
@@ -964,7 +973,8 @@ kvk_status kvk_export_layer(const kvk_cache *c, int32_t layer, void *k_out, void
     e = launch_gqa_export(c->gqa_view(layer), k_out, v_out, k_scale, k_zero, v_scale, v_zero,
                           k_residual, c->desc.max_ctx, st);
   else
-    e = launch_mla_export(c->mla_view(layer), k_out, v_out, c->desc.max_ctx, st);
+    e = launch_mla_export(c->mla_view(layer), k_out, v_out, k_scale, k_zero, v_scale, v_zero,
+                          c->desc.max_ctx, st);
   if (e != cudaSuccess) return cuda_fail(e, "export launch");
   return KVK_OK;
 }

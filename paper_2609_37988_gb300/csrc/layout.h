@@ -208,6 +208,28 @@ KVK_HD int sym_phys(int lb, int t, int rec_bytes) {
 
 KVK_HD int64_t align256(int64_t x) { return (x + 255) & ~(int64_t)255; }
 
+// ---- quantised MLA latents --------------------------------------------------
+// A position of a quantised MLA anchor stores two vectors, the kept latent
+// c[:width] and the positional key k^R, as unsigned codes (symmetric: code +
+// q; grouped: the code), in one record of (width + rope) * bits / 8 bytes:
+// coordinate k of the concatenation [c[:width] | k^R] in chunk k / 8 of
+// `bits` bytes, within which code k % 8 = 2 p + h sits at
+//   8 bits: byte 2 p + h;
+//   4 bits: bits 4 p + 16 h of the chunk's 32-bit word;
+//   2 bits: bits 2 p + 8 h of the chunk's 16-bit half-word;
+// so that the f16 pair (code 2p, code 2p+1) is one byte permute (8 bits) or
+// one shift and mask (4 and 2 bits) away.  Beside the records, a plane of
+// per-position metadata: symmetric, one 32-bit word (bf16 scale of the
+// latent, bf16 scale of k^R in the high half); grouped, a float4 (latent
+// scale, latent zero, k^R scale, k^R zero).
+KVK_HD int mla_q_rec_bytes(int width, int rope, int bits) { return (width + rope) * bits / 8; }
+KVK_HD int mla_q_meta_bytes(int scheme) { return scheme == kSchemeSym ? 4 : 16; }
+// bit offset of code k (0..7) inside its chunk
+KVK_HD int mla_q_bit(int k, int bits) {
+  const int p = k >> 1, h = k & 1;
+  return bits == 8 ? 8 * (2 * p + h) : bits == 4 ? 4 * p + 16 * h : 2 * p + 8 * h;
+}
+
 // Offsets inside one anchor's arena.
 struct ArenaLayout {
   int64_t lens;      // int32[B]
@@ -241,9 +263,13 @@ KVK_HD ArenaLayout arena_layout(int mla, int B, int Hkv, int max_ctx, int D, int
   A.rec = off;
   A.scales = -1;
   if (mla) {
-    A.rec_bytes = (width + rope) * 2;
+    A.rec_bytes = bits == 16 ? (width + rope) * 2 : mla_q_rec_bytes(width, rope, bits);
     off = align256(off + (int64_t)B * A.cap * A.rec_bytes);
     A.gmeta = A.resid = -1;
+    if (bits != 16) {
+      A.scales = off;  // per-position metadata plane
+      off = align256(off + (int64_t)B * A.cap * mla_q_meta_bytes(scheme));
+    }
   } else if (bits != 16 && scheme == kSchemeSym) {
     A.rec_bytes = sym_rec_bytes(bits, D);
     off = align256(off + (int64_t)B * Hkv * A.cap * A.rec_bytes);

@@ -1,0 +1,629 @@
+// mla_q.cu -- MLA decode over a quantised latent cache: the three axes of a
+// layer's plan together (Sec. 2.1: a kept latent width, codes of 8, 4 or 2
+// bits, and sharing by later layers; Appendix C.2 truncation with the
+// quantisers of Appendix C.3).
+//
+// Each position stores its kept latent c[:W] and its positional key k^R as
+// one quantised vector each: x = s u + z with unsigned codes u and, per
+// vector, a scale s and an offset z (symmetric scheme: z = -q s; grouped
+// scheme: z = the vector's minimum); the decode reads them centred, x =
+// s (u - C0) + (z + C0 s).  A vector's (s, z) are constant over its
+// coordinates, so both products keep the (centred) codes as operands:
+//   score_t  = sigma ( s_t <q_lat, u_t> + z_t sum(q_lat)
+//                    + s^R_t <q_pe, u^R_t> + z^R_t sum(q_pe) )
+//   o_lat    = sum_t p_t (s_t u_t + z_t) / sum_t p_t
+//            = ( sum_t (p_t s_t) u_t + sum_t p_t z_t ) / sum_t p_t .
+// The codes enter the tcgen05 products as exact f16 subnormals (the bit
+// pattern u is the half u 2^-24), the query and the value weights p s as f16
+// hi + lo halves, fp32 accumulation in TMEM; the latent and positional parts
+// of the score accumulate in separate TMEM columns so that each gets its
+// own scale.  The tensor-core work per position equals the bf16 latent
+// decode's (mla.cu): the quantisation only changes the bytes read and adds
+// an expansion of the codes into the operand layout in shared memory.
+#include <math.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "layout.h"
+#include "mla_common.cuh"
+#include "umma.cuh"
+
+namespace kvk {
+namespace {
+
+// Grid (split, sequence); 12 warps:
+//   0-3   softmax and epilogue (TMEM lane = tile position, as in mla.cu);
+//   4, 7  score products of the even and the odd tiles;
+//   5     bulk copies of the raw records and metadata of each tile;
+//   6     value products;
+//   8-11  expansion of a tile's codes into the f16 operand layout.
+// Rings: NR raw stages (codes as stored + metadata), NST operand stages
+// (the f16 tile as (W + 64) / 64 boxes of TR rows x 128 bytes in the 128-byte
+// swizzled K-major layout, plus the tile's per-position (s, z, s^R, z^R)).
+constexpr int kMlaQThreads = 384;
+
+template <int W, int BITS, bool SYM>
+struct MlaQCfg {
+  static constexpr int TR = W == 512 ? 32 : 64;      // positions per tile
+  static constexpr int KH = W + kRope;
+  static constexpr int BOXES = KH / 64;
+  static constexpr int BOX = TR * 128;
+  static constexpr int OSTAGE = BOXES * BOX;          // f16 operand tile
+  static constexpr int NST = 3;
+  static constexpr int REC = KH * BITS / 8;           // stored record bytes
+  static constexpr int MB = SYM ? 4 : 16;             // metadata bytes per position
+  static constexpr int RAW_META = TR * REC;           // offset of the metadata in a raw stage
+  static constexpr int RAW = TR * REC + TR * MB;
+  static constexpr int NR = 2;
+  static constexpr int OMETA = TR * 16;               // float4 (s, z, s^R, z^R) per position
+  static constexpr int QB = 32 * KH * 2;
+  static constexpr int PB = 4 * 1024;
+  static constexpr int OFF_OM = NST * OSTAGE;
+  static constexpr int OFF_RAW = OFF_OM + NST * OMETA;
+  static constexpr int OFF_Q = OFF_RAW + NR * RAW;
+  static constexpr int OFF_P = OFF_Q + QB;
+  static constexpr int OFF_QS = OFF_P + 2 * PB;       // float [2][16] query sums (latent, rope)
+  static constexpr int OFF_RED = OFF_QS + 128;        // float [4][16] maxima, sums, zero sums
+  static constexpr int OFF_BAR = OFF_RED + 3 * 256;
+  // full[NST], sbar[2], pbar[2], obar[NST], dbar[3], rfull[NR], rfree[NR]
+  static constexpr int NBAR = 2 * NST + 7 + 2 * NR;
+  static constexpr int OFF_TB = OFF_BAR + 8 * NBAR;
+  static constexpr int SMEM = OFF_TB + 16 + 1024;
+  static constexpr int MV = W >= 128 ? 128 : 64;
+  static constexpr int MBL = W / MV;                  // value M-blocks
+  static constexpr int OCOLS = 32 * MBL;
+  static constexpr int SCOLS = 128;                   // two buffers of [latent hi|lo, rope hi|lo]
+  static constexpr int TCOLS = 256;
+  static_assert(OCOLS + SCOLS <= TCOLS, "TMEM columns");
+  static_assert(REC % 16 == 0 && RAW_META % 16 == 0 && (TR * MB) % 16 == 0, "bulk copy sizes");
+  static_assert(OSTAGE % 1024 == 0 && OFF_RAW % 16 == 0 && OFF_Q % 16 == 0, "alignment");
+  static_assert(SMEM <= 232448, "shared memory");
+  static_assert(BITS == 8 || BITS == 4 || (BITS == 2 && SYM), "code widths");
+};
+
+// barrier over the four expansion warps (named barrier 3, 128 threads)
+__device__ __forceinline__ void expand_sync() { asm volatile("bar.sync 3, 128;" ::: "memory"); }
+
+// f16 pairs (code 2p, code 2p + 1) * 2^-24 of one stored chunk of 8 codes
+template <int BITS>
+__device__ __forceinline__ uint4 expand_chunk(const uint8_t *src) {
+  if constexpr (BITS == 8) {
+    const uint2 w = *reinterpret_cast<const uint2 *>(src);
+    return make_uint4(__byte_perm(w.x, 0u, 0x4140), __byte_perm(w.x, 0u, 0x4342),
+                      __byte_perm(w.y, 0u, 0x4140), __byte_perm(w.y, 0u, 0x4342));
+  } else if constexpr (BITS == 4) {
+    const uint32_t w = *reinterpret_cast<const uint32_t *>(src);
+    return make_uint4(w & 0x000F000Fu, (w >> 4) & 0x000F000Fu, (w >> 8) & 0x000F000Fu,
+                      (w >> 12) & 0x000F000Fu);
+  } else {
+    const uint32_t x = *reinterpret_cast<const uint16_t *>(src);
+    const uint32_t z = __byte_perm(x, 0u, 0x4140);  // byte 1 to bits 16..23
+    return make_uint4(z & 0x00030003u, (z >> 2) & 0x00030003u, (z >> 4) & 0x00030003u,
+                      (z >> 6) & 0x00030003u);
+  }
+}
+
+template <int W, int BITS, bool SYM>
+__global__ void __launch_bounds__(kMlaQThreads, 1)
+    mla_decode_q_kernel(const MlaView v, const uint16_t *__restrict__ qlat,
+                        const uint16_t *__restrict__ q_pe, int H, float sig, int items_per_split,
+                        int n_splits, float *__restrict__ partial, int32_t *err) {
+  using C = MlaQCfg<W, BITS, SYM>;
+  constexpr int TR = C::TR, KH = C::KH;
+  constexpr float kCodeScale = 16777216.f;  // codes enter the products as u * 2^-24
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t *full = reinterpret_cast<uint64_t *>(sm + C::OFF_BAR);
+  uint64_t *sbar = full + C::NST, *pbar = sbar + 2, *obar = pbar + 2, *dbar = obar + C::NST;
+  uint64_t *rfull = dbar + 3, *rfree = rfull + C::NR;
+  uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + C::OFF_TB);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + C::OFF_TB + 4);
+  float *red = reinterpret_cast<float *>(sm + C::OFF_RED);  // [4 warps][16] maxima
+  float *lsum = red + 4 * kHeads;                           // [4 warps][16] sums
+  float *zsum = lsum + 4 * kHeads;                          // [4 warps][16] value zero terms
+  float *qsum = reinterpret_cast<float *>(sm + C::OFF_QS);  // [latent, rope][16]
+  uint8_t *q_s = sm + C::OFF_Q;
+
+  const int split = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int len = v.lens[b];
+  const int i0 = split * items_per_split;
+  const int i1 = (split == n_splits - 1) ? len : min(i0 + items_per_split, len);
+  const int n_tiles = i1 > i0 ? (i1 - i0 + TR - 1) / TR : 0;
+  const size_t pos0 = (size_t)b * v.cap;  // slab of sequence b
+  constexpr uint32_t kLimit = 1u << 22;
+
+  if (tid == 0) {
+    for (int i = 0; i < C::NBAR; ++i) {
+      // full and pbar: one arrival per expansion / softmax warp; rfree: per
+      // expansion warp; the rest: one arrival (commit, or expect_tx)
+      const bool four = (i < C::NST) || (i >= C::NST + 2 && i < C::NST + 4) ||
+                        (i >= 2 * C::NST + 7 + C::NR);
+      mbar_init(&full[i], four ? 4 : 1);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 4) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tbase)),
+                 "r"(C::TCOLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();  // barriers initialised, TMEM address published
+  tc_fence_after();
+  // Query operand (f16), K-major core layout: row n, coordinate k at
+  // (n/8) SBO + (k/8) 128 + (n%8) 16 + (k%8) 2, SBO = KH/8 128.  Rows 0-15:
+  // [q_lat hi | q_pe hi] of head n; rows 16-31: [q_lat lo | q_pe lo] of head
+  // n - 16.  The latent halves come from the absorb (f16 hi/lo); q_pe (bf16)
+  // is split here.  Warps 0-4 stage it; the second score warp waits for it.
+  if (warp < 5 || warp == 7) {
+    pdl_wait();
+    constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (64 unused) | lo(W)]
+    const uint16_t *qb = qlat + (size_t)b * H * QROW;
+    auto qdst = [&](int n, int c) { return q_s + (n / 8) * (KH / 8 * 128) + c * 128 + (n % 8) * 16; };
+    if (warp < 5) {
+      for (int q = tid; q < 32 * (W / 8); q += 160) {  // latent parts: 16-byte cp.async
+        const int n = q / (W / 8), c = q % (W / 8), h = n & 15;
+        const bool valid = h < H;
+        const uint16_t *src = valid ? qb + (size_t)h * QROW + (n >= 16 ? KH : 0) + 8 * c : qb;
+        cp_async16(qdst(n, c), src, valid);
+      }
+      for (int q = tid; q < 16 * (kRope / 8); q += 160) {  // positional parts: hi and lo rows
+        const int h = q / (kRope / 8), c = q % (kRope / 8);
+        uint4 hi = make_uint4(0, 0, 0, 0), lo = hi;
+        if (h < H) {
+          const uint4 w = *reinterpret_cast<const uint4 *>(q_pe + ((size_t)b * H + h) * kRope + 8 * c);
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+          uint32_t hs[4], ls[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            split2<false>(__uint_as_float(ws[i] << 16), __uint_as_float(ws[i] & 0xffff0000u), hs[i], ls[i]);
+          hi = make_uint4(hs[0], hs[1], hs[2], hs[3]);
+          lo = make_uint4(ls[0], ls[1], ls[2], ls[3]);
+        }
+        *reinterpret_cast<uint4 *>(qdst(h, W / 8 + c)) = hi;
+        *reinterpret_cast<uint4 *>(qdst(16 + h, W / 8 + c)) = lo;
+      }
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    fence_proxy_async();
+    tc_fence_before();
+    asm volatile("bar.sync 2, 192;" ::: "memory");  // warps 0-4 and 7: the query is staged
+    tc_fence_after();
+  }
+  const uint32_t tmem = *tbase;
+  const uint32_t t_o = tmem, t_s = tmem + C::OCOLS;  // O columns, then two S buffers of 64
+  auto ostage = [&](int s) { return sm + s * C::OSTAGE; };
+  auto ometa = [&](int s) { return reinterpret_cast<float4 *>(sm + C::OFF_OM + s * C::OMETA); };
+  auto rawst = [&](int r) { return sm + C::OFF_RAW + r * C::RAW; };
+  auto pbuf = [&](int ps) { return sm + C::OFF_P + ps * C::PB; };
+  bool failed = false;
+
+  if (warp == 5) {
+    // ======================= copy warp ====================================
+    int issued = 0;
+    if (lane == 0) {
+      for (; issued < n_tiles; ++issued) {
+        const int r = issued % C::NR;
+        // the raw stage's previous tile was expanded
+        if (issued >= C::NR &&
+            !mbar_wait_or_abort(&rfree[r], ((issued - C::NR) / C::NR) & 1, kLimit, abort_flag)) {
+          *abort_flag = 1;
+          set_err(err, 8);
+          break;
+        }
+        const int base = i0 + issued * TR, nval = min(TR, i1 - base);
+        // metadata rows rounded up to 16 bytes (within the slab: capacity
+        // and split starts are multiples of 64 positions)
+        const int mbytes = ((nval * C::MB + 15) / 16) * 16;
+        fence_proxy_async();
+        mbar_expect_tx(&rfull[r], nval * C::REC + mbytes);
+        bulk_g2s(rawst(r), v.rec + (pos0 + base) * C::REC, nval * C::REC, &rfull[r]);
+        bulk_g2s(rawst(r) + C::RAW_META, v.meta + (pos0 + base) * C::MB, mbytes, &rfull[r]);
+      }
+      for (int u = max(0, issued - C::NR); u < issued; ++u)
+        mbar_wait(&rfull[u % C::NR], (u / C::NR) & 1, kLimit);
+    }
+    __syncwarp();
+    pdl_trigger();
+  } else if (warp >= 8) {
+    // ======================= expansion warps ==============================
+    // tile t: raw stage t % NR -> operand stage t % NST (free once the
+    // values of tile t - NST were computed); rows past the split's end are
+    // zero, with zero scales
+    const int et = tid - 256;
+    // codes are centred on C0 (symmetric: q, so the operand is the signed
+    // code itself and the offset term vanishes; grouped: the mid code), by an
+    // exact f16 subtraction of subnormals: u - C0 with the offset moved into
+    // z' = z + C0 s, which keeps the fp32 accumulations free of a large
+    // common offset that would cancel at the end
+    constexpr int kC0 = SYM ? (1 << (BITS - 1)) - 1 : 1 << (BITS - 1);
+    constexpr uint32_t kC0Pair = (uint32_t)kC0 * 0x00010001u;
+    for (int t = 0; t < n_tiles; ++t) {
+      const int r = t % C::NR, s = t % C::NST;
+      bool ok = mbar_wait_or_abort(&rfull[r], (t / C::NR) & 1, kLimit, abort_flag);
+      if (ok && t >= C::NST)
+        ok = mbar_wait_or_abort(&obar[s], ((t - C::NST) / C::NST) & 1, kLimit, abort_flag);
+      if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+      const int nval = min(TR, i1 - (i0 + t * TR));
+      const uint8_t *raw = rawst(r);
+      uint8_t *ost = ostage(s);
+      for (int q = et; q < TR * (KH / 8); q += 128) {
+        const int row = q / (KH / 8), c8 = q - row * (KH / 8);
+        uint4 x = make_uint4(0, 0, 0, 0);
+        if (row < nval) {
+          x = expand_chunk<BITS>(raw + row * C::REC + c8 * BITS);
+          x = make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
+                         hsub2_u32(x.w, kC0Pair));
+        }
+        *reinterpret_cast<uint4 *>(ost + (c8 / 8) * C::BOX + row * 128 + 16 * ((c8 % 8) ^ (row % 8))) = x;
+      }
+      for (int row = et; row < TR; row += 128) {
+        float4 m = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (row < nval) {
+          if constexpr (SYM) {
+            // x = s (u - q): centred on q, no offset
+            const uint32_t w = reinterpret_cast<const uint32_t *>(raw + C::RAW_META)[row];
+            m = make_float4(__uint_as_float(w << 16), 0.f, __uint_as_float(w & 0xffff0000u), 0.f);
+          } else {
+            m = reinterpret_cast<const float4 *>(raw + C::RAW_META)[row];
+            m.y = fmaf((float)kC0, m.x, m.y);
+            m.w = fmaf((float)kC0, m.z, m.w);
+          }
+        }
+        ometa(s)[row] = m;
+      }
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&full[s]);
+        mbar_arrive(&rfree[r]);
+      }
+    }
+    if (failed && lane == 0) {
+      *abort_flag = 1;
+      set_err(err, 8);
+    }
+    __syncwarp();
+    pdl_trigger();
+  }
+  else if (warp == 4 || warp == 7) {
+    // ======================= score warps ==================================
+    // as in mla.cu (warp 4 the even tiles, warp 7 the odd ones; a warp waits
+    // for softmax(t-2) before the operand of tile t, whose stage's previous
+    // tile t - 3 is then known to have been expanded); the latent k-steps
+    // accumulate into S columns 0-31, the positional ones into 32-63
+    const int role = warp == 4 ? 0 : 1;
+    constexpr uint32_t ID_S = umma_idesc_f16(64, 32, false, false);
+    for (int t = role; t < n_tiles && !failed; t += 2) {
+      const int s = t % C::NST;
+      bool ok = true;
+      if (t >= 2) ok = mbar_wait_or_abort(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag);
+      if (ok) ok = mbar_wait_or_abort(&full[s], (t / C::NST) & 1, kLimit, abort_flag);
+      if (ok && lane == 0) {
+        tc_fence_after();
+        const uint64_t dc = umma_desc(smem_u32(ostage(s)), 16, 1024, 2);
+        const uint64_t dq = umma_desc(smem_u32(q_s), 128, KH / 8 * 128, 0);
+        const uint32_t S = t_s + 64 * (t & 1);
+#pragma unroll
+        for (int ks = 0; ks < KH / 16; ++ks) {
+          const bool rope = ks >= W / 16;
+          umma_f16(rope ? S + 32 : S, dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
+                   dq + (uint64_t)(ks * 16), ID_S, rope ? ks > W / 16 : ks > 0);
+        }
+        umma_commit(&sbar[t & 1]);
+      }
+      failed = !__all_sync(0xffffffffu, ok);
+    }
+    if (failed && lane == 0) {
+      *abort_flag = 1;
+      set_err(err, 8);
+    }
+    if (lane == 0) {
+      umma_commit(&dbar[2 * role]);
+      mbar_wait(&dbar[2 * role], 0, kLimit);
+    }
+    __syncwarp();
+    pdl_trigger();
+  } else if (warp == 6) {
+    // ======================= value warp ===================================
+    constexpr uint32_t ID_V = umma_idesc_f16(C::MV, 32, true, true);
+    for (int t = 0; t < n_tiles && !failed; ++t) {
+      const bool ok = mbar_wait_or_abort(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
+      if (ok && lane == 0) {  // O^T[:, hi | lo] += U^T [P'_hi | P'_lo]
+        tc_fence_after();
+        const uint64_t da = umma_desc(smem_u32(ostage(t % C::NST)), C::BOX, 1024, 2);
+        const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, 1024, 0);
+#pragma unroll
+        for (int ks = 0; ks < TR / 16; ++ks)
+#pragma unroll
+          for (int mb = 0; mb < C::MBL; ++mb)
+            umma_f16(t_o + 32 * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
+                     dp + (uint64_t)(ks * 16), ID_V, t > 0 || ks > 0);
+        umma_commit(&obar[t % C::NST]);
+      }
+      failed = !__all_sync(0xffffffffu, ok);
+    }
+    if (failed && lane == 0) {
+      *abort_flag = 1;
+      set_err(err, 8);
+    }
+    if (lane == 0) {
+      umma_commit(&dbar[1]);
+      mbar_wait(&dbar[1], 0, kLimit);
+    }
+    __syncwarp();
+    pdl_trigger();
+  } else {
+    // ======================= softmax warps ================================
+    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+    const int prow = 16 * warp + lane;  // this lane's tile position (lanes 0-15)
+    // per-head sums of the query halves as the products use them: thread
+    // (h = tid / 8, j = tid % 8) adds chunks j, j + 8, ... of rows h and 16 + h
+    {
+      const int h = tid >> 3, j = tid & 7;
+      float sl = 0.f, sr = 0.f;
+      for (int c = j; c < KH / 8; c += 8) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          const int n = h + 16 * half;
+          const uint4 w = *reinterpret_cast<const uint4 *>(q_s + (n / 8) * (KH / 8 * 128) + c * 128 + (n % 8) * 16);
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+          float acc = 0.f;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float2 f = unpack2<false>(ws[i]);
+            acc += f.x + f.y;
+          }
+          if (c < W / 8) sl += acc; else sr += acc;
+        }
+      }
+#pragma unroll
+      for (int off = 1; off < 8; off <<= 1) {
+        sl += __shfl_xor_sync(0xffffffffu, sl, off);
+        sr += __shfl_xor_sync(0xffffffffu, sr, off);
+      }
+      if (j == 0) {
+        qsum[h] = sl;
+        qsum[kHeads + h] = sr;
+      }
+      softmax_sync();
+    }
+    float qsl[kHeads], qsr[kHeads];
+#pragma unroll
+    for (int h = 0; h < kHeads; ++h) { qsl[h] = qsum[h]; qsr[h] = qsum[kHeads + h]; }
+    float m_run[kHeads], l_part[kHeads], z_part[kHeads];
+#pragma unroll
+    for (int h = 0; h < kHeads; ++h) { m_run[h] = -1e30f; l_part[h] = 0.f; z_part[h] = 0.f; }
+    for (int t = 0; t < n_tiles; ++t) {
+      const int base = i0 + t * TR, nval = min(TR, i1 - base);
+      bool ok = mbar_wait_or_abort(&sbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
+      // the tile's scales were written before its operand was published:
+      // acquire them (the phase of tile t is complete, the next cannot be)
+      if (ok) ok = mbar_wait_or_abort(&full[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag);
+      // P buffer (t & 1) was read by values(t-2)
+      if (ok && t >= 2)
+        ok = mbar_wait_or_abort(&obar[(t - 2) % C::NST], ((t - 2) / C::NST) & 1, kLimit, abort_flag);
+      if (softmax_sync_or(!ok)) { failed = true; break; }
+      tc_fence_after();
+      const bool live = lane < 16 && prow < nval;
+      const float4 md = live ? ometa(t % C::NST)[prow] : make_float4(0.f, 0.f, 0.f, 0.f);
+      float x[kHeads];
+      {
+        const uint32_t S = t_s + 64 * (t & 1);
+        float lo[16], rh[16], rl[16];
+        tmem_ld16(S + lane_off, x);
+        tmem_ld16(S + 16 + lane_off, lo);
+        tmem_ld16(S + 32 + lane_off, rh);
+        tmem_ld16(S + 48 + lane_off, rl);
+        const float scl = md.x * kCodeScale, scr = md.z * kCodeScale;
+#pragma unroll
+        for (int h = 0; h < kHeads; ++h)
+          x[h] = live ? fmaf(x[h] + lo[h], scl, fmaf(rh[h] + rl[h], scr, fmaf(md.y, qsl[h], md.w * qsr[h])))
+                      : -INFINITY;
+      }
+      bool need = false;
+#pragma unroll
+      for (int h = 0; h < kHeads; ++h) need |= x[h] * sig > m_run[h] + 8.f;
+      if (softmax_sync_or(need)) {
+#pragma unroll
+        for (int h = 0; h < kHeads; ++h) {
+          float mx = x[h];
+#pragma unroll
+          for (int off = 1; off < 16; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+          if (lane == 0) red[warp * kHeads + h] = mx;
+        }
+        softmax_sync();
+        float alpha[kHeads];
+        bool any = false;
+#pragma unroll
+        for (int h = 0; h < kHeads; ++h) {
+          const float mt =
+              fmaxf(fmaxf(red[h], red[kHeads + h]), fmaxf(red[2 * kHeads + h], red[3 * kHeads + h])) * sig;
+          alpha[h] = 1.f;
+          if (mt > m_run[h] + 8.f) {
+            alpha[h] = fast_exp2(m_run[h] - mt);
+            m_run[h] = mt;
+            any = true;
+          }
+          l_part[h] *= alpha[h];
+          z_part[h] *= alpha[h];
+        }
+        if (t >= 1 && any) {
+          ok = mbar_wait_or_abort(&obar[(t - 1) % C::NST], ((t - 1) / C::NST) & 1, kLimit, abort_flag);
+          if (softmax_sync_or(!ok)) { failed = true; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int mb = 0; mb < C::MBL; ++mb)
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+              float o[16];
+              tmem_ld16(t_o + 32 * mb + 16 * half + lane_off, o);
+#pragma unroll
+              for (int h = 0; h < 16; ++h) o[h] *= alpha[h];
+              tmem_st16(t_o + 32 * mb + 16 * half + lane_off, o);
+            }
+        }
+        softmax_sync();
+      }
+      // value weights P' = p s (the latent scale of the position) as f16 hi
+      // + lo into the MN-major P operand: position k, column n (0-15 hi,
+      // 16-31 lo) at (k/8) 128 + (n/8) 1024 + (k%8) 16 + (n%8) 2
+      if (lane < 16 && prow < TR) {
+        uint32_t hw[8], lw[8];
+#pragma unroll
+        for (int h = 0; h < kHeads; h += 2) {
+          const float p0 = fast_exp2(fmaf(x[h], sig, -m_run[h]));
+          const float p1 = fast_exp2(fmaf(x[h + 1], sig, -m_run[h + 1]));
+          l_part[h] += p0;
+          l_part[h + 1] += p1;
+          z_part[h] = fmaf(p0, md.y, z_part[h]);
+          z_part[h + 1] = fmaf(p1, md.y, z_part[h + 1]);
+          split2<false>(p0 * md.x, p1 * md.x, hw[h / 2], lw[h / 2]);
+        }
+        uint8_t *pp = pbuf(t & 1) + (prow / 8) * 128 + (prow % 8) * 16;
+        *reinterpret_cast<uint4 *>(pp) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *reinterpret_cast<uint4 *>(pp + 1024) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+        *reinterpret_cast<uint4 *>(pp + 2048) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        *reinterpret_cast<uint4 *>(pp + 3072) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&pbar[t & 1]);
+    }
+    pdl_trigger();
+    // ---- partial of this split: o_lat rows, m, l ----------------------------
+    if (!failed && n_tiles > 0) {
+      const int t = n_tiles - 1;
+      const bool ok = mbar_wait_or_abort(&obar[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag);
+      failed = softmax_sync_or(!ok);
+    }
+    if (failed && tid == 0) {
+      *abort_flag = 1;
+      set_err(err, 8);
+    }
+    if (!failed) {
+      tc_fence_after();
+      const size_t RS = (size_t)W + 2;
+      const size_t prow_base = ((size_t)split * v.B + b) * H;
+#pragma unroll
+      for (int h = 0; h < kHeads; ++h) {
+        float sum = l_part[h], zs = z_part[h];
+#pragma unroll
+        for (int off = 1; off < 16; off <<= 1) {
+          sum += __shfl_xor_sync(0xffffffffu, sum, off);
+          zs += __shfl_xor_sync(0xffffffffu, zs, off);
+        }
+        if (lane == 0) {
+          lsum[warp * kHeads + h] = sum;
+          zsum[warp * kHeads + h] = zs;
+        }
+      }
+      softmax_sync();
+      float zt[kHeads];
+#pragma unroll
+      for (int h = 0; h < kHeads; ++h)
+        zt[h] = zsum[h] + zsum[kHeads + h] + zsum[2 * kHeads + h] + zsum[3 * kHeads + h];
+#pragma unroll
+      for (int mb = 0; mb < C::MBL; ++mb) {
+        float o[16];
+        if (n_tiles > 0) {
+          float lo[16];
+          tmem_ld16(t_o + 32 * mb + lane_off, o);
+          tmem_ld16(t_o + 32 * mb + 16 + lane_off, lo);
+#pragma unroll
+          for (int h = 0; h < 16; ++h) o[h] = fmaf(o[h] + lo[h], kCodeScale, zt[h]);
+        } else {
+#pragma unroll
+          for (int h = 0; h < 16; ++h) o[h] = 0.f;
+        }
+        const int r = C::MV == 128 ? 128 * mb + 32 * warp + lane : 16 * warp + lane;
+        if (C::MV == 128 || lane < 16) {
+#pragma unroll
+          for (int h = 0; h < kHeads; ++h)
+            if (h < H) partial[(prow_base + h) * RS + r] = o[h];
+        }
+      }
+      if (tid < H) {
+        const float L = lsum[tid] + lsum[kHeads + tid] + lsum[2 * kHeads + tid] + lsum[3 * kHeads + tid];
+        float mh = m_run[0];
+#pragma unroll
+        for (int h = 1; h < kHeads; ++h) mh = (tid == h) ? m_run[h] : mh;
+        float *pr = partial + (prow_base + tid) * RS;
+        pr[W] = (L > 0.f) ? mh : -INFINITY;
+        pr[W + 1] = L;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TCOLS)
+                 : "memory");
+}
+
+template <int W, int BITS, bool SYM>
+cudaError_t launch_mla_q_t(const MlaDecodeArgs &a, cudaStream_t st) {
+  using C = MlaQCfg<W, BITS, SYM>;
+  if (a.n_splits > 64) return cudaErrorInvalidValue;  // merge weights hold 64 splits
+  const int B = a.v.B;
+  auto k = mla_decode_q_kernel<W, BITS, SYM>;
+  constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(mla_merge_upv_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               MU_SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  cudaError_t e = launch_pdl(mla_absorb_kernel<W, true>, dim3(W / 64, a.H, (B + 15) / 16),
+                             dim3(128), 0, st, static_cast<const uint16_t *>(a.q_nope),
+                             static_cast<const uint16_t *>(a.q_pe),
+                             static_cast<const uint16_t *>(a.w_uk), B, a.H, a.r, a.qlat);
+  if (e == cudaSuccess)
+    e = launch_pdl(k, dim3(a.n_splits, B), dim3(kMlaQThreads), C::SMEM, st, a.v,
+                   static_cast<const uint16_t *>(a.qlat), static_cast<const uint16_t *>(a.q_pe),
+                   a.H, a.sig_log2, a.items_per_split, a.n_splits, a.partial, a.err);
+  if (e == cudaSuccess)
+    e = launch_pdl(mla_merge_upv_kernel<W>, dim3(a.H, (B + 15) / 16, 4), dim3(128), MU_SMEM, st,
+                   static_cast<const float *>(a.partial), a.n_splits,
+                   static_cast<const uint16_t *>(a.w_uv), B, a.H, a.r, a.out);
+  return e;
+}
+
+template <int W>
+cudaError_t launch_mla_q_w(const MlaDecodeArgs &a, cudaStream_t st) {
+  const bool sym = a.v.scheme == kSchemeSym;
+  switch (a.v.bits) {
+    case 8: return sym ? launch_mla_q_t<W, 8, true>(a, st) : launch_mla_q_t<W, 8, false>(a, st);
+    case 4: return sym ? launch_mla_q_t<W, 4, true>(a, st) : launch_mla_q_t<W, 4, false>(a, st);
+    case 2: return sym ? launch_mla_q_t<W, 2, true>(a, st) : cudaErrorInvalidValue;
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+// MLA decode over a quantised latent anchor: absorb (f16 halves), the
+// latent decode above, then the merge fused with the up-projection.
+cudaError_t launch_mla_decode_q(const MlaDecodeArgs &a, cudaStream_t st) {
+  if (a.v.rope != kRope || !a.v.meta) return cudaErrorInvalidValue;
+  switch (a.v.width) {
+    case 512: return launch_mla_q_w<512>(a, st);
+    case 256: return launch_mla_q_w<256>(a, st);
+    case 128: return launch_mla_q_w<128>(a, st);
+    case 64: return launch_mla_q_w<64>(a, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace kvk

@@ -78,12 +78,16 @@ def _layer(inherit=False, bits=16, group=64, key_axis="token", width=0, evict_ca
 
 
 def config(n: int, seed: int = None, *, batch: int = None, context: int = None,
-           n_layers: int = None, sym_bits: int = None) -> Workload:
+           n_layers: int = None, sym_bits: int = None, mla_bits: int = None,
+           mla_scheme: str = "symmetric") -> Workload:
     """Workload ``n`` (1..5).  ``batch``/``context``/``n_layers`` shrink it
     for oracle-sized tests while keeping the per-layer draws.  ``sym_bits``
     (8, 4 or 2) stores every quantised anchor with the paper's symmetric
     per-vector quantiser at that bit-width instead (per-token rows; the
-    plan, shapes and inputs are otherwise unchanged)."""
+    plan, shapes and inputs are otherwise unchanged).  ``mla_bits`` (8, 4 or
+    2; MLA workload only) stores every latent layer quantised as well (all
+    three axes), each position's kept latent and positional key one vector
+    each, with ``mla_scheme`` ``"symmetric"`` or ``"grouped"``."""
     seed = n if seed is None else seed
     rng = np.random.default_rng(seed)
     if n == 1:
@@ -140,6 +144,13 @@ def config(n: int, seed: int = None, *, batch: int = None, context: int = None,
             w.name = re.sub(r"int\d", f"sym{sym_bits}", w.name)
         else:
             w.name += f"-sym{sym_bits}"
+    if mla_bits is not None:
+        if mla_bits not in (8, 4, 2) or w.kind != "mla" or mla_scheme not in ("symmetric", "grouped") \
+                or (mla_bits == 2 and mla_scheme == "grouped"):
+            raise ValueError("quantised latents: symmetric 8/4/2 or grouped 8/4 bits on the MLA workload")
+        for a in w.layers:
+            a.update(bits=mla_bits, scheme=mla_scheme)
+        w.name += f"-{'sym' if mla_scheme == 'symmetric' else 'int'}{mla_bits}"
     if batch is not None:
         w.batch = batch
     if n_layers is not None:

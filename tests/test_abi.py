@@ -138,10 +138,14 @@ def test_symmetric_plan_validation(lib):
     # unknown scheme; 3 bits
     assert _plan_status(lib, d, _plan(lib, (0, 4, 32, 0, 0, 0, 0, 2), BF16, BF16, BF16))[0] == 2
     assert _plan_status(lib, d, _plan(lib, _sym(3), BF16, BF16, BF16))[0] == 2
-    # head_dim 64 and MLA latents are outside what the library supports
+    # head_dim 64 is outside what the library supports; MLA latents take
+    # the symmetric 8/4/2-bit and grouped 8/4-bit vectors, not grouped 2-bit
     assert _plan_status(lib, _desc(lib, head_dim=64), _plan(lib, _sym(4), BF16, BF16, BF16))[0] == 5
     m = _desc(lib, kind=1, n_layers=1, n_q_heads=16, head_dim=128, latent_dim=512, rope_dim=64)
-    assert _plan_status(lib, m, _plan(lib, (0, 4, 0, 0, 0, 512, 0, 1)))[0] == 5
+    for bits, scheme in ((8, 1), (4, 1), (2, 1), (8, 0), (4, 0)):
+        ok, sizes = _plan_status(lib, m, _plan(lib, (0, bits, 0, 0, 0, 256, 0, scheme)))
+        assert ok == 0 and sizes[0] > 0
+    assert _plan_status(lib, m, _plan(lib, (0, 2, 0, 0, 0, 256, 0, 0)))[0] == 5
     # grouped 2-bit stays unsupported, and says where 2-bit codes are
     assert _plan_status(lib, d, _plan(lib, BF16, (0, 2, 32, 0, 0, 0, 0, 0), BF16, BF16))[0] == 5
     assert "symmetric" in lib.load().kvk_last_error().decode()
