@@ -23,6 +23,7 @@
 #include <math.h>
 
 #include <algorithm>
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -33,20 +34,45 @@
 namespace kvk {
 namespace {
 
-// Grid (split, sequence); 12 warps:
+// Grid (split, sequence); 16 warps:
 //   0-3   softmax and epilogue (TMEM lane = tile position, as in mla.cu);
 //   4, 7  score products of the even and the odd tiles;
 //   5     bulk copies of the raw records and metadata of each tile;
 //   6     value products;
-//   8-11  expansion of a tile's codes into the f16 operand layout.
+//   8-15  expansion of a tile's codes into the f16 operand layout.
 // Rings: NR raw stages (codes as stored + metadata), NST operand stages
 // (the f16 tile as (W + 64) / 64 boxes of TR rows x 128 bytes in the 128-byte
 // swizzled K-major layout, plus the tile's per-position (s, z, s^R, z^R)).
-constexpr int kMlaQThreads = 384;
+// Tiles of 128 positions (score products M = 128, TMEM lane = position)
+// where three operand stages fit beside at least three raw stages, else 64
+// or 32 (M = 64, lanes 0-15 of each lane quarter); the raw ring takes the
+// rest of the shared memory, up to 8 stages, so that several tiles' bytes
+// are in flight while earlier tiles are expanded and multiplied.
+constexpr int kMlaQThreads = 512;
+constexpr int kExpWarps = 8;                 // warps 8-15
+constexpr int kExpThreads = 32 * kExpWarps;
+constexpr uint32_t kSleepNs = 256;           // suspend hint of the role loops' barrier waits
+constexpr int kMlaQSmemMax = 232448;
+
+template <int W, int BITS, bool SYM>
+struct MlaQTile {
+  static constexpr int KH = W + kRope;
+  static constexpr int REC = KH * BITS / 8;
+  static constexpr int MB = SYM ? 4 : 16;
+  // shared memory of everything but the raw ring, for TR positions and NST stages
+  static constexpr int fixed(int TR, int NST) {
+    return NST * (KH / 64) * TR * 128 + NST * TR * 16 + 32 * KH * 2 + 2 * 4 * (TR * 16 > 1024 ? TR * 16 : 1024) +
+           128 + 768 + 8 * (2 * NST + 7 + 16) + 16 + 1024;
+  }
+  static constexpr int raw(int TR) { return TR * REC + TR * MB; }
+  static constexpr int nr(int TR, int NST) { return (kMlaQSmemMax - fixed(TR, NST)) / raw(TR); }
+  static constexpr int TR = nr(128, 3) >= 3 ? 128 : nr(64, 3) >= 3 ? 64 : 32;
+};
 
 template <int W, int BITS, bool SYM>
 struct MlaQCfg {
-  static constexpr int TR = W == 512 ? 32 : 64;      // positions per tile
+  static constexpr int TR = MlaQTile<W, BITS, SYM>::TR;  // positions per tile
+  static constexpr int SM = TR == 128 ? 128 : 64;       // score product M
   static constexpr int KH = W + kRope;
   static constexpr int BOXES = KH / 64;
   static constexpr int BOX = TR * 128;
@@ -56,10 +82,12 @@ struct MlaQCfg {
   static constexpr int MB = SYM ? 4 : 16;             // metadata bytes per position
   static constexpr int RAW_META = TR * REC;           // offset of the metadata in a raw stage
   static constexpr int RAW = TR * REC + TR * MB;
-  static constexpr int NR = 2;
+  static constexpr int NR_FIT = MlaQTile<W, BITS, SYM>::nr(TR, NST);
+  static constexpr int NR = NR_FIT < 8 ? NR_FIT : 8;
   static constexpr int OMETA = TR * 16;               // float4 (s, z, s^R, z^R) per position
   static constexpr int QB = 32 * KH * 2;
-  static constexpr int PB = 4 * 1024;
+  static constexpr int PNS = TR * 16 > 1024 ? TR * 16 : 1024;  // P: stride of 8-column groups
+  static constexpr int PB = 4 * PNS;
   static constexpr int OFF_OM = NST * OSTAGE;
   static constexpr int OFF_RAW = OFF_OM + NST * OMETA;
   static constexpr int OFF_Q = OFF_RAW + NR * RAW;
@@ -76,30 +104,37 @@ struct MlaQCfg {
   static constexpr int OCOLS = 32 * MBL;
   static constexpr int SCOLS = 128;                   // two buffers of [latent hi|lo, rope hi|lo]
   static constexpr int TCOLS = 256;
+  static_assert(NR >= 2, "raw stages");
   static_assert(OCOLS + SCOLS <= TCOLS, "TMEM columns");
   static_assert(REC % 16 == 0 && RAW_META % 16 == 0 && (TR * MB) % 16 == 0, "bulk copy sizes");
-  static_assert(OSTAGE % 1024 == 0 && OFF_RAW % 16 == 0 && OFF_Q % 16 == 0, "alignment");
-  static_assert(SMEM <= 232448, "shared memory");
+  static_assert(OSTAGE % 1024 == 0 && OFF_RAW % 16 == 0 && OFF_Q % 16 == 0 && OFF_P % 16 == 0, "alignment");
+  static_assert(SMEM <= kMlaQSmemMax, "shared memory");
   static_assert(BITS == 8 || BITS == 4 || (BITS == 2 && SYM), "code widths");
 };
 
-// barrier over the four expansion warps (named barrier 3, 128 threads)
-__device__ __forceinline__ void expand_sync() { asm volatile("bar.sync 3, 128;" ::: "memory"); }
 
-// f16 pairs (code 2p, code 2p + 1) * 2^-24 of one stored chunk of 8 codes
+// The stored bytes of one chunk of 8 codes (BITS bytes) and their f16 pairs
+// (code 2p, code 2p + 1) * 2^-24.
 template <int BITS>
-__device__ __forceinline__ uint4 expand_chunk(const uint8_t *src) {
+struct RawChunk {
+  using T = typename std::conditional<BITS == 8, uint2, uint32_t>::type;
+};
+template <int BITS>
+__device__ __forceinline__ typename RawChunk<BITS>::T load_chunk(const uint8_t *src) {
+  if constexpr (BITS == 8) return *reinterpret_cast<const uint2 *>(src);
+  else if constexpr (BITS == 4) return *reinterpret_cast<const uint32_t *>(src);
+  else return *reinterpret_cast<const uint16_t *>(src);
+}
+template <int BITS>
+__device__ __forceinline__ uint4 expand_chunk(typename RawChunk<BITS>::T w) {
   if constexpr (BITS == 8) {
-    const uint2 w = *reinterpret_cast<const uint2 *>(src);
     return make_uint4(__byte_perm(w.x, 0u, 0x4140), __byte_perm(w.x, 0u, 0x4342),
                       __byte_perm(w.y, 0u, 0x4140), __byte_perm(w.y, 0u, 0x4342));
   } else if constexpr (BITS == 4) {
-    const uint32_t w = *reinterpret_cast<const uint32_t *>(src);
     return make_uint4(w & 0x000F000Fu, (w >> 4) & 0x000F000Fu, (w >> 8) & 0x000F000Fu,
                       (w >> 12) & 0x000F000Fu);
   } else {
-    const uint32_t x = *reinterpret_cast<const uint16_t *>(src);
-    const uint32_t z = __byte_perm(x, 0u, 0x4140);  // byte 1 to bits 16..23
+    const uint32_t z = __byte_perm(w, 0u, 0x4140);  // byte 1 to bits 16..23
     return make_uint4(z & 0x00030003u, (z >> 2) & 0x00030003u, (z >> 4) & 0x00030003u,
                       (z >> 6) & 0x00030003u);
   }
@@ -139,9 +174,9 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     for (int i = 0; i < C::NBAR; ++i) {
       // full and pbar: one arrival per expansion / softmax warp; rfree: per
       // expansion warp; the rest: one arrival (commit, or expect_tx)
-      const bool four = (i < C::NST) || (i >= C::NST + 2 && i < C::NST + 4) ||
-                        (i >= 2 * C::NST + 7 + C::NR);
-      mbar_init(&full[i], four ? 4 : 1);
+      const bool exp = (i < C::NST) || (i >= 2 * C::NST + 7 + C::NR);
+      const bool four = i >= C::NST + 2 && i < C::NST + 4;
+      mbar_init(&full[i], exp ? kExpWarps : four ? 4 : 1);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -205,39 +240,17 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   auto pbuf = [&](int ps) { return sm + C::OFF_P + ps * C::PB; };
   bool failed = false;
 
-  if (warp == 5) {
-    // ======================= copy warp ====================================
-    int issued = 0;
-    if (lane == 0) {
-      for (; issued < n_tiles; ++issued) {
-        const int r = issued % C::NR;
-        // the raw stage's previous tile was expanded
-        if (issued >= C::NR &&
-            !mbar_wait_or_abort(&rfree[r], ((issued - C::NR) / C::NR) & 1, kLimit, abort_flag)) {
-          *abort_flag = 1;
-          set_err(err, 8);
-          break;
-        }
-        const int base = i0 + issued * TR, nval = min(TR, i1 - base);
-        // metadata rows rounded up to 16 bytes (within the slab: capacity
-        // and split starts are multiples of 64 positions)
-        const int mbytes = ((nval * C::MB + 15) / 16) * 16;
-        fence_proxy_async();
-        mbar_expect_tx(&rfull[r], nval * C::REC + mbytes);
-        bulk_g2s(rawst(r), v.rec + (pos0 + base) * C::REC, nval * C::REC, &rfull[r]);
-        bulk_g2s(rawst(r) + C::RAW_META, v.meta + (pos0 + base) * C::MB, mbytes, &rfull[r]);
-      }
-      for (int u = max(0, issued - C::NR); u < issued; ++u)
-        mbar_wait(&rfull[u % C::NR], (u / C::NR) & 1, kLimit);
-    }
-    __syncwarp();
-    pdl_trigger();
-  } else if (warp >= 8) {
+  // Register split over the warpgroups (launched with 128 per thread, 65536
+  // in all): expansion 80 + 80, products and copies 96, softmax 256, in all
+  // (80 + 80 + 96 + 256) x 128 = 65536; each warpgroup's role begins with its
+  // own (the softmax increase waits for the decreases).
+  if (warp >= 8) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 80;\n" ::: "memory");
     // ======================= expansion warps ==============================
     // tile t: raw stage t % NR -> operand stage t % NST (free once the
     // values of tile t - NST were computed); rows past the split's end are
     // zero, with zero scales
-    const int et = tid - 256;
+    const int et = tid - 256;  // 0 .. kExpThreads - 1
     // codes are centred on C0 (symmetric: q, so the operand is the signed
     // code itself and the offset term vanishes; grouped: the mid code), by an
     // exact f16 subtraction of subnormals: u - C0 with the offset moved into
@@ -245,26 +258,54 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     // common offset that would cancel at the end
     constexpr int kC0 = SYM ? (1 << (BITS - 1)) - 1 : 1 << (BITS - 1);
     constexpr uint32_t kC0Pair = (uint32_t)kC0 * 0x00010001u;
+    // chunk q = et + 256 i of a tile (8 codes): row q / (KH / 8), chunk
+    // q % (KH / 8); its raw and operand offsets are the same in every tile
+    // (threads past the last chunk repeat it: the same bytes, written twice)
+    constexpr int kCpr = KH / 8, kJobs = TR * kCpr;
+    constexpr int kPer = (kJobs + kExpThreads - 1) / kExpThreads;
+    uint32_t roff[kPer], soff[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      const int q = min(et + kExpThreads * i, kJobs - 1);
+      const int row = q / kCpr, c8 = q - row * kCpr;
+      roff[i] = row * C::REC + c8 * BITS;
+      soff[i] = (c8 / 8) * C::BOX + row * 128 + 16 * ((c8 % 8) ^ (row % 8));
+    }
     for (int t = 0; t < n_tiles; ++t) {
       const int r = t % C::NR, s = t % C::NST;
-      bool ok = mbar_wait_or_abort(&rfull[r], (t / C::NR) & 1, kLimit, abort_flag);
+      bool ok = mbar_wait_sleepy(&rfull[r], (t / C::NR) & 1, kLimit, abort_flag, kSleepNs);
       if (ok && t >= C::NST)
-        ok = mbar_wait_or_abort(&obar[s], ((t - C::NST) / C::NST) & 1, kLimit, abort_flag);
+        ok = mbar_wait_sleepy(&obar[s], ((t - C::NST) / C::NST) & 1, kLimit, abort_flag, kSleepNs);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       const int nval = min(TR, i1 - (i0 + t * TR));
       const uint8_t *raw = rawst(r);
       uint8_t *ost = ostage(s);
-      for (int q = et; q < TR * (KH / 8); q += 128) {
-        const int row = q / (KH / 8), c8 = q - row * (KH / 8);
-        uint4 x = make_uint4(0, 0, 0, 0);
-        if (row < nval) {
-          x = expand_chunk<BITS>(raw + row * C::REC + c8 * BITS);
-          x = make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
+      if (nval == TR) {
+        // every load before the first use
+        typename RawChunk<BITS>::T w[kPer];
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) w[i] = load_chunk<BITS>(raw + roff[i]);
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) {
+          const uint4 x = expand_chunk<BITS>(w[i]);
+          *reinterpret_cast<uint4 *>(ost + soff[i]) =
+              make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
                          hsub2_u32(x.w, kC0Pair));
         }
-        *reinterpret_cast<uint4 *>(ost + (c8 / 8) * C::BOX + row * 128 + 16 * ((c8 % 8) ^ (row % 8))) = x;
+      } else {
+        // the split's last, partial tile: rows past its end are zero
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) {
+          uint4 x = make_uint4(0, 0, 0, 0);
+          if ((int)(roff[i] / C::REC) < nval) {
+            x = expand_chunk<BITS>(load_chunk<BITS>(raw + roff[i]));
+            x = make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
+                           hsub2_u32(x.w, kC0Pair));
+          }
+          *reinterpret_cast<uint4 *>(ost + soff[i]) = x;
+        }
       }
-      for (int row = et; row < TR; row += 128) {
+      for (int row = et; row < TR; row += kExpThreads) {
         float4 m = make_float4(0.f, 0.f, 0.f, 0.f);
         if (row < nval) {
           if constexpr (SYM) {
@@ -292,78 +333,111 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     }
     __syncwarp();
     pdl_trigger();
-  }
-  else if (warp == 4 || warp == 7) {
-    // ======================= score warps ==================================
-    // as in mla.cu (warp 4 the even tiles, warp 7 the odd ones; a warp waits
-    // for softmax(t-2) before the operand of tile t, whose stage's previous
-    // tile t - 3 is then known to have been expanded); the latent k-steps
-    // accumulate into S columns 0-31, the positional ones into 32-63
-    const int role = warp == 4 ? 0 : 1;
-    constexpr uint32_t ID_S = umma_idesc_f16(64, 32, false, false);
-    for (int t = role; t < n_tiles && !failed; t += 2) {
-      const int s = t % C::NST;
-      bool ok = true;
-      if (t >= 2) ok = mbar_wait_or_abort(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag);
-      if (ok) ok = mbar_wait_or_abort(&full[s], (t / C::NST) & 1, kLimit, abort_flag);
-      if (ok && lane == 0) {
-        tc_fence_after();
-        const uint64_t dc = umma_desc(smem_u32(ostage(s)), 16, 1024, 2);
-        const uint64_t dq = umma_desc(smem_u32(q_s), 128, KH / 8 * 128, 0);
-        const uint32_t S = t_s + 64 * (t & 1);
-#pragma unroll
-        for (int ks = 0; ks < KH / 16; ++ks) {
-          const bool rope = ks >= W / 16;
-          umma_f16(rope ? S + 32 : S, dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
-                   dq + (uint64_t)(ks * 16), ID_S, rope ? ks > W / 16 : ks > 0);
+  } else if (warp >= 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 96;\n" ::: "memory");
+    if (warp == 5) {
+      // ======================= copy warp ====================================
+      int issued = 0;
+      if (lane == 0) {
+        for (; issued < n_tiles; ++issued) {
+          const int r = issued % C::NR;
+          // the raw stage's previous tile was expanded
+          if (issued >= C::NR &&
+              !mbar_wait_sleepy(&rfree[r], ((issued - C::NR) / C::NR) & 1, kLimit, abort_flag, kSleepNs)) {
+            *abort_flag = 1;
+            set_err(err, 8);
+            break;
+          }
+          const int base = i0 + issued * TR, nval = min(TR, i1 - base);
+          // metadata rows rounded up to 16 bytes (within the slab: capacity
+          // and split starts are multiples of 64 positions)
+          const int mbytes = ((nval * C::MB + 15) / 16) * 16;
+          fence_proxy_async();
+          mbar_expect_tx(&rfull[r], nval * C::REC + mbytes);
+          bulk_g2s(rawst(r), v.rec + (pos0 + base) * C::REC, nval * C::REC, &rfull[r]);
+          bulk_g2s(rawst(r) + C::RAW_META, v.meta + (pos0 + base) * C::MB, mbytes, &rfull[r]);
         }
-        umma_commit(&sbar[t & 1]);
+        for (int u = max(0, issued - C::NR); u < issued; ++u)
+          mbar_wait(&rfull[u % C::NR], (u / C::NR) & 1, kLimit);
       }
-      failed = !__all_sync(0xffffffffu, ok);
-    }
-    if (failed && lane == 0) {
-      *abort_flag = 1;
-      set_err(err, 8);
-    }
-    if (lane == 0) {
-      umma_commit(&dbar[2 * role]);
-      mbar_wait(&dbar[2 * role], 0, kLimit);
-    }
-    __syncwarp();
-    pdl_trigger();
-  } else if (warp == 6) {
-    // ======================= value warp ===================================
-    constexpr uint32_t ID_V = umma_idesc_f16(C::MV, 32, true, true);
-    for (int t = 0; t < n_tiles && !failed; ++t) {
-      const bool ok = mbar_wait_or_abort(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
-      if (ok && lane == 0) {  // O^T[:, hi | lo] += U^T [P'_hi | P'_lo]
-        tc_fence_after();
-        const uint64_t da = umma_desc(smem_u32(ostage(t % C::NST)), C::BOX, 1024, 2);
-        const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, 1024, 0);
-#pragma unroll
-        for (int ks = 0; ks < TR / 16; ++ks)
-#pragma unroll
-          for (int mb = 0; mb < C::MBL; ++mb)
-            umma_f16(t_o + 32 * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
-                     dp + (uint64_t)(ks * 16), ID_V, t > 0 || ks > 0);
-        umma_commit(&obar[t % C::NST]);
+      __syncwarp();
+      pdl_trigger();
+    } else if (warp == 4 || warp == 7) {
+      // ======================= score warps ==================================
+      // as in mla.cu (warp 4 the even tiles, warp 7 the odd ones; a warp waits
+      // for softmax(t-2) before the operand of tile t, whose stage's previous
+      // tile t - 3 is then known to have been expanded); the latent k-steps
+      // accumulate into S columns 0-31, the positional ones into 32-63
+      const int role = warp == 4 ? 0 : 1;
+      constexpr uint32_t ID_S = umma_idesc_f16(C::SM, 32, false, false);
+      for (int t = role; t < n_tiles && !failed; t += 2) {
+        const int s = t % C::NST;
+        bool ok = true;
+        if (t >= 2) ok = mbar_wait_sleepy(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag, kSleepNs);
+        if (ok) ok = mbar_wait_sleepy(&full[s], (t / C::NST) & 1, kLimit, abort_flag, kSleepNs);
+        if (ok && lane == 0) {
+          tc_fence_after();
+          const uint64_t dc = umma_desc(smem_u32(ostage(s)), 16, 1024, 2);
+          const uint64_t dq = umma_desc(smem_u32(q_s), 128, KH / 8 * 128, 0);
+          const uint32_t S = t_s + 64 * (t & 1);
+  #pragma unroll
+          for (int ks = 0; ks < KH / 16; ++ks) {
+            const bool rope = ks >= W / 16;
+            umma_f16(rope ? S + 32 : S, dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
+                     dq + (uint64_t)(ks * 16), ID_S, rope ? ks > W / 16 : ks > 0);
+          }
+          umma_commit(&sbar[t & 1]);
+        }
+        failed = !__all_sync(0xffffffffu, ok);
       }
-      failed = !__all_sync(0xffffffffu, ok);
+      if (failed && lane == 0) {
+        *abort_flag = 1;
+        set_err(err, 8);
+      }
+      if (lane == 0) {
+        umma_commit(&dbar[2 * role]);
+        mbar_wait(&dbar[2 * role], 0, kLimit);
+      }
+      __syncwarp();
+      pdl_trigger();
+    } else {
+      // ======================= value warp ===================================
+      constexpr uint32_t ID_V = umma_idesc_f16(C::MV, 32, true, true);
+      for (int t = 0; t < n_tiles && !failed; ++t) {
+        const bool ok = mbar_wait_sleepy(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag, kSleepNs);
+        if (ok && lane == 0) {  // O^T[:, hi | lo] += U^T [P'_hi | P'_lo]
+          tc_fence_after();
+          const uint64_t da = umma_desc(smem_u32(ostage(t % C::NST)), C::BOX, 1024, 2);
+          const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, C::PNS, 0);
+  #pragma unroll
+          for (int ks = 0; ks < TR / 16; ++ks)
+  #pragma unroll
+            for (int mb = 0; mb < C::MBL; ++mb)
+              umma_f16(t_o + 32 * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
+                       dp + (uint64_t)(ks * 16), ID_V, t > 0 || ks > 0);
+          umma_commit(&obar[t % C::NST]);
+        }
+        failed = !__all_sync(0xffffffffu, ok);
+      }
+      if (failed && lane == 0) {
+        *abort_flag = 1;
+        set_err(err, 8);
+      }
+      if (lane == 0) {
+        umma_commit(&dbar[1]);
+        mbar_wait(&dbar[1], 0, kLimit);
+      }
+      __syncwarp();
+      pdl_trigger();
     }
-    if (failed && lane == 0) {
-      *abort_flag = 1;
-      set_err(err, 8);
-    }
-    if (lane == 0) {
-      umma_commit(&dbar[1]);
-      mbar_wait(&dbar[1], 0, kLimit);
-    }
-    __syncwarp();
-    pdl_trigger();
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 256;\n" ::: "memory");
     // ======================= softmax warps ================================
     const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
-    const int prow = 16 * warp + lane;  // this lane's tile position (lanes 0-15)
+    // this lane's tile position: M = 128 puts row r in lane r; M = 64 puts
+    // row r in lane 32 (r / 16) + r % 16 (lanes 0-15 of each quarter)
+    constexpr int kRowLanes = C::SM == 128 ? 32 : 16;
+    const int prow = kRowLanes * warp + lane;
     // per-head sums of the query halves as the products use them: thread
     // (h = tid / 8, j = tid % 8) adds chunks j, j + 8, ... of rows h and 16 + h
     {
@@ -403,29 +477,27 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     for (int h = 0; h < kHeads; ++h) { m_run[h] = -1e30f; l_part[h] = 0.f; z_part[h] = 0.f; }
     for (int t = 0; t < n_tiles; ++t) {
       const int base = i0 + t * TR, nval = min(TR, i1 - base);
-      bool ok = mbar_wait_or_abort(&sbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
+      bool ok = mbar_wait_sleepy(&sbar[t & 1], (t >> 1) & 1, kLimit, abort_flag, kSleepNs);
       // the tile's scales were written before its operand was published:
       // acquire them (the phase of tile t is complete, the next cannot be)
-      if (ok) ok = mbar_wait_or_abort(&full[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag);
+      if (ok) ok = mbar_wait_sleepy(&full[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag, kSleepNs);
       // P buffer (t & 1) was read by values(t-2)
       if (ok && t >= 2)
-        ok = mbar_wait_or_abort(&obar[(t - 2) % C::NST], ((t - 2) / C::NST) & 1, kLimit, abort_flag);
+        ok = mbar_wait_sleepy(&obar[(t - 2) % C::NST], ((t - 2) / C::NST) & 1, kLimit, abort_flag, kSleepNs);
       if (softmax_sync_or(!ok)) { failed = true; break; }
       tc_fence_after();
-      const bool live = lane < 16 && prow < nval;
+      const bool live = lane < kRowLanes && prow < nval;
       const float4 md = live ? ometa(t % C::NST)[prow] : make_float4(0.f, 0.f, 0.f, 0.f);
       float x[kHeads];
       {
-        const uint32_t S = t_s + 64 * (t & 1);
-        float lo[16], rh[16], rl[16];
-        tmem_ld16(S + lane_off, x);
-        tmem_ld16(S + 16 + lane_off, lo);
-        tmem_ld16(S + 32 + lane_off, rh);
-        tmem_ld16(S + 48 + lane_off, rl);
+        // [latent hi | latent lo | rope hi | rope lo] of the 16 heads
+        float sv[64];
+        tmem_ld64(t_s + 64 * (t & 1) + lane_off, sv);
         const float scl = md.x * kCodeScale, scr = md.z * kCodeScale;
 #pragma unroll
         for (int h = 0; h < kHeads; ++h)
-          x[h] = live ? fmaf(x[h] + lo[h], scl, fmaf(rh[h] + rl[h], scr, fmaf(md.y, qsl[h], md.w * qsr[h])))
+          x[h] = live ? fmaf(sv[h] + sv[16 + h], scl,
+                             fmaf(sv[32 + h] + sv[48 + h], scr, fmaf(md.y, qsl[h], md.w * qsr[h])))
                       : -INFINITY;
       }
       bool need = false;
@@ -436,7 +508,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
         for (int h = 0; h < kHeads; ++h) {
           float mx = x[h];
 #pragma unroll
-          for (int off = 1; off < 16; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+          for (int off = 1; off < kRowLanes; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
           if (lane == 0) red[warp * kHeads + h] = mx;
         }
         softmax_sync();
@@ -456,7 +528,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
           z_part[h] *= alpha[h];
         }
         if (t >= 1 && any) {
-          ok = mbar_wait_or_abort(&obar[(t - 1) % C::NST], ((t - 1) / C::NST) & 1, kLimit, abort_flag);
+          ok = mbar_wait_sleepy(&obar[(t - 1) % C::NST], ((t - 1) / C::NST) & 1, kLimit, abort_flag, kSleepNs);
           if (softmax_sync_or(!ok)) { failed = true; break; }
           tc_fence_after();
 #pragma unroll
@@ -474,8 +546,8 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
       }
       // value weights P' = p s (the latent scale of the position) as f16 hi
       // + lo into the MN-major P operand: position k, column n (0-15 hi,
-      // 16-31 lo) at (k/8) 128 + (n/8) 1024 + (k%8) 16 + (n%8) 2
-      if (lane < 16 && prow < TR) {
+      // 16-31 lo) at (k/8) 128 + (n/8) PNS + (k%8) 16 + (n%8) 2
+      if (lane < kRowLanes && prow < TR) {
         uint32_t hw[8], lw[8];
 #pragma unroll
         for (int h = 0; h < kHeads; h += 2) {
@@ -489,9 +561,9 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
         }
         uint8_t *pp = pbuf(t & 1) + (prow / 8) * 128 + (prow % 8) * 16;
         *reinterpret_cast<uint4 *>(pp) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-        *reinterpret_cast<uint4 *>(pp + 1024) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
-        *reinterpret_cast<uint4 *>(pp + 2048) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-        *reinterpret_cast<uint4 *>(pp + 3072) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
+        *reinterpret_cast<uint4 *>(pp + C::PNS) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+        *reinterpret_cast<uint4 *>(pp + 2 * C::PNS) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        *reinterpret_cast<uint4 *>(pp + 3 * C::PNS) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
       }
       fence_proxy_async();
       tc_fence_before();
@@ -502,7 +574,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     // ---- partial of this split: o_lat rows, m, l ----------------------------
     if (!failed && n_tiles > 0) {
       const int t = n_tiles - 1;
-      const bool ok = mbar_wait_or_abort(&obar[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag);
+      const bool ok = mbar_wait_sleepy(&obar[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag, kSleepNs);
       failed = softmax_sync_or(!ok);
     }
     if (failed && tid == 0) {
@@ -517,7 +589,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
       for (int h = 0; h < kHeads; ++h) {
         float sum = l_part[h], zs = z_part[h];
 #pragma unroll
-        for (int off = 1; off < 16; off <<= 1) {
+        for (int off = 1; off < kRowLanes; off <<= 1) {
           sum += __shfl_xor_sync(0xffffffffu, sum, off);
           zs += __shfl_xor_sync(0xffffffffu, zs, off);
         }
