@@ -382,6 +382,19 @@ kvk_status kvk_export_layer(const kvk_cache *cache, int32_t layer, void *k_out, 
                             float *k_scale, float *k_zero, float *v_scale, float *v_zero,
                             void *k_residual, kvk_stream stream);
 
+/* Number of polls a decode kernel's bounded wait on its own asynchronous
+ * copies makes, inside the tile loop, before it gives up
+ * (kvk_decode_attention, kvk_decode_partial, the no-alloc decode and the
+ * MLA decode of quantised latents).  KVK_WAIT_LIMIT_DEFAULT unless changed
+ * here; the setting applies to the calls enqueued after it.  A wait that
+ * gives up makes its CTA stop consuming tiles, let the copies it has in
+ * flight land (with a limit of its own), set KVK_DEVERR_TIMEOUT and return;
+ * the outputs of that call are unspecified and later calls are unaffected.
+ * 0 makes every such wait give up at its first poll: a way to exercise that
+ * path without a fault.  Errors: KVK_ERR_INVALID_ARG for a null cache. */
+#define KVK_WAIT_LIMIT_DEFAULT 4194304u
+kvk_status kvk_set_wait_limit(kvk_cache *cache, uint32_t polls);
+
 /* Synchronise `stream`, read the device error word into *code and clear it.
  * Returns KVK_ERR_DEVICE if the word was non-zero.  After a
  * KVK_DEVERR_TIMEOUT the outputs of the affected calls are unspecified. */

@@ -116,6 +116,13 @@ class Cache:
     def reset(self, stream=None):
         check(self.lib.kvk_cache_reset(self.handle, _stream(stream)))
 
+    WAIT_LIMIT_DEFAULT = 4194304
+
+    def set_wait_limit(self, polls: int):
+        """Polls a decode kernel's bounded wait makes in its tile loop before
+        giving up (0: at the first poll, setting the timeout error)."""
+        check(self.lib.kvk_set_wait_limit(self.handle, int(polls)))
+
     # -- plan ----------------------------------------------------------------
     def source(self, layer: int) -> int:
         out = ctypes.c_int32()

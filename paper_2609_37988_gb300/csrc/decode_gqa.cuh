@@ -952,7 +952,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       }
       const int nt = t + C::NST - 1;
       if (nt < n_tiles) issue(nt, nt % C::NST);
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22));
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, a.wait_limit));
       if (ok) compute(t, t % C::NST);
     }
     if (t_fail < 0 && __syncthreads_or(!ok)) t_fail = n_tiles - 1;
@@ -969,7 +969,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       if (use_cp)
         cp_async_wait<C::NST - 2>();
       else
-        ok = mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, 1u << 22);
+        ok = mbar_wait(&bars[t % C::NST], (t / C::NST) & 1, a.wait_limit);
       // every thread has finished tile t-1, and all agree whether a wait gave up
       if (__syncthreads_or(!ok)) {
         timed_out = true;

@@ -45,6 +45,7 @@ struct GqaDecodeArgs {
   float *partial;      // [n_splits, B*Hq, D+2], written when out is null
   float *out;          // [B, Hq, D]: normalised output (single split)
   int32_t *err;
+  uint32_t wait_limit = 1u << 22;  // polls of a bounded wait on this CTA's copies before it gives up
 };
 
 // Returns cudaSuccess or the launch error.  Template dispatch on
@@ -137,6 +138,7 @@ struct MlaDecodeArgs {
   float *out;          // [B, H, Dv]
   int32_t *err;
   const void *tmap;    // host copy of the anchor's 128-byte tensor map (mla_make_tmap)
+  uint32_t wait_limit = 1u << 22;  // polls of a bounded wait in the tile loop before it gives up
 };
 cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st);
 // the same for an anchor of quantised latents (mla_q.cu; one CTA per SM)

@@ -178,6 +178,7 @@ struct kvk_cache {
   int sm_count;
   int device;
   std::vector<int> ctas;  // per layer, decode CTAs per SM (0 = not queried)
+  uint32_t wait_limit = KVK_WAIT_LIMIT_DEFAULT;  // decode tile-loop waits (kvk_set_wait_limit)
   struct alignas(64) Tmap {
     uint8_t bytes[128];
   };
@@ -422,6 +423,12 @@ kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg
 
 kvk_status kvk_cache_destroy(kvk_cache *cache) {
   delete cache;
+  return KVK_OK;
+}
+
+kvk_status kvk_set_wait_limit(kvk_cache *c, uint32_t polls) {
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
+  c->wait_limit = polls;
   return KVK_OK;
 }
 
@@ -771,6 +778,7 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   const int tps = ((tiles + n_splits - 1) / n_splits + per - 1) / per * per;
   args.items_per_split = tps * kTile;
   args.err = c->err();
+  args.wait_limit = c->wait_limit;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (merge && n_splits == 1) {
     args.out = out;  // one split: the kernel normalises and writes the output
@@ -904,6 +912,7 @@ kvk_status kvk_decode_attention_mla(kvk_cache *c, int32_t layer, const void *q_n
   args.olat = reinterpret_cast<float *>(c->ws + c->wl.olat);
   args.out = out;
   args.err = c->err();
+  args.wait_limit = c->wait_limit;
   cudaError_t e = launch_mla_decode(args, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "MLA decode launch");
   return KVK_OK;

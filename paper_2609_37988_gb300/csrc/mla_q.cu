@@ -144,7 +144,7 @@ template <int W, int BITS, bool SYM>
 __global__ void __launch_bounds__(kMlaQThreads, 1)
     mla_decode_q_kernel(const MlaView v, const uint16_t *__restrict__ qlat,
                         const uint16_t *__restrict__ q_pe, int H, float sig, int items_per_split,
-                        int n_splits, float *__restrict__ partial, int32_t *err) {
+                        int n_splits, float *__restrict__ partial, int32_t *err, uint32_t wait_limit) {
   using C = MlaQCfg<W, BITS, SYM>;
   constexpr int TR = C::TR, KH = C::KH;
   constexpr float kCodeScale = 16777216.f;  // codes enter the products as u * 2^-24
@@ -168,6 +168,8 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   const int i1 = (split == n_splits - 1) ? len : min(i0 + items_per_split, len);
   const int n_tiles = i1 > i0 ? (i1 - i0 + TR - 1) / TR : 0;
   const size_t pos0 = (size_t)b * v.cap;  // slab of sequence b
+  // waits in the tile loops poll at most wait_limit times; the final waits
+  // for a role's own copies and products (before the CTA leaves) kLimit
   constexpr uint32_t kLimit = 1u << 22;
 
   if (tid == 0) {
@@ -273,9 +275,9 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     }
     for (int t = 0; t < n_tiles; ++t) {
       const int r = t % C::NR, s = t % C::NST;
-      bool ok = mbar_wait_sleepy(&rfull[r], (t / C::NR) & 1, kLimit, abort_flag, kSleepNs);
+      bool ok = mbar_wait_sleepy(&rfull[r], (t / C::NR) & 1, wait_limit, abort_flag, kSleepNs);
       if (ok && t >= C::NST)
-        ok = mbar_wait_sleepy(&obar[s], ((t - C::NST) / C::NST) & 1, kLimit, abort_flag, kSleepNs);
+        ok = mbar_wait_sleepy(&obar[s], ((t - C::NST) / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       const int nval = min(TR, i1 - (i0 + t * TR));
       const uint8_t *raw = rawst(r);
@@ -343,7 +345,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
           const int r = issued % C::NR;
           // the raw stage's previous tile was expanded
           if (issued >= C::NR &&
-              !mbar_wait_sleepy(&rfree[r], ((issued - C::NR) / C::NR) & 1, kLimit, abort_flag, kSleepNs)) {
+              !mbar_wait_sleepy(&rfree[r], ((issued - C::NR) / C::NR) & 1, wait_limit, abort_flag, kSleepNs)) {
             *abort_flag = 1;
             set_err(err, 8);
             break;
@@ -373,8 +375,8 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
       for (int t = role; t < n_tiles && !failed; t += 2) {
         const int s = t % C::NST;
         bool ok = true;
-        if (t >= 2) ok = mbar_wait_sleepy(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag, kSleepNs);
-        if (ok) ok = mbar_wait_sleepy(&full[s], (t / C::NST) & 1, kLimit, abort_flag, kSleepNs);
+        if (t >= 2) ok = mbar_wait_sleepy(&pbar[t & 1], ((t - 2) >> 1) & 1, wait_limit, abort_flag, kSleepNs);
+        if (ok) ok = mbar_wait_sleepy(&full[s], (t / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
         if (ok && lane == 0) {
           tc_fence_after();
           const uint64_t dc = umma_desc(smem_u32(ostage(s)), 16, 1024, 2);
@@ -404,7 +406,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
       // ======================= value warp ===================================
       constexpr uint32_t ID_V = umma_idesc_f16(C::MV, 32, true, true);
       for (int t = 0; t < n_tiles && !failed; ++t) {
-        const bool ok = mbar_wait_sleepy(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag, kSleepNs);
+        const bool ok = mbar_wait_sleepy(&pbar[t & 1], (t >> 1) & 1, wait_limit, abort_flag, kSleepNs);
         if (ok && lane == 0) {  // O^T[:, hi | lo] += U^T [P'_hi | P'_lo]
           tc_fence_after();
           const uint64_t da = umma_desc(smem_u32(ostage(t % C::NST)), C::BOX, 1024, 2);
@@ -477,13 +479,13 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     for (int h = 0; h < kHeads; ++h) { m_run[h] = -1e30f; l_part[h] = 0.f; z_part[h] = 0.f; }
     for (int t = 0; t < n_tiles; ++t) {
       const int base = i0 + t * TR, nval = min(TR, i1 - base);
-      bool ok = mbar_wait_sleepy(&sbar[t & 1], (t >> 1) & 1, kLimit, abort_flag, kSleepNs);
+      bool ok = mbar_wait_sleepy(&sbar[t & 1], (t >> 1) & 1, wait_limit, abort_flag, kSleepNs);
       // the tile's scales were written before its operand was published:
       // acquire them (the phase of tile t is complete, the next cannot be)
-      if (ok) ok = mbar_wait_sleepy(&full[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag, kSleepNs);
+      if (ok) ok = mbar_wait_sleepy(&full[t % C::NST], (t / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
       // P buffer (t & 1) was read by values(t-2)
       if (ok && t >= 2)
-        ok = mbar_wait_sleepy(&obar[(t - 2) % C::NST], ((t - 2) / C::NST) & 1, kLimit, abort_flag, kSleepNs);
+        ok = mbar_wait_sleepy(&obar[(t - 2) % C::NST], ((t - 2) / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
       if (softmax_sync_or(!ok)) { failed = true; break; }
       tc_fence_after();
       const bool live = lane < kRowLanes && prow < nval;
@@ -528,7 +530,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
           z_part[h] *= alpha[h];
         }
         if (t >= 1 && any) {
-          ok = mbar_wait_sleepy(&obar[(t - 1) % C::NST], ((t - 1) / C::NST) & 1, kLimit, abort_flag, kSleepNs);
+          ok = mbar_wait_sleepy(&obar[(t - 1) % C::NST], ((t - 1) / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
           if (softmax_sync_or(!ok)) { failed = true; break; }
           tc_fence_after();
 #pragma unroll
@@ -574,7 +576,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     // ---- partial of this split: o_lat rows, m, l ----------------------------
     if (!failed && n_tiles > 0) {
       const int t = n_tiles - 1;
-      const bool ok = mbar_wait_sleepy(&obar[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag, kSleepNs);
+      const bool ok = mbar_wait_sleepy(&obar[t % C::NST], (t / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
       failed = softmax_sync_or(!ok);
     }
     if (failed && tid == 0) {
@@ -664,7 +666,7 @@ cudaError_t launch_mla_q_t(const MlaDecodeArgs &a, cudaStream_t st) {
   if (e == cudaSuccess)
     e = launch_pdl(k, dim3(a.n_splits, B), dim3(kMlaQThreads), C::SMEM, st, a.v,
                    static_cast<const uint16_t *>(a.qlat), static_cast<const uint16_t *>(a.q_pe),
-                   a.H, a.sig_log2, a.items_per_split, a.n_splits, a.partial, a.err);
+                   a.H, a.sig_log2, a.items_per_split, a.n_splits, a.partial, a.err, a.wait_limit);
   if (e == cudaSuccess)
     e = launch_pdl(mla_merge_upv_kernel<W>, dim3(a.H, (B + 15) / 16, 4), dim3(128), MU_SMEM, st,
                    static_cast<const float *>(a.partial), a.n_splits,

@@ -169,3 +169,7 @@ def test_symmetric_arena_and_cost(lib):
         per_elem = stored * 8 / (2 * 8 * 128)
         assert per_elem == pytest.approx(cost.bits_per_element_symmetric(bits))
         assert rho == pytest.approx(16 / bits)
+
+
+def test_wait_limit_rejects_a_null_cache(lib):
+    assert lib.load().kvk_set_wait_limit(None, 5) == 1  # KVK_ERR_INVALID_ARG
