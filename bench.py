@@ -19,6 +19,7 @@ path) and the line reports the sum over ranks divided by the slowest rank.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import math
 import os
@@ -45,6 +46,20 @@ def peaks():
     return 6800.0, "fallback"
 
 
+def _record_bytes(w, l):
+    """Bytes stored per (position, kv head) by anchor l: one record, with the
+    group metadata (per-token formats) or the two bf16 scales (symmetric)."""
+    return _rec_bytes(w.layers[l], w.head_dim)
+
+
+def _rec_bytes(a, D):
+    if a["bits"] == 16:
+        return 4 * D
+    if a.get("scheme") == "symmetric":
+        return 2 * D * a["bits"] // 8 + 2 * 2
+    return 2 * D * a["bits"] // 8 + 2 * 8 * D // a["group"]
+
+
 def algorithmic_bytes(w, lens_after_append):
     """Bytes one step must move: each layer reads its source anchor's records
     at the current length (per-token formats: rec bytes per (position, kv
@@ -55,12 +70,7 @@ def algorithmic_bytes(w, lens_after_append):
     per_layer = []
     for l in range(w.n_layers):
         a = w.layers[src[l]]
-        if a["bits"] == 16:
-            rec = 4 * D
-        elif a.get("scheme") == "symmetric":
-            rec = 2 * D * a["bits"] // 8 + 2 * 2      # codes + two bf16 scales
-        else:
-            rec = 2 * D * a["bits"] // 8 + 2 * 8 * D // a["group"]
+        rec = _record_bytes(w, src[l])
         n = w.keep if w.keep else lens_after_append
         cache = B * H * n * rec
         qo = B * w.n_q_heads * D * (2 + 4)
@@ -327,9 +337,12 @@ def _layer_kind(w, l, src):
 def kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer, src, layer_call, dev,
                      splitk_reduce, reps=5):
     """Per-layer decode-kernel durations (ms) grouped by kind, with the
-    algorithmic bytes of each layer: ``{kind: [(ms, bytes), ...]}``."""
+    algorithmic bytes of each layer: ``{kind: [(ms, bytes), ...]}``; for
+    GQA steps also the appends and the split-K merges in ``aux`` (same
+    form, kinds "append" and "merge").  Returns (kt, aux, how)."""
     import torch
     L = w.n_layers
+    aux = {}
     parts = {}
     if w.kind == "gqa":
         for l in range(L):
@@ -349,19 +362,40 @@ def kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer, src,
         if w.kind == "gqa" and splits[l] > 1:
             splitk_reduce(parts[l], out=outs[l].view(-1, w.head_dim))
 
+    def append_bytes(l):
+        # the new rows read (bf16 keys and values) and one record written per
+        # (sequence, new position, kv head)
+        k, v = new_kv[l]
+        rows = k.shape[0] * k.shape[1] * k.shape[2]
+        return k.numel() * k.element_size() + v.numel() * v.element_size() + rows * _record_bytes(w, l)
+
+    def merge_bytes(l):
+        rows = w.batch * w.n_q_heads
+        return splits[l] * rows * (w.head_dim + 2) * 4 + rows * w.head_dim * 4
+
     kt = {}
     try:
-        evs = [(torch.cuda.Event(enable_timing=True, external=True),
-                torch.cuda.Event(enable_timing=True, external=True)) for _ in range(L)]
+        def ev():
+            return (torch.cuda.Event(enable_timing=True, external=True),
+                    torch.cuda.Event(enable_timing=True, external=True))
+        evs = [ev() for _ in range(L)]
+        aev = {l: ev() for l in new_kv}
+        mev = {l: ev() for l in range(L) if w.kind == "gqa" and splits[l] > 1}
 
         def tstep():
             for l in range(L):
                 if l in new_kv:
+                    aev[l][0].record(stream)
                     cache.append(l, *new_kv[l])
+                    aev[l][1].record(stream)
                 evs[l][0].record(stream)
                 run_layer(l)
                 evs[l][1].record(stream)
+                if l in mev:
+                    mev[l][0].record(stream)
                 merge(l)
+                if l in mev:
+                    mev[l][1].record(stream)
             if w.append_per_step:
                 cache.rewind(1)
 
@@ -379,11 +413,15 @@ def kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer, src,
                 for l in range(L):
                     kt.setdefault(_layer_kind(w, l, src), []).append(
                         (evs[l][0].elapsed_time(evs[l][1]), per_layer[l]))
+                for l, (e0, e1) in aev.items():
+                    aux.setdefault("append", []).append((e0.elapsed_time(e1), append_bytes(l)))
+                for l, (e0, e1) in mev.items():
+                    aux.setdefault("merge", []).append((e0.elapsed_time(e1), merge_bytes(l)))
         del g
-        return kt, "event nodes in a graph replay of the step"
+        return kt, aux, "event nodes in a graph replay of the step"
     except (TypeError, RuntimeError):
         torch.cuda.synchronize()
-        kt = {}
+        kt, aux = {}, {}
     with torch.cuda.stream(stream):
         for l in range(L):
             if l in new_kv:
@@ -399,7 +437,7 @@ def kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer, src,
         if w.append_per_step:
             cache.rewind(1)
         torch.cuda.synchronize()
-    return kt, "eager launches between events (includes host launch gaps)"
+    return kt, aux, "eager launches between events (includes host launch gaps)"
 
 
 
@@ -421,12 +459,15 @@ def main():
                          "quantiser at this bit-width")
     ap.add_argument("--profile-case",
                     choices=["gqa", "kpc", "mla", "mla64", "gather", "sym", "evict", "evict-small",
-                             "prefill", "prefill-small"],
+                             "prefill", "prefill-small", "append"],
                     default=None,
                     help="small ncu case: decode (or eviction) launches only, no timing line")
     ap.add_argument("--prefill", action="store_true",
                     help="time causal chunk attention (pre-fill) over one compressed 14B anchor "
                          "instead of the decode step (one JSON line of its own)")
+    ap.add_argument("--append", action="store_true",
+                    help="time bulk appends (quantise on write) at the 14B shape instead of the "
+                         "decode step (one JSON line of its own)")
     ap.add_argument("--evict", action="store_true",
                     help="time the window-vote evictor at the long-context 14B shape instead "
                          "of the decode step (one JSON line of its own)")
@@ -442,6 +483,9 @@ def main():
         return
     if args.prefill:
         prefill_bench(args)
+        return
+    if args.append:
+        append_bench(args)
         return
 
     import torch
@@ -565,7 +609,7 @@ def main():
     # back to eager launches bracketed by events where graph event nodes are
     # not available.
     from paper_2609_37988_gb300.cache import splitk_reduce
-    kt, kernel_timing = kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer,
+    kt, aux, kernel_timing = kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer,
                                          src, layer_call if w.kind == "mla" else None, dev,
                                          splitk_reduce)
     hbm, peak_kind = peaks()
@@ -575,12 +619,16 @@ def main():
     bts = [b for _, b in kt[dom]]
     avg_ms = sum(durs) / len(durs)
     achieved = (sum(bts) / len(bts)) / (avg_ms / 1e3) / 1e9
-    kernels = {}
-    for k, v in kt.items():
+    def summary(v):
         d = sum(t for t, _ in v) / len(v)
         b = sum(x for _, x in v) / len(v)
-        kernels[k] = {"avg_us": round(d * 1e3, 2), "gbs": round(b / (d / 1e3) / 1e9, 1),
-                      "frac": round(b / (d / 1e3) / 1e9 / hbm, 4)}
+        return {"avg_us": round(d * 1e3, 2), "bytes": int(b), "gbs": round(b / (d / 1e3) / 1e9, 1),
+                "frac": round(b / (d / 1e3) / 1e9 / hbm, 4)}
+    kernels = {k: summary(v) for k, v in kt.items()}
+    # the step's other kernels: a decode-step append (one new row per
+    # sequence and kv head) and a split-K merge move a few hundred KB to a
+    # few MB each, so their time is launch and memory latency, not bandwidth
+    other_kernels = {k: summary(v) for k, v in aux.items()}
     # DRAM bytes per launch of the dominant kernel from the committed ncu
     # summary, used only while the decode sources still hash to the value
     # recorded with it (null otherwise: the counters would be stale)
@@ -704,6 +752,7 @@ def main():
                          "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
                          "peak_source": f"MEASURED_PEAKS.json hbm_gbs ({peak_kind})"},
             "kernels": kernels,
+            "other_kernels": other_kernels,
             "kernel_timing": kernel_timing,
             "cpu_baseline": cpu,
             "e2e": e2e,
@@ -899,6 +948,78 @@ def prefill_bench(args):
     print(json.dumps(line))
 
 
+APPEND_CHUNK = 2048
+
+
+def append_bench(args):
+    """Bulk append (quantise on write) at the 14B shape: B=32 sequences, a
+    chunk of 2048 new positions each (a pre-fill chunk), 8 KV heads, head_dim
+    128, bf16 keys and values (268 MB read per call, larger than L2), into
+    one anchor of each format; the cache is reset between calls so every
+    call writes positions 0..2047.  CUDA events around each append on the
+    launching stream.  value = GB/s of the int4 g32 per-token append."""
+    import torch
+    from __graft_entry__ import build
+    build()
+    from paper_2609_37988_gb300 import workloads as W
+    from paper_2609_37988_gb300.cache import Cache, Layer
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    B, n, Hkv, D = 32, APPEND_CHUNK, 8, 128
+    w = W.config(3)
+    k, v = W.kv_inputs(w, 0, 0, n, device=dev)
+    formats = {"int4 g32": dict(bits=4, group=32), "int8 g64": dict(bits=8, group=64),
+               "bf16": dict(bits=16), "sym4": dict(bits=4, scheme="symmetric"),
+               "sym8": dict(bits=8, scheme="symmetric"),
+               "int4 g32 per-channel keys": dict(bits=4, group=32, key_axis="channel")}
+    res = {}
+    hbm, peak_kind = peaks()
+    with Clocks(0) as clk:
+        for name, cfg in formats.items():
+            c = Cache(n_layers=1, n_q_heads=40, n_kv_heads=Hkv, head_dim=D, max_batch=B,
+                      max_ctx=n, layers=[Layer(**cfg)], max_splits=8, device=dev)
+            stored = B * n * Hkv * _rec_bytes(dataclasses.asdict(Layer(**cfg)), D)
+            nbytes = k.numel() * k.element_size() + v.numel() * v.element_size() + stored
+            stream = torch.cuda.current_stream()
+            for _ in range(max(3, args.warmup)):
+                c.reset()
+                c.append(0, k, v)
+            torch.cuda.synchronize()
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                  for _ in range(args.steps)]
+            if name == "int4 g32":
+                clk.mark("start")
+            for s0, e0 in ev:
+                c.reset()
+                s0.record(stream)
+                c.append(0, k, v)
+                e0.record(stream)
+            torch.cuda.synchronize()
+            if name == "int4 g32":
+                clk.mark("end")
+            assert c.device_error() == 0
+            ms = statistics.mean(s0.elapsed_time(e0) for s0, e0 in ev)
+            res[name] = {"us": round(ms * 1e3, 2), "bytes": int(nbytes),
+                         "gbs": round(nbytes / (ms * 1e-3) / 1e9, 1),
+                         "frac": round(nbytes / (ms * 1e-3) / 1e9 / hbm, 4)}
+            del c
+    main_ = res["int4 g32"]
+    line = {"metric": "bulk append with quantise on write: GB/s of algorithmic bytes",
+            "value": main_["gbs"], "unit": "GB/s", "higher_is_better": True,
+            "steps": args.steps, "warmup": max(3, args.warmup), "n_gpus": 1,
+            "dtype": "bf16 in, int4 codes + f32 scale/zero out", "data": "synthetic",
+            "config": {"workload": f"qwen2.5-14b kv, B={B}, {n} new positions per sequence, "
+                                   f"{Hkv} kv heads, d_h {D}",
+                       "l2": "inputs (268 MB) larger than L2"},
+            "roofline": {"bound": "hbm", "kernel": "append (int4 g32, per token)",
+                         "achieved": main_["gbs"], "peak": hbm, "unit": "GB/s",
+                         "frac": main_["frac"], "traffic": None,
+                         "peak_source": f"MEASURED_PEAKS.json hbm_gbs ({peak_kind})",
+                         "work": "keys and values read once (bf16), records and metadata written once"},
+            "formats": res, "gpu_launches": args.steps, "clocks": clk.summary()}
+    print(json.dumps(line))
+
+
 def profile_case(kind):
     """The kernel-level ncu case.  gqa: one int4 g32 and one bf16 anchor at
     the 14B step shape (B=32, 8 kv / 40 q heads, d_h 128, T=8192; 1.5 GB of
@@ -930,6 +1051,16 @@ def profile_case(kind):
         for _ in range(3):
             for l in range(2):
                 c.decode(l, q, w.sigma)
+    elif kind == "append":
+        # bulk append at the 14B shape: 32 sequences x 2048 new positions x
+        # 8 kv heads into an int4 g32 anchor (268 MB of bf16 inputs), 3 calls
+        w = W.config(3)
+        c = Cache(n_layers=1, n_q_heads=40, n_kv_heads=8, head_dim=128, max_batch=32,
+                  max_ctx=APPEND_CHUNK, layers=[Layer(bits=4, group=32)])
+        k, v = W.kv_inputs(w, 0, 0, APPEND_CHUNK, device="cuda")
+        for _ in range(3):
+            c.reset()
+            c.append(0, k, v)
     elif kind == "kpc":
         # per-channel keys at the 7B step shape: one int4 g32 and one int8
         # g64 anchor (B=16, 4 kv / 28 q heads, T=8192)

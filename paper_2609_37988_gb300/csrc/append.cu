@@ -37,6 +37,19 @@ __device__ __forceinline__ int seq_count(const int32_t *n_per_seq, int b, int n_
   return n;
 }
 
+// rint(fl(d / s)) for s > 0 and |d / s| at most a few hundred, without a
+// division in the common case: y = fl(d fl(1/s)) is within 1.2e-7 |d/s| of
+// d/s, and fl(d/s) within 6e-8 |d/s|, so for |d/s| <= 300 the two differ by
+// less than 6e-5; when y is further than 1e-4 from the nearest half-integer
+// both round to the same integer.  Otherwise (or when y is not finite) the
+// correctly rounded division decides.  `near` reports that case.
+__device__ __forceinline__ float rint_quot_fast(float d, float rs, bool &near) {
+  const float y = __fmul_rn(d, rs);
+  const float r = rintf(y);
+  near = !(fabsf(__fsub_rn(y, r)) < 0.4999f);
+  return r;
+}
+
 // Quantise one lane's E elements belonging to groups of GS channels spread
 // over GS/E consecutive lanes.  Returns codes, writes the group's scale and
 // zero into (sc, zr) on every lane of the group.
@@ -53,16 +66,22 @@ __device__ __forceinline__ void quant_lane(const float (&x)[E], int GS, int leve
   }
   const float lev = (float)levels;
   const float scale = __fdiv_rn(__fsub_rn(mx, mn), lev);
+  const float rs = scale == 0.f ? 0.f : __frcp_rn(scale);
+  float r[E];
+  bool any_near = false;
 #pragma unroll
   for (int e = 0; e < E; ++e) {
-    if (scale == 0.f) {
-      code[e] = 0;
-    } else {
-      float r = rintf(__fdiv_rn(__fsub_rn(x[e], mn), scale));
-      r = fminf(fmaxf(r, 0.f), lev);
-      code[e] = (uint32_t)r;
-    }
+    bool near;
+    r[e] = rint_quot_fast(__fsub_rn(x[e], mn), rs, near);
+    any_near |= near;
   }
+  if (__any_sync(0xffffffffu, any_near && scale != 0.f)) {
+#pragma unroll
+    for (int e = 0; e < E; ++e)
+      if (scale != 0.f) r[e] = rintf(__fdiv_rn(__fsub_rn(x[e], mn), scale));
+  }
+#pragma unroll
+  for (int e = 0; e < E; ++e) code[e] = scale == 0.f ? 0u : (uint32_t)fminf(fmaxf(r[e], 0.f), lev);
   sc = scale;
   zr = mn;
 }
@@ -83,10 +102,24 @@ __device__ __forceinline__ uint16_t quant_sym_lane(const float (&x)[E], int bits
   const float q = (float)sym_levels(bits);
   const uint16_t sb = f32_to_bf16_bits(__fdiv_rn(am, q));
   const float s = bf16_to_f32(sb);
+  const float rs = s == 0.f ? 0.f : __frcp_rn(s);
+  float rq[E];
+  bool any_near = false;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    bool near;
+    rq[e] = rint_quot_fast(x[e], rs, near);
+    any_near |= near;
+  }
+  if (__any_sync(0xffffffffu, any_near && s != 0.f)) {
+#pragma unroll
+    for (int e = 0; e < E; ++e)
+      if (s != 0.f) rq[e] = rintf(__fdiv_rn(x[e], s));
+  }
 #pragma unroll
   for (int e = 0; e < E; ++e) {
     float r = 0.f;
-    if (s != 0.f) r = fminf(fmaxf(rintf(__fdiv_rn(x[e], s)), -q), q);
+    if (s != 0.f) r = fminf(fmaxf(rq[e], -q), q);
     u[e] = (uint32_t)(int)(r + q);
   }
   return sb;
@@ -150,15 +183,43 @@ __device__ void put_section(uint32_t *buf, int bits, bool is_k, const uint32_t (
   __syncwarp();
 }
 
+// E = D / 32 consecutive elements of one lane, one vector load (inputs are
+// 16-byte aligned and rows are D elements long)
+template <int E>
+__device__ __forceinline__ void load_lane(const void *in, size_t i, int f32, float (&x)[E]) {
+  static_assert(E == 2 || E == 4, "two or four elements per lane");
+  if (f32) {
+    const float *p = static_cast<const float *>(in) + i;
+    if constexpr (E == 4) {
+      const float4 w = *reinterpret_cast<const float4 *>(p);
+      x[0] = w.x; x[1] = w.y; x[2] = w.z; x[3] = w.w;
+    } else {
+      const float2 w = *reinterpret_cast<const float2 *>(p);
+      x[0] = w.x; x[1] = w.y;
+    }
+  } else {
+    const uint16_t *p = static_cast<const uint16_t *>(in) + i;
+    uint32_t w[E / 2];
+    if constexpr (E == 4) {
+      const uint2 u = *reinterpret_cast<const uint2 *>(p);
+      w[0] = u.x; w[1] = u.y;
+    } else {
+      w[0] = *reinterpret_cast<const uint32_t *>(p);
+    }
+#pragma unroll
+    for (int j = 0; j < E / 2; ++j) {
+      x[2 * j] = __uint_as_float(w[j] << 16);
+      x[2 * j + 1] = __uint_as_float(w[j] & 0xffff0000u);
+    }
+  }
+}
+
 template <int D>
 __device__ __forceinline__ void load_row(const void *kin, const void *vin, int in_f32,
                                          size_t ibase, int lane, float (&xk)[D / 32],
                                          float (&xv)[D / 32]) {
-#pragma unroll
-  for (int e = 0; e < D / 32; ++e) {
-    xk[e] = load_in(kin, ibase + lane * (D / 32) + e, in_f32);
-    xv[e] = load_in(vin, ibase + lane * (D / 32) + e, in_f32);
-  }
+  load_lane<D / 32>(kin, ibase + lane * (D / 32), in_f32, xk);
+  load_lane<D / 32>(vin, ibase + lane * (D / 32), in_f32, xv);
 }
 
 // Quantises and writes one (sequence b, position t, KV head kvh) record from
@@ -222,9 +283,10 @@ __global__ void __launch_bounds__(128)
   constexpr int E = D / 32;
   __shared__ __align__(16) uint32_t sbuf[4][(2 * D * 2 + 2 * 64) / 4];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const size_t wid = (size_t)blockIdx.x * 4 + warp;
   const size_t total = (size_t)v.B * n_new * v.Hkv;
-  if (wid < total) {
+  // rows wid, wid + 4 gridDim.x, ...: a bounded grid, so that the completion
+  // counter below takes one atomic per CTA, not one per four rows
+  for (size_t wid = (size_t)blockIdx.x * 4 + warp; wid < total; wid += (size_t)gridDim.x * 4) {
     const int kvh = (int)(wid % v.Hkv);
     const int i = (int)((wid / v.Hkv) % n_new);
     const int b = (int)(wid / ((size_t)v.Hkv * n_new));
@@ -240,6 +302,7 @@ __global__ void __launch_bounds__(128)
       load_row<D>(kin, vin, in_f32, (((size_t)b * n_new + i) * v.Hkv + kvh) * D, lane, xk, xv);
       append_row<D>(v, xk, xv, b, kvh, t, sbuf[warp], lane);
     }
+    __syncwarp();  // the row buffer is free again
   }
   // The last CTA advances the lengths (per-token layouts only; per-channel
   // keys advance them in the residual kernel, which runs last).
@@ -258,6 +321,265 @@ __global__ void __launch_bounds__(128)
       }
       if (threadIdx.x == 0) *v.counter = 0;
     }
+  }
+}
+
+// ---- bulk appends, head_dim 128, per-token layouts -------------------------
+// One warp per (sequence, new position, KV head) row over a bounded grid,
+// lane L holding channels 4L .. 4L+3.  Each lane packs its codes into one
+// register per section; the record's 32-bit words are then gathered from
+// the lanes that hold their channels by warp shuffles (the channel order of
+// layout.h, derived per format below) and stored as whole words, the 128-
+// to 512-byte record in one to four coalesced store instructions.
+
+// 4-bit codes (grouped int4 or symmetric 4-bit): p = K codes | V codes << 16.
+// Lanes 0-15 build K word T = lane (lane column c = T / 4, word w = T % 4
+// holds k-steps 2w, 2w+1: nibble h + 2 jj from lane 4 (2w + jj) + c/2 + 2h
+// element 2 (c%2), nibble 4 + h + 2 jj from its element 2 (c%2) + 1).
+// Lanes 16-31 build logical V word U = lane - 16 (chunk k = U / 4, word
+// wd = U % 4: M-blocks 2k + mm, rows g = 2 wd + gg, g + 8 e: bits
+// 8 (2 gg + mm) + 4 e from lane 4 (2k + mm) + 2e + wd/2, element
+// 2 (wd%2) + gg).
+struct Gather4 {
+  int src[4], sh, dlo[4], dhi[4];
+  __device__ explicit Gather4(int lane) {
+    if (lane < 16) {
+      const int c = lane >> 2, w = lane & 3;
+      sh = 8 * (c & 1);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int jj = q >> 1, h = q & 1;
+        src[q] = 4 * (2 * w + jj) + (c >> 1) + 2 * h;
+        dlo[q] = 4 * (h + 2 * jj);
+        dhi[q] = 4 * (4 + h + 2 * jj);
+      }
+    } else {
+      const int u = lane - 16, k = u >> 2, wd = u & 3;
+      sh = 16 + 8 * (wd & 1);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int mm = q >> 1, e = q & 1;
+        src[q] = 4 * (2 * k + mm) + 2 * e + (wd >> 1);
+        dlo[q] = 8 * mm + 4 * e;
+        dhi[q] = 16 + 8 * mm + 4 * e;
+      }
+    }
+  }
+  __device__ __forceinline__ uint32_t word(uint32_t p) const {
+    uint32_t x = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t b = __shfl_sync(0xffffffffu, p, src[q]) >> sh;
+      x |= ((b & 0xFu) << dlo[q]) | (((b >> 4) & 0xFu) << dhi[q]);
+    }
+    return x;
+  }
+};
+
+// 8-bit codes: every lane builds K word T = lane (chunk T / 4 = 4 (bp / 16)
+// + c, k-step j = 4 (chunk / 4) + T % 4: bytes 0-1 from lane 4j + c/2,
+// bytes 2-3 from lane 4j + c/2 + 2, each lane's elements 2 (c%2), +1) and
+// logical V word U = lane (M-block m = U / 4, word wd = U % 4: bytes 2 gg + e
+// from lane 4m + 2e + wd/2, element 2 (wd%2) + gg).
+struct Gather8 {
+  int ks0, ks1, ksh, vs0, vs1, vsh;
+  __device__ explicit Gather8(int lane) {
+    const int chunk = lane >> 2, c = chunk & 3, j = 4 * (chunk >> 2) + (lane & 3);
+    ks0 = 4 * j + (c >> 1);
+    ks1 = ks0 + 2;
+    ksh = 16 * (c & 1);
+    const int m = lane >> 2, wd = lane & 3;
+    vs0 = 4 * m + (wd >> 1);
+    vs1 = vs0 + 2;
+    vsh = 16 * (wd & 1);
+  }
+  __device__ __forceinline__ uint32_t kword(uint32_t pk) const {
+    const uint32_t a = (__shfl_sync(0xffffffffu, pk, ks0) >> ksh) & 0xFFFFu;
+    const uint32_t b = (__shfl_sync(0xffffffffu, pk, ks1) >> ksh) & 0xFFFFu;
+    return a | (b << 16);
+  }
+  __device__ __forceinline__ uint32_t vword(uint32_t pv) const {
+    const uint32_t a = __shfl_sync(0xffffffffu, pv, vs0) >> vsh;
+    const uint32_t b = __shfl_sync(0xffffffffu, pv, vs1) >> vsh;
+    return __byte_perm(a, b, 0x5140);
+  }
+};
+
+// bf16 values: lane owns K words T = lane, lane + 32 (chunk T / 4, c =
+// chunk % 4, j = 2 (chunk / 4) + (T % 4) / 2, h = T % 2: the bf16 pair of
+// elements 2 (c%2), +1 of lane 4j + c/2 + 2h) and V words W = lane, lane + 32
+// (row g = W / 8, M-block m = W % 8: element g % 4 of lanes 4m + g/4 (low
+// half) and 4m + g/4 + 2 (high half)).
+struct Gather16 {
+  int ks[2], kreg, vs[2], vreg, vhalf;
+  __device__ explicit Gather16(int lane) {
+    const int c = (lane >> 2) & 3;
+    kreg = c & 1;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int T = lane + 32 * i, chunk = T >> 2;
+      const int j = 2 * (chunk >> 2) + ((T & 3) >> 1);
+      ks[i] = 4 * j + (c >> 1) + 2 * (T & 1);
+    }
+    const int g0 = lane >> 3;  // rows g0 (W = lane) and g0 + 4 (W = lane + 32)
+    const int m = lane & 7;
+    vs[0] = 4 * m + (g0 >> 2);
+    vs[1] = 4 * m + ((g0 + 4) >> 2);
+    vreg = ((g0 & 3) >> 1);  // the same for g0 + 4
+    vhalf = 16 * (g0 & 1);
+  }
+  __device__ __forceinline__ uint32_t kword(uint32_t k0, uint32_t k1, int i) const {
+    const uint32_t a = __shfl_sync(0xffffffffu, k0, ks[i]);
+    const uint32_t b = __shfl_sync(0xffffffffu, k1, ks[i]);
+    return kreg ? b : a;
+  }
+  __device__ __forceinline__ uint32_t vword(uint32_t v0, uint32_t v1, int i) const {
+    const uint32_t a0 = __shfl_sync(0xffffffffu, v0, vs[i]);
+    const uint32_t a1 = __shfl_sync(0xffffffffu, v1, vs[i]);
+    const uint32_t b0 = __shfl_sync(0xffffffffu, v0, vs[i] + 2);
+    const uint32_t b1 = __shfl_sync(0xffffffffu, v1, vs[i] + 2);
+    const uint32_t lo = ((vreg ? a1 : a0) >> vhalf) & 0xFFFFu;
+    const uint32_t hi = ((vreg ? b1 : b0) >> vhalf) & 0xFFFFu;
+    return lo | (hi << 16);
+  }
+};
+
+// Codes of one lane's four channels in one register (code e at bits BITS e).
+template <int BITS>
+__device__ __forceinline__ uint32_t pack_codes(const uint32_t (&c)[4]) {
+  return c[0] | (c[1] << BITS) | (c[2] << (2 * BITS)) | (c[3] << (3 * BITS));
+}
+
+template <int BITS, int GS, bool SYM>
+__global__ void __launch_bounds__(256)
+    gqa_append_bulk(const GqaView v, const void *kin, const void *vin, int in_f32, int n_new,
+                    const int32_t *n_per_seq, int32_t *err) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int D = 128, E = 4;
+  constexpr int SEC = D * BITS / 8;                       // bytes per section
+  constexpr int REC = SYM ? 2 * SEC : BITS == 16 ? 2 * SEC : 2 * SEC + 2 * (((D / GS) * 8 + 15) & ~15);
+  constexpr int KM = 2 * SEC, VM = KM + (((D / GS) * 8 + 15) & ~15);
+  constexpr int NC = SEC / 16;                            // chunks per code section
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int wpb = blockDim.x >> 5;
+  const size_t total = (size_t)v.B * n_new * v.Hkv;
+  Gather4 g4(lane);
+  Gather8 g8(lane);
+  Gather16 g16(lane);
+  (void)g4; (void)g8; (void)g16;
+  // two rows per iteration, their loads issued together and their
+  // arithmetic independent (rows past the end compute on row 0's inputs and
+  // store nothing)
+  auto process = [&](const float (&xk)[E], const float (&xv)[E], bool ok, size_t row, int t) {
+    uint8_t *rec = v.rec + row * REC;
+    if constexpr (BITS == 16) {
+      uint32_t k0 = pack2<true>(xk[0], xk[1]), k1 = pack2<true>(xk[2], xk[3]);
+      uint32_t v0 = pack2<true>(xv[0], xv[1]), v1 = pack2<true>(xv[2], xv[3]);
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const uint32_t kw = g16.kword(k0, k1, h), vw = g16.vword(v0, v1, h);
+        if (ok) {
+          reinterpret_cast<uint32_t *>(rec)[lane + 32 * h] = kw;
+          reinterpret_cast<uint32_t *>(rec + SEC)[lane + 32 * h] = vw;
+        }
+      }
+    } else {
+      uint32_t ck[E], cv[E];
+      if constexpr (SYM) {
+        const uint32_t sk = quant_sym_lane<E>(xk, BITS, ck);
+        const uint32_t sv = quant_sym_lane<E>(xv, BITS, cv);
+        if (ok && lane == 0) v.scales[row] = sk | (sv << 16);
+      } else {
+        float ks, kz, vs, vz;
+        quant_lane<E>(xk, GS, (1 << BITS) - 1, ck, ks, kz);
+        quant_lane<E>(xv, GS, (1 << BITS) - 1, cv, vs, vz);
+        if (ok && (lane * E) % GS == 0) {
+          reinterpret_cast<float2 *>(rec + KM)[(lane * E) / GS] = make_float2(ks, kz);
+          reinterpret_cast<float2 *>(rec + VM)[(lane * E) / GS] = make_float2(vs, vz);
+        }
+      }
+      const uint32_t pk = pack_codes<BITS>(ck), pv = pack_codes<BITS>(cv);
+      // logical chunk of this lane's word(s) and its physical 16-byte slot:
+      // symmetric records rotate all chunks by sym_rot(t), grouped ones the
+      // V chunks by v_rot(t)
+      if constexpr (BITS == 4) {
+        const uint32_t w = g4.word(pk | (pv << 16));
+        int off;
+        if (lane < 16) {
+          off = SYM ? 16 * (((lane >> 2) + sym_rot(t, REC / 16)) & (REC / 16 - 1)) + 4 * (lane & 3)
+                    : 4 * lane;
+        } else {
+          const int u = lane - 16, k = u >> 2;
+          off = SYM ? 16 * ((NC + k + sym_rot(t, REC / 16)) & (REC / 16 - 1)) + 4 * (u & 3)
+                    : SEC + 16 * ((k + v_rot(t, REC, NC)) & (NC - 1)) + 4 * (u & 3);
+        }
+        if (ok) *reinterpret_cast<uint32_t *>(rec + off) = w;
+      } else {
+        const uint32_t kw = g8.kword(pk), vw = g8.vword(pv);
+        const int kc = lane >> 2;
+        const int koff = SYM ? 16 * ((kc + sym_rot(t, REC / 16)) & (REC / 16 - 1)) + 4 * (lane & 3)
+                             : 4 * lane;
+        const int voff = SYM ? 16 * ((NC + kc + sym_rot(t, REC / 16)) & (REC / 16 - 1)) + 4 * (lane & 3)
+                             : SEC + 16 * ((kc + v_rot(t, REC, NC)) & (NC - 1)) + 4 * (lane & 3);
+        if (ok) {
+          *reinterpret_cast<uint32_t *>(rec + koff) = kw;
+          *reinterpret_cast<uint32_t *>(rec + voff) = vw;
+        }
+      }
+    }
+  };
+  const size_t step = (size_t)gridDim.x * wpb;
+  for (size_t w0 = (size_t)blockIdx.x * wpb + warp; w0 < total; w0 += 2 * step) {
+    bool ok[2];
+    size_t row[2];
+    int tt[2];
+    float xk[2][E], xv[2][E];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const size_t wid = w0 + u * step;
+      ok[u] = false;
+      row[u] = 0;
+      tt[u] = 0;
+      size_t in_off = 0;
+      if (wid < total) {
+        // 32-bit index arithmetic (the launcher sends fewer than 2^31 rows)
+        const uint32_t w = (uint32_t)wid, q = w / (uint32_t)v.Hkv;
+        const int kvh = (int)(w - q * (uint32_t)v.Hkv);
+        const uint32_t bq = q / (uint32_t)n_new;
+        const int i = (int)(q - bq * (uint32_t)n_new), b = (int)bq;
+        in_off = wid * D;  // inputs are [B, n_new, H_kv, D], row wid
+        const int nb = seq_count(n_per_seq, b, n_new, err);
+        const int t = v.lens[b] + i;
+        if (i < nb) {
+          if (t >= v.cap) {
+            if (lane == 0) set_err(err, 2);
+          } else {
+            ok[u] = true;
+            row[u] = ((size_t)b * v.Hkv + kvh) * v.cap + t;
+            tt[u] = t;
+          }
+        }
+      }
+      load_row<D>(kin, vin, in_f32, in_off, lane, xk[u], xv[u]);
+    }
+    process(xk[0], xv[0], ok[0], row[0], tt[0]);
+    process(xk[1], xv[1], ok[1], row[1], tt[1]);
+  }
+  // the last CTA advances the lengths
+  __syncthreads();
+  __shared__ int last;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    last = (atomicAdd(v.counter, 1) == (int)gridDim.x - 1);
+  }
+  __syncthreads();
+  if (last) {
+    for (int b = threadIdx.x; b < v.B; b += blockDim.x) {
+      const int nb = seq_count(n_per_seq, b, n_new, nullptr);
+      v.lens[b] = min((long long)v.lens[b] + nb, (long long)v.cap);
+    }
+    if (threadIdx.x == 0) *v.counter = 0;
   }
 }
 
@@ -417,8 +739,8 @@ __global__ void __launch_bounds__(128)
   pdl_wait();
   pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const size_t wid = (size_t)blockIdx.x * 4 + warp;
-  if (wid < (size_t)v.B * n_new) {
+  for (size_t wid = (size_t)blockIdx.x * 4 + warp; wid < (size_t)v.B * n_new;
+       wid += (size_t)gridDim.x * 4) {
     const int i = (int)(wid % n_new), b = (int)(wid / n_new);
     const int nb = seq_count(n_per_seq, b, n_new, err);
     const int t = v.lens[b] + i;
@@ -464,8 +786,8 @@ __global__ void __launch_bounds__(128)
   constexpr int R = 64, KH = W + R, EC = W / 32, ER = R / 32;
   __shared__ uint8_t buf[4][KH];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const size_t wid = (size_t)blockIdx.x * 4 + warp;
-  if (wid < (size_t)v.B * n_new) {
+  for (size_t wid = (size_t)blockIdx.x * 4 + warp; wid < (size_t)v.B * n_new;
+       wid += (size_t)gridDim.x * 4) {
     const int i = (int)(wid % n_new), b = (int)(wid / n_new);
     const int nb = seq_count(n_per_seq, b, n_new, err);
     const int t = v.lens[b] + i;
@@ -522,6 +844,7 @@ __global__ void __launch_bounds__(128)
         }
       }
     }
+    __syncwarp();  // the row buffer is free again
   }
   __syncthreads();
   __shared__ int last;
@@ -539,13 +862,27 @@ __global__ void __launch_bounds__(128)
   }
 }
 
+// CTAs of `wpc` row warps for `rows` rows: one per wpc rows, up to 2048
+// threads per SM of the current device; the kernels loop over the rest
+unsigned row_blocks(size_t rows, int wpc = 4) {
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+      sms = 148;
+  }
+  const size_t need = (rows + wpc - 1) / wpc, cap = (size_t)sms * (64 / wpc);
+  return (unsigned)(need < cap ? (need > 0 ? need : 1) : cap);
+}
+
 }  // namespace
 
 cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, int in_f32,
                               int n_new, const int32_t *n_per_seq, int32_t *err,
                               cudaStream_t st) {
   const size_t rows = (size_t)v.B * n_new * v.Hkv;
-  const unsigned blocks = (unsigned)((rows + 3) / 4);
+  const unsigned blocks = row_blocks(rows);
   const bool kpc = v.bits != 16 && v.key_axis == 1;
   const bool d128 = v.D == 128;
   cudaError_t e = cudaSuccess;
@@ -558,7 +895,19 @@ cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, i
                    v, k, in_f32, n_new, n_per_seq, err, max_groups);
   }
   if (e == cudaSuccess) {
-    if (!kpc && (size_t)n_new * v.Hkv <= 64)
+    const dim3 bg(row_blocks(rows, 8));
+    if (!kpc && (size_t)n_new * v.Hkv > 64 && d128 && rows < (1u << 31) &&
+        (v.bits == 16 || v.bits == 8 || v.bits == 4)) {
+      // bulk appends of the per-token layouts with head_dim 128
+      const bool sym = v.scheme == kSchemeSym;
+      auto bulk = [&](auto kern) {
+        return launch_pdl(kern, bg, dim3(256), 0, st, v, k, vv, in_f32, n_new, n_per_seq, err);
+      };
+      if (v.bits == 16) e = bulk(gqa_append_bulk<16, 64, false>);
+      else if (sym) e = v.bits == 8 ? bulk(gqa_append_bulk<8, 64, true>) : bulk(gqa_append_bulk<4, 64, true>);
+      else if (v.bits == 8) e = v.group == 32 ? bulk(gqa_append_bulk<8, 32, false>) : bulk(gqa_append_bulk<8, 64, false>);
+      else e = v.group == 32 ? bulk(gqa_append_bulk<4, 32, false>) : bulk(gqa_append_bulk<4, 64, false>);
+    } else if (!kpc && (size_t)n_new * v.Hkv <= 64)
       e = launch_pdl(d128 ? gqa_append_seq<128> : gqa_append_seq<64>, dim3(v.B), dim3(256), 0, st,
                      v, k, vv, in_f32, n_new, n_per_seq, err);
     else
@@ -575,7 +924,7 @@ cudaError_t launch_mla_append(const MlaView &v, const void *c, const void *kr, i
                               int n_new, const int32_t *n_per_seq, int32_t *err,
                               cudaStream_t st) {
   const size_t rows = (size_t)v.B * n_new;
-  const dim3 grid((unsigned)((rows + 3) / 4));
+  const dim3 grid(row_blocks(rows));
   const uint16_t *cc = static_cast<const uint16_t *>(c), *kk = static_cast<const uint16_t *>(kr);
   if (v.bits != 16) {
     if (v.rope != 64) return cudaErrorInvalidValue;

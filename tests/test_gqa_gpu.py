@@ -241,3 +241,55 @@ def test_per_channel_keys_one_position_at_a_time():
     assert torch.equal(ea["k_residual"][:, :, :6], eb["k_residual"][:, :, :6])
     q = torch.randn((2, 4, 128)).to(torch.bfloat16).cuda()
     assert torch.equal(a.decode(0, q, 0.1, n_splits=1), b.decode(0, q, 0.1, n_splits=1))
+
+
+def _tie_rows(B, n, Hkv, D, group, levels, symmetric, seed):
+    """Rows whose quantiser quotients land exactly on half-integers and one
+    float32 ulp either side of them: each group (or row, for the symmetric
+    quantiser) spans a range that makes the scale a power of two, so
+    (x - min) / scale or x / scale is exactly k + 1/2 for the tie channels."""
+    rng = np.random.default_rng(seed)
+    x = np.zeros((B, n, Hkv, D), np.float32)
+    span = D if symmetric else group
+    for idx in np.ndindex(B, n, Hkv):
+        e = float(2.0 ** rng.integers(-6, 6))
+        for g0 in range(0, D, span):
+            k = rng.integers(0, levels, size=span).astype(np.float32)
+            vals = (k + 0.5) * e
+            if symmetric:
+                vals *= rng.choice([-1.0, 1.0], size=span).astype(np.float32)
+                vals[0], vals[1] = levels * e, -levels * e   # max |x| = q 2^e: scale 2^e
+                base = 0.0
+            else:
+                base = float(rng.normal()) * 4.0 * e
+                vals[0], vals[1] = 0.0, levels * e            # range = levels 2^e: scale 2^e
+            nudge = rng.integers(-1, 2, size=span)            # a third exact, a third 1 ulp off
+            vals = np.where(nudge > 0, np.nextafter(vals, np.float32(np.inf)),
+                            np.where(nudge < 0, np.nextafter(vals, np.float32(-np.inf)), vals))
+            vals[0] = 0.0 if not symmetric else vals[0]
+            vals[1] = levels * e if not symmetric else vals[1]
+            x[idx][g0:g0 + span] = (np.float32(base) + vals.astype(np.float32)) if not symmetric else vals
+    return x
+
+
+@pytest.mark.parametrize("fmt", [dict(bits=4, group=32, key_axis="token"),
+                                 dict(bits=8, group=64, key_axis="token"),
+                                 dict(bits=4, scheme="symmetric"), dict(bits=8, scheme="symmetric")],
+                         ids=["int4g32", "int8g64", "sym4", "sym8"])
+def test_append_rounding_ties(fmt):
+    # float32 inputs exactly on the quantiser's rounding boundaries (and one
+    # ulp away): the codes must still equal the oracle's (round half to even
+    # of the correctly rounded quotient), on the bulk append path
+    B, Hkv, D, n = 2, 2, 128, 40
+    sym = fmt.get("scheme") == "symmetric"
+    levels = (1 << (fmt["bits"] - 1)) - 1 if sym else (1 << fmt["bits"]) - 1
+    group = fmt.get("group", D)
+    k = _tie_rows(B, n, Hkv, D, group, levels, sym, seed=fmt["bits"] + 10 * sym)
+    v = _tie_rows(B, n, Hkv, D, group, levels, sym, seed=fmt["bits"] + 10 * sym + 1)
+    c = _cache(B, 4, Hkv, D, n, [dict(**fmt)])
+    c.append(0, torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda())
+    lens = np.full(B, n)
+    cfg = dict(fmt, key_axis="token")
+    st = oracle_state(k, v, lens, cfg)
+    check_codes(c.export(0), st, lens, cfg)
+    assert c.device_error() == 0
