@@ -459,7 +459,7 @@ def main():
                          "quantiser at this bit-width")
     ap.add_argument("--profile-case",
                     choices=["gqa", "kpc", "mla", "mla64", "gather", "sym", "evict", "evict-small",
-                             "prefill", "prefill-small", "append"],
+                             "prefill", "prefill-small", "append", "mlaq", "mlaq64"],
                     default=None,
                     help="small ncu case: decode (or eviction) launches only, no timing line")
     ap.add_argument("--prefill", action="store_true",
@@ -1025,7 +1025,8 @@ def profile_case(kind):
     the 14B step shape (B=32, 8 kv / 40 q heads, d_h 128, T=8192; 1.5 GB of
     cache, both anchors larger than L2); each decode runs 3 times in the order
     int4, bf16.  mla / mla64: one d=512 (302 MB) / d=64 (67 MB) latent layer
-    at B=64, T=4096.
+    at B=64, T=4096; mlaq / mlaq64: the same layer stored with the symmetric
+    8-bit quantiser (152 / 35 MB).  append: bulk appends at the 14B shape.
     gather: one int4 g32 anchor at B=4, T=131072 with a kept list of T/8
     positions per sequence (805 MB cache, 101 MB read per decode), 3 decodes.
     sym: one symmetric anchor of each bit-width (8, 4, 2) at the 14B step
@@ -1121,11 +1122,15 @@ def profile_case(kind):
         for _ in range(3):
             c.decode(0, q, w.sigma)
     else:
-        width = 64 if kind == "mla64" else 512
+        # mla / mla64: one bf16 latent layer of width 512 / 64; mlaq / mlaq64:
+        # the same stored with the symmetric 8-bit quantiser (B=64, T=4096)
+        width = 64 if kind.endswith("64") else 512
+        bits = 8 if kind.startswith("mlaq") else 16
         w = W.config(4, n_layers=1)
         w.layers[0]["width"] = width
         c = Cache(kind="mla", n_layers=1, n_q_heads=16, head_dim=128, latent_dim=512, rope_dim=64,
-                  max_batch=w.batch, max_ctx=w.context, layers=[Layer(bits=16, width=width)])
+                  max_batch=w.batch, max_ctx=w.context,
+                  layers=[Layer(bits=bits, width=width, scheme="symmetric")])
         cl, kr = W.mla_inputs(w, 0, 0, w.context, device="cuda")
         c.append(0, cl, kr)
         wk, wv = W.mla_weights(w, 0, device="cuda")
