@@ -244,7 +244,9 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
  * 0 .. len_b - n_q + i of the dequantised stored keys and values (the ones
  * decode reads), with its own query heads (an inheriting layer reads its
  * anchor).  Queries before position 0 (len_b < n_q) give zeros.  Kept lists
- * are not used: pre-fill reads every position.
+ * are not used: pre-fill reads every position.  Keys with per-channel groups
+ * are read as decode reads them: complete groups of positions from their
+ * codes and the group plane, the open group from the bf16 residual.
  *  q:       device [B, n_q, H_q, head_dim] in q_dtype (post-RoPE),
  *           16-byte aligned;
  *  out:     device float32 [B, n_q, H_q, head_dim], 16-byte aligned;
@@ -252,7 +254,7 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
  *           bytes: per-row softmax statistics and the anchor's cache
  *           dequantised once into the products' operand layout (1 KB per
  *           position and KV head for quantised anchors, 512 B for bf16).
- * Errors: UNSUPPORTED (MLA, head_dim != 128, grouped per-channel keys),
+ * Errors: UNSUPPORTED (MLA, head_dim != 128),
  * INVALID_ARG (n_q outside [1, max_ctx], null or misaligned pointers,
  * scale not finite and positive, scratch too small). */
 kvk_status kvk_prefill_scratch_size(const kvk_cache *cache, int32_t layer, int32_t n_q,

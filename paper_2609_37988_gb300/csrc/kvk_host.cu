@@ -654,9 +654,6 @@ kvk_status check_prefill(const kvk_cache *c, int32_t layer, int32_t n_q) {
   if (s) return s;
   if (c->desc.kind != KVK_KIND_GQA) return fail(KVK_ERR_UNSUPPORTED, "pre-fill on an MLA cache");
   if (c->desc.head_dim != 128) return fail(KVK_ERR_UNSUPPORTED, "pre-fill needs head_dim 128");
-  const kvk_layer_cfg &L = c->cfg[c->src[layer]];
-  if (L.bits != 16 && L.key_axis == KVK_AXIS_CHANNEL && L.scheme != KVK_QUANT_SYMMETRIC)
-    return fail(KVK_ERR_UNSUPPORTED, "pre-fill over per-channel key groups");
   if (n_q < 1 || n_q > c->desc.max_ctx)
     return fail(KVK_ERR_INVALID_ARG, "n_q %d outside [1, max_ctx]", n_q);
   return KVK_OK;

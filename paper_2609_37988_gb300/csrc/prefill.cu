@@ -53,6 +53,7 @@ constexpr int kPfBarBytes = 320;             // barriers and the CTA's shared wo
 struct PfPlan {
   int n_rb, n_jobs, grid, n_t64;
   int q_lo, k_lo, fmt, gshift;
+  int kpc;            // keys with per-channel groups (codes + group plane + residual)
   int ks16, nrec;
   uint32_t nc_magic;  // expand: ceil(2^32 / nrec), e / nrec = umulhi(e, nc_magic)
   int b_stride;       // expand: staged record stride (odd multiple of 16 bytes)
@@ -108,6 +109,20 @@ __global__ void __launch_bounds__(kPfWorkers) prefill_expand_kernel(const PfArgs
       const bool ok = t < len;
       cp_async4(stg + pos * p.b_stride + v.rec_bytes, v.scales + (size_t)unit * v.cap + (ok ? t : t0), ok);
     }
+  // per-channel keys: the (scale, zero) rows of the tile's complete groups
+  // of positions (kPfT >> gshift groups of 128 channels; rows of the open
+  // group are zero and unused: those positions come from the residual)
+  const int g0 = t0 >> p.gshift, full = (len >> p.gshift) << p.gshift;
+  float2 *mrows = reinterpret_cast<float2 *>(stg + kPfT * p.b_stride);
+  if (p.kpc) {
+    const int ng = kPfT >> p.gshift;
+    for (int i = tid; i < ng * 128 * 8 / 16; i += kPfWorkers) {
+      const int gi = i / 64, c = i - gi * 64;  // 64 chunks of 16 bytes per row
+      const bool ok = ((g0 + gi) << p.gshift) < full;
+      const float2 *src = v.gmeta + ((size_t)unit * (v.cap >> p.gshift) + (ok ? g0 + gi : 0)) * 128;
+      cp_async16(reinterpret_cast<uint8_t *>(mrows) + 16 * i, reinterpret_cast<const uint8_t *>(src) + 16 * c, ok);
+    }
+  }
   cp_async_commit();
   cp_async_wait<0>();
   __syncthreads();
@@ -117,7 +132,29 @@ __global__ void __launch_bounds__(kPfWorkers) prefill_expand_kernel(const PfArgs
   const int ks = 16 * p.ks16;
   const int mb = (p.nrec * 16 - 2 * ks) / 2;  // grouped: one metadata block
   uint8_t *kh = sm, *kl = sm + 2 * kPfBox;
-  if (part < 4) {
+  if (part < 4 && p.kpc) {
+    // per-channel keys: complete groups from codes and the group rows, the
+    // open group from the bf16 residual (row t mod g), zero past the length
+    const int t = t0 + pidx;
+    if (t < full) {
+      const float2 *mr = mrows + ((t >> p.gshift) - g0) * 128;
+      if (p.fmt == kFmtG8)
+        tc_dequant_kpc<8, kPfBox>(bundle, mr, pidx, part, kh, kl);
+      else
+        tc_dequant_kpc<4, kPfBox>(bundle, mr, pidx, part, kh, kl);
+    } else {
+      const uint4 z = make_uint4(0, 0, 0, 0);
+      if (t < len) {
+        const uint8_t *res = v.resid + ((size_t)unit * ((size_t)1 << p.gshift) + (t & ((1 << p.gshift) - 1))) * 256;
+        tc_dequant<kFmtBf16, kPfBox>(res, nullptr, pidx, part, p.gshift, kh, kl);
+      } else {
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) put_chunk(kh, pidx, 32 * part + 8 * cc, kPfBox, z);
+      }
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) put_chunk(kl, pidx, 32 * part + 8 * cc, kPfBox, z);
+    }
+  } else if (part < 4) {
     const uint8_t *kmeta = sym ? bundle + v.rec_bytes : bundle + 2 * ks;
     switch (p.fmt) {
       case kFmtBf16: tc_dequant<kFmtBf16, kPfBox>(bundle, kmeta, pidx, part, p.gshift, kh, kl); break;
@@ -130,7 +167,7 @@ __global__ void __launch_bounds__(kPfWorkers) prefill_expand_kernel(const PfArgs
   } else {
     const int qc = part - 4;
     uint8_t *vh = sm + p.kbytes, *vl = vh + 2 * kPfBox;
-    const uint8_t *vsec = bundle + ks, *vmeta = bundle + 2 * ks + mb;
+    const uint8_t *vsec = bundle + ks, *vmeta = bundle + 2 * ks + (p.kpc ? 0 : mb);
     const float svs =
         sym ? __uint_as_float(*reinterpret_cast<const uint32_t *>(bundle + v.rec_bytes) & 0xFFFF0000u) : 0.f;
     switch (p.fmt) {
@@ -623,6 +660,7 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
           : a.v.scheme == kSchemeSym ? (a.v.bits == 8 ? kFmtS8 : a.v.bits == 4 ? kFmtS4 : kFmtS2)
                                      : (a.v.bits == 8 ? kFmtG8 : kFmtG4);
   p.gshift = a.v.group == 64 ? 6 : 5;
+  p.kpc = a.v.bits != 16 && a.v.key_axis == 1 ? 1 : 0;
   p.ks16 = TcFmtKs16(p.fmt);
   p.nrec = a.v.rec_bytes / 16;
   p.nc_magic = (uint32_t)((0x100000000ull + p.nrec - 1) / p.nrec);
@@ -631,7 +669,8 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   p.b_stride = 16 * (bchunks % 2 ? bchunks : bchunks + 1);
   p.kbytes = 2 * kPfBox * (p.k_lo ? 2 : 1);
   p.tbytes = 2 * p.kbytes;
-  p.smem_x = p.tbytes + kPfT * p.b_stride + 1024;
+  // + the (scale, zero) rows of the tile's position groups (per-channel keys)
+  p.smem_x = p.tbytes + kPfT * p.b_stride + (p.kpc ? 2 * 128 * 8 : 0) + 1024;
   const int vb = out ? p.tbytes - p.kbytes : 0;
   const int nbytes = out ? kPfRows * 4 : 0;
   const int rbytes = out ? 0 : 4 * kPfRows * 8;

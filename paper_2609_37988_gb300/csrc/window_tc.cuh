@@ -153,6 +153,48 @@ __device__ __forceinline__ void tc_dequant(const uint8_t *bundle, const uint8_t 
   }
 }
 
+// The same for keys with per-channel groups (KIVI layout): the position's
+// codes (K section in the same channel order as per-token codes) and the
+// (scale, zero) of each channel for the position's group of positions, mrow
+// [128] float2.
+template <int BITS, int KBOX = 128 * 128>
+__device__ __forceinline__ void tc_dequant_kpc(const uint8_t *bundle, const float2 *mrow, int row,
+                                               int qc, uint8_t *kh, uint8_t *kl) {
+  static_assert(BITS == 8 || BITS == 4, "per-channel keys: 8- or 4-bit codes");
+  constexpr int D = 128;
+  const uint32_t *bw = reinterpret_cast<const uint32_t *>(bundle);
+  constexpr int NW = BITS == 8 ? 8 : 4;
+  uint32_t w[NW];
+  if constexpr (BITS == 8) {
+    const int ob = 16 * (qc >> 1) + 2 * (qc & 1);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const uint2 u = *reinterpret_cast<const uint2 *>(bw + 4 * c + ob);
+      w[2 * c] = u.x; w[2 * c + 1] = u.y;
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < 4; ++c) w[c] = bw[4 * c + qc];
+  }
+#pragma unroll
+  for (int cc = 0; cc < 4; ++cc) {
+    const int ch0 = 32 * qc + 8 * cc;
+    float x[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int l = 8 * cc + i;  // channel of quarter 0
+      int byte, hi;
+      k_pos(l, BITS, D, &byte, &hi);
+      const int wi = BITS == 8 ? 2 * (byte >> 4) + ((byte & 15) >> 2) : byte >> 4;
+      const int sh = 8 * (byte & 3) + 4 * hi;
+      const uint32_t u = (w[wi] >> sh) & ((1u << BITS) - 1u);
+      const float2 m = mrow[ch0 + i];
+      x[i] = fmaf(u2f(u), m.x, m.y);
+    }
+    put8(kh, kl, true, row, ch0, KBOX, x);
+  }
+}
+
 // Channels 32 qc .. 32 qc + 31 of one position's value, from the V section
 // of its staged record (logical order, rotation undone) and its metadata
 // (grouped: the (scale, zero) pairs of the value groups; symmetric: the

@@ -23,11 +23,13 @@ FORMATS = [
     dict(bits=8, group=64, key_axis="token", scheme="symmetric"),
     dict(bits=4, group=64, key_axis="token", scheme="symmetric"),
     dict(bits=2, group=64, key_axis="token", scheme="symmetric"),
+    dict(bits=8, group=64, key_axis="channel"),
+    dict(bits=4, group=32, key_axis="channel"),
 ]
 
 
 def _fid(f):
-    return f"{f.get('scheme', 'grouped')[:3]}{f['bits']}g{f['group']}"
+    return f"{f.get('scheme', 'grouped')[:3]}{f['bits']}g{f['group']}{'-kpc' if f['key_axis'] == 'channel' else ''}"
 
 
 def _cache(B, Hq, Hkv, T, layers):
@@ -75,7 +77,7 @@ def test_prefill_parity(fmt, G, n_q):
     assert c.device_error() == 0
 
 
-@pytest.mark.parametrize("fmt", [FORMATS[0], FORMATS[2], FORMATS[6]], ids=_fid)
+@pytest.mark.parametrize("fmt", [FORMATS[0], FORMATS[2], FORMATS[6], FORMATS[9]], ids=_fid)
 def test_prefill_long_chunk_many_tiles(fmt):
     # a 256-query chunk over 1000 positions: 1280 rows (ten row blocks) per
     # unit, 16 tiles of 64 positions for the last block
@@ -108,8 +110,6 @@ def test_prefill_rejections():
     from paper_2609_37988_gb300._lib import KVKError
     c = _cache(2, 4, 2, 300, [dict(bits=8, group=64, key_axis="channel"), dict(bits=16)])
     q = torch.zeros((2, 8, 4, 128), dtype=torch.bfloat16, device="cuda")
-    with pytest.raises(KVKError):
-        c.prefill(0, q, 0.1)  # per-channel key groups
     with pytest.raises(KVKError):
         c.prefill(1, q, 0.0)  # scale
     with pytest.raises(KVKError):
