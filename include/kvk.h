@@ -254,7 +254,7 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
  *           bytes: per-row softmax statistics and the anchor's cache
  *           dequantised once into the products' operand layout (1 KB per
  *           position and KV head for quantised anchors, 512 B for bf16).
- * Errors: UNSUPPORTED (MLA, head_dim != 128),
+ * Errors: UNSUPPORTED (MLA: see kvk_prefill_attention_mla; head_dim != 128),
  * INVALID_ARG (n_q outside [1, max_ctx], null or misaligned pointers,
  * scale not finite and positive, scratch too small). */
 kvk_status kvk_prefill_scratch_size(const kvk_cache *cache, int32_t layer, int32_t n_q,
@@ -262,6 +262,30 @@ kvk_status kvk_prefill_scratch_size(const kvk_cache *cache, int32_t layer, int32
 kvk_status kvk_prefill_attention(kvk_cache *cache, int32_t layer, const void *q, int32_t q_dtype,
                                  int32_t n_q, float softmax_scale, float *out, void *scratch,
                                  size_t scratch_bytes, kvk_stream stream);
+
+/* Causal chunk attention (pre-fill) of MLA layer `layer` over its latent
+ * cache (bf16 or quantised, at its kept width d): the chunk is the last n_q
+ * positions of every sequence, already written with kvk_append; query i of
+ * sequence b, at position len_b - n_q + i, attends to positions 0 .. itself
+ * with the absorbed query of each head (Appendix C.2, as
+ * kvk_decode_attention_mla: q_lat = W_UK[h][:, :d]^T q_nope, scores
+ * sigma (q_lat . c[:d] + q_pe . k^R), output W_UV[h][:, :d] o_lat).  Each
+ * query row runs the decode path over its own causal prefix (one CTA per
+ * row).  Queries before position 0 give zeros.
+ *  q_nope:  device bf16 [B, n_q, H, head_dim]; q_pe: bf16 [B, n_q, H, rope]
+ *           (post-RoPE);
+ *  w_uk, w_uv: device bf16 [H, head_dim, latent] as for decode;
+ *  out:     device float32 [B, n_q, H, head_dim];
+ *  scratch: device, 256-byte aligned, at least kvk_prefill_scratch_size
+ *           bytes (which answers for MLA layers too): the rows' absorbed
+ *           queries and latent partials;
+ * all 16-byte aligned.  Errors: INVALID_ARG (not an MLA cache, n_q outside
+ * [1, max_ctx], null or misaligned pointers, scale not finite and positive,
+ * scratch too small). */
+kvk_status kvk_prefill_attention_mla(kvk_cache *cache, int32_t layer, const void *q_nope,
+                                     const void *q_pe, const void *w_uk, const void *w_uv,
+                                     int32_t n_q, float softmax_scale, float *out, void *scratch,
+                                     size_t scratch_bytes, kvk_stream stream);
 
 /* Copy anchor `layer`'s kept lists out, device to device, on `stream`.
  * *per_head (host) = -1: no list installed (nothing copied); 0: lists per

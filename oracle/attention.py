@@ -24,6 +24,10 @@ Everything here runs in float64 on already-dequantised caches.
   ``W_UK^h[:, :d] c[:d]`` and value ``W_UV^h[:, :d] c[:d]`` explicitly; the
   score adds ``<q_pe^h, k^R>``.  The GPU computes the absorbed form; the
   algebraic identity between the two is pinned by a test.
+* ``mla_prefill_unabsorbed`` -- the chunk attention of an MLA layer: query
+  ``i`` of the chunk (the last ``C`` positions of each sequence) at position
+  ``len - C + i`` attends causally to positions ``0 .. len - C + i`` with the
+  explicitly reconstructed keys and values of ``mla_decode_unabsorbed``.
 """
 from __future__ import annotations
 
@@ -151,4 +155,36 @@ def mla_decode_unabsorbed(q_nope, q_pe, c, k_r, w_uk, w_uv, d, lens, sigma):
             Vh = C @ Wv.T                                 # [T, Dv] values
             s = sigma * (Kc @ q_nope[b, h] + KR @ q_pe[b, h])
             out[b, h] = softmax_weights(s) @ Vh
+    return out
+
+
+def mla_prefill_unabsorbed(q_nope, q_pe, c, k_r, w_uk, w_uv, d, lens, sigma):
+    """MLA chunk attention, content keys and values reconstructed explicitly.
+
+    q_nope : ``[B, C, H, Dn]``   q_pe : ``[B, C, H, dR]`` (post-RoPE), the
+             queries of each sequence's last ``C`` positions
+    c, k_r, w_uk, w_uv : as for ``mla_decode_unabsorbed``; ``lens`` the
+             positions held (the chunk included)
+    Returns ``[B, C, H, Dv]`` float64; queries before position 0 give zeros.
+    """
+    q_nope = np.asarray(q_nope, np.float64)
+    q_pe = np.asarray(q_pe, np.float64)
+    B, C, H, _ = q_nope.shape
+    Dv = w_uv.shape[1]
+    out = np.zeros((B, C, H, Dv), np.float64)
+    for b in range(B):
+        L = int(lens[b])
+        Cb = np.asarray(c[b, :L, :d], np.float64)           # [L, d]
+        KR = np.asarray(k_r[b, :L], np.float64)             # [L, dR]
+        for h in range(H):
+            Wk = np.asarray(w_uk[h, :, :d], np.float64)     # [Dn, d]
+            Wv = np.asarray(w_uv[h, :, :d], np.float64)     # [Dv, d]
+            Kc = Cb @ Wk.T                                  # [L, Dn] content keys
+            Vh = Cb @ Wv.T                                  # [L, Dv] values
+            for i in range(C):
+                p = L - C + i  # position of query i
+                if p < 0:
+                    continue
+                s = sigma * (Kc[:p + 1] @ q_nope[b, i, h] + KR[:p + 1] @ q_pe[b, i, h])
+                out[b, i, h] = softmax_weights(s) @ Vh[:p + 1]
     return out

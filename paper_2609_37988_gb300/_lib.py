@@ -66,6 +66,7 @@ _SIGS = {
     "kvk_export_kept": [_P, _I, _P, _P, ctypes.POINTER(_I), _P],
     "kvk_prefill_scratch_size": [_P, _I, _I, ctypes.POINTER(_SZ)],
     "kvk_prefill_attention": [_P, _I, _P, _I, _I, _F, _P, _P, _SZ, _P],
+    "kvk_prefill_attention_mla": [_P, _I, _P, _P, _P, _P, _I, _F, _P, _P, _SZ, _P],
     "kvk_rewind": [_P, _I, _P],
     "kvk_decode_plan_splits": [_P, _I, ctypes.POINTER(_I)],
     "kvk_decode_attention": [_P, _I, _P, _I, _F, _P, _I, _P],

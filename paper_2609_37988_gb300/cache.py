@@ -203,6 +203,30 @@ class Cache:
         self._prefill_scratch = scratch  # kept alive until the stream is done with it
         return out
 
+    def prefill_mla(self, layer: int, q_nope: torch.Tensor, q_pe: torch.Tensor, w_uk: torch.Tensor,
+                    w_uv: torch.Tensor, scale: float, out: torch.Tensor = None, stream=None) -> torch.Tensor:
+        """MLA causal chunk attention: ``q_nope`` ``[B, n_q, H, head_dim]`` and
+        ``q_pe`` ``[B, n_q, H, rope_dim]`` (bf16), the queries of each
+        sequence's last ``n_q`` positions (appended first); returns float32
+        ``[B, n_q, H, head_dim]``."""
+        for t, n in ((q_nope, "q_nope"), (q_pe, "q_pe"), (w_uk, "w_uk"), (w_uv, "w_uv")):
+            _need(t, n)
+        d = self.desc
+        if q_nope.dim() != 4 or (q_nope.shape[0], q_nope.shape[2], q_nope.shape[3]) != \
+                (d.max_batch, d.n_q_heads, d.head_dim) or q_pe.shape != q_nope.shape[:3] + (d.rope_dim,):
+            raise ValueError("q_nope must be [max_batch, n_q, n_q_heads, head_dim], q_pe [.., rope_dim]")
+        n_q = q_nope.shape[1]
+        if out is None:
+            out = torch.empty(q_nope.shape, dtype=torch.float32, device=q_nope.device)
+        nbytes = ctypes.c_size_t()
+        check(self.lib.kvk_prefill_scratch_size(self.handle, layer, n_q, ctypes.byref(nbytes)))
+        scratch = torch.empty(nbytes.value, dtype=torch.uint8, device=self.device)
+        check(self.lib.kvk_prefill_attention_mla(self.handle, layer, _ptr(q_nope), _ptr(q_pe), _ptr(w_uk),
+                                                 _ptr(w_uv), n_q, float(scale), _ptr(out), _ptr(scratch),
+                                                 nbytes.value, _stream(stream)))
+        self._prefill_scratch = scratch  # kept alive until the stream is done with it
+        return out
+
     def kept_lists(self, layer: int, stream=None):
         """Installed kept lists: ``(idx, n, per_head)`` device tensors shaped
         per head ``[B, H_kv, cap]`` / ``[B, H_kv]`` (or per sequence), or

@@ -31,7 +31,18 @@ struct MlaView {
   int B, width, rope, rec_bytes;
   int bits;            // 16, or 8 / 4 / 2 for quantised latents
   int scheme;          // kSchemeGrouped or kSchemeSym (quantised latents)
+  // 0: decode, one query row per sequence.  n > 0: pre-fill, n query rows
+  // per sequence: row b n + i is query i of sequence b, at position
+  // lens[b] - n + i, attending to positions 0 .. itself
+  int n_q = 0;
 };
+// query rows of an MLA launch, and for row vb its sequence and the positions it reads
+__host__ __device__ __forceinline__ int mla_rows(const MlaView &v) { return v.n_q ? v.B * v.n_q : v.B; }
+__device__ __forceinline__ int mla_row_seq(const MlaView &v, int vb) { return v.n_q ? vb / v.n_q : vb; }
+__device__ __forceinline__ int mla_row_len(const MlaView &v, int vb, int b) {
+  const int L = v.lens[b];
+  return v.n_q ? max(0, min(L, L - v.n_q + (vb - b * v.n_q) + 1)) : L;
+}
 
 struct GqaDecodeArgs {
   GqaView v;

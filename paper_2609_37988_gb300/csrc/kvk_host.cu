@@ -676,7 +676,40 @@ PrefillScratch prefill_scratch(const kvk_cache *c, int32_t layer, int32_t n_q) {
 }
 }  // namespace
 
+namespace {
+// MLA pre-fill scratch: the absorbed queries of every query row, then the
+// rows' latent partials (one split)
+struct MlaPrefillScratch {
+  size_t qlat, partial, total;
+};
+MlaPrefillScratch mla_prefill_scratch(const kvk_cache *c, int32_t layer, int32_t n_q) {
+  const int a = c->src[layer];
+  const size_t rows = (size_t)c->desc.max_batch * n_q * c->desc.n_q_heads;
+  const int W = c->cfg[a].width;
+  MlaPrefillScratch p;
+  p.qlat = 0;
+  p.partial = (size_t)align256((int64_t)(rows * (2 * W + c->desc.rope_dim) * 2));
+  p.total = p.partial + rows * (W + 2) * 4;
+  return p;
+}
+kvk_status check_prefill_mla(const kvk_cache *c, int32_t layer, int32_t n_q) {
+  kvk_status s = check_layer_index(c, layer);
+  if (s) return s;
+  if (c->desc.kind != KVK_KIND_MLA) return fail(KVK_ERR_INVALID_ARG, "cache is not MLA");
+  if (n_q < 1 || n_q > c->desc.max_ctx)
+    return fail(KVK_ERR_INVALID_ARG, "n_q %d outside [1, max_ctx]", n_q);
+  return KVK_OK;
+}
+}  // namespace
+
 kvk_status kvk_prefill_scratch_size(const kvk_cache *c, int32_t layer, int32_t n_q, size_t *bytes) {
+  if (c && c->desc.kind == KVK_KIND_MLA) {
+    kvk_status s = check_prefill_mla(c, layer, n_q);
+    if (s) return s;
+    if (!bytes) return fail(KVK_ERR_INVALID_ARG, "null output");
+    *bytes = mla_prefill_scratch(c, layer, n_q).total;
+    return KVK_OK;
+  }
   kvk_status s = check_prefill(c, layer, n_q);
   if (s) return s;
   if (!bytes) return fail(KVK_ERR_INVALID_ARG, "null output");
@@ -912,6 +945,48 @@ kvk_status kvk_decode_attention_mla(kvk_cache *c, int32_t layer, const void *q_n
   args.wait_limit = c->wait_limit;
   cudaError_t e = launch_mla_decode(args, reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "MLA decode launch");
+  return KVK_OK;
+}
+
+
+kvk_status kvk_prefill_attention_mla(kvk_cache *c, int32_t layer, const void *q_nope,
+                                     const void *q_pe, const void *w_uk, const void *w_uv,
+                                     int32_t n_q, float softmax_scale, float *out, void *scratch,
+                                     size_t scratch_bytes, kvk_stream stream) {
+  kvk_status s = check_prefill_mla(c, layer, n_q);
+  if (s) return s;
+  if (!q_nope || !q_pe || !w_uk || !w_uv || !out || !aligned16(q_nope) || !aligned16(q_pe) ||
+      !aligned16(w_uk) || !aligned16(w_uv) || !aligned16(out))
+    return fail(KVK_ERR_INVALID_ARG, "null or misaligned MLA operand");
+  if (!std::isfinite(softmax_scale) || !(softmax_scale > 0.f))
+    return fail(KVK_ERR_INVALID_ARG, "softmax scale must be finite and positive");
+  const MlaPrefillScratch ps = mla_prefill_scratch(c, layer, n_q);
+  if (!scratch || (reinterpret_cast<uintptr_t>(scratch) & 255u) || scratch_bytes < ps.total)
+    return fail(KVK_ERR_INVALID_ARG, "scratch null, not 256-byte aligned or smaller than %zu bytes",
+                ps.total);
+  const int a = c->src[layer];
+  MlaDecodeArgs args;
+  args.v = c->mla_view(a);
+  args.v.n_q = n_q;  // query row b n_q + i: query i of sequence b over its causal prefix
+  args.tmap = c->tmap[a].bytes;
+  args.q_nope = q_nope;
+  args.q_pe = q_pe;
+  args.w_uk = w_uk;
+  args.w_uv = w_uv;
+  args.H = c->desc.n_q_heads;
+  args.Dn = c->desc.head_dim;
+  args.r = c->desc.latent_dim;
+  args.sig_log2 = softmax_scale * 1.4426950408889634f;
+  args.n_splits = 1;  // every row's prefix in one CTA (rows are plentiful)
+  args.items_per_split = layer_tiles(c, a) * kTile;
+  args.qlat = reinterpret_cast<uint16_t *>(static_cast<uint8_t *>(scratch) + ps.qlat);
+  args.partial = reinterpret_cast<float *>(static_cast<uint8_t *>(scratch) + ps.partial);
+  args.olat = nullptr;
+  args.out = out;
+  args.err = c->err();
+  args.wait_limit = c->wait_limit;
+  cudaError_t e = launch_mla_decode(args, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "MLA pre-fill launch");
   return KVK_OK;
 }
 

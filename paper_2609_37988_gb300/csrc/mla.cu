@@ -125,9 +125,10 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
   float *lsum = red + 4 * kHeads;                           // [4 warps][16]
   uint8_t *q_s = sm + C::OFF_Q;
 
-  const int split = blockIdx.x, b = blockIdx.y;
+  const int split = blockIdx.x, vb = blockIdx.y;  // vb: the query row (decode: sequence)
+  const int b = mla_row_seq(v, vb);              // the sequence whose cache it reads
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int len = v.lens[b];
+  const int len = mla_row_len(v, vb, b);
   const int i0 = split * items_per_split;
   const int i1 = (split == n_splits - 1) ? len : min(i0 + items_per_split, len);
   const int n_tiles = i1 > i0 ? (i1 - i0 + TR - 1) / TR : 0;
@@ -163,7 +164,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
   if (warp < 5 || warp == 7) {
     pdl_wait();
     constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (unused 64) | lo(W)]
-    const uint16_t *qb = qlat + (size_t)b * H * QROW;
+    const uint16_t *qb = qlat + (size_t)vb * H * QROW;
     // warps 0-4 stage it; the second score warp only waits for it
     for (int q = tid; warp < 5 && q < 32 * (C::KH / 8); q += 160) {  // 16-byte cp.async, zero-filled
       const int n = q / (C::KH / 8), c = q % (C::KH / 8);
@@ -173,7 +174,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
       if (valid)
         src = n >= 16     ? qb + (size_t)h * QROW + C::KH + 8 * c
               : c < W / 8 ? qb + (size_t)h * QROW + 8 * c
-                          : q_pe + ((size_t)b * H + h) * kRope + 8 * (c - W / 8);
+                          : q_pe + ((size_t)vb * H + h) * kRope + 8 * (c - W / 8);
       cp_async16(q_s + (n / 8) * (C::KH / 8 * 128) + c * 128 + (n % 8) * 16, src, valid);
     }
     cp_async_commit();
@@ -400,7 +401,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     if (!failed) {
       tc_fence_after();
       const size_t RS = (size_t)W + 2;
-      const size_t prow_base = ((size_t)split * v.B + b) * H;
+      const size_t prow_base = ((size_t)split * mla_rows(v) + vb) * H;
 #pragma unroll
       for (int h = 0; h < kHeads; ++h) {
         float sum = l_part[h];
@@ -468,7 +469,7 @@ template <int W>
 cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
   using C = MlaCfg<W>;
   if (a.n_splits > 64) return cudaErrorInvalidValue;  // merge weights hold 64 splits
-  const int B = a.v.B;
+  const int B = mla_rows(a.v);  // query rows
   auto k = mla_decode_kernel<W>;
   constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
   static bool attr = false;
@@ -568,7 +569,7 @@ cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st) {
 }
 
 int mla_decode_ctas_per_sm(int width, int bits) {
-  if (bits != 16) return 1;  // quantised latents: 12 warps and ~200 KB of shared memory
+  if (bits != 16) return 1;  // quantised latents: 16 warps and up to 227 KB of shared memory
   switch (width) {
     case 512: return mla_ctas_t<512>();
     case 256: return mla_ctas_t<256>();

@@ -161,9 +161,10 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   float *qsum = reinterpret_cast<float *>(sm + C::OFF_QS);  // [latent, rope][16]
   uint8_t *q_s = sm + C::OFF_Q;
 
-  const int split = blockIdx.x, b = blockIdx.y;
+  const int split = blockIdx.x, vb = blockIdx.y;  // vb: the query row (decode: sequence)
+  const int b = mla_row_seq(v, vb);              // the sequence whose cache it reads
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int len = v.lens[b];
+  const int len = mla_row_len(v, vb, b);
   const int i0 = split * items_per_split;
   const int i1 = (split == n_splits - 1) ? len : min(i0 + items_per_split, len);
   const int n_tiles = i1 > i0 ? (i1 - i0 + TR - 1) / TR : 0;
@@ -201,7 +202,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   if (warp < 5 || warp == 7) {
     pdl_wait();
     constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (64 unused) | lo(W)]
-    const uint16_t *qb = qlat + (size_t)b * H * QROW;
+    const uint16_t *qb = qlat + (size_t)vb * H * QROW;
     auto qdst = [&](int n, int c) { return q_s + (n / 8) * (KH / 8 * 128) + c * 128 + (n % 8) * 16; };
     if (warp < 5) {
       for (int q = tid; q < 32 * (W / 8); q += 160) {  // latent parts: 16-byte cp.async
@@ -214,7 +215,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
         const int h = q / (kRope / 8), c = q % (kRope / 8);
         uint4 hi = make_uint4(0, 0, 0, 0), lo = hi;
         if (h < H) {
-          const uint4 w = *reinterpret_cast<const uint4 *>(q_pe + ((size_t)b * H + h) * kRope + 8 * c);
+          const uint4 w = *reinterpret_cast<const uint4 *>(q_pe + ((size_t)vb * H + h) * kRope + 8 * c);
           const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
           uint32_t hs[4], ls[4];
 #pragma unroll
@@ -586,7 +587,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     if (!failed) {
       tc_fence_after();
       const size_t RS = (size_t)W + 2;
-      const size_t prow_base = ((size_t)split * v.B + b) * H;
+      const size_t prow_base = ((size_t)split * mla_rows(v) + vb) * H;
 #pragma unroll
       for (int h = 0; h < kHeads; ++h) {
         float sum = l_part[h], zs = z_part[h];
@@ -647,7 +648,7 @@ template <int W, int BITS, bool SYM>
 cudaError_t launch_mla_q_t(const MlaDecodeArgs &a, cudaStream_t st) {
   using C = MlaQCfg<W, BITS, SYM>;
   if (a.n_splits > 64) return cudaErrorInvalidValue;  // merge weights hold 64 splits
-  const int B = a.v.B;
+  const int B = mla_rows(a.v);  // query rows
   auto k = mla_decode_q_kernel<W, BITS, SYM>;
   constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
   static bool attr = false;

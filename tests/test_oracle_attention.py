@@ -216,3 +216,44 @@ def test_prefill_first_position_returns_its_value_and_last_query_is_decode():
     # the last query sees every position: one decode step
     np.testing.assert_allclose(got[:, -1], attention.gqa_decode(q[:, -1], K, V, [C], 1.0),
                                rtol=1e-13, atol=1e-13)
+
+
+# ---- MLA chunk (prefill) attention ------------------------------------------
+def _mla_case(seed, B=2, C=5, H=3, Dn=4, dR=2, r=6, d=4, T=11):
+    rng = np.random.default_rng(seed)
+    return (rng.standard_normal((B, C, H, Dn)), rng.standard_normal((B, C, H, dR)),
+            rng.standard_normal((B, T, r)), rng.standard_normal((B, T, dR)),
+            rng.standard_normal((H, Dn, r)), rng.standard_normal((H, Dn + 1, r)), d)
+
+
+def test_mla_prefill_matches_library_causal_sdpa():
+    # per head: keys [W_UK c[:d] ; k^R], queries [q_nope ; q_pe], values
+    # W_UV c[:d]; torch's scaled_dot_product_attention with the causal mask
+    # shifted by the cached prefix, in float64
+    qn, qp, c, kr, wk, wv, d = _mla_case(6)
+    B, C, H, _ = qn.shape
+    T = c.shape[1]
+    lens = [T, T]
+    Kc = np.einsum("hnk,btk->bhtn", wk[:, :, :d], c[:, :, :d])
+    K = np.concatenate([Kc, np.broadcast_to(kr[:, None], (B, H) + kr.shape[1:])], -1)
+    V = np.einsum("hvk,btk->bhtv", wv[:, :, :d], c[:, :, :d])
+    Q = np.concatenate([qn, qp], -1).transpose(0, 2, 1, 3)
+    mask = torch.arange(T)[None, :] <= (T - C + torch.arange(C))[:, None]
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(np.ascontiguousarray(Q)), torch.from_numpy(np.ascontiguousarray(K)),
+        torch.from_numpy(V), attn_mask=mask, scale=0.4)
+    got = attention.mla_prefill_unabsorbed(qn, qp, c, kr, wk, wv, d, lens, 0.4)
+    np.testing.assert_allclose(got, ref.permute(0, 2, 1, 3).numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_mla_prefill_short_sequence_and_last_query_is_decode():
+    qn, qp, c, kr, wk, wv, d = _mla_case(7)
+    C = qn.shape[1]
+    lens = [c.shape[1], 3]  # sequence 1: its first C - 3 queries sit before position 0
+    got = attention.mla_prefill_unabsorbed(qn, qp, c, kr, wk, wv, d, lens, 0.5)
+    assert (got[1, :C - 3] == 0).all()
+    dec = attention.mla_decode_unabsorbed(qn[:, -1], qp[:, -1], c, kr, wk, wv, d, lens, 0.5)
+    np.testing.assert_allclose(got[:, -1], dec, rtol=1e-13, atol=1e-13)
+    # query C - 3 of sequence 1 sits at position 0: it returns that position's value
+    np.testing.assert_allclose(got[1, C - 3], np.einsum("hvk,k->hv", wv[:, :, :d], c[1, 0, :d]),
+                               rtol=1e-12, atol=1e-12)
