@@ -465,6 +465,9 @@ def main():
     ap.add_argument("--prefill", action="store_true",
                     help="time causal chunk attention (pre-fill) over one compressed 14B anchor "
                          "instead of the decode step (one JSON line of its own)")
+    ap.add_argument("--prefill-mla", action="store_true",
+                    help="time MLA pre-fill (a 1024-query chunk over B=4 x 4096 positions) at every "
+                         "kept width instead of the decode step (one JSON line of its own)")
     ap.add_argument("--append", action="store_true",
                     help="time bulk appends (quantise on write) at the 14B shape instead of the "
                          "decode step (one JSON line of its own)")
@@ -486,6 +489,9 @@ def main():
         return
     if args.append:
         append_bench(args)
+        return
+    if args.prefill_mla:
+        prefill_mla_bench(args)
         return
 
     import torch
@@ -945,6 +951,79 @@ def prefill_bench(args):
                          "work": f"scores and value products counted once ({flops / 1e9:.1f} GFLOP)"},
             "ms_min": round(min(ms), 4), "ms_max": round(max(ms), 4),
             "gpu_launches": 2 * args.steps, "clocks": clk.summary()}
+    print(json.dumps(line))
+
+
+MLA_PREFILL_CHUNK = 1024
+
+
+def prefill_mla_bench(args):
+    """MLA pre-fill over one latent layer of the MLA workload (16 heads,
+    latent 512 + k^R 64) at B=4 sequences of 4096 positions, the last 1024
+    of which are the chunk, for every kept width (bf16 latents, or quantised
+    with --mla-bits / --mla-scheme).  CUDA events on the launching stream.
+    value = ms per call at width 512; the roofline counts the attention's
+    score and value products once against the measured bf16 dense peak."""
+    import torch
+    from __graft_entry__ import build
+    build()
+    from paper_2609_37988_gb300 import workloads as W
+    from paper_2609_37988_gb300.cache import Cache, Layer
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    B, T, n_q = 4, 4096, MLA_PREFILL_CHUNK
+    w = W.config(4, batch=B, mla_bits=args.mla_bits, mla_scheme=args.mla_scheme)
+    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+        peak = float(json.load(f)["bf16_tflops"])
+    res = {}
+    with Clocks(0) as clk:
+        for width in (512, 256, 128, 64):
+            l = next(i for i, a in enumerate(w.layers) if a["width"] == width)
+            a = dict(w.layers[l])
+            c = Cache(kind="mla", n_layers=1, n_q_heads=w.n_q_heads, head_dim=w.head_dim,
+                      latent_dim=w.latent_dim, rope_dim=w.rope_dim, max_batch=B, max_ctx=T,
+                      layers=[Layer(**a)], device=dev)
+            cl, kr = W.mla_inputs(w, l, 0, T, device=dev)
+            c.append(0, cl, kr)
+            del cl, kr
+            wk, wv = W.mla_weights(w, l, device=dev)
+            qn = W.randn((B, n_q, w.n_q_heads, w.head_dim), w.seed, l, 12, dtype=torch.bfloat16, device=dev)
+            qp = W.randn((B, n_q, w.n_q_heads, w.rope_dim), w.seed, l, 13, dtype=torch.bfloat16, device=dev)
+            out = torch.empty(qn.shape, dtype=torch.float32, device=dev)
+            for _ in range(max(3, args.warmup)):
+                c.prefill_mla(0, qn, qp, wk, wv, w.sigma, out=out)
+            torch.cuda.synchronize()
+            stream = torch.cuda.current_stream()
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                  for _ in range(args.steps)]
+            if width == 512:
+                clk.mark("start")
+            for s0, e0 in ev:
+                s0.record(stream)
+                c.prefill_mla(0, qn, qp, wk, wv, w.sigma, out=out)
+                e0.record(stream)
+            torch.cuda.synchronize()
+            if width == 512:
+                clk.mark("end")
+            assert c.device_error() == 0
+            ms = statistics.mean(s0.elapsed_time(e0) for s0, e0 in ev)
+            rows = sum(T - n_q + i + 1 for i in range(n_q)) * B * w.n_q_heads
+            flops = rows * 2 * (2 * width + w.rope_dim)
+            res[f"d{width}"] = {"ms": round(ms, 4), "tflops": round(flops / (ms * 1e-3) / 1e12, 2),
+                                "frac": round(flops / (ms * 1e-3) / 1e12 / peak, 4)}
+            del c
+    m = res["d512"]
+    q = "bf16" if args.mla_bits is None else f"{'sym' if args.mla_scheme == 'symmetric' else 'int'}{args.mla_bits}"
+    line = {"metric": "MLA pre-fill over the latent cache: ms per call, TFLOP/s of the attention",
+            "value": m["ms"], "unit": "ms", "higher_is_better": False, "steps": args.steps,
+            "warmup": max(3, args.warmup), "n_gpus": 1, "dtype": f"{q} latents, f16/bf16 hi+lo products",
+            "data": "synthetic",
+            "config": {"workload": f"mla-h16-r512 {q}, B={B}, T={T}, chunk {n_q}",
+                       "l2": "each sequence's latent cache fits in L2; the rows re-read it from there"},
+            "roofline": {"bound": "tensor", "achieved": m["tflops"], "peak": round(peak, 1), "unit": "TFLOP/s",
+                         "frac": m["frac"], "traffic": None, "peak_source": "measured bf16 dense (burst)",
+                         "work": "score and value products of every row over its causal range, once"},
+            "widths": res, "gpu_launches": 3 * args.steps, "clocks": clk.summary()}
     print(json.dumps(line))
 
 

@@ -62,7 +62,7 @@ struct MlaQTile {
   // shared memory of everything but the raw ring, for TR positions and NST stages
   static constexpr int fixed(int TR, int NST) {
     return NST * (KH / 64) * TR * 128 + NST * TR * 16 + 32 * KH * 2 + 2 * 4 * (TR * 16 > 1024 ? TR * 16 : 1024) +
-           128 + 768 + 8 * (2 * NST + 7 + 16) + 16 + 1024;
+           128 + 768 + 8 * (2 * NST + 2 * 4 + 5 + 16) + 16 + 1024;
   }
   static constexpr int raw(int TR) { return TR * REC + TR * MB; }
   static constexpr int nr(int TR, int NST) { return (kMlaQSmemMax - fixed(TR, NST)) / raw(TR); }
@@ -95,15 +95,21 @@ struct MlaQCfg {
   static constexpr int OFF_QS = OFF_P + 2 * PB;       // float [2][16] query sums (latent, rope)
   static constexpr int OFF_RED = OFF_QS + 128;        // float [4][16] maxima, sums, zero sums
   static constexpr int OFF_BAR = OFF_RED + 3 * 256;
-  // full[NST], sbar[2], pbar[2], obar[NST], dbar[3], rfull[NR], rfree[NR]
-  static constexpr int NBAR = 2 * NST + 7 + 2 * NR;
+  static constexpr int NSB = 4;                       // score buffers in TMEM
+  // full[NST], sbar[NSB], pbar[2], obar[NST], dbar[3], rfull[NR], rfree[NR], sfree[NSB]
+  static constexpr int NBAR = 2 * NST + 2 * NSB + 5 + 2 * NR;
   static constexpr int OFF_TB = OFF_BAR + 8 * NBAR;
   static constexpr int SMEM = OFF_TB + 16 + 1024;
   static constexpr int MV = W >= 128 ? 128 : 64;
   static constexpr int MBL = W / MV;                  // value M-blocks
   static constexpr int OCOLS = 32 * MBL;
-  static constexpr int SCOLS = 128;                   // two buffers of [latent hi|lo, rope hi|lo]
-  static constexpr int TCOLS = 256;
+  // the score k-steps of a tile split between the two score warps: warp 4
+  // takes latent k-steps [0, KA), warp 7 the rest and the positional ones,
+  // each into accumulators of its own (32 columns: 16 heads hi | lo)
+  static constexpr int KL = W / 16, KA = (KL + kRope / 16) / 2, KB = KL - KA;
+  static constexpr int SBUF = KB > 0 ? 96 : 64;      // [A | B | rope] columns per buffer
+  static constexpr int SCOLS = SBUF * NSB;
+  static constexpr int TCOLS = 512;
   static_assert(NR >= 2, "raw stages");
   static_assert(OCOLS + SCOLS <= TCOLS, "TMEM columns");
   static_assert(REC % 16 == 0 && RAW_META % 16 == 0 && (TR * MB) % 16 == 0, "bulk copy sizes");
@@ -151,8 +157,8 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t *full = reinterpret_cast<uint64_t *>(sm + C::OFF_BAR);
-  uint64_t *sbar = full + C::NST, *pbar = sbar + 2, *obar = pbar + 2, *dbar = obar + C::NST;
-  uint64_t *rfull = dbar + 3, *rfree = rfull + C::NR;
+  uint64_t *sbar = full + C::NST, *pbar = sbar + C::NSB, *obar = pbar + 2, *dbar = obar + C::NST;
+  uint64_t *rfull = dbar + 3, *rfree = rfull + C::NR, *sfree = rfree + C::NR;
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + C::OFF_TB);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + C::OFF_TB + 4);
   float *red = reinterpret_cast<float *>(sm + C::OFF_RED);  // [4 warps][16] maxima
@@ -177,9 +183,11 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     for (int i = 0; i < C::NBAR; ++i) {
       // full and pbar: one arrival per expansion / softmax warp; rfree: per
       // expansion warp; the rest: one arrival (commit, or expect_tx)
-      const bool exp = (i < C::NST) || (i >= 2 * C::NST + 7 + C::NR);
-      const bool four = i >= C::NST + 2 && i < C::NST + 4;
-      mbar_init(&full[i], exp ? kExpWarps : four ? 4 : 1);
+      const int o_pbar = C::NST + C::NSB, o_rfree = 2 * C::NST + C::NSB + 5 + C::NR;
+      const bool exp = (i < C::NST) || (i >= o_rfree && i < o_rfree + C::NR);
+      const bool four = (i >= o_pbar && i < o_pbar + 2) || i >= o_rfree + C::NR;
+      const bool two = i >= C::NST && i < C::NST + C::NSB;  // sbar: both score warps commit
+      mbar_init(&full[i], exp ? kExpWarps : four ? 4 : two ? 2 : 1);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -236,7 +244,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     tc_fence_after();
   }
   const uint32_t tmem = *tbase;
-  const uint32_t t_o = tmem, t_s = tmem + C::OCOLS;  // O columns, then two S buffers of 64
+  const uint32_t t_o = tmem, t_s = tmem + C::OCOLS;  // O columns, then NSB S buffers of 64
   auto ostage = [&](int s) { return sm + s * C::OSTAGE; };
   auto ometa = [&](int s) { return reinterpret_cast<float4 *>(sm + C::OFF_OM + s * C::OMETA); };
   auto rawst = [&](int r) { return sm + C::OFF_RAW + r * C::RAW; };
@@ -367,29 +375,38 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
       pdl_trigger();
     } else if (warp == 4 || warp == 7) {
       // ======================= score warps ==================================
-      // as in mla.cu (warp 4 the even tiles, warp 7 the odd ones; a warp waits
-      // for softmax(t-2) before the operand of tile t, whose stage's previous
-      // tile t - 3 is then known to have been expanded); the latent k-steps
-      // accumulate into S columns 0-31, the positional ones into 32-63
+      // both warps work on every tile, warp 4 the latent k-steps [0, KA)
+      // into S columns [0, 32), warp 7 the latent ones [KA, KL) into
+      // [32, 64) and the positional ones into the last 32 columns; each
+      // waits for the tile's expansion and for softmax(t - NSB) to have read
+      // the buffer, and commits to the buffer's barrier (two arrivals)
       const int role = warp == 4 ? 0 : 1;
       constexpr uint32_t ID_S = umma_idesc_f16(C::SM, 32, false, false);
-      for (int t = role; t < n_tiles && !failed; t += 2) {
+      for (int t = 0; t < n_tiles && !failed; ++t) {
         const int s = t % C::NST;
         bool ok = true;
-        if (t >= 2) ok = mbar_wait_sleepy(&pbar[t & 1], ((t - 2) >> 1) & 1, wait_limit, abort_flag, kSleepNs);
+        if (t >= C::NSB)
+          ok = mbar_wait_sleepy(&sfree[t % C::NSB], ((t - C::NSB) / C::NSB) & 1, wait_limit, abort_flag, kSleepNs);
         if (ok) ok = mbar_wait_sleepy(&full[s], (t / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
         if (ok && lane == 0) {
           tc_fence_after();
           const uint64_t dc = umma_desc(smem_u32(ostage(s)), 16, 1024, 2);
           const uint64_t dq = umma_desc(smem_u32(q_s), 128, KH / 8 * 128, 0);
-          const uint32_t S = t_s + 64 * (t & 1);
-  #pragma unroll
-          for (int ks = 0; ks < KH / 16; ++ks) {
-            const bool rope = ks >= W / 16;
-            umma_f16(rope ? S + 32 : S, dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
-                     dq + (uint64_t)(ks * 16), ID_S, rope ? ks > W / 16 : ks > 0);
+          const uint32_t S = t_s + C::SBUF * (t % C::NSB);
+          auto mma = [&](uint32_t d, int ks, bool acc) {
+            umma_f16(d, dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4), dq + (uint64_t)(ks * 16),
+                     ID_S, acc);
+          };
+          if (role == 0) {
+#pragma unroll
+            for (int ks = 0; ks < C::KA; ++ks) mma(S, ks, ks > 0);
+          } else {
+#pragma unroll
+            for (int ks = C::KA; ks < C::KL; ++ks) mma(S + 32, ks, ks > C::KA);
+#pragma unroll
+            for (int ks = C::KL; ks < KH / 16; ++ks) mma(S + C::SBUF - 32, ks, ks > C::KL);
           }
-          umma_commit(&sbar[t & 1]);
+          umma_commit(&sbar[t % C::NSB]);
         }
         failed = !__all_sync(0xffffffffu, ok);
       }
@@ -480,7 +497,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     for (int h = 0; h < kHeads; ++h) { m_run[h] = -1e30f; l_part[h] = 0.f; z_part[h] = 0.f; }
     for (int t = 0; t < n_tiles; ++t) {
       const int base = i0 + t * TR, nval = min(TR, i1 - base);
-      bool ok = mbar_wait_sleepy(&sbar[t & 1], (t >> 1) & 1, wait_limit, abort_flag, kSleepNs);
+      bool ok = mbar_wait_sleepy(&sbar[t % C::NSB], (t / C::NSB) & 1, wait_limit, abort_flag, kSleepNs);
       // the tile's scales were written before its operand was published:
       // acquire them (the phase of tile t is complete, the next cannot be)
       if (ok) ok = mbar_wait_sleepy(&full[t % C::NST], (t / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
@@ -493,15 +510,24 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
       const float4 md = live ? ometa(t % C::NST)[prow] : make_float4(0.f, 0.f, 0.f, 0.f);
       float x[kHeads];
       {
-        // [latent hi | latent lo | rope hi | rope lo] of the 16 heads
-        float sv[64];
-        tmem_ld64(t_s + 64 * (t & 1) + lane_off, sv);
+        // [A hi | A lo | (B hi | B lo |) rope hi | rope lo] of the 16 heads
+        float sv[64], sr[32];
+        const uint32_t S = t_s + C::SBUF * (t % C::NSB) + lane_off;
+        tmem_ld64(S, sv);
+        if constexpr (C::KB > 0) tmem_ld32(S + 64, sr);
+        // the score buffer is free for tile t + NSB
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sfree[t % C::NSB]);
         const float scl = md.x * kCodeScale, scr = md.z * kCodeScale;
 #pragma unroll
-        for (int h = 0; h < kHeads; ++h)
-          x[h] = live ? fmaf(sv[h] + sv[16 + h], scl,
-                             fmaf(sv[32 + h] + sv[48 + h], scr, fmaf(md.y, qsl[h], md.w * qsr[h])))
-                      : -INFINITY;
+        for (int h = 0; h < kHeads; ++h) {
+          // latent and positional parts (with one accumulator pair each
+          // when the latent k-steps were not split)
+          const float lat = C::KB > 0 ? (sv[h] + sv[16 + h]) + (sv[32 + h] + sv[48 + h]) : sv[h] + sv[16 + h];
+          const float rp = C::KB > 0 ? sr[h] + sr[16 + h] : sv[32 + h] + sv[48 + h];
+          x[h] = live ? fmaf(lat, scl, fmaf(rp, scr, fmaf(md.y, qsl[h], md.w * qsr[h]))) : -INFINITY;
+        }
       }
       bool need = false;
 #pragma unroll
