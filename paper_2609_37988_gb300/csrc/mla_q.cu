@@ -34,20 +34,19 @@
 namespace kvk {
 namespace {
 
-// Grid (split, sequence); 16 warps:
+// Grid (split, query row); 16 warps:
 //   0-3   softmax and epilogue (TMEM lane = tile position, as in mla.cu);
-//   4, 7  score products of the even and the odd tiles;
-//   5     bulk copies of the raw records and metadata of each tile;
+//   4, 7  score products (each tile's k-steps split between the two);
+//   5     idle (keeps the warpgroups aligned);
 //   6     value products;
-//   8-15  expansion of a tile's codes into the f16 operand layout.
-// Rings: NR raw stages (codes as stored + metadata), NST operand stages
-// (the f16 tile as (W + 64) / 64 boxes of TR rows x 128 bytes in the 128-byte
-// swizzled K-major layout, plus the tile's per-position (s, z, s^R, z^R)).
-// Tiles of 128 positions (score products M = 128, TMEM lane = position)
-// where three operand stages fit beside at least three raw stages, else 64
-// or 32 (M = 64, lanes 0-15 of each lane quarter); the raw ring takes the
-// rest of the shared memory, up to 8 stages, so that several tiles' bytes
-// are in flight while earlier tiles are expanded and multiplied.
+//   8-15  expansion of a tile's codes, read from global memory (L2
+//         prefetched a few tiles ahead), into the f16 operand layout.
+// NST operand stages (the f16 tile as (W + 64) / 64 boxes of TR rows x 128
+// bytes in the 128-byte swizzled K-major layout, plus the tile's
+// per-position (s, z', s^R, z'^R)): tiles of 128 positions (score products
+// M = 128, TMEM lane = position) where two stages fit, else 64 (M = 64,
+// lanes 0-15 of each lane quarter), and as many stages (up to 4) as shared
+// memory holds beside the query and the weights.
 constexpr int kMlaQThreads = 512;
 constexpr int kExpWarps = 8;                 // warps 8-15
 constexpr int kExpThreads = 32 * kExpWarps;
@@ -57,16 +56,13 @@ constexpr int kMlaQSmemMax = 232448;
 template <int W, int BITS, bool SYM>
 struct MlaQTile {
   static constexpr int KH = W + kRope;
-  static constexpr int REC = KH * BITS / 8;
-  static constexpr int MB = SYM ? 4 : 16;
-  // shared memory of everything but the raw ring, for TR positions and NST stages
-  static constexpr int fixed(int TR, int NST) {
-    return NST * (KH / 64) * TR * 128 + NST * TR * 16 + 32 * KH * 2 + 2 * 4 * (TR * 16 > 1024 ? TR * 16 : 1024) +
-           128 + 768 + 8 * (2 * NST + 2 * 4 + 5 + 16) + 16 + 1024;
-  }
-  static constexpr int raw(int TR) { return TR * REC + TR * MB; }
-  static constexpr int nr(int TR, int NST) { return (kMlaQSmemMax - fixed(TR, NST)) / raw(TR); }
-  static constexpr int TR = nr(128, 3) >= 3 ? 128 : nr(64, 3) >= 3 ? 64 : 32;
+  static constexpr int pns(int TR) { return TR * 16 > 1024 ? TR * 16 : 1024; }
+  // shared memory besides the stages: query, weights, sums, barriers
+  static constexpr int fixed(int TR) { return 32 * KH * 2 + 2 * 4 * pns(TR) + 128 + 768 + 8 * 24 + 16 + 1024; }
+  static constexpr int stage(int TR) { return (KH / 64) * TR * 128 + TR * 16; }
+  static constexpr int nst(int TR) { return (kMlaQSmemMax - fixed(TR)) / stage(TR); }
+  static constexpr int TR = nst(128) >= 2 ? 128 : 64;
+  static constexpr int NST = nst(TR) < 4 ? nst(TR) : 4;
 };
 
 template <int W, int BITS, bool SYM>
@@ -77,27 +73,23 @@ struct MlaQCfg {
   static constexpr int BOXES = KH / 64;
   static constexpr int BOX = TR * 128;
   static constexpr int OSTAGE = BOXES * BOX;          // f16 operand tile
-  static constexpr int NST = 3;
+  static constexpr int NST = MlaQTile<W, BITS, SYM>::NST;
   static constexpr int REC = KH * BITS / 8;           // stored record bytes
   static constexpr int MB = SYM ? 4 : 16;             // metadata bytes per position
-  static constexpr int RAW_META = TR * REC;           // offset of the metadata in a raw stage
-  static constexpr int RAW = TR * REC + TR * MB;
-  static constexpr int NR_FIT = MlaQTile<W, BITS, SYM>::nr(TR, NST);
-  static constexpr int NR = NR_FIT < 8 ? NR_FIT : 8;
+  static constexpr int PF = 4;                        // tiles prefetched into L2 ahead
   static constexpr int OMETA = TR * 16;               // float4 (s, z, s^R, z^R) per position
   static constexpr int QB = 32 * KH * 2;
   static constexpr int PNS = TR * 16 > 1024 ? TR * 16 : 1024;  // P: stride of 8-column groups
   static constexpr int PB = 4 * PNS;
   static constexpr int OFF_OM = NST * OSTAGE;
-  static constexpr int OFF_RAW = OFF_OM + NST * OMETA;
-  static constexpr int OFF_Q = OFF_RAW + NR * RAW;
+  static constexpr int OFF_Q = OFF_OM + NST * OMETA;
   static constexpr int OFF_P = OFF_Q + QB;
   static constexpr int OFF_QS = OFF_P + 2 * PB;       // float [2][16] query sums (latent, rope)
   static constexpr int OFF_RED = OFF_QS + 128;        // float [4][16] maxima, sums, zero sums
   static constexpr int OFF_BAR = OFF_RED + 3 * 256;
   static constexpr int NSB = 4;                       // score buffers in TMEM
-  // full[NST], sbar[NSB], pbar[2], obar[NST], dbar[3], rfull[NR], rfree[NR], sfree[NSB]
-  static constexpr int NBAR = 2 * NST + 2 * NSB + 5 + 2 * NR;
+  // full[NST], sbar[NSB], pbar[2], obar[NST], dbar[3], sfree[NSB]
+  static constexpr int NBAR = 2 * NST + 2 * NSB + 5;
   static constexpr int OFF_TB = OFF_BAR + 8 * NBAR;
   static constexpr int SMEM = OFF_TB + 16 + 1024;
   static constexpr int MV = W >= 128 ? 128 : 64;
@@ -110,10 +102,10 @@ struct MlaQCfg {
   static constexpr int SBUF = KB > 0 ? 96 : 64;      // [A | B | rope] columns per buffer
   static constexpr int SCOLS = SBUF * NSB;
   static constexpr int TCOLS = 512;
-  static_assert(NR >= 2, "raw stages");
+  static_assert(NST >= 2, "operand stages");
   static_assert(OCOLS + SCOLS <= TCOLS, "TMEM columns");
-  static_assert(REC % 16 == 0 && RAW_META % 16 == 0 && (TR * MB) % 16 == 0, "bulk copy sizes");
-  static_assert(OSTAGE % 1024 == 0 && OFF_RAW % 16 == 0 && OFF_Q % 16 == 0 && OFF_P % 16 == 0, "alignment");
+  static_assert(REC % 16 == 0 && (TR * MB) % 16 == 0, "prefetch sizes");
+  static_assert(OSTAGE % 1024 == 0 && OFF_Q % 16 == 0 && OFF_P % 16 == 0, "alignment");
   static_assert(SMEM <= kMlaQSmemMax, "shared memory");
   static_assert(BITS == 8 || BITS == 4 || (BITS == 2 && SYM), "code widths");
 };
@@ -125,11 +117,16 @@ template <int BITS>
 struct RawChunk {
   using T = typename std::conditional<BITS == 8, uint2, uint32_t>::type;
 };
+// one chunk's stored bytes, from global memory through the read-only path
 template <int BITS>
-__device__ __forceinline__ typename RawChunk<BITS>::T load_chunk(const uint8_t *src) {
-  if constexpr (BITS == 8) return *reinterpret_cast<const uint2 *>(src);
-  else if constexpr (BITS == 4) return *reinterpret_cast<const uint32_t *>(src);
-  else return *reinterpret_cast<const uint16_t *>(src);
+__device__ __forceinline__ typename RawChunk<BITS>::T ldg_chunk(const uint8_t *src) {
+  if constexpr (BITS == 8) return __ldg(reinterpret_cast<const uint2 *>(src));
+  else if constexpr (BITS == 4) return __ldg(reinterpret_cast<const unsigned int *>(src));
+  else return __ldg(reinterpret_cast<const unsigned short *>(src));
+}
+// prefetch `bytes` (a multiple of 16, from a 16-byte aligned address) into L2
+__device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 template <int BITS>
 __device__ __forceinline__ uint4 expand_chunk(typename RawChunk<BITS>::T w) {
@@ -158,7 +155,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t *full = reinterpret_cast<uint64_t *>(sm + C::OFF_BAR);
   uint64_t *sbar = full + C::NST, *pbar = sbar + C::NSB, *obar = pbar + 2, *dbar = obar + C::NST;
-  uint64_t *rfull = dbar + 3, *rfree = rfull + C::NR, *sfree = rfree + C::NR;
+  uint64_t *sfree = dbar + 3;
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + C::OFF_TB);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + C::OFF_TB + 4);
   float *red = reinterpret_cast<float *>(sm + C::OFF_RED);  // [4 warps][16] maxima
@@ -181,11 +178,11 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
 
   if (tid == 0) {
     for (int i = 0; i < C::NBAR; ++i) {
-      // full and pbar: one arrival per expansion / softmax warp; rfree: per
-      // expansion warp; the rest: one arrival (commit, or expect_tx)
-      const int o_pbar = C::NST + C::NSB, o_rfree = 2 * C::NST + C::NSB + 5 + C::NR;
-      const bool exp = (i < C::NST) || (i >= o_rfree && i < o_rfree + C::NR);
-      const bool four = (i >= o_pbar && i < o_pbar + 2) || i >= o_rfree + C::NR;
+      // full: one arrival per expansion warp; pbar and sfree: per softmax
+      // warp; sbar: per score warp; the rest: one (a commit)
+      const int o_pbar = C::NST + C::NSB, o_sfree = 2 * C::NST + C::NSB + 5;
+      const bool exp = i < C::NST;
+      const bool four = (i >= o_pbar && i < o_pbar + 2) || i >= o_sfree;
       const bool two = i >= C::NST && i < C::NST + C::NSB;  // sbar: both score warps commit
       mbar_init(&full[i], exp ? kExpWarps : four ? 4 : two ? 2 : 1);
     }
@@ -247,20 +244,18 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   const uint32_t t_o = tmem, t_s = tmem + C::OCOLS;  // O columns, then NSB S buffers of 64
   auto ostage = [&](int s) { return sm + s * C::OSTAGE; };
   auto ometa = [&](int s) { return reinterpret_cast<float4 *>(sm + C::OFF_OM + s * C::OMETA); };
-  auto rawst = [&](int r) { return sm + C::OFF_RAW + r * C::RAW; };
   auto pbuf = [&](int ps) { return sm + C::OFF_P + ps * C::PB; };
   bool failed = false;
 
   // Register split over the warpgroups (launched with 128 per thread, 65536
-  // in all): expansion 80 + 80, products and copies 96, softmax 256, in all
+  // in all): expansion 80 + 80, products 96, softmax 256, in all
   // (80 + 80 + 96 + 256) x 128 = 65536; each warpgroup's role begins with its
   // own (the softmax increase waits for the decreases).
   if (warp >= 8) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 80;\n" ::: "memory");
     // ======================= expansion warps ==============================
-    // tile t: raw stage t % NR -> operand stage t % NST (free once the
-    // values of tile t - NST were computed); rows past the split's end are
-    // zero, with zero scales
+    // tile t -> operand stage t % NST (free once the values of tile t - NST
+    // were computed); rows past the split's end are zero, with zero scales
     const int et = tid - 256;  // 0 .. kExpThreads - 1
     // codes are centred on C0 (symmetric: q, so the operand is the signed
     // code itself and the offset term vanishes; grouped: the mid code), by an
@@ -282,26 +277,52 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
       roff[i] = row * C::REC + c8 * BITS;
       soff[i] = (c8 / 8) * C::BOX + row * 128 + 16 * ((c8 % 8) ^ (row % 8));
     }
+    // the split's records and metadata rows in global memory; tiles are
+    // prefetched into L2 PF ahead of the expansion (a hint, no completion)
+    const uint8_t *grec = v.rec + (pos0 + i0) * C::REC;
+    const uint8_t *gmeta = v.meta + (pos0 + i0) * C::MB;
+    auto prefetch = [&](int u) {
+      if (et == 0 && u < n_tiles) {
+        const int nv = min(TR, i1 - (i0 + u * TR));
+        prefetch_l2(grec + (size_t)u * TR * C::REC, (uint32_t)(nv * C::REC));
+        prefetch_l2(gmeta + (size_t)u * TR * C::MB, (uint32_t)(((nv * C::MB + 15) / 16) * 16));
+      }
+    };
+    for (int u = 0; u < C::PF; ++u) prefetch(u);
     for (int t = 0; t < n_tiles; ++t) {
-      const int r = t % C::NR, s = t % C::NST;
-      bool ok = mbar_wait_sleepy(&rfull[r], (t / C::NR) & 1, wait_limit, abort_flag, kSleepNs);
-      if (ok && t >= C::NST)
+      const int s = t % C::NST;
+      prefetch(t + C::PF);
+      bool ok = true;
+      if (t >= C::NST)
         ok = mbar_wait_sleepy(&obar[s], ((t - C::NST) / C::NST) & 1, wait_limit, abort_flag, kSleepNs);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       const int nval = min(TR, i1 - (i0 + t * TR));
-      const uint8_t *raw = rawst(r);
+      const uint8_t *raw = grec + (size_t)t * TR * C::REC;
+      const uint8_t *rmeta = gmeta + (size_t)t * TR * C::MB;
       uint8_t *ost = ostage(s);
+      // this thread's metadata row (at most one: TR <= 256), loaded first
+      const int mrow = et;
+      uint4 mw = make_uint4(0, 0, 0, 0);
+      if (mrow < nval) {
+        if constexpr (SYM) mw.x = __ldg(reinterpret_cast<const uint32_t *>(rmeta) + mrow);
+        else mw = __ldg(reinterpret_cast<const uint4 *>(rmeta) + mrow);
+      }
       if (nval == TR) {
-        // every load before the first use
-        typename RawChunk<BITS>::T w[kPer];
+        // loads in groups of eight, each group's loads before their use
 #pragma unroll
-        for (int i = 0; i < kPer; ++i) w[i] = load_chunk<BITS>(raw + roff[i]);
+        for (int j0 = 0; j0 < kPer; j0 += 8) {
+          typename RawChunk<BITS>::T w[8];
 #pragma unroll
-        for (int i = 0; i < kPer; ++i) {
-          const uint4 x = expand_chunk<BITS>(w[i]);
-          *reinterpret_cast<uint4 *>(ost + soff[i]) =
-              make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
-                         hsub2_u32(x.w, kC0Pair));
+          for (int i = 0; i < 8; ++i)
+            if (j0 + i < kPer) w[i] = ldg_chunk<BITS>(raw + roff[j0 + i]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (j0 + i < kPer) {
+              const uint4 x = expand_chunk<BITS>(w[i]);
+              *reinterpret_cast<uint4 *>(ost + soff[j0 + i]) =
+                  make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
+                             hsub2_u32(x.w, kC0Pair));
+            }
         }
       } else {
         // the split's last, partial tile: rows past its end are zero
@@ -309,33 +330,32 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
         for (int i = 0; i < kPer; ++i) {
           uint4 x = make_uint4(0, 0, 0, 0);
           if ((int)(roff[i] / C::REC) < nval) {
-            x = expand_chunk<BITS>(load_chunk<BITS>(raw + roff[i]));
+            x = expand_chunk<BITS>(ldg_chunk<BITS>(raw + roff[i]));
             x = make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
                            hsub2_u32(x.w, kC0Pair));
           }
           *reinterpret_cast<uint4 *>(ost + soff[i]) = x;
         }
       }
-      for (int row = et; row < TR; row += kExpThreads) {
+      if (mrow < TR) {
         float4 m = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (row < nval) {
+        if (mrow < nval) {
           if constexpr (SYM) {
             // x = s (u - q): centred on q, no offset
-            const uint32_t w = reinterpret_cast<const uint32_t *>(raw + C::RAW_META)[row];
-            m = make_float4(__uint_as_float(w << 16), 0.f, __uint_as_float(w & 0xffff0000u), 0.f);
+            m = make_float4(__uint_as_float(mw.x << 16), 0.f, __uint_as_float(mw.x & 0xffff0000u), 0.f);
           } else {
-            m = reinterpret_cast<const float4 *>(raw + C::RAW_META)[row];
+            m = make_float4(__uint_as_float(mw.x), __uint_as_float(mw.y), __uint_as_float(mw.z),
+                            __uint_as_float(mw.w));
             m.y = fmaf((float)kC0, m.x, m.y);
             m.w = fmaf((float)kC0, m.z, m.w);
           }
         }
-        ometa(s)[row] = m;
+        ometa(s)[mrow] = m;
       }
       fence_proxy_async();
       __syncwarp();
       if (lane == 0) {
         mbar_arrive(&full[s]);
-        mbar_arrive(&rfree[r]);
       }
     }
     if (failed && lane == 0) {
@@ -347,31 +367,7 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
   } else if (warp >= 4) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 96;\n" ::: "memory");
     if (warp == 5) {
-      // ======================= copy warp ====================================
-      int issued = 0;
-      if (lane == 0) {
-        for (; issued < n_tiles; ++issued) {
-          const int r = issued % C::NR;
-          // the raw stage's previous tile was expanded
-          if (issued >= C::NR &&
-              !mbar_wait_sleepy(&rfree[r], ((issued - C::NR) / C::NR) & 1, wait_limit, abort_flag, kSleepNs)) {
-            *abort_flag = 1;
-            set_err(err, 8);
-            break;
-          }
-          const int base = i0 + issued * TR, nval = min(TR, i1 - base);
-          // metadata rows rounded up to 16 bytes (within the slab: capacity
-          // and split starts are multiples of 64 positions)
-          const int mbytes = ((nval * C::MB + 15) / 16) * 16;
-          fence_proxy_async();
-          mbar_expect_tx(&rfull[r], nval * C::REC + mbytes);
-          bulk_g2s(rawst(r), v.rec + (pos0 + base) * C::REC, nval * C::REC, &rfull[r]);
-          bulk_g2s(rawst(r) + C::RAW_META, v.meta + (pos0 + base) * C::MB, mbytes, &rfull[r]);
-        }
-        for (int u = max(0, issued - C::NR); u < issued; ++u)
-          mbar_wait(&rfull[u % C::NR], (u / C::NR) & 1, kLimit);
-      }
-      __syncwarp();
+      // no role: the tiles come from global memory (see the expansion warps)
       pdl_trigger();
     } else if (warp == 4 || warp == 7) {
       // ======================= score warps ==================================
