@@ -46,7 +46,9 @@ namespace {
 // per-position (s, z', s^R, z'^R)): tiles of 128 positions (score products
 // M = 128, TMEM lane = position) where two stages fit, else 64 (M = 64,
 // lanes 0-15 of each lane quarter), and as many stages (up to 4) as shared
-// memory holds beside the query and the weights.
+// memory holds beside the query and the weights (a tile's stage is busy
+// from its expansion through its value products, so the stage count bounds
+// how many tiles are in that chain at once).
 constexpr int kMlaQThreads = 512;
 constexpr int kExpWarps = 8;                 // warps 8-15
 constexpr int kExpThreads = 32 * kExpWarps;
@@ -269,14 +271,16 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
     // (threads past the last chunk repeat it: the same bytes, written twice)
     constexpr int kCpr = KH / 8, kJobs = TR * kCpr;
     constexpr int kPer = (kJobs + kExpThreads - 1) / kExpThreads;
-    uint32_t roff[kPer], soff[kPer];
-#pragma unroll
-    for (int i = 0; i < kPer; ++i) {
-      const int q = min(et + kExpThreads * i, kJobs - 1);
-      const int row = q / kCpr, c8 = q - row * kCpr;
-      roff[i] = row * C::REC + c8 * BITS;
-      soff[i] = (c8 / 8) * C::BOX + row * 128 + 16 * ((c8 % 8) ^ (row % 8));
-    }
+    // offsets of chunk i of this thread, recomputed where used (registers go
+    // to the loads in flight)
+    auto roff = [&](int i) {
+      const int q = min(et + kExpThreads * i, kJobs - 1), row = q / kCpr;
+      return row * C::REC + (q - row * kCpr) * BITS;
+    };
+    auto soff = [&](int i) {
+      const int q = min(et + kExpThreads * i, kJobs - 1), row = q / kCpr, c8 = q - row * kCpr;
+      return (c8 / 8) * C::BOX + row * 128 + 16 * ((c8 % 8) ^ (row % 8));
+    };
     // the split's records and metadata rows in global memory; tiles are
     // prefetched into L2 PF ahead of the expansion (a hint, no completion)
     const uint8_t *grec = v.rec + (pos0 + i0) * C::REC;
@@ -308,33 +312,28 @@ __global__ void __launch_bounds__(kMlaQThreads, 1)
         else mw = __ldg(reinterpret_cast<const uint4 *>(rmeta) + mrow);
       }
       if (nval == TR) {
-        // loads in groups of eight, each group's loads before their use
+        // every load of the tile before the first use
+        typename RawChunk<BITS>::T w[kPer];
 #pragma unroll
-        for (int j0 = 0; j0 < kPer; j0 += 8) {
-          typename RawChunk<BITS>::T w[8];
+        for (int i = 0; i < kPer; ++i) w[i] = ldg_chunk<BITS>(raw + roff(i));
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
-            if (j0 + i < kPer) w[i] = ldg_chunk<BITS>(raw + roff[j0 + i]);
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            if (j0 + i < kPer) {
-              const uint4 x = expand_chunk<BITS>(w[i]);
-              *reinterpret_cast<uint4 *>(ost + soff[j0 + i]) =
-                  make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
-                             hsub2_u32(x.w, kC0Pair));
-            }
+        for (int i = 0; i < kPer; ++i) {
+          const uint4 x = expand_chunk<BITS>(w[i]);
+          *reinterpret_cast<uint4 *>(ost + soff(i)) =
+              make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
+                         hsub2_u32(x.w, kC0Pair));
         }
       } else {
         // the split's last, partial tile: rows past its end are zero
 #pragma unroll
         for (int i = 0; i < kPer; ++i) {
           uint4 x = make_uint4(0, 0, 0, 0);
-          if ((int)(roff[i] / C::REC) < nval) {
-            x = expand_chunk<BITS>(ldg_chunk<BITS>(raw + roff[i]));
+          if ((int)(roff(i) / C::REC) < nval) {
+            x = expand_chunk<BITS>(ldg_chunk<BITS>(raw + roff(i)));
             x = make_uint4(hsub2_u32(x.x, kC0Pair), hsub2_u32(x.y, kC0Pair), hsub2_u32(x.z, kC0Pair),
                            hsub2_u32(x.w, kC0Pair));
           }
-          *reinterpret_cast<uint4 *>(ost + soff[i]) = x;
+          *reinterpret_cast<uint4 *>(ost + soff(i)) = x;
         }
       }
       if (mrow < TR) {
