@@ -213,11 +213,12 @@ def cpu_baseline(w, seconds=12.0):
     for a in w.anchors:
         kinds.setdefault(w.layers[a]["bits"], a)
     units = []
+    w1 = dataclasses.replace(w, batch=1)  # one sequence's inputs: the sample needs one unit
     for bits, a in sorted(kinds.items()):
-        k, v = W.kv_inputs(w, a, 0, T, device="cpu")
+        k, v = W.kv_inputs(w1, a, 0, T, device="cpu")
         kk = k[0, :, 0].float().numpy()
         vv = v[0, :, 0].float().numpy()
-        q = W.queries(w, a)[0, :G].float().numpy()
+        q = W.queries(w1, a)[0, :G].float().numpy()
         if bits == 16:
             units.append((bits, q, kk, vv, None))
         elif w.layers[a].get("scheme") == "symmetric":
