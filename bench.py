@@ -355,7 +355,9 @@ def kernel_durations(w, cache, stream, new_kv, qs, outs, splits, per_layer, src,
         if w.kind == "mla":
             layer_call(l)  # the whole MLA call (4 launches)
         elif splits[l] > 1:
-            cache.decode_partial(l, qs[l], w.sigma, splits[l], partials=parts[l])
+            # the automatic schedule, as the step's decode (splits or runs;
+            # splits[l] partial slots either way)
+            cache.decode_partial(l, qs[l], w.sigma, 0, partials=parts[l])
         else:
             cache.decode(l, qs[l], w.sigma, out=outs[l], n_splits=1)
 
@@ -458,6 +460,12 @@ def main():
     ap.add_argument("--sym-bits", type=int, choices=[8, 4, 2], default=None,
                     help="store the quantised anchors with the symmetric per-vector "
                          "quantiser at this bit-width")
+    ap.add_argument("--schedule", choices=["auto", "splits", "runs"], default="auto",
+                    help="partition of the GQA decodes over CTAs (kvk_set_decode_schedule)")
+    ap.add_argument("--run-ctas", type=int, default=0,
+                    help="CTAs of a run-schedule decode (0: whole waves of resident CTAs)")
+    ap.add_argument("--run-setup", type=int, default=-1,
+                    help="planned tiles charged to each unit's start in a run decode (-1: default)")
     ap.add_argument("--profile-case",
                     choices=["gqa", "kpc", "mla", "mla64", "gather", "sym", "evict", "evict-small",
                              "prefill", "prefill-small", "append", "mlaq", "mlaq64"],
@@ -542,6 +550,8 @@ def main():
         cache = Cache(n_layers=w.n_layers, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
                       head_dim=w.head_dim, max_batch=w.batch, max_ctx=T,
                       layers=[Layer(**a) for a in w.layers], max_splits=64, device=dev)
+        cache.set_decode_schedule({"auto": 0, "splits": 1, "runs": 2}[args.schedule], args.run_ctas,
+                                  args.run_setup)
         for a in w.anchors:
             k, v = W.kv_inputs(w, a, 0, pre, device=dev)
             cache.append(a, k, v)
@@ -751,7 +761,9 @@ def main():
                        "l2": (f"no flush; smallest per-layer read {min(per_layer) / 1e6:.0f} MB vs 126 MB L2"
                               + (" (every layer's read exceeds L2)" if min(per_layer) > 126e6 else
                                  " (some layers fit in L2; consecutive inheritors may hit it)")),
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": f"replicas x{world}",
+                       "decode_schedule": (args.schedule if args.run_ctas == 0 else
+                                           f"{args.schedule}, {args.run_ctas} run CTAs")},
             "fraction_of_peak": value / hbm, "peak_gbs": hbm, "peak_kind": peak_kind,
             "fraction_of_nominal_8tbs": value / 8000.0,
             "roofline": {"bound": "hbm", "kernel": (f"gqa_decode ({dom})" if w.kind == "gqa" else

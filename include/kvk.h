@@ -192,7 +192,9 @@ kvk_status kvk_rewind(kvk_cache *cache, int32_t n, kvk_stream stream);
 
 /* The split count kvk_decode_attention / kvk_decode_attention_mla would use
  * for `layer` with n_splits = 0 (host only; depends on the host-side bound
- * on the anchor's lengths and on the SM count). */
+ * on the anchor's lengths, the SM count and the decode schedule).  Under the
+ * run schedule (kvk_set_decode_schedule) it is the number of partial slots
+ * per (sequence, KV head) that kvk_decode_partial with n_splits = 0 writes. */
 kvk_status kvk_decode_plan_splits(kvk_cache *cache, int32_t layer, int32_t *n_splits);
 
 /* Install the kept-position list of anchor `layer` (eviction, Sec. 3.4):
@@ -324,7 +326,11 @@ kvk_status kvk_decode_attention_mla(kvk_cache *cache, int32_t layer, const void 
  * partials device float [n_splits, B*H_q, head_dim + 2]: per row the
  * unnormalised accumulator sum_t 2^(x_t - m) v_t (head_dim floats), then m,
  * then l = sum_t 2^(x_t - m), with x_t = scale * log2(e) * <q, k_t>.  A split
- * that reads no position stores m = -inf, l = 0. */
+ * that reads no position stores m = -inf, l = 0.  n_splits >= 2: equal
+ * contiguous context splits.  n_splits = 0: the automatic schedule, with
+ * kvk_decode_plan_splits slots; under the run schedule each slot holds one
+ * piece of a partition of the positions (not an equal split), and merging
+ * all slots with kvk_splitk_reduce gives the attention output. */
 kvk_status kvk_decode_partial(kvk_cache *cache, int32_t layer, const void *q,
                               int32_t q_dtype, float softmax_scale, float *partials,
                               int32_t n_splits, kvk_stream stream);
@@ -420,6 +426,34 @@ kvk_status kvk_export_layer(const kvk_cache *cache, int32_t layer, void *k_out, 
  * path without a fault.  Errors: KVK_ERR_INVALID_ARG for a null cache. */
 #define KVK_WAIT_LIMIT_DEFAULT 4194304u
 kvk_status kvk_set_wait_limit(kvk_cache *cache, uint32_t polls);
+
+/* How an automatic GQA decode (n_splits = 0) partitions the work over CTAs
+ * (a scheduling choice; the paper's method is the same either way):
+ *  KVK_SCHEDULE_SPLITS: a grid of (context split, KV head, sequence), every
+ *      split the same number of positions;
+ *  KVK_SCHEDULE_RUNS: one or a few whole waves of resident CTAs, each taking
+ *      an equal run of the flattened (sequence, KV head, tile) grid, a run
+ *      meeting at most two (sequence, KV head) units; quantised anchors with
+ *      per-token keys or the symmetric scheme read without a kept list
+ *      (other anchors use the splits);
+ *  KVK_SCHEDULE_AUTO (default): the runs where the split grid would give
+ *      each CTA at most 13 tiles and leave its last wave of CTAs less than
+ *      90 % full (and every run CTA gets at least four tiles), else the
+ *      splits.
+ * run_ctas: the number of run CTAs (clamped to [units, tiles], units = B *
+ * H_kv, tiles of 64 or 128 positions per unit); 0 = the fewest whole waves
+ * of resident CTAs that are at least the units.  run_setup: planned tiles
+ * charged to each unit's start (query set-up, first copies, epilogue) in
+ * the partition, so that runs that start a second unit carry fewer data
+ * tiles; -1 = the library's default, else 0..64.
+ * Results agree to rounding (the merge order of partial sums differs).
+ * Applies to calls enqueued after it.  Errors: INVALID_ARG for a null cache,
+ * an unknown schedule, run_ctas < 0 or run_setup outside [-1, 64]. */
+#define KVK_SCHEDULE_AUTO 0
+#define KVK_SCHEDULE_SPLITS 1
+#define KVK_SCHEDULE_RUNS 2
+kvk_status kvk_set_decode_schedule(kvk_cache *cache, int32_t schedule, int32_t run_ctas,
+                                   int32_t run_setup);
 
 /* Synchronise `stream`, read the device error word into *code and clear it.
  * Returns KVK_ERR_DEVICE if the word was non-zero.  After a

@@ -57,6 +57,7 @@ _SIGS = {
     "kvk_cache_destroy": [_P],
     "kvk_cache_reset": [_P, _P],
     "kvk_set_wait_limit": [_P, ctypes.c_uint32],
+    "kvk_set_decode_schedule": [_P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32],
     "kvk_layer_source": [_P, _I, ctypes.POINTER(_I)],
     "kvk_layer_lengths": [_P, _I, ctypes.POINTER(_P)],
     "kvk_append": [_P, _I, _P, _P, _I, _I, _P, _P],

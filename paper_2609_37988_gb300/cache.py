@@ -123,6 +123,17 @@ class Cache:
         giving up (0: at the first poll, setting the timeout error)."""
         check(self.lib.kvk_set_wait_limit(self.handle, int(polls)))
 
+    SCHEDULE_AUTO, SCHEDULE_SPLITS, SCHEDULE_RUNS = 0, 1, 2
+
+    def set_decode_schedule(self, schedule: int, run_ctas: int = 0, run_setup: int = -1):
+        """How automatic GQA decodes partition the work: SCHEDULE_SPLITS (equal
+        context splits per unit), SCHEDULE_RUNS (equal runs of the flattened
+        unit x tile grid, where the format has them) or SCHEDULE_AUTO;
+        run_ctas: CTAs of a run decode (0: whole waves of resident CTAs);
+        run_setup: planned tiles charged to each unit's start (-1: default)."""
+        check(self.lib.kvk_set_decode_schedule(self.handle, int(schedule), int(run_ctas),
+                                               int(run_setup)))
+
     # -- plan ----------------------------------------------------------------
     def source(self, layer: int) -> int:
         out = ctypes.c_int32()
@@ -270,7 +281,8 @@ class Cache:
         _need(q, "q")
         B, Hq, D = q.shape
         if partials is None:
-            partials = torch.empty((n_splits, B * Hq, D + 2), dtype=torch.float32, device=q.device)
+            n = n_splits if n_splits > 0 else self.plan_splits(layer)
+            partials = torch.empty((n, B * Hq, D + 2), dtype=torch.float32, device=q.device)
         check(self.lib.kvk_decode_partial(self.handle, layer, _ptr(q), _dtype_code(q), float(scale),
                                           _ptr(partials), n_splits, _stream(stream)))
         return partials

@@ -104,7 +104,7 @@ struct GqaCfg {
                                    : (STAGE <= 13312 ? 4 : (STAGE <= 20480 ? 3 : 2));
   static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");
   static constexpr int BAR_OFF = Q_BYTES + NST * STAGE;
-  static constexpr int GMASK_OFF = BAR_OFF + (TMA ? 8 * NST : 0);
+  static constexpr int GMASK_OFF = BAR_OFF + (TMA ? 16 * NST : 0);  // two mbarrier sets
   static constexpr int FOLD_OFF = (GMASK_OFF + (TMA ? 16 * NST : 0) + 15) & ~15;  // 16-byte stores
   static constexpr int SMEM = FOLD_OFF + FOLD_BYTES + ZRED_BYTES;
   // CTAs per SM the register budget is sized for: four where four fit in
@@ -156,12 +156,19 @@ __device__ __forceinline__ float key_weight(int ch, int sgn) {
   return __int_as_float((127 + 2 * sgn * key_weight_exp<BITS>(ch)) << 23);
 }
 
+// The decode of one unit (sequence b, KV head kvh) over items [i0, i1) of
+// its positions or kept list (i1 < 0: to the end), written to partial slot
+// `slot`, or normalised to the output when a.out is set.  The copy ring
+// starts at tile 0 on mbarrier set `bset` (NST fresh mbarriers, initialised
+// by the caller; a CTA decoding two units uses one set for each, so that
+// both run the same code with stage and phase fixed by the tile number).
+// Returns false when a bounded wait gave up.
 // GATHER: the rows come from the anchor's kept-position list (compiled
 // separately so that the contiguous path carries none of its state).
 template <int BITS, int D, int KAX, int GS, bool GATHER>
-__global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
-    gqa_decode_kernel(const GqaDecodeArgs a) {
-  pdl_wait();
+__device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const int b, const int kvh,
+                                                const int i0, const int i1_req, const int slot,
+                                                const int bset) {
   using C = GqaCfg<BITS, D, KAX, GS>;
   constexpr bool BF = C::BF;
   constexpr int KS = C::KS, NG = C::NG;
@@ -172,19 +179,15 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   uint8_t *stages = smem + C::Q_BYTES;
 
   const GqaView &v = a.v;
-  const int split = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, c = lane & 3;
   const int len = v.lens[b];
   // kept-position lists exist only with per-token key metadata or bf16
   // caches (rejected by the host for per-channel keys)
   constexpr bool gather = GATHER && !C::KPC;
-  const int kunit = v.kept_per_head ? b * v.Hkv + blockIdx.y : b;  // whose kept list
+  const int kunit = v.kept_per_head ? b * v.Hkv + kvh : b;  // whose kept list
   const int n_items = gather ? min(v.kept_n[kunit], v.kept_cap) : len;
-  const int i0 = split * a.items_per_split;
-  // the last split runs to the end, so a launch recorded for shorter
-  // sequences (a replayed graph) still covers every position
-  const int i1 = (split == a.n_splits - 1) ? n_items : min(i0 + a.items_per_split, n_items);
+  const int i1 = i1_req < 0 ? n_items : min(i1_req, n_items);
   const int Tq = C::KPC ? (len / GS) * GS : len;  // positions held as codes
   const bool use_lo = a.q_f32 != 0;
   const int32_t *kept = v.kept_idx + (size_t)kunit * v.kept_cap;
@@ -263,15 +266,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
   // bulk-copy producer (quantised caches): one copy per tile, or one per
   // kept record; rows that get no copy are zero-filled so stale bytes never
   // reach the arithmetic.
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::BAR_OFF);
-  if constexpr (C::TMA) {
-    if (tid == 0) {
-#pragma unroll
-      for (int s = 0; s < C::NST; ++s) mbar_init(&bars[s], 1);
-      fence_mbar_init();
-    }
-    __syncthreads();
-  }
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::BAR_OFF) + bset * C::NST;
   // gather: kept position of row (TILE/4) warp + lane of the next tile to
   // issue, and per stage one row-validity word per warp
   uint32_t *gmask = reinterpret_cast<uint32_t *>(smem + C::GMASK_OFF);
@@ -1057,38 +1052,164 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
       if (a.out) {
         a.out[(row0 + h) * D + ch] = (L > 0.f) ? A / L : 0.f;
       } else {
-        float *pr = a.partial + ((size_t)split * gridDim.z * a.Hq + row0 + h) * RS;
+        float *pr = a.partial + ((size_t)slot * v.B * a.Hq + row0 + h) * RS;
         pr[ch] = A;
         if (ch == 0) { pr[D] = (L > 0.f) ? M : -INFINITY; pr[D + 1] = L; }
       }
     }
   }
+  return !timed_out;
 }
 
-template <int BITS, int D, int KAX, int GS, bool GATHER>
+// Formats with a run-schedule kernel: the contiguous bulk-copy formats
+// (quantised, per-token keys or the symmetric scheme).
+template <int BITS, int D, int KAX, int GS>
+__host__ __device__ constexpr bool gqa_has_run() {
+  using C = GqaCfg<BITS, D, KAX, GS>;
+  return C::TMA && !C::KPC;
+}
+
+// Segment k (0 or 1) of run-schedule CTA blockIdx.x (see gqa_decode_kernel):
+// unit (b, kvh), items [i0, i1) (i1 = -1: to the sequence's end), partial
+// slot, and the number of slots the unit's pieces fill when this CTA holds
+// its last planned tile (else 0).  False when the run has no segment k.
+// Each unit spans a.run_tpu planned tiles of the run grid: a.run_setup
+// tiles standing for the cost of starting a unit (query set-up, the first
+// copies, the epilogue), then its data tiles, so that a run that starts a
+// second unit carries fewer data tiles.  32-bit arithmetic only (the host
+// keeps W < 2^31 and n < 2^16): with W = q n + r, run c starts at planned
+// tile floor(c W / n) = c q + floor(c r / n).
+struct GqaRunSeg {
+  int b, kvh, i0, i1, slot, n_used;
+};
+__device__ __forceinline__ int gqa_run_start(const GqaDecodeArgs &a, int c) {
+  return c * a.run_q + (int)(((uint32_t)c * (uint32_t)a.run_r) / (uint32_t)a.run_ctas);
+}
+template <int TILE>
+__device__ __forceinline__ bool gqa_run_segment(const GqaDecodeArgs &a, int k, GqaRunSeg &sg) {
+  const int x = blockIdx.x, tpu = a.run_tpu, su = a.run_setup;
+  const int w1 = gqa_run_start(a, x + 1);
+  int w = gqa_run_start(a, x);
+  if (k == 1) w = (w / tpu + 1) * tpu;  // the next unit's first planned tile
+  if (w >= w1) return false;
+  const int u = w / tpu;
+  const int ub = u * tpu, we = min(w1, ub + tpu);
+  const bool owns_end = we == ub + tpu;
+  // the first CTA whose run meets unit u: this one, or an earlier one whose
+  // run holds planned tile ub (runs are at least q >= 1 tiles, so at most a
+  // unit's worth of steps back)
+  int c0 = x;
+  while (gqa_run_start(a, c0) > ub) --c0;
+  sg.b = u / a.v.Hkv;
+  sg.kvh = u - sg.b * a.v.Hkv;
+  sg.i0 = max(0, w - ub - su) * TILE;
+  sg.i1 = owns_end ? -1 : max(0, we - ub - su) * TILE;
+  sg.slot = x - c0;
+  sg.n_used = owns_end ? sg.slot + 1 : 0;
+  return true;
+}
+
+// RUN = false: grid (split, kv head, sequence); CTA (x, y, z) decodes items
+// [x ips, (x + 1) ips) of unit (z, y) into partial slot x (ips =
+// a.items_per_split; the last split runs to the end, so a launch recorded
+// for shorter sequences, as in a replayed graph, still covers every
+// position).
+// RUN = true: a one-dimensional grid of equal runs.  The (unit, tile) grid,
+// u = b Hkv + kvh with a.run_tpu planned tiles each (set-up tiles, then
+// data tiles), is flattened and CTA x takes planned tiles [w0, w1), w0 =
+// floor(x W / n) (W tiles, n CTAs).  The host
+// keeps runs no longer than a unit, so a run meets at most two units; each
+// is one segment, decoded into partial slot x - (the first CTA meeting the
+// unit), each on its own set of mbarriers.  The CTA that holds a unit's
+// last planned tile runs to the sequence's end and marks the unit's unused
+// slots (up to a.run_slots) empty.  Every CTA does
+// W / n tiles of work, so one wave of resident CTAs ends together instead
+// of a second, partial wave of splits.
+template <int BITS, int D, int KAX, int GS, bool GATHER, bool RUN>
+__global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
+    gqa_decode_kernel(const GqaDecodeArgs a) {
+  pdl_wait();
+  using C = GqaCfg<BITS, D, KAX, GS>;
+  extern __shared__ __align__(128) uint8_t smem[];
+  if constexpr (C::TMA) {
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::BAR_OFF);
+    if (threadIdx.x == 0) {
+#pragma unroll
+      for (int s = 0; s < (RUN ? 2 : 1) * C::NST; ++s) mbar_init(&bars[s], 1);
+      fence_mbar_init();
+    }
+    __syncthreads();
+  }
+  if constexpr (!RUN) {
+    const int split = blockIdx.x;
+    const int i0 = split * a.items_per_split;
+    const int i1 = split == a.n_splits - 1 ? -1 : i0 + a.items_per_split;
+    gqa_decode_unit<BITS, D, KAX, GS, GATHER>(a, blockIdx.z, blockIdx.y, i0, i1, split, 0);
+  } else {
+    static_assert(gqa_has_run<BITS, D, KAX, GS>() && !GATHER, "runs cover the contiguous bulk-copy formats");
+    // Every thread derives the segments from blockIdx.x and the arguments
+    // alone (warp-uniform values, as the split grid's are), the second one
+    // after the first segment.  The two segments are two call sites, not a
+    // loop: inside a loop the decode body compiles to slower code.
+    auto mark_unused = [&](const GqaRunSeg &sg) {
+      if (sg.n_used == 0) return;
+      // slots past the unit's last CTA, for its G heads: whole empty rows
+      // (accumulator 0, m = -inf, l = 0), like a split that reads nothing
+      const size_t row0 = (size_t)sg.b * a.Hq + (size_t)sg.kvh * a.G;
+      constexpr int RS = D + 2;
+      for (int i = threadIdx.x; i < (a.run_slots - sg.n_used) * a.G * RS; i += blockDim.x) {
+        const int r = i / RS, col = i - r * RS;
+        float *pr = a.partial + ((size_t)(sg.n_used + r / a.G) * a.v.B * a.Hq + row0 + r % a.G) * RS;
+        pr[col] = col == D ? -INFINITY : 0.f;
+      }
+    };
+    GqaRunSeg sg;
+    if (!gqa_run_segment<C::TILE>(a, 0, sg)) return;
+    // false: a wait gave up (the error word is set)
+    if (!gqa_decode_unit<BITS, D, KAX, GS, false>(a, sg.b, sg.kvh, sg.i0, sg.i1, sg.slot, 0)) return;
+    mark_unused(sg);
+    if (!gqa_run_segment<C::TILE>(a, 1, sg)) return;
+    __syncthreads();  // the next unit's query and copies reuse shared memory
+    if (!gqa_decode_unit<BITS, D, KAX, GS, false>(a, sg.b, sg.kvh, sg.i0, sg.i1, sg.slot, 1)) return;
+    mark_unused(sg);
+  }
+}
+
+template <int BITS, int D, int KAX, int GS, bool GATHER, bool RUN>
 cudaError_t launch_gqa_decode_g(const GqaDecodeArgs &a, cudaStream_t st) {
   using C = GqaCfg<BITS, D, KAX, GS>;
-  auto k = gqa_decode_kernel<BITS, D, KAX, GS, GATHER>;
+  auto k = gqa_decode_kernel<BITS, D, KAX, GS, GATHER, RUN>;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
+  if constexpr (RUN) return launch_pdl(k, dim3(a.run_ctas), dim3(128), C::SMEM, st, a);
   dim3 grid(a.n_splits, a.v.Hkv, a.v.B);
   return launch_pdl(k, grid, dim3(128), C::SMEM, st, a);
 }
 
 template <int BITS, int D, int KAX, int GS>
 cudaError_t launch_gqa_decode_t(const GqaDecodeArgs &a, cudaStream_t st) {
+  if (a.run_ctas > 0) {
+    // run schedule: contiguous bulk-copy formats, partials only
+    if constexpr (gqa_has_run<BITS, D, KAX, GS>()) {
+      if (a.gather || a.out || a.run_tpu < 1 || a.run_slots < 1) return cudaErrorInvalidValue;
+      return launch_gqa_decode_g<BITS, D, KAX, GS, false, true>(a, st);
+    } else {
+      return cudaErrorInvalidValue;
+    }
+  }
   if constexpr (GqaCfg<BITS, D, KAX, GS>::KPC) {
     if (a.gather) return cudaErrorInvalidValue;  // no kept lists with per-channel keys
-    return launch_gqa_decode_g<BITS, D, KAX, GS, false>(a, st);
+    return launch_gqa_decode_g<BITS, D, KAX, GS, false, false>(a, st);
   } else {
-    return a.gather ? launch_gqa_decode_g<BITS, D, KAX, GS, true>(a, st)
-                    : launch_gqa_decode_g<BITS, D, KAX, GS, false>(a, st);
+    return a.gather ? launch_gqa_decode_g<BITS, D, KAX, GS, true, false>(a, st)
+                    : launch_gqa_decode_g<BITS, D, KAX, GS, false, false>(a, st);
   }
 }
+
 
 template <int BITS, int D, int KAX, int GS>
 int gqa_tile_t() {
@@ -1098,7 +1219,7 @@ int gqa_tile_t() {
 template <int BITS, int D, int KAX, int GS>
 int gqa_ctas_per_sm_t() {
   using C = GqaCfg<BITS, D, KAX, GS>;
-  auto k = gqa_decode_kernel<BITS, D, KAX, GS, false>;
+  auto k = gqa_decode_kernel<BITS, D, KAX, GS, false, false>;
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   int n = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, 128, C::SMEM) != cudaSuccess) n = 1;

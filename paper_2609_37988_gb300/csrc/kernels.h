@@ -57,6 +57,14 @@ struct GqaDecodeArgs {
   float *out;          // [B, Hq, D]: normalised output (single split)
   int32_t *err;
   uint32_t wait_limit = 1u << 22;  // polls of a bounded wait on this CTA's copies before it gives up
+  // run schedule (quantised formats with per-token keys or the symmetric
+  // scheme, contiguous reads, partials only): run_ctas > 0 CTAs take equal
+  // runs of the (unit, tile) grid of run_tpu kernel tiles per unit, into
+  // run_slots partial slots per unit; 0 = the (split, kv head, sequence) grid.
+  // run_tpu counts run_setup planned tiles per unit for its start-up cost
+  // before its data tiles; run_q, run_r: the planned tile count W = B Hkv
+  // run_tpu as q run_ctas + r.
+  int run_ctas = 0, run_tpu = 0, run_slots = 0, run_q = 0, run_r = 0, run_setup = 0;
 };
 
 // Returns cudaSuccess or the launch error.  Template dispatch on

@@ -163,6 +163,11 @@ WsLayout ws_layout(const kvk_model_desc *d, int max_splits) {
 
 }  // namespace
 
+// planned set-up tiles per unit of a run-schedule decode unless set
+// (4: the best of 0..8 measured on int4 and symmetric 4-bit anchors at the
+// 14B step shape, B = 20..64)
+constexpr int kRunSetupDefault = 4;
+
 struct kvk_cache {
   kvk_model_desc desc;
   std::vector<kvk_layer_cfg> cfg;
@@ -179,6 +184,9 @@ struct kvk_cache {
   int device;
   std::vector<int> ctas;  // per layer, decode CTAs per SM (0 = not queried)
   uint32_t wait_limit = KVK_WAIT_LIMIT_DEFAULT;  // decode tile-loop waits (kvk_set_wait_limit)
+  int schedule = KVK_SCHEDULE_AUTO;              // decode partition (kvk_set_decode_schedule)
+  int run_ctas = 0;                              // CTAs of a run-schedule decode (0: whole waves)
+  int run_setup = kRunSetupDefault;              // planned set-up tiles per unit of a run decode
   struct alignas(64) Tmap {
     uint8_t bytes[128];
   };
@@ -313,6 +321,71 @@ int auto_splits(kvk_cache *c, int a) {
   return choose_splits(units, layer_tiles(c, a), kt / kTile, slots, c->max_splits);
 }
 
+// The run schedule of an automatic decode of anchor a (kernel side in
+// decode_gqa.cuh): n CTAs, each an equal run of the (unit, kernel tile)
+// grid, n >= units so that a run meets at most two units.  n is the
+// smallest whole number of waves of resident CTAs that is at least the
+// number of units, or the count set with kvk_set_decode_schedule (clamped
+// to [units, tiles]).  Formats: quantised with per-token keys or the
+// symmetric scheme, contiguous reads.  Returns false (split grid) when the
+// format has no run kernel, the schedule is off, there are fewer tiles than
+// CTAs, or the partial slots would exceed max_splits.  The automatic choice
+// takes the runs only where the split grid gives each CTA at most 13 kernel
+// tiles and leaves its last wave less than 90 % full: the decode is bound
+// by HBM even with a partly filled last wave, so what the runs save is the
+// per-CTA start-up of many short splits.  Measured at the 14B step shape
+// (int4 g32, one anchor): B = 20 (6 splits of 11 tiles) 54.1 -> 48.6 us,
+// B = 24 (5 of 13) 58.9 -> 56.5 us; with 16 or more tiles per split the
+// runs were 1-4 % slower (B = 32 and 64, symmetric 8-bit at B = 32).
+struct RunPlan {
+  int ctas = 0, tpu = 0, slots = 0, q = 0, r = 0, setup = 0;
+};
+bool plan_runs(kvk_cache *c, int a, RunPlan *p) {
+  const kvk_layer_cfg &L = c->cfg[a];
+  if (c->schedule == KVK_SCHEDULE_SPLITS || c->desc.kind != KVK_KIND_GQA) return false;
+  if (L.bits == 16 || c->kept_on[a]) return false;
+  if (layer_scheme(&L) != kSchemeSym && L.key_axis != 0) return false;  // per-channel keys
+  const int kt = gqa_decode_tile(L.bits, c->desc.head_dim, L.key_axis, layer_group(&c->desc, &L),
+                                 layer_scheme(&L));
+  const int per = kt / kTile;
+  const long long tdata = (layer_tiles(c, a) + per - 1) / per;  // data tiles per unit
+  const long long tpu = tdata + c->run_setup;                   // planned tiles per unit
+  const long long units = (long long)c->desc.max_batch * c->desc.n_kv_heads;
+  const long long total = units * tpu;
+  auto_splits(c, a);  // queries the CTAs per SM
+  const long long slots = (long long)c->sm_count * c->ctas[a];
+  long long n;
+  if (c->run_ctas > 0) {
+    n = std::min<long long>(std::max<long long>(c->run_ctas, units), total);
+  } else {
+    n = slots;
+    while (n < units) n += slots;
+  }
+  // the kernel's run arithmetic is 32-bit: W < 2^31, n < 2^16
+  if (n > total || total >= (1LL << 31) || n >= (1LL << 16)) return false;
+  if (c->schedule == KVK_SCHEDULE_AUTO) {
+    if (total < 4 * n) return false;
+    const int s = std::min(auto_splits(c, a), layer_tiles(c, a));
+    const long long nt = (tdata + s - 1) / s;                 // kernel tiles per split
+    const long long grid = units * ((tdata + nt - 1) / nt);   // CTAs that get work
+    const double fill = (double)(grid % slots) / (double)slots;
+    if (nt > 13 || grid % slots == 0 || fill >= 0.9) return false;
+  }
+  int kmax = 0;
+  for (long long u = 0; u < units; ++u) {
+    const long long c0 = ((u * tpu + 1) * n - 1) / total, c1 = ((u + 1) * tpu * n - 1) / total;
+    kmax = std::max<int>(kmax, (int)(c1 - c0 + 1));
+  }
+  if (kmax > c->max_splits) return false;
+  p->ctas = (int)n;
+  p->tpu = (int)tpu;
+  p->slots = kmax;
+  p->q = (int)(total / n);
+  p->r = (int)(total % n);
+  p->setup = c->run_setup;
+  return true;
+}
+
 }  // namespace
 
 extern "C" {
@@ -432,6 +505,20 @@ kvk_status kvk_set_wait_limit(kvk_cache *c, uint32_t polls) {
   return KVK_OK;
 }
 
+kvk_status kvk_set_decode_schedule(kvk_cache *c, int32_t schedule, int32_t run_ctas,
+                                   int32_t run_setup) {
+  if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
+  if (schedule != KVK_SCHEDULE_AUTO && schedule != KVK_SCHEDULE_SPLITS && schedule != KVK_SCHEDULE_RUNS)
+    return fail(KVK_ERR_INVALID_ARG, "unknown decode schedule %d", schedule);
+  if (run_ctas < 0) return fail(KVK_ERR_INVALID_ARG, "run_ctas %d < 0", run_ctas);
+  if (run_setup < -1 || run_setup > 64)
+    return fail(KVK_ERR_INVALID_ARG, "run_setup %d outside [-1, 64]", run_setup);
+  c->schedule = schedule;
+  c->run_ctas = run_ctas;
+  c->run_setup = run_setup < 0 ? kRunSetupDefault : run_setup;
+  return KVK_OK;
+}
+
 kvk_status kvk_cache_reset(kvk_cache *c, kvk_stream stream) {
   if (!c) return fail(KVK_ERR_INVALID_ARG, "null cache");
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -531,7 +618,10 @@ kvk_status kvk_decode_plan_splits(kvk_cache *c, int32_t layer, int32_t *n_splits
   kvk_status s = check_layer_index(c, layer);
   if (s) return s;
   if (!n_splits) return fail(KVK_ERR_INVALID_ARG, "null output");
-  *n_splits = std::min(auto_splits(c, c->src[layer]), layer_tiles(c, c->src[layer]));
+  RunPlan rp;
+  *n_splits = plan_runs(c, c->src[layer], &rp)
+                  ? rp.slots
+                  : std::min(auto_splits(c, c->src[layer]), layer_tiles(c, c->src[layer]));
   return KVK_OK;
 }
 
@@ -790,11 +880,14 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   args.v = c->gqa_view(a);
   args.gather = c->kept_on[a];
   const int tiles = layer_tiles(c, a);
+  RunPlan rp;
+  const bool runs = n_splits == 0 && plan_runs(c, a, &rp);
+  if (runs) n_splits = rp.slots;
   if (n_splits == 0) n_splits = auto_splits(c, a);
   // a partial-only call keeps the caller's split count (extra splits are
   // empty and write m = -inf, l = 0); a full call never uses more splits
   // than tiles.
-  if (merge) n_splits = std::min(n_splits, tiles);
+  if (merge && !runs) n_splits = std::min(n_splits, tiles);
   args.q = q;
   args.q_f32 = q_dtype == KVK_DTYPE_F32;
   args.Hq = c->desc.n_q_heads;
@@ -809,8 +902,16 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   args.items_per_split = tps * kTile;
   args.err = c->err();
   args.wait_limit = c->wait_limit;
+  if (runs) {
+    args.run_ctas = rp.ctas;
+    args.run_tpu = rp.tpu;
+    args.run_slots = rp.slots;
+    args.run_q = rp.q;
+    args.run_r = rp.r;
+    args.run_setup = rp.setup;
+  }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (merge && n_splits == 1) {
+  if (merge && n_splits == 1 && !runs) {
     args.out = out;  // one split: the kernel normalises and writes the output
     args.partial = nullptr;
   } else {
@@ -819,7 +920,7 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   }
   cudaError_t e = launch_gqa_decode(args, st);
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
-  if (merge && n_splits > 1) {
+  if (merge && (n_splits > 1 || runs)) {
     e = launch_splitk_merge(args.partial, n_splits, c->desc.max_batch * c->desc.n_q_heads,
                             c->desc.head_dim, out, st);
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");
@@ -862,9 +963,10 @@ kvk_status kvk_internal_decode_with_partials(kvk_cache *c, int32_t layer, const 
     return fail(KVK_ERR_INVALID_ARG, "n_splits %d outside [0, %d]", n_splits, c->max_splits);
   const int a = c->src[layer];
   const int tiles = layer_tiles(c, a);
-  int ns = n_splits == 0 ? auto_splits(c, a) : n_splits;
-  ns = std::min(ns, tiles);
-  const size_t need = ns > 1 ? (size_t)ns * c->desc.max_batch * c->desc.n_q_heads *
+  RunPlan rp;
+  const bool runs = n_splits == 0 && plan_runs(c, a, &rp);
+  int ns = runs ? rp.slots : std::min(n_splits == 0 ? auto_splits(c, a) : n_splits, tiles);
+  const size_t need = (ns > 1 || runs) ? (size_t)ns * c->desc.max_batch * c->desc.n_q_heads *
                                    ((size_t)c->desc.head_dim + 2)
                              : 0;
   if (need > partial_floats)
@@ -872,7 +974,7 @@ kvk_status kvk_internal_decode_with_partials(kvk_cache *c, int32_t layer, const 
                 "layer %d: %d splits x %d rows need %zu partial floats; the fixed buffer "
                 "holds %zu (use fewer splits or kvk_decode_attention)",
                 layer, ns, c->desc.max_batch * c->desc.n_q_heads, need, partial_floats);
-  return gqa_decode_common(c, layer, q, q_dtype, scale, out, partial, ns, true, stream);
+  return gqa_decode_common(c, layer, q, q_dtype, scale, out, partial, runs ? 0 : ns, true, stream);
 }
 
 extern "C" {
@@ -890,7 +992,8 @@ kvk_status kvk_decode_partial(kvk_cache *c, int32_t layer, const void *q, int32_
                               kvk_stream stream) {
   if (!partials || !aligned16(partials))
     return fail(KVK_ERR_INVALID_ARG, "null or misaligned partials");
-  if (n_splits < 2) return fail(KVK_ERR_INVALID_ARG, "kvk_decode_partial needs n_splits >= 2");
+  if (n_splits == 1 || n_splits < 0)
+    return fail(KVK_ERR_INVALID_ARG, "kvk_decode_partial needs n_splits 0 (automatic) or >= 2");
   return gqa_decode_common(c, layer, q, q_dtype, softmax_scale, nullptr, partials, n_splits,
                            false, stream);
 }

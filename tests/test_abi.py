@@ -173,3 +173,7 @@ def test_symmetric_arena_and_cost(lib):
 
 def test_wait_limit_rejects_a_null_cache(lib):
     assert lib.load().kvk_set_wait_limit(None, 5) == 1  # KVK_ERR_INVALID_ARG
+
+
+def test_decode_schedule_rejects_a_null_cache(lib):
+    assert lib.load().kvk_set_decode_schedule(None, 0, 0, -1) == 1  # KVK_ERR_INVALID_ARG

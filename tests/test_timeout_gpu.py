@@ -5,8 +5,8 @@ nothing else), let the copies it had in flight land and return; the context
 stays usable, so with the default limit restored the next decode on the same
 cache matches the fp64 oracle and leaves the error word clear.
 
-Covered: the GQA decode's bulk-copy ring with early refill (per-token int8),
-its per-channel-key loop (bulk copies awaited at the top of each tile), and
+Covered: the GQA decode's bulk-copy ring with early refill (per-token int8,
+split grid and run schedule), its per-channel-key loop (bulk copies awaited at the top of each tile), and
 the quantised MLA decode (every role of the warp-specialised kernel gives
 up, the copy warp drains what it issued)."""
 import math
@@ -45,12 +45,18 @@ def test_gqa_decode_gives_up_and_recovers(cfg):
     for ns in (1, 4):
         c.decode(0, q.cuda(), scale, n_splits=ns)
         assert c.device_error() == TIMEOUT, f"splits={ns}: the timeout was not reported"
+    if cfg["key_axis"] == "token":
+        # the run schedule: a CTA whose first segment gives up skips its second
+        c.set_decode_schedule(c.SCHEDULE_RUNS, 5)
+        c.decode(0, q.cuda(), scale)
+        assert c.device_error() == TIMEOUT, "runs: the timeout was not reported"
 
     c.set_wait_limit(c.WAIT_LIMIT_DEFAULT)
     expected = gqa_expected(q, st, LENS, scale)
     for ns in (0, 1, 4):
         out = c.decode(0, q.cuda(), scale, n_splits=ns)
         assert_close(f32(out), expected, what=f"after timeout, splits={ns}")
+    c.set_decode_schedule(c.SCHEDULE_AUTO)
     assert c.device_error() == 0
 
 
