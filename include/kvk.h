@@ -73,7 +73,9 @@ enum {
   KVK_DEVERR_KEPT_RANGE = 1,   /* kept position >= sequence length           */
   KVK_DEVERR_CAPACITY = 2,     /* append position >= capacity                */
   KVK_DEVERR_COUNT = 4,        /* per-sequence append count out of range     */
-  KVK_DEVERR_TIMEOUT = 8       /* a bounded wait on an async copy gave up    */
+  KVK_DEVERR_TIMEOUT = 8,      /* a bounded wait on an async copy gave up    */
+  KVK_DEVERR_ALIGN = 16        /* shared memory not aligned for a copy; the  */
+                               /* call computed nothing                      */
 };
 
 /* Model geometry.  GQA: n_q_heads query heads, n_kv_heads KV heads of

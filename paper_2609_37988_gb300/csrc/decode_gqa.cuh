@@ -36,7 +36,9 @@
 // fields of a word at weights 4^e that the query (keys) or the final
 // accumulator scale (values) undoes.
 #pragma once
+#include <cuda.h>  // CUtensorMap (the gather's row copies)
 #include <math.h>
+#include <string.h>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -90,7 +92,8 @@ struct GqaCfg {
   static constexpr int STAGE = TMA ? KG_OFF_T + KG_ROWS * D * 8 + (SYM ? TILE * 4 : 0)
                                    : KG_OFF + KG_ROWS * D * 8;
   static constexpr int QSTR = D + 4;  // padded query row (floats): conflict-free head rows
-  static constexpr int Q_BYTES = 8 * QSTR * 4 + 2 * 8 * NG * 4;
+  // padded to 128 bytes: stages (tensor-map copy destinations) start 128-byte aligned
+  static constexpr int Q_BYTES = (8 * QSTR * 4 + 2 * 8 * NG * 4 + 127) & ~127;
   // per-channel keys: the query folded with each group's scales, once per
   // tile, in the score MMA's fragment order ([KG_ROWS][KS][32] x 16 bytes),
   // and the zero-point terms per warp ([4][KG_ROWS][8] floats)
@@ -105,13 +108,21 @@ struct GqaCfg {
   static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");
   static constexpr int BAR_OFF = Q_BYTES + NST * STAGE;
   static constexpr int GMASK_OFF = BAR_OFF + (TMA ? 16 * NST : 0);  // two mbarrier sets
-  static constexpr int FOLD_OFF = (GMASK_OFF + (TMA ? 16 * NST : 0) + 15) & ~15;  // 16-byte stores
+  // The kept-list gather of grouped per-token records copies whole records
+  // with tensor-map row copies (four rows per instruction): the records land
+  // as stored, so the consumer reads each row's value-chunk rotation (one
+  // byte per row and stage) instead of deriving it from the row.
+  static constexpr bool GTMA = QUANT && !SYM && KPT;
+  static constexpr int ROT_OFF = GMASK_OFF + (TMA ? 16 * NST : 0);
+  static constexpr int FOLD_OFF = (ROT_OFF + (GTMA ? NST * TILE : 0) + 15) & ~15;  // 16-byte stores
   static constexpr int SMEM = FOLD_OFF + FOLD_BYTES + ZRED_BYTES;
   // CTAs per SM the register budget is sized for: four where four fit in
   // shared memory (228 KB per SM, 1 KB reserved per CTA), else three
   static constexpr int MIN_CTAS = (!BF && 4 * (SMEM + 1024) <= 233472) ? 4 : 3;
   static_assert(REC % 16 == 0, "records are 16-byte multiples");
   static_assert(Q_BYTES % 16 == 0 && STAGE % 16 == 0 && FOLD_OFF % 16 == 0, "16-byte aligned regions");
+  static_assert(!GTMA || (Q_BYTES % 128 == 0 && STAGE % 128 == 0 && (4 * REC) % 128 == 0),
+                "row-copy destinations 128-byte aligned");
   static_assert(BITS != 2 || SYM, "2-bit codes exist for the symmetric scheme only");
   static_assert(!SYM || (D == 128 && GS == D), "symmetric rows are 128 channels, one group");
   static_assert(!QUANT || (GS % 16 == 0 && D % GS == 0), "groups are whole k-steps");
@@ -123,6 +134,18 @@ __device__ __forceinline__ int vswz(int mode, int t, int u) {
   if (mode == 1) return u ^ (t & 6);
   if (mode == 2) return u ^ (((t >> 1) & 1) | (((t >> 2) & 1) << 2));
   return u;
+}
+
+// Tensor-map row copy of four records: rows r0..r3 of the anchor's record
+// table (one box = one record) land back to back at dst, completing on bar.
+__device__ __forceinline__ void tma_rows4(void *dst, const CUtensorMap *map, int r0, int r1, int r2,
+                                          int r3, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(r0), "r"(r1), "r"(r2), "r"(r3),
+      "r"(smem_u32(bar))
+      : "memory");
 }
 
 // Codes as f16 operands: a code c placed in the low bits of a zero f16 bit
@@ -162,13 +185,14 @@ __device__ __forceinline__ float key_weight(int ch, int sgn) {
 // starts at tile 0 on mbarrier set `bset` (NST fresh mbarriers, initialised
 // by the caller; a CTA decoding two units uses one set for each, so that
 // both run the same code with stage and phase fixed by the tile number).
-// Returns false when a bounded wait gave up.
+// rows: the anchor's record table as a tensor map (kept-list gather of
+// grouped per-token records).  Returns false when a bounded wait gave up.
 // GATHER: the rows come from the anchor's kept-position list (compiled
 // separately so that the contiguous path carries none of its state).
 template <int BITS, int D, int KAX, int GS, bool GATHER>
-__device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const int b, const int kvh,
-                                                const int i0, const int i1_req, const int slot,
-                                                const int bset) {
+__device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const CUtensorMap *rows,
+                                                const int b, const int kvh, const int i0,
+                                                const int i1_req, const int slot, const int bset) {
   using C = GqaCfg<BITS, D, KAX, GS>;
   constexpr bool BF = C::BF;
   constexpr int KS = C::KS, NG = C::NG;
@@ -270,6 +294,7 @@ __device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const in
   // gather: kept position of row (TILE/4) warp + lane of the next tile to
   // issue, and per stage one row-validity word per warp
   uint32_t *gmask = reinterpret_cast<uint32_t *>(smem + C::GMASK_OFF);
+  uint8_t *rotb = smem + C::ROT_OFF;  // [stage][row] value-chunk rotation (row gather)
   int gidx_next = -1;
   if constexpr (C::TMA) {
     if (gather) {
@@ -322,6 +347,25 @@ __device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const in
       }
       const uint32_t vm = __ballot_sync(0xffffffffu, mine);
       if (lane == 0) gmask[s * 4 + warp] = vm;
+      if constexpr (C::GTMA) {
+        // whole records by tensor-map row copies, four rows per copy: lane j
+        // < RPW / 4 copies the warp's rows 4j .. 4j + 3.  A row without a
+        // valid position copies the slab's position 0 instead (a real
+        // record: the consumer masks the row and zeroes its value scales).
+        // Each row's value-chunk rotation goes to the stage's rotation bytes.
+        const int trow = (int)(slab * (size_t)v.cap) + (mine ? myidx : 0);
+        if (lane < RPW)
+          rotb[s * C::TILE + RPW * warp + lane] = (uint8_t)(mine ? v_rot(myidx, C::REC, C::KB / 16) : 0);
+        const int q = 4 * (lane & 7);
+        const int r0 = __shfl_sync(0xffffffffu, trow, q), r1 = __shfl_sync(0xffffffffu, trow, q + 1);
+        const int r2 = __shfl_sync(0xffffffffu, trow, q + 2), r3 = __shfl_sync(0xffffffffu, trow, q + 3);
+        if (tid == 0) mbar_expect_tx(&bars[s], C::TILE * C::REC);
+        if (lane < RPW / 4) {
+          fence_proxy_async();
+          tma_rows4(st + (RPW * warp + 4 * lane) * C::REC, rows, r0, r1, r2, r3, &bars[s]);
+        }
+        return;
+      }
       // value chunks (grouped) or whole records (symmetric) are stored
       // rotated by the position and read rotated by the shared-memory row:
       // chunk u of the record moves accordingly
@@ -356,7 +400,9 @@ __device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const in
       issue_cp(t, s);
   };
 
-  const bool use_cp = !C::TMA || gather;  // completion by cp.async groups
+  // completion by cp.async groups (bf16 planes, the chunked gather) or by
+  // the stages' mbarriers (bulk and tensor-map row copies)
+  const bool use_cp = !C::TMA || (gather && !C::GTMA);
 #pragma unroll
   for (int s = 0; s < C::NST - 1; ++s) {
     if (s < n_tiles) issue(s, s);
@@ -842,9 +888,12 @@ __device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const in
           const int mi = 4 * q + (lane >> 3);  // this lane addresses matrix mi
           const int j = mi / NC, k = mi % NC;
           const int t = wr0 + 16 * rb + 8 * j + (lane & 7);
+          // rotation of the row's record: by its shared-memory row, or (row
+          // gather) by its position, read from the stage's rotation bytes
+          const int vr = (C::GTMA && gather) ? rotb[s * C::TILE + t] : v_rot(t, C::REC, NC);
           const uint8_t *src =
               C::SYM ? st + t * C::REC + 16 * ((NC + k + sym_rot(t, C::NCH)) & (C::NCH - 1))
-                     : st + t * C::REC + C::KB + 16 * ((k + v_rot(t, C::REC, NC)) & (NC - 1));
+                     : st + t * C::REC + C::KB + 16 * ((k + vr) & (NC - 1));
           ldmatrix_x4_t(vw[rb][4 * q], vw[rb][4 * q + 1], vw[rb][4 * q + 2], vw[rb][4 * q + 3],
                         src);
         }
@@ -873,6 +922,12 @@ __device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const in
             } else if ((gi & 1) == 0) {
               vA4[rb] = reinterpret_cast<const float4 *>(vm_row(st, tA))[gi >> 1];
               vB4[rb] = reinterpret_cast<const float4 *>(vm_row(st, tA + 8))[gi >> 1];
+              if constexpr (C::GTMA && gather) {
+                // rows without a position hold another record's bytes
+                // (p = 0 there, but 0 * a non-finite scale would poison)
+                if (!vA[rb]) vA4[rb] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (!vB[rb]) vB4[rb] = make_float4(0.f, 0.f, 0.f, 0.f);
+              }
             }
             const float2 mA = (gi & 1) ? make_float2(vA4[rb].z, vA4[rb].w)
                                        : make_float2(vA4[rb].x, vA4[rb].y);
@@ -930,13 +985,14 @@ __device__ __forceinline__ bool gqa_decode_unit(const GqaDecodeArgs &a, const in
   // ---- copy ring over the split's tiles -----------------------------------
   bool timed_out = false;
   int t_stop = n_tiles;  // first tile not consumed
-  // Bulk-copy ring (quantised, contiguous, per-token keys): the stage that
+  // Bulk-copy ring (quantised per-token keys, contiguous or gathered by row
+  // copies): the stage that
   // tile t - 1 used is refilled as soon as every warp has finished it,
   // before tile t is awaited, so NST copies are in flight during each wait.
   // The barrier at the top of an iteration both frees that stage and lets
   // all threads agree whether a wait of the previous iteration gave up
   // (a warp whose wait gave up skips that tile's arithmetic).
-  constexpr bool kEarly = C::TMA && !gather && !C::KPC;
+  constexpr bool kEarly = C::TMA && !C::KPC && (!gather || C::GTMA);
   if constexpr (kEarly) {
     bool ok = true;
     int t_fail = -1;
@@ -1127,10 +1183,17 @@ __device__ __forceinline__ bool gqa_run_segment(const GqaDecodeArgs &a, int k, G
 // of a second, partial wave of splits.
 template <int BITS, int D, int KAX, int GS, bool GATHER, bool RUN>
 __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
-    gqa_decode_kernel(const GqaDecodeArgs a) {
+    gqa_decode_kernel(const __grid_constant__ CUtensorMap rows, const GqaDecodeArgs a) {
   pdl_wait();
   using C = GqaCfg<BITS, D, KAX, GS>;
   extern __shared__ __align__(128) uint8_t smem[];
+  if constexpr (GATHER && C::GTMA) {
+    // row-copy destinations are 128-byte aligned relative to the base
+    if (smem_u32(smem) & 127u) {
+      if (threadIdx.x == 0) set_err(a.err, 16);  // KVK_DEVERR_ALIGN
+      return;
+    }
+  }
   if constexpr (C::TMA) {
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + C::BAR_OFF);
     if (threadIdx.x == 0) {
@@ -1144,7 +1207,7 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     const int split = blockIdx.x;
     const int i0 = split * a.items_per_split;
     const int i1 = split == a.n_splits - 1 ? -1 : i0 + a.items_per_split;
-    gqa_decode_unit<BITS, D, KAX, GS, GATHER>(a, blockIdx.z, blockIdx.y, i0, i1, split, 0);
+    gqa_decode_unit<BITS, D, KAX, GS, GATHER>(a, &rows, blockIdx.z, blockIdx.y, i0, i1, split, 0);
   } else {
     static_assert(gqa_has_run<BITS, D, KAX, GS>() && !GATHER, "runs cover the contiguous bulk-copy formats");
     // Every thread derives the segments from blockIdx.x and the arguments
@@ -1166,11 +1229,13 @@ __global__ void __launch_bounds__(128, GqaCfg<BITS, D, KAX, GS>::MIN_CTAS)
     GqaRunSeg sg;
     if (!gqa_run_segment<C::TILE>(a, 0, sg)) return;
     // false: a wait gave up (the error word is set)
-    if (!gqa_decode_unit<BITS, D, KAX, GS, false>(a, sg.b, sg.kvh, sg.i0, sg.i1, sg.slot, 0)) return;
+    if (!gqa_decode_unit<BITS, D, KAX, GS, false>(a, &rows, sg.b, sg.kvh, sg.i0, sg.i1, sg.slot, 0))
+      return;
     mark_unused(sg);
     if (!gqa_run_segment<C::TILE>(a, 1, sg)) return;
     __syncthreads();  // the next unit's query and copies reuse shared memory
-    if (!gqa_decode_unit<BITS, D, KAX, GS, false>(a, sg.b, sg.kvh, sg.i0, sg.i1, sg.slot, 1)) return;
+    if (!gqa_decode_unit<BITS, D, KAX, GS, false>(a, &rows, sg.b, sg.kvh, sg.i0, sg.i1, sg.slot, 1))
+      return;
     mark_unused(sg);
   }
 }
@@ -1185,9 +1250,16 @@ cudaError_t launch_gqa_decode_g(const GqaDecodeArgs &a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  if constexpr (RUN) return launch_pdl(k, dim3(a.run_ctas), dim3(128), C::SMEM, st, a);
+  // the record table's tensor map (row gather), else an unused zero map
+  CUtensorMap rows;
+  memset(&rows, 0, sizeof rows);
+  if (GATHER && C::GTMA) {
+    if (!a.rows) return cudaErrorInvalidValue;
+    memcpy(&rows, a.rows, sizeof rows);
+  }
+  if constexpr (RUN) return launch_pdl(k, dim3(a.run_ctas), dim3(128), C::SMEM, st, rows, a);
   dim3 grid(a.n_splits, a.v.Hkv, a.v.B);
-  return launch_pdl(k, grid, dim3(128), C::SMEM, st, a);
+  return launch_pdl(k, grid, dim3(128), C::SMEM, st, rows, a);
 }
 
 template <int BITS, int D, int KAX, int GS>

@@ -57,6 +57,9 @@ struct GqaDecodeArgs {
   float *out;          // [B, Hq, D]: normalised output (single split)
   int32_t *err;
   uint32_t wait_limit = 1u << 22;  // polls of a bounded wait on this CTA's copies before it gives up
+  // host copy of the anchor's record-table tensor map (gqa_make_rows_tmap),
+  // required by the kept-list gather of grouped per-token records
+  const void *rows = nullptr;
   // run schedule (quantised formats with per-token keys or the symmetric
   // scheme, contiguous reads, partials only): run_ctas > 0 CTAs take equal
   // runs of the (unit, tile) grid of run_tpu kernel tiles per unit, into
@@ -72,6 +75,19 @@ struct GqaDecodeArgs {
 cudaError_t launch_gqa_decode(const GqaDecodeArgs &a, cudaStream_t st);
 int gqa_decode_ctas_per_sm(int bits, int D, int key_axis, int group, int scheme);
 int gqa_decode_tile(int bits, int D, int key_axis, int group, int scheme);
+// Whether the format's kept-list gather copies records by tensor-map rows,
+// and the 128-byte tensor map of an anchor's record table for it: rows
+// slab * cap + position, one record per row (B * Hkv * cap < 2^31).
+bool gqa_decode_row_gather(int bits, int key_axis, int scheme);
+cudaError_t gqa_make_rows_tmap(void *out, const GqaView &v);
+
+// cuTensorMapEncodeTiled reached through the runtime's driver entry point
+// (no link against the driver library); arguments in the driver's order,
+// enums as their integer values.  cudaErrorInvalidValue if it refuses.
+cudaError_t encode_tensor_map_tiled(void *map, int dtype, int rank, void *base,
+                                    const uint64_t *dims, const uint64_t *strides,
+                                    const uint32_t *box, const uint32_t *elem_strides,
+                                    int interleave, int swizzle, int l2_promotion, int oob_fill);
 
 struct RewindArgs {
   int32_t *lens[64];

@@ -190,7 +190,10 @@ struct kvk_cache {
   struct alignas(64) Tmap {
     uint8_t bytes[128];
   };
-  std::vector<Tmap> tmap;  // per MLA anchor, the decode kernel's tensor map
+  // per anchor: MLA, the decode kernel's tensor map; GQA with kept lists in
+  // a row-gather format, the record table's (gqa_make_rows_tmap)
+  std::vector<Tmap> tmap;
+  std::vector<char> has_tmap;
 
   GqaView gqa_view(int l) const {
     const ArenaLayout &A = lay[l];
@@ -479,16 +482,24 @@ kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg
     delete c;
     return cuda_fail(e, "querying the device");
   }
-  if (desc->kind == KVK_KIND_MLA) {
-    c->tmap.resize(desc->n_layers);
-    for (int l = 0; l < desc->n_layers; ++l) {
-      if (cfg[l].inherit || cfg[l].bits != 16) continue;  // quantised tiles use bulk copies
+  c->tmap.resize(desc->n_layers);
+  c->has_tmap.assign(desc->n_layers, 0);
+  for (int l = 0; l < desc->n_layers; ++l) {
+    if (cfg[l].inherit) continue;
+    if (desc->kind == KVK_KIND_MLA) {
+      if (cfg[l].bits != 16) continue;  // quantised tiles use bulk copies
       e = mla_make_tmap(c->tmap[l].bytes, c->mla_view(l));
-      if (e != cudaSuccess) {
-        delete c;
-        return cuda_fail(e, "encoding the tensor map of an MLA anchor");
-      }
+    } else {
+      if (cfg[l].evict_capacity <= 0 ||
+          !gqa_decode_row_gather(cfg[l].bits, cfg[l].key_axis, layer_scheme(&cfg[l])))
+        continue;
+      e = gqa_make_rows_tmap(c->tmap[l].bytes, c->gqa_view(l));
     }
+    if (e != cudaSuccess) {
+      delete c;
+      return cuda_fail(e, "encoding an anchor's tensor map");
+    }
+    c->has_tmap[l] = 1;
   }
   *out = c;
   return KVK_OK;
@@ -902,6 +913,7 @@ static kvk_status gqa_decode_common(kvk_cache *c, int32_t layer, const void *q, 
   args.items_per_split = tps * kTile;
   args.err = c->err();
   args.wait_limit = c->wait_limit;
+  args.rows = c->has_tmap[a] ? c->tmap[a].bytes : nullptr;
   if (runs) {
     args.run_ctas = rp.ctas;
     args.run_tpu = rp.tpu;

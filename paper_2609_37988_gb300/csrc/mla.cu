@@ -531,29 +531,13 @@ int mla_ctas_t() {
 // cuTensorMapEncodeTiled, reached through the runtime's entry-point query so
 // the library links the static runtime only.
 cudaError_t mla_make_tmap(void *out, const MlaView &v) {
-  using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
-                              const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
-                              const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
-                              CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-  static Encode encode = nullptr;
-  if (!encode) {
-    void *fn = nullptr;
-    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
-    const cudaError_t e =
-        cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-    if (e != cudaSuccess) return e;
-    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
-    encode = reinterpret_cast<Encode>(fn);
-  }
-  const cuuint64_t dims[2] = {(cuuint64_t)(v.width + v.rope), (cuuint64_t)v.B * (cuuint64_t)v.cap};
-  const cuuint64_t strides[1] = {(cuuint64_t)v.rec_bytes};
-  const cuuint32_t box[2] = {64, (cuuint32_t)mla_tile_rows(v.width)};
-  const cuuint32_t estr[2] = {1, 1};
-  const CUresult r = encode(static_cast<CUtensorMap *>(out), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                            v.rec, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+  const uint64_t dims[2] = {(uint64_t)(v.width + v.rope), (uint64_t)v.B * (uint64_t)v.cap};
+  const uint64_t strides[1] = {(uint64_t)v.rec_bytes};
+  const uint32_t box[2] = {64, (uint32_t)mla_tile_rows(v.width)};
+  const uint32_t estr[2] = {1, 1};
+  return encode_tensor_map_tiled(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, v.rec, dims, strides, box,
+                                 estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
 cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st) {
