@@ -262,8 +262,8 @@ kvk_status check_layer_index(const kvk_cache *c, int layer) {
 // waves of `slots`, and a partial last wave costs at least half a wave (its
 // CTAs have the SMs to themselves but run at most ~2x faster).  Measured on
 // the 7B and 14B step shapes, the 131k-context gather and the symmetric
-// formats, this model's pick is within 1 % of the best split count except
-// for the gather (10 %), where it keeps the previous choice.
+// formats, this model's pick is within 1 % of the best split count; the
+// kept-list gather has a rule of its own (auto_splits).
 int choose_splits(int units, int tiles, int per, int slots, int max_splits) {
   const double F = 2.0, tail = 0.5;
   if (tiles <= 1) return 1;
@@ -321,6 +321,16 @@ int auto_splits(kvk_cache *c, int a) {
   const kvk_layer_cfg &L = c->cfg[a];
   const int kt = gqa_decode_tile(L.bits, c->desc.head_dim, L.bits == 16 ? 0 : L.key_axis,
                                  layer_group(&c->desc, &L), layer_scheme(&L));
+  if (c->kept_on[a]) {
+    // Kept-list gathers (random record reads) run best with one wave of
+    // CTAs filling at most 85 % of the resident slots: at the 131k-context
+    // shape (32 units, int4 g32, 608 slots) 16 splits (512 CTAs) took 32.0
+    // us per call against 36.1 with 19 (every slot), 37.4 with 14, 35.5
+    // with 20; the same held for the earlier chunked gather (36.9 / 40.4).
+    const int ktiles = (layer_tiles(c, a) + kt / kTile - 1) / (kt / kTile);
+    const int s = (int)(0.85 * slots) / std::max(1, units);
+    return std::max(1, std::min(std::min(s, ktiles), c->max_splits));
+  }
   return choose_splits(units, layer_tiles(c, a), kt / kTile, slots, c->max_splits);
 }
 
