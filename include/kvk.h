@@ -347,10 +347,12 @@ kvk_status kvk_decode_partial(kvk_cache *cache, int32_t layer, const void *q,
  *    into the library; every GPU that loads the library holds that buffer
  *    until the process exits.
  *  - The partials take S * max_batch * n_q_heads * (head_dim + 2) floats,
- *    where S is the split count the call actually uses: n_splits, or the
- *    automatic count when n_splits is 0, in either case capped at the number
- *    of 64-position tiles of the context; a call that resolves to one split
- *    writes its output directly and needs no partials.  A call needing more
+ *    where S is the split count the call actually uses: n_splits capped at
+ *    the number of 64-position tiles of the context, or with n_splits = 0
+ *    the automatic plan's count (kvk_decode_plan_splits: the split count, or
+ *    under the run schedule the partial slots per (sequence, KV head)); a
+ *    call that resolves to one split of the split grid writes its output
+ *    directly and needs no partials.  A call needing more
  *    than 4,194,304 floats returns KVK_ERR_CAPACITY and enqueues nothing;
  *    pass fewer splits or use kvk_decode_attention.
  *  - The cache's device must be the current device (the buffer is per
