@@ -659,11 +659,42 @@ def main():
             traffic = ent.get("bytes_per_launch")
 
     # ---- end to end through the public API, host buffers --------------------
+    # The step's host copies run on a copy stream beside the layers, as a
+    # serving loop would issue them: the first layer's inputs, then the rest
+    # of the step's inputs, while the first layer runs; each group of
+    # OUT_CHUNK layers' outputs leave as soon as that group is done.  Every
+    # copy is inside the timed region; events order each layer after its
+    # inputs and each output copy after its layers.
+    OUT_CHUNK = 8
+    copy_stream = torch.cuda.Stream(device=dev)
+    n_out_chunks = (w.n_layers + OUT_CHUNK - 1) // OUT_CHUNK
+    ev_in = [torch.cuda.Event() for _ in range(2)]
+    ev_out = [torch.cuda.Event() for _ in range(n_out_chunks)]
+
+    def copies_in(first, rest):
+        # first(), rest(): the copies of layer 0's inputs and of the others'
+        copy_stream.wait_stream(stream)
+        with torch.cuda.stream(copy_stream):
+            first()
+            ev_in[0].record(copy_stream)
+            rest()
+            ev_in[1].record(copy_stream)
+        stream.wait_event(ev_in[0])
+
+    def copy_out(l, h_all, d_all):
+        # after layer l: the outputs of its group, when it is the group's last
+        if (l + 1) % OUT_CHUNK and l != w.n_layers - 1:
+            return
+        c = l // OUT_CHUNK
+        ev_out[c].record(stream)
+        copy_stream.wait_event(ev_out[c])
+        with torch.cuda.stream(copy_stream):
+            lo = c * OUT_CHUNK
+            h_all[lo:l + 1].copy_(d_all[lo:l + 1], non_blocking=True)
+
     e2e = None
     if args.e2e_steps > 0:
-        # one pinned host buffer and one device buffer per kind of tensor, so
-        # that a step's inputs arrive in two copies and its outputs leave in one
-        # (per-layer copies cost more in fixed latency than in bytes)
+        # one pinned host buffer and one device buffer per kind of tensor
         e_out_all = torch.empty((w.n_layers,) + tuple(outs[0].shape), dtype=outs[0].dtype, device=dev)
         e_outs = list(e_out_all.unbind(0))
         h_out_all = torch.empty(e_out_all.shape, dtype=e_out_all.dtype).pin_memory()
@@ -678,11 +709,20 @@ def main():
             h2d = h_qn.numel() * h_qn.element_size() + h_qp.numel() * h_qp.element_size()
 
             def e2e_body():
-                d_qn.copy_(h_qn, non_blocking=True)
-                d_qp.copy_(h_qp, non_blocking=True)
+                def first():
+                    d_qn[:1].copy_(h_qn[:1], non_blocking=True)
+                    d_qp[:1].copy_(h_qp[:1], non_blocking=True)
+
+                def rest():
+                    d_qn[1:].copy_(h_qn[1:], non_blocking=True)
+                    d_qp[1:].copy_(h_qp[1:], non_blocking=True)
+                copies_in(first, rest)
                 for l in range(w.n_layers):
+                    if l == 1:
+                        stream.wait_event(ev_in[1])
                     cache.decode_mla(l, d_qn[l], d_qp[l], mw[l][0], mw[l][1], w.sigma, out=e_outs[l])
-                h_out_all.copy_(e_out_all, non_blocking=True)
+                    copy_out(l, h_out_all, e_out_all)
+                stream.wait_stream(copy_stream)
     if args.e2e_steps > 0 and w.kind == "gqa":
         h_q_all = torch.stack([q.cpu() for q in qs]).pin_memory()
         d_q_all = torch.empty_like(h_q_all, device=dev)
@@ -695,15 +735,28 @@ def main():
         h2d = h_q_all.numel() * h_q_all.element_size() + \
             (h_kv_all.numel() * h_kv_all.element_size() if kv_layers else 0)
 
+        # layer 0's K/V, when it appends, are the first pair of the stack
+        n_kv0 = 2 if kv_layers and kv_layers[0] == 0 else 0
+
         def e2e_body():
-            d_q_all.copy_(h_q_all, non_blocking=True)
-            if kv_layers:
-                d_kv_all.copy_(h_kv_all, non_blocking=True)
+            def first():
+                d_q_all[:1].copy_(h_q_all[:1], non_blocking=True)
+                if n_kv0:
+                    d_kv_all[:n_kv0].copy_(h_kv_all[:n_kv0], non_blocking=True)
+
+            def rest():
+                d_q_all[1:].copy_(h_q_all[1:], non_blocking=True)
+                if kv_layers:
+                    d_kv_all[n_kv0:].copy_(h_kv_all[n_kv0:], non_blocking=True)
+            copies_in(first, rest)
             for l in range(w.n_layers):
+                if l == 1:
+                    stream.wait_event(ev_in[1])
                 if l in d_kv:
                     cache.append(l, *d_kv[l])
                 cache.decode(l, d_q[l], w.sigma, out=e_outs[l])
-            h_out_all.copy_(e_out_all, non_blocking=True)
+                copy_out(l, h_out_all, e_out_all)
+            stream.wait_stream(copy_stream)
             if w.append_per_step:
                 cache.rewind(1)
     if args.e2e_steps > 0:
@@ -724,7 +777,8 @@ def main():
                     g_e2e.replay()
                     stream.synchronize()
                 e2e_step()
-                e2e_mode = "cuda graph of the API calls and host copies"
+                e2e_mode = ("cuda graph of the API calls and host copies (copies on a second "
+                            "stream beside the layers)")
             except Exception:  # capture unsupported: stay eager
                 torch.cuda.synchronize()
             barrier()

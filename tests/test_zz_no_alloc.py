@@ -3,8 +3,9 @@ cannot provide scratch device memory.  Its split-K partials live in a fixed
 buffer inside the library; these checks call it through the C ABI on two
 calls in a row (the second call reuses a buffer still holding the first
 call's partials) and compare each result with the fp64 oracle on the same
-inputs and with kvk_decode_attention, and check that a request too large for
-the buffer is refused before anything runs.
+inputs and with kvk_decode_attention (split grid and run schedule), and
+check that a request too large for the buffer is refused before anything
+runs.
 
 Kept in a file of its own, collected last."""
 import ctypes
@@ -63,6 +64,26 @@ def test_matches_oracle_and_decode_on_two_calls_in_a_row():
         ref = c.decode(layer, q, scale, n_splits=ns)
         torch.cuda.synchronize()
         assert_close(out.cpu().numpy(), ref.cpu().numpy(), what=f"noalloc layer {layer} vs decode")
+    assert c.device_error() == 0
+
+
+def test_run_schedule():
+    """With the run schedule the automatic call (n_splits = 0) writes the
+    plan's partial slots into the fixed buffer and merges them: equal to the
+    oracle and to kvk_decode_attention on the same schedule."""
+    c, states = _cache_with_data(seed=3)
+    c.set_decode_schedule(c.SCHEDULE_RUNS, 11)
+    scale = 1.0 / math.sqrt(D)
+    q = torch.randn((B, HQ, D), generator=torch.Generator().manual_seed(4)).to(torch.bfloat16)
+    expected = gqa_expected(q, states[0], LENS, scale)
+    q = q.cuda()
+    out = torch.full((B, HQ, D), float("nan"), device="cuda")
+    assert _noalloc(c, 0, q, scale, out, 0) == 0
+    torch.cuda.synchronize()
+    assert_close(out.cpu().numpy(), expected, what="noalloc runs vs oracle")
+    ref = c.decode(0, q, scale)
+    torch.cuda.synchronize()
+    assert torch.equal(out, ref)
     assert c.device_error() == 0
 
 
