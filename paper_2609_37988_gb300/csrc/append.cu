@@ -38,10 +38,12 @@ __device__ __forceinline__ int seq_count(const int32_t *n_per_seq, int b, int n_
 }
 
 // rint(fl(d / s)) for s > 0 and |d / s| at most a few hundred, without a
-// division in the common case: y = fl(d fl(1/s)) is within 1.2e-7 |d/s| of
-// d/s, and fl(d/s) within 6e-8 |d/s|, so for |d/s| <= 300 the two differ by
-// less than 6e-5; when y is further than 1e-4 from the nearest half-integer
-// both round to the same integer.  Otherwise (or when y is not finite) the
+// division in the common case.  rs is the fast reciprocal of s
+// (__fdividef(1, s): within 2 ulp of 1/s for normal s), so y = fl(d rs) is
+// within 1.8e-7 |d/s| of d/s, and fl(d/s) within 6e-8 |d/s|: for |d/s| <=
+// 300 the two differ by less than 7.2e-5, and when y is further than 1e-4
+// from the nearest half-integer both round to the same integer.  Otherwise
+// (or when y is not finite, as for a scale whose reciprocal overflows) the
 // correctly rounded division decides.  `near` reports that case.
 __device__ __forceinline__ float rint_quot_fast(float d, float rs, bool &near) {
   const float y = __fmul_rn(d, rs);
@@ -66,7 +68,7 @@ __device__ __forceinline__ void quant_lane(const float (&x)[E], int GS, int leve
   }
   const float lev = (float)levels;
   const float scale = __fdiv_rn(__fsub_rn(mx, mn), lev);
-  const float rs = scale == 0.f ? 0.f : __frcp_rn(scale);
+  const float rs = scale == 0.f ? 0.f : __fdividef(1.f, scale);
   float r[E];
   bool any_near = false;
 #pragma unroll
@@ -102,7 +104,7 @@ __device__ __forceinline__ uint16_t quant_sym_lane(const float (&x)[E], int bits
   const float q = (float)sym_levels(bits);
   const uint16_t sb = f32_to_bf16_bits(__fdiv_rn(am, q));
   const float s = bf16_to_f32(sb);
-  const float rs = s == 0.f ? 0.f : __frcp_rn(s);
+  const float rs = s == 0.f ? 0.f : __fdividef(1.f, s);
   float rq[E];
   bool any_near = false;
 #pragma unroll
@@ -274,6 +276,36 @@ __device__ void append_row(const GqaView &v, const float (&xk)[D / 32], const fl
   }
 }
 
+// Row wid = (b n_new + i) Hkv + kvh of an append, tracked as (b, i, kvh)
+// and advanced by a fixed stride with carries instead of divided per row:
+// the stride's own decomposition is computed once.
+struct RowIdx {
+  uint32_t b, i, kvh;
+};
+struct RowStep {
+  uint32_t Hkv, n_new, db, di, dk;
+  __device__ RowStep(uint32_t step, uint32_t Hkv_, uint32_t n_new_) : Hkv(Hkv_), n_new(n_new_) {
+    const uint32_t q = step / Hkv;
+    dk = step - q * Hkv;
+    db = q / n_new;
+    di = q - db * n_new;
+  }
+  __device__ RowIdx at(uint32_t w) const {
+    const uint32_t q = w / Hkv, b = q / n_new;
+    return RowIdx{b, q - b * n_new, w - q * Hkv};
+  }
+  __device__ RowIdx next(RowIdx r) const {  // the row `step` further on
+    r.kvh += dk;
+    const uint32_t c = r.kvh >= Hkv;
+    r.kvh -= c ? Hkv : 0u;
+    r.i += di + c;
+    const uint32_t c2 = r.i >= n_new;
+    r.i -= c2 ? n_new : 0u;
+    r.b += db + c2;
+    return r;
+  }
+};
+
 template <int D>
 __global__ void __launch_bounds__(128)
     gqa_append_rows(const GqaView v, const void *kin, const void *vin, int in_f32, int n_new,
@@ -286,10 +318,13 @@ __global__ void __launch_bounds__(128)
   const size_t total = (size_t)v.B * n_new * v.Hkv;
   // rows wid, wid + 4 gridDim.x, ...: a bounded grid, so that the completion
   // counter below takes one atomic per CTA, not one per four rows
+  // (the grid stride and the first row fit 32 bits; the row index itself
+  // stays 64-bit, its (b, i, kvh) advance by the stride)
+  const RowStep rstep((uint32_t)gridDim.x * 4u, (uint32_t)v.Hkv, (uint32_t)n_new);
+  RowIdx ridx = rstep.at((uint32_t)min((size_t)blockIdx.x * 4 + warp, total));
   for (size_t wid = (size_t)blockIdx.x * 4 + warp; wid < total; wid += (size_t)gridDim.x * 4) {
-    const int kvh = (int)(wid % v.Hkv);
-    const int i = (int)((wid / v.Hkv) % n_new);
-    const int b = (int)(wid / ((size_t)v.Hkv * n_new));
+    const int kvh = (int)ridx.kvh, i = (int)ridx.i, b = (int)ridx.b;
+    ridx = rstep.next(ridx);
     const int nb = seq_count(n_per_seq, b, n_new, err);
     const int t = v.lens[b] + i;
     bool ok = i < nb;
@@ -530,6 +565,9 @@ __global__ void __launch_bounds__(256)
     }
   };
   const size_t step = (size_t)gridDim.x * wpb;
+  // 32-bit index arithmetic (the launcher sends fewer than 2^31 rows)
+  const RowStep rstep((uint32_t)step, (uint32_t)v.Hkv, (uint32_t)n_new);
+  RowIdx ridx = rstep.at((uint32_t)min((size_t)blockIdx.x * wpb + warp, total));
   for (size_t w0 = (size_t)blockIdx.x * wpb + warp; w0 < total; w0 += 2 * step) {
     bool ok[2];
     size_t row[2];
@@ -538,16 +576,14 @@ __global__ void __launch_bounds__(256)
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
       const size_t wid = w0 + u * step;
+      const RowIdx r = ridx;
+      ridx = rstep.next(ridx);  // row wid + step
       ok[u] = false;
       row[u] = 0;
       tt[u] = 0;
       size_t in_off = 0;
       if (wid < total) {
-        // 32-bit index arithmetic (the launcher sends fewer than 2^31 rows)
-        const uint32_t w = (uint32_t)wid, q = w / (uint32_t)v.Hkv;
-        const int kvh = (int)(w - q * (uint32_t)v.Hkv);
-        const uint32_t bq = q / (uint32_t)n_new;
-        const int i = (int)(q - bq * (uint32_t)n_new), b = (int)bq;
+        const int kvh = (int)r.kvh, i = (int)r.i, b = (int)r.b;
         in_off = wid * D;  // inputs are [B, n_new, H_kv, D], row wid
         const int nb = seq_count(n_per_seq, b, n_new, err);
         const int t = v.lens[b] + i;
