@@ -255,9 +255,9 @@ kvk_status kvk_evict_window(kvk_cache *cache, int32_t layer, const void *q_win, 
  *           16-byte aligned;
  *  out:     device float32 [B, n_q, H_q, head_dim], 16-byte aligned;
  *  scratch: device, 256-byte aligned, at least kvk_prefill_scratch_size
- *           bytes: per-row softmax statistics and the anchor's cache
- *           dequantised once into the products' operand layout (1 KB per
- *           position and KV head for quantised anchors, 512 B for bf16).
+ *           bytes: the anchor's cache dequantised once into the products'
+ *           operand layout (1 KB per position and KV head for quantised
+ *           anchors, 512 B for bf16) and a job counter.
  * Errors: UNSUPPORTED (MLA: see kvk_prefill_attention_mla; head_dim != 128),
  * INVALID_ARG (n_q outside [1, max_ctx], null or misaligned pointers,
  * scale not finite and positive, scratch too small). */

@@ -135,9 +135,8 @@ struct PfArgs {
   int q_f32;
   int Hq, G, n_q;
   float sig_log2;      // softmax scale * log2(e)
-  float2 *stats;       // [B * Hkv][n_q * G] (max, sum) per row
   float *out;          // [B, n_q, Hq, D]
-  int *counter;        // two job counters (statistics, output), zeroed by the launch
+  int *counter;        // the job counter, zeroed by the launch
   uint8_t *tiles;      // [B * Hkv][cap / 64] expanded tiles of prefill_tile_bytes(bits)
   int32_t *err;
 };

@@ -250,21 +250,21 @@ kvk_status check_layer_index(const kvk_cache *c, int layer) {
   return KVK_OK;
 }
 
-// Split count that best fills the GPU: whole waves of CTAs, equal tile
-// counts per split, and at least 16 64-position tiles per CTA so the
-// per-CTA query set-up and the split partials stay a small share of the
-// work.  Among choices within 1% the fewer splits win.
 // Split count of a GQA decode: `tiles` 64-item tiles per (sequence, KV head)
 // unit, kernel tiles of `per` such tiles, `slots` resident CTAs.  Cost model
 // of a split count s: the launch rounds split boundaries to the kernel tile,
 // so each working CTA runs nt kernel tiles plus a fixed cost of about two
 // tiles (query set-up, merge of the warps' states, the partial); CTAs run in
 // waves of `slots`, and a partial last wave costs at least half a wave (its
-// CTAs have the SMs to themselves but run at most ~2x faster).  Measured on
-// the 7B and 14B step shapes, the 131k-context gather and the symmetric
-// formats, this model's pick is within 1 % of the best split count; the
-// kept-list gather has a rule of its own (auto_splits).
-int choose_splits(int units, int tiles, int per, int slots, int max_splits) {
+// CTAs have the SMs to themselves but run at most ~2x faster).  For the
+// bf16 kernel (`full_tail`), bound by HBM rather than by its issue rate, a
+// partial last wave costs a whole wave.  Among choices within
+// 1 % the fewer splits win.  Measured on the 7B and 14B step shapes and
+// every format, this model's pick is within 1 % of the best split count
+// (bf16 at the 14B step: 5 splits, 163.6 us, against 167.2 with the 3 of
+// the quantised kernels' rule; B = 16..48 and T = 4096..16384 likewise);
+// the kept-list gather has a rule of its own (auto_splits).
+int choose_splits(int units, int tiles, int per, int slots, int max_splits, bool full_tail) {
   const double F = 2.0, tail = 0.5;
   if (tiles <= 1) return 1;
   per = std::max(1, per);
@@ -281,7 +281,8 @@ int choose_splits(int units, int tiles, int per, int slots, int max_splits) {
       t = F + nt;
     } else {
       const double fl = std::floor(w), f = w - fl;
-      t = (F + nt) * (fl + (f > 1e-9 ? std::max(f, tail) : 0.0));
+      const double last = f <= 1e-9 ? 0.0 : full_tail ? 1.0 : std::max(f, tail);
+      t = (F + nt) * (fl + last);
     }
     if (t < best_t * 0.99) {
       best_t = t;
@@ -331,7 +332,7 @@ int auto_splits(kvk_cache *c, int a) {
     const int s = (int)(0.85 * slots) / std::max(1, units);
     return std::max(1, std::min(std::min(s, ktiles), c->max_splits));
   }
-  return choose_splits(units, layer_tiles(c, a), kt / kTile, slots, c->max_splits);
+  return choose_splits(units, layer_tiles(c, a), kt / kTile, slots, c->max_splits, L.bits == 16);
 }
 
 // The run schedule of an automatic decode of anchor a (kernel side in
@@ -769,18 +770,17 @@ kvk_status check_prefill(const kvk_cache *c, int32_t layer, int32_t n_q) {
     return fail(KVK_ERR_INVALID_ARG, "n_q %d outside [1, max_ctx]", n_q);
   return KVK_OK;
 }
-// Pre-fill scratch: the rows' statistics, the two job counters, then the
-// expanded tiles (every 64-position tile of every unit, dequantised once).
+// Pre-fill scratch: the job counter, then the expanded tiles (every
+// 64-position tile of every unit, dequantised once).
 struct PrefillScratch {
-  size_t stats, counters, tiles, total;
+  size_t counters, tiles, total;
 };
 PrefillScratch prefill_scratch(const kvk_cache *c, int32_t layer, int32_t n_q) {
+  (void)n_q;
   PrefillScratch p;
   const int a = c->src[layer];
-  const size_t rows = (size_t)c->desc.max_batch * c->desc.n_q_heads * n_q;  // units x n_q G
-  p.stats = 0;
-  p.counters = (size_t)align256((int64_t)(rows * 8));
-  p.tiles = (size_t)((p.counters + 256 + 1023) & ~(size_t)1023);
+  p.counters = 0;
+  p.tiles = 1024;
   const size_t units = (size_t)c->desc.max_batch * c->desc.n_kv_heads;
   p.total = p.tiles + units * (size_t)(c->lay[a].cap / 64) * prefill_tile_bytes(c->cfg[a].bits);
   return p;
@@ -851,7 +851,6 @@ kvk_status kvk_prefill_attention(kvk_cache *c, int32_t layer, const void *q, int
   a.G = c->desc.n_q_heads / c->desc.n_kv_heads;
   a.n_q = n_q;
   a.sig_log2 = softmax_scale * 1.4426950408889634f;
-  a.stats = static_cast<float2 *>(scratch);
   a.counter = reinterpret_cast<int *>(static_cast<uint8_t *>(scratch) + ps.counters);
   a.tiles = static_cast<uint8_t *>(scratch) + ps.tiles;
   a.out = out;

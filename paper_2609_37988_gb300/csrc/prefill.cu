@@ -8,19 +8,20 @@
 // Rows: row r = i G + h of a (sequence, KV head) unit is chunk query i and
 // head h of the KV head's group; query i sits at position len - n_q + i and
 // sees positions 0 .. len - n_q + i.  A job is 128 consecutive rows of one
-// unit.  Three launches:
+// unit.  Two launches:
 //  * expand: every 64-position tile of the cache is dequantised once into
 //    the layout the products read (bf16 hi and lo halves, K-major
 //    128-byte-swizzled boxes), in caller scratch;
-//  * statistics: per row, the maximum M and the sum L of 2^(x - M) of its
-//    scaled scores x = sigma log2(e) <q, k> over its causal range, online
-//    over the tiles (S = Q K^T with TMEM lane = row);
-//  * outputs: per tile, S = Q K^T, P = 2^(x - M - log2 L) (zero past the
-//    row's limit) as bf16 hi and lo pairs into TMEM, O += P V (P the A
-//    operand from TMEM, the value tile an MN-major B operand); after the
-//    job's last tile O (TMEM lane = row) is written out.  The normalisers
-//    being final, O is never rescaled.
-// The two attention kernels run one persistent CTA per SM: a copy warp
+//  * attention, one pass over the tiles: per tile, S = Q K^T (TMEM lane =
+//    row) with x = sigma log2(e) <q, k>; each row's maximum over the tile
+//    (its four slices' maxima through shared memory) against the row's
+//    reference m, which moves only when a score rises more than 8 above it
+//    (O and the row's sums then rescaled by 2^(m_old - m_new) in place);
+//    P = 2^(x - m) (zero past the row's limit, at most 2^8) as bf16 hi and
+//    lo pairs into TMEM, O += P V (P the A operand from TMEM, the value
+//    tile an MN-major B operand); after the job's last tile O (TMEM lane =
+//    row) is divided by the row's sum of P and written out.
+// The attention kernel runs one persistent CTA per SM: a copy warp
 // brings each job's tiles in with bulk copies, three MMA warps issue the
 // tcgen05 products (one thread issues at most one product per ~45 cycles:
 // the scores of even and of odd tiles, and the value products, are three
@@ -61,7 +62,7 @@ struct PfPlan {
   int ns;             // key stages of the attention kernels
   int nv;             // value stages (output pass)
   int band;           // units per band of the job order
-  int off_v, off_norm, off_red, off_bar, smem, smem_x;  // key stages at offset 0
+  int off_v, off_red, off_bar, smem, smem_x;  // key stages at offset 0
 };
 
 // Tiles a job reads: positions up to that of the job's last row.
@@ -218,7 +219,6 @@ __device__ __forceinline__ void pf_issue_values(uint32_t t_o, uint32_t pa, uint3
   }
 }
 
-template <bool OUT>
 __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, const PfPlan p) {
   constexpr int D = 128;
   constexpr uint32_t kLimit = 1u << 20;  // polls of up to 2 us each
@@ -240,8 +240,6 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + p.off_bar + kBars * 8);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + p.off_bar + kBars * 8 + 4);
   volatile int *s_job = reinterpret_cast<volatile int *>(sm + p.off_bar + kBars * 8 + 8);
-  float *norm = reinterpret_cast<float *>(sm + p.off_norm);  // [128] log-normaliser per job row
-  float2 *red = reinterpret_cast<float2 *>(sm + p.off_red);  // [4][128] slice statistics
   const GqaView &v = a.v;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int R = a.n_q * a.G;
@@ -259,7 +257,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     fence_mbar_init();
   }
   pdl_wait();  // the expanded tiles, lengths and (output pass) statistics are complete
-  constexpr uint32_t kCols = OUT ? 512 : 256;
+  constexpr uint32_t kCols = 512;
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(tbase)),
@@ -277,7 +275,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   // (fp32, 128 channels) and P of tile k at 256 + 64 (k & 1) (bf16 pairs,
   // hi 32 columns, then lo), the A operand of the value products.
   const uint32_t t_o = tmem + 128;
-  const uint32_t t_q = tmem + (OUT ? 384 : 128);
+  const uint32_t t_q = tmem + 384;
   auto t_p = [&](int k) { return tmem + 256 + 64 * (k & 1); };
 
   // Jobs are handed out one at a time from a counter, so CTAs finish
@@ -288,7 +286,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   // keeps taking jobs (and skips them) until none is left, so no barrier
   // waits for threads that left.
   const int units = v.B * v.Hkv;
-  int *counter = a.counter + (OUT ? 1 : 0);
+  int *counter = a.counter;
   auto next_job = [&]() -> int {
     asm volatile("bar.sync 2, %0;" ::"n"(kPfThreads) : "memory");  // the previous id is read
     if (tid == 0) *s_job = atomicAdd(counter, 1);
@@ -338,7 +336,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
             mbar_expect_tx(&kfull[s], p.kbytes);
             bulk_g2s(sm + s * p.kbytes, src0 + (size_t)k * p.tbytes, p.kbytes, &kfull[s]);
           }
-          if (OUT && ok) {
+          if (ok) {
             const int sv = kk % p.nv, uv = kk / p.nv;
             if (uv > 0) ok = sleepy(&vfree[sv], (uv - 1) & 1);
             if (ok) {
@@ -356,7 +354,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
     if (lane == 0)
       for (int c = max(0, kk - max(p.ns, p.nv)); c < kk; ++c) {
         if (c >= kk - p.ns) mbar_wait(&kfull[c % p.ns], (c / p.ns) & 1, 1u << 22);
-        if (OUT && c >= kk - p.nv) mbar_wait(&vfull[c % p.nv], (c / p.nv) & 1, 1u << 22);
+        if (c >= kk - p.nv) mbar_wait(&vfull[c % p.nv], (c / p.nv) & 1, 1u << 22);
       }
     __syncwarp();
   } else if (warp >= kPfWorkers / 32) {
@@ -418,7 +416,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
             if (ok) ok = sleepy(&kfull[s], (kk / p.ns) & 1);
             if (ok) issue_s(kk, s);
             ++issued;
-          } else if (OUT && role == 2) {
+          } else if (role == 2) {
             ok = pv(kk, k > 0);
             ++issued;
           }
@@ -477,22 +475,13 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       for (int i = 0; i < 16; ++i) split2<true>(x[2 * i], x[2 * i + 1], hw[i], lw[i]);
       tmem_st16_nw(t_q + 16 * slice + lane_off, hw);
       if (p.q_lo) tmem_st16_nw(t_q + 64 + 16 * slice + lane_off, lw);
-      if constexpr (OUT) {
-        for (int r2 = tid; r2 < kPfRows; r2 += kPfWorkers) {
-          float nv = INFINITY;
-          if (r2 < J.nr) {
-            const float2 f = a.stats[(size_t)J.unit * R + J.r0 + r2];
-            if (f.y > 0.f) nv = f.x + log2f(f.y);
-          }
-          norm[r2] = nv;
-        }
-      }
       tmem_wait_st();
       tc_fence_before();  // the rows, stored here, are read by the tensor cores
       workers_sync<kPfWorkers>();
     };
 
     int kk = 0;
+    float *smax = reinterpret_cast<float *>(sm + p.off_red);  // [4 slices][128 rows]
     for (int job = next_job(); job < p.n_jobs; job = next_job()) {
       if (failed) continue;
       const Job J = job_at(job);
@@ -500,16 +489,21 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
       load_q(J);
       __syncwarp();
       if (lane == 0) mbar_arrive(qready);
-      // this thread's row of the job in the score epilogues
+      // this thread's row of the job (and slice of each tile's positions)
       const int rl = 32 * quarter + lane;
       const bool row_live = rl < J.nr;
       const int last = base + (J.r0 + rl) / a.G;  // the last position the row sees
-      const bool warp_live = 32 * quarter < J.nr;
-      float m_run = -INFINITY, l_run = 0.f;  // statistics: this slice's running pair
+      // The row's reference maximum (scaled scores, base 2) and this slice's
+      // sum of weights.  The reference stays while no score of the row rises
+      // more than 8 above it (P <= 2^8); when one does, the row's four
+      // threads move it and rescale their channels of O (in TMEM, after the
+      // value product of the previous tile) and their sums.  The weights
+      // are not normalised: O is divided by the row's sum at the end.
+      float c_ref = -INFINITY, l_run = 0.f;
       for (int k = 0; k < J.n_t; ++k, ++kk) {
-        // scores of this tile; output pass: its P buffer is free
-        bool ok = sleepy(&sdone[kk & 1], (kk >> 1) & 1);
-        if (OUT && ok) ok = wait_pv(kk - 2);  // its P buffer is free
+        // scores of this tile, and its P buffer free
+        bool ok = !failed && sleepy(&sdone[kk & 1], (kk >> 1) & 1);
+        if (ok) ok = wait_pv(kk - 2);
         if (workers_sync_or<kPfWorkers>(!ok)) {
           failed = true;
           *abort_flag = 1;
@@ -517,121 +511,123 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
         }
         tc_fence_after();
         const int tb = k * kPfT + 16 * slice;  // first position of this thread's slice
-        if constexpr (!OUT) {
-          // online (max, sum) of this row over the slice's 16 positions
-          if (warp_live) {
-            float y[16];
-            tmem_ld16(tmem + 64u * (kk & 1) + 16 * slice + lane_off, y);
-            const int nv = min(16, last - tb + 1);
-            if (row_live && nv > 0) {
-              float ll[4] = {0.f, 0.f, 0.f, 0.f}, mn;
-              if (nv == 16) {  // the whole slice is in the row's range (most tiles)
-                float mm[4];
+        const int nv = row_live ? min(16, last - tb + 1) : 0;  // live positions (<= 0: none)
+        float y[16];
+        tmem_ld16(tmem + 64u * (kk & 1) + 16 * slice + lane_off, y);
+        float mx = -INFINITY;
+        if (nv >= 16) {  // the whole slice is in the row's range (most tiles)
+          float mm[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) mm[i] = fmaxf(fmaxf(y[i], y[4 + i]), fmaxf(y[8 + i], y[12 + i]));
-                mn = fmaxf(m_run, fmaxf(fmaxf(mm[0], mm[1]), fmaxf(mm[2], mm[3])) * sg);
+          for (int i = 0; i < 4; ++i) mm[i] = fmaxf(fmaxf(y[i], y[4 + i]), fmaxf(y[8 + i], y[12 + i]));
+          mx = fmaxf(fmaxf(mm[0], mm[1]), fmaxf(mm[2], mm[3]));
+        } else {
 #pragma unroll
-                for (int i = 0; i < 16; ++i) ll[i & 3] += fast_exp2(fmaf(y[i], sg, -mn));
-              } else {
-                float mm = -INFINITY;
+          for (int i = 0; i < 16; ++i)
+            if (i < nv) mx = fmaxf(mx, y[i]);
+        }
+        smax[slice * kPfRows + rl] = mx;
+        workers_sync<kPfWorkers>();  // the row's four slice maxima
+        const float M = sg * fmaxf(fmaxf(smax[rl], smax[kPfRows + rl]),
+                                   fmaxf(smax[2 * kPfRows + rl], smax[3 * kPfRows + rl]));
+        if (M > c_ref + 8.f) {  // the same decision on the row's four threads
+          if (c_ref != -INFINITY) {
+            // O holds this job's earlier tiles: rescale this thread's 32
+            // channels once the previous tile's value product is done
+            if (!wait_pv(kk - 1)) {
+              failed = true;
+              *abort_flag = 1;
+            } else {
+              tc_fence_after();
+              const float f = fast_exp2(c_ref - M);
+              float z[16];
+              uint32_t zw[16];
 #pragma unroll
-                for (int i = 0; i < 16; ++i)
-                  if (i < nv) mm = fmaxf(mm, y[i]);
-                mn = fmaxf(m_run, mm * sg);
+              for (int h = 0; h < 2; ++h) {
+                tmem_ld16(t_o + 32 * slice + 16 * h + lane_off, z);
 #pragma unroll
-                for (int i = 0; i < 16; ++i)
-                  if (i < nv) ll[i & 3] += fast_exp2(fmaf(y[i], sg, -mn));
+                for (int i = 0; i < 16; ++i) zw[i] = __float_as_uint(z[i] * f);
+                tmem_st16_nw(t_o + 32 * slice + 16 * h + lane_off, zw);
               }
-              l_run = l_run * fast_exp2(m_run - mn) + ((ll[0] + ll[1]) + (ll[2] + ll[3]));
-              m_run = mn;
+              l_run *= f;
             }
+          }
+          c_ref = M;
+        }
+        // P of this row over the slice's 16 positions, hi and lo halves
+        float x0[8], x1[8];
+        if (nv >= 16) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            x0[i] = fast_exp2(fmaf(y[i], sg, -c_ref));
+            x1[i] = fast_exp2(fmaf(y[8 + i], sg, -c_ref));
           }
         } else {
-          // P of this row over the slice's 16 positions, hi and lo halves
-          float y[16];
-          tmem_ld16(tmem + 64u * (kk & 1) + 16 * slice + lane_off, y);
-          const float c = norm[rl];
-          float x0[8], x1[8];
-          if (tb + 15 <= last) {  // the whole slice is in the row's range (most tiles)
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              x0[i] = fast_exp2(fmaf(y[i], sg, -c));
-              x1[i] = fast_exp2(fmaf(y[8 + i], sg, -c));
-            }
-          } else {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              x0[i] = tb + i <= last ? fast_exp2(fmaf(y[i], sg, -c)) : 0.f;
-              x1[i] = tb + 8 + i <= last ? fast_exp2(fmaf(y[8 + i], sg, -c)) : 0.f;
-            }
+          for (int i = 0; i < 8; ++i) {
+            x0[i] = i < nv ? fast_exp2(fmaf(y[i], sg, -c_ref)) : 0.f;
+            x1[i] = 8 + i < nv ? fast_exp2(fmaf(y[8 + i], sg, -c_ref)) : 0.f;
           }
-          // positions 16 slice .. 16 slice + 15 of the tile: 8 columns of
-          // bf16 pairs (hi), the same 32 columns on (lo)
-          uint32_t hw[8], lw[8];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            split2<true>(x0[2 * i], x0[2 * i + 1], hw[i], lw[i]);
-            split2<true>(x1[2 * i], x1[2 * i + 1], hw[4 + i], lw[4 + i]);
-          }
-          tmem_st8_nw(t_p(kk) + 8 * slice + lane_off, hw);
-          tmem_st8_nw(t_p(kk) + 32 + 8 * slice + lane_off, lw);
-          tmem_wait_st();
         }
+        // positions 16 slice .. 16 slice + 15 of the tile: 8 columns of
+        // bf16 pairs (hi), the same 32 columns on (lo)
+        uint32_t hw[8], lw[8];
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          split2<true>(x0[2 * i], x0[2 * i + 1], hw[i], lw[i]);
+          split2<true>(x1[2 * i], x1[2 * i + 1], hw[4 + i], lw[4 + i]);
+          ls[i] += (x0[2 * i] + x0[2 * i + 1]) + (x1[2 * i] + x1[2 * i + 1]);
+        }
+        l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        tmem_st8_nw(t_p(kk) + 8 * slice + lane_off, hw);
+        tmem_st8_nw(t_p(kk) + 32 + 8 * slice + lane_off, lw);
+        tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&epi[kk & 1]);
       }
-      if (failed) continue;
-      if constexpr (!OUT) {
-        // the four slices' pairs of each row, combined
-        red[slice * kPfRows + rl] = make_float2(m_run, l_run);
-        workers_sync<kPfWorkers>();
-        if (slice == 0 && row_live) {
-          float M = -INFINITY;
-#pragma unroll
-          for (int s2 = 0; s2 < 4; ++s2) M = fmaxf(M, red[s2 * kPfRows + rl].x);
-          float L = 0.f;
-          if (M != -INFINITY)
-#pragma unroll
-            for (int s2 = 0; s2 < 4; ++s2) {
-              const float2 e = red[s2 * kPfRows + rl];
-              if (e.x != -INFINITY) L += e.y * fast_exp2(e.x - M);
-            }
-          a.stats[(size_t)J.unit * R + J.r0 + rl] = make_float2(M, L);
-        }
-        workers_sync<kPfWorkers>();
-      } else {
-        // O: lane = the job's row, 32 channels per slice
-        float o[32];
-        if (J.n_t > 0) {
-          const bool ok = wait_pv(kk - 1);
-          if (workers_sync_or<kPfWorkers>(!ok)) {
-            failed = true;
-            *abort_flag = 1;
-            continue;
-          }
-          tc_fence_after();
-          float z[16];
-          tmem_ld16(t_o + 32 * slice + lane_off, z);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) o[i] = z[i];
-          tmem_ld16(t_o + 32 * slice + 16 + lane_off, z);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) o[16 + i] = z[i];
-        } else {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] = 0.f;
-        }
-        if (row_live) {
-          const int r = J.r0 + rl;
-          const int qi = r / a.G, h = J.j * a.G + (r - qi * a.G);
-          float4 *dst = reinterpret_cast<float4 *>(a.out + (((size_t)J.b * a.n_q + qi) * a.Hq + h) * D + 32 * slice);
-#pragma unroll
-          for (int c = 0; c < 8; ++c) dst[c] = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
-        }
-        tc_fence_before();
-        workers_sync<kPfWorkers>();  // O read before the next job's first value product
+      // a rescale's wait that gave up on the last tile is seen by every worker
+      if (workers_sync_or<kPfWorkers>(failed)) {
+        failed = true;
+        *abort_flag = 1;
+        continue;
       }
+      // O: lane = the job's row, 32 channels per slice, divided by the sum
+      // of the row's weights (the four slices' sums, same reference)
+      float o[32];
+      if (J.n_t > 0) {
+        const bool ok = wait_pv(kk - 1);
+        if (workers_sync_or<kPfWorkers>(!ok)) {
+          failed = true;
+          *abort_flag = 1;
+          continue;
+        }
+        tc_fence_after();
+        float z[16];
+        tmem_ld16(t_o + 32 * slice + lane_off, z);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o[i] = z[i];
+        tmem_ld16(t_o + 32 * slice + 16 + lane_off, z);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o[16 + i] = z[i];
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) o[i] = 0.f;
+      }
+      smax[slice * kPfRows + rl] = l_run;
+      workers_sync<kPfWorkers>();
+      const float L = (smax[rl] + smax[kPfRows + rl]) + (smax[2 * kPfRows + rl] + smax[3 * kPfRows + rl]);
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      if (row_live) {
+        const int r = J.r0 + rl;
+        const int qi = r / a.G, h = J.j * a.G + (r - qi * a.G);
+        float4 *dst = reinterpret_cast<float4 *>(a.out + (((size_t)J.b * a.n_q + qi) * a.Hq + h) * D + 32 * slice);
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          dst[c] = make_float4(o[4 * c] * inv, o[4 * c + 1] * inv, o[4 * c + 2] * inv, o[4 * c + 3] * inv);
+      }
+      tc_fence_before();
+      workers_sync<kPfWorkers>();  // O and the sums read before the next job's first products
     }
     if (failed && tid == 0) set_err(a.err, 8);
   }
@@ -644,11 +640,11 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const PfArgs a, 
   pdl_trigger();
 }
 
-// Shared-memory plan.  Attention kernels: the job's query rows (hi, then
-// lo), the key stages, the value stages and P (output pass), normalisers,
-// slice statistics (statistics pass), barriers; as many stages (up to three)
-// as fit.  Expand kernel: one tile and its staged records.
-PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
+// Shared-memory plan.  Attention kernel: the key stages, the value stages,
+// the rows' slice maxima (and at a job's end their sums of weights),
+// barriers; the query rows, S, P and O live in TMEM.  Expand kernel: one
+// tile and its staged records.
+PfPlan pf_plan(const PfArgs &a, int sms) {
   PfPlan p;
   const int R = a.n_q * a.G;
   p.n_rb = (R + kPfRows - 1) / kPfRows;
@@ -671,29 +667,21 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
   p.tbytes = 2 * p.kbytes;
   // + the (scale, zero) rows of the tile's position groups (per-channel keys)
   p.smem_x = p.tbytes + kPfT * p.b_stride + (p.kpc ? 2 * 128 * 8 : 0) + 1024;
-  const int vb = out ? p.tbytes - p.kbytes : 0;
-  const int nbytes = out ? kPfRows * 4 : 0;
-  const int rbytes = out ? 0 : 4 * kPfRows * 8;
-  // the most stages that fit (query rows and P live in TMEM).  Output
-  // pass: value tiles wait for the value product three tiles back, key
-  // tiles only for the score product, so values get the larger share
-  // (int4: 2 key and 5 value stages of 32 KB); keys keep at least two
-  // (a score warp's wait for the stage it skipped relies on ns >= 2).
-  const int avail = 232448 - (nbytes + rbytes + kPfBarBytes + 1024);
-  if (!out) {
-    p.ns = std::max(1, std::min(kPfMaxStages, avail / p.kbytes));
-    p.nv = 1;
-  } else {
-    const int T = avail / p.kbytes;  // key and value tiles are the same size
-    p.ns = std::min(kPfMaxStages, std::max(2, T / 3));
-    p.nv = std::max(1, std::min(kPfMaxStages, T - p.ns));
-  }
+  const int vb = p.tbytes - p.kbytes;
+  const int rbytes = 4 * kPfRows * 4;
+  // the most stages that fit.  Value tiles wait for the value product three
+  // tiles back, key tiles only for the score product, so values get the
+  // larger share (int4: 2 key and 5 value stages of 32 KB); keys keep at
+  // least two (a score warp's wait for the stage it skipped relies on ns >= 2).
+  const int avail = 232448 - (rbytes + kPfBarBytes + 1024);
+  const int T = avail / p.kbytes;  // key and value tiles are the same size
+  p.ns = std::min(kPfMaxStages, std::max(2, T / 3));
+  p.nv = std::max(1, std::min(kPfMaxStages, T - p.ns));
   // bands of units whose tiles take up to 32 MB (L2 holds two bands)
-  const long long unit_bytes = (long long)p.n_t64 * (out ? p.tbytes : p.kbytes);
+  const long long unit_bytes = (long long)p.n_t64 * p.tbytes;
   p.band = (int)std::max(1LL, std::min<long long>(a.v.B * a.v.Hkv, (32LL << 20) / std::max(1LL, unit_bytes)));
   p.off_v = p.ns * p.kbytes;
-  p.off_norm = p.off_v + p.nv * vb;
-  p.off_red = p.off_norm + nbytes;
+  p.off_red = p.off_v + p.nv * vb;
   p.off_bar = p.off_red + rbytes;
   // + alignment of the base to 1024 bytes; at least half the SM's shared
   // memory, so that one CTA (holding its TMEM columns) runs per SM
@@ -707,8 +695,8 @@ PfPlan pf_plan(const PfArgs &a, bool out, int sms) {
 size_t prefill_tile_bytes(int bits) { return (size_t)2 * 2 * kPfBox * (bits != 16 ? 2 : 1); }
 
 bool prefill_plan_fits(const PfArgs &a) {
-  const PfPlan s = pf_plan(a, false, 1), o = pf_plan(a, true, 1);
-  return s.smem <= 232448 && o.smem <= 232448 && o.ns >= 2 && o.nv >= 2;
+  const PfPlan o = pf_plan(a, 1);
+  return o.smem <= 232448 && o.ns >= 2 && o.nv >= 2;
 }
 
 cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st) {
@@ -719,22 +707,18 @@ cudaError_t launch_gqa_prefill(const PfArgs &a, cudaStream_t st) {
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
   }
-  const PfPlan ps = pf_plan(a, false, sms), po = pf_plan(a, true, sms);
+  const PfPlan po = pf_plan(a, sms);
   cudaError_t e = cudaFuncSetAttribute(prefill_expand_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       ps.smem_x);
+                                       po.smem_x);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(prefill_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, ps.smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(prefill_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, po.smem);
+    e = cudaFuncSetAttribute(prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, po.smem);
   if (e != cudaSuccess) return e;
-  e = cudaMemsetAsync(a.counter, 0, 2 * sizeof(int), st);  // the job counters
+  e = cudaMemsetAsync(a.counter, 0, sizeof(int), st);  // the job counter
   if (e == cudaSuccess)
-    e = launch_pdl(prefill_expand_kernel, dim3(ps.n_t64, a.v.B * a.v.Hkv), dim3(kPfWorkers), ps.smem_x, st,
-                   a, ps);
+    e = launch_pdl(prefill_expand_kernel, dim3(po.n_t64, a.v.B * a.v.Hkv), dim3(kPfWorkers), po.smem_x, st,
+                   a, po);
   if (e == cudaSuccess)
-    e = launch_pdl(prefill_kernel<false>, dim3(ps.grid), dim3(kPfThreads), ps.smem, st, a, ps);
-  if (e == cudaSuccess)
-    e = launch_pdl(prefill_kernel<true>, dim3(po.grid), dim3(kPfThreads), po.smem, st, a, po);
+    e = launch_pdl(prefill_kernel, dim3(po.grid), dim3(kPfThreads), po.smem, st, a, po);
   return e;
 }
 
