@@ -485,16 +485,22 @@ __device__ __forceinline__ uint32_t pack_codes(const uint32_t (&c)[4]) {
   return c[0] | (c[1] << BITS) | (c[2] << (2 * BITS)) | (c[3] << (3 * BITS));
 }
 
-template <int BITS, int GS, bool SYM>
+// KPC: keys with per-channel groups -- the kernel writes the value section
+// and its metadata only (the key codes are written when a group of
+// positions completes, by gqa_append_kgroups) and leaves the lengths to the
+// residual kernel, which runs last.
+template <int BITS, int GS, bool SYM, bool KPC = false>
 __global__ void __launch_bounds__(256)
     gqa_append_bulk(const GqaView v, const void *kin, const void *vin, int in_f32, int n_new,
                     const int32_t *n_per_seq, int32_t *err) {
   pdl_wait();
   pdl_trigger();
+  static_assert(!KPC || (!SYM && BITS != 16), "per-channel keys: grouped codes");
   constexpr int D = 128, E = 4;
   constexpr int SEC = D * BITS / 8;                       // bytes per section
-  constexpr int REC = SYM ? 2 * SEC : BITS == 16 ? 2 * SEC : 2 * SEC + 2 * (((D / GS) * 8 + 15) & ~15);
-  constexpr int KM = 2 * SEC, VM = KM + (((D / GS) * 8 + 15) & ~15);
+  constexpr int MBY = ((D / GS) * 8 + 15) & ~15;          // one section's group metadata
+  constexpr int REC = SYM ? 2 * SEC : BITS == 16 ? 2 * SEC : 2 * SEC + (KPC ? 1 : 2) * MBY;
+  constexpr int KM = 2 * SEC, VM = KPC ? 2 * SEC : KM + MBY;
   constexpr int NC = SEC / 16;                            // chunks per code section
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int wpb = blockDim.x >> 5;
@@ -526,11 +532,12 @@ __global__ void __launch_bounds__(256)
         const uint32_t sv = quant_sym_lane<E>(xv, BITS, cv);
         if (ok && lane == 0) v.scales[row] = sk | (sv << 16);
       } else {
-        float ks, kz, vs, vz;
-        quant_lane<E>(xk, GS, (1 << BITS) - 1, ck, ks, kz);
+        float ks = 0.f, kz = 0.f, vs, vz;
+        if constexpr (!KPC) quant_lane<E>(xk, GS, (1 << BITS) - 1, ck, ks, kz);
+        else for (int e = 0; e < E; ++e) ck[e] = 0u;
         quant_lane<E>(xv, GS, (1 << BITS) - 1, cv, vs, vz);
         if (ok && (lane * E) % GS == 0) {
-          reinterpret_cast<float2 *>(rec + KM)[(lane * E) / GS] = make_float2(ks, kz);
+          if constexpr (!KPC) reinterpret_cast<float2 *>(rec + KM)[(lane * E) / GS] = make_float2(ks, kz);
           reinterpret_cast<float2 *>(rec + VM)[(lane * E) / GS] = make_float2(vs, vz);
         }
       }
@@ -549,7 +556,7 @@ __global__ void __launch_bounds__(256)
           off = SYM ? 16 * ((NC + k + sym_rot(t, REC / 16)) & (REC / 16 - 1)) + 4 * (u & 3)
                     : SEC + 16 * ((k + v_rot(t, REC, NC)) & (NC - 1)) + 4 * (u & 3);
         }
-        if (ok) *reinterpret_cast<uint32_t *>(rec + off) = w;
+        if (ok && (!KPC || lane >= 16)) *reinterpret_cast<uint32_t *>(rec + off) = w;
       } else {
         const uint32_t kw = g8.kword(pk), vw = g8.vword(pv);
         const int kc = lane >> 2;
@@ -558,7 +565,7 @@ __global__ void __launch_bounds__(256)
         const int voff = SYM ? 16 * ((NC + kc + sym_rot(t, REC / 16)) & (REC / 16 - 1)) + 4 * (lane & 3)
                              : SEC + 16 * ((kc + v_rot(t, REC, NC)) & (NC - 1)) + 4 * (lane & 3);
         if (ok) {
-          *reinterpret_cast<uint32_t *>(rec + koff) = kw;
+          if constexpr (!KPC) *reinterpret_cast<uint32_t *>(rec + koff) = kw;
           *reinterpret_cast<uint32_t *>(rec + voff) = vw;
         }
       }
@@ -602,7 +609,9 @@ __global__ void __launch_bounds__(256)
     process(xk[0], xv[0], ok[0], row[0], tt[0]);
     process(xk[1], xv[1], ok[1], row[1], tt[1]);
   }
-  // the last CTA advances the lengths
+  // the last CTA advances the lengths (per-channel keys: the residual
+  // kernel does, after this one)
+  if constexpr (KPC) return;
   __syncthreads();
   __shared__ int last;
   if (threadIdx.x == 0) {
@@ -661,79 +670,141 @@ __global__ void __launch_bounds__(256)
   if (threadIdx.x == 0) v.lens[b] = min((long long)len + nb, (long long)v.cap);
 }
 
-// Per-channel key groups completed by this append: one thread per
-// (sequence, kv head, group, channel pair {ch, ch+8} sharing 4-bit bytes).
+// Per-channel key groups completed by this append: one warp per (sequence,
+// KV head, group of GS positions).  The group's keys (residual rows for
+// positions already stored, the appended rows for new ones, rounded to
+// bf16 as the residual holds them) are staged in natural channel order in
+// shared memory; lane L quantises the channel pairs {c, c + 8} of pairs L
+// (and L + 32 when D = 128; c = 16 (p / 8) + p % 8: the two channels of one
+// 4-bit byte)
+// over the group's positions: scale = fl((max - min) / levels) correctly
+// rounded, codes rint((x - min) / scale) through the fast reciprocal with
+// the rounding check of rint_quot_fast (the correctly rounded division
+// where it cannot decide), the codes packed into the positions' key
+// sections in shared memory and stored as whole 16-byte chunks.
+constexpr int kKgWarps = 4;
+// dynamic shared memory of gqa_append_kgroups: per warp the staged keys
+// (GS rows of D + 8 bf16) and the key sections (GS rows of D bits / 8 bytes)
+__host__ __device__ constexpr int kg_warp_bytes(int D, int GS, int bits) {
+  return ((GS * (D + 8) * 2 + GS * D * bits / 8) + 15) & ~15;
+}
 template <int D>
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(32 * kKgWarps)
     gqa_append_kgroups(const GqaView v, const void *kin, int in_f32, int n_new,
                        const int32_t *n_per_seq, int32_t *err, int max_groups) {
   pdl_wait();
   pdl_trigger();
-  const int pairs = D / 2;
-  const size_t id = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const size_t total = (size_t)v.B * v.Hkv * max_groups * pairs;
-  if (id >= total) return;
-  const int pr = (int)(id % pairs);
-  const int gidx = (int)((id / pairs) % max_groups);
-  const int kvh = (int)((id / ((size_t)pairs * max_groups)) % v.Hkv);
-  const int b = (int)(id / ((size_t)pairs * max_groups * v.Hkv));
+  constexpr int PAD = D + 8;                      // bf16 per staged row (conflict-free columns)
+  extern __shared__ __align__(16) uint8_t kg_smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const size_t wid = (size_t)blockIdx.x * kKgWarps + warp;
+  const size_t total = (size_t)v.B * v.Hkv * max_groups;
+  if (wid >= total) return;
+  const int gidx = (int)(wid % max_groups);
+  const int kvh = (int)((wid / max_groups) % v.Hkv);
+  const int b = (int)(wid / ((size_t)max_groups * v.Hkv));
   const int GS = v.group;
   const int nb = seq_count(n_per_seq, b, n_new, nullptr);
   const int len0 = v.lens[b];
   const int G = len0 / GS + gidx;  // candidate group
-  if ((G + 1) * GS > len0 + nb || (G + 1) * GS > v.cap) return;  // not completed now
-  const int ch0 = (pr / 8) * 16 + (pr % 8);  // channels ch0 and ch0 + 8
+  if ((G + 1) * GS > len0 + nb || (G + 1) * GS > v.cap) return;  // not completed now (warp-uniform)
   const size_t slab = (size_t)b * v.Hkv + kvh;
   const RecLayout L = rec_layout(v.bits, D, GS, 1);
+  const int sec = D * v.bits / 8;
   const uint8_t *res = v.resid + slab * (size_t)GS * D * 2;
-  const int levels = (1 << v.bits) - 1;
-  uint32_t codes[2][64];
-  float scs[2], zrs[2];
-  for (int h = 0; h < 2; ++h) {
-    const int ch = ch0 + 8 * h;
-    int kb, khi;
-    k_pos(ch, 16, D, &kb, &khi);
-    float mn = INFINITY, mx = -INFINITY;
-    float xs[64];
-    for (int r = 0; r < GS; ++r) {
-      const int p = G * GS + r;
-      float x;
-      if (p < len0) {
-        x = bf16_to_f32(*reinterpret_cast<const uint16_t *>(res + (size_t)r * D * 2 + kb));
-      } else {
-        const size_t ii = (((size_t)b * n_new + (p - len0)) * v.Hkv + kvh) * D + ch;
-        x = bf16_to_f32(f32_to_bf16_bits(load_in(kin, ii, in_f32)));  // keys buffer as bf16
+  uint8_t *wbase = kg_smem + warp * kg_warp_bytes(D, GS, v.bits);
+  uint16_t *xs = reinterpret_cast<uint16_t *>(wbase);
+  uint8_t *ks = wbase + GS * PAD * 2;
+  // ---- the group's keys, natural channel order ----
+  constexpr int CPR = D / 8;  // 8-channel pieces per row
+  for (int q = lane; q < GS * CPR; q += 32) {
+    const int r = q / CPR, c8 = 8 * (q - r * CPR);
+    const int p = G * GS + r;
+    uint16_t h[8];
+    if (p < len0) {
+      // residual row r: bf16 in the key fragment order
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        int kb, khi;
+        k_pos(c8 + e, 16, D, &kb, &khi);
+        h[e] = *reinterpret_cast<const uint16_t *>(res + (size_t)r * D * 2 + kb);
       }
-      xs[r] = x;
-      mn = fminf(mn, x);
-      mx = fmaxf(mx, x);
-    }
-    const float scale = __fdiv_rn(__fsub_rn(mx, mn), (float)levels);
-    for (int r = 0; r < GS; ++r) {
-      if (scale == 0.f) {
-        codes[h][r] = 0;
-      } else {
-        float q = rintf(__fdiv_rn(__fsub_rn(xs[r], mn), scale));
-        codes[h][r] = (uint32_t)fminf(fmaxf(q, 0.f), (float)levels);
-      }
-    }
-    scs[h] = scale;
-    zrs[h] = mn;
-  }
-  for (int h = 0; h < 2; ++h)
-    v.gmeta[(slab * (v.cap / GS) + G) * D + ch0 + 8 * h] = make_float2(scs[h], zrs[h]);
-  for (int r = 0; r < GS; ++r) {
-    uint8_t *rec = v.rec + (slab * v.cap + (size_t)G * GS + r) * L.rec + L.k_off;
-    int b0, h0, b1, h1;
-    k_pos(ch0, v.bits, D, &b0, &h0);
-    k_pos(ch0 + 8, v.bits, D, &b1, &h1);
-    if (v.bits == 8) {
-      rec[b0] = (uint8_t)codes[0][r];
-      rec[b1] = (uint8_t)codes[1][r];
     } else {
-      // 4-bit: channels ch0 and ch0+8 share one byte (low and high nibble)
-      rec[b0] = (uint8_t)(codes[0][r] | (codes[1][r] << 4));
+      const size_t ii = (((size_t)b * n_new + (p - len0)) * v.Hkv + kvh) * D + c8;
+      if (in_f32) {
+        const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(kin) + ii);
+        const float4 u0 = src[0], u1 = src[1];
+        const float f[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) h[e] = f32_to_bf16_bits(f[e]);
+      } else {
+        const uint4 u = *reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(kin) + ii);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) { h[2 * e] = (uint16_t)(w[e] & 0xffffu); h[2 * e + 1] = (uint16_t)(w[e] >> 16); }
+      }
     }
+    uint4 o;
+    o.x = h[0] | ((uint32_t)h[1] << 16); o.y = h[2] | ((uint32_t)h[3] << 16);
+    o.z = h[4] | ((uint32_t)h[5] << 16); o.w = h[6] | ((uint32_t)h[7] << 16);
+    *reinterpret_cast<uint4 *>(xs + r * PAD + c8) = o;
+  }
+  for (int q = lane; q < GS * sec / 16; q += 32) reinterpret_cast<uint4 *>(ks)[q] = make_uint4(0, 0, 0, 0);
+  __syncwarp();
+  // ---- per channel: scale, zero, codes ----
+  const float lev = (float)((1 << v.bits) - 1);
+#pragma unroll
+  for (int pp = 0; pp < D / 64; ++pp) {  // D / 2 channel pairs, 32 per pass
+    const int pr = lane + 32 * pp;
+    const int ch0 = (pr >> 3) * 16 + (pr & 7);
+    float sc[2], zr[2], rs[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int ch = ch0 + 8 * h;
+      float mn = INFINITY, mx = -INFINITY;
+      for (int r = 0; r < GS; ++r) {
+        const float x = bf16_to_f32(xs[r * PAD + ch]);
+        mn = fminf(mn, x);
+        mx = fmaxf(mx, x);
+      }
+      sc[h] = __fdiv_rn(__fsub_rn(mx, mn), lev);
+      zr[h] = mn;
+      rs[h] = sc[h] == 0.f ? 0.f : __fdividef(1.f, sc[h]);
+      v.gmeta[(slab * (v.cap / GS) + G) * D + ch] = make_float2(sc[h], mn);
+    }
+    int kb0, kh0, kb1, kh1;
+    k_pos(ch0, v.bits, D, &kb0, &kh0);
+    k_pos(ch0 + 8, v.bits, D, &kb1, &kh1);
+    for (int r = 0; r < GS; ++r) {
+      uint32_t c[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (sc[h] == 0.f) {
+          c[h] = 0u;
+        } else {
+          const float d = __fsub_rn(bf16_to_f32(xs[r * PAD + ch0 + 8 * h]), zr[h]);
+          bool near;
+          float q = rint_quot_fast(d, rs[h], near);
+          if (near) q = rintf(__fdiv_rn(d, sc[h]));
+          c[h] = (uint32_t)fminf(fmaxf(q, 0.f), lev);
+        }
+      }
+      if (v.bits == 8) {
+        ks[r * sec + kb0] = (uint8_t)c[0];
+        ks[r * sec + kb1] = (uint8_t)c[1];
+      } else {
+        // channels ch0 and ch0 + 8 share one byte (low and high nibble)
+        ks[r * sec + kb0] = (uint8_t)(c[0] | (c[1] << 4));
+      }
+    }
+  }
+  __syncwarp();
+  // ---- the group's key sections, whole 16-byte chunks ----
+  const int cps = sec / 16;
+  for (int q = lane; q < GS * cps; q += 32) {
+    const int r = q / cps, u = q - r * cps;
+    uint8_t *rec = v.rec + (slab * v.cap + (size_t)G * GS + r) * L.rec + L.k_off;
+    reinterpret_cast<uint4 *>(rec)[u] = reinterpret_cast<const uint4 *>(ks + r * sec)[u];
   }
   (void)err;
 }
@@ -925,14 +996,33 @@ cudaError_t launch_gqa_append(const GqaView &v, const void *k, const void *vv, i
   if (kpc) {
     // groups first (they read residual rows the open group may overwrite)
     const int max_groups = (n_new + v.group - 1) / v.group + 1;
-    const size_t thr = (size_t)v.B * v.Hkv * max_groups * (v.D / 2);
-    const dim3 grid((unsigned)((thr + 127) / 128));
-    e = launch_pdl(d128 ? gqa_append_kgroups<128> : gqa_append_kgroups<64>, grid, dim3(128), 0, st,
-                   v, k, in_f32, n_new, n_per_seq, err, max_groups);
+    const size_t warps = (size_t)v.B * v.Hkv * max_groups;
+    const dim3 grid((unsigned)((warps + kKgWarps - 1) / kKgWarps));
+    auto kern = d128 ? gqa_append_kgroups<128> : gqa_append_kgroups<64>;
+    const int smem = kKgWarps * kg_warp_bytes(v.D, v.group, v.bits);
+    static bool attr_set = false;
+    if (!attr_set) {
+      // the largest need: head_dim 128, groups of 64, 8-bit codes
+      const int most = kKgWarps * kg_warp_bytes(128, 64, 8);
+      e = cudaFuncSetAttribute(gqa_append_kgroups<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(gqa_append_kgroups<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+      if (e != cudaSuccess) return e;
+      attr_set = true;
+    }
+    e = launch_pdl(kern, grid, dim3(32 * kKgWarps), (size_t)smem, st, v, k, in_f32, n_new, n_per_seq, err,
+                   max_groups);
   }
   if (e == cudaSuccess) {
     const dim3 bg(row_blocks(rows, 8));
-    if (!kpc && (size_t)n_new * v.Hkv > 64 && d128 && rows < (1u << 31) &&
+    if (kpc && (size_t)n_new * v.Hkv > 64 && d128 && rows < (1u << 31) && (v.bits == 8 || v.bits == 4)) {
+      // bulk appends of the values beside per-channel keys (head_dim 128)
+      auto bulk = [&](auto kern) {
+        return launch_pdl(kern, bg, dim3(256), 0, st, v, k, vv, in_f32, n_new, n_per_seq, err);
+      };
+      if (v.bits == 8) e = v.group == 32 ? bulk(gqa_append_bulk<8, 32, false, true>) : bulk(gqa_append_bulk<8, 64, false, true>);
+      else e = v.group == 32 ? bulk(gqa_append_bulk<4, 32, false, true>) : bulk(gqa_append_bulk<4, 64, false, true>);
+    } else if (!kpc && (size_t)n_new * v.Hkv > 64 && d128 && rows < (1u << 31) &&
         (v.bits == 16 || v.bits == 8 || v.bits == 4)) {
       // bulk appends of the per-token layouts with head_dim 128
       const bool sym = v.scheme == kSchemeSym;
