@@ -99,10 +99,12 @@ struct GqaCfg {
   // and the zero-point terms per warp ([4][KG_ROWS][8] floats)
   static constexpr int FOLD_BYTES = KPC ? KG_ROWS * KS * 32 * 16 : 0;
   static constexpr int ZRED_BYTES = KPC ? 4 * KG_ROWS * 8 * 4 : 0;
-  // stages: four where they and the rest fit four CTAs per SM (57 KB each),
-  // else three or two by stage size
+  // stages: bf16 planes three (head_dim 128: two CTAs per SM, ~190 KB of
+  // copies in flight per SM, the decode bound by HBM); quantised stages
+  // four where they and the rest fit four CTAs per SM (57 KB each), else
+  // three or two by stage size
   static constexpr int FIXED = Q_BYTES + FOLD_BYTES + ZRED_BYTES + 24 * 4;
-  static constexpr int NST = !TMA ? 2
+  static constexpr int NST = !TMA ? 3
                              : KPC ? (FIXED + 4 * STAGE <= 57344 ? 4 : (FIXED + 3 * STAGE <= 57344 ? 3 : (STAGE <= 20480 ? 3 : 2)))
                                    : (STAGE <= 13312 ? 4 : (STAGE <= 20480 ? 3 : 2));
   static_assert(TMA || RB == 1, "plane layout holds 64-row tiles");

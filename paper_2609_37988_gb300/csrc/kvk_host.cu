@@ -257,15 +257,16 @@ kvk_status check_layer_index(const kvk_cache *c, int layer) {
 // tiles (query set-up, merge of the warps' states, the partial); CTAs run in
 // waves of `slots`, and a partial last wave costs at least half a wave (its
 // CTAs have the SMs to themselves but run at most ~2x faster).  For the
-// bf16 kernel (`full_tail`), bound by HBM rather than by its issue rate, a
-// partial last wave costs a whole wave.  Among choices within
-// 1 % the fewer splits win.  Measured on the 7B and 14B step shapes and
-// every format, this model's pick is within 1 % of the best split count
-// (bf16 at the 14B step: 5 splits, 163.6 us, against 167.2 with the 3 of
-// the quantised kernels' rule; B = 16..48 and T = 4096..16384 likewise);
-// the kept-list gather has a rule of its own (auto_splits).
+// bf16 kernel (`full_tail`), bound by HBM rather than by its issue rate and
+// running two CTAs per SM with three stages each, a partial last wave costs
+// a whole wave and a CTA's fixed cost is about four tiles.  Among choices
+// within 1 % the fewer splits win.  Measured on the 7B and 14B step shapes
+// and every format, this model's pick is within 1 % of the best split count
+// for the quantised kernels; for bf16 at B = 8..64 and T = 2048..16384 it
+// is the best or within 1 % except at B = 40 (4 %) (the 14B step: one
+// split, 160.5 us); the kept-list gather has a rule of its own (auto_splits).
 int choose_splits(int units, int tiles, int per, int slots, int max_splits, bool full_tail) {
-  const double F = 2.0, tail = 0.5;
+  const double F = full_tail ? 4.0 : 2.0, tail = 0.5;
   if (tiles <= 1) return 1;
   per = std::max(1, per);
   const int ktiles = (tiles + per - 1) / per;
