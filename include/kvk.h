@@ -151,7 +151,10 @@ kvk_status kvk_workspace_size(const kvk_model_desc *desc, int32_t max_splits,
  * n_layers device pointers (NULL for inheritors), each of at least the size
  * kvk_cache_plan reported; workspace: device buffer of ws_bytes.  The cache
  * starts empty; call kvk_cache_reset (or zero the arenas) before first use.
- * The cache keeps the pointers; the caller keeps the memory alive. */
+ * The cache keeps the pointers; the caller keeps the memory alive.
+ * INVALID_CONFIG also when a grouped 8- or 4-bit anchor with per-token keys
+ * and evict_capacity > 0 holds max_batch x n_kv_heads x capacity >= 2^31
+ * records (its kept-list gather addresses records as 31-bit rows). */
 kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg,
                             void *const *arenas, void *workspace, size_t ws_bytes,
                             int32_t max_splits, kvk_cache **out);

@@ -505,7 +505,15 @@ kvk_status kvk_cache_create(const kvk_model_desc *desc, const kvk_layer_cfg *cfg
       if (cfg[l].evict_capacity <= 0 ||
           !gqa_decode_row_gather(cfg[l].bits, cfg[l].key_axis, layer_scheme(&cfg[l])))
         continue;
-      e = gqa_make_rows_tmap(c->tmap[l].bytes, c->gqa_view(l));
+      const GqaView gv = c->gqa_view(l);
+      if ((long long)gv.B * gv.Hkv * gv.cap >= (1LL << 31)) {
+        delete c;
+        return fail(KVK_ERR_INVALID_CONFIG,
+                    "layer %d: kept lists on grouped per-token anchors need max_batch x n_kv_heads x "
+                    "capacity below 2^31 records",
+                    l);
+      }
+      e = gqa_make_rows_tmap(c->tmap[l].bytes, gv);
     }
     if (e != cudaSuccess) {
       delete c;
