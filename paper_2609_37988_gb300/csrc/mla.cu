@@ -32,9 +32,12 @@ namespace kvk {
 namespace {
 
 // Latent split-K decode on the 5th-generation tensor cores.  Grid (split,
-// sequence); 6 warps: warps 0-3 run the softmax and the epilogue, warp 4
-// issues the UMMAs, warp 5 the TMA copies.  Tiles of TR positions of
-// [c[:W] | k^R] (TR = 48 for W = 512, so that three stages fit, else 64).
+// query row / R); 8 warps: warps 0-3 run the softmax and the epilogue,
+// warps 4, 6 and 7 issue the UMMAs, warp 5 the TMA copies.  Below, the
+// operands are described for R = 1 (decode); with R = 2 (pairs of pre-fill
+// rows) the query operand, S, P and O carry the two rows' 32 columns side by
+// side.  Tiles of TR positions of [c[:W] | k^R] (TR = 48 for W = 512, so
+// that three stages fit (two with R = 2), else 64).
 //
 // Shared memory per stage: the tile as (W + 64)/64 boxes of TR positions x
 // 64 coordinates, each box TR rows of 128 bytes in the 128-byte swizzled
@@ -61,32 +64,39 @@ namespace {
 // positions per decode tile (and rows of a TMA box) for kept width w
 __host__ __device__ constexpr int mla_tile_rows(int w) { return w == 512 ? 48 : 64; }
 
-template <int W>
+// R: query rows per CTA (pre-fill rows of one sequence share every tile;
+// decode: R = 1).  The query operand, S, P and O have NQ = 32 R columns:
+// row rho of the CTA, head h at 32 rho + h (hi part, with q_pe) and
+// 32 rho + 16 + h (lo part).
+template <int W, int R = 1>
 struct MlaCfg {
+  static constexpr int NQ = 32 * R;                   // Q rows; S, P, O columns
+  static constexpr int NH = 16 * R;                   // (row, head) pairs of a CTA
   static constexpr int TR = mla_tile_rows(W);         // positions per tile
   static constexpr int KH = W + kRope;                // hi extent: latent + rope
   static constexpr int BOXES = KH / 64;               // 64-coordinate boxes per tile
   static constexpr int BOX = TR * 128;                // bytes per box
   static constexpr int STAGE = BOXES * BOX;
-  static constexpr int NST = 3;
-  static constexpr int QB = 32 * KH * 2;              // [Q_hi ; Q_lo] operand (32 rows)
-  static constexpr int PB = 4 * 1024;                 // [P_hi | P_lo] operand, 4 column blocks
+  static constexpr int NST = (R > 1 && W == 512) ? 2 : 3;  // two where the wider query operand needs the room
+  static constexpr int QB = NQ * KH * 2;              // [Q_hi ; Q_lo] operand (NQ rows)
+  static constexpr int PB = 4 * 1024 * R;             // [P_hi | P_lo] operand, 4 R column blocks
   static constexpr int OFF_Q = NST * STAGE;
   static constexpr int OFF_P = OFF_Q + QB;            // two buffers
-  static constexpr int OFF_RED = OFF_P + 2 * PB;      // float [4][16] maxima, [4][16] sums
-  static constexpr int OFF_BAR = OFF_RED + 512;       // full[NST], sbar[2], pbar[2], obar[NST], dbar[3]
+  static constexpr int OFF_RED = OFF_P + 2 * PB;      // float [4][NH] maxima, [4][NH] sums
+  static constexpr int OFF_BAR = OFF_RED + 512 * R;   // full[NST], sbar[2], pbar[2], obar[NST], dbar[3]
   static constexpr int NBAR = 2 * NST + 7;
   static constexpr int OFF_TB = OFF_BAR + 8 * NBAR;   // TMEM base address, abort flag
   static constexpr int SMEM = OFF_TB + 16 + 1024;     // + slack to align the base to 1024
   static constexpr int MV = W >= 128 ? 128 : 64;      // value UMMA M
   static constexpr int MB = W / MV;                   // value M-blocks
-  static constexpr int OCOLS = 32 * MB;               // TMEM columns of O
-  static constexpr int SCOLS = 64;                    // two 32-column S buffers
-  static constexpr int TCOLS = OCOLS + SCOLS <= 128 ? 128 : 256;
+  static constexpr int OCOLS = NQ * MB;               // TMEM columns of O
+  static constexpr int SCOLS = 2 * NQ;                // two NQ-column S buffers
+  static constexpr int TCOLS = OCOLS + SCOLS <= 128 ? 128 : OCOLS + SCOLS <= 256 ? 256 : 512;
   static_assert(KH % 64 == 0 && W % 64 == 0, "whole boxes");
   static_assert(TR % 16 == 0 && TR <= 64, "tile rows");
   static_assert(OCOLS + SCOLS <= TCOLS, "TMEM columns");
   static_assert(SMEM <= 232448, "shared memory");
+  static_assert(R == 1 || R == 2, "one or two query rows per CTA");
 };
 
 // 2-D TMA tile load (x = coordinate, y = row) completing on `bar`
@@ -104,13 +114,14 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *tmap, 
 // per ~45 cycles: the products come as three streams)
 constexpr int kMlaThreads = 256;
 
-template <int W>
+template <int W, int R>
 __global__ void __launch_bounds__(kMlaThreads, 1)
     mla_decode_kernel(const __grid_constant__ CUtensorMap tmap, const MlaView v,
                       const uint16_t *__restrict__ qlat, const uint16_t *__restrict__ q_pe, int H,
                       float sig, int items_per_split, int n_splits, float *__restrict__ partial,
                       int32_t *err) {
-  using C = MlaCfg<W>;
+  using C = MlaCfg<W, R>;
+  constexpr int NQ = C::NQ, NH = C::NH;
   constexpr int TR = C::TR;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -121,14 +132,16 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
   uint64_t *sbar = full + C::NST, *pbar = sbar + 2, *obar = pbar + 2, *dbar = obar + C::NST;
   uint32_t *tbase = reinterpret_cast<uint32_t *>(sm + C::OFF_TB);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + C::OFF_TB + 4);
-  float *red = reinterpret_cast<float *>(sm + C::OFF_RED);  // [4 warps][16]
-  float *lsum = red + 4 * kHeads;                           // [4 warps][16]
+  float *red = reinterpret_cast<float *>(sm + C::OFF_RED);  // [4 warps][NH]
+  float *lsum = red + 4 * NH;                               // [4 warps][NH]
   uint8_t *q_s = sm + C::OFF_Q;
 
-  const int split = blockIdx.x, vb = blockIdx.y;  // vb: the query row (decode: sequence)
-  const int b = mla_row_seq(v, vb);              // the sequence whose cache it reads
+  // query rows vb0 .. vb0 + R - 1 (decode: the sequence; pre-fill: R
+  // consecutive chunk rows of one sequence, the last seeing the most)
+  const int split = blockIdx.x, vb0 = blockIdx.y * R;
+  const int b = mla_row_seq(v, vb0);             // the sequence whose cache it reads
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int len = mla_row_len(v, vb, b);
+  const int len = mla_row_len(v, vb0 + R - 1, b);
   const int i0 = split * items_per_split;
   const int i1 = (split == n_splits - 1) ? len : min(i0 + items_per_split, len);
   const int n_tiles = i1 > i0 ? (i1 - i0 + TR - 1) / TR : 0;
@@ -159,20 +172,20 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
   // other warps wait for the absorb itself before reading its q_lat.
   // Query operand, K-major core layout: row n, coordinate k at
   // (n/8) SBO + (k/8) 128 + (n%8) 16 + (k%8) 2 with SBO = (W+64)/8 128.
-  // Rows 0-15: [q_lat hi | q_pe] of head n; rows 16-31: [q_lat lo | 0] of
-  // head n-16.
+  // Rows 32 rho + h: [q_lat hi | q_pe] of head h of query row vb0 + rho;
+  // rows 32 rho + 16 + h: [q_lat lo | 0].
   if (warp < 5 || warp == 7) {
     pdl_wait();
     constexpr int QROW = 2 * W + kRope;  // qlat row: [hi(W) | (unused 64) | lo(W)]
-    const uint16_t *qb = qlat + (size_t)vb * H * QROW;
     // warps 0-4 stage it; the second score warp only waits for it
-    for (int q = tid; warp < 5 && q < 32 * (C::KH / 8); q += 160) {  // 16-byte cp.async, zero-filled
+    for (int q = tid; warp < 5 && q < NQ * (C::KH / 8); q += 160) {  // 16-byte cp.async, zero-filled
       const int n = q / (C::KH / 8), c = q % (C::KH / 8);
-      const int h = n & 15;
+      const int vb = vb0 + n / 32, nn = n & 31, h = nn & 15;
+      const uint16_t *qb = qlat + (size_t)vb * H * QROW;
       const uint16_t *src = qb;
-      const bool valid = h < H && (n < 16 || c < W / 8);
+      const bool valid = h < H && (nn < 16 || c < W / 8);
       if (valid)
-        src = n >= 16     ? qb + (size_t)h * QROW + C::KH + 8 * c
+        src = nn >= 16    ? qb + (size_t)h * QROW + C::KH + 8 * c
               : c < W / 8 ? qb + (size_t)h * QROW + 8 * c
                           : q_pe + ((size_t)vb * H + h) * kRope + 8 * (c - W / 8);
       cp_async16(q_s + (n / 8) * (C::KH / 8 * 128) + c * 128 + (n % 8) * 16, src, valid);
@@ -224,7 +237,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     // (t - NST <= t - 2): its wait for full[t % NST] is then for the phase
     // right after the last completed one.
     const int role = warp == 4 ? 0 : 1;
-    constexpr uint32_t ID_S = umma_idesc(64, 32, false, false);
+    constexpr uint32_t ID_S = umma_idesc(64, NQ, false, false);
     for (int t = role; t < n_tiles && !failed; t += 2) {
       const int s = t % C::NST;
       bool ok = true;
@@ -247,7 +260,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         const uint64_t dq = umma_desc(smem_u32(q_s), 128, C::KH / 8 * 128, 0);
 #pragma unroll
         for (int ks = 0; ks < C::KH / 16; ++ks)
-          umma_f16(t_s + 32 * (t & 1), dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
+          umma_f16(t_s + NQ * (t & 1), dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
                    dq + (uint64_t)(ks * 16), ID_S, ks > 0);
         umma_commit(&sbar[t & 1]);
       }
@@ -268,7 +281,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     // ======================= value warp ===================================
     // values(t) once P(t) is written; it waits for every pbar phase in
     // order, and pbar(t + 2) needs obar(t), committed after values(t)
-    constexpr uint32_t ID_V = umma_idesc(C::MV, 32, true, true);
+    constexpr uint32_t ID_V = umma_idesc(C::MV, NQ, true, true);
     for (int t = 0; t < n_tiles && !failed; ++t) {
       const bool ok = mbar_wait_or_abort(&pbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
       if (ok && lane == 0) {  // O^T[:, hi | lo] += C^T [P_hi | P_lo]
@@ -279,7 +292,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         for (int ks = 0; ks < TR / 16; ++ks)
 #pragma unroll
           for (int mb = 0; mb < C::MB; ++mb)
-            umma_f16(t_o + 32 * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
+            umma_f16(t_o + NQ * mb, da + (uint64_t)(((2 * mb) * C::BOX + ks * 2048) >> 4),
                      dp + (uint64_t)(ks * 16), ID_V, t > 0 || ks > 0);
         umma_commit(&obar[t % C::NST]);
       }
@@ -299,52 +312,56 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     // ======================= softmax warps ================================
     const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
     const int prow = 16 * warp + lane;  // this lane's tile position (lanes 0-15)
-    float m_run[kHeads], l_part[kHeads];
+    // each row's own end: row rho sees the positions below its causal limit
+    int i1r[R];
 #pragma unroll
-    for (int h = 0; h < kHeads; ++h) { m_run[h] = -1e30f; l_part[h] = 0.f; }
+    for (int r = 0; r < R; ++r) i1r[r] = R == 1 ? i1 : min(i1, mla_row_len(v, vb0 + r, b));
+    float m_run[NH], l_part[NH];  // (row, head) pair j = 16 rho + h
+#pragma unroll
+    for (int j = 0; j < NH; ++j) { m_run[j] = -1e30f; l_part[j] = 0.f; }
     for (int t = 0; t < n_tiles; ++t) {
-      const int base = i0 + t * TR, nval = min(TR, i1 - base);
+      const int base = i0 + t * TR;
       bool ok = mbar_wait_or_abort(&sbar[t & 1], (t >> 1) & 1, kLimit, abort_flag);
       // P buffer (t & 1) was read by values(t-2)
       if (ok && t >= 2)
         ok = mbar_wait_or_abort(&obar[(t - 2) % C::NST], ((t - 2) / C::NST) & 1, kLimit, abort_flag);
       if (softmax_sync_or(!ok)) { failed = true; break; }
       tc_fence_after();
-      float x[kHeads];
-      {
-        float lo[16];
-        tmem_ld16(t_s + 32 * (t & 1) + lane_off, x);
-        tmem_ld16(t_s + 32 * (t & 1) + 16 + lane_off, lo);
-        const bool live = lane < 16 && prow < nval;
+      float x[NH];
 #pragma unroll
-        for (int h = 0; h < kHeads; ++h) x[h] = live ? x[h] + lo[h] : -INFINITY;
+      for (int r = 0; r < R; ++r) {
+        float hi[16], lo[16];
+        tmem_ld16(t_s + NQ * (t & 1) + 32 * r + lane_off, hi);
+        tmem_ld16(t_s + NQ * (t & 1) + 32 * r + 16 + lane_off, lo);
+        const bool live = lane < 16 && prow < min(TR, i1r[r] - base);
+#pragma unroll
+        for (int h = 0; h < 16; ++h) x[16 * r + h] = live ? hi[h] + lo[h] : -INFINITY;
       }
       bool need = false;
 #pragma unroll
-      for (int h = 0; h < kHeads; ++h) need |= x[h] * sig > m_run[h] + 8.f;
+      for (int j = 0; j < NH; ++j) need |= x[j] * sig > m_run[j] + 8.f;
       if (softmax_sync_or(need)) {
         // new maxima: reduce over the 16 rows of each warp, then the 4 warps
 #pragma unroll
-        for (int h = 0; h < kHeads; ++h) {
-          float mx = x[h];
+        for (int j = 0; j < NH; ++j) {
+          float mx = x[j];
 #pragma unroll
           for (int off = 1; off < 16; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-          if (lane == 0) red[warp * kHeads + h] = mx;
+          if (lane == 0) red[warp * NH + j] = mx;
         }
         softmax_sync();
-        float alpha[kHeads];
+        float alpha[NH];
         bool any = false;
 #pragma unroll
-        for (int h = 0; h < kHeads; ++h) {
-          const float mt =
-              fmaxf(fmaxf(red[h], red[kHeads + h]), fmaxf(red[2 * kHeads + h], red[3 * kHeads + h])) * sig;
-          alpha[h] = 1.f;
-          if (mt > m_run[h] + 8.f) {  // stale maximum kept while within 2^8
-            alpha[h] = fast_exp2(m_run[h] - mt);
-            m_run[h] = mt;
+        for (int j = 0; j < NH; ++j) {
+          const float mt = fmaxf(fmaxf(red[j], red[NH + j]), fmaxf(red[2 * NH + j], red[3 * NH + j])) * sig;
+          alpha[j] = 1.f;
+          if (mt > m_run[j] + 8.f) {  // stale maximum kept while within 2^8
+            alpha[j] = fast_exp2(m_run[j] - mt);
+            m_run[j] = mt;
             any = true;
           }
-          l_part[h] *= alpha[h];
+          l_part[j] *= alpha[j];
         }
         if (t >= 1 && any) {
           // O holds values up to t-1: wait for them, scale per head in TMEM
@@ -354,33 +371,38 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
 #pragma unroll
           for (int mb = 0; mb < C::MB; ++mb)
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
+            for (int c = 0; c < 2 * R; ++c) {  // column block c: row c/2, hi or lo
               float o[16];
-              tmem_ld16(t_o + 32 * mb + 16 * half + lane_off, o);
+              tmem_ld16(t_o + NQ * mb + 16 * c + lane_off, o);
 #pragma unroll
-              for (int h = 0; h < 16; ++h) o[h] *= alpha[h];
-              tmem_st16(t_o + 32 * mb + 16 * half + lane_off, o);
+              for (int h = 0; h < 16; ++h) o[h] *= alpha[16 * (c / 2) + h];
+              tmem_st16(t_o + NQ * mb + 16 * c + lane_off, o);
             }
         }
         softmax_sync();  // `red` is reused by the next vote
       }
       // weights hi/lo in bf16 into the MN-major P operand: position k, column
-      // n (0-15 hi, 16-31 lo) at (k/8) 128 + (n/8) 1024 + (k%8) 16 + (n%8) 2
+      // n (32 rho + h hi, 32 rho + 16 + h lo) at (k/8) 128 + (n/8) 1024 +
+      // (k%8) 16 + (n%8) 2
       if (lane < 16 && prow < TR) {
-        uint32_t hw[8], lw[8];
 #pragma unroll
-        for (int h = 0; h < kHeads; h += 2) {
-          const float p0 = fast_exp2(fmaf(x[h], sig, -m_run[h]));
-          const float p1 = fast_exp2(fmaf(x[h + 1], sig, -m_run[h + 1]));
-          l_part[h] += p0;
-          l_part[h + 1] += p1;
-          split2<true>(p0, p1, hw[h / 2], lw[h / 2]);
+        for (int r = 0; r < R; ++r) {
+          uint32_t hw[8], lw[8];
+#pragma unroll
+          for (int h = 0; h < 16; h += 2) {
+            const int j = 16 * r + h;
+            const float p0 = fast_exp2(fmaf(x[j], sig, -m_run[j]));
+            const float p1 = fast_exp2(fmaf(x[j + 1], sig, -m_run[j + 1]));
+            l_part[j] += p0;
+            l_part[j + 1] += p1;
+            split2<true>(p0, p1, hw[h / 2], lw[h / 2]);
+          }
+          uint8_t *pp = pbuf(t & 1) + 4096 * r + (prow / 8) * 128 + (prow % 8) * 16;
+          *reinterpret_cast<uint4 *>(pp) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+          *reinterpret_cast<uint4 *>(pp + 1024) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+          *reinterpret_cast<uint4 *>(pp + 2048) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+          *reinterpret_cast<uint4 *>(pp + 3072) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
         }
-        uint8_t *pp = pbuf(t & 1) + (prow / 8) * 128 + (prow % 8) * 16;
-        *reinterpret_cast<uint4 *>(pp) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-        *reinterpret_cast<uint4 *>(pp + 1024) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
-        *reinterpret_cast<uint4 *>(pp + 2048) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-        *reinterpret_cast<uint4 *>(pp + 3072) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
       }
       fence_proxy_async();
       tc_fence_before();
@@ -388,7 +410,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
       if (lane == 0) mbar_arrive(&pbar[t & 1]);  // one of the four arrivals
     }
     pdl_trigger();
-    // ---- partial of this split: O^T columns h + 16+h, m, l ------------------
+    // ---- partial of this split: O^T columns 32 rho + h + 32 rho + 16 + h, m, l
     if (!failed && n_tiles > 0) {
       const int t = n_tiles - 1;
       const bool ok = mbar_wait_or_abort(&obar[t % C::NST], (t / C::NST) & 1, kLimit, abort_flag);
@@ -401,42 +423,45 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     if (!failed) {
       tc_fence_after();
       const size_t RS = (size_t)W + 2;
-      const size_t prow_base = ((size_t)split * mla_rows(v) + vb) * H;
+      const size_t prow_base = ((size_t)split * mla_rows(v) + vb0) * H;  // + rho H: row rho
 #pragma unroll
-      for (int h = 0; h < kHeads; ++h) {
-        float sum = l_part[h];
+      for (int j = 0; j < NH; ++j) {
+        float sum = l_part[j];
 #pragma unroll
         for (int off = 1; off < 16; off <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-        if (lane == 0) lsum[warp * kHeads + h] = sum;
+        if (lane == 0) lsum[warp * NH + j] = sum;
       }
 #pragma unroll
-      for (int mb = 0; mb < C::MB; ++mb) {
-        float o[16];
-        if (n_tiles > 0) {
-          float lo[16];
-          tmem_ld16(t_o + 32 * mb + lane_off, o);
-          tmem_ld16(t_o + 32 * mb + 16 + lane_off, lo);
+      for (int mb = 0; mb < C::MB; ++mb)
 #pragma unroll
-          for (int h = 0; h < 16; ++h) o[h] += lo[h];
-        } else {
+        for (int rho = 0; rho < R; ++rho) {
+          float o[16];
+          if (n_tiles > 0) {
+            float lo[16];
+            tmem_ld16(t_o + NQ * mb + 32 * rho + lane_off, o);
+            tmem_ld16(t_o + NQ * mb + 32 * rho + 16 + lane_off, lo);
 #pragma unroll
-          for (int h = 0; h < 16; ++h) o[h] = 0.f;
+            for (int h = 0; h < 16; ++h) o[h] += lo[h];
+          } else {
+#pragma unroll
+            for (int h = 0; h < 16; ++h) o[h] = 0.f;
+          }
+          // latent row of this lane: M=128 blocks use every lane; the M=64
+          // block (W = 64) holds row 16 warp + lane in lanes 0-15
+          const int r = C::MV == 128 ? 128 * mb + 32 * warp + lane : 16 * warp + lane;
+          if (C::MV == 128 || lane < 16) {
+#pragma unroll
+            for (int h = 0; h < 16; ++h)
+              if (h < H) partial[(prow_base + (size_t)rho * H + h) * RS + r] = o[h];
+          }
         }
-        // latent row of this lane: M=128 blocks use every lane; the M=64
-        // block (W = 64) holds row 16 warp + lane in lanes 0-15
-        const int r = C::MV == 128 ? 128 * mb + 32 * warp + lane : 16 * warp + lane;
-        if (C::MV == 128 || lane < 16) {
-#pragma unroll
-          for (int h = 0; h < kHeads; ++h)
-            if (h < H) partial[(prow_base + h) * RS + r] = o[h];
-        }
-      }
       softmax_sync();
-      if (tid < H) {
-        const float L = lsum[tid] + lsum[kHeads + tid] + lsum[2 * kHeads + tid] + lsum[3 * kHeads + tid];
+      if (tid < H * R) {
+        const int rho = R == 1 ? 0 : tid / H, j = 16 * rho + tid - rho * H;
+        const float L = lsum[j] + lsum[NH + j] + lsum[2 * NH + j] + lsum[3 * NH + j];
         float mh = m_run[0];
 #pragma unroll
-        for (int h = 1; h < kHeads; ++h) mh = (tid == h) ? m_run[h] : mh;
+        for (int jj = 1; jj < NH; ++jj) mh = (j == jj) ? m_run[jj] : mh;
         float *pr = partial + (prow_base + tid) * RS;
         pr[W] = (L > 0.f) ? mh : -INFINITY;
         pr[W + 1] = L;
@@ -455,26 +480,30 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
 // largest shared-memory carveout (with no preference the occupancy query
 // sizes the carveout for one CTA per SM, although two CTAs of the narrower
 // widths fit).
-template <int W>
+template <int W, int R = 1>
 cudaError_t mla_decode_attrs() {
-  auto k = mla_decode_kernel<W>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, MlaCfg<W>::SMEM);
+  auto k = mla_decode_kernel<W, R>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, MlaCfg<W, R>::SMEM);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);
   return e;
 }
 
-template <int W>
+// R = 2 (two query rows per CTA) for pre-fill calls whose sequences hold an
+// even number of query rows, so that the pairs never straddle two sequences:
+// every tile then serves both rows (the score product's N = 64, one issue).
+template <int W, int R>
 cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
-  using C = MlaCfg<W>;
+  using C = MlaCfg<W, R>;
   if (a.n_splits > 64) return cudaErrorInvalidValue;  // merge weights hold 64 splits
   const int B = mla_rows(a.v);  // query rows
-  auto k = mla_decode_kernel<W>;
+  if (R > 1 && (a.v.n_q % R != 0)) return cudaErrorInvalidValue;
+  auto k = mla_decode_kernel<W, R>;
   constexpr int MU_SMEM = (64 * (W + 8)) * 2 + (2 * 64 * 16 + 16) * 4;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = mla_decode_attrs<W>();
+    cudaError_t e = mla_decode_attrs<W, R>();
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(mla_merge_upv_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                MU_SMEM);
@@ -486,7 +515,7 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
                              static_cast<const uint16_t *>(a.q_pe),
                              static_cast<const uint16_t *>(a.w_uk), B, a.H, a.r, a.qlat);
   if (e == cudaSuccess)
-    e = launch_pdl(k, dim3(a.n_splits, B), dim3(kMlaThreads), C::SMEM, st,
+    e = launch_pdl(k, dim3(a.n_splits, B / R), dim3(kMlaThreads), C::SMEM, st,
                    *static_cast<const CUtensorMap *>(a.tmap), a.v,
                    static_cast<const uint16_t *>(a.qlat), static_cast<const uint16_t *>(a.q_pe),
                    a.H, a.sig_log2, a.items_per_split, a.n_splits, a.partial, a.err);
@@ -504,7 +533,7 @@ cudaError_t launch_mla_t(const MlaDecodeArgs &a, cudaStream_t st) {
 template <int W>
 int mla_ctas_t() {
   using C = MlaCfg<W>;
-  auto k = mla_decode_kernel<W>;
+  auto k = mla_decode_kernel<W, 1>;
   if (mla_decode_attrs<W>() != cudaSuccess) return 1;
   cudaFuncAttributes fa;
   int dev = 0, smem_sm = 0, regs_sm = 0, resv = 0;
@@ -543,11 +572,15 @@ cudaError_t mla_make_tmap(void *out, const MlaView &v) {
 cudaError_t launch_mla_decode(const MlaDecodeArgs &a, cudaStream_t st) {
   if (a.v.bits != 16) return launch_mla_decode_q(a, st);
   if (!a.tmap) return cudaErrorInvalidValue;
+  // pre-fill rows in pairs where the score products bound a tile (d >= 256:
+  // 2.75 -> 2.19 ms at d = 512, 1.54 -> 1.01 ms at d = 256 for 4 x 1024
+  // rows); at d <= 128 the softmax bounds it and pairs gain nothing
+  const bool pairs = a.v.n_q > 0 && a.v.n_q % 2 == 0;
   switch (a.v.width) {
-    case 512: return launch_mla_t<512>(a, st);
-    case 256: return launch_mla_t<256>(a, st);
-    case 128: return launch_mla_t<128>(a, st);
-    case 64: return launch_mla_t<64>(a, st);
+    case 512: return pairs ? launch_mla_t<512, 2>(a, st) : launch_mla_t<512, 1>(a, st);
+    case 256: return pairs ? launch_mla_t<256, 2>(a, st) : launch_mla_t<256, 1>(a, st);
+    case 128: return launch_mla_t<128, 1>(a, st);
+    case 64: return launch_mla_t<64, 1>(a, st);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -2,7 +2,9 @@
 bf16 and quantised, through the C ABI: every query row of the chunk attends
 to its own causal prefix with the absorbed query (the decode path per row),
 against the oracle's unabsorbed chunk attention on the dequantised cache.
-Ragged lengths, one sequence shorter than the chunk, an inheriting layer."""
+Ragged lengths, one sequence shorter than the chunk, an inheriting layer;
+bf16 chunks of an even number of rows decode two rows per CTA at d >= 256
+(a pair may hold an empty row beside a one-position row), odd ones one."""
 import math
 
 import numpy as np
@@ -18,7 +20,7 @@ pytestmark = pytest.mark.gpu
 H = 16
 
 
-def _setup(width, fmt, lens, T, seed):
+def _setup(width, fmt, lens, T, seed, H=H):
     from paper_2609_37988_gb300.cache import Cache, Layer
     B = len(lens)
     layer = dict(bits=16, width=width) if fmt is None else dict(bits=fmt[1], scheme=fmt[0], width=width)
@@ -75,3 +77,25 @@ def test_mla_prefill_rejections():
         c.prefill_mla(0, torch.zeros((2, 65, H, 128), dtype=torch.bfloat16, device="cuda"),
                       torch.zeros((2, 65, H, 64), dtype=torch.bfloat16, device="cuda"), wk.cuda(),
                       wv.cuda(), 0.1)  # n_q > max_ctx
+
+
+@pytest.mark.parametrize("width,n_q,heads", [(512, 40, 10), (512, 39, 16), (256, 40, 5), (256, 2, 16),
+                                              (128, 40, 16)],
+                         ids=["d512-pairs-h10", "d512-odd-rows", "d256-pairs-h5", "d256-one-pair", "d128-rows"])
+def test_mla_prefill_row_pairs(width, n_q, heads):
+    """Two rows per CTA: each row masks its own causal end inside the shared
+    tiles; fewer than 16 heads; an odd row count keeps one row per CTA."""
+    lens = [301, 130, 21]
+    c, wk, wv, c_hat, kr_hat = _setup(width, None, lens, 320, seed=width + n_q, H=heads)
+    g = torch.Generator().manual_seed(6)
+    qn = torch.randn((len(lens), n_q, heads, 128), generator=g).to(torch.bfloat16)
+    qp = torch.randn((len(lens), n_q, heads, 64), generator=g).to(torch.bfloat16)
+    sigma = 1.0 / math.sqrt(192)
+    out = c.prefill_mla(0, qn.cuda(), qp.cuda(), wk.cuda(), wv.cuda(), sigma)
+    ref = oatt.mla_prefill_unabsorbed(f32(qn), f32(qp), c_hat, kr_hat, f32(wk), f32(wv), width, lens, sigma)
+    assert_close(f32(out), ref, what=f"mla prefill pairs d={width} n_q={n_q} H={heads}")
+    empty = max(0, n_q - lens[2])
+    assert (f32(out[2, :empty]) == 0).all()
+    if empty < n_q:
+        assert (np.abs(f32(out[2, empty])) > 0).any()  # the one-position row
+    assert c.device_error() == 0
