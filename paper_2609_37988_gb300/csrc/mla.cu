@@ -37,21 +37,22 @@ namespace {
 // operands are described for R = 1 (decode); with R = 2 (pairs of pre-fill
 // rows) the query operand, S, P and O carry the two rows' 32 columns side by
 // side.  Tiles of TR positions of [c[:W] | k^R] (TR = 48 for W = 512, so
-// that three stages fit (two with R = 2), else 64).
+// that three stages fit (two with R = 2), 128 for W = 64, else 64).
 //
 // Shared memory per stage: the tile as (W + 64)/64 boxes of TR positions x
 // 64 coordinates, each box TR rows of 128 bytes in the 128-byte swizzled
-// layout, written by TMA tensor copies (one per box, completing on the
+// layout, written by TMA tensor copies (TR/BR per box, completing on the
 // stage's mbarrier).  The same bytes serve both products:
 //   scores  S[pos x 32] = C[pos x (W+64)] [Q_hi ; Q_lo]^T
-//           (UMMA M=64 (rows past TR are ignored), N=32: columns 0-15 are
-//           the heads' q_lat hi (+ q_pe) parts, 16-31 their q_lat lo parts;
-//           A = the tile K-major);
+//           (UMMA M=64 (rows past TR are ignored; M=128 for TR = 128),
+//           N=32: columns 0-15 are the heads' q_lat hi (+ q_pe) parts,
+//           16-31 their q_lat lo parts; A = the tile K-major);
 //   values  O^T[W x 32] += C^T[W x TR pos] [P_hi | P_lo]
 //           (UMMA M=128 latent rows (64 for W = 64), N = 16 heads hi + 16
 //           heads lo, A = the tile read MN-major); O = columns h + 16+h.
 // Score rows come back with tcgen05.ld (M=64 accumulator: row r in TMEM
-// lane 32 (r/16) + r%16), so lane r%16 of softmax warp r/16 owns position r:
+// lane 32 (r/16) + r%16, so lane r%16 of softmax warp r/16 owns position r;
+// M=128: lane r%32 of warp r/32):
 // its 16 scores stay in registers; the online softmax is base 2 with a stale
 // maximum kept within 2^8 (one vote per tile; maxima are reduced only when
 // one rises).  The weights go hi/lo in bf16 into the P operand; O stays in
@@ -61,8 +62,17 @@ namespace {
 // copy warp refills a stage as soon as the values that read it completed.
 // Every wait is bounded (an abort flag stops the other role); the CTA frees
 // its TMEM on every path.
-// positions per decode tile (and rows of a TMA box) for kept width w
-__host__ __device__ constexpr int mla_tile_rows(int w) { return w == 512 ? 48 : 64; }
+// rows of one TMA box (the anchor's tensor map) for kept width w
+__host__ __device__ constexpr int mla_box_rows(int w) { return w == 512 ? 48 : 64; }
+// positions per tile: 48 at d = 512 (three stages fit), 128 at d = 64 (M =
+// 128 score products, every softmax lane owning a position, two CTAs per SM
+// with two stages each), 64 otherwise.  Measured (B = 64, T = 4096 decode
+// call; 4 x 1024-row pre-fill): 128-position tiles took d = 64 from 29.2 to
+// 28.4 us per call and 0.63 to 0.54 ms per pre-fill; at d = 128 and 256 the
+// calls were unchanged and the d = 128 pre-fill went 0.74 -> 0.80 ms.
+__host__ __device__ constexpr int mla_tile_rows(int w, int r) {
+  return w == 512 ? 48 : (r == 1 && w == 64) ? 128 : 64;
+}
 
 // R: query rows per CTA (pre-fill rows of one sequence share every tile;
 // decode: R = 1).  The query operand, S, P and O have NQ = 32 R columns:
@@ -72,14 +82,19 @@ template <int W, int R = 1>
 struct MlaCfg {
   static constexpr int NQ = 32 * R;                   // Q rows; S, P, O columns
   static constexpr int NH = 16 * R;                   // (row, head) pairs of a CTA
-  static constexpr int TR = mla_tile_rows(W);         // positions per tile
+  static constexpr int TR = mla_tile_rows(W, R);      // positions per tile
+  static constexpr int BR = mla_box_rows(W);          // rows per TMA copy
+  static constexpr int MS = TR > 64 ? 128 : 64;       // score UMMA M
+  static constexpr int PNS = TR > 64 ? 2048 : 1024;   // P operand: bytes between 8-column blocks
   static constexpr int KH = W + kRope;                // hi extent: latent + rope
   static constexpr int BOXES = KH / 64;               // 64-coordinate boxes per tile
   static constexpr int BOX = TR * 128;                // bytes per box
   static constexpr int STAGE = BOXES * BOX;
-  static constexpr int NST = (R > 1 && W == 512) ? 2 : 3;  // two where the wider query operand needs the room
+  // stages: two where the wider query operand (R = 2, d = 512) or the
+  // 128-position tile (d = 64: two CTAs per SM) needs the room
+  static constexpr int NST = (R > 1 && W == 512) || TR > 64 ? 2 : 3;
   static constexpr int QB = NQ * KH * 2;              // [Q_hi ; Q_lo] operand (NQ rows)
-  static constexpr int PB = 4 * 1024 * R;             // [P_hi | P_lo] operand, 4 R column blocks
+  static constexpr int PB = 4 * PNS * R;              // [P_hi | P_lo] operand, 4 R column blocks
   static constexpr int OFF_Q = NST * STAGE;
   static constexpr int OFF_P = OFF_Q + QB;            // two buffers
   static constexpr int OFF_RED = OFF_P + 2 * PB;      // float [4][NH] maxima, [4][NH] sums
@@ -93,7 +108,7 @@ struct MlaCfg {
   static constexpr int SCOLS = 2 * NQ;                // two NQ-column S buffers
   static constexpr int TCOLS = OCOLS + SCOLS <= 128 ? 128 : OCOLS + SCOLS <= 256 ? 256 : 512;
   static_assert(KH % 64 == 0 && W % 64 == 0, "whole boxes");
-  static_assert(TR % 16 == 0 && TR <= 64, "tile rows");
+  static_assert(TR % 16 == 0 && TR % BR == 0 && (TR <= 64 || TR == 128), "tile rows");
   static_assert(OCOLS + SCOLS <= TCOLS, "TMEM columns");
   static_assert(SMEM <= 232448, "shared memory");
   static_assert(R == 1 || R == 2, "one or two query rows per CTA");
@@ -220,7 +235,10 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         mbar_expect_tx(&full[s], C::STAGE);
 #pragma unroll
         for (int j = 0; j < C::BOXES; ++j)
-          tma_load_2d(stage(s) + j * C::BOX, &tmap, 64 * j, row0 + issued * TR, &full[s]);
+#pragma unroll
+          for (int h = 0; h < TR / C::BR; ++h)
+            tma_load_2d(stage(s) + j * C::BOX + h * C::BR * 128, &tmap, 64 * j,
+                        row0 + issued * TR + h * C::BR, &full[s]);
       }
       // the last copies land before the CTA leaves (bounded; done at once
       // when they were consumed)
@@ -237,7 +255,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     // (t - NST <= t - 2): its wait for full[t % NST] is then for the phase
     // right after the last completed one.
     const int role = warp == 4 ? 0 : 1;
-    constexpr uint32_t ID_S = umma_idesc(64, NQ, false, false);
+    constexpr uint32_t ID_S = umma_idesc(C::MS, NQ, false, false);
     for (int t = role; t < n_tiles && !failed; t += 2) {
       const int s = t % C::NST;
       bool ok = true;
@@ -287,7 +305,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
       if (ok && lane == 0) {  // O^T[:, hi | lo] += C^T [P_hi | P_lo]
         tc_fence_after();
         const uint64_t da = umma_desc(smem_u32(stage(t % C::NST)), C::BOX, 1024, 2);
-        const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, 1024, 0);
+        const uint64_t dp = umma_desc(smem_u32(pbuf(t & 1)), 128, C::PNS, 0);
 #pragma unroll
         for (int ks = 0; ks < TR / 16; ++ks)
 #pragma unroll
@@ -311,7 +329,11 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
   } else {
     // ======================= softmax warps ================================
     const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
-    const int prow = 16 * warp + lane;  // this lane's tile position (lanes 0-15)
+    // this lane's tile position: M = 128 scores put position r in TMEM lane
+    // r; M = 64 in lane 32 (r/16) + r%16 (lanes 0-15 of each warp)
+    constexpr bool ALL = C::MS == 128;
+    constexpr int RL = ALL ? 32 : 16;  // lanes holding positions
+    const int prow = ALL ? 32 * warp + lane : 16 * warp + lane;
     // each row's own end: row rho sees the positions below its causal limit
     int i1r[R];
 #pragma unroll
@@ -333,7 +355,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         float hi[16], lo[16];
         tmem_ld16(t_s + NQ * (t & 1) + 32 * r + lane_off, hi);
         tmem_ld16(t_s + NQ * (t & 1) + 32 * r + 16 + lane_off, lo);
-        const bool live = lane < 16 && prow < min(TR, i1r[r] - base);
+        const bool live = (ALL || lane < 16) && prow < min(TR, i1r[r] - base);
 #pragma unroll
         for (int h = 0; h < 16; ++h) x[16 * r + h] = live ? hi[h] + lo[h] : -INFINITY;
       }
@@ -346,7 +368,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         for (int j = 0; j < NH; ++j) {
           float mx = x[j];
 #pragma unroll
-          for (int off = 1; off < 16; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+          for (int off = 1; off < RL; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
           if (lane == 0) red[warp * NH + j] = mx;
         }
         softmax_sync();
@@ -382,9 +404,9 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         softmax_sync();  // `red` is reused by the next vote
       }
       // weights hi/lo in bf16 into the MN-major P operand: position k, column
-      // n (32 rho + h hi, 32 rho + 16 + h lo) at (k/8) 128 + (n/8) 1024 +
+      // n (32 rho + h hi, 32 rho + 16 + h lo) at (k/8) 128 + (n/8) PNS +
       // (k%8) 16 + (n%8) 2
-      if (lane < 16 && prow < TR) {
+      if ((ALL || lane < 16) && prow < TR) {
 #pragma unroll
         for (int r = 0; r < R; ++r) {
           uint32_t hw[8], lw[8];
@@ -397,11 +419,11 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
             l_part[j + 1] += p1;
             split2<true>(p0, p1, hw[h / 2], lw[h / 2]);
           }
-          uint8_t *pp = pbuf(t & 1) + 4096 * r + (prow / 8) * 128 + (prow % 8) * 16;
+          uint8_t *pp = pbuf(t & 1) + 4 * C::PNS * r + (prow / 8) * 128 + (prow % 8) * 16;
           *reinterpret_cast<uint4 *>(pp) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-          *reinterpret_cast<uint4 *>(pp + 1024) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
-          *reinterpret_cast<uint4 *>(pp + 2048) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-          *reinterpret_cast<uint4 *>(pp + 3072) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
+          *reinterpret_cast<uint4 *>(pp + C::PNS) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+          *reinterpret_cast<uint4 *>(pp + 2 * C::PNS) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+          *reinterpret_cast<uint4 *>(pp + 3 * C::PNS) = make_uint4(lw[4], lw[5], lw[6], lw[7]);
         }
       }
       fence_proxy_async();
@@ -428,7 +450,7 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
       for (int j = 0; j < NH; ++j) {
         float sum = l_part[j];
 #pragma unroll
-        for (int off = 1; off < 16; off <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+        for (int off = 1; off < RL; off <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
         if (lane == 0) lsum[warp * NH + j] = sum;
       }
 #pragma unroll
@@ -562,7 +584,7 @@ int mla_ctas_t() {
 cudaError_t mla_make_tmap(void *out, const MlaView &v) {
   const uint64_t dims[2] = {(uint64_t)(v.width + v.rope), (uint64_t)v.B * (uint64_t)v.cap};
   const uint64_t strides[1] = {(uint64_t)v.rec_bytes};
-  const uint32_t box[2] = {64, (uint32_t)mla_tile_rows(v.width)};
+  const uint32_t box[2] = {64, (uint32_t)mla_box_rows(v.width)};
   const uint32_t estr[2] = {1, 1};
   return encode_tensor_map_tiled(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, v.rec, dims, strides, box,
                                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
