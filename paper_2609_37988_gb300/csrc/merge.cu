@@ -13,13 +13,16 @@
 namespace kvk {
 namespace {
 
+// P is written by the decode this launch overlaps (programmatic dependent
+// launch), so it is read with coherent loads after the grid-dependency wait,
+// not through the read-only path (no __restrict__).
 // One thread per output element: every load of the row's partials (the S
 // maxima, sums and this element's accumulators) is issued before any is
 // used, so the merge costs one memory round trip.  Rows per CTA: 128 / dim
 // (dim <= 128), else one row with a channel loop.
 template <int SB>
 __global__ void __launch_bounds__(128)
-    splitk_merge_kernel(const float *__restrict__ P, int S, int n_rows, int dim,
+    splitk_merge_kernel(const float *P, int S, int n_rows, int dim,
                         float *__restrict__ out) {
   pdl_wait();
   pdl_trigger();
@@ -59,7 +62,7 @@ __global__ void __launch_bounds__(128)
 
 // more than 16 splits: the same, with the split loop not unrolled
 __global__ void __launch_bounds__(128)
-    splitk_merge_kernel_n(const float *__restrict__ P, int S, int n_rows, int dim,
+    splitk_merge_kernel_n(const float *P, int S, int n_rows, int dim,
                           float *__restrict__ out) {
   pdl_wait();
   pdl_trigger();

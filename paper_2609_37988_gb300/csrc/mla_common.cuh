@@ -93,9 +93,14 @@ __global__ void __launch_bounds__(128)
 // W_UV rows are prefetched into shared memory (cp.async) while phase 1
 // merges the 16 rows into o_lat (split hi/lo bf16, shared memory); phase 2:
 // warp w computes 16 sequences x 8 outputs over K = d on the tensor cores.
+// `partial` is written by the decode kernel this launch overlaps
+// (programmatic dependent launch): it is read with coherent loads after the
+// grid-dependency wait, never through the read-only path (no __restrict__),
+// whose loads may be scheduled as if the data were constant for the whole
+// kernel.
 template <int W>
 __global__ void __launch_bounds__(128)
-    mla_merge_upv_kernel(const float *__restrict__ partial, int n_splits,
+    mla_merge_upv_kernel(const float *partial, int n_splits,
                          const uint16_t *__restrict__ w_uv, int B, int H, int r,
                          float *__restrict__ out) {
   constexpr int Dv = 128;
@@ -122,6 +127,29 @@ __global__ void __launch_bounds__(128)
   pdl_wait();
   const size_t RS = (size_t)W + 2;
   const size_t pstride = (size_t)B * H * RS;
+  // o_lat = sum_s w_s acc_s / L, (row, pair) elements of the 16 rows: each
+  // thread keeps its PER elements in registers and issues a split group's
+  // loads together; the first group's loads go out with the (m, l) loads
+  // below, so that a merge of up to SG splits takes one memory round trip
+  constexpr int PER = 16 * (W / 2) / 128;
+  constexpr int SG = PER >= 16 ? 1 : 16 / PER;  // splits whose loads are in flight together
+  float2 x[SG][PER];
+  auto load_group = [&](int sp0) {
+#pragma unroll
+    for (int g2 = 0; g2 < SG; ++g2) {
+      const int sp = sp0 + g2;
+#pragma unroll
+      for (int k = 0; k < PER; ++k) {
+        const int e = tid + 128 * k, row = e / (W / 2), i = 2 * (e % (W / 2));
+        const int b = b0 + row;
+        x[g2][k] = (sp < n_splits && b < B)
+                       ? *reinterpret_cast<const float2 *>(partial + sp * pstride +
+                                                           ((size_t)b * H + h) * RS + i)
+                       : make_float2(0.f, 0.f);
+      }
+    }
+  };
+  load_group(0);
   // merge weights: every split's (m, l) of the 16 rows loaded at once
   float *l_s = linv_s + 16;  // [64][16] split sums, then 1/L
   for (int q = tid; q < n_splits * 16; q += 128) {
@@ -148,29 +176,11 @@ __global__ void __launch_bounds__(128)
     linv_s[tid] = (L > 0.f) ? 1.f / L : 0.f;
   }
   __syncthreads();
-  // o_lat = sum_s w_s acc_s / L, (row, pair) elements of the 16 rows: each
-  // thread keeps its PER elements in registers and issues a split's loads
-  // together, one memory round trip per split
-  constexpr int PER = 16 * (W / 2) / 128;
-  constexpr int SG = PER >= 16 ? 1 : 16 / PER;  // splits whose loads are in flight together
   float2 oacc[PER];
 #pragma unroll
   for (int k = 0; k < PER; ++k) oacc[k] = make_float2(0.f, 0.f);
   for (int sp0 = 0; sp0 < n_splits; sp0 += SG) {
-    float2 x[SG][PER];
-#pragma unroll
-    for (int g2 = 0; g2 < SG; ++g2) {
-      const int sp = sp0 + g2;
-#pragma unroll
-      for (int k = 0; k < PER; ++k) {
-        const int e = tid + 128 * k, row = e / (W / 2), i = 2 * (e % (W / 2));
-        const int b = b0 + row;
-        x[g2][k] = (sp < n_splits && b < B)
-                       ? *reinterpret_cast<const float2 *>(partial + sp * pstride +
-                                                           ((size_t)b * H + h) * RS + i)
-                       : make_float2(0.f, 0.f);
-      }
-    }
+    if (sp0 > 0) load_group(sp0);
 #pragma unroll
     for (int g2 = 0; g2 < SG; ++g2) {
       const int sp = sp0 + g2;
