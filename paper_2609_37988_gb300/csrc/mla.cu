@@ -57,8 +57,10 @@ namespace {
 // maximum kept within 2^8 (one vote per tile; maxima are reduced only when
 // one rises).  The weights go hi/lo in bf16 into the P operand; O stays in
 // TMEM until the end (rescaled in place on the rare tiles that raise a
-// maximum).  The MMA warp keeps the tensor core fed: scores(t) goes out as
-// soon as tile t has landed, values(t-1) as soon as P(t-1) is written; the
+// maximum).  Two score warps issue a tile's score products as soon as it
+// has landed, each half of the K-steps into its own accumulator (the softmax
+// adds the two), so a stage's chain (landing, scores, softmax, values) is
+// short; the value warp issues values(t) as soon as P(t) is written; the
 // copy warp refills a stage as soon as the values that read it completed.
 // Every wait is bounded (an abort flag stops the other role); the CTA frees
 // its TMEM on every path.
@@ -105,7 +107,7 @@ struct MlaCfg {
   static constexpr int MV = W >= 128 ? 128 : 64;      // value UMMA M
   static constexpr int MB = W / MV;                   // value M-blocks
   static constexpr int OCOLS = NQ * MB;               // TMEM columns of O
-  static constexpr int SCOLS = 2 * NQ;                // two NQ-column S buffers
+  static constexpr int SCOLS = 4 * NQ;                // two S buffers of two K-halves
   static constexpr int TCOLS = OCOLS + SCOLS <= 128 ? 128 : OCOLS + SCOLS <= 256 ? 256 : 512;
   static_assert(KH % 64 == 0 && W % 64 == 0, "whole boxes");
   static_assert(TR % 16 == 0 && TR % BR == 0 && (TR <= 64 || TR == 128), "tile rows");
@@ -165,8 +167,9 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
 
   if (tid == 0) {
     for (int i = 0; i < C::NBAR; ++i) {
-      const bool pb = i >= C::NST + 2 && i < C::NST + 4;
-      mbar_init(&full[i], pb ? 4 : 1);
+      const bool sb = i >= C::NST && i < C::NST + 2;      // both score warps commit
+      const bool pb = i >= C::NST + 2 && i < C::NST + 4;  // the four softmax warps
+      mbar_init(&full[i], pb ? 4 : sb ? 2 : 1);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -249,14 +252,16 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
     pdl_trigger();
   } else if (warp == 4 || warp == 7) {
     // ======================= score warps ==================================
-    // warp 4 the even tiles, warp 7 the odd ones.  Before tile t a warp
-    // waits for softmax(t-2) (its S buffer is free), which follows softmax
-    // of every earlier tile, hence the landing of the stage's previous tile
-    // (t - NST <= t - 2): its wait for full[t % NST] is then for the phase
-    // right after the last completed one.
+    // Both warps take every tile: warp 4 the first half of the K-steps into
+    // its own accumulator, warp 7 the second half into another (the softmax
+    // adds the two), so that a tile's scores take half the issue time.
+    // Before tile t a warp waits for softmax(t-2) (the S buffer is free),
+    // then for the tile's landing; both waits are for consecutive phases.
     const int role = warp == 4 ? 0 : 1;
     constexpr uint32_t ID_S = umma_idesc(C::MS, NQ, false, false);
-    for (int t = role; t < n_tiles && !failed; t += 2) {
+    constexpr int KS = C::KH / 16, KHALF = KS / 2;
+    static_assert(KS % 2 == 0, "K-steps split evenly over the two score warps");
+    for (int t = 0; t < n_tiles && !failed; ++t) {
       const int s = t % C::NST;
       bool ok = true;
       if (t >= 2) ok = mbar_wait_or_abort(&pbar[t & 1], ((t - 2) >> 1) & 1, kLimit, abort_flag);
@@ -272,15 +277,18 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
         fence_proxy_async();
         __syncwarp();
       }
-      if (ok && lane == 0) {  // scores(t) -> S[t & 1]
+      if (ok && lane == 0) {  // this warp's half of scores(t) -> S[t & 1][role]
         tc_fence_after();
         const uint64_t dc = umma_desc(smem_u32(stage(s)), 16, 1024, 2);
         const uint64_t dq = umma_desc(smem_u32(q_s), 128, C::KH / 8 * 128, 0);
 #pragma unroll
-        for (int ks = 0; ks < C::KH / 16; ++ks)
-          umma_f16(t_s + NQ * (t & 1), dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4),
-                   dq + (uint64_t)(ks * 16), ID_S, ks > 0);
-        umma_commit(&sbar[t & 1]);
+        for (int kk = 0; kk < KHALF; ++kk) {
+          const int ks = role * KHALF + kk;
+          umma_f16(t_s + NQ * (2 * (t & 1) + role),
+                   dc + (uint64_t)(((ks / 4) * C::BOX + (ks % 4) * 32) >> 4), dq + (uint64_t)(ks * 16),
+                   ID_S, kk > 0);
+        }
+        umma_commit(&sbar[t & 1]);  // one of the two arrivals
       }
       failed = !__all_sync(0xffffffffu, ok);
     }
@@ -352,12 +360,16 @@ __global__ void __launch_bounds__(kMlaThreads, 1)
       float x[NH];
 #pragma unroll
       for (int r = 0; r < R; ++r) {
-        float hi[16], lo[16];
-        tmem_ld16(t_s + NQ * (t & 1) + 32 * r + lane_off, hi);
-        tmem_ld16(t_s + NQ * (t & 1) + 32 * r + 16 + lane_off, lo);
+        // hi and lo columns of both K-halves
+        float hi[16], lo[16], hi2[16], lo2[16];
+        const uint32_t sa = t_s + 2 * NQ * (t & 1) + 32 * r + lane_off;
+        tmem_ld16(sa, hi);
+        tmem_ld16(sa + 16, lo);
+        tmem_ld16(sa + NQ, hi2);
+        tmem_ld16(sa + NQ + 16, lo2);
         const bool live = (ALL || lane < 16) && prow < min(TR, i1r[r] - base);
 #pragma unroll
-        for (int h = 0; h < 16; ++h) x[16 * r + h] = live ? hi[h] + lo[h] : -INFINITY;
+        for (int h = 0; h < 16; ++h) x[16 * r + h] = live ? (hi[h] + hi2[h]) + (lo[h] + lo2[h]) : -INFINITY;
       }
       bool need = false;
 #pragma unroll
