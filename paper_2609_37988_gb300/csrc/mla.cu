@@ -92,9 +92,13 @@ struct MlaCfg {
   static constexpr int BOXES = KH / 64;               // 64-coordinate boxes per tile
   static constexpr int BOX = TR * 128;                // bytes per box
   static constexpr int STAGE = BOXES * BOX;
-  // stages: two where the wider query operand (R = 2, d = 512) or the
-  // 128-position tile (d = 64: two CTAs per SM) needs the room
-  static constexpr int NST = (R > 1 && W == 512) || TR > 64 ? 2 : 3;
+  // stages: the decode is bound by the bytes in flight per SM, so as many
+  // as shared memory holds beside the rest at the CTAs per SM each width
+  // runs: four at d = 256 (the call 49.1 -> 45.5 us), three at d = 512 (two
+  // with R = 2, whose query operand takes the room), three at d = 128 and
+  // two at d = 64 (two CTAs per SM; one CTA per SM with eight or six stages
+  // took the d = 128 call 33.9 -> 34.8 us and both pre-fills 15-45 % longer)
+  static constexpr int NST = (R > 1 && W == 512) ? 2 : W == 256 ? 4 : TR > 64 ? 2 : 3;
   static constexpr int QB = NQ * KH * 2;              // [Q_hi ; Q_lo] operand (NQ rows)
   static constexpr int PB = 4 * PNS * R;              // [P_hi | P_lo] operand, 4 R column blocks
   static constexpr int OFF_Q = NST * STAGE;
