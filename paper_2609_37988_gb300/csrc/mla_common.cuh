@@ -132,7 +132,7 @@ __global__ void __launch_bounds__(128)
   // loads together; the first group's loads go out with the (m, l) loads
   // below, so that a merge of up to SG splits takes one memory round trip
   constexpr int PER = 16 * (W / 2) / 128;
-  constexpr int SG = PER >= 16 ? 1 : 16 / PER;  // splits whose loads are in flight together
+  constexpr int SG = PER >= 32 ? 1 : 32 / PER;  // splits whose loads are in flight together
   float2 x[SG][PER];
   auto load_group = [&](int sp0) {
 #pragma unroll
