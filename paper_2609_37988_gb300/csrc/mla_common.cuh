@@ -132,7 +132,9 @@ __global__ void __launch_bounds__(128)
   // loads together; the first group's loads go out with the (m, l) loads
   // below, so that a merge of up to SG splits takes one memory round trip
   constexpr int PER = 16 * (W / 2) / 128;
-  constexpr int SG = PER >= 32 ? 1 : 32 / PER;  // splits whose loads are in flight together
+  // splits whose loads are in flight together: 32 elements per thread, and
+  // both splits of the widest latent (64 registers of loads there)
+  constexpr int SG = PER >= 32 ? 2 : 32 / PER;
   float2 x[SG][PER];
   auto load_group = [&](int sp0) {
 #pragma unroll
