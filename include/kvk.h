@@ -278,8 +278,8 @@ kvk_status kvk_prefill_attention(kvk_cache *cache, int32_t layer, const void *q,
  * kvk_decode_attention_mla: q_lat = W_UK[h][:, :d]^T q_nope, scores
  * sigma (q_lat . c[:d] + q_pe . k^R), output W_UV[h][:, :d] o_lat).  Each
  * query row runs the decode path over its own causal prefix (one CTA per
- * row, or per pair of consecutive rows of a sequence at widths >= 256 when
- * n_q is even).  Queries before position 0 give zeros.
+ * row, or per pair of consecutive rows of a sequence for bf16 latents of
+ * width >= 256 when n_q is even).  Queries before position 0 give zeros.
  *  q_nope:  device bf16 [B, n_q, H, head_dim]; q_pe: bf16 [B, n_q, H, rope]
  *           (post-RoPE);
  *  w_uk, w_uv: device bf16 [H, head_dim, latent] as for decode;
